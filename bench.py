@@ -1,0 +1,376 @@
+"""Benchmark of the stage-decode step on GB300.
+
+One step = one decode step of the 7B-shaped body stage (blocks [0, 14) of a 28-block Qwen
+7B-shaped decoder, d_model 3584, 28/4 heads of 128, FFN 18944, bf16 weights, batch 1, KV
+context 2048 pre-filled) unless --config picks another workload.  Each timed step decodes the
+next position of the workload's 64-step run (positions wrap after 64 steps).
+
+Prints one JSON line: metric "stage decode us/layer/token" (lower is better), the roofline of
+the dominant kernel (gate/up GEMV) against the measured HBM copy bandwidth, the whole step's
+HBM fraction, an end-to-end figure through the host-buffer C-ABI call, SM clocks sampled
+during the timed region, and the CPU oracle timed on a bounded sample (cpu_baseline).
+
+``--impl reference`` times the CPU oracle instead (this workload has no runnable reference
+implementation: the paper ships none).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "stage decode us/layer/token"
+UNIT = "us/layer/token"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", type=int, default=2)
+    ap.add_argument("--profile-steps", type=int, default=20)
+    ap.add_argument("--e2e-steps", type=int, default=500)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)), int(os.environ.get("WORLD_SIZE", 1))
+
+
+# ---------------------------------------------------------------------------- bytes
+
+def kernel_bytes(work, kind: str) -> int:
+    """Algorithmic HBM bytes of one launch of a kernel kind at the workload's first step:
+    weights as stored once, activations in and out once, KV rows read over [0, P_b]."""
+    from paper_2609_34045_gb300 import workload as wl
+    m, b = work.model, work.batch
+    d, q, kv, f, v = m.d_model, m.q_dim, m.kv_dim, m.ffn, m.vocab
+    mb = lambda r, c: wl.matrix_bytes(r, c, m.weight_fmt)  # noqa: E731
+    if kind == "qkv":
+        return mb(q + 2 * kv, d) + b * (d + q) * 4 + b * 2 * kv * 2
+    if kind == "attn":
+        return sum(2 * kv * 2 * (p + 1) for p in work.contexts[:b]) + 2 * b * q * 4
+    if kind == "oproj":
+        return mb(d, q) + b * (q + 3 * d) * 4
+    if kind == "gateup":
+        return mb(2 * f, d) + b * (d + f) * 4
+    if kind == "down":
+        return mb(d, f) + b * (f + 3 * d) * 4
+    if kind == "lmhead":
+        return mb(v, d) + b * d * 4
+    return 0
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return float(j["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for name in ("gemv.cu", "common.cuh"):
+        with open(os.path.join(ROOT, "paper_2609_34045_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(kind: str, config: int):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on the current
+    kernel source (else None)."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        j = json.load(f)
+    e = j.get(f"config{config}", {}).get(kind)
+    if not e or e.get("source_hash") != kernel_source_hash():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+# ---------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(prefix="kfl_clocks_", suffix=".csv")
+            os.close(fd)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------------------- CPU oracle
+
+def oracle_layer_seconds(work, n_layer_steps: int, warmup: int = 1):
+    """Time the CPU oracle on single-block decode steps of the workload (weights and KV made
+    before timing).  Returns (seconds per layer-token, layer-steps timed, threads)."""
+    import numpy as np
+
+    import oracle
+    from paper_2609_34045_gb300 import workload as wl
+    m = work.model
+    st = oracle.OracleStage(m, work.l0, work.l0 + 1, False, False, work.batch, work.max_ctx)
+    st.load_layer(0, wl.layer_weights(m, work.l0, work.seed))
+    for u in range(work.batch):
+        k, v = wl.kv_prefill(m, work.l0, u, work.contexts[u], work.seed)
+        st.set_kv(0, u, k, v)
+    h = wl.hidden_in(m, 0, work.batch, work.seed)
+    pos = wl.positions(work, 0)
+    for _ in range(warmup):
+        st.decode(pos, hidden_in=h)
+    t0 = time.perf_counter()
+    for _ in range(n_layer_steps):
+        st.decode(pos, hidden_in=h)
+    dt = (time.perf_counter() - t0) / n_layer_steps
+    return dt / work.batch, n_layer_steps, os.cpu_count()
+
+
+def run_reference(args, work):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return 0
+    sec, n, cores = oracle_layer_seconds(work, max(1, min(args.steps, 8)), warmup=min(args.warmup, 1))
+    us = sec * 1e6
+    line = {
+        "impl": "reference", "metric": METRIC, "value": us, "unit": UNIT, "n_gpus": args.gpus, "steps": n,
+        "warmup": min(args.warmup, 1), "ms_per_step": sec * 1e3 * work.batch, "higher_is_better": False,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded)",
+        "config": {"workload": work.name, "layers_timed": 1, "batch": work.batch, "ctx": list(work.contexts),
+                   "note": "the paper ships no implementation; the reference arm is the fp64 CPU oracle"},
+        "cpu_baseline": {"value": us, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": f"{n} decode steps of one block (block {work.l0}) of {work.name}"},
+        "e2e": {"value": us, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------------------- ours
+
+def run_ours(args, work):
+    import numpy as np
+    import torch
+
+    from paper_2609_34045_gb300 import device_inputs as di
+    from paper_2609_34045_gb300 import stage as K
+    from paper_2609_34045_gb300 import workload as wl
+
+    rank, local, world = dist_env()
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    if not os.path.exists(K.LIB_PATH):
+        from paper_2609_34045_gb300.build import build
+        build()
+
+    m = work.model
+    flags = (K.KFL_EMBED_IN if work.embed_in else 0) | (K.KFL_LOGITS_OUT if work.logits_out else 0)
+    cfg = K.model_cfg(m, work.max_ctx, work.batch)
+    st = K.kfl_stage_create(cfg, work.l0, work.l1, flags)
+    di.load_stage_seeded(st, work)
+    b, d = work.batch, m.d_model
+    stream = torch.cuda.current_stream()
+    n_pos = work.steps
+    pos_all = torch.tensor(np.stack([wl.positions(work, s) for s in range(n_pos)]), dtype=torch.int32,
+                           device="cuda")
+    if work.embed_in:
+        ids_all = torch.tensor(np.stack([wl.token_ids(work.seed, wl.ids_tag(s), b, m.vocab) for s in range(n_pos)]),
+                               dtype=torch.int32, device="cuda")
+        hid_all = None
+    else:
+        ids_all = None
+        hid_all = torch.tensor(np.stack([wl.hidden_in(m, s, b, work.seed) for s in range(n_pos)]),
+                               dtype=torch.float32, device="cuda")
+    out = torch.empty(b, d, dtype=torch.float32, device="cuda")
+    nxt = torch.empty(b, dtype=torch.int32, device="cuda") if work.logits_out else None
+
+    def step(s):
+        i = s % n_pos
+        K.kfl_stage_decode(st, ids_all[i] if ids_all is not None else None,
+                           hid_all[i] if hid_all is not None else None, pos_all[i], b, out, nxt,
+                           stream.cuda_stream)
+
+    for s in range(args.warmup):
+        step(s)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)  # let the sampler take its first reading
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for s in range(args.steps):
+        step(s)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    if dist:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+        dist.barrier()
+    status = K.kfl_stage_status(st)
+    if status != 0:
+        raise RuntimeError(f"device reported {K.kfl_strerror(status)} during the benchmark")
+
+    n_layers = max(1, work.n_layers)
+    value = ms * 1e3 / (n_layers * b) / world
+    launches = K.kfl_stage_launches_per_step(st, b) * args.steps
+
+    # per-kernel timing (kernels one by one with CUDA events on the launching stream)
+    K.kfl_stage_profile(st, True)
+    for s in range(args.profile_steps):
+        step(s)
+    prof = K.kfl_stage_profile_read(st)
+    K.kfl_stage_profile(st, False)
+    kinds = [k for k in ("qkv", "attn", "oproj", "gateup", "down", "lmhead") if prof[k][1] > 0]
+    dom = max(kinds, key=lambda k: prof[k][0])
+    dom_ms = prof[dom][0] / prof[dom][1]
+    dom_bytes = kernel_bytes(work, dom)
+    peak, peak_kind = measured_peaks()
+    achieved = dom_bytes / (dom_ms * 1e-3) / 1e9
+    step_bytes = work.step_bytes(0)
+    step_gbs = step_bytes / (ms * 1e-3) / 1e9
+    per_kernel = {k: {"us": 1e3 * prof[k][0] / prof[k][1], "launches_per_step": prof[k][1] / args.profile_steps,
+                      "gbs": (kernel_bytes(work, k) / (prof[k][0] / prof[k][1] * 1e-3) / 1e9) if prof[k][0] else None}
+                  for k in kinds}
+
+    # end to end through the host-buffer C-ABI call (pinned host memory, copies timed)
+    e2e_steps = min(args.e2e_steps, args.steps)
+    pos_h = torch.from_numpy(np.stack([wl.positions(work, s) for s in range(n_pos)])).pin_memory()
+    if work.embed_in:
+        in_h = torch.from_numpy(np.stack([wl.token_ids(work.seed, wl.ids_tag(s), b, m.vocab)
+                                          for s in range(n_pos)])).pin_memory()
+        h2d = b * 4 + b * 4
+    else:
+        in_h = torch.from_numpy(np.stack([wl.hidden_in(m, s, b, work.seed) for s in range(n_pos)])).pin_memory()
+        h2d = b * d * 4 + b * 4
+    out_h = torch.empty(b, d, dtype=torch.float32).pin_memory()
+    nxt_h = torch.empty(b, dtype=torch.int32).pin_memory() if work.logits_out else None
+    d2h = (b * 4) if work.logits_out else (b * d * 4)
+
+    def e2e_step(s):
+        i = s % n_pos
+        K.kfl_stage_decode_host(st, in_h[i] if work.embed_in else None, None if work.embed_in else in_h[i],
+                                pos_h[i], b, None if work.logits_out else out_h, nxt_h, stream.cuda_stream)
+
+    for s in range(3):
+        e2e_step(s)
+    if dist:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for s in range(e2e_steps):
+        e2e_step(s)
+    e2e_s = (time.perf_counter() - t0) / e2e_steps
+    if dist:
+        t = torch.tensor([e2e_s], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    e2e_value = e2e_s * 1e6 / (n_layers * b) / world
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        sec, n, cores = oracle_layer_seconds(work, 3)
+        cpu = {"value": sec * 1e6, "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": f"{n} decode steps of one block (block {work.l0}) of {work.name}, fp64 numpy"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": False, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16 weights, fp32 accumulate", "data": "synthetic (seeded)",
+            "config": {"workload": work.name, "stage_layers": [work.l0, work.l1], "batch": b,
+                       "ctx": list(work.contexts), "weights": m.weight_fmt,
+                       "l2": "inputs larger than L2 (weights streamed once per step)",
+                       "parallelism": f"replicas x{world}"},
+            "tokens_per_s": b * world / (ms * 1e-3),
+            "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "peak_kind": f"{peak_kind} copy (MEASURED_PEAKS.json hbm_gbs)",
+                         "bytes_per_launch": dom_bytes, "us_per_launch": dom_ms * 1e3,
+                         "traffic": ncu_traffic(dom, args.config)},
+            "step_roofline": {"bytes_per_step": step_bytes, "achieved_gbs": step_gbs, "frac_of_measured": step_gbs / peak,
+                              "frac_of_8tbs": step_gbs / 8000.0},
+            "per_kernel": per_kernel,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "steps": e2e_steps},
+            "gpu_launches": launches,
+            "clocks": clk,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    K.kfl_stage_destroy(st)
+    if dist:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse()
+    from paper_2609_34045_gb300 import workload as wl
+    work = wl.CONFIGS[args.config]
+    if args.impl == "reference":
+        return run_reference(args, work)
+    return run_ours(args, work)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,218 @@
+// Internal definitions shared by the stage-decode kernels and the runtime (sm_103a only).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#if defined(__CUDA_ARCH__) && (__CUDA_ARCH__ < 1000)
+#error "this library targets sm_103a (Blackwell) only"
+#endif
+
+namespace kfl {
+
+// ---- tiling of the weight-streaming GEMV ------------------------------------------------
+// A matrix [N][K] is stored as tiles [N/RB][K/KT][RB][KT] (zero-padded), each tile one
+// contiguous 16 KiB chunk of HBM, so a CTA streams its share of the matrix with 1-D bulk
+// copies and every warp reads a whole tile row from shared memory without bank conflicts.
+constexpr int RB = 64;            // rows per row block (and per tile)
+constexpr int KT = 128;           // K per bf16 tile
+constexpr int TILE_BYTES = RB * KT * 2;
+constexpr int MAXB = 4;           // users per step
+constexpr int XCHUNK_BYTES = KT * 4;          // one user's fp32 activation chunk of a tile
+constexpr int STAGE_BYTES = TILE_BYTES + MAXB * XCHUNK_BYTES;
+constexpr int CONSUMER_WARPS = 8;
+constexpr int GEMV_THREADS = (CONSUMER_WARPS + 1) * 32;
+constexpr int MAX_STAGES = 10;
+
+// int4 group-64 tiles: [N/RB][K/KT4][RB][KT4/8] uint32 codes then [RB][KT4/64] bf16 scales
+constexpr int KT4 = 256;
+constexpr int TILE4_CODE_BYTES = RB * KT4 / 2;     // 8 KiB
+constexpr int TILE4_SCALE_BYTES = RB * (KT4 / 64) * 2;  // 512 B
+constexpr int TILE4_BYTES = TILE4_CODE_BYTES + TILE4_SCALE_BYTES;
+
+// ---- device error word bits ---------------------------------------------------------------
+constexpr unsigned ERR_POSITION = 1u;
+constexpr unsigned ERR_TOKEN = 2u;
+constexpr unsigned ERR_TIMEOUT = 4u;
+
+// bounded waits: spins before backing off, total polls before giving up (~1-2 s)
+constexpr uint32_t WAIT_FAST_SPINS = 1024;
+constexpr uint32_t WAIT_LIMIT = 1u << 24;
+
+enum Epilogue : int {
+  EPI_STORE = 0,   // out[b][n] = y
+  EPI_QKV = 1,     // RoPE on q/k row pairs, q to fp32, k/v appended to the bf16 cache
+  EPI_RESID = 2,   // h[b][n] += y; xn = h * g_next; per-row-block sum of squares
+  EPI_SWIGLU = 3,  // rows (2j, 2j+1) = (gate_j, up_j) -> a[b][j] = silu(gate) * up
+  EPI_ARGMAX = 4,  // greedy argmax over rows, lowest index on ties
+};
+
+struct GemvParams {
+  const uint8_t *w;  // tiled weights
+  int fmt;           // 0 bf16, 1 int4
+  int n_rows;        // valid rows N
+  int n_rb, n_kt;    // row blocks, K tiles
+  int tile_bytes;
+  int kt;            // K per tile
+  const float *x;    // activations [batch][ldx]
+  int ldx;
+  int batch;
+  int stages;
+  // RMSNorm folded into the GEMV: y = inv_rms[b] * (W . x) with x = h * g precomputed by the
+  // producer of h; inv_rms from the per-row-block sums of squares of h
+  const float *sumsq;  // [n_parts][MAXB] or NULL
+  int n_parts;
+  int d_norm;
+  float eps;
+  // EPI_STORE / EPI_SWIGLU
+  float *out;
+  int ldo;
+  // EPI_RESID
+  float *h;
+  float *xn;
+  const float *g_next;
+  float *sumsq_out;
+  float *capture;  // [MAXB? no: batch rows][ldh] per-layer hidden, or NULL
+  int ldh;
+  // EPI_QKV
+  float *q;
+  uint16_t *kcache, *vcache;  // this layer's [max_batch][Hkv][max_ctx][hd]
+  const int *positions;
+  const float *rope_cos, *rope_sin;  // [max_ctx][hd/2]
+  int n_q_rows, n_kv_rows, head_dim, max_ctx, n_kv_heads;
+  // EPI_ARGMAX
+  float *cand_val;
+  int *cand_idx;
+  int *argmax_ticket;
+  int *next_ids;
+  // stream-K bookkeeping
+  float *partial;  // [grid][2][RB][MAXB]
+  int *tickets;    // [n_rb], zero between launches
+  unsigned *err;
+};
+
+struct AttnParams {
+  const float *q;            // [batch][Hq*hd] (RoPE applied)
+  const uint16_t *kcache;    // this layer's [max_batch][Hkv][max_ctx][hd]
+  const uint16_t *vcache;
+  const int *positions;
+  float *o;                  // [batch][ldo]
+  int ldo;
+  float *partial;            // [batch][Hkv][n_chunks][G][hd + 2]
+  int *tickets;              // [batch][Hkv]
+  int batch, n_heads, n_kv_heads, max_ctx, chunk, n_chunks;
+  float scale_log2;          // log2(e) / sqrt(hd)
+  unsigned *err;
+};
+
+// ---- PTX helpers --------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait on an mbarrier phase; false after WAIT_LIMIT polls.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+  for (uint32_t i = 0; i < WAIT_LIMIT; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (i >= WAIT_FAST_SPINS) __nanosleep(64);
+  }
+  return false;
+}
+
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
+// 1-D bulk copy global -> shared (TMA), completion counted in bytes on `bar`.
+// dst, src 16-byte aligned; bytes a multiple of 16.
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar,
+                                         uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1], %2, [%3], %4;" ::"r"(dst),
+      "l"(src), "r"(bytes), "r"(bar), "l"(policy)
+      : "memory");
+}
+
+// Programmatic dependent launch (PDL)
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+__device__ __forceinline__ void named_bar_sync(int id, int n) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t u) { return __uint_as_float(u << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t u) { return __uint_as_float(u & 0xFFFF0000u); }
+__device__ __forceinline__ float bf16_to_f32(uint16_t b) { return __uint_as_float(uint32_t(b) << 16); }
+
+// fp32 -> bf16, round to nearest even (NaN -> quiet NaN)
+__device__ __forceinline__ uint16_t f32_to_bf16_rne(float f) {
+  uint32_t u = __float_as_uint(f);
+  if ((u & 0x7FFFFFFFu) > 0x7F800000u) return 0x7FC0;
+  u += 0x7FFFu + ((u >> 16) & 1u);
+  return static_cast<uint16_t>(u >> 16);
+}
+
+__device__ __forceinline__ float ld_cg(const float *p) { return __ldcg(p); }
+
+}  // namespace kfl
+
+// Kernel launchers (defined in the .cu files; used by the runtime).
+namespace kfl {
+cudaError_t prepare_gemv();
+cudaError_t prepare_attention();
+cudaError_t launch_gemv(const GemvParams &p, int epi, int grid, cudaStream_t s, bool pdl);
+cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s, bool pdl);
+cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in,
+                               int batch, const uint16_t *embed, int vocab, int d, int ldh,
+                               const float *g_next, float *h, float *xn, float *sumsq,
+                               int *positions, int max_ctx, unsigned *err, cudaStream_t s);
+cudaError_t launch_stage_output(const float *h, int ldh, int d, int batch, float *hidden_out,
+                                const int *next_in, int *next_ids, cudaStream_t s, bool pdl);
+cudaError_t launch_repack_bf16(const uint16_t *src, int n_src_rows, int k, const int *row_map,
+                               int n_rows_out, int n_rb, int n_kt, uint8_t *dst, cudaStream_t s);
+cudaError_t launch_repack_int4(const uint32_t *words, const uint16_t *scales, int n_src_rows, int k,
+                               const int *row_map, int n_rows_out, int n_rb, int n_kt, uint8_t *dst,
+                               cudaStream_t s);
+cudaError_t launch_bf16_to_f32(const uint16_t *src, float *dst, int n, cudaStream_t s);
+}  // namespace kfl

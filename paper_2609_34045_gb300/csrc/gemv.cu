@@ -1,0 +1,502 @@
+// Weight-streaming GEMV y[b] = W . x[b] for batch 1..4 on sm_103a.
+//
+// Decode at batch one is memory-bandwidth bound: a stage reads each of its weights once per
+// token and does two flops per weight (Kafila, section V-A, Eq. 2).  So the kernel is built
+// around one thing, keeping HBM busy:
+//
+//   * weights are pre-tiled at load time ([N/64][K/128][64][128] bf16), so each 16 KiB tile is
+//     one contiguous HBM chunk;
+//   * the grid is persistent (one CTA per SM) and split "stream-K" style: CTA c streams the
+//     contiguous tile range [c*T/G, (c+1)*T/G) of the flattened tile sequence, so every SM
+//     moves the same number of bytes whatever the matrix shape;
+//   * one producer thread per CTA feeds a ring of shared-memory stages with 1-D TMA bulk
+//     copies (cp.async.bulk + mbarrier complete_tx); eight consumer warps read tiles and the
+//     matching fp32 activation chunks from shared memory and accumulate in fp32;
+//   * under programmatic dependent launch the producer starts streaming weights, which do not
+//     depend on the previous kernel, before griddepcontrol.wait, hiding launch and tail gaps;
+//   * row blocks split between CTAs are combined deterministically: each CTA writes its partial
+//     sums, the last to arrive (atomic ticket, no spin) adds them in CTA order;
+//   * epilogues are fused: RoPE + KV append, residual add + next RMSNorm input + sum of squares,
+//     SwiGLU, greedy argmax.
+#include "common.cuh"
+
+#include <math.h>
+
+namespace kfl {
+
+__device__ __forceinline__ int cta_of_tile(long long t, long long T, int G) {
+  // the largest c with floor(c*T/G) <= t
+  return static_cast<int>(((t + 1) * G - 1) / T);
+}
+
+__device__ __forceinline__ bool consumer_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag,
+                                              unsigned *err) {
+  if (*abort_flag) return false;
+  for (uint32_t i = 0; i < WAIT_LIMIT; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (i >= WAIT_FAST_SPINS) {
+      if (*abort_flag) return false;
+      __nanosleep(64);
+    }
+  }
+  *abort_flag = 1;
+  atomicOr(err, ERR_TIMEOUT);
+  return false;
+}
+
+// ---------------------------------------------------------------------------- epilogues
+// red[r * MAXB + b] holds the finished dot product of row rb*RB + r for user b (before the
+// RMSNorm scale inv[b]).  Called by the 256 consumer threads; every thread reaches every
+// barrier.
+template <int B, int EPI>
+__device__ __forceinline__ void epilogue(const GemvParams &p, int rb, const float *red, const float *inv,
+                                         float *scr, int tid) {
+  const int warp = tid >> 5, lane = tid & 31;
+  if constexpr (EPI == EPI_STORE) {
+    if (tid < RB * B) {
+      const int b = tid / RB, r = tid % RB, n = rb * RB + r;
+      if (n < p.n_rows) p.out[(size_t)b * p.ldo + n] = red[r * MAXB + b] * inv[b];
+    }
+  } else if constexpr (EPI == EPI_RESID) {
+    float sq = 0.f;
+    if (tid < RB * B) {
+      const int b = tid >> 6, r = tid & 63, n = rb * RB + r;
+      if (n < p.n_rows) {
+        const size_t o = (size_t)b * p.ldh + n;
+        const float hn = p.h[o] + red[r * MAXB + b] * inv[b];
+        p.h[o] = hn;
+        if (p.g_next) p.xn[o] = hn * p.g_next[n];
+        if (p.capture) p.capture[(size_t)b * p.n_rows + n] = hn;
+        sq = hn * hn;
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
+    if (lane == 0) scr[warp] = sq;
+    named_bar_sync(1, CONSUMER_WARPS * 32);
+    if (tid < B) p.sumsq_out[rb * MAXB + tid] = scr[2 * tid] + scr[2 * tid + 1];
+  } else if constexpr (EPI == EPI_SWIGLU) {
+    if (tid < 32 * B) {
+      const int b = tid >> 5, pr = tid & 31, j = rb * (RB / 2) + pr;
+      if (2 * j < p.n_rows) {
+        const float g = red[(2 * pr) * MAXB + b] * inv[b];
+        const float u = red[(2 * pr + 1) * MAXB + b] * inv[b];
+        p.out[(size_t)b * p.ldo + j] = g / (1.0f + expf(-g)) * u;
+      }
+    }
+  } else if constexpr (EPI == EPI_QKV) {
+    if (tid < 32 * B) {
+      const int b = tid >> 5, pr = tid & 31, r0 = rb * RB + 2 * pr;
+      int pos = p.positions[b];
+      const bool ok = pos >= 0 && pos < p.max_ctx;
+      if (!ok) pos = 0;
+      if (r0 < p.n_rows) {
+        const int hd = p.head_dim, half = hd >> 1;
+        const float v1 = red[(2 * pr) * MAXB + b] * inv[b];
+        const float v2 = red[(2 * pr + 1) * MAXB + b] * inv[b];
+        if (r0 < p.n_q_rows + p.n_kv_rows) {
+          const bool is_q = r0 < p.n_q_rows;
+          const int rr = is_q ? r0 : r0 - p.n_q_rows;
+          const int head = rr / hd, i = (rr % hd) >> 1;
+          const float cs = p.rope_cos[(size_t)pos * half + i];
+          const float sn = p.rope_sin[(size_t)pos * half + i];
+          const float a = v1 * cs - v2 * sn;
+          const float c = v2 * cs + v1 * sn;
+          if (is_q) {
+            float *qd = p.q + (size_t)b * p.n_q_rows + head * hd;
+            qd[i] = a;
+            qd[i + half] = c;
+          } else if (ok) {
+            uint16_t *kd = p.kcache + (((size_t)b * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
+            kd[i] = f32_to_bf16_rne(a);
+            kd[i + half] = f32_to_bf16_rne(c);
+          }
+        } else if (ok) {
+          const int rr = r0 - p.n_q_rows - p.n_kv_rows;
+          const int head = rr / hd, j = rr % hd;
+          uint16_t *vd = p.vcache + (((size_t)b * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
+          vd[j] = f32_to_bf16_rne(v1);
+          vd[j + 1] = f32_to_bf16_rne(v2);
+        }
+      }
+    }
+  } else if constexpr (EPI == EPI_ARGMAX) {
+    int *scri = reinterpret_cast<int *>(scr + CONSUMER_WARPS);
+    __shared__ int s_last_am;
+    float v = -INFINITY;
+    int idx = 0x7fffffff;
+    if (tid < RB * B) {
+      const int b = tid >> 6, r = tid & 63, n = rb * RB + r;
+      if (n < p.n_rows) {
+        v = red[r * MAXB + b] * inv[b];
+        idx = n;
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, v, off);
+      const int oi = __shfl_xor_sync(0xffffffffu, idx, off);
+      if (ov > v || (ov == v && oi < idx)) { v = ov; idx = oi; }
+    }
+    if (lane == 0) { scr[warp] = v; scri[warp] = idx; }
+    named_bar_sync(1, CONSUMER_WARPS * 32);
+    if (tid < B) {
+      float bv = scr[2 * tid];
+      int bi = scri[2 * tid];
+      const float ov = scr[2 * tid + 1];
+      const int oi = scri[2 * tid + 1];
+      if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
+      p.cand_val[rb * MAXB + tid] = bv;
+      p.cand_idx[rb * MAXB + tid] = bi;
+      __threadfence();
+    }
+    named_bar_sync(1, CONSUMER_WARPS * 32);
+    if (tid == 0) {
+      const int prev = atomicAdd(p.argmax_ticket, 1);
+      s_last_am = (prev == p.n_rb - 1);
+      if (s_last_am) atomicExch(p.argmax_ticket, 0);
+    }
+    named_bar_sync(1, CONSUMER_WARPS * 32);
+    if (s_last_am) {
+      __threadfence();
+      for (int b = 0; b < B; ++b) {
+        float bv = -INFINITY;
+        int bi = 0x7fffffff;
+        for (int r = tid; r < p.n_rb; r += CONSUMER_WARPS * 32) {
+          const float ov = __ldcg(p.cand_val + r * MAXB + b);
+          const int oi = __ldcg(p.cand_idx + r * MAXB + b);
+          if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+          const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+          const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+          if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
+        }
+        named_bar_sync(1, CONSUMER_WARPS * 32);
+        if (lane == 0) { scr[warp] = bv; scri[warp] = bi; }
+        named_bar_sync(1, CONSUMER_WARPS * 32);
+        if (tid == 0) {
+          bv = scr[0];
+          bi = scri[0];
+          for (int w = 1; w < CONSUMER_WARPS; ++w) {
+            if (scr[w] > bv || (scr[w] == bv && scri[w] < bi)) { bv = scr[w]; bi = scri[w]; }
+          }
+          p.next_ids[b] = (bi == 0x7fffffff) ? 0 : bi;
+        }
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------- the kernel
+// FMT 0: bf16 tiles [RB][KT].  FMT 1: int4 tiles, codes [RB][KT4/8] uint32 + scales [RB][KT4/64].
+template <int B, int EPI, int FMT>
+__global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const __grid_constant__ GemvParams p) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  const int S = p.stages;
+  uint64_t *full = reinterpret_cast<uint64_t *>(smem + (size_t)S * STAGE_BYTES);
+  uint64_t *empty = full + S;
+  float *red = reinterpret_cast<float *>(empty + S);  // [RB][MAXB]
+  float *scr = red + RB * MAXB;                       // 2 * CONSUMER_WARPS words
+  __shared__ float s_inv[MAXB];
+  __shared__ int s_last;
+  __shared__ volatile int s_abort;
+  __shared__ int s_issued;
+
+  constexpr int KTILE = FMT == 0 ? KT : KT4;
+  constexpr uint32_t WBYTES = FMT == 0 ? TILE_BYTES : TILE4_BYTES;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const long long T = (long long)p.n_rb * p.n_kt;
+  const int G = gridDim.x, c = blockIdx.x;
+  const long long t0 = (long long)c * T / G, t1 = (long long)(c + 1) * T / G;
+  const int n = static_cast<int>(t1 - t0);
+
+  if (tid == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(smem_addr(&full[s]), 1);
+      mbar_init(smem_addr(&empty[s]), CONSUMER_WARPS);
+    }
+    s_abort = 0;
+    s_issued = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  pdl_launch_dependents();
+
+  if (warp == CONSUMER_WARPS) {
+    // ------------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint64_t pol_w = policy_evict_first();
+      const uint64_t pol_x = policy_evict_last();
+      const uint32_t xbytes = B * (KTILE * 4);
+      const int pre = n < S ? n : S;
+      for (int i = 0; i < pre; ++i) {
+        const uint32_t fb = smem_addr(&full[i]);
+        mbar_arrive_expect_tx(fb, WBYTES + xbytes);
+        bulk_g2s(smem_addr(smem + (size_t)i * STAGE_BYTES), p.w + (size_t)(t0 + i) * WBYTES, WBYTES, fb, pol_w);
+      }
+      pdl_wait();
+      auto issue_x = [&](int i, int s) {
+        const long long t = t0 + i;
+        const int kt = static_cast<int>(t % p.n_kt);
+        const uint32_t fb = smem_addr(&full[s]);
+        const uint32_t dst = smem_addr(smem + (size_t)s * STAGE_BYTES + WBYTES);
+#pragma unroll
+        for (int b = 0; b < B; ++b)
+          bulk_g2s(dst + b * (KTILE * 4), p.x + (size_t)b * p.ldx + (size_t)kt * KTILE, KTILE * 4, fb, pol_x);
+      };
+      for (int i = 0; i < pre; ++i) issue_x(i, i);
+      int issued = pre;
+      for (int i = pre; i < n; ++i) {
+        const int s = i % S;
+        const uint32_t par = ((i / S) - 1) & 1;
+        if (!consumer_wait(smem_addr(&empty[s]), par, &s_abort, p.err)) break;
+        const uint32_t fb = smem_addr(&full[s]);
+        mbar_arrive_expect_tx(fb, WBYTES + xbytes);
+        bulk_g2s(smem_addr(smem + (size_t)s * STAGE_BYTES), p.w + (size_t)(t0 + i) * WBYTES, WBYTES, fb, pol_w);
+        issue_x(i, s);
+        issued = i + 1;
+      }
+      s_issued = issued;
+    }
+    return;
+  }
+
+  // -------------------------------------------------------------------- consumers
+  pdl_wait();
+  if (tid < B) {
+    float inv = 1.0f;
+    if (p.sumsq) {
+      float s = 0.f;
+      for (int i = 0; i < p.n_parts; ++i) s += p.sumsq[i * MAXB + tid];
+      inv = 1.0f / sqrtf(s / static_cast<float>(p.d_norm) + p.eps);
+    }
+    s_inv[tid] = inv;
+  }
+  named_bar_sync(1, CONSUMER_WARPS * 32);
+
+  // bf16: lane -> 8 consecutive K (chunk kc) of rows warp*8 + rsub + 2j, j < 4
+  // int4: lane -> 16 consecutive K (chunk kc) of the same rows
+  const int kc = lane & 15, rsub = lane >> 4;
+  float acc[B][4];
+  int seg_kt0 = 0;
+  for (int i = 0; i < n; ++i) {
+    const long long t = t0 + i;
+    const int rb = static_cast<int>(t / p.n_kt);
+    const int kt = static_cast<int>(t - (long long)rb * p.n_kt);
+    if (i == 0 || kt == 0) {
+#pragma unroll
+      for (int b = 0; b < B; ++b)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[b][j] = 0.f;
+      seg_kt0 = kt;
+    }
+    const int s = i % S;
+    consumer_wait(smem_addr(&full[s]), (i / S) & 1, &s_abort, p.err);
+    const uint8_t *st = smem + (size_t)s * STAGE_BYTES;
+    if constexpr (FMT == 0) {
+      float xv[B][8];
+      const float4 *xp = reinterpret_cast<const float4 *>(st + TILE_BYTES) + kc * 2;
+#pragma unroll
+      for (int b = 0; b < B; ++b) {
+        const float4 a0 = xp[b * (KT / 4)], a1 = xp[b * (KT / 4) + 1];
+        xv[b][0] = a0.x; xv[b][1] = a0.y; xv[b][2] = a0.z; xv[b][3] = a0.w;
+        xv[b][4] = a1.x; xv[b][5] = a1.y; xv[b][6] = a1.z; xv[b][7] = a1.w;
+      }
+      const uint4 *wp = reinterpret_cast<const uint4 *>(st) + (warp * 8 + rsub) * (KT / 8) + kc;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint4 w4 = wp[j * 2 * (KT / 8)];
+        float w[8];
+        w[0] = bf16_lo(w4.x); w[1] = bf16_hi(w4.x); w[2] = bf16_lo(w4.y); w[3] = bf16_hi(w4.y);
+        w[4] = bf16_lo(w4.z); w[5] = bf16_hi(w4.z); w[6] = bf16_lo(w4.w); w[7] = bf16_hi(w4.w);
+#pragma unroll
+        for (int b = 0; b < B; ++b)
+#pragma unroll
+          for (int e = 0; e < 8; ++e) acc[b][j] = fmaf(w[e], xv[b][e], acc[b][j]);
+      }
+    } else {
+      // int4 tile: codes [RB][KT4/8] uint32 (32 words = 128 B per row), scales [RB][4] bf16
+      const float4 *xp = reinterpret_cast<const float4 *>(st + TILE4_BYTES) + kc * 4;
+      float xv[B][16];
+#pragma unroll
+      for (int b = 0; b < B; ++b) {
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          const float4 a = xp[b * (KT4 / 4) + v];
+          xv[b][4 * v] = a.x; xv[b][4 * v + 1] = a.y; xv[b][4 * v + 2] = a.z; xv[b][4 * v + 3] = a.w;
+        }
+      }
+      const uint2 *cp = reinterpret_cast<const uint2 *>(st) + (warp * 8 + rsub) * (KT4 / 16) + kc;
+      const uint16_t *sp = reinterpret_cast<const uint16_t *>(st + TILE4_CODE_BYTES);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int r = warp * 8 + rsub + 2 * j;
+        const uint2 cw = cp[j * 2 * (KT4 / 16)];
+        const float sc = bf16_to_f32(sp[r * (KT4 / 64) + (kc >> 2)]);
+        float part[B];
+#pragma unroll
+        for (int b = 0; b < B; ++b) part[b] = 0.f;
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          const uint32_t word = e < 8 ? cw.x : cw.y;
+          const int q = static_cast<int>(word << (28 - 4 * (e & 7))) >> 28;  // sign-extended nibble
+          const float wq = static_cast<float>(q);
+#pragma unroll
+          for (int b = 0; b < B; ++b) part[b] = fmaf(wq, xv[b][e], part[b]);
+        }
+#pragma unroll
+        for (int b = 0; b < B; ++b) acc[b][j] = fmaf(sc, part[b], acc[b][j]);
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_addr(&empty[s]));
+
+    if (kt == p.n_kt - 1 || i == n - 1) {
+      // ---- segment end: reduce over the 16 lanes sharing a row
+#pragma unroll
+      for (int b = 0; b < B; ++b)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          float v = acc[b][j];
+          v += __shfl_xor_sync(0xffffffffu, v, 8);
+          v += __shfl_xor_sync(0xffffffffu, v, 4);
+          v += __shfl_xor_sync(0xffffffffu, v, 2);
+          v += __shfl_xor_sync(0xffffffffu, v, 1);
+          acc[b][j] = v;
+        }
+      if (kc == 0) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+#pragma unroll
+          for (int b = 0; b < B; ++b) red[(warp * 8 + rsub + 2 * j) * MAXB + b] = acc[b][j];
+      }
+      named_bar_sync(1, CONSUMER_WARPS * 32);
+      bool do_epi = true;
+      if (!(seg_kt0 == 0 && kt == p.n_kt - 1)) {
+        // this row block is shared with neighbouring CTAs
+        const int first_rb = static_cast<int>(t0 / p.n_kt);
+        const int slot = (rb == first_rb) ? 0 : 1;
+        float *mine = p.partial + (size_t)(c * 2 + slot) * (RB * MAXB);
+        for (int e = tid; e < RB * MAXB; e += CONSUMER_WARPS * 32) mine[e] = red[e];
+        __threadfence();
+        named_bar_sync(1, CONSUMER_WARPS * 32);
+        const int c_lo = cta_of_tile((long long)rb * p.n_kt, T, G);
+        const int c_hi = cta_of_tile((long long)(rb + 1) * p.n_kt - 1, T, G);
+        if (tid == 0) {
+          const int prev = atomicAdd(p.tickets + rb, 1);
+          s_last = (prev == c_hi - c_lo);
+          if (s_last) atomicExch(p.tickets + rb, 0);
+        }
+        named_bar_sync(1, CONSUMER_WARPS * 32);
+        do_epi = s_last != 0;
+        if (do_epi) {
+          __threadfence();
+          for (int e = tid; e < RB * MAXB; e += CONSUMER_WARPS * 32) {
+            float sum = 0.f;
+            for (int cc = c_lo; cc <= c_hi; ++cc) {
+              const int frb = static_cast<int>(((long long)cc * T / G) / p.n_kt);
+              const int sl = (rb == frb) ? 0 : 1;
+              sum += __ldcg(p.partial + (size_t)(cc * 2 + sl) * (RB * MAXB) + e);
+            }
+            red[e] = sum;
+          }
+          named_bar_sync(1, CONSUMER_WARPS * 32);
+        }
+      }
+      if (do_epi) epilogue<B, EPI>(p, rb, red, s_inv, scr, tid);
+      named_bar_sync(1, CONSUMER_WARPS * 32);
+    }
+  }
+
+  if (s_abort && tid == 0) {
+    // drain copies still in flight before the CTA's shared memory goes away (bounded)
+    const int issued = s_issued;
+    for (int i = (issued > S ? issued - S : 0); i < issued; ++i)
+      mbar_wait(smem_addr(&full[i % S]), (i / S) & 1);
+  }
+}
+
+// ---------------------------------------------------------------------------- launch
+static size_t gemv_smem_bytes(int stages) {
+  return (size_t)stages * STAGE_BYTES + 2 * stages * sizeof(uint64_t) + (RB * MAXB + 2 * CONSUMER_WARPS) * sizeof(float);
+}
+
+template <int B, int EPI, int FMT>
+static cudaError_t launch_one(const GemvParams &p, int grid, cudaStream_t s, bool pdl) {
+  cudaLaunchConfig_t cfg = {};
+  const size_t smem = gemv_smem_bytes(p.stages);
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(GEMV_THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, gemv_kernel<B, EPI, FMT>, p);
+}
+
+template <int EPI, int FMT>
+static cudaError_t launch_b(const GemvParams &p, int grid, cudaStream_t s, bool pdl) {
+  switch (p.batch) {
+    case 1: return launch_one<1, EPI, FMT>(p, grid, s, pdl);
+    case 2: return launch_one<2, EPI, FMT>(p, grid, s, pdl);
+    case 3: return launch_one<3, EPI, FMT>(p, grid, s, pdl);
+    case 4: return launch_one<4, EPI, FMT>(p, grid, s, pdl);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+template <int FMT>
+static cudaError_t launch_f(const GemvParams &p, int epi, int grid, cudaStream_t s, bool pdl) {
+  switch (epi) {
+    case EPI_STORE: return launch_b<EPI_STORE, FMT>(p, grid, s, pdl);
+    case EPI_QKV: return launch_b<EPI_QKV, FMT>(p, grid, s, pdl);
+    case EPI_RESID: return launch_b<EPI_RESID, FMT>(p, grid, s, pdl);
+    case EPI_SWIGLU: return launch_b<EPI_SWIGLU, FMT>(p, grid, s, pdl);
+    case EPI_ARGMAX: return launch_b<EPI_ARGMAX, FMT>(p, grid, s, pdl);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+template <int B, int EPI, int FMT>
+static cudaError_t prepare_one() {
+  return cudaFuncSetAttribute(gemv_kernel<B, EPI, FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)gemv_smem_bytes(MAX_STAGES));
+}
+
+template <int EPI, int FMT>
+static cudaError_t prepare_b() {
+  cudaError_t e;
+  if ((e = prepare_one<1, EPI, FMT>()) != cudaSuccess) return e;
+  if ((e = prepare_one<2, EPI, FMT>()) != cudaSuccess) return e;
+  if ((e = prepare_one<3, EPI, FMT>()) != cudaSuccess) return e;
+  return prepare_one<4, EPI, FMT>();
+}
+
+template <int FMT>
+static cudaError_t prepare_f() {
+  cudaError_t e;
+  if ((e = prepare_b<EPI_STORE, FMT>()) != cudaSuccess) return e;
+  if ((e = prepare_b<EPI_QKV, FMT>()) != cudaSuccess) return e;
+  if ((e = prepare_b<EPI_RESID, FMT>()) != cudaSuccess) return e;
+  if ((e = prepare_b<EPI_SWIGLU, FMT>()) != cudaSuccess) return e;
+  return prepare_b<EPI_ARGMAX, FMT>();
+}
+
+// Raise the dynamic shared-memory limit of every GEMV instantiation (once per device, before
+// any launch or stream capture).
+cudaError_t prepare_gemv() {
+  cudaError_t e = prepare_f<0>();
+  return e != cudaSuccess ? e : prepare_f<1>();
+}
+
+cudaError_t launch_gemv(const GemvParams &p, int epi, int grid, cudaStream_t s, bool pdl) {
+  if (p.stages < 2 || p.stages > MAX_STAGES) return cudaErrorInvalidValue;
+  return p.fmt == 0 ? launch_f<0>(p, epi, grid, s, pdl) : launch_f<1>(p, epi, grid, s, pdl);
+}
+
+}  // namespace kfl

@@ -1,0 +1,167 @@
+// Stage input/output and load-time kernels.
+#include "common.cuh"
+
+namespace kfl {
+
+// Stage input (Kafila section III: the head embeds the token; other members receive the
+// hidden state from the previous ring member).  One CTA of 64 threads per (64-row block,
+// user): writes h, the next RMSNorm input xn = h * g_next and the block's sum of squares,
+// and copies/validates the positions.
+__global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const float *hidden_in,
+                                                         const int *positions_in, const uint16_t *embed,
+                                                         int vocab, int d, int ldh, const float *g_next,
+                                                         float *h, float *xn, float *sumsq, int *positions,
+                                                         int max_ctx, unsigned *err) {
+  __shared__ float part[2];
+  const int b = blockIdx.y, tid = threadIdx.x, r = blockIdx.x * 64 + tid;
+  pdl_launch_dependents();
+  pdl_wait();
+  if (blockIdx.x == 0 && tid == 0) {
+    const int pos = positions_in[b];
+    if (pos < 0 || pos >= max_ctx) atomicOr(err, ERR_POSITION);
+    positions[b] = pos;
+  }
+  float v = 0.f;
+  if (r < d) {
+    if (embed) {
+      int id = ids[b];
+      if (id < 0 || id >= vocab) {
+        if (tid == 0 && blockIdx.x == 0) atomicOr(err, ERR_TOKEN);
+        id = 0;
+      }
+      v = bf16_to_f32(embed[(size_t)id * d + r]);
+    } else {
+      v = hidden_in[(size_t)b * d + r];
+    }
+    h[(size_t)b * ldh + r] = v;
+    if (g_next) xn[(size_t)b * ldh + r] = v * g_next[r];
+  }
+  float sq = v * v;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
+  if ((tid & 31) == 0) part[tid >> 5] = sq;
+  __syncthreads();
+  if (tid == 0) sumsq[blockIdx.x * MAXB + b] = part[0] + part[1];
+}
+
+cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in, int batch,
+                               const uint16_t *embed, int vocab, int d, int ldh, const float *g_next, float *h,
+                               float *xn, float *sumsq, int *positions, int max_ctx, unsigned *err,
+                               cudaStream_t s) {
+  dim3 grid((d + 63) / 64, batch);
+  stage_input_kernel<<<grid, 64, 0, s>>>(ids, hidden_in, positions_in, embed, vocab, d, ldh, g_next, h, xn, sumsq,
+                                         positions, max_ctx, err);
+  return cudaGetLastError();
+}
+
+__global__ void stage_output_kernel(const float *h, int ldh, int d, float *hidden_out, const int *next_in,
+                                    int *next_ids) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int b = blockIdx.y;
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (hidden_out && r < d) hidden_out[(size_t)b * d + r] = h[(size_t)b * ldh + r];
+  if (next_ids && blockIdx.x == 0 && threadIdx.x == 0) next_ids[b] = next_in[b];
+}
+
+cudaError_t launch_stage_output(const float *h, int ldh, int d, int batch, float *hidden_out, const int *next_in,
+                                int *next_ids, cudaStream_t s, bool pdl) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((d + 255) / 256, batch);
+  cfg.blockDim = dim3(256);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, stage_output_kernel, h, ldh, d, hidden_out, next_in, next_ids);
+}
+
+// Repack a bf16 matrix src [n_src_rows][k] into tiles [n_rb][n_kt][RB][KT]: output row r is
+// source row row_map[r] (or r when row_map is NULL); rows >= n_rows_out and columns >= k are 0.
+__global__ void repack_bf16_kernel(const uint16_t *src, int n_src_rows, int k, const int *row_map, int n_rows_out,
+                                   int n_rb, int n_kt, uint8_t *dst) {
+  const long long total = (long long)n_rb * n_kt * RB * (KT / 8);
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int ch = static_cast<int>(e % (KT / 8));
+    const long long rest = e / (KT / 8);
+    const int r = static_cast<int>(rest % RB);
+    const long long t = rest / RB;
+    const int kt = static_cast<int>(t % n_kt);
+    const int rb = static_cast<int>(t / n_kt);
+    const int orow = rb * RB + r;
+    int srow = -1;
+    if (orow < n_rows_out) srow = row_map ? row_map[orow] : orow;
+    if (srow >= n_src_rows) srow = -1;
+    const int k0 = kt * KT + ch * 8;
+    uint16_t v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) v[j] = (srow >= 0 && k0 + j < k) ? src[(size_t)srow * k + k0 + j] : uint16_t(0);
+    uint4 o;
+    o.x = v[0] | (uint32_t(v[1]) << 16);
+    o.y = v[2] | (uint32_t(v[3]) << 16);
+    o.z = v[4] | (uint32_t(v[5]) << 16);
+    o.w = v[6] | (uint32_t(v[7]) << 16);
+    reinterpret_cast<uint4 *>(dst)[e] = o;
+  }
+}
+
+cudaError_t launch_repack_bf16(const uint16_t *src, int n_src_rows, int k, const int *row_map, int n_rows_out,
+                               int n_rb, int n_kt, uint8_t *dst, cudaStream_t s) {
+  repack_bf16_kernel<<<4 * 152 * 4, 256, 0, s>>>(src, n_src_rows, k, row_map, n_rows_out, n_rb, n_kt, dst);
+  return cudaGetLastError();
+}
+
+// Repack an int4 group-64 matrix (words [n_src_rows][k/8], scales [n_src_rows][k/64]) into
+// tiles [n_rb][n_kt][RB][KT4/8 words] followed by [RB][KT4/64] bf16 scales per tile.
+__global__ void repack_int4_kernel(const uint32_t *words, const uint16_t *scales, int n_src_rows, int k,
+                                   const int *row_map, int n_rows_out, int n_rb, int n_kt, uint8_t *dst) {
+  constexpr int WPR = KT4 / 8;   // words per tile row
+  constexpr int SPR = KT4 / 64;  // scales per tile row
+  const long long total = (long long)n_rb * n_kt * RB;
+  const int kw = k / 8, ks = k / 64;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int r = static_cast<int>(e % RB);
+    const long long t = e / RB;
+    const int kt = static_cast<int>(t % n_kt);
+    const int rb = static_cast<int>(t / n_kt);
+    const int orow = rb * RB + r;
+    int srow = -1;
+    if (orow < n_rows_out) srow = row_map ? row_map[orow] : orow;
+    if (srow >= n_src_rows) srow = -1;
+    uint8_t *tile = dst + (size_t)t * TILE4_BYTES;
+    uint32_t *wd = reinterpret_cast<uint32_t *>(tile) + r * WPR;
+    uint16_t *sd = reinterpret_cast<uint16_t *>(tile + TILE4_CODE_BYTES) + r * SPR;
+    for (int j = 0; j < WPR; ++j) {
+      const int w = kt * WPR + j;
+      wd[j] = (srow >= 0 && w < kw) ? words[(size_t)srow * kw + w] : 0u;
+    }
+    for (int j = 0; j < SPR; ++j) {
+      const int g = kt * SPR + j;
+      sd[j] = (srow >= 0 && g < ks) ? scales[(size_t)srow * ks + g] : uint16_t(0);
+    }
+  }
+}
+
+cudaError_t launch_repack_int4(const uint32_t *words, const uint16_t *scales, int n_src_rows, int k,
+                               const int *row_map, int n_rows_out, int n_rb, int n_kt, uint8_t *dst,
+                               cudaStream_t s) {
+  repack_int4_kernel<<<4 * 152, 256, 0, s>>>(words, scales, n_src_rows, k, row_map, n_rows_out, n_rb, n_kt, dst);
+  return cudaGetLastError();
+}
+
+__global__ void bf16_to_f32_kernel(const uint16_t *src, float *dst, int n) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
+    dst[i] = bf16_to_f32(src[i]);
+}
+
+cudaError_t launch_bf16_to_f32(const uint16_t *src, float *dst, int n, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  bf16_to_f32_kernel<<<(n + 255) / 256 < 1024 ? (n + 255) / 256 : 1024, 256, 0, s>>>(src, dst, n);
+  return cudaGetLastError();
+}
+
+}  // namespace kfl

@@ -1,0 +1,947 @@
+// Stage runtime and C ABI (kafila_stage.h).
+//
+// A stage owns its repacked weights, its KV cache (reserved at max_ctx x max_batch, the
+// declared context and concurrency of Kafila section V-C/V-D) and a small workspace.  A decode
+// step is: stage input kernel -> one CUDA graph of the block kernels (captured once per batch
+// size, kernels chained with programmatic dependent launch) -> stage output kernel.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <vector>
+
+#include "../../include/kafila_stage.h"
+#include "../../include/kafila_synth.h"
+#include "common.cuh"
+
+using namespace kfl;
+
+namespace {
+
+int round_up(int x, int m) { return (x + m - 1) / m * m; }
+
+struct Mat {
+  uint8_t *tiles = nullptr;
+  int N = 0, K = 0, n_rb = 0, n_kt = 0, fmt = 0;
+  size_t bytes = 0;
+};
+
+Mat mat_shape(int N, int K, int fmt) {
+  Mat m;
+  m.N = N;
+  m.K = K;
+  m.fmt = fmt;
+  m.n_rb = (N + RB - 1) / RB;
+  const int kt = fmt == KFL_BF16 ? KT : KT4;
+  m.n_kt = (K + kt - 1) / kt;
+  m.bytes = (size_t)m.n_rb * m.n_kt * (fmt == KFL_BF16 ? TILE_BYTES : TILE4_BYTES);
+  return m;
+}
+
+struct LayerDev {
+  Mat qkv, o, gu, down;
+  float *g_attn = nullptr, *g_ffn = nullptr;
+  bool loaded = false;
+};
+
+// Every size the stage allocates, computed once for kfl_stage_memory_bytes and create.
+struct Plan {
+  int d, hq, hkv, hd, F, V, qdim, kvdim, nl;
+  int ldh, ldq, lda;  // activation row strides, multiples of 256 floats
+  Mat qkv, o, gu, down, lm;
+  size_t kv_elems_per_layer;  // per cache (K or V)
+  int n_sm, ctas_per_sm, stages, gemv_grid_max, n_rb_max, n_parts, attn_nchunks_max;
+  size_t bytes_weights, bytes_kv, bytes_ws;
+};
+
+int env_int(const char *name, int dflt) {
+  const char *v = std::getenv(name);
+  return (v && *v) ? std::atoi(v) : dflt;
+}
+
+int validate_cfg(const kfl_model_cfg *c, int l0, int l1, int flags) {
+  if (!c) return KFL_ERR_ARG;
+  if (c->n_layers_total <= 0 || c->d_model <= 0 || c->n_heads <= 0 || c->n_kv_heads <= 0 || c->head_dim <= 0 ||
+      c->ffn <= 0 || c->vocab <= 0)
+    return KFL_ERR_ARG;
+  if (c->n_heads % c->n_kv_heads != 0 || c->n_heads / c->n_kv_heads > 8) return KFL_ERR_ARG;
+  if (c->head_dim != 64 && c->head_dim != 128) return KFL_ERR_ARG;
+  if (c->d_model % 8 != 0 || c->ffn % 8 != 0) return KFL_ERR_ARG;
+  if (c->weight_fmt != KFL_BF16 && c->weight_fmt != KFL_INT4_G64) return KFL_ERR_ARG;
+  if (c->weight_fmt == KFL_INT4_G64 &&
+      (c->d_model % 64 != 0 || c->ffn % 64 != 0 || (c->n_heads * c->head_dim) % 64 != 0))
+    return KFL_ERR_ARG;
+  if (c->max_ctx <= 0 || c->max_batch <= 0 || c->max_batch > MAXB) return KFL_ERR_ARG;
+  if (c->max_ctx > (1 << 20)) return KFL_ERR_ARG;
+  if (c->qk_norm != 0) return KFL_ERR_ARG;
+  if (!(c->rms_eps > 0.f) || !(c->rope_theta > 0.f)) return KFL_ERR_ARG;
+  if (l0 < 0 || l1 < l0 || l1 > c->n_layers_total) return KFL_ERR_ARG;
+  if (flags & ~KFL_IS_HEAD) return KFL_ERR_ARG;
+  if (l0 == l1 && !(flags & KFL_LOGITS_OUT) && !(flags & KFL_EMBED_IN)) return KFL_ERR_ARG;
+  return KFL_OK;
+}
+
+void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan *p) {
+  p->d = c->d_model;
+  p->hq = c->n_heads;
+  p->hkv = c->n_kv_heads;
+  p->hd = c->head_dim;
+  p->F = c->ffn;
+  p->V = c->vocab;
+  p->qdim = p->hq * p->hd;
+  p->kvdim = p->hkv * p->hd;
+  p->nl = l1 - l0;
+  p->ldh = round_up(p->d, 256);
+  p->ldq = round_up(p->qdim, 256);
+  p->lda = round_up(p->F, 256);
+  const int f = c->weight_fmt;
+  p->qkv = mat_shape(p->qdim + 2 * p->kvdim, p->d, f);
+  p->o = mat_shape(p->d, p->qdim, f);
+  p->gu = mat_shape(2 * p->F, p->d, f);
+  p->down = mat_shape(p->d, p->F, f);
+  p->lm = mat_shape(p->V, p->d, f);
+  p->kv_elems_per_layer = (size_t)c->max_batch * p->hkv * c->max_ctx * p->hd;
+  p->n_sm = n_sm;
+  p->ctas_per_sm = env_int("KFL_GEMV_CTAS_PER_SM", 1);
+  if (p->ctas_per_sm < 1 || p->ctas_per_sm > 2) p->ctas_per_sm = 1;
+  p->stages = env_int("KFL_GEMV_STAGES", 6);
+  if (p->stages < 2 || p->stages > MAX_STAGES) p->stages = 6;
+  p->gemv_grid_max = n_sm * p->ctas_per_sm;
+  int nrb = 1;
+  if (p->nl > 0) {
+    nrb = p->qkv.n_rb;
+    if (p->o.n_rb > nrb) nrb = p->o.n_rb;
+    if (p->gu.n_rb > nrb) nrb = p->gu.n_rb;
+    if (p->down.n_rb > nrb) nrb = p->down.n_rb;
+  }
+  if ((flags & KFL_LOGITS_OUT) && p->lm.n_rb > nrb) nrb = p->lm.n_rb;
+  p->n_rb_max = nrb;
+  p->n_parts = (p->d + RB - 1) / RB;
+  p->attn_nchunks_max = (c->max_ctx + 63) / 64;
+
+  size_t w = 0;
+  if (p->nl > 0)
+    w += (size_t)p->nl * (p->qkv.bytes + p->o.bytes + p->gu.bytes + p->down.bytes + 2 * (size_t)p->d * 4);
+  if (flags & KFL_EMBED_IN) w += (size_t)p->V * p->d * 2;
+  if (flags & KFL_LOGITS_OUT) w += p->lm.bytes + (size_t)p->d * 4;
+  p->bytes_weights = w;
+  p->bytes_kv = 2 * (size_t)p->nl * p->kv_elems_per_layer * 2;
+  size_t ws = 0;
+  ws += (size_t)c->max_ctx * (p->hd / 2) * 4 * 2;                      // rope tables
+  ws += (size_t)MAXB * (2 * p->ldh + 2 * p->ldq + p->lda) * 4;         // h, xn, q, o, a
+  ws += (size_t)p->n_parts * MAXB * 4;                                 // sum of squares
+  ws += 2 * MAXB * 4;                                                  // positions, next ids
+  ws += (size_t)p->gemv_grid_max * 2 * RB * MAXB * 4;                  // stream-K partials
+  ws += (size_t)(p->n_rb_max + 1) * 4;                                 // tickets + argmax ticket
+  ws += (size_t)p->n_rb_max * MAXB * 8;                                // argmax candidates
+  ws += (size_t)MAXB * p->hkv * p->attn_nchunks_max * 8 * (p->hd + 2) * 4;  // attention partials
+  ws += (size_t)MAXB * p->hkv * 4;                                     // attention tickets
+  ws += 16;                                                            // error word
+  ws += (size_t)MAXB * (2 + p->d) * 4;                                 // host-decode staging
+  p->bytes_ws = ws;
+}
+
+}  // namespace
+
+struct kfl_stage {
+  kfl_model_cfg cfg;
+  int l0 = 0, l1 = 0, flags = 0;
+  int dev = 0;
+  Plan P;
+  std::vector<LayerDev> layers;
+  Mat lm;
+  uint16_t *embed = nullptr;
+  float *g_final = nullptr;
+  bool head_loaded = false;
+  uint16_t *kc = nullptr, *vc = nullptr;
+  float *rope_cos = nullptr, *rope_sin = nullptr;
+  float *h = nullptr, *xn = nullptr, *q = nullptr, *o = nullptr, *a = nullptr, *sumsq = nullptr;
+  int *pos = nullptr, *next_int = nullptr;
+  int *io_pos = nullptr, *io_ids = nullptr;  // host-buffer decode staging
+  float *io_hin = nullptr;
+  float *gemv_partial = nullptr;
+  int *tickets = nullptr, *am_ticket = nullptr;
+  float *cand_val = nullptr;
+  int *cand_idx = nullptr;
+  float *attn_partial = nullptr;
+  int *attn_tickets = nullptr;
+  unsigned *err = nullptr;
+  float *capture = nullptr;
+  std::vector<void *> allocs;
+  int alloc_count = 0, fault_at = 0;
+  cudaStream_t cap_stream = nullptr;
+  cudaGraphExec_t graph[MAXB + 1] = {};
+  bool profile = false;
+  std::vector<cudaEvent_t> ev;
+  double prof_ms[KFL_KERNEL_KINDS] = {};
+  int64_t prof_n[KFL_KERNEL_KINDS] = {};
+  int magic = 0x4B464C53;
+
+  int alloc(void **p, size_t bytes) {
+    ++alloc_count;
+    if (fault_at > 0 && alloc_count == fault_at) return KFL_ERR_OOM;
+    if (bytes == 0) bytes = 16;
+    if (cudaMalloc(p, bytes) != cudaSuccess) {
+      cudaGetLastError();
+      *p = nullptr;
+      return KFL_ERR_OOM;
+    }
+    allocs.push_back(*p);
+    return KFL_OK;
+  }
+  bool loaded() const {
+    for (const auto &l : layers)
+      if (!l.loaded) return false;
+    if ((flags & (KFL_EMBED_IN | KFL_LOGITS_OUT)) && !head_loaded) return false;
+    return true;
+  }
+  void drop_graphs() {
+    for (auto &g : graph)
+      if (g) {
+        cudaGraphExecDestroy(g);
+        g = nullptr;
+      }
+  }
+};
+
+namespace {
+
+bool valid(const kfl_stage *st) { return st && st->magic == 0x4B464C53; }
+
+#define CK(x)                               \
+  do {                                      \
+    if ((x) != cudaSuccess) {               \
+      cudaGetLastError();                   \
+      return KFL_ERR_CUDA;                  \
+    }                                       \
+  } while (0)
+
+int attn_chunk_for(const kfl_stage *st, int batch) {
+  const Plan &P = st->P;
+  const long long work = (long long)st->cfg.max_ctx * batch * P.hkv;
+  long long want = (work + 2LL * P.n_sm - 1) / (2LL * P.n_sm);
+  int chunk = round_up((int)(want < 64 ? 64 : want), 64);
+  if (chunk > round_up(st->cfg.max_ctx, 64)) chunk = round_up(st->cfg.max_ctx, 64);
+  return chunk;
+}
+
+GemvParams base_gemv(kfl_stage *st, const Mat &m, const float *x, int ldx, int batch) {
+  GemvParams g = {};
+  g.w = m.tiles;
+  g.fmt = m.fmt;
+  g.n_rows = m.N;
+  g.n_rb = m.n_rb;
+  g.n_kt = m.n_kt;
+  g.tile_bytes = m.fmt == KFL_BF16 ? TILE_BYTES : TILE4_BYTES;
+  g.kt = m.fmt == KFL_BF16 ? KT : KT4;
+  g.x = x;
+  g.ldx = ldx;
+  g.batch = batch;
+  g.stages = st->P.stages;
+  g.partial = st->gemv_partial;
+  g.tickets = st->tickets;
+  g.err = st->err;
+  return g;
+}
+
+int gemv_grid(const kfl_stage *st, const Mat &m) {
+  const long long T = (long long)m.n_rb * m.n_kt;
+  return (int)(T < st->P.gemv_grid_max ? T : st->P.gemv_grid_max);
+}
+
+// Enqueue the kernels of the blocks (and lm_head) on stream s.  With `kinds` (profiling mode,
+// no PDL), the k-th kernel is bracketed by events ev[2(ev_base+k)], ev[2(ev_base+k)+1] and
+// its kind is appended to *kinds.
+int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector<int> *kinds, int ev_base) {
+  const Plan &P = st->P;
+  const kfl_model_cfg &c = st->cfg;
+  int k = ev_base;
+  auto pre = [&](int kind) -> int {
+    if (kinds) {
+      CK(cudaEventRecord(st->ev[2 * k], s));
+      kinds->push_back(kind);
+    }
+    return KFL_OK;
+  };
+  auto post = [&]() -> int {
+    if (kinds) CK(cudaEventRecord(st->ev[2 * k + 1], s));
+    ++k;
+    return KFL_OK;
+  };
+  const int chunk = attn_chunk_for(st, batch);
+  for (int l = 0; l < P.nl; ++l) {
+    const LayerDev &L = st->layers[l];
+    uint16_t *kcl = st->kc + (size_t)l * P.kv_elems_per_layer;
+    uint16_t *vcl = st->vc + (size_t)l * P.kv_elems_per_layer;
+    // Q/K/V with RoPE and KV append
+    {
+      GemvParams g = base_gemv(st, L.qkv, st->xn, P.ldh, batch);
+      g.sumsq = st->sumsq;
+      g.n_parts = P.n_parts;
+      g.d_norm = P.d;
+      g.eps = c.rms_eps;
+      g.q = st->q;
+      g.kcache = kcl;
+      g.vcache = vcl;
+      g.positions = st->pos;
+      g.rope_cos = st->rope_cos;
+      g.rope_sin = st->rope_sin;
+      g.n_q_rows = P.qdim;
+      g.n_kv_rows = P.kvdim;
+      g.head_dim = P.hd;
+      g.max_ctx = c.max_ctx;
+      g.n_kv_heads = P.hkv;
+      pre(KFL_KERNEL_QKV);
+      CK(launch_gemv(g, EPI_QKV, gemv_grid(st, L.qkv), s, pdl));
+      post();
+    }
+    // attention
+    {
+      AttnParams a = {};
+      a.q = st->q;
+      a.kcache = kcl;
+      a.vcache = vcl;
+      a.positions = st->pos;
+      a.o = st->o;
+      a.ldo = P.ldq;
+      a.partial = st->attn_partial;
+      a.tickets = st->attn_tickets;
+      a.batch = batch;
+      a.n_heads = P.hq;
+      a.n_kv_heads = P.hkv;
+      a.max_ctx = c.max_ctx;
+      a.chunk = chunk;
+      a.n_chunks = (c.max_ctx + chunk - 1) / chunk;
+      a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)P.hd));
+      a.err = st->err;
+      pre(KFL_KERNEL_ATTN);
+      CK(launch_attention(a, P.hd, s, pdl));
+      post();
+    }
+    // O projection + residual; produces the FFN norm input
+    {
+      GemvParams g = base_gemv(st, L.o, st->o, P.ldq, batch);
+      g.h = st->h;
+      g.ldh = P.ldh;
+      g.xn = st->xn;
+      g.g_next = L.g_ffn;
+      g.sumsq_out = st->sumsq;
+      pre(KFL_KERNEL_OPROJ);
+      CK(launch_gemv(g, EPI_RESID, gemv_grid(st, L.o), s, pdl));
+      post();
+    }
+    // gate/up + SwiGLU
+    {
+      GemvParams g = base_gemv(st, L.gu, st->xn, P.ldh, batch);
+      g.sumsq = st->sumsq;
+      g.n_parts = P.n_parts;
+      g.d_norm = P.d;
+      g.eps = c.rms_eps;
+      g.out = st->a;
+      g.ldo = P.lda;
+      pre(KFL_KERNEL_GATEUP);
+      CK(launch_gemv(g, EPI_SWIGLU, gemv_grid(st, L.gu), s, pdl));
+      post();
+    }
+    // down + residual; produces the next block's (or the final) norm input
+    {
+      GemvParams g = base_gemv(st, L.down, st->a, P.lda, batch);
+      g.h = st->h;
+      g.ldh = P.ldh;
+      g.xn = st->xn;
+      g.g_next = (l + 1 < P.nl) ? st->layers[l + 1].g_attn : ((st->flags & KFL_LOGITS_OUT) ? st->g_final : nullptr);
+      g.sumsq_out = st->sumsq;
+      g.capture = st->capture ? st->capture + (size_t)l * c.max_batch * P.d : nullptr;
+      pre(KFL_KERNEL_DOWN);
+      CK(launch_gemv(g, EPI_RESID, gemv_grid(st, L.down), s, pdl));
+      post();
+    }
+  }
+  if (st->flags & KFL_LOGITS_OUT) {
+    GemvParams g = base_gemv(st, st->lm, st->xn, P.ldh, batch);
+    g.sumsq = st->sumsq;
+    g.n_parts = P.n_parts;
+    g.d_norm = P.d;
+    g.eps = c.rms_eps;
+    g.cand_val = st->cand_val;
+    g.cand_idx = st->cand_idx;
+    g.argmax_ticket = st->am_ticket;
+    g.next_ids = st->next_int;
+    pre(KFL_KERNEL_LMHEAD);
+    CK(launch_gemv(g, EPI_ARGMAX, gemv_grid(st, st->lm), s, pdl));
+    post();
+  }
+  return KFL_OK;
+}
+
+int ensure_graph(kfl_stage *st, int batch) {
+  if (st->graph[batch]) return KFL_OK;
+  if (!st->cap_stream) CK(cudaStreamCreateWithFlags(&st->cap_stream, cudaStreamNonBlocking));
+  cudaGraph_t g = nullptr;
+  CK(cudaStreamBeginCapture(st->cap_stream, cudaStreamCaptureModeThreadLocal));
+  int rc = enqueue_body(st, batch, st->cap_stream, true, nullptr, 0);
+  cudaError_t e = cudaStreamEndCapture(st->cap_stream, &g);
+  if (rc != KFL_OK || e != cudaSuccess) {
+    if (g) cudaGraphDestroy(g);
+    cudaGetLastError();
+    return KFL_ERR_CUDA;
+  }
+  e = cudaGraphInstantiate(&st->graph[batch], g, 0);
+  cudaGraphDestroy(g);
+  if (e != cudaSuccess) {
+    st->graph[batch] = nullptr;
+    cudaGetLastError();
+    return KFL_ERR_CUDA;
+  }
+  return KFL_OK;
+}
+
+const float *input_g_next(const kfl_stage *st) {
+  if (st->P.nl > 0) return st->layers[0].g_attn;
+  if (st->flags & KFL_LOGITS_OUT) return st->g_final;
+  return nullptr;
+}
+
+int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const int32_t *positions, int batch,
+             float *hidden_out, int32_t *next_ids, cudaStream_t s) {
+  const Plan &P = st->P;
+  const bool embed = (st->flags & KFL_EMBED_IN) != 0;
+  if (st->profile) {
+    const int n_k = kfl_stage_launches_per_step(st, batch);
+    while ((int)st->ev.size() < 2 * n_k) {
+      cudaEvent_t e;
+      CK(cudaEventCreate(&e));
+      st->ev.push_back(e);
+    }
+    std::vector<int> kinds;
+    CK(cudaEventRecord(st->ev[0], s));
+    CK(launch_stage_input(ids, hidden_in, positions, batch, embed ? st->embed : nullptr, P.V, P.d, P.ldh,
+                          input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, s));
+    CK(cudaEventRecord(st->ev[1], s));
+    kinds.push_back(KFL_KERNEL_INPUT);
+    int rc = enqueue_body(st, batch, s, false, &kinds, 1);
+    if (rc != KFL_OK) return rc;
+    const int ko = (int)kinds.size();
+    CK(cudaEventRecord(st->ev[2 * ko], s));
+    CK(launch_stage_output(st->h, P.ldh, P.d, batch, hidden_out, st->next_int, next_ids, s, false));
+    CK(cudaEventRecord(st->ev[2 * ko + 1], s));
+    kinds.push_back(KFL_KERNEL_OUTPUT);
+    CK(cudaEventSynchronize(st->ev[2 * ko + 1]));
+    for (size_t k = 0; k < kinds.size(); ++k) {
+      float ms = 0.f;
+      CK(cudaEventElapsedTime(&ms, st->ev[2 * k], st->ev[2 * k + 1]));
+      st->prof_ms[kinds[k]] += ms;
+      st->prof_n[kinds[k]] += 1;
+    }
+    return KFL_OK;
+  }
+  CK(launch_stage_input(ids, hidden_in, positions, batch, embed ? st->embed : nullptr, P.V, P.d, P.ldh,
+                        input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, s));
+  if (P.nl > 0 || (st->flags & KFL_LOGITS_OUT)) {
+    int rc = ensure_graph(st, batch);
+    if (rc != KFL_OK) return rc;
+    CK(cudaGraphLaunch(st->graph[batch], s));
+  }
+  CK(launch_stage_output(st->h, P.ldh, P.d, batch, hidden_out, st->next_int, next_ids, s, false));
+  return KFL_OK;
+}
+
+// host or device source -> device pointer (a temporary copy for host sources)
+int to_device(kfl_stage *st, const void *src, size_t bytes, int on_device, void **out, std::vector<void *> &tmp) {
+  if (on_device) {
+    *out = const_cast<void *>(src);
+    return KFL_OK;
+  }
+  void *d = nullptr;
+  if (cudaMalloc(&d, bytes ? bytes : 16) != cudaSuccess) {
+    cudaGetLastError();
+    return KFL_ERR_OOM;
+  }
+  tmp.push_back(d);
+  CK(cudaMemcpy(d, src, bytes, cudaMemcpyHostToDevice));
+  *out = d;
+  return KFL_OK;
+}
+
+void free_tmp(std::vector<void *> &tmp) {
+  for (void *p : tmp) cudaFree(p);
+  tmp.clear();
+}
+
+int load_gain(kfl_stage *st, const uint16_t *src, int n, int on_device, float *dst, std::vector<void *> &tmp) {
+  void *d = nullptr;
+  int rc = to_device(st, src, (size_t)n * 2, on_device, &d, tmp);
+  if (rc) return rc;
+  CK(launch_bf16_to_f32(static_cast<const uint16_t *>(d), dst, n, nullptr));
+  return KFL_OK;
+}
+
+// Concatenate matrices (rows stacked) into one device buffer and repack with an optional row
+// map.  parts: (matrix, rows).  For int4 the words and scales are concatenated separately.
+int load_matrix(kfl_stage *st, Mat &m, const std::vector<std::pair<const kfl_matrix *, int>> &parts, int K,
+                const std::vector<int> &row_map, int on_device, std::vector<void *> &tmp) {
+  const bool bf = m.fmt == KFL_BF16;
+  int n_src = 0;
+  for (auto &pp : parts) {
+    if (!pp.first || !pp.first->w || (!bf && !pp.first->scales)) return KFL_ERR_ARG;
+    n_src += pp.second;
+  }
+  const size_t row_w = bf ? (size_t)K * 2 : (size_t)K / 2;  // bytes of codes per row
+  const size_t row_s = bf ? 0 : (size_t)(K / 64) * 2;
+  void *wcat = nullptr, *scat = nullptr;
+  if (parts.size() == 1 && on_device) {
+    wcat = const_cast<void *>(parts[0].first->w);
+    scat = const_cast<void *>(parts[0].first->scales);
+  } else {
+    if (cudaMalloc(&wcat, n_src * row_w) != cudaSuccess) {
+      cudaGetLastError();
+      return KFL_ERR_OOM;
+    }
+    tmp.push_back(wcat);
+    if (!bf) {
+      if (cudaMalloc(&scat, n_src * row_s) != cudaSuccess) {
+        cudaGetLastError();
+        return KFL_ERR_OOM;
+      }
+      tmp.push_back(scat);
+    }
+    size_t off = 0;
+    for (auto &pp : parts) {
+      CK(cudaMemcpy(static_cast<uint8_t *>(wcat) + off * row_w, pp.first->w, pp.second * row_w, cudaMemcpyDefault));
+      if (!bf)
+        CK(cudaMemcpy(static_cast<uint8_t *>(scat) + off * row_s, pp.first->scales, pp.second * row_s,
+                      cudaMemcpyDefault));
+      off += pp.second;
+    }
+  }
+  int *dmap = nullptr;
+  if (!row_map.empty()) {
+    if (cudaMalloc(&dmap, row_map.size() * sizeof(int)) != cudaSuccess) {
+      cudaGetLastError();
+      return KFL_ERR_OOM;
+    }
+    tmp.push_back(dmap);
+    CK(cudaMemcpy(dmap, row_map.data(), row_map.size() * sizeof(int), cudaMemcpyHostToDevice));
+  }
+  if (bf)
+    CK(launch_repack_bf16(static_cast<const uint16_t *>(wcat), n_src, K, dmap, m.N, m.n_rb, m.n_kt, m.tiles,
+                          nullptr));
+  else
+    CK(launch_repack_int4(static_cast<const uint32_t *>(wcat), static_cast<const uint16_t *>(scat), n_src, K, dmap,
+                          m.N, m.n_rb, m.n_kt, m.tiles, nullptr));
+  CK(cudaDeviceSynchronize());
+  return KFL_OK;
+}
+
+}  // namespace
+
+// ============================================================================ C ABI
+
+extern "C" int kfl_stage_memory_bytes(const kfl_model_cfg *cfg, int l0, int l1, int flags, size_t *out) {
+  if (!out) return KFL_ERR_ARG;
+  int rc = validate_cfg(cfg, l0, l1, flags);
+  if (rc) return rc;
+  Plan P;
+  int n_sm = 152;
+  int dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && v > 0) n_sm = v;
+  }
+  cudaGetLastError();
+  make_plan(cfg, l0, l1, flags, n_sm, &P);
+  *out = P.bytes_weights + P.bytes_kv + P.bytes_ws;
+  return KFL_OK;
+}
+
+extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int flags, kfl_stage **out) {
+  if (!out) return KFL_ERR_ARG;
+  *out = nullptr;
+  int rc = validate_cfg(cfg, l0, l1, flags);
+  if (rc) return rc;
+  int dev = 0, n_sm = 0;
+  CK(cudaGetDevice(&dev));
+  CK(cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev));
+  CK(prepare_gemv());
+  CK(prepare_attention());
+  kfl_stage *st = new kfl_stage();
+  st->cfg = *cfg;
+  st->l0 = l0;
+  st->l1 = l1;
+  st->flags = flags;
+  st->dev = dev;
+  st->fault_at = env_int("KFL_FAULT_ALLOC_AT", 0);
+  make_plan(cfg, l0, l1, flags, n_sm, &st->P);
+  Plan &P = st->P;
+  auto fail = [&](int code) {
+    kfl_stage_destroy(st);
+    return code;
+  };
+#define AL(ptr, bytes)                                                  \
+  do {                                                                  \
+    int _r = st->alloc(reinterpret_cast<void **>(&(ptr)), (bytes));     \
+    if (_r) return fail(_r);                                            \
+  } while (0)
+  st->layers.resize(P.nl);
+  for (int l = 0; l < P.nl; ++l) {
+    LayerDev &L = st->layers[l];
+    L.qkv = P.qkv;
+    L.o = P.o;
+    L.gu = P.gu;
+    L.down = P.down;
+    AL(L.qkv.tiles, L.qkv.bytes);
+    AL(L.o.tiles, L.o.bytes);
+    AL(L.gu.tiles, L.gu.bytes);
+    AL(L.down.tiles, L.down.bytes);
+    AL(L.g_attn, (size_t)P.d * 4);
+    AL(L.g_ffn, (size_t)P.d * 4);
+  }
+  if (flags & KFL_EMBED_IN) AL(st->embed, (size_t)P.V * P.d * 2);
+  if (flags & KFL_LOGITS_OUT) {
+    st->lm = P.lm;
+    AL(st->lm.tiles, st->lm.bytes);
+    AL(st->g_final, (size_t)P.d * 4);
+  }
+  if (P.nl > 0) {
+    AL(st->kc, (size_t)P.nl * P.kv_elems_per_layer * 2);
+    AL(st->vc, (size_t)P.nl * P.kv_elems_per_layer * 2);
+  }
+  AL(st->rope_cos, (size_t)cfg->max_ctx * (P.hd / 2) * 4);
+  AL(st->rope_sin, (size_t)cfg->max_ctx * (P.hd / 2) * 4);
+  AL(st->h, (size_t)MAXB * P.ldh * 4);
+  AL(st->xn, (size_t)MAXB * P.ldh * 4);
+  AL(st->q, (size_t)MAXB * P.ldq * 4);
+  AL(st->o, (size_t)MAXB * P.ldq * 4);
+  AL(st->a, (size_t)MAXB * P.lda * 4);
+  AL(st->sumsq, (size_t)P.n_parts * MAXB * 4);
+  AL(st->pos, MAXB * 4);
+  AL(st->next_int, MAXB * 4);
+  AL(st->gemv_partial, (size_t)P.gemv_grid_max * 2 * RB * MAXB * 4);
+  AL(st->tickets, (size_t)(P.n_rb_max + 1) * 4);
+  st->am_ticket = st->tickets + P.n_rb_max;
+  AL(st->cand_val, (size_t)P.n_rb_max * MAXB * 4);
+  AL(st->cand_idx, (size_t)P.n_rb_max * MAXB * 4);
+  AL(st->attn_partial, (size_t)MAXB * P.hkv * P.attn_nchunks_max * 8 * (P.hd + 2) * 4);
+  AL(st->attn_tickets, (size_t)MAXB * P.hkv * 4);
+  AL(st->err, 16);
+  AL(st->io_pos, MAXB * 4);
+  AL(st->io_ids, MAXB * 4);
+  AL(st->io_hin, (size_t)MAXB * P.d * 4);
+#undef AL
+  // zero everything that is read before it is written or whose padding must stay zero
+  if (P.nl > 0) {
+    if (cudaMemset(st->kc, 0, (size_t)P.nl * P.kv_elems_per_layer * 2) != cudaSuccess) return fail(KFL_ERR_CUDA);
+    if (cudaMemset(st->vc, 0, (size_t)P.nl * P.kv_elems_per_layer * 2) != cudaSuccess) return fail(KFL_ERR_CUDA);
+  }
+  if (cudaMemset(st->h, 0, (size_t)MAXB * P.ldh * 4) || cudaMemset(st->xn, 0, (size_t)MAXB * P.ldh * 4) ||
+      cudaMemset(st->q, 0, (size_t)MAXB * P.ldq * 4) || cudaMemset(st->o, 0, (size_t)MAXB * P.ldq * 4) ||
+      cudaMemset(st->a, 0, (size_t)MAXB * P.lda * 4) || cudaMemset(st->sumsq, 0, (size_t)P.n_parts * MAXB * 4) ||
+      cudaMemset(st->pos, 0, MAXB * 4) || cudaMemset(st->next_int, 0, MAXB * 4) ||
+      cudaMemset(st->tickets, 0, (size_t)(P.n_rb_max + 1) * 4) ||
+      cudaMemset(st->attn_tickets, 0, (size_t)MAXB * P.hkv * 4) || cudaMemset(st->err, 0, 16))
+    return fail(KFL_ERR_CUDA);
+  // RoPE table: angle pos * theta^(-2i/hd) in fp64, stored as fp32 cos / sin
+  {
+    const int half = P.hd / 2;
+    std::vector<float> cs((size_t)cfg->max_ctx * half), sn((size_t)cfg->max_ctx * half);
+    for (int p = 0; p < cfg->max_ctx; ++p)
+      for (int i = 0; i < half; ++i) {
+        const double a = (double)p * std::pow((double)cfg->rope_theta, -2.0 * i / P.hd);
+        cs[(size_t)p * half + i] = (float)std::cos(a);
+        sn[(size_t)p * half + i] = (float)std::sin(a);
+      }
+    if (cudaMemcpy(st->rope_cos, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(st->rope_sin, sn.data(), sn.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+      return fail(KFL_ERR_CUDA);
+  }
+  *out = st;
+  return KFL_OK;
+}
+
+extern "C" int kfl_stage_load_layer(kfl_stage *st, int local, const kfl_layer_weights *w, int on_device) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  if (!w) return KFL_ERR_ARG;
+  if (local < 0 || local >= st->P.nl) return KFL_ERR_RANGE;
+  if (!w->attn_norm || !w->ffn_norm) return KFL_ERR_ARG;
+  CK(cudaSetDevice(st->dev));
+  const Plan &P = st->P;
+  LayerDev &L = st->layers[local];
+  std::vector<void *> tmp;
+  int rc = KFL_OK;
+  do {
+    if ((rc = load_gain(st, w->attn_norm, P.d, on_device, L.g_attn, tmp))) break;
+    if ((rc = load_gain(st, w->ffn_norm, P.d, on_device, L.g_ffn, tmp))) break;
+    // Q/K/V: q and k rows of each head reordered so that the RoPE pair (i, i + hd/2) is adjacent
+    std::vector<int> map(P.qdim + 2 * P.kvdim);
+    for (int r = 0; r < (int)map.size(); ++r) {
+      if (r < P.qdim + P.kvdim) {
+        const int base = (r / P.hd) * P.hd, j = r % P.hd;
+        map[r] = base + ((j & 1) ? (j >> 1) + P.hd / 2 : (j >> 1));
+      } else {
+        map[r] = r;
+      }
+    }
+    if ((rc = load_matrix(st, L.qkv, {{&w->wq, P.qdim}, {&w->wk, P.kvdim}, {&w->wv, P.kvdim}}, P.d, map, on_device,
+                          tmp)))
+      break;
+    if ((rc = load_matrix(st, L.o, {{&w->wo, P.d}}, P.qdim, {}, on_device, tmp))) break;
+    // gate/up interleaved: row 2j = gate j, row 2j + 1 = up j
+    std::vector<int> gmap(2 * P.F);
+    for (int j = 0; j < P.F; ++j) {
+      gmap[2 * j] = j;
+      gmap[2 * j + 1] = P.F + j;
+    }
+    if ((rc = load_matrix(st, L.gu, {{&w->wg, P.F}, {&w->wu, P.F}}, P.d, gmap, on_device, tmp))) break;
+    if ((rc = load_matrix(st, L.down, {{&w->wd, P.d}}, P.F, {}, on_device, tmp))) break;
+    if (cudaDeviceSynchronize() != cudaSuccess) {
+      rc = KFL_ERR_CUDA;
+      break;
+    }
+    L.loaded = true;
+    st->drop_graphs();
+  } while (0);
+  cudaGetLastError();
+  free_tmp(tmp);
+  return rc;
+}
+
+extern "C" int kfl_stage_load_head(kfl_stage *st, const uint16_t *embed, const uint16_t *final_norm,
+                                   const kfl_matrix *lm_head, int on_device) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  if (!(st->flags & (KFL_EMBED_IN | KFL_LOGITS_OUT))) return KFL_OK;
+  if ((st->flags & KFL_EMBED_IN) && !embed) return KFL_ERR_ARG;
+  if ((st->flags & KFL_LOGITS_OUT) && (!final_norm || !lm_head)) return KFL_ERR_ARG;
+  CK(cudaSetDevice(st->dev));
+  const Plan &P = st->P;
+  std::vector<void *> tmp;
+  int rc = KFL_OK;
+  do {
+    if (st->flags & KFL_EMBED_IN) {
+      if (cudaMemcpy(st->embed, embed, (size_t)P.V * P.d * 2, cudaMemcpyDefault) != cudaSuccess) {
+        rc = KFL_ERR_CUDA;
+        break;
+      }
+    }
+    if (st->flags & KFL_LOGITS_OUT) {
+      if ((rc = load_gain(st, final_norm, P.d, on_device, st->g_final, tmp))) break;
+      if ((rc = load_matrix(st, st->lm, {{lm_head, P.V}}, P.d, {}, on_device, tmp))) break;
+    }
+    if (cudaDeviceSynchronize() != cudaSuccess) {
+      rc = KFL_ERR_CUDA;
+      break;
+    }
+    st->head_loaded = true;
+    st->drop_graphs();
+  } while (0);
+  cudaGetLastError();
+  free_tmp(tmp);
+  return rc;
+}
+
+extern "C" int kfl_stage_load_weights(kfl_stage *st, const kfl_weights *w) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  if (!w || w->n_layers != st->P.nl || (st->P.nl > 0 && !w->layers)) return KFL_ERR_ARG;
+  for (int l = 0; l < st->P.nl; ++l) {
+    int rc = kfl_stage_load_layer(st, l, &w->layers[l], w->on_device);
+    if (rc) return rc;
+  }
+  return kfl_stage_load_head(st, w->embed, w->final_norm, &w->lm_head, w->on_device);
+}
+
+static int check_decode_args(kfl_stage *st, const int32_t *ids, const float *hidden_in, const int32_t *positions,
+                             int batch, float *hidden_out, int32_t *next_ids) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  if (batch < 1) return KFL_ERR_ARG;
+  if (batch > st->cfg.max_batch) return KFL_ERR_RANGE;
+  if (!positions) return KFL_ERR_ARG;
+  if ((st->flags & KFL_EMBED_IN) ? !ids : !hidden_in) return KFL_ERR_ARG;
+  if ((st->flags & KFL_LOGITS_OUT) ? !next_ids : !hidden_out) return KFL_ERR_ARG;
+  if (!st->loaded()) return KFL_ERR_STATE;
+  return KFL_OK;
+}
+
+extern "C" int kfl_stage_decode(kfl_stage *st, const int32_t *token_ids, const float *hidden_in,
+                                const int32_t *positions, int batch, float *hidden_out, int32_t *next_ids,
+                                void *cuda_stream) {
+  int rc = check_decode_args(st, token_ids, hidden_in, positions, batch, hidden_out, next_ids);
+  if (rc) return rc;
+  CK(cudaSetDevice(st->dev));
+  return run_step(st, token_ids, hidden_in, positions, batch, hidden_out, next_ids,
+                  static_cast<cudaStream_t>(cuda_stream));
+}
+
+extern "C" int kfl_stage_decode_host(kfl_stage *st, const int32_t *token_ids, const float *hidden_in,
+                                     const int32_t *positions, int batch, float *hidden_out, int32_t *next_ids,
+                                     void *cuda_stream) {
+  int rc = check_decode_args(st, token_ids, hidden_in, positions, batch, hidden_out, next_ids);
+  if (rc) return rc;
+  CK(cudaSetDevice(st->dev));
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  const Plan &P = st->P;
+  const bool embed = (st->flags & KFL_EMBED_IN) != 0;
+  CK(cudaMemcpyAsync(st->io_pos, positions, (size_t)batch * 4, cudaMemcpyHostToDevice, s));
+  if (embed) CK(cudaMemcpyAsync(st->io_ids, token_ids, (size_t)batch * 4, cudaMemcpyHostToDevice, s));
+  else CK(cudaMemcpyAsync(st->io_hin, hidden_in, (size_t)batch * P.d * 4, cudaMemcpyHostToDevice, s));
+  rc = run_step(st, embed ? st->io_ids : nullptr, embed ? nullptr : st->io_hin, st->io_pos, batch, nullptr, nullptr, s);
+  if (rc) return rc;
+  if (hidden_out)
+    CK(cudaMemcpy2DAsync(hidden_out, (size_t)P.d * 4, st->h, (size_t)P.ldh * 4, (size_t)P.d * 4, batch,
+                         cudaMemcpyDeviceToHost, s));
+  if (next_ids) CK(cudaMemcpyAsync(next_ids, st->next_int, (size_t)batch * 4, cudaMemcpyDeviceToHost, s));
+  CK(cudaStreamSynchronize(s));
+  return KFL_OK;
+}
+
+extern "C" int kfl_kv_reset(kfl_stage *st, int user) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  if (user < -1 || user >= st->cfg.max_batch) return KFL_ERR_RANGE;
+  CK(cudaSetDevice(st->dev));
+  CK(cudaDeviceSynchronize());
+  const Plan &P = st->P;
+  const size_t per_user = (size_t)P.hkv * st->cfg.max_ctx * P.hd;
+  for (int l = 0; l < P.nl; ++l) {
+    for (int u = 0; u < st->cfg.max_batch; ++u) {
+      if (user >= 0 && u != user) continue;
+      const size_t off = (size_t)l * P.kv_elems_per_layer + (size_t)u * per_user;
+      CK(cudaMemset(st->kc + off, 0, per_user * 2));
+      CK(cudaMemset(st->vc + off, 0, per_user * 2));
+    }
+  }
+  CK(cudaDeviceSynchronize());
+  return KFL_OK;
+}
+
+extern "C" int kfl_kv_fill_seeded(kfl_stage *st, int user, int len, uint64_t seed) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  if (user < -1 || user >= st->cfg.max_batch || len < 0 || len > st->cfg.max_ctx) return KFL_ERR_RANGE;
+  CK(cudaSetDevice(st->dev));
+  CK(cudaDeviceSynchronize());
+  const Plan &P = st->P;
+  const float c = (float)(1.0 * (1.0 / std::sqrt((65536.0 * 65536.0 - 1.0) / 3.0)));
+  const size_t per_user = (size_t)P.hkv * st->cfg.max_ctx * P.hd;
+  for (int l = 0; l < P.nl; ++l) {
+    const int gl = st->l0 + l;
+    for (int u = 0; u < st->cfg.max_batch; ++u) {
+      if (user >= 0 && u != user) continue;
+      for (int h = 0; h < P.hkv; ++h) {
+        const size_t off = (size_t)l * P.kv_elems_per_layer + (size_t)u * per_user + (size_t)h * st->cfg.max_ctx * P.hd;
+        const int64_t start = (((int64_t)u * P.hkv + h) << 20) * P.hd;
+        for (int which = 0; which < 2; ++which) {
+          uint16_t *dst = (which == 0 ? st->kc : st->vc) + off;
+          int rc = kfl_synth_fill(dst, (int64_t)len * P.hd, seed, 0x4B560000ull + 2ull * gl + which,
+                                  KFL_SYNTH_NORMAL_BF16, c, 0.0f, start, nullptr);
+          if (rc) return rc;
+        }
+      }
+    }
+  }
+  CK(cudaDeviceSynchronize());
+  return KFL_OK;
+}
+
+extern "C" int kfl_kv_write(kfl_stage *st, int local, int user, const uint16_t *k, const uint16_t *v, int len,
+                            int on_device) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  if (!k || !v) return KFL_ERR_ARG;
+  if (local < 0 || local >= st->P.nl || user < 0 || user >= st->cfg.max_batch || len < 0 || len > st->cfg.max_ctx)
+    return KFL_ERR_RANGE;
+  if (len == 0) return KFL_OK;
+  CK(cudaSetDevice(st->dev));
+  CK(cudaDeviceSynchronize());
+  const Plan &P = st->P;
+  const size_t per_user = (size_t)P.hkv * st->cfg.max_ctx * P.hd;
+  const size_t off = (size_t)local * P.kv_elems_per_layer + (size_t)user * per_user;
+  const size_t dpitch = (size_t)st->cfg.max_ctx * P.hd * 2, spitch = (size_t)len * P.hd * 2;
+  const cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+  CK(cudaMemcpy2D(st->kc + off, dpitch, k, spitch, spitch, P.hkv, kind));
+  CK(cudaMemcpy2D(st->vc + off, dpitch, v, spitch, spitch, P.hkv, kind));
+  return KFL_OK;
+}
+
+extern "C" int kfl_kv_read(kfl_stage *st, int local, int user, uint16_t *k, uint16_t *v, int on_device) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  if (!k || !v) return KFL_ERR_ARG;
+  if (local < 0 || local >= st->P.nl || user < 0 || user >= st->cfg.max_batch) return KFL_ERR_RANGE;
+  CK(cudaSetDevice(st->dev));
+  CK(cudaDeviceSynchronize());
+  const Plan &P = st->P;
+  const size_t per_user = (size_t)P.hkv * st->cfg.max_ctx * P.hd;
+  const size_t off = (size_t)local * P.kv_elems_per_layer + (size_t)user * per_user;
+  const cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
+  CK(cudaMemcpy(k, st->kc + off, per_user * 2, kind));
+  CK(cudaMemcpy(v, st->vc + off, per_user * 2, kind));
+  return KFL_OK;
+}
+
+extern "C" int kfl_stage_debug_capture(kfl_stage *st, float *per_layer_hidden) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  if (st->capture != per_layer_hidden) {
+    st->capture = per_layer_hidden;
+    st->drop_graphs();
+  }
+  return KFL_OK;
+}
+
+extern "C" int kfl_stage_status(kfl_stage *st) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  CK(cudaSetDevice(st->dev));
+  CK(cudaDeviceSynchronize());
+  unsigned e = 0;
+  CK(cudaMemcpy(&e, st->err, 4, cudaMemcpyDeviceToHost));
+  CK(cudaMemset(st->err, 0, 4));
+  if (e & ERR_TIMEOUT) return KFL_ERR_TIMEOUT;
+  if (e & (ERR_POSITION | ERR_TOKEN)) return KFL_ERR_RANGE;
+  return KFL_OK;
+}
+
+extern "C" int kfl_stage_profile(kfl_stage *st, int enable) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  st->profile = enable != 0;
+  return KFL_OK;
+}
+
+extern "C" int kfl_stage_profile_read(kfl_stage *st, double *ms, int64_t *launches, int n) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  CK(cudaSetDevice(st->dev));
+  CK(cudaDeviceSynchronize());
+  for (int k = 0; k < KFL_KERNEL_KINDS && k < n; ++k) {
+    if (ms) ms[k] = st->prof_ms[k];
+    if (launches) launches[k] = st->prof_n[k];
+    st->prof_ms[k] = 0.0;
+    st->prof_n[k] = 0;
+  }
+  return KFL_KERNEL_KINDS;
+}
+
+extern "C" int kfl_stage_launches_per_step(kfl_stage *st, int batch) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  (void)batch;
+  return 2 + 5 * st->P.nl + ((st->flags & KFL_LOGITS_OUT) ? 1 : 0);
+}
+
+extern "C" void kfl_stage_destroy(kfl_stage *st) {
+  if (!valid(st)) return;
+  cudaSetDevice(st->dev);
+  cudaDeviceSynchronize();
+  st->drop_graphs();
+  for (cudaEvent_t e : st->ev) cudaEventDestroy(e);
+  if (st->cap_stream) cudaStreamDestroy(st->cap_stream);
+  for (void *p : st->allocs) cudaFree(p);
+  cudaGetLastError();
+  st->magic = 0;
+  delete st;
+}
+
+extern "C" const char *kfl_strerror(int code) {
+  switch (code) {
+    case KFL_OK: return "ok";
+    case KFL_ERR_ARG: return "invalid argument";
+    case KFL_ERR_RANGE: return "index, size, position or token id out of range";
+    case KFL_ERR_OOM: return "device memory allocation failed";
+    case KFL_ERR_CUDA: return "CUDA runtime error";
+    case KFL_ERR_STATE: return "stage not ready (weights not loaded) or invalid";
+    case KFL_ERR_TIMEOUT: return "a bounded device-side wait gave up";
+    default: return "unknown error";
+  }
+}

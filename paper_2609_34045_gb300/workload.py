@@ -30,8 +30,10 @@ for bit):
 """
 from __future__ import annotations
 
+import concurrent.futures as _cf
 import math
-from dataclasses import dataclass, field, replace
+import os
+from dataclasses import dataclass, replace
 
 import numpy as np
 
@@ -48,7 +50,21 @@ KIND_NORMAL_BF16 = 0
 KIND_INT4_WORDS = 1
 KIND_INT4_SCALES_BF16 = 2
 
-_CHUNK = 1 << 22
+_CHUNK = 1 << 21
+_THREADS = min(16, os.cpu_count() or 1)
+
+
+def _chunked(n: int, out: np.ndarray, fill) -> np.ndarray:
+    """Run ``fill(c0, c1)`` (which writes out[c0:c1]) over chunks, on threads for large n
+    (numpy releases the GIL inside its array loops)."""
+    starts = range(0, n, _CHUNK)
+    if n > 4 * _CHUNK and _THREADS > 1:
+        with _cf.ThreadPoolExecutor(_THREADS) as ex:
+            list(ex.map(lambda c0: fill(c0, min(n, c0 + _CHUNK)), starts))
+    else:
+        for c0 in starts:
+            fill(c0, min(n, c0 + _CHUNK))
+    return out
 
 
 def _mix64_int(z: int) -> int:
@@ -116,10 +132,10 @@ def normal_bf16(seed: int, tag: int, n: int, std: float, mean: float = 0.0, star
     """``n`` bf16 bit patterns of the ``normal`` kind, stream ``(seed, tag)``, from index ``start``."""
     key = stream_key(seed, tag)
     out = np.empty(n, dtype=np.uint16)
-    for c0 in range(0, n, _CHUNK):
-        c1 = min(n, c0 + _CHUNK)
+
+    def fill(c0, c1):
         out[c0:c1] = f32_to_bf16_bits(_normal_from_draws(draws(key, start + c0, c1 - c0), std, mean))
-    return out
+    return _chunked(n, out, fill)
 
 
 def normal_bf16_at(seed: int, tag: int, idx: np.ndarray, std: float, mean: float = 0.0) -> np.ndarray:
@@ -130,21 +146,21 @@ def normal_bf16_at(seed: int, tag: int, idx: np.ndarray, std: float, mean: float
 def int4_words(seed: int, tag: int, n: int) -> np.ndarray:
     key = stream_key(seed, tag)
     out = np.empty(n, dtype=np.uint32)
-    for c0 in range(0, n, _CHUNK):
-        c1 = min(n, c0 + _CHUNK)
+
+    def fill(c0, c1):
         out[c0:c1] = (draws(key, c0, c1 - c0) & np.uint64(0xFFFFFFFF)).astype(np.uint32)
-    return out
+    return _chunked(n, out, fill)
 
 
 def int4_scales_bf16(seed: int, tag: int, n: int) -> np.ndarray:
     key = stream_key(seed, tag)
     out = np.empty(n, dtype=np.uint16)
     c1s = np.float32(INT4_SCALE_C1)
-    for c0 in range(0, n, _CHUNK):
-        c1 = min(n, c0 + _CHUNK)
+
+    def fill(c0, c1):
         u = (draws(key, c0, c1 - c0) >> np.uint64(40)).astype(np.float32) * np.float32(2.0 ** -24)
         out[c0:c1] = f32_to_bf16_bits(c1s * (np.float32(0.5) + u))
-    return out
+    return _chunked(n, out, fill)
 
 
 def token_ids(seed: int, tag: int, n: int, vocab: int) -> np.ndarray:

@@ -1,0 +1,259 @@
+"""GPU parity: the CUDA stage-decode path against the fp64 oracle on the same seeded inputs.
+
+Bar (element by element): hidden states within max-abs 1e-2 of the oracle's per-layer RMS, per
+user and step; greedy ids identical where the oracle's top-2 logit margin exceeds 1e-2; KV slot
+addressing bit-exact (every slot not written is unchanged, written slots hold the new K/V).
+Everything goes through the C ABI.
+"""
+import numpy as np
+import pytest
+import torch
+
+from gpu_helpers import Pair, ensure_built
+from paper_2609_34045_gb300 import stage as K
+from paper_2609_34045_gb300 import workload as wl
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    ensure_built()
+    torch.cuda.init()
+
+
+# small shapes that span several tiles and leave ragged tails everywhere: d = 320 is 2.5 bf16
+# K tiles and 1.25 int4 K tiles; 2F = 1424 rows is 22.25 row blocks; vocab 1000 is 15.6 row
+# blocks; G = 3 query heads per KV head; contexts cross the 64-position sub-tiles
+RAGGED = wl.ModelShape(n_layers_total=3, d_model=320, n_heads=6, n_kv_heads=2, head_dim=64, ffn=712, vocab=1000)
+RAGGED128 = wl.ModelShape(n_layers_total=2, d_model=384, n_heads=4, n_kv_heads=1, head_dim=128, ffn=520,
+                          vocab=777)
+RAGGED_INT4 = wl.ModelShape(n_layers_total=2, d_model=320, n_heads=6, n_kv_heads=2, head_dim=64, ffn=704,
+                            vocab=1000, weight_fmt="int4_g64")
+
+
+def _greedy(pair, steps, first_ids):
+    ids = first_ids
+    for s in range(steps):
+        o, _, _ = pair.step(s, ids=ids)
+        ids = o["next_ids"]
+    pair.compare_kv()
+
+
+def test_config1_tiny_head_greedy():
+    w = wl.CONFIGS[1]
+    p = Pair(w.model, w.l0, w.l1, K.KFL_IS_HEAD, w.batch, w.contexts, w.max_ctx, w.seed)
+    _greedy(p, w.steps, wl.first_token_ids(w.model, w.batch, w.seed))
+    p.close()
+
+
+@pytest.mark.parametrize("batch,contexts", [(1, (0,)), (3, (5, 130, 67)), (4, (1, 64, 200, 63))])
+def test_ragged_head_stage(batch, contexts):
+    p = Pair(RAGGED, 1, 3, K.KFL_IS_HEAD, batch, contexts, 272, seed=11)
+    _greedy(p, 3, wl.token_ids(11, 99, batch, RAGGED.vocab))
+    p.close()
+
+
+@pytest.mark.parametrize("batch", [1, 2, 3, 4])
+def test_ragged_body_stage_hidden_in(batch):
+    contexts = tuple(17 + 40 * u for u in range(batch))
+    p = Pair(RAGGED, 0, 3, 0, batch, contexts, 192, seed=12)
+    for s in range(2):
+        p.step(s, hidden=wl.hidden_in(RAGGED, s, batch, 12))
+    p.compare_kv()
+    p.close()
+
+
+def test_head_dim_128_single_kv_head():
+    p = Pair(RAGGED128, 0, 2, K.KFL_IS_HEAD, 2, (100, 3), 192, seed=13)
+    _greedy(p, 3, np.array([5, 700], dtype=np.int32))
+    p.close()
+
+
+@pytest.mark.parametrize("batch", [1, 4])
+def test_int4_head_stage(batch):
+    contexts = (9, 70, 131, 2)[:batch]
+    p = Pair(RAGGED_INT4, 0, 2, K.KFL_IS_HEAD, batch, contexts, 192, seed=14)
+    _greedy(p, 2, wl.token_ids(14, 98, batch, RAGGED_INT4.vocab))
+    p.close()
+
+
+def test_empty_tail_stage_is_head_return_leg():
+    # l0 == l1 with LOGITS_OUT: final norm, lm_head and argmax of a received hidden state
+    p = Pair(RAGGED, 3, 3, K.KFL_LOGITS_OUT, 2, (0, 0), 64, seed=15)
+    h = wl.hidden_in(RAGGED, 0, 2, 15)
+    o, g_out, g_next = p.step(0, hidden=h)
+    p.close()
+
+
+def test_stage_split_associativity_bit_exact():
+    m = RAGGED
+    full = Pair(m, 0, 3, K.KFL_IS_HEAD, 2, (30, 90), 128, seed=16)
+    a = Pair(m, 0, 1, K.KFL_EMBED_IN, 2, (30, 90), 128, seed=16)
+    b = Pair(m, 1, 3, K.KFL_LOGITS_OUT, 2, (30, 90), 128, seed=16)
+    ids = np.array([3, 900], dtype=np.int32)
+    for s in range(3):
+        pos = np.array([30 + s, 90 + s], dtype=np.int32)
+        hf, nf = full.gpu_step(pos, ids=ids)
+        ha, _ = a.gpu_step(pos, ids=ids)
+        hb, nb = b.gpu_step(pos, hidden=ha)
+        assert np.array_equal(hf, hb)
+        assert np.array_equal(nf, nb)
+        cf = full.cap.cpu().numpy()
+        assert np.array_equal(cf[:1], a.cap.cpu().numpy()) and np.array_equal(cf[1:], b.cap.cpu().numpy())
+        ids = nf
+    for p in (full, a, b):
+        p.close()
+
+
+def test_deterministic_replay_and_profile_mode():
+    p = Pair(RAGGED, 0, 3, K.KFL_IS_HEAD, 3, (10, 20, 30), 64, seed=17)
+    pos = np.array([10, 20, 30], dtype=np.int32)
+    ids = np.array([1, 2, 3], dtype=np.int32)
+    h1, n1 = p.gpu_step(pos, ids=ids)
+    c1 = p.cap.cpu().numpy().copy()
+    h2, n2 = p.gpu_step(pos, ids=ids)  # rewrites the same slots with the same values
+    assert np.array_equal(h1, h2) and np.array_equal(n1, n2)
+    K.kfl_stage_profile(p.st, True)
+    h3, n3 = p.gpu_step(pos, ids=ids)
+    prof = K.kfl_stage_profile_read(p.st)
+    K.kfl_stage_profile(p.st, False)
+    assert np.array_equal(h1, h3) and np.array_equal(n1, n3)
+    assert np.array_equal(c1, p.cap.cpu().numpy())
+    assert prof["qkv"][1] == 3 and prof["attn"][1] == 3 and prof["lmhead"][1] == 1
+    assert all(ms > 0 for ms, n in prof.values() if n > 0)
+    assert K.kfl_stage_launches_per_step(p.st, 3) == 2 + 5 * 3 + 1
+    p.close()
+
+
+def test_decode_host_buffers_match_device_buffers():
+    p = Pair(RAGGED, 0, 2, K.KFL_LOGITS_OUT, 2, (10, 11), 64, seed=18)
+    pos = np.array([10, 11], dtype=np.int32)
+    h = wl.hidden_in(RAGGED, 0, 2, 18)
+    hd, nd = p.gpu_step(pos, hidden=h)
+    hh, nh = p.gpu_step(pos, hidden=h, host=True)
+    assert np.array_equal(hd, hh) and np.array_equal(nd, nh)
+    p.close()
+
+
+def test_bad_position_and_token_are_reported_not_faulted():
+    p = Pair(RAGGED, 0, 1, K.KFL_IS_HEAD, 2, (5, 6), 64, seed=19)
+    k_before = np.zeros((2, 64, 64), dtype=np.uint16)
+    v_before = np.zeros_like(k_before)
+    K.kfl_kv_read(p.st, 0, 1, k_before, v_before, False)
+    p.gpu_step(np.array([5, 64], dtype=np.int32), ids=np.array([1, 2], dtype=np.int32))
+    assert K.kfl_stage_status(p.st) == -2
+    k_after = np.zeros_like(k_before)
+    v_after = np.zeros_like(k_before)
+    K.kfl_kv_read(p.st, 0, 1, k_after, v_after, False)
+    assert np.array_equal(k_before, k_after) and np.array_equal(v_before, v_after)
+    p.gpu_step(np.array([5, 6], dtype=np.int32), ids=np.array([1, RAGGED.vocab], dtype=np.int32))
+    assert K.kfl_stage_status(p.st) == -2
+    # the stage stays usable
+    p.step(0, ids=np.array([1, 2], dtype=np.int32))
+    assert K.kfl_stage_status(p.st) == 0
+    p.close()
+
+
+def test_batch_above_max_and_unloaded_stage_are_refused():
+    cfg = K.model_cfg(RAGGED, 64, 2)
+    st = K.kfl_stage_create(cfg, 0, 1, 0)
+    d = torch.zeros(3, RAGGED.d_model, device="cuda")
+    pos = torch.zeros(3, dtype=torch.int32, device="cuda")
+    with pytest.raises(K.KflError) as e:
+        K.kfl_stage_decode(st, None, d, pos, 1, d, None)
+    assert e.value.code == -5  # weights not loaded
+    K.kfl_stage_load_layer(st, 0, wl.layer_weights(RAGGED, 0, 1), on_device=False)
+    with pytest.raises(K.KflError) as e:
+        K.kfl_stage_decode(st, None, d, pos, 3, d, None)
+    assert e.value.code == -2
+    K.kfl_stage_destroy(st)
+
+
+def test_allocation_failure_is_reported_and_recoverable(monkeypatch):
+    cfg = K.model_cfg(RAGGED, 64, 2)
+    for n in (1, 5, 12):
+        monkeypatch.setenv("KFL_FAULT_ALLOC_AT", str(n))
+        with pytest.raises(K.KflError) as e:
+            K.kfl_stage_create(cfg, 0, 2, K.KFL_IS_HEAD)
+        assert e.value.code == -3
+    monkeypatch.delenv("KFL_FAULT_ALLOC_AT")
+    st = K.kfl_stage_create(cfg, 0, 2, K.KFL_IS_HEAD)
+    K.kfl_stage_destroy(st)
+
+
+def test_kv_reset_and_seeded_fill_match_the_host_generator():
+    m = RAGGED
+    cfg = K.model_cfg(m, 96, 3)
+    st = K.kfl_stage_create(cfg, 1, 3, 0)
+    K.kfl_kv_fill_seeded(st, -1, 70, 21)
+    for local, layer in enumerate((1, 2)):
+        for u in range(3):
+            kg = np.zeros((m.n_kv_heads, 96, m.head_dim), dtype=np.uint16)
+            vg = np.zeros_like(kg)
+            K.kfl_kv_read(st, local, u, kg, vg, False)
+            kh, vh = wl.kv_prefill(m, layer, u, 70, 21)
+            assert np.array_equal(kg[:, :70], kh) and np.array_equal(vg[:, :70], vh)
+            assert not kg[:, 70:].any()
+    K.kfl_kv_reset(st, 1)
+    kg = np.ones((m.n_kv_heads, 96, m.head_dim), dtype=np.uint16)
+    vg = np.ones_like(kg)
+    K.kfl_kv_read(st, 0, 1, kg, vg, False)
+    assert not kg.any() and not vg.any()
+    K.kfl_kv_read(st, 0, 0, kg, vg, False)
+    assert kg.any()
+    K.kfl_stage_destroy(st)
+
+
+def test_device_generator_is_bit_identical_to_host():
+    from paper_2609_34045_gb300 import device_inputs as di
+    n = 3_000_017
+    for std, mean in ((0.02, 0.0), (0.02, 1.0), (1.0, 0.0)):
+        g = di.normal_bf16(7, 1234, n, std, mean).cpu().numpy().view(np.uint16)
+        assert np.array_equal(g, wl.normal_bf16(7, 1234, n, std, mean))
+    words, scales = di.matrix("int4_g64", 7, 55, 56, 64, 4096)
+    hw, hs = wl.matrix("int4_g64", 7, 55, 56, 64, 4096)
+    assert np.array_equal(words.cpu().numpy().view(np.uint32), hw)
+    assert np.array_equal(scales.cpu().numpy().view(np.uint16), hs)
+    # far into a stream (index > 2^32)
+    t = torch.empty(1000, dtype=torch.int16, device="cuda")
+    K.kfl_synth_fill(t, 1000, 7, 9, K.SYNTH_NORMAL_BF16, float(wl.normal_scale(1.0)), 0.0, start=(1 << 33) + 5)
+    idx = np.arange((1 << 33) + 5, (1 << 33) + 1005, dtype=np.uint64)
+    assert np.array_equal(t.cpu().numpy().view(np.uint16), wl.normal_bf16_at(7, 9, idx, 1.0))
+
+
+# ---------------------------------------------------------------------------- full widths
+
+def test_config2_width_bench_launch_shape():
+    """The 7B-shaped body stage at its full width and context, b = 1 (the benchmark's kernels
+    and launch shapes), on two of its blocks."""
+    w = wl.CONFIGS[2]
+    p = Pair(w.model, 0, 2, 0, 1, w.contexts, w.max_ctx, w.seed, device_weights=True)
+    for s in range(2):
+        p.step(s, hidden=wl.hidden_in(w.model, s, 1, w.seed))
+    p.compare_kv()
+    p.close()
+
+
+def test_config3_width_head_with_full_vocab():
+    """The 32B-shaped head: embedding and lm_head over the full 152064-token vocabulary."""
+    w = wl.CONFIGS[3]
+    p = Pair(w.model, 56, 57, K.KFL_IS_HEAD, 1, w.contexts, w.max_ctx, w.seed, device_weights=True)
+    _greedy(p, 2, wl.first_token_ids(w.model, 1, w.seed))
+    p.close()
+
+
+def test_config4_width_four_ragged_users():
+    w = wl.CONFIGS[4]
+    p = Pair(w.model, 0, 1, 0, 4, w.contexts, w.max_ctx, w.seed, device_weights=True)
+    for s in range(2):
+        p.step(s, hidden=wl.hidden_in(w.model, s, 4, w.seed))
+    p.compare_kv()
+    p.close()
+
+
+def test_config5_width_int4_head_b4():
+    w = wl.CONFIGS[6]
+    p = Pair(w.model, 79, 80, K.KFL_IS_HEAD, 4, w.contexts, w.max_ctx, w.seed, device_weights=True)
+    _greedy(p, 1, wl.token_ids(w.seed, 97, 4, w.model.vocab))
+    p.close()
