@@ -16,6 +16,7 @@ namespace kfl {
 constexpr int ATT_THREADS = 128;
 constexpr int ATT_SUB = 64;  // positions per shared-memory sub-tile
 constexpr int ATT_MAXG = 8;
+constexpr int ATT_MERGE_MAX = 2048;  // chunks x heads merged in shared memory (fits the K buffers)
 
 __device__ __forceinline__ void cp_async16(void *dst, const void *src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
@@ -224,21 +225,52 @@ __global__ void __launch_bounds__(ATT_THREADS) attn_kernel(const __grid_constant
   __syncthreads();
   if (!s_last) return;
   __threadfence();
+  // merge: stage every chunk's (m, l) in shared memory (the K buffers are free now), turn them
+  // into per-chunk weights 2^(m_c - M) / L once per head, then each thread sums its outputs
+  // over the chunks with independent loads
   const float *base = p.partial + (((size_t)b * p.n_kv_heads + kvh) * p.n_chunks) * (ATT_MAXG * pstride);
+  float *wm = reinterpret_cast<float *>(sk);  // [nc][G] weights (host keeps nc * G <= ATT_MERGE_MAX)
+  float *wl = wm + ATT_MERGE_MAX;             // [nc][G] l values
+  for (int e = tid; e < nc * G; e += ATT_THREADS) {
+    const int cc = e / G, g = e % G;
+    const float *pc = base + (size_t)cc * ATT_MAXG * pstride + g * pstride;
+    wm[e] = __ldcg(pc + HD);
+    wl[e] = __ldcg(pc + HD + 1);
+  }
+  __syncthreads();
+  for (int g = warp; g < G; g += ATT_THREADS / 32) {
+    float M = -INFINITY;
+    for (int cc = lane; cc < nc; cc += 32) M = fmaxf(M, wm[cc * G + g]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    float Lsum = 0.f;
+    for (int cc = lane; cc < nc; cc += 32) Lsum += wl[cc * G + g] * exp2f(wm[cc * G + g] - M);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, off);
+    __syncwarp();
+    const float invL = 1.0f / Lsum;
+    for (int cc = lane; cc < nc; cc += 32) wm[cc * G + g] = exp2f(wm[cc * G + g] - M) * invL;
+  }
+  __syncthreads();
 #pragma unroll 1
   for (int k = 0; k < ATT_MAXG / DSPLIT; ++k) {
     const int g = gpar + DSPLIT * k;
     if (g >= G) continue;
-    float M = -INFINITY;
-    for (int cc = 0; cc < nc; ++cc) M = fmaxf(M, __ldcg(base + (size_t)cc * ATT_MAXG * pstride + g * pstride + HD));
-    float Lsum = 0.f, O = 0.f;
-    for (int cc = 0; cc < nc; ++cc) {
-      const float *pc = base + (size_t)cc * ATT_MAXG * pstride + g * pstride;
-      const float w = exp2f(__ldcg(pc + HD) - M);
-      Lsum = fmaf(__ldcg(pc + HD + 1), w, Lsum);
-      O = fmaf(__ldcg(pc + d), w, O);
+    const float *pg = base + g * pstride + d;
+    float O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
+    int cc = 0;
+    for (; cc + 4 <= nc; cc += 4) {
+      const float a0 = __ldcg(pg + (size_t)cc * ATT_MAXG * pstride);
+      const float a1 = __ldcg(pg + (size_t)(cc + 1) * ATT_MAXG * pstride);
+      const float a2 = __ldcg(pg + (size_t)(cc + 2) * ATT_MAXG * pstride);
+      const float a3 = __ldcg(pg + (size_t)(cc + 3) * ATT_MAXG * pstride);
+      O0 = fmaf(wm[cc * G + g], a0, O0);
+      O1 = fmaf(wm[(cc + 1) * G + g], a1, O1);
+      O2 = fmaf(wm[(cc + 2) * G + g], a2, O2);
+      O3 = fmaf(wm[(cc + 3) * G + g], a3, O3);
     }
-    o[g * HD + d] = O / Lsum;
+    for (; cc < nc; ++cc) O0 = fmaf(wm[cc * G + g], __ldcg(pg + (size_t)cc * ATT_MAXG * pstride), O0);
+    o[g * HD + d] = (O0 + O1) + (O2 + O3);
   }
 }
 
@@ -266,6 +298,7 @@ static cudaError_t launch_hd(const AttnParams &p, cudaStream_t s, bool pdl) {
 
 cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s, bool pdl) {
   if (p.n_heads % p.n_kv_heads != 0 || p.n_heads / p.n_kv_heads > ATT_MAXG) return cudaErrorInvalidValue;
+  if (p.n_chunks * (p.n_heads / p.n_kv_heads) > ATT_MERGE_MAX) return cudaErrorInvalidValue;
   if (head_dim == 128) return launch_hd<128>(p, s, pdl);
   if (head_dim == 64) return launch_hd<64>(p, s, pdl);
   return cudaErrorInvalidValue;

@@ -24,6 +24,21 @@
 
 namespace kfl {
 
+// (a0, a1) += (w0, w1) * (x0, x1) with one packed fp32x2 FMA (sm_100+)
+__device__ __forceinline__ void ffma2(float &a0, float &a1, float w0, float w1, float x0, float x1) {
+  asm("{\n\t.reg .b64 a, w, x;\n\t"
+      "mov.b64 a, {%0, %1};\n\tmov.b64 w, {%2, %3};\n\tmov.b64 x, {%4, %5};\n\t"
+      "fma.rn.f32x2 a, w, x, a;\n\tmov.b64 {%0, %1}, a;\n\t}"
+      : "+f"(a0), "+f"(a1)
+      : "f"(w0), "f"(w1), "f"(x0), "f"(x1));
+}
+
+// Signed 4-bit code j of a word as an exact float: the offset-binary nibble (code ^ 8) is
+// placed in the mantissa of 2^23, and 2^23 + 8 is subtracted.
+__device__ __forceinline__ float int4_code(uint32_t word, int j) {
+  return __uint_as_float(((word >> (4 * j)) & 0xFu) ^ 0x4B000008u) - 8388616.0f;
+}
+
 __device__ __forceinline__ int cta_of_tile(long long t, long long T, int G) {
   // the largest c with floor(c*T/G) <= t
   return static_cast<int>(((t + 1) * G - 1) / T);
@@ -192,7 +207,7 @@ __device__ __forceinline__ void epilogue(const GemvParams &p, int rb, const floa
 // ---------------------------------------------------------------------------- the kernel
 // FMT 0: bf16 tiles [RB][KT].  FMT 1: int4 tiles, codes [RB][KT4/8] uint32 + scales [RB][KT4/64].
 template <int B, int EPI, int FMT>
-__global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const __grid_constant__ GemvParams p) {
+__global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) gemv_kernel(const __grid_constant__ GemvParams p) {
   extern __shared__ __align__(1024) uint8_t smem[];
   const int S = p.stages;
   uint64_t *full = reinterpret_cast<uint64_t *>(smem + (size_t)S * STAGE_BYTES);
@@ -202,7 +217,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const __grid_cons
   __shared__ float s_inv[MAXB];
   __shared__ int s_last;
   __shared__ volatile int s_abort;
-  __shared__ int s_issued;
+  __shared__ volatile int s_issued;
 
   constexpr int KTILE = FMT == 0 ? KT : KT4;
   constexpr uint32_t WBYTES = FMT == 0 ? TILE_BYTES : TILE4_BYTES;
@@ -235,30 +250,36 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const __grid_cons
         const uint32_t fb = smem_addr(&full[i]);
         mbar_arrive_expect_tx(fb, WBYTES + xbytes);
         bulk_g2s(smem_addr(smem + (size_t)i * STAGE_BYTES), p.w + (size_t)(t0 + i) * WBYTES, WBYTES, fb, pol_w);
+        s_issued = i + 1;
       }
       pdl_wait();
-      auto issue_x = [&](int i, int s) {
-        const long long t = t0 + i;
-        const int kt = static_cast<int>(t % p.n_kt);
+      auto issue_x = [&](int kt, int s) {
         const uint32_t fb = smem_addr(&full[s]);
         const uint32_t dst = smem_addr(smem + (size_t)s * STAGE_BYTES + WBYTES);
 #pragma unroll
         for (int b = 0; b < B; ++b)
           bulk_g2s(dst + b * (KTILE * 4), p.x + (size_t)b * p.ldx + (size_t)kt * KTILE, KTILE * 4, fb, pol_x);
       };
-      for (int i = 0; i < pre; ++i) issue_x(i, i);
-      int issued = pre;
+      int kt_x = static_cast<int>(t0 % p.n_kt);
+      for (int i = 0; i < pre; ++i) {
+        issue_x(kt_x, i);
+        if (++kt_x == p.n_kt) kt_x = 0;
+      }
+      int s = 0;
+      uint32_t eph = 0;
       for (int i = pre; i < n; ++i) {
-        const int s = i % S;
-        const uint32_t par = ((i / S) - 1) & 1;
-        if (!consumer_wait(smem_addr(&empty[s]), par, &s_abort, p.err)) break;
+        if (!consumer_wait(smem_addr(&empty[s]), eph, &s_abort, p.err)) break;
         const uint32_t fb = smem_addr(&full[s]);
         mbar_arrive_expect_tx(fb, WBYTES + xbytes);
         bulk_g2s(smem_addr(smem + (size_t)s * STAGE_BYTES), p.w + (size_t)(t0 + i) * WBYTES, WBYTES, fb, pol_w);
-        issue_x(i, s);
-        issued = i + 1;
+        issue_x(kt_x, s);
+        s_issued = i + 1;
+        if (++kt_x == p.n_kt) kt_x = 0;
+        if (++s == S) {
+          s = 0;
+          eph ^= 1u;
+        }
       }
-      s_issued = issued;
     }
     return;
   }
@@ -279,21 +300,22 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const __grid_cons
   // bf16: lane -> 8 consecutive K (chunk kc) of rows warp*8 + rsub + 2j, j < 4
   // int4: lane -> 16 consecutive K (chunk kc) of the same rows
   const int kc = lane & 15, rsub = lane >> 4;
-  float acc[B][4];
+  // accumulators: (even-K, odd-K) partial sums per (user, row), added at the segment end
+  float acc[B][4][2];
   int seg_kt0 = 0;
+  int rb = static_cast<int>(t0 / p.n_kt);
+  int kt = static_cast<int>(t0 - (long long)rb * p.n_kt);
+  int s = 0;
+  uint32_t phase = 0;
   for (int i = 0; i < n; ++i) {
-    const long long t = t0 + i;
-    const int rb = static_cast<int>(t / p.n_kt);
-    const int kt = static_cast<int>(t - (long long)rb * p.n_kt);
     if (i == 0 || kt == 0) {
 #pragma unroll
       for (int b = 0; b < B; ++b)
 #pragma unroll
-        for (int j = 0; j < 4; ++j) acc[b][j] = 0.f;
+        for (int j = 0; j < 4; ++j) acc[b][j][0] = acc[b][j][1] = 0.f;
       seg_kt0 = kt;
     }
-    const int s = i % S;
-    consumer_wait(smem_addr(&full[s]), (i / S) & 1, &s_abort, p.err);
+    consumer_wait(smem_addr(&full[s]), phase, &s_abort, p.err);
     const uint8_t *st = smem + (size_t)s * STAGE_BYTES;
     if constexpr (FMT == 0) {
       float xv[B][8];
@@ -308,46 +330,52 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const __grid_cons
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const uint4 w4 = wp[j * 2 * (KT / 8)];
-        float w[8];
-        w[0] = bf16_lo(w4.x); w[1] = bf16_hi(w4.x); w[2] = bf16_lo(w4.y); w[3] = bf16_hi(w4.y);
-        w[4] = bf16_lo(w4.z); w[5] = bf16_hi(w4.z); w[6] = bf16_lo(w4.w); w[7] = bf16_hi(w4.w);
+        const uint32_t wu[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
-        for (int b = 0; b < B; ++b)
+        for (int e = 0; e < 4; ++e) {
+          const float wl = bf16_lo(wu[e]), wh = bf16_hi(wu[e]);
 #pragma unroll
-          for (int e = 0; e < 8; ++e) acc[b][j] = fmaf(w[e], xv[b][e], acc[b][j]);
+          for (int b = 0; b < B; ++b) ffma2(acc[b][j][0], acc[b][j][1], wl, wh, xv[b][2 * e], xv[b][2 * e + 1]);
+        }
       }
     } else {
-      // int4 tile: codes [RB][KT4/8] uint32 (32 words = 128 B per row), scales [RB][4] bf16
+      // int4 tile: codes [RB][KT4/8] uint32 (32 words = 128 B per row), scales [RB][4] bf16.
+      // The lane's 16 codes of a row (two words, one scale group) are taken a word at a time
+      // so that only 8 activations per user are live.
       const float4 *xp = reinterpret_cast<const float4 *>(st + TILE4_BYTES) + kc * 4;
-      float xv[B][16];
-#pragma unroll
-      for (int b = 0; b < B; ++b) {
-#pragma unroll
-        for (int v = 0; v < 4; ++v) {
-          const float4 a = xp[b * (KT4 / 4) + v];
-          xv[b][4 * v] = a.x; xv[b][4 * v + 1] = a.y; xv[b][4 * v + 2] = a.z; xv[b][4 * v + 3] = a.w;
-        }
-      }
       const uint2 *cp = reinterpret_cast<const uint2 *>(st) + (warp * 8 + rsub) * (KT4 / 16) + kc;
       const uint16_t *sp = reinterpret_cast<const uint16_t *>(st + TILE4_CODE_BYTES);
+      uint2 cw[4];
+      float sc[4];
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        const int r = warp * 8 + rsub + 2 * j;
-        const uint2 cw = cp[j * 2 * (KT4 / 16)];
-        const float sc = bf16_to_f32(sp[r * (KT4 / 64) + (kc >> 2)]);
-        float part[B];
+        cw[j] = cp[j * 2 * (KT4 / 16)];
+        sc[j] = bf16_to_f32(sp[(warp * 8 + rsub + 2 * j) * (KT4 / 64) + (kc >> 2)]);
+      }
 #pragma unroll
-        for (int b = 0; b < B; ++b) part[b] = 0.f;
+      for (int hw = 0; hw < 2; ++hw) {
+        float xv[B][8];
 #pragma unroll
-        for (int e = 0; e < 16; ++e) {
-          const uint32_t word = e < 8 ? cw.x : cw.y;
-          const int q = static_cast<int>(word << (28 - 4 * (e & 7))) >> 28;  // sign-extended nibble
-          const float wq = static_cast<float>(q);
-#pragma unroll
-          for (int b = 0; b < B; ++b) part[b] = fmaf(wq, xv[b][e], part[b]);
+        for (int b = 0; b < B; ++b) {
+          const float4 a0 = xp[b * (KT4 / 4) + 2 * hw], a1 = xp[b * (KT4 / 4) + 2 * hw + 1];
+          xv[b][0] = a0.x; xv[b][1] = a0.y; xv[b][2] = a0.z; xv[b][3] = a0.w;
+          xv[b][4] = a1.x; xv[b][5] = a1.y; xv[b][6] = a1.z; xv[b][7] = a1.w;
         }
 #pragma unroll
-        for (int b = 0; b < B; ++b) acc[b][j] = fmaf(sc, part[b], acc[b][j]);
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t word = hw ? cw[j].y : cw[j].x;
+          float part[B][2];
+#pragma unroll
+          for (int b = 0; b < B; ++b) part[b][0] = part[b][1] = 0.f;
+#pragma unroll
+          for (int e = 0; e < 8; e += 2) {
+            const float q0 = int4_code(word, e), q1 = int4_code(word, e + 1);
+#pragma unroll
+            for (int b = 0; b < B; ++b) ffma2(part[b][0], part[b][1], q0, q1, xv[b][e], xv[b][e + 1]);
+          }
+#pragma unroll
+          for (int b = 0; b < B; ++b) ffma2(acc[b][j][0], acc[b][j][1], sc[j], sc[j], part[b][0], part[b][1]);
+        }
       }
     }
     __syncwarp();
@@ -355,22 +383,23 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const __grid_cons
 
     if (kt == p.n_kt - 1 || i == n - 1) {
       // ---- segment end: reduce over the 16 lanes sharing a row
+      float tot[B][4];
 #pragma unroll
       for (int b = 0; b < B; ++b)
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          float v = acc[b][j];
+          float v = acc[b][j][0] + acc[b][j][1];
           v += __shfl_xor_sync(0xffffffffu, v, 8);
           v += __shfl_xor_sync(0xffffffffu, v, 4);
           v += __shfl_xor_sync(0xffffffffu, v, 2);
           v += __shfl_xor_sync(0xffffffffu, v, 1);
-          acc[b][j] = v;
+          tot[b][j] = v;
         }
       if (kc == 0) {
 #pragma unroll
         for (int j = 0; j < 4; ++j)
 #pragma unroll
-          for (int b = 0; b < B; ++b) red[(warp * 8 + rsub + 2 * j) * MAXB + b] = acc[b][j];
+          for (int b = 0; b < B; ++b) red[(warp * 8 + rsub + 2 * j) * MAXB + b] = tot[b][j];
       }
       named_bar_sync(1, CONSUMER_WARPS * 32);
       bool do_epi = true;
@@ -407,6 +436,14 @@ __global__ void __launch_bounds__(GEMV_THREADS, 1) gemv_kernel(const __grid_cons
       }
       if (do_epi) epilogue<B, EPI>(p, rb, red, s_inv, scr, tid);
       named_bar_sync(1, CONSUMER_WARPS * 32);
+    }
+    if (++kt == p.n_kt) {
+      kt = 0;
+      ++rb;
+    }
+    if (++s == S) {
+      s = 0;
+      phase ^= 1u;
     }
   }
 

@@ -217,12 +217,20 @@ bool valid(const kfl_stage *st) { return st && st->magic == 0x4B464C53; }
     }                                       \
   } while (0)
 
+// Positions per attention CTA: about three CTAs per SM over the reserved context, at least two
+// 64-position sub-tiles each, and few enough chunks for the merge (chunks x group <= 2048).
 int attn_chunk_for(const kfl_stage *st, int batch) {
   const Plan &P = st->P;
-  const long long work = (long long)st->cfg.max_ctx * batch * P.hkv;
-  long long want = (work + 2LL * P.n_sm - 1) / (2LL * P.n_sm);
-  int chunk = round_up((int)(want < 64 ? 64 : want), 64);
-  if (chunk > round_up(st->cfg.max_ctx, 64)) chunk = round_up(st->cfg.max_ctx, 64);
+  const int max_ctx = st->cfg.max_ctx;
+  const long long work = (long long)max_ctx * batch * P.hkv;
+  long long want = (work + 3LL * P.n_sm - 1) / (3LL * P.n_sm);
+  const int group = P.hq / P.hkv;
+  const long long min_for_merge = ((long long)max_ctx * group + 2047) / 2048;
+  if (want < min_for_merge) want = min_for_merge;
+  if (want < 128) want = 128;
+  int chunk = round_up((int)want, 64);
+  while ((long long)((max_ctx + chunk - 1) / chunk) * group > 2048) chunk += 64;
+  if (chunk > round_up(max_ctx, 64)) chunk = round_up(max_ctx, 64);
   return chunk;
 }
 
