@@ -1,0 +1,297 @@
+// Grouped-query decode attention over one chunk of cached positions (flash-decoding unit),
+// shared by the standalone attention kernel (attention.cu) and the persistent stage kernel.
+//
+// User b's token at position P_b attends to its cached slots [0, P_b] (its own K/V were
+// appended by the QKV epilogue), query head h reading KV head h / G.  A unit is one (user, KV
+// head, chunk of positions): the chunk's K and V rows are loaded once (cp.async, 64-position
+// sub-tiles, double buffered) for all G query heads that share the KV head; an online-softmax
+// state (running max m, running sum l, weighted sum of V) is kept per head.  A single-chunk
+// unit writes its output directly; otherwise each unit writes (m, l, acc) and the last unit of
+// its (user, KV head) to finish (atomic ticket, no spin) merges the chunks in chunk order.
+// Scores are in the log2 domain (q pre-scaled by log2(e)/sqrt(hd)).
+//
+// 256 threads.  Scores: 4 lanes per position, each a quarter of the head dimension, for every
+// head.  P.V: one warp per head (two per warp at hd 64), 4 dimensions per lane.
+#pragma once
+
+#include <math.h>
+
+#include "common.cuh"
+
+namespace kfl {
+
+constexpr int ATT_THREADS = 256;
+constexpr int ATT_SUB = 64;          // positions per shared-memory sub-tile
+constexpr int ATT_MAXG = 8;          // query heads per KV head
+constexpr int ATT_MERGE_MAX = 2048;  // chunks x heads merged in shared memory (fits the K buffers)
+constexpr int ATT_BAR = 2;           // named barrier of the attention threads
+
+__device__ __forceinline__ void att_sync() { named_bar_sync(ATT_BAR, ATT_THREADS); }
+
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+template <int HD>
+struct AttnLayout {
+  // K row: four quarters of hd/4 dims, each padded by 16 bytes, so the four lanes reading the
+  // quarters of one position and the next position's lanes hit distinct banks
+  static constexpr int QB = HD / 2 + 16;
+  static constexpr int KROW = 4 * QB;
+  static constexpr int VROW = HD * 2;
+  static constexpr int QQ = HD / 4 + 4;     // floats per padded quarter of a q row
+  static constexpr int K_OFF = 0;
+  static constexpr int V_OFF = K_OFF + 2 * ATT_SUB * KROW;
+  static constexpr int Q_OFF = V_OFF + 2 * ATT_SUB * VROW;
+  static constexpr int S_OFF = Q_OFF + ATT_MAXG * 4 * QQ * 4;
+  static constexpr int M_OFF = S_OFF + ATT_MAXG * ATT_SUB * 4;
+  static constexpr int BYTES = M_OFF + 4 * ATT_MAXG * 4;
+  static_assert(2 * ATT_MERGE_MAX * 4 <= 2 * ATT_SUB * KROW, "merge scratch must fit the K buffers");
+};
+
+__host__ __device__ constexpr int attn_pstride(int hd) { return hd + 4; }
+
+// Number of chunks of user b (1 for an invalid position: that unit writes zeros).
+__device__ __forceinline__ int attn_chunks(const AttnParams &p, int b) {
+  const int P = __ldcg(p.positions + b);
+  if (P < 0 || P >= p.max_ctx) return 1;
+  return (P + 1 + p.chunk - 1) / p.chunk;
+}
+
+template <int HD>
+__device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, uint8_t *sm, int *s_last, int tid) {
+  using L = AttnLayout<HD>;
+  uint8_t *sk = sm + L::K_OFF;
+  uint8_t *sv = sm + L::V_OFF;
+  float *sq = reinterpret_cast<float *>(sm + L::Q_OFF);
+  float *ss = reinterpret_cast<float *>(sm + L::S_OFF);
+  float *s_m = reinterpret_cast<float *>(sm + L::M_OFF);
+  float *s_l = s_m + ATT_MAXG;
+  float *s_alpha = s_l + ATT_MAXG;
+  const int warp = tid >> 5, lane = tid & 31;
+  const int G = p.n_heads / p.n_kv_heads;
+  // P.V / output mapping: head og, dimensions od .. od + 3
+  const int og = (HD == 128) ? warp : 2 * warp + (lane >> 4);
+  const int od = 4 * ((HD == 128) ? lane : (lane & 15));
+  const bool owns = og < G;
+  float *o = p.o + (size_t)b * p.ldo + (size_t)kvh * G * HD;
+
+  const int P = __ldcg(p.positions + b);
+  if (P < 0 || P >= p.max_ctx) {
+    // the stage input flagged the position; leave a defined (zero) output
+    if (owns) *reinterpret_cast<float4 *>(o + og * HD + od) = make_float4(0.f, 0.f, 0.f, 0.f);
+    return;
+  }
+  const int ntok = P + 1;
+  const int start = c * p.chunk;
+  const int end = min(ntok, start + p.chunk);
+  const size_t head_base = ((size_t)b * p.n_kv_heads + kvh) * p.max_ctx;
+  const uint16_t *kg = p.kcache + head_base * HD;
+  const uint16_t *vg = p.vcache + head_base * HD;
+
+  for (int e = tid; e < G * HD; e += ATT_THREADS) {
+    const int g = e / HD, d = e % HD;
+    sq[g * 4 * L::QQ + (d / (HD / 4)) * L::QQ + d % (HD / 4)] =
+        __ldcg(p.q + (size_t)b * p.n_heads * HD + (size_t)kvh * G * HD + e) * p.scale_log2;
+  }
+  if (tid < ATT_MAXG) {
+    s_m[tid] = -INFINITY;
+    s_l[tid] = 0.f;
+  }
+
+  auto load_sub = [&](int sub, int buf) {
+    const int p0 = start + sub * ATT_SUB;
+    const int cnt = min(ATT_SUB, end - p0);
+    constexpr int CH = HD / 8;   // 16-byte chunks per row
+    constexpr int CQ = HD / 32;  // chunks per quarter
+    for (int e = tid; e < cnt * CH; e += ATT_THREADS) {
+      const int r = e / CH, ch = e % CH;
+      cp_async16(sk + buf * ATT_SUB * L::KROW + r * L::KROW + (ch / CQ) * L::QB + (ch % CQ) * 16,
+                 kg + (size_t)(p0 + r) * HD + ch * 8);
+      cp_async16(sv + buf * ATT_SUB * L::VROW + r * L::VROW + ch * 16, vg + (size_t)(p0 + r) * HD + ch * 8);
+    }
+    cp_async_commit();
+  };
+
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  const int nsub = (end - start + ATT_SUB - 1) / ATT_SUB;
+  load_sub(0, 0);
+  for (int it = 0; it < nsub; ++it) {
+    const int buf = it & 1;
+    if (it + 1 < nsub) {
+      load_sub(it + 1, buf ^ 1);
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    att_sync();
+    const int p0 = start + it * ATT_SUB;
+    const int cnt = min(ATT_SUB, end - p0);
+    const uint8_t *kb = sk + buf * ATT_SUB * L::KROW;
+    const uint8_t *vb = sv + buf * ATT_SUB * L::VROW;
+
+    // scores: lanes 4i..4i+3 share position i, each a quarter of the head dimension
+    {
+      const int pp = tid >> 2, qq = tid & 3;
+      const bool valid = pp < cnt;
+      float kf[HD / 4];
+      const uint4 *kr = reinterpret_cast<const uint4 *>(kb + pp * L::KROW + qq * L::QB);
+#pragma unroll
+      for (int ch = 0; ch < HD / 32; ++ch) {
+        const uint4 k4 = valid ? kr[ch] : make_uint4(0u, 0u, 0u, 0u);
+        kf[8 * ch] = bf16_lo(k4.x); kf[8 * ch + 1] = bf16_hi(k4.x);
+        kf[8 * ch + 2] = bf16_lo(k4.y); kf[8 * ch + 3] = bf16_hi(k4.y);
+        kf[8 * ch + 4] = bf16_lo(k4.z); kf[8 * ch + 5] = bf16_hi(k4.z);
+        kf[8 * ch + 6] = bf16_lo(k4.w); kf[8 * ch + 7] = bf16_hi(k4.w);
+      }
+#pragma unroll
+      for (int g = 0; g < ATT_MAXG; ++g) {
+        if (g < G) {
+          const float4 *qr = reinterpret_cast<const float4 *>(sq + g * 4 * L::QQ + qq * L::QQ);
+          float d0 = 0.f, d1 = 0.f;
+#pragma unroll
+          for (int i = 0; i < HD / 16; ++i) {
+            const float4 q4 = qr[i];
+            d0 = fmaf(kf[4 * i], q4.x, d0);
+            d1 = fmaf(kf[4 * i + 1], q4.y, d1);
+            d0 = fmaf(kf[4 * i + 2], q4.z, d0);
+            d1 = fmaf(kf[4 * i + 3], q4.w, d1);
+          }
+          float dot = d0 + d1;
+          dot += __shfl_xor_sync(0xffffffffu, dot, 1);
+          dot += __shfl_xor_sync(0xffffffffu, dot, 2);
+          if (qq == 0) ss[g * ATT_SUB + pp] = valid ? dot : -INFINITY;
+        }
+      }
+    }
+    att_sync();
+    // online softmax update: warp g owns head g
+    if (warp < G) {
+      const int g = warp;
+      const float a0 = ss[g * ATT_SUB + lane], a1 = ss[g * ATT_SUB + lane + 32];
+      float mx = fmaxf(a0, a1);
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+      const float m_old = s_m[g];
+      const float m_new = fmaxf(m_old, mx);
+      const float e0 = exp2f(a0 - m_new), e1 = exp2f(a1 - m_new);
+      float sum = e0 + e1;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+      ss[g * ATT_SUB + lane] = e0;
+      ss[g * ATT_SUB + lane + 32] = e1;
+      __syncwarp();
+      if (lane == 0) {
+        const float alpha = exp2f(m_old - m_new);
+        s_alpha[g] = alpha;
+        s_l[g] = s_l[g] * alpha + sum;
+        s_m[g] = m_new;
+      }
+    }
+    att_sync();
+    // acc = acc * alpha + P . V over the sub-tile's valid positions
+    if (owns) {
+      const float al = s_alpha[og];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) acc[i] *= al;
+      const float *pr = ss + og * ATT_SUB;
+      int pp = 0;
+      for (; pp + 4 <= cnt; pp += 4) {
+        const float4 p4 = *reinterpret_cast<const float4 *>(pr + pp);
+        const float pw[4] = {p4.x, p4.y, p4.z, p4.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const uint2 v2 = *reinterpret_cast<const uint2 *>(vb + (pp + k) * L::VROW + od * 2);
+          acc[0] = fmaf(pw[k], bf16_lo(v2.x), acc[0]);
+          acc[1] = fmaf(pw[k], bf16_hi(v2.x), acc[1]);
+          acc[2] = fmaf(pw[k], bf16_lo(v2.y), acc[2]);
+          acc[3] = fmaf(pw[k], bf16_hi(v2.y), acc[3]);
+        }
+      }
+      for (; pp < cnt; ++pp) {
+        const float pw = pr[pp];
+        const uint2 v2 = *reinterpret_cast<const uint2 *>(vb + pp * L::VROW + od * 2);
+        acc[0] = fmaf(pw, bf16_lo(v2.x), acc[0]);
+        acc[1] = fmaf(pw, bf16_hi(v2.x), acc[1]);
+        acc[2] = fmaf(pw, bf16_lo(v2.y), acc[2]);
+        acc[3] = fmaf(pw, bf16_hi(v2.y), acc[3]);
+      }
+    }
+    att_sync();
+  }
+
+  if (nc == 1) {
+    if (owns) {
+      const float il = 1.0f / s_l[og];
+      *reinterpret_cast<float4 *>(o + og * HD + od) = make_float4(acc[0] * il, acc[1] * il, acc[2] * il, acc[3] * il);
+    }
+    return;
+  }
+  constexpr int PS = attn_pstride(HD);
+  const size_t unit_base = ((size_t)b * p.n_kv_heads + kvh) * p.n_chunks;
+  float *part = p.partial + (unit_base + c) * (ATT_MAXG * PS);
+  if (owns) *reinterpret_cast<float4 *>(part + og * PS + od) = make_float4(acc[0], acc[1], acc[2], acc[3]);
+  if (tid < G) {
+    part[tid * PS + HD] = s_m[tid];
+    part[tid * PS + HD + 1] = s_l[tid];
+  }
+  __threadfence();
+  att_sync();
+  if (tid == 0) {
+    int *tk = p.tickets + b * p.n_kv_heads + kvh;
+    const int prev = atomicAdd(tk, 1);
+    *s_last = (prev == nc - 1);
+    if (*s_last) atomicExch(tk, 0);
+  }
+  att_sync();
+  if (!*s_last) return;
+  __threadfence();
+  // merge: per-chunk weights 2^(m_c - M) / L staged in shared memory (the K buffers), then each
+  // thread sums its 4 outputs over the chunks
+  const float *base = p.partial + unit_base * (ATT_MAXG * PS);
+  float *wm = reinterpret_cast<float *>(sk);
+  float *wl = wm + ATT_MERGE_MAX;
+  for (int e = tid; e < nc * G; e += ATT_THREADS) {
+    const int cc = e / G, g = e % G;
+    const float *pc = base + (size_t)cc * ATT_MAXG * PS + g * PS;
+    wm[e] = __ldcg(pc + HD);
+    wl[e] = __ldcg(pc + HD + 1);
+  }
+  att_sync();
+  if (warp < G) {
+    const int g = warp;
+    float M = -INFINITY;
+    for (int cc = lane; cc < nc; cc += 32) M = fmaxf(M, wm[cc * G + g]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    float Lsum = 0.f;
+    for (int cc = lane; cc < nc; cc += 32) Lsum += wl[cc * G + g] * exp2f(wm[cc * G + g] - M);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, off);
+    __syncwarp();
+    const float invL = 1.0f / Lsum;
+    for (int cc = lane; cc < nc; cc += 32) wm[cc * G + g] = exp2f(wm[cc * G + g] - M) * invL;
+  }
+  att_sync();
+  if (owns) {
+    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+    const float *pg = base + og * PS + od;
+#pragma unroll 4
+    for (int cc = 0; cc < nc; ++cc) {
+      const float w = wm[cc * G + og];
+      const float4 a = __ldcg(reinterpret_cast<const float4 *>(pg + (size_t)cc * ATT_MAXG * PS));
+      O.x = fmaf(w, a.x, O.x);
+      O.y = fmaf(w, a.y, O.y);
+      O.z = fmaf(w, a.z, O.z);
+      O.w = fmaf(w, a.w, O.w);
+    }
+    *reinterpret_cast<float4 *>(o + og * HD + od) = O;
+  }
+}
+
+}  // namespace kfl

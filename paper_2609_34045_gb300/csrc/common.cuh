@@ -105,6 +105,27 @@ struct AttnParams {
   unsigned *err;
 };
 
+// One phase of the persistent stage kernel: a GEMV (with its epilogue) or an attention pass.
+enum PhaseKind : int { PH_GEMV = 0, PH_ATTN = 1 };
+
+struct Phase {
+  int kind;
+  int epi;
+  GemvParams g;
+  AttnParams a;
+};
+
+struct StageKernelParams {
+  const Phase *phases;  // device array
+  int n_phases;
+  int stages;      // ring stages
+  int head_dim;
+  int attn_bytes;  // shared memory of the attention unit
+  unsigned *bar;   // grid-barrier counter, zeroed by the stage input kernel
+  int *abort_flag; // set when any wait gives up; zeroed by the stage input kernel
+  unsigned *err;
+};
+
 // ---- PTX helpers --------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t smem_addr(const void *p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -206,7 +227,12 @@ cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s, 
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in,
                                int batch, const uint16_t *embed, int vocab, int d, int ldh,
                                const float *g_next, float *h, float *xn, float *sumsq,
-                               int *positions, int max_ctx, unsigned *err, cudaStream_t s);
+                               int *positions, int max_ctx, unsigned *err, unsigned *bar, cudaStream_t s);
+size_t stage_kernel_smem(int stages, int head_dim);
+int stage_kernel_attn_bytes(int head_dim);
+cudaError_t prepare_stage_kernel(size_t smem);
+cudaError_t launch_stage_kernel(const StageKernelParams &kp, int batch, int fmt, int grid, size_t smem,
+                                cudaStream_t s);
 cudaError_t launch_stage_output(const float *h, int ldh, int d, int batch, float *hidden_out,
                                 const int *next_in, int *next_ids, cudaStream_t s, bool pdl);
 cudaError_t launch_repack_bf16(const uint16_t *src, int n_src_rows, int k, const int *row_map,

@@ -11,7 +11,7 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
                                                          const int *positions_in, const uint16_t *embed,
                                                          int vocab, int d, int ldh, const float *g_next,
                                                          float *h, float *xn, float *sumsq, int *positions,
-                                                         int max_ctx, unsigned *err) {
+                                                         int max_ctx, unsigned *err, unsigned *bar) {
   __shared__ float part[2];
   const int b = blockIdx.y, tid = threadIdx.x, r = blockIdx.x * 64 + tid;
   pdl_launch_dependents();
@@ -20,6 +20,11 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
     const int pos = positions_in[b];
     if (pos < 0 || pos >= max_ctx) atomicOr(err, ERR_POSITION);
     positions[b] = pos;
+    // grid-barrier counter and abort flag of the persistent stage kernel that follows
+    if (b == 0 && bar) {
+      bar[0] = 0u;
+      bar[1] = 0u;
+    }
   }
   float v = 0.f;
   if (r < d) {
@@ -47,10 +52,10 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in, int batch,
                                const uint16_t *embed, int vocab, int d, int ldh, const float *g_next, float *h,
                                float *xn, float *sumsq, int *positions, int max_ctx, unsigned *err,
-                               cudaStream_t s) {
+                               unsigned *bar, cudaStream_t s) {
   dim3 grid((d + 63) / 64, batch);
   stage_input_kernel<<<grid, 64, 0, s>>>(ids, hidden_in, positions_in, embed, vocab, d, ldh, g_next, h, xn, sumsq,
-                                         positions, max_ctx, err);
+                                         positions, max_ctx, err, bar);
   return cudaGetLastError();
 }
 

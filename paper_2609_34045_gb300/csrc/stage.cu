@@ -135,10 +135,11 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   ws += (size_t)p->gemv_grid_max * 2 * RB * MAXB * 4;                  // stream-K partials
   ws += (size_t)(p->n_rb_max + 1) * 4;                                 // tickets + argmax ticket
   ws += (size_t)p->n_rb_max * MAXB * 8;                                // argmax candidates
-  ws += (size_t)MAXB * p->hkv * p->attn_nchunks_max * 8 * (p->hd + 2) * 4;  // attention partials
+  ws += (size_t)MAXB * p->hkv * p->attn_nchunks_max * 8 * (p->hd + 4) * 4;  // attention partials
   ws += (size_t)MAXB * p->hkv * 4;                                     // attention tickets
   ws += 16;                                                            // error word
   ws += (size_t)MAXB * (2 + p->d) * 4;                                 // host-decode staging
+  ws += 16;                                                            // grid barrier
   p->bytes_ws = ws;
 }
 
@@ -172,6 +173,14 @@ struct kfl_stage {
   int alloc_count = 0, fault_at = 0;
   cudaStream_t cap_stream = nullptr;
   cudaGraphExec_t graph[MAXB + 1] = {};
+  // persistent stage kernel
+  bool persistent = true;
+  int mk_stages = 0;
+  size_t mk_smem = 0;
+  unsigned *bar = nullptr;  // [0] grid-barrier counter, [1] abort flag
+  Phase *phases_dev[MAXB + 1] = {};
+  int n_phases = 0;
+  int persist_chunk[MAXB + 1] = {};
   bool profile = false;
   std::vector<cudaEvent_t> ev;
   double prof_ms[KFL_KERNEL_KINDS] = {};
@@ -202,6 +211,11 @@ struct kfl_stage {
         cudaGraphExecDestroy(g);
         g = nullptr;
       }
+    for (auto &p : phases_dev)
+      if (p) {
+        cudaFree(p);
+        p = nullptr;
+      }
   }
 };
 
@@ -217,22 +231,8 @@ bool valid(const kfl_stage *st) { return st && st->magic == 0x4B464C53; }
     }                                       \
   } while (0)
 
-// Positions per attention CTA: about three CTAs per SM over the reserved context, at least two
-// 64-position sub-tiles each, and few enough chunks for the merge (chunks x group <= 2048).
-int attn_chunk_for(const kfl_stage *st, int batch) {
-  const Plan &P = st->P;
-  const int max_ctx = st->cfg.max_ctx;
-  const long long work = (long long)max_ctx * batch * P.hkv;
-  long long want = (work + 3LL * P.n_sm - 1) / (3LL * P.n_sm);
-  const int group = P.hq / P.hkv;
-  const long long min_for_merge = ((long long)max_ctx * group + 2047) / 2048;
-  if (want < min_for_merge) want = min_for_merge;
-  if (want < 128) want = 128;
-  int chunk = round_up((int)want, 64);
-  while ((long long)((max_ctx + chunk - 1) / chunk) * group > 2048) chunk += 64;
-  if (chunk > round_up(max_ctx, 64)) chunk = round_up(max_ctx, 64);
-  return chunk;
-}
+// Positions per attention unit: the same in both execution modes, so they give identical bits.
+int attn_chunk_for(const kfl_stage *st, int batch) { return st->persist_chunk[batch]; }
 
 GemvParams base_gemv(kfl_stage *st, const Mat &m, const float *x, int ldx, int batch) {
   GemvParams g = {};
@@ -253,36 +253,25 @@ GemvParams base_gemv(kfl_stage *st, const Mat &m, const float *x, int ldx, int b
   return g;
 }
 
-int gemv_grid(const kfl_stage *st, const Mat &m) {
-  const long long T = (long long)m.n_rb * m.n_kt;
-  return (int)(T < st->P.gemv_grid_max ? T : st->P.gemv_grid_max);
-}
 
-// Enqueue the kernels of the blocks (and lm_head) on stream s.  With `kinds` (profiling mode,
-// no PDL), the k-th kernel is bracketed by events ev[2(ev_base+k)], ev[2(ev_base+k)+1] and
-// its kind is appended to *kinds.
-int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector<int> *kinds, int ev_base) {
+// The phases of one decode step of the stage at this batch size: for every block Q/K/V (+RoPE,
+// KV append), attention, O (+residual), gate/up (+SwiGLU), down (+residual); then lm_head
+// (+argmax) for the head.  Both execution modes run exactly these.
+std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk) {
   const Plan &P = st->P;
   const kfl_model_cfg &c = st->cfg;
-  int k = ev_base;
-  auto pre = [&](int kind) -> int {
-    if (kinds) {
-      CK(cudaEventRecord(st->ev[2 * k], s));
-      kinds->push_back(kind);
-    }
-    return KFL_OK;
+  std::vector<Phase> ph;
+  auto gemv = [&](int epi, const GemvParams &g) {
+    Phase x = {};
+    x.kind = PH_GEMV;
+    x.epi = epi;
+    x.g = g;
+    ph.push_back(x);
   };
-  auto post = [&]() -> int {
-    if (kinds) CK(cudaEventRecord(st->ev[2 * k + 1], s));
-    ++k;
-    return KFL_OK;
-  };
-  const int chunk = attn_chunk_for(st, batch);
   for (int l = 0; l < P.nl; ++l) {
     const LayerDev &L = st->layers[l];
     uint16_t *kcl = st->kc + (size_t)l * P.kv_elems_per_layer;
     uint16_t *vcl = st->vc + (size_t)l * P.kv_elems_per_layer;
-    // Q/K/V with RoPE and KV append
     {
       GemvParams g = base_gemv(st, L.qkv, st->xn, P.ldh, batch);
       g.sumsq = st->sumsq;
@@ -300,13 +289,12 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
       g.head_dim = P.hd;
       g.max_ctx = c.max_ctx;
       g.n_kv_heads = P.hkv;
-      pre(KFL_KERNEL_QKV);
-      CK(launch_gemv(g, EPI_QKV, gemv_grid(st, L.qkv), s, pdl));
-      post();
+      gemv(EPI_QKV, g);
     }
-    // attention
     {
-      AttnParams a = {};
+      Phase x = {};
+      x.kind = PH_ATTN;
+      AttnParams &a = x.a;
       a.q = st->q;
       a.kcache = kcl;
       a.vcache = vcl;
@@ -319,15 +307,12 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
       a.n_heads = P.hq;
       a.n_kv_heads = P.hkv;
       a.max_ctx = c.max_ctx;
-      a.chunk = chunk;
-      a.n_chunks = (c.max_ctx + chunk - 1) / chunk;
+      a.chunk = attn_chunk;
+      a.n_chunks = (c.max_ctx + attn_chunk - 1) / attn_chunk;
       a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)P.hd));
       a.err = st->err;
-      pre(KFL_KERNEL_ATTN);
-      CK(launch_attention(a, P.hd, s, pdl));
-      post();
+      ph.push_back(x);
     }
-    // O projection + residual; produces the FFN norm input
     {
       GemvParams g = base_gemv(st, L.o, st->o, P.ldq, batch);
       g.h = st->h;
@@ -335,11 +320,8 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
       g.xn = st->xn;
       g.g_next = L.g_ffn;
       g.sumsq_out = st->sumsq;
-      pre(KFL_KERNEL_OPROJ);
-      CK(launch_gemv(g, EPI_RESID, gemv_grid(st, L.o), s, pdl));
-      post();
+      gemv(EPI_RESID, g);
     }
-    // gate/up + SwiGLU
     {
       GemvParams g = base_gemv(st, L.gu, st->xn, P.ldh, batch);
       g.sumsq = st->sumsq;
@@ -348,11 +330,8 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
       g.eps = c.rms_eps;
       g.out = st->a;
       g.ldo = P.lda;
-      pre(KFL_KERNEL_GATEUP);
-      CK(launch_gemv(g, EPI_SWIGLU, gemv_grid(st, L.gu), s, pdl));
-      post();
+      gemv(EPI_SWIGLU, g);
     }
-    // down + residual; produces the next block's (or the final) norm input
     {
       GemvParams g = base_gemv(st, L.down, st->a, P.lda, batch);
       g.h = st->h;
@@ -361,9 +340,7 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
       g.g_next = (l + 1 < P.nl) ? st->layers[l + 1].g_attn : ((st->flags & KFL_LOGITS_OUT) ? st->g_final : nullptr);
       g.sumsq_out = st->sumsq;
       g.capture = st->capture ? st->capture + (size_t)l * c.max_batch * P.d : nullptr;
-      pre(KFL_KERNEL_DOWN);
-      CK(launch_gemv(g, EPI_RESID, gemv_grid(st, L.down), s, pdl));
-      post();
+      gemv(EPI_RESID, g);
     }
   }
   if (st->flags & KFL_LOGITS_OUT) {
@@ -376,24 +353,91 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
     g.cand_idx = st->cand_idx;
     g.argmax_ticket = st->am_ticket;
     g.next_ids = st->next_int;
-    pre(KFL_KERNEL_LMHEAD);
-    CK(launch_gemv(g, EPI_ARGMAX, gemv_grid(st, st->lm), s, pdl));
-    post();
+    gemv(EPI_ARGMAX, g);
   }
+  return ph;
+}
+
+// Kernel kind of phase i of a step (phases come in blocks of five, then lm_head).
+int phase_kind_code(const Phase &ph, size_t i) {
+  if (ph.kind == PH_ATTN) return KFL_KERNEL_ATTN;
+  switch (ph.epi) {
+    case EPI_QKV: return KFL_KERNEL_QKV;
+    case EPI_SWIGLU: return KFL_KERNEL_GATEUP;
+    case EPI_ARGMAX: return KFL_KERNEL_LMHEAD;
+    default: return (i % 5 == 2) ? KFL_KERNEL_OPROJ : KFL_KERNEL_DOWN;
+  }
+}
+
+// Per-kernel mode: one launch per phase on stream s (chained with PDL when pdl is set).  With
+// `kinds` (profiling, no PDL) the k-th launch is bracketed by events ev[2(ev_base+k)] and
+// ev[2(ev_base+k)+1] and its kind appended to *kinds.
+int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector<int> *kinds, int ev_base) {
+  const std::vector<Phase> phases = build_phases(st, batch, attn_chunk_for(st, batch));
+  int k = ev_base;
+  for (size_t i = 0; i < phases.size(); ++i) {
+    const Phase &ph = phases[i];
+    if (kinds) {
+      CK(cudaEventRecord(st->ev[2 * k], s));
+      kinds->push_back(phase_kind_code(ph, i));
+    }
+    if (ph.kind == PH_GEMV) {
+      const long long T = (long long)ph.g.n_rb * ph.g.n_kt;
+      const int grid = (int)(T < st->P.gemv_grid_max ? T : st->P.gemv_grid_max);
+      CK(launch_gemv(ph.g, ph.epi, grid, s, pdl));
+    } else {
+      CK(launch_attention(ph.a, st->P.hd, s, pdl));
+    }
+    if (kinds) CK(cudaEventRecord(st->ev[2 * k + 1], s));
+    ++k;
+  }
+  return KFL_OK;
+}
+
+// Persistent mode: the whole step as one cooperative launch of the stage kernel.
+int enqueue_persistent(kfl_stage *st, int batch, cudaStream_t s) {
+  if (!st->phases_dev[batch]) {
+    const std::vector<Phase> phases = build_phases(st, batch, st->persist_chunk[batch]);
+    void *d = nullptr;
+    if (cudaMalloc(&d, phases.size() * sizeof(Phase)) != cudaSuccess) {
+      cudaGetLastError();
+      return KFL_ERR_OOM;
+    }
+    st->phases_dev[batch] = static_cast<Phase *>(d);
+    st->n_phases = (int)phases.size();
+    CK(cudaMemcpy(d, phases.data(), phases.size() * sizeof(Phase), cudaMemcpyHostToDevice));
+  }
+  StageKernelParams kp = {};
+  kp.phases = st->phases_dev[batch];
+  kp.n_phases = st->n_phases;
+  kp.stages = st->mk_stages;
+  kp.head_dim = st->P.hd;
+  kp.attn_bytes = stage_kernel_attn_bytes(st->P.hd);
+  kp.bar = st->bar;
+  kp.abort_flag = reinterpret_cast<int *>(st->bar + 1);
+  kp.err = st->err;
+  CK(launch_stage_kernel(kp, batch, st->cfg.weight_fmt, st->P.n_sm, st->mk_smem, s));
   return KFL_OK;
 }
 
 int ensure_graph(kfl_stage *st, int batch) {
   if (st->graph[batch]) return KFL_OK;
   if (!st->cap_stream) CK(cudaStreamCreateWithFlags(&st->cap_stream, cudaStreamNonBlocking));
+  if (st->persistent && !st->phases_dev[batch]) {
+    // the phase table is uploaded outside the capture
+    int rc = enqueue_persistent(st, batch, nullptr);
+    CK(cudaDeviceSynchronize());
+    if (rc != KFL_OK) return rc;
+  }
   cudaGraph_t g = nullptr;
   CK(cudaStreamBeginCapture(st->cap_stream, cudaStreamCaptureModeThreadLocal));
-  int rc = enqueue_body(st, batch, st->cap_stream, true, nullptr, 0);
+  int rc = st->persistent ? enqueue_persistent(st, batch, st->cap_stream)
+                          : enqueue_body(st, batch, st->cap_stream, true, nullptr, 0);
   cudaError_t e = cudaStreamEndCapture(st->cap_stream, &g);
   if (rc != KFL_OK || e != cudaSuccess) {
     if (g) cudaGraphDestroy(g);
     cudaGetLastError();
-    return KFL_ERR_CUDA;
+    return rc != KFL_OK ? rc : KFL_ERR_CUDA;
   }
   e = cudaGraphInstantiate(&st->graph[batch], g, 0);
   cudaGraphDestroy(g);
@@ -415,8 +459,9 @@ int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const in
              float *hidden_out, int32_t *next_ids, cudaStream_t s) {
   const Plan &P = st->P;
   const bool embed = (st->flags & KFL_EMBED_IN) != 0;
+  const bool body = P.nl > 0 || (st->flags & KFL_LOGITS_OUT);
   if (st->profile) {
-    const int n_k = kfl_stage_launches_per_step(st, batch);
+    const int n_k = 2 + (int)build_phases(st, batch, attn_chunk_for(st, batch)).size();
     while ((int)st->ev.size() < 2 * n_k) {
       cudaEvent_t e;
       CK(cudaEventCreate(&e));
@@ -425,7 +470,7 @@ int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const in
     std::vector<int> kinds;
     CK(cudaEventRecord(st->ev[0], s));
     CK(launch_stage_input(ids, hidden_in, positions, batch, embed ? st->embed : nullptr, P.V, P.d, P.ldh,
-                          input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, s));
+                          input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, st->bar, s));
     CK(cudaEventRecord(st->ev[1], s));
     kinds.push_back(KFL_KERNEL_INPUT);
     int rc = enqueue_body(st, batch, s, false, &kinds, 1);
@@ -445,8 +490,8 @@ int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const in
     return KFL_OK;
   }
   CK(launch_stage_input(ids, hidden_in, positions, batch, embed ? st->embed : nullptr, P.V, P.d, P.ldh,
-                        input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, s));
-  if (P.nl > 0 || (st->flags & KFL_LOGITS_OUT)) {
+                        input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, st->bar, s));
+  if (body) {
     int rc = ensure_graph(st, batch);
     if (rc != KFL_OK) return rc;
     CK(cudaGraphLaunch(st->graph[batch], s));
@@ -573,6 +618,8 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
   CK(cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev));
   CK(prepare_gemv());
   CK(prepare_attention());
+  int smem_optin = 0;
+  CK(cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev));
   kfl_stage *st = new kfl_stage();
   st->cfg = *cfg;
   st->l0 = l0;
@@ -630,12 +677,13 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
   st->am_ticket = st->tickets + P.n_rb_max;
   AL(st->cand_val, (size_t)P.n_rb_max * MAXB * 4);
   AL(st->cand_idx, (size_t)P.n_rb_max * MAXB * 4);
-  AL(st->attn_partial, (size_t)MAXB * P.hkv * P.attn_nchunks_max * 8 * (P.hd + 2) * 4);
+  AL(st->attn_partial, (size_t)MAXB * P.hkv * P.attn_nchunks_max * 8 * (P.hd + 4) * 4);
   AL(st->attn_tickets, (size_t)MAXB * P.hkv * 4);
   AL(st->err, 16);
   AL(st->io_pos, MAXB * 4);
   AL(st->io_ids, MAXB * 4);
   AL(st->io_hin, (size_t)MAXB * P.d * 4);
+  AL(st->bar, 16);
 #undef AL
   // zero everything that is read before it is written or whose padding must stay zero
   if (P.nl > 0) {
@@ -647,7 +695,8 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
       cudaMemset(st->a, 0, (size_t)MAXB * P.lda * 4) || cudaMemset(st->sumsq, 0, (size_t)P.n_parts * MAXB * 4) ||
       cudaMemset(st->pos, 0, MAXB * 4) || cudaMemset(st->next_int, 0, MAXB * 4) ||
       cudaMemset(st->tickets, 0, (size_t)(P.n_rb_max + 1) * 4) ||
-      cudaMemset(st->attn_tickets, 0, (size_t)MAXB * P.hkv * 4) || cudaMemset(st->err, 0, 16))
+      cudaMemset(st->attn_tickets, 0, (size_t)MAXB * P.hkv * 4) || cudaMemset(st->err, 0, 16) ||
+      cudaMemset(st->bar, 0, 16))
     return fail(KFL_ERR_CUDA);
   // RoPE table: angle pos * theta^(-2i/hd) in fp64, stored as fp32 cos / sin
   {
@@ -662,6 +711,30 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
     if (cudaMemcpy(st->rope_cos, cs.data(), cs.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
         cudaMemcpy(st->rope_sin, sn.data(), sn.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
       return fail(KFL_ERR_CUDA);
+  }
+  // persistent stage kernel: the deepest ring that fits next to the attention buffers
+  st->persistent = env_int("KFL_PERSISTENT", 1) != 0;
+  {
+    int stages = env_int("KFL_STAGE_KERNEL_STAGES", MAX_STAGES);
+    if (stages > MAX_STAGES) stages = MAX_STAGES;
+    const size_t static_smem = 4096;  // the kernel's own __shared__ variables
+    while (stages > 2 && stage_kernel_smem(stages, P.hd) + static_smem > (size_t)smem_optin) --stages;
+    st->mk_stages = stages;
+    st->mk_smem = stage_kernel_smem(stages, P.hd);
+    if (prepare_stage_kernel(st->mk_smem) != cudaSuccess) {
+      cudaGetLastError();
+      st->persistent = false;
+    }
+    for (int b = 1; b <= cfg->max_batch; ++b) {
+      // about one attention unit per SM over the reserved context
+      const long long work = (long long)cfg->max_ctx * b * P.hkv;
+      long long want = (work + P.n_sm - 1) / P.n_sm;
+      if (want < 64) want = 64;
+      int chunk = round_up((int)want, 64);
+      while ((long long)((cfg->max_ctx + chunk - 1) / chunk) * (P.hq / P.hkv) > 2048) chunk += 64;
+      if (chunk > round_up(cfg->max_ctx, 64)) chunk = round_up(cfg->max_ctx, 64);
+      st->persist_chunk[b] = chunk;
+    }
   }
   *out = st;
   return KFL_OK;
@@ -925,7 +998,9 @@ extern "C" int kfl_stage_profile_read(kfl_stage *st, double *ms, int64_t *launch
 extern "C" int kfl_stage_launches_per_step(kfl_stage *st, int batch) {
   if (!valid(st)) return KFL_ERR_STATE;
   (void)batch;
-  return 2 + 5 * st->P.nl + ((st->flags & KFL_LOGITS_OUT) ? 1 : 0);
+  const int body = 5 * st->P.nl + ((st->flags & KFL_LOGITS_OUT) ? 1 : 0);
+  if (st->profile || !st->persistent) return 2 + body;
+  return 2 + (body > 0 ? 1 : 0);
 }
 
 extern "C" void kfl_stage_destroy(kfl_stage *st) {

@@ -114,15 +114,29 @@ def test_deterministic_replay_and_profile_mode():
     c1 = p.cap.cpu().numpy().copy()
     h2, n2 = p.gpu_step(pos, ids=ids)  # rewrites the same slots with the same values
     assert np.array_equal(h1, h2) and np.array_equal(n1, n2)
+    # per-kernel mode (one launch per phase, events around each) gives the same bits as the
+    # persistent stage kernel
+    assert K.kfl_stage_launches_per_step(p.st, 3) == 3
     K.kfl_stage_profile(p.st, True)
+    assert K.kfl_stage_launches_per_step(p.st, 3) == 2 + 5 * 3 + 1
     h3, n3 = p.gpu_step(pos, ids=ids)
     prof = K.kfl_stage_profile_read(p.st)
     K.kfl_stage_profile(p.st, False)
     assert np.array_equal(h1, h3) and np.array_equal(n1, n3)
     assert np.array_equal(c1, p.cap.cpu().numpy())
-    assert prof["qkv"][1] == 3 and prof["attn"][1] == 3 and prof["lmhead"][1] == 1
+    assert prof["qkv"][1] == 3 and prof["attn"][1] == 3 and prof["oproj"][1] == 3 and prof["down"][1] == 3
+    assert prof["lmhead"][1] == 1 and prof["gateup"][1] == 3
     assert all(ms > 0 for ms, n in prof.values() if n > 0)
-    assert K.kfl_stage_launches_per_step(p.st, 3) == 2 + 5 * 3 + 1
+    p.close()
+
+
+@pytest.mark.parametrize("fmt_model", [RAGGED, RAGGED_INT4], ids=["bf16", "int4"])
+def test_per_kernel_mode_parity(fmt_model, monkeypatch):
+    """The stage run as one launch per phase (CUDA graph with programmatic dependent launch)."""
+    monkeypatch.setenv("KFL_PERSISTENT", "0")
+    p = Pair(fmt_model, 0, 2, K.KFL_IS_HEAD, 3, (4, 77, 150), 192, seed=23)
+    assert K.kfl_stage_launches_per_step(p.st, 3) == 2 + 5 * 2 + 1
+    _greedy(p, 2, np.array([1, 500, 999], dtype=np.int32))
     p.close()
 
 
