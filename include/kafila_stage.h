@@ -159,6 +159,16 @@ int kfl_kv_read(kfl_stage *st, int local, int user, uint16_t *k, uint16_t *v, in
  * Changing it rebuilds the stage's CUDA graphs on the next decode. */
 int kfl_stage_debug_capture(kfl_stage *st, float *per_layer_hidden);
 
+/* Phase trace of the persistent stage kernel (tuning aid).  When buf (device uint64
+ * [n_phases][grid][slots], shape from kfl_stage_trace_shape) is not NULL, every later decode
+ * writes %globaltimer stamps (ns) per phase and CTA: 0 consumers reach the phase, 1 they pass
+ * its grid barrier, 2 they finish it, 3 the activation producer passes the barrier, 4 it issues
+ * the phase's last chunk, 5/6 the weight producer issues the phase's first/last tile (slots of
+ * events that do not happen are left as they were).  NULL turns it off.  Changing it rebuilds
+ * the stage's CUDA graphs on the next decode. */
+int kfl_stage_trace(kfl_stage *st, uint64_t *buf);
+int kfl_stage_trace_shape(kfl_stage *st, int batch, int *n_phases, int *grid, int *slots);
+
 /* Sticky device-side error word of the stage: waits for the device, then returns KFL_OK,
  * KFL_ERR_RANGE (a bad position or token id was seen) or KFL_ERR_TIMEOUT (a bounded wait
  * gave up), and clears it. */
@@ -186,6 +196,10 @@ int kfl_stage_launches_per_step(kfl_stage *st, int batch);
 
 void kfl_stage_destroy(kfl_stage *st);
 const char *kfl_strerror(int code);
+
+/* Text of the last CUDA runtime error behind a KFL_ERR_CUDA on this thread (the failing call
+ * and its error string), or "" if none.  The pointer stays valid until the next failing call. */
+const char *kfl_last_error_detail(void);
 
 #ifdef __cplusplus
 }

@@ -14,14 +14,14 @@ __global__ void __launch_bounds__(ATT_THREADS) attn_kernel(const __grid_constant
   pdl_wait();
   const int nc = attn_chunks(p, b);
   if (c >= nc) return;
-  attn_unit<HD>(p, b, kvh, c, nc, sm, &s_last, threadIdx.x);
+  attn_unit<HD, 2>(p, b, kvh, c, nc, sm, &s_last, threadIdx.x, 0);
 }
 
 cudaError_t prepare_attention() {
   cudaError_t e = cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       AttnLayout<128>::BYTES);
+                                       AttnLayout<128, 2>::BYTES);
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, AttnLayout<64>::BYTES);
+  return cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, AttnLayout<64, 2>::BYTES);
 }
 
 template <int HD>
@@ -29,7 +29,7 @@ static cudaError_t launch_hd(const AttnParams &p, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.n_chunks, p.n_kv_heads, p.batch);
   cfg.blockDim = dim3(ATT_THREADS);
-  cfg.dynamicSmemBytes = AttnLayout<HD>::BYTES;
+  cfg.dynamicSmemBytes = AttnLayout<HD, 2>::BYTES;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -42,6 +42,7 @@ static cudaError_t launch_hd(const AttnParams &p, cudaStream_t s, bool pdl) {
 cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s, bool pdl) {
   if (p.n_heads % p.n_kv_heads != 0 || p.n_heads / p.n_kv_heads > ATT_MAXG) return cudaErrorInvalidValue;
   if (p.n_chunks * (p.n_heads / p.n_kv_heads) > ATT_MERGE_MAX) return cudaErrorInvalidValue;
+  static_assert(AttnLayout<64, 1>::MERGE_MAX >= ATT_MERGE_MAX, "merge scratch");
   if (head_dim == 128) return launch_hd<128>(p, s, pdl);
   if (head_dim == 64) return launch_hd<64>(p, s, pdl);
   return cudaErrorInvalidValue;

@@ -23,7 +23,7 @@ namespace kfl {
 constexpr int ATT_THREADS = 256;
 constexpr int ATT_SUB = 64;          // positions per shared-memory sub-tile
 constexpr int ATT_MAXG = 8;          // query heads per KV head
-constexpr int ATT_MERGE_MAX = 2048;  // chunks x heads merged in shared memory (fits the K buffers)
+constexpr int ATT_MERGE_MAX = 1024;  // chunks x heads merged in shared memory (fits the K buffers)
 constexpr int ATT_BAR = 2;           // named barrier of the attention threads
 
 __device__ __forceinline__ void att_sync() { named_bar_sync(ATT_BAR, ATT_THREADS); }
@@ -37,7 +37,7 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-template <int HD>
+template <int HD, int NBUF>
 struct AttnLayout {
   // K row: four quarters of hd/4 dims, each padded by 16 bytes, so the four lanes reading the
   // quarters of one position and the next position's lanes hit distinct banks
@@ -46,26 +46,71 @@ struct AttnLayout {
   static constexpr int VROW = HD * 2;
   static constexpr int QQ = HD / 4 + 4;     // floats per padded quarter of a q row
   static constexpr int K_OFF = 0;
-  static constexpr int V_OFF = K_OFF + 2 * ATT_SUB * KROW;
-  static constexpr int Q_OFF = V_OFF + 2 * ATT_SUB * VROW;
+  static constexpr int V_OFF = K_OFF + NBUF * ATT_SUB * KROW;
+  static constexpr int Q_OFF = V_OFF + NBUF * ATT_SUB * VROW;
   static constexpr int S_OFF = Q_OFF + ATT_MAXG * 4 * QQ * 4;
   static constexpr int M_OFF = S_OFF + ATT_MAXG * ATT_SUB * 4;
   static constexpr int BYTES = M_OFF + 4 * ATT_MAXG * 4;
-  static_assert(2 * ATT_MERGE_MAX * 4 <= 2 * ATT_SUB * KROW, "merge scratch must fit the K buffers");
+  static constexpr int MERGE_MAX = (NBUF * ATT_SUB * KROW) / 8;  // chunks x heads in the K buffers
+  static_assert(MERGE_MAX >= 1024, "merge scratch too small");
 };
 
 __host__ __device__ constexpr int attn_pstride(int hd) { return hd + 4; }
 
-// Number of chunks of user b (1 for an invalid position: that unit writes zeros).
+// Number of chunks of user b (1 for an invalid position: that unit writes zeros).  The
+// positions are never written while a step runs, so they need no L2-coherent load.
 __device__ __forceinline__ int attn_chunks(const AttnParams &p, int b) {
-  const int P = __ldcg(p.positions + b);
+  const int P = p.positions[b];
   if (P < 0 || P >= p.max_ctx) return 1;
   return (P + 1 + p.chunk - 1) / p.chunk;
 }
 
-template <int HD>
-__device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, uint8_t *sm, int *s_last, int tid) {
-  using L = AttnLayout<HD>;
+// Rows [p0, p0 + cnt) of user b / KV head kvh into K/V buffer `buf`, except `skip` (the new
+// token's row, written in this step) when skip >= 0; one cp.async group.
+template <int HD, int NBUF>
+__device__ __forceinline__ void attn_load_rows(const AttnParams &p, int b, int kvh, int p0, int cnt, int buf,
+                                               int only, int skip, uint8_t *sm, int tid) {
+  using L = AttnLayout<HD, NBUF>;
+  const size_t head_base = ((size_t)b * p.n_kv_heads + kvh) * p.max_ctx;
+  const uint16_t *kg = p.kcache + head_base * HD;
+  const uint16_t *vg = p.vcache + head_base * HD;
+  uint8_t *sk = sm + L::K_OFF + buf * ATT_SUB * L::KROW;
+  uint8_t *sv = sm + L::V_OFF + buf * ATT_SUB * L::VROW;
+  constexpr int CH = HD / 8;   // 16-byte chunks per row
+  constexpr int CQ = HD / 32;  // chunks per quarter
+  for (int e = tid; e < cnt * CH; e += ATT_THREADS) {
+    const int r = e / CH, ch = e % CH;
+    const int row = p0 + r;
+    if ((only >= 0 && row != only) || row == skip) continue;
+    cp_async16(sk + r * L::KROW + (ch / CQ) * L::QB + (ch % CQ) * 16, kg + (size_t)row * HD + ch * 8);
+    cp_async16(sv + r * L::VROW + ch * 16, vg + (size_t)row * HD + ch * 8);
+  }
+  cp_async_commit();
+}
+
+// Issue the loads of a unit's first sub-tile that do not depend on the current step: every row
+// but the new token's (which the QKV phase writes).  The unit then runs with prefetched = 1.
+template <int HD, int NBUF>
+__device__ __forceinline__ void attn_prefetch(const AttnParams &p, int b, int kvh, int c, uint8_t *sm, int tid) {
+  const int P = p.positions[b];
+  if (P < 0 || P >= p.max_ctx) return;
+  const int start = c * p.chunk;
+  const int end = min(P + 1, start + p.chunk);
+  attn_load_rows<HD, NBUF>(p, b, kvh, start, min(ATT_SUB, end - start), 0, -1, P, sm, tid);
+}
+
+// The (user, KV head) output is written: publish it (persistent kernel; the bar.sync orders every
+// thread's stores before the release).
+__device__ __forceinline__ void attn_publish(const AttnParams &p, int kvh, int tid) {
+  if (!p.out_ready) return;
+  att_sync();
+  if (tid == 0) red_add_release(p.out_ready + kvh, 1u);
+}
+
+template <int HD, int NBUF>
+__device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, uint8_t *sm, int *s_last, int tid,
+                          int prefetched) {
+  using L = AttnLayout<HD, NBUF>;
   uint8_t *sk = sm + L::K_OFF;
   uint8_t *sv = sm + L::V_OFF;
   float *sq = reinterpret_cast<float *>(sm + L::Q_OFF);
@@ -81,18 +126,16 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
   const bool owns = og < G;
   float *o = p.o + (size_t)b * p.ldo + (size_t)kvh * G * HD;
 
-  const int P = __ldcg(p.positions + b);
+  const int P = p.positions[b];
   if (P < 0 || P >= p.max_ctx) {
     // the stage input flagged the position; leave a defined (zero) output
     if (owns) *reinterpret_cast<float4 *>(o + og * HD + od) = make_float4(0.f, 0.f, 0.f, 0.f);
+    attn_publish(p, kvh, tid);
     return;
   }
   const int ntok = P + 1;
   const int start = c * p.chunk;
   const int end = min(ntok, start + p.chunk);
-  const size_t head_base = ((size_t)b * p.n_kv_heads + kvh) * p.max_ctx;
-  const uint16_t *kg = p.kcache + head_base * HD;
-  const uint16_t *vg = p.vcache + head_base * HD;
 
   for (int e = tid; e < G * HD; e += ATT_THREADS) {
     const int g = e / HD, d = e % HD;
@@ -106,27 +149,22 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
 
   auto load_sub = [&](int sub, int buf) {
     const int p0 = start + sub * ATT_SUB;
-    const int cnt = min(ATT_SUB, end - p0);
-    constexpr int CH = HD / 8;   // 16-byte chunks per row
-    constexpr int CQ = HD / 32;  // chunks per quarter
-    for (int e = tid; e < cnt * CH; e += ATT_THREADS) {
-      const int r = e / CH, ch = e % CH;
-      cp_async16(sk + buf * ATT_SUB * L::KROW + r * L::KROW + (ch / CQ) * L::QB + (ch % CQ) * 16,
-                 kg + (size_t)(p0 + r) * HD + ch * 8);
-      cp_async16(sv + buf * ATT_SUB * L::VROW + r * L::VROW + ch * 16, vg + (size_t)(p0 + r) * HD + ch * 8);
-    }
-    cp_async_commit();
+    attn_load_rows<HD, NBUF>(p, b, kvh, p0, min(ATT_SUB, end - p0), buf, -1, -1, sm, tid);
   };
 
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
   const int nsub = (end - start + ATT_SUB - 1) / ATT_SUB;
-  load_sub(0, 0);
+  if (prefetched)  // only the new token's row of the first sub-tile is still to load
+    attn_load_rows<HD, NBUF>(p, b, kvh, start, min(ATT_SUB, end - start), 0, P, -1, sm, tid);
+  else
+    load_sub(0, 0);
   for (int it = 0; it < nsub; ++it) {
-    const int buf = it & 1;
-    if (it + 1 < nsub) {
+    const int buf = NBUF == 2 ? (it & 1) : 0;
+    if (NBUF == 2 && it + 1 < nsub) {
       load_sub(it + 1, buf ^ 1);
       cp_async_wait<1>();
     } else {
+      if (NBUF == 1 && it > 0) load_sub(it, 0);
       cp_async_wait<0>();
     }
     att_sync();
@@ -230,6 +268,7 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
       const float il = 1.0f / s_l[og];
       *reinterpret_cast<float4 *>(o + og * HD + od) = make_float4(acc[0] * il, acc[1] * il, acc[2] * il, acc[3] * il);
     }
+    attn_publish(p, kvh, tid);
     return;
   }
   constexpr int PS = attn_pstride(HD);
@@ -240,22 +279,20 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
     part[tid * PS + HD] = s_m[tid];
     part[tid * PS + HD + 1] = s_l[tid];
   }
-  __threadfence();
   att_sync();
   if (tid == 0) {
     int *tk = p.tickets + b * p.n_kv_heads + kvh;
-    const int prev = atomicAdd(tk, 1);
-    *s_last = (prev == nc - 1);
+    const unsigned prev = atom_add_acq_rel(reinterpret_cast<unsigned *>(tk), 1u);
+    *s_last = (prev == (unsigned)(nc - 1));
     if (*s_last) atomicExch(tk, 0);
   }
   att_sync();
   if (!*s_last) return;
-  __threadfence();
   // merge: per-chunk weights 2^(m_c - M) / L staged in shared memory (the K buffers), then each
   // thread sums its 4 outputs over the chunks
   const float *base = p.partial + unit_base * (ATT_MAXG * PS);
   float *wm = reinterpret_cast<float *>(sk);
-  float *wl = wm + ATT_MERGE_MAX;
+  float *wl = wm + L::MERGE_MAX;
   for (int e = tid; e < nc * G; e += ATT_THREADS) {
     const int cc = e / G, g = e % G;
     const float *pc = base + (size_t)cc * ATT_MAXG * PS + g * PS;
@@ -292,6 +329,7 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
     }
     *reinterpret_cast<float4 *>(o + og * HD + od) = O;
   }
+  attn_publish(p, kvh, tid);
 }
 
 }  // namespace kfl

@@ -18,17 +18,23 @@ constexpr int RB = 64;            // rows per row block (and per tile)
 constexpr int KT = 128;           // K per bf16 tile
 constexpr int TILE_BYTES = RB * KT * 2;
 constexpr int MAXB = 4;           // users per step
-constexpr int XCHUNK_BYTES = KT * 4;          // one user's fp32 activation chunk of a tile
-constexpr int STAGE_BYTES = TILE_BYTES + MAXB * XCHUNK_BYTES;
 constexpr int CONSUMER_WARPS = 8;
 constexpr int GEMV_THREADS = (CONSUMER_WARPS + 1) * 32;
-constexpr int MAX_STAGES = 10;
+constexpr int MAX_STAGES = 12;
 
 // int4 group-64 tiles: [N/RB][K/KT4][RB][KT4/8] uint32 codes then [RB][KT4/64] bf16 scales
 constexpr int KT4 = 256;
 constexpr int TILE4_CODE_BYTES = RB * KT4 / 2;     // 8 KiB
 constexpr int TILE4_SCALE_BYTES = RB * (KT4 / 64) * 2;  // 512 B
 constexpr int TILE4_BYTES = TILE4_CODE_BYTES + TILE4_SCALE_BYTES;
+
+// A ring stage holds one weight tile and the B users' fp32 activation chunks of its K range.
+__host__ __device__ constexpr int tile_k(int fmt) { return fmt == 0 ? KT : KT4; }
+__host__ __device__ constexpr int tile_bytes(int fmt) { return fmt == 0 ? TILE_BYTES : TILE4_BYTES; }
+__host__ __device__ constexpr int stage_bytes(int batch, int fmt) {
+  return (tile_bytes(fmt) + batch * tile_k(fmt) * 4 + 127) / 128 * 128;
+}
+constexpr int STAGE_BYTES_MAX = stage_bytes(MAXB, 0);
 
 // ---- device error word bits ---------------------------------------------------------------
 constexpr unsigned ERR_POSITION = 1u;
@@ -77,8 +83,9 @@ struct GemvParams {
   // EPI_QKV
   float *q;
   uint16_t *kcache, *vcache;  // this layer's [max_batch][Hkv][max_ctx][hd]
-  const int *positions;
-  const float *rope_cos, *rope_sin;  // [max_ctx][hd/2]
+  const int *positions;       // [batch]; never written while a step runs
+  const float *rope_cos, *rope_sin;  // [max_ctx][hd/2], or [batch][hd/2] when rope_per_user
+  int rope_per_user;
   int n_q_rows, n_kv_rows, head_dim, max_ctx, n_kv_heads;
   // EPI_ARGMAX
   float *cand_val;
@@ -89,6 +96,20 @@ struct GemvParams {
   float *partial;  // [grid][2][RB][MAXB]
   int *tickets;    // [n_rb], zero between launches
   unsigned *err;
+  // dataflow (persistent stage kernel only; all NULL / 0 otherwise)
+  int in_kind;                // 0 inputs complete at launch, 1 per-chunk counters, 2 per-KV-head counters
+  const unsigned *in_ready;   // counters of the producing phase
+  int in_len;                 // kind 1: length of the input vector (elements)
+  int in_unit;                // kind 1: input elements one producing row block completes
+  int in_group;               // kind 2: query heads per KV head
+  int in_head_dim;            // kind 2
+  int in_need;                // kind 2: completions per KV head (the batch)
+  const unsigned *norm_done;  // row blocks of h completed by the phase producing h (NULL: ready)
+  int norm_need;
+  unsigned *out_ready;        // per consumer chunk (RESID, SWIGLU) or per KV head (QKV)
+  int out_unit;               // output elements per row block (RESID 64, SWIGLU 32)
+  int out_kt;                 // the consumer's tile K
+  unsigned *out_done;         // row blocks completed
 };
 
 struct AttnParams {
@@ -103,6 +124,10 @@ struct AttnParams {
   int batch, n_heads, n_kv_heads, max_ctx, chunk, n_chunks;
   float scale_log2;          // log2(e) / sqrt(hd)
   unsigned *err;
+  // dataflow (persistent stage kernel only)
+  const unsigned *in_ready;  // per KV head: Q/K/V row blocks completed
+  int in_need;
+  unsigned *out_ready;       // per KV head: (user, KV head) outputs completed
 };
 
 // One phase of the persistent stage kernel: a GEMV (with its epilogue) or an attention pass.
@@ -121,10 +146,30 @@ struct StageKernelParams {
   int stages;      // ring stages
   int head_dim;
   int attn_bytes;  // shared memory of the attention unit
-  unsigned *bar;   // grid-barrier counter, zeroed by the stage input kernel
+  unsigned *bar;   // [1] is the abort flag, zeroed by the stage input kernel
   int *abort_flag; // set when any wait gives up; zeroed by the stage input kernel
   unsigned *err;
+  unsigned long long *trace;  // [n_phases][grid][TRACE_SLOTS] globaltimer stamps, or NULL
+  const int *positions;       // [batch] (static during the step)
+  const float *rope_cos, *rope_sin;  // [max_ctx][hd/2]
+  int max_ctx;
 };
+
+// phase trace slots (ns, %globaltimer)
+constexpr int TRACE_SLOTS = 8;
+constexpr int TR_CONS_ENTER = 0;   // consumers reach the phase
+constexpr int TR_CONS_GO = 1;      // consumers start its work
+constexpr int TR_CONS_DONE = 2;    // consumers finished the phase
+constexpr int TR_X_GO = 3;         // activation producer issued the phase's first chunk
+constexpr int TR_X_LAST = 4;       // activation producer issued the phase's last chunk
+constexpr int TR_W_FIRST = 5;      // weight producer issued the phase's first tile
+constexpr int TR_W_LAST = 6;       // weight producer issued the phase's last tile
+
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
 
 // ---- PTX helpers --------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t smem_addr(const void *p) {
@@ -158,6 +203,29 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "r"(bar), "r"(parity)
       : "memory");
   return ok != 0;
+}
+
+// Non-blocking test of an mbarrier phase.
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ int ld_acquire_cta_shared(const volatile int *p) {
+  int v;
+  asm volatile("ld.acquire.cta.shared.b32 %0, [%1];" : "=r"(v) : "r"(smem_addr((const void *)p)) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_release_cta_shared(volatile int *p, int v) {
+  asm volatile("st.release.cta.shared.b32 [%0], %1;" ::"r"(smem_addr((const void *)p)), "r"(v) : "memory");
 }
 
 // Bounded wait on an mbarrier phase; false after WAIT_LIMIT polls.
@@ -216,6 +284,22 @@ __device__ __forceinline__ uint16_t f32_to_bf16_rne(float f) {
 
 __device__ __forceinline__ float ld_cg(const float *p) { return __ldcg(p); }
 
+// gpu-scope atomics with release / acquire-release semantics: the writes a CTA made before a
+// bar.sync become visible with the atomic, without a separate membar
+__device__ __forceinline__ unsigned atom_add_acq_rel(unsigned *p, unsigned v) {
+  unsigned old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+__device__ __forceinline__ void red_add_release(unsigned *p, unsigned v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned *p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
 }  // namespace kfl
 
 // Kernel launchers (defined in the .cu files; used by the runtime).
@@ -228,7 +312,7 @@ cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int
                                int batch, const uint16_t *embed, int vocab, int d, int ldh,
                                const float *g_next, float *h, float *xn, float *sumsq,
                                int *positions, int max_ctx, unsigned *err, unsigned *bar, cudaStream_t s);
-size_t stage_kernel_smem(int stages, int head_dim);
+size_t stage_kernel_smem(int stages, int head_dim, int batch, int fmt);
 int stage_kernel_attn_bytes(int head_dim);
 cudaError_t prepare_stage_kernel(size_t smem);
 cudaError_t launch_stage_kernel(const StageKernelParams &kp, int batch, int fmt, int grid, size_t smem,

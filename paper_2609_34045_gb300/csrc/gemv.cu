@@ -22,13 +22,16 @@
 
 namespace kfl {
 
+constexpr int GEMV_MAX_STAGES = 10;  // standalone kernel: two CTAs (this and the next) per SM
+
 // ---------------------------------------------------------------------------- the kernel
 // FMT 0: bf16 tiles [RB][KT].  FMT 1: int4 tiles, codes [RB][KT4/8] uint32 + scales [RB][KT4/64].
 template <int B, int EPI, int FMT>
 __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) gemv_kernel(const __grid_constant__ GemvParams p) {
   extern __shared__ __align__(1024) uint8_t smem[];
   const int S = p.stages;
-  uint64_t *full = reinterpret_cast<uint64_t *>(smem + (size_t)S * STAGE_BYTES);
+  constexpr int SB = stage_bytes(B, FMT);
+  uint64_t *full = reinterpret_cast<uint64_t *>(smem + (size_t)S * SB);
   uint64_t *empty = full + S;
   float *red = reinterpret_cast<float *>(empty + S);  // [RB][MAXB]
   float *scr = red + RB * MAXB;                       // 2 * CONSUMER_WARPS words
@@ -67,13 +70,13 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
       for (int i = 0; i < pre; ++i) {
         const uint32_t fb = smem_addr(&full[i]);
         mbar_arrive_expect_tx(fb, WBYTES + xbytes);
-        bulk_g2s(smem_addr(smem + (size_t)i * STAGE_BYTES), p.w + (size_t)(t0 + i) * WBYTES, WBYTES, fb, pol_w);
+        bulk_g2s(smem_addr(smem + (size_t)i * SB), p.w + (size_t)(t0 + i) * WBYTES, WBYTES, fb, pol_w);
         s_issued = i + 1;
       }
       pdl_wait();
       auto issue_x = [&](int kt, int s) {
         const uint32_t fb = smem_addr(&full[s]);
-        const uint32_t dst = smem_addr(smem + (size_t)s * STAGE_BYTES + WBYTES);
+        const uint32_t dst = smem_addr(smem + (size_t)s * SB + WBYTES);
 #pragma unroll
         for (int b = 0; b < B; ++b)
           bulk_g2s(dst + b * (KTILE * 4), p.x + (size_t)b * p.ldx + (size_t)kt * KTILE, KTILE * 4, fb, pol_x);
@@ -89,7 +92,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
         if (!consumer_wait(smem_addr(&empty[s]), eph, &s_abort, p.err)) break;
         const uint32_t fb = smem_addr(&full[s]);
         mbar_arrive_expect_tx(fb, WBYTES + xbytes);
-        bulk_g2s(smem_addr(smem + (size_t)s * STAGE_BYTES), p.w + (size_t)(t0 + i) * WBYTES, WBYTES, fb, pol_w);
+        bulk_g2s(smem_addr(smem + (size_t)s * SB), p.w + (size_t)(t0 + i) * WBYTES, WBYTES, fb, pol_w);
         issue_x(kt_x, s);
         s_issued = i + 1;
         if (++kt_x == p.n_kt) kt_x = 0;
@@ -108,8 +111,9 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
   consumer_sync();
   int s = 0;
   uint32_t phase = 0;
-  gemv_consume<B, EPI, FMT>(p, smem, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv, &s_last, &s_abort,
-                            tid);
+  int inv_ready = 1;
+  gemv_consume<B, EPI, FMT>(p, smem, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv, &inv_ready, &s_last,
+                            &s_abort, tid);
 
   if (s_abort && tid == 0) {
     // drain copies still in flight before the CTA's shared memory goes away (bounded)
@@ -120,14 +124,15 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
 }
 
 // ---------------------------------------------------------------------------- launch
-static size_t gemv_smem_bytes(int stages) {
-  return (size_t)stages * STAGE_BYTES + 2 * stages * sizeof(uint64_t) + (RB * MAXB + 2 * CONSUMER_WARPS) * sizeof(float);
+static size_t gemv_smem_bytes(int stages, int batch, int fmt) {
+  return (size_t)stages * stage_bytes(batch, fmt) + 2 * stages * sizeof(uint64_t) +
+         (RB * MAXB + 2 * CONSUMER_WARPS) * sizeof(float);
 }
 
 template <int B, int EPI, int FMT>
 static cudaError_t launch_one(const GemvParams &p, int grid, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
-  const size_t smem = gemv_smem_bytes(p.stages);
+  const size_t smem = gemv_smem_bytes(p.stages, B, FMT);
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(GEMV_THREADS);
   cfg.dynamicSmemBytes = smem;
@@ -166,7 +171,7 @@ static cudaError_t launch_f(const GemvParams &p, int epi, int grid, cudaStream_t
 template <int B, int EPI, int FMT>
 static cudaError_t prepare_one() {
   return cudaFuncSetAttribute(gemv_kernel<B, EPI, FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)gemv_smem_bytes(MAX_STAGES));
+                              (int)gemv_smem_bytes(GEMV_MAX_STAGES, B, FMT));
 }
 
 template <int EPI, int FMT>
@@ -196,7 +201,7 @@ cudaError_t prepare_gemv() {
 }
 
 cudaError_t launch_gemv(const GemvParams &p, int epi, int grid, cudaStream_t s, bool pdl) {
-  if (p.stages < 2 || p.stages > MAX_STAGES) return cudaErrorInvalidValue;
+  if (p.stages < 2 || p.stages > GEMV_MAX_STAGES) return cudaErrorInvalidValue;
   return p.fmt == 0 ? launch_f<0>(p, epi, grid, s, pdl) : launch_f<1>(p, epi, grid, s, pdl);
 }
 

@@ -99,7 +99,7 @@ __device__ __forceinline__ void epilogue(const GemvParams &p, int rb, const floa
   } else if constexpr (EPI == EPI_QKV) {
     if (tid < 32 * B) {
       const int b = tid >> 5, pr = tid & 31, r0 = rb * RB + 2 * pr;
-      int pos = __ldcg(p.positions + b);
+      int pos = p.positions[b];
       const bool ok = pos >= 0 && pos < p.max_ctx;
       if (!ok) pos = 0;
       if (r0 < p.n_rows) {
@@ -110,8 +110,9 @@ __device__ __forceinline__ void epilogue(const GemvParams &p, int rb, const floa
           const bool is_q = r0 < p.n_q_rows;
           const int rr = is_q ? r0 : r0 - p.n_q_rows;
           const int head = rr / hd, i = (rr % hd) >> 1;
-          const float cs = p.rope_cos[(size_t)pos * half + i];
-          const float sn = p.rope_sin[(size_t)pos * half + i];
+          const size_t ri = (size_t)(p.rope_per_user ? b : pos) * half + i;
+          const float cs = p.rope_cos[ri];
+          const float sn = p.rope_sin[ri];
           const float a = v1 * cs - v2 * sn;
           const float c = v2 * cs + v1 * sn;
           if (is_q) {
@@ -160,17 +161,15 @@ __device__ __forceinline__ void epilogue(const GemvParams &p, int rb, const floa
       if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
       p.cand_val[rb * MAXB + tid] = bv;
       p.cand_idx[rb * MAXB + tid] = bi;
-      __threadfence();
     }
     named_bar_sync(1, CONSUMER_WARPS * 32);
     if (tid == 0) {
-      const int prev = atomicAdd(p.argmax_ticket, 1);
-      s_last_am = (prev == p.n_rb - 1);
+      const unsigned prev = atom_add_acq_rel(reinterpret_cast<unsigned *>(p.argmax_ticket), 1u);
+      s_last_am = (prev == (unsigned)(p.n_rb - 1));
       if (s_last_am) atomicExch(p.argmax_ticket, 0);
     }
     named_bar_sync(1, CONSUMER_WARPS * 32);
     if (s_last_am) {
-      __threadfence();
       for (int b = 0; b < B; ++b) {
         float bv = -INFINITY;
         int bi = 0x7fffffff;
@@ -269,18 +268,22 @@ __device__ __forceinline__ void tile_compute(const uint8_t *st, int warp, int la
   }
 }
 
-// RMSNorm scale of the GEMV input (1 without a norm), from the per-row-block sums of squares
-// of h, summed in block order; written to inv[0..B) by the first B consumer threads.
+// RMSNorm scale of the GEMV input (1 without a norm): warp b sums the per-row-block sums of
+// squares of user b's h (lane j takes parts j, j+32, ... in order, then a fixed butterfly), so
+// the loads are independent and the order is the same on every call.  Writes inv[0..B).
 template <int B>
 __device__ __forceinline__ void norm_scale(const GemvParams &p, float *inv, int tid) {
-  if (tid < B) {
+  const int warp = tid >> 5, lane = tid & 31;
+  if (warp < B) {
     float v = 1.0f;
     if (p.sumsq) {
       float s = 0.f;
-      for (int i = 0; i < p.n_parts; ++i) s += __ldcg(p.sumsq + i * MAXB + tid);
+      for (int i = lane; i < p.n_parts; i += 32) s += __ldcg(p.sumsq + i * MAXB + warp);
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
       v = 1.0f / sqrtf(s / static_cast<float>(p.d_norm) + p.eps);
     }
-    inv[tid] = v;
+    if (lane == 0) inv[warp] = v;
   }
 }
 
@@ -288,10 +291,23 @@ __device__ __forceinline__ void norm_scale(const GemvParams &p, float *inv, int 
 // starts at t0: reduce the lanes of each row, combine with the neighbouring CTAs that share the
 // row block (partials + atomic ticket; the last to arrive sums them in CTA order), and run the
 // epilogue once per row block.  All consumer threads call it.
+// Wait (one thread, bounded) until a counter written by other CTAs reaches `need`.
+__device__ __forceinline__ bool wait_counter(const unsigned *ctr, unsigned need, volatile int *abort_flag,
+                                             unsigned *err) {
+  for (uint32_t i = 0; i < 64u * WAIT_LIMIT; ++i) {
+    if (ld_acquire_gpu(ctr) >= need) return true;
+    if ((i & 255) == 255 && *abort_flag) return false;
+  }
+  *abort_flag = 1;
+  atomicOr(err, ERR_TIMEOUT);
+  return false;
+}
+
 template <int B, int EPI>
 __device__ __forceinline__ void segment_end(const GemvParams &p, int rb, int kt, int seg_kt0, long long t0,
                                             long long T, int G, int c, float (&acc)[B][4][2], float *red,
-                                            float *scr, const float *inv, int *s_last, int tid) {
+                                            float *scr, float *inv, int *inv_ready, int *s_last,
+                                            volatile int *abort_flag, int tid) {
   const int warp = tid >> 5, lane = tid & 31, kc = lane & 15, rsub = lane >> 4;
   float tot[B][4];
 #pragma unroll
@@ -319,33 +335,74 @@ __device__ __forceinline__ void segment_end(const GemvParams &p, int rb, int kt,
     const int slot = (rb == first_rb) ? 0 : 1;
     float *mine = p.partial + (size_t)(c * 2 + slot) * (RB * MAXB);
     for (int e = tid; e < RB * MAXB; e += CONSUMER_THREADS) mine[e] = red[e];
-    __threadfence();
     consumer_sync();
     const int c_lo = cta_of_tile((long long)rb * p.n_kt, T, G);
     const int c_hi = cta_of_tile((long long)(rb + 1) * p.n_kt - 1, T, G);
     if (tid == 0) {
-      const int prev = atomicAdd(p.tickets + rb, 1);
-      *s_last = (prev == c_hi - c_lo);
+      // release this CTA's partials; the last to arrive acquires everyone's
+      const unsigned prev = atom_add_acq_rel(reinterpret_cast<unsigned *>(p.tickets + rb), 1u);
+      *s_last = (prev == (unsigned)(c_hi - c_lo));
       if (*s_last) atomicExch(p.tickets + rb, 0);
     }
     consumer_sync();
     do_epi = *s_last != 0;
     if (do_epi) {
-      __threadfence();
+      // issue every partial's load first (independent), then add them in CTA order
+      constexpr int MAXPART = 8;
       for (int e = tid; e < RB * MAXB; e += CONSUMER_THREADS) {
         float sum = 0.f;
-        for (int cc = c_lo; cc <= c_hi; ++cc) {
-          const int frb = static_cast<int>(((long long)cc * T / G) / p.n_kt);
-          const int sl = (rb == frb) ? 0 : 1;
-          sum += __ldcg(p.partial + (size_t)(cc * 2 + sl) * (RB * MAXB) + e);
+        for (int c0 = c_lo; c0 <= c_hi; c0 += MAXPART) {
+          float v[MAXPART];
+#pragma unroll
+          for (int j = 0; j < MAXPART; ++j) {
+            const int cc = c0 + j;
+            v[j] = 0.f;
+            if (cc <= c_hi) {
+              const int frb = static_cast<int>(((long long)cc * T / G) / p.n_kt);
+              const int sl = (rb == frb) ? 0 : 1;
+              v[j] = __ldcg(p.partial + (size_t)(cc * 2 + sl) * (RB * MAXB) + e);
+            }
+          }
+#pragma unroll
+          for (int j = 0; j < MAXPART; ++j)
+            if (c0 + j <= c_hi) sum += v[j];
         }
         red[e] = sum;
       }
       consumer_sync();
     }
   }
+  if (do_epi && !*inv_ready) {
+    // the RMSNorm scale needs every row block of h: in the persistent kernel wait for the
+    // phase that produces h to complete them
+    if (tid == 0 && p.norm_done) wait_counter(p.norm_done, (unsigned)p.norm_need, abort_flag, p.err);
+    consumer_sync();
+    norm_scale<B>(p, inv, tid);
+    consumer_sync();
+    if (tid == 0) *inv_ready = 1;
+  }
   if (do_epi) epilogue<B, EPI>(p, rb, red, inv, scr, tid);
   consumer_sync();
+  if (do_epi && tid == 0) {
+    // publish this row block (the bar.sync above ordered every consumer's stores before it)
+    if (p.out_ready) {
+      int idx;
+      if constexpr (EPI == EPI_QKV) {
+        const int r0 = rb * RB, hd = p.head_dim;
+        const int group = p.n_q_rows / p.n_kv_rows;
+        if (r0 < p.n_q_rows)
+          idx = (r0 / hd) / group;
+        else if (r0 < p.n_q_rows + p.n_kv_rows)
+          idx = (r0 - p.n_q_rows) / hd;
+        else
+          idx = (r0 - p.n_q_rows - p.n_kv_rows) / hd;
+      } else {
+        idx = (rb * p.out_unit) / p.out_kt;
+      }
+      red_add_release(p.out_ready + idx, 1u);
+    }
+    if (p.out_done) red_add_release(p.out_done, 1u);
+  }
 }
 
 // Consumer side of one GEMV over this CTA's tile range [t0, t0 + n): wait for each tile's ring
@@ -354,8 +411,8 @@ __device__ __forceinline__ void segment_end(const GemvParams &p, int rb, int kt,
 template <int B, int EPI, int FMT>
 __device__ __forceinline__ void gemv_consume(const GemvParams &p, uint8_t *ring, uint64_t *full, uint64_t *empty,
                                              int S, int &s, uint32_t &phase, long long t0, int n, long long T,
-                                             int G, int c, float *red, float *scr, const float *inv, int *s_last,
-                                             volatile int *abort_flag, int tid) {
+                                             int G, int c, float *red, float *scr, float *inv, int *inv_ready,
+                                             int *s_last, volatile int *abort_flag, int tid) {
   const int warp = tid >> 5, lane = tid & 31;
   float acc[B][4][2];
   int seg_kt0 = 0;
@@ -370,10 +427,11 @@ __device__ __forceinline__ void gemv_consume(const GemvParams &p, uint8_t *ring,
       seg_kt0 = kt;
     }
     consumer_wait(smem_addr(&full[s]), phase, abort_flag, p.err);
-    tile_compute<B, FMT>(ring + (size_t)s * STAGE_BYTES, warp, lane, acc);
+    tile_compute<B, FMT>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc);
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_addr(&empty[s]));
-    if (kt == p.n_kt - 1 || i == n - 1) segment_end<B, EPI>(p, rb, kt, seg_kt0, t0, T, G, c, acc, red, scr, inv, s_last, tid);
+    if (kt == p.n_kt - 1 || i == n - 1)
+      segment_end<B, EPI>(p, rb, kt, seg_kt0, t0, T, G, c, acc, red, scr, inv, inv_ready, s_last, abort_flag, tid);
     if (++kt == p.n_kt) {
       kt = 0;
       ++rb;

@@ -7,7 +7,9 @@
 #include <cuda_runtime.h>
 
 #include <cmath>
+#include <algorithm>
 #include <cstdlib>
+#include <cstdio>
 #include <cstring>
 #include <vector>
 
@@ -52,6 +54,7 @@ struct Plan {
   Mat qkv, o, gu, down, lm;
   size_t kv_elems_per_layer;  // per cache (K or V)
   int n_sm, ctas_per_sm, stages, gemv_grid_max, n_rb_max, n_parts, attn_nchunks_max;
+  int n_phases, ctr_stride;  // persistent kernel: phases per step, readiness counters per phase
   size_t bytes_weights, bytes_kv, bytes_ws;
 };
 
@@ -106,7 +109,7 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   p->ctas_per_sm = env_int("KFL_GEMV_CTAS_PER_SM", 1);
   if (p->ctas_per_sm < 1 || p->ctas_per_sm > 2) p->ctas_per_sm = 1;
   p->stages = env_int("KFL_GEMV_STAGES", 6);
-  if (p->stages < 2 || p->stages > MAX_STAGES) p->stages = 6;
+  if (p->stages < 2 || p->stages > 10) p->stages = 6;
   p->gemv_grid_max = n_sm * p->ctas_per_sm;
   int nrb = 1;
   if (p->nl > 0) {
@@ -119,6 +122,14 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   p->n_rb_max = nrb;
   p->n_parts = (p->d + RB - 1) / RB;
   p->attn_nchunks_max = (c->max_ctx + 63) / 64;
+  p->n_phases = 5 * p->nl + ((flags & KFL_LOGITS_OUT) ? 1 : 0);
+  {
+    const int kk = tile_k(f);
+    int m = p->hkv;
+    const int lens[3] = {p->d, p->qdim, p->F};
+    for (int i = 0; i < 3; ++i) m = std::max(m, (lens[i] + kk - 1) / kk);
+    p->ctr_stride = round_up(m + 2, 32);
+  }
 
   size_t w = 0;
   if (p->nl > 0)
@@ -132,8 +143,9 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   ws += (size_t)MAXB * (2 * p->ldh + 2 * p->ldq + p->lda) * 4;         // h, xn, q, o, a
   ws += (size_t)p->n_parts * MAXB * 4;                                 // sum of squares
   ws += 2 * MAXB * 4;                                                  // positions, next ids
-  ws += (size_t)p->gemv_grid_max * 2 * RB * MAXB * 4;                  // stream-K partials
-  ws += (size_t)(p->n_rb_max + 1) * 4;                                 // tickets + argmax ticket
+  ws += (size_t)4 * p->gemv_grid_max * 2 * RB * MAXB * 4;              // stream-K partials (x4)
+  ws += (size_t)(4 * p->n_rb_max + 1) * 4;                             // tickets (x4) + argmax ticket
+  ws += (size_t)std::max(1, p->n_phases) * p->ctr_stride * 4;          // readiness counters
   ws += (size_t)p->n_rb_max * MAXB * 8;                                // argmax candidates
   ws += (size_t)MAXB * p->hkv * p->attn_nchunks_max * 8 * (p->hd + 4) * 4;  // attention partials
   ws += (size_t)MAXB * p->hkv * 4;                                     // attention tickets
@@ -167,16 +179,18 @@ struct kfl_stage {
   int *cand_idx = nullptr;
   float *attn_partial = nullptr;
   int *attn_tickets = nullptr;
+  unsigned *counters = nullptr;  // persistent kernel readiness counters [n_phases][ctr_stride]
   unsigned *err = nullptr;
   float *capture = nullptr;
+  unsigned long long *trace = nullptr;
   std::vector<void *> allocs;
   int alloc_count = 0, fault_at = 0;
   cudaStream_t cap_stream = nullptr;
   cudaGraphExec_t graph[MAXB + 1] = {};
   // persistent stage kernel
   bool persistent = true;
-  int mk_stages = 0;
-  size_t mk_smem = 0;
+  int mk_stages[MAXB + 1] = {};
+  size_t mk_smem[MAXB + 1] = {};
   unsigned *bar = nullptr;  // [0] grid-barrier counter, [1] abort flag
   Phase *phases_dev[MAXB + 1] = {};
   int n_phases = 0;
@@ -223,12 +237,18 @@ namespace {
 
 bool valid(const kfl_stage *st) { return st && st->magic == 0x4B464C53; }
 
-#define CK(x)                               \
-  do {                                      \
-    if ((x) != cudaSuccess) {               \
-      cudaGetLastError();                   \
-      return KFL_ERR_CUDA;                  \
-    }                                       \
+thread_local char g_last_error[256] = "";
+
+int record_cuda_error(cudaError_t e, const char *what, int line) {
+  snprintf(g_last_error, sizeof(g_last_error), "%s (%s) at stage.cu:%d", cudaGetErrorString(e), what, line);
+  cudaGetLastError();
+  return KFL_ERR_CUDA;
+}
+
+#define CK(x)                                                   \
+  do {                                                          \
+    cudaError_t _e = (x);                                       \
+    if (_e != cudaSuccess) return record_cuda_error(_e, #x, __LINE__); \
   } while (0)
 
 // Positions per attention unit: the same in both execution modes, so they give identical bits.
@@ -247,6 +267,7 @@ GemvParams base_gemv(kfl_stage *st, const Mat &m, const float *x, int ldx, int b
   g.ldx = ldx;
   g.batch = batch;
   g.stages = st->P.stages;
+  g.rope_per_user = 0;
   g.partial = st->gemv_partial;
   g.tickets = st->tickets;
   g.err = st->err;
@@ -257,7 +278,7 @@ GemvParams base_gemv(kfl_stage *st, const Mat &m, const float *x, int ldx, int b
 // The phases of one decode step of the stage at this batch size: for every block Q/K/V (+RoPE,
 // KV append), attention, O (+residual), gate/up (+SwiGLU), down (+residual); then lm_head
 // (+argmax) for the head.  Both execution modes run exactly these.
-std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk) {
+std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk, bool dataflow = false) {
   const Plan &P = st->P;
   const kfl_model_cfg &c = st->cfg;
   std::vector<Phase> ph;
@@ -266,6 +287,11 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk) {
     x.kind = PH_GEMV;
     x.epi = epi;
     x.g = g;
+    // stream-K partials and tickets rotate over four buffers, so a phase never reuses those
+    // of the three before it (in the persistent kernel phases overlap)
+    const int r = (int)ph.size() % 4;
+    x.g.partial = st->gemv_partial + (size_t)r * P.gemv_grid_max * 2 * RB * MAXB;
+    x.g.tickets = st->tickets + (size_t)r * P.n_rb_max;
     ph.push_back(x);
   };
   for (int l = 0; l < P.nl; ++l) {
@@ -355,6 +381,61 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk) {
     g.next_ids = st->next_int;
     gemv(EPI_ARGMAX, g);
   }
+  if (dataflow) {
+    // readiness counters: phase k publishes in region k, the phase after it reads region k
+    const int kk = tile_k(c.weight_fmt);
+    const int G = P.hq / P.hkv;
+    auto region = [&](int k) { return st->counters + (size_t)k * P.ctr_stride; };
+    auto done = [&](int k) { return st->counters + (size_t)k * P.ctr_stride + P.ctr_stride - 1; };
+    const int rb_d = (P.d + RB - 1) / RB;
+    for (size_t k = 0; k < ph.size(); ++k) {
+      Phase &x = ph[k];
+      const bool lm = (int)k == 5 * P.nl;
+      const int j = lm ? 5 : (int)(k % 5);  // 0 QKV, 1 attention, 2 O, 3 gate/up, 4 down, 5 lm_head
+      if (x.kind == PH_ATTN) {
+        x.a.in_ready = region((int)k - 1);
+        x.a.in_need = (G + 2) * P.hd / RB;
+        x.a.out_ready = region((int)k);
+        continue;
+      }
+      GemvParams &g = x.g;
+      if (j == 0 || j == 5) {  // input xn and the norm of h from the previous down (or none)
+        if (k > 0) {
+          g.in_kind = 1;
+          g.in_ready = region((int)k - 1);
+          g.in_len = P.d;
+          g.in_unit = RB;
+          g.norm_done = done((int)k - 1);
+          g.norm_need = rb_d;
+        }
+      } else if (j == 2) {  // attention output o
+        g.in_kind = 2;
+        g.in_ready = region((int)k - 1);
+        g.in_len = P.qdim;
+        g.in_group = G;
+        g.in_head_dim = P.hd;
+        g.in_need = batch;
+      } else if (j == 3) {  // xn and the norm of h from O
+        g.in_kind = 1;
+        g.in_ready = region((int)k - 1);
+        g.in_len = P.d;
+        g.in_unit = RB;
+        g.norm_done = done((int)k - 1);
+        g.norm_need = rb_d;
+      } else if (j == 4) {  // a from gate/up
+        g.in_kind = 1;
+        g.in_ready = region((int)k - 1);
+        g.in_len = P.F;
+        g.in_unit = RB / 2;
+      }
+      if (j != 5) {
+        g.out_ready = region((int)k);
+        g.out_done = done((int)k);
+        g.out_unit = (j == 3) ? RB / 2 : RB;
+        g.out_kt = kk;
+      }
+    }
+  }
   return ph;
 }
 
@@ -394,39 +475,47 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
   return KFL_OK;
 }
 
+// Persistent mode: the phase table of this batch size, uploaded once (outside any capture).
+int upload_phases(kfl_stage *st, int batch) {
+  if (st->phases_dev[batch]) return KFL_OK;
+  const std::vector<Phase> phases = build_phases(st, batch, st->persist_chunk[batch], true);
+  void *d = nullptr;
+  if (cudaMalloc(&d, phases.size() * sizeof(Phase)) != cudaSuccess) {
+    cudaGetLastError();
+    return KFL_ERR_OOM;
+  }
+  st->phases_dev[batch] = static_cast<Phase *>(d);
+  st->n_phases = (int)phases.size();
+  CK(cudaMemcpy(d, phases.data(), phases.size() * sizeof(Phase), cudaMemcpyHostToDevice));
+  return KFL_OK;
+}
+
 // Persistent mode: the whole step as one cooperative launch of the stage kernel.
 int enqueue_persistent(kfl_stage *st, int batch, cudaStream_t s) {
-  if (!st->phases_dev[batch]) {
-    const std::vector<Phase> phases = build_phases(st, batch, st->persist_chunk[batch]);
-    void *d = nullptr;
-    if (cudaMalloc(&d, phases.size() * sizeof(Phase)) != cudaSuccess) {
-      cudaGetLastError();
-      return KFL_ERR_OOM;
-    }
-    st->phases_dev[batch] = static_cast<Phase *>(d);
-    st->n_phases = (int)phases.size();
-    CK(cudaMemcpy(d, phases.data(), phases.size() * sizeof(Phase), cudaMemcpyHostToDevice));
-  }
   StageKernelParams kp = {};
   kp.phases = st->phases_dev[batch];
   kp.n_phases = st->n_phases;
-  kp.stages = st->mk_stages;
+  kp.stages = st->mk_stages[batch];
   kp.head_dim = st->P.hd;
   kp.attn_bytes = stage_kernel_attn_bytes(st->P.hd);
   kp.bar = st->bar;
   kp.abort_flag = reinterpret_cast<int *>(st->bar + 1);
   kp.err = st->err;
-  CK(launch_stage_kernel(kp, batch, st->cfg.weight_fmt, st->P.n_sm, st->mk_smem, s));
+  kp.trace = st->trace;
+  kp.positions = st->pos;
+  kp.rope_cos = st->rope_cos;
+  kp.rope_sin = st->rope_sin;
+  kp.max_ctx = st->cfg.max_ctx;
+  CK(cudaMemsetAsync(st->counters, 0, (size_t)std::max(1, st->n_phases) * st->P.ctr_stride * 4, s));
+  CK(launch_stage_kernel(kp, batch, st->cfg.weight_fmt, st->P.n_sm, st->mk_smem[batch], s));
   return KFL_OK;
 }
 
 int ensure_graph(kfl_stage *st, int batch) {
   if (st->graph[batch]) return KFL_OK;
   if (!st->cap_stream) CK(cudaStreamCreateWithFlags(&st->cap_stream, cudaStreamNonBlocking));
-  if (st->persistent && !st->phases_dev[batch]) {
-    // the phase table is uploaded outside the capture
-    int rc = enqueue_persistent(st, batch, nullptr);
-    CK(cudaDeviceSynchronize());
+  if (st->persistent) {
+    int rc = upload_phases(st, batch);
     if (rc != KFL_OK) return rc;
   }
   cudaGraph_t g = nullptr;
@@ -672,9 +761,10 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
   AL(st->sumsq, (size_t)P.n_parts * MAXB * 4);
   AL(st->pos, MAXB * 4);
   AL(st->next_int, MAXB * 4);
-  AL(st->gemv_partial, (size_t)P.gemv_grid_max * 2 * RB * MAXB * 4);
-  AL(st->tickets, (size_t)(P.n_rb_max + 1) * 4);
-  st->am_ticket = st->tickets + P.n_rb_max;
+  AL(st->gemv_partial, (size_t)4 * P.gemv_grid_max * 2 * RB * MAXB * 4);
+  AL(st->tickets, (size_t)(4 * P.n_rb_max + 1) * 4);
+  st->am_ticket = st->tickets + 4 * P.n_rb_max;
+  AL(st->counters, (size_t)std::max(1, P.n_phases) * P.ctr_stride * 4);
   AL(st->cand_val, (size_t)P.n_rb_max * MAXB * 4);
   AL(st->cand_idx, (size_t)P.n_rb_max * MAXB * 4);
   AL(st->attn_partial, (size_t)MAXB * P.hkv * P.attn_nchunks_max * 8 * (P.hd + 4) * 4);
@@ -694,7 +784,8 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
       cudaMemset(st->q, 0, (size_t)MAXB * P.ldq * 4) || cudaMemset(st->o, 0, (size_t)MAXB * P.ldq * 4) ||
       cudaMemset(st->a, 0, (size_t)MAXB * P.lda * 4) || cudaMemset(st->sumsq, 0, (size_t)P.n_parts * MAXB * 4) ||
       cudaMemset(st->pos, 0, MAXB * 4) || cudaMemset(st->next_int, 0, MAXB * 4) ||
-      cudaMemset(st->tickets, 0, (size_t)(P.n_rb_max + 1) * 4) ||
+      cudaMemset(st->tickets, 0, (size_t)(4 * P.n_rb_max + 1) * 4) ||
+      cudaMemset(st->counters, 0, (size_t)std::max(1, P.n_phases) * P.ctr_stride * 4) ||
       cudaMemset(st->attn_tickets, 0, (size_t)MAXB * P.hkv * 4) || cudaMemset(st->err, 0, 16) ||
       cudaMemset(st->bar, 0, 16))
     return fail(KFL_ERR_CUDA);
@@ -715,13 +806,18 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
   // persistent stage kernel: the deepest ring that fits next to the attention buffers
   st->persistent = env_int("KFL_PERSISTENT", 1) != 0;
   {
-    int stages = env_int("KFL_STAGE_KERNEL_STAGES", MAX_STAGES);
-    if (stages > MAX_STAGES) stages = MAX_STAGES;
-    const size_t static_smem = 4096;  // the kernel's own __shared__ variables
-    while (stages > 2 && stage_kernel_smem(stages, P.hd) + static_smem > (size_t)smem_optin) --stages;
-    st->mk_stages = stages;
-    st->mk_smem = stage_kernel_smem(stages, P.hd);
-    if (prepare_stage_kernel(st->mk_smem) != cudaSuccess) {
+    const size_t static_smem = 8192;  // the kernel's own __shared__ variables
+    size_t smem_max = 0;
+    for (int b = 1; b <= cfg->max_batch; ++b) {
+      int stages = env_int("KFL_STAGE_KERNEL_STAGES", MAX_STAGES);
+      if (stages > MAX_STAGES) stages = MAX_STAGES;
+      while (stages > 2 && stage_kernel_smem(stages, P.hd, b, cfg->weight_fmt) + static_smem > (size_t)smem_optin)
+        --stages;
+      st->mk_stages[b] = stages;
+      st->mk_smem[b] = stage_kernel_smem(stages, P.hd, b, cfg->weight_fmt);
+      if (st->mk_smem[b] > smem_max) smem_max = st->mk_smem[b];
+    }
+    if (prepare_stage_kernel(smem_max) != cudaSuccess) {
       cudaGetLastError();
       st->persistent = false;
     }
@@ -731,7 +827,7 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
       long long want = (work + P.n_sm - 1) / P.n_sm;
       if (want < 64) want = 64;
       int chunk = round_up((int)want, 64);
-      while ((long long)((cfg->max_ctx + chunk - 1) / chunk) * (P.hq / P.hkv) > 2048) chunk += 64;
+      while ((long long)((cfg->max_ctx + chunk - 1) / chunk) * (P.hq / P.hkv) > 1024) chunk += 64;
       if (chunk > round_up(cfg->max_ctx, 64)) chunk = round_up(cfg->max_ctx, 64);
       st->persist_chunk[b] = chunk;
     }
@@ -964,6 +1060,24 @@ extern "C" int kfl_stage_debug_capture(kfl_stage *st, float *per_layer_hidden) {
   return KFL_OK;
 }
 
+extern "C" int kfl_stage_trace(kfl_stage *st, uint64_t *buf) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  if (st->trace != reinterpret_cast<unsigned long long *>(buf)) {
+    st->trace = reinterpret_cast<unsigned long long *>(buf);
+    st->drop_graphs();
+  }
+  return KFL_OK;
+}
+
+extern "C" int kfl_stage_trace_shape(kfl_stage *st, int batch, int *n_phases, int *grid, int *slots) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  if (batch < 1 || batch > st->cfg.max_batch) return KFL_ERR_RANGE;
+  if (n_phases) *n_phases = (int)build_phases(st, batch, st->persist_chunk[batch]).size();
+  if (grid) *grid = st->P.n_sm;
+  if (slots) *slots = TRACE_SLOTS;
+  return KFL_OK;
+}
+
 extern "C" int kfl_stage_status(kfl_stage *st) {
   if (!valid(st)) return KFL_ERR_STATE;
   CK(cudaSetDevice(st->dev));
@@ -1015,6 +1129,8 @@ extern "C" void kfl_stage_destroy(kfl_stage *st) {
   st->magic = 0;
   delete st;
 }
+
+extern "C" const char *kfl_last_error_detail(void) { return g_last_error; }
 
 extern "C" const char *kfl_strerror(int code) {
   switch (code) {

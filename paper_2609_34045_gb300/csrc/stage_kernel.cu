@@ -4,19 +4,22 @@
 // A stage's cost is the time to stream its weights once (Kafila, section V-A, Eq. 2).  Split
 // into one kernel per operation, every boundary drains the memory pipe: the launch, the ramp of
 // the next kernel and the tail of the previous one.  Here the weights of every phase stream back
-// to back through one TMA ring per SM, and only the consumers synchronise between phases:
+// to back through one TMA ring per SM, and phases overlap as far as the data allows:
 //
-//   warps 0-7  consumers: GEMV tiles, epilogues and attention units of each phase in turn; a
-//              grid barrier (counter in global memory) separates a phase from its inputs
-//   warp 8     weight producer: the tiles of every GEMV phase of this CTA, in order, into the
-//              ring (cp.async.bulk), limited only by free stages, never by a grid barrier
-//   warp 9     activation producer: after the grid barrier that makes a phase's input ready,
-//              the matching activation chunks into the stages the weight producer armed
+//   warps 0-7  consumers: GEMV tiles, epilogues and attention units of each phase in turn;
+//              every finished piece of output is published on a readiness counter in global
+//              memory (release), per activation chunk, per KV head, and per phase
+//   warp 8     weight producer (one thread): the weight tiles of every GEMV phase of this CTA,
+//              in order, into the ring (cp.async.bulk) as soon as a stage is free; weights
+//              never wait for data, so HBM keeps streaming while the consumers wait
+//   warp 9     activation producer: for each tile, once the counters of its activation chunk
+//              say the producing phase has written it (polled a warp at a time, 32 chunks per
+//              L2 round trip), the chunk into the stage the weight producer armed
 //
-// While the consumers wait at a barrier or run attention, the weight producer keeps filling the
-// ring with the next phase's tiles, so HBM stays busy across phase boundaries.  Every wait is
-// bounded; a timeout sets the error word and a global abort flag that ends every other wait, so
-// the kernel always returns.
+// There is no grid-wide barrier: a CTA starts the next phase's tiles as soon as their inputs
+// exist, so the tail of one phase overlaps the start of the next.  Every wait is bounded; a
+// timeout sets the error word and a global abort flag that ends every other wait, so the kernel
+// always returns.
 #include "attn_core.cuh"
 #include "gemv_core.cuh"
 
@@ -24,30 +27,6 @@ namespace kfl {
 
 constexpr int MK_WARPS = CONSUMER_WARPS + 2;
 constexpr int MK_THREADS = MK_WARPS * 32;
-
-__device__ __forceinline__ unsigned ld_acquire(const unsigned *p) {
-  unsigned v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-
-// Wait until the grid-barrier counter reaches `target` (bounded; false on timeout or abort).
-__device__ bool grid_wait(const StageKernelParams &kp, unsigned target, volatile int *s_abort) {
-  for (uint32_t i = 0; i < WAIT_LIMIT; ++i) {
-    if (ld_acquire(kp.bar) >= target) return true;
-    if (i >= 64) {
-      if (*s_abort || *reinterpret_cast<volatile int *>(kp.abort_flag)) {
-        *s_abort = 1;
-        return false;
-      }
-      __nanosleep(i < 4096 ? 32 : 256);
-    }
-  }
-  *s_abort = 1;
-  atomicExch(kp.abort_flag, 1);
-  atomicOr(kp.err, ERR_TIMEOUT);
-  return false;
-}
 
 // Tile range of CTA c in a GEMV phase: stream-K over min(T, grid) CTAs; the rest get none.
 __device__ __forceinline__ void phase_range(const GemvParams &g, int c, int grid, long long &T, int &G,
@@ -63,51 +42,117 @@ __device__ __forceinline__ void phase_range(const GemvParams &g, int c, int grid
   n = static_cast<int>((long long)(c + 1) * T / G - t0);
 }
 
+// Is activation chunk kt of a GEMV phase written?  (acquire loads of the producers' counters)
+__device__ __forceinline__ bool chunk_ready(const GemvParams &g, int kt) {
+  if (g.in_kind == 1) {
+    const int kk = tile_k(g.fmt);
+    const int len = min(kk, g.in_len - kt * kk);
+    const unsigned need = (unsigned)((len + g.in_unit - 1) / g.in_unit);
+    return ld_acquire_gpu(g.in_ready + kt) >= need;
+  }
+  if (g.in_kind == 2) {
+    const int kk = tile_k(g.fmt);
+    const int h0 = (kt * kk) / g.in_head_dim;
+    const int h1 = min(((kt + 1) * kk - 1) / g.in_head_dim, g.in_len / g.in_head_dim - 1);
+    for (int kvh = h0 / g.in_group; kvh <= h1 / g.in_group; ++kvh)
+      if (ld_acquire_gpu(g.in_ready + kvh) < (unsigned)g.in_need) return false;
+    return true;
+  }
+  return true;
+}
+
 // Phase bodies as separate (not inlined) functions: each gets its own register allocation, so
 // the widest one does not raise the pressure of the rest of the kernel.
 template <int B, int EPI, int FMT>
-__device__ __noinline__ void gemv_phase(const GemvParams &g, uint8_t *ring, uint64_t *full, uint64_t *empty, int S,
-                                        int &s, uint32_t &phase, long long t0, int n, long long T, int G, int c,
-                                        float *red, float *scr, const float *inv, int *s_last, volatile int *abort_flag,
-                                        int tid) {
-  gemv_consume<B, EPI, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, inv, s_last, abort_flag,
-                            tid);
+__device__ __noinline__ void gemv_phase_call(const GemvParams &g, uint8_t *ring, uint64_t *full, uint64_t *empty,
+                                             int S, int &s, uint32_t &phase, long long t0, int n, long long T, int G,
+                                             int c, float *red, float *scr, float *inv, int *inv_ready, int *s_last,
+                                             volatile int *abort_flag, int tid) {
+  gemv_consume<B, EPI, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, inv, inv_ready, s_last,
+                            abort_flag, tid);
+}
+
+// Batches 1-2 inline the loop (shared-memory addressing known to the compiler); wider batches
+// call the out-of-line copy.
+template <int B, int EPI, int FMT>
+__device__ __forceinline__ void gemv_phase(const GemvParams &g, uint8_t *ring, uint64_t *full, uint64_t *empty, int S,
+                                           int &s, uint32_t &phase, long long t0, int n, long long T, int G, int c,
+                                           float *red, float *scr, float *inv, int *inv_ready, int *s_last,
+                                           volatile int *abort_flag, int tid) {
+  if constexpr (B <= 2)
+    gemv_consume<B, EPI, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, inv, inv_ready, s_last,
+                              abort_flag, tid);
+  else
+    gemv_phase_call<B, EPI, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, inv, inv_ready,
+                                 s_last, abort_flag, tid);
 }
 
 template <int HD>
 __device__ __noinline__ void attn_phase_unit(const AttnParams &a, int b, int kvh, int ch, int nc, uint8_t *att,
-                                             int *s_last, int tid) {
-  attn_unit<HD>(a, b, kvh, ch, nc, att, s_last, tid);
+                                             int *s_last, int tid, int prefetched) {
+  attn_unit<HD, 1>(a, b, kvh, ch, nc, att, s_last, tid, prefetched);
+}
+
+// (user, KV head, chunk) of attention unit u: users in order, n_kv_heads * nc_b units each.
+__device__ __forceinline__ void attn_unit_coords(int u, int hk, int nc0, int nc1, int nc2, int nc3, int &b, int &kvh,
+                                                 int &ch, int &ncb) {
+  int rem = u;
+  b = 0;
+  ncb = nc0;
+  if (rem >= nc0 * hk) {
+    rem -= nc0 * hk;
+    b = 1;
+    ncb = nc1;
+    if (rem >= nc1 * hk) {
+      rem -= nc1 * hk;
+      b = 2;
+      ncb = nc2;
+      if (rem >= nc2 * hk) {
+        rem -= nc2 * hk;
+        b = 3;
+        ncb = nc3;
+      }
+    }
+  }
+  kvh = rem / ncb;
+  ch = rem % ncb;
 }
 
 template <int B, int FMT>
-__global__ void __maxnreg__(200) stage_kernel(const __grid_constant__ StageKernelParams kp) {
+__global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_constant__ StageKernelParams kp) {
   extern __shared__ __align__(1024) uint8_t smem[];
+  constexpr int SB = stage_bytes(B, FMT);
   const int S = kp.stages;
   uint8_t *ring = smem;
-  uint8_t *att = smem + (size_t)S * STAGE_BYTES;
+  uint8_t *att = smem + (size_t)S * SB;
   uint64_t *full = reinterpret_cast<uint64_t *>(att + kp.attn_bytes);
   uint64_t *empty = full + S;
-  float *red = reinterpret_cast<float *>(empty + S);  // [RB][MAXB]
+  uint64_t *armed = empty + S;                        // weight tile issued (for the x producer)
+  float *red = reinterpret_cast<float *>(armed + S);  // [RB][MAXB]
   float *scr = red + RB * MAXB;                       // 2 * CONSUMER_WARPS words
-  volatile int *armed = reinterpret_cast<volatile int *>(scr + 2 * CONSUMER_WARPS);  // [S]
   __shared__ GemvParams s_gp;
   __shared__ AttnParams s_ap;
   __shared__ float s_inv[MAXB];
   __shared__ int s_last;
+  __shared__ int s_inv_ready;
   __shared__ volatile int s_abort;
   __shared__ volatile int s_issued;
+  __shared__ int s_pos[MAXB];                           // this step's positions
+  __shared__ float s_cos[MAXB * 64], s_sin[MAXB * 64];  // their RoPE rows
 
   constexpr int KTILE = FMT == 0 ? KT : KT4;
   constexpr uint32_t WBYTES = FMT == 0 ? TILE_BYTES : TILE4_BYTES;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int c = blockIdx.x, grid = gridDim.x;
+  auto stamp = [&](int k, int slot) {
+    if (kp.trace) kp.trace[((size_t)k * grid + c) * TRACE_SLOTS + slot] = global_ns();
+  };
 
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_addr(&full[s]), 1);
       mbar_init(smem_addr(&empty[s]), CONSUMER_WARPS);
-      armed[s] = -1;
+      mbar_init(smem_addr(&armed[s]), 1);
     }
     s_abort = 0;
     s_issued = 0;
@@ -116,7 +161,7 @@ __global__ void __maxnreg__(200) stage_kernel(const __grid_constant__ StageKerne
   __syncthreads();
 
   if (warp == CONSUMER_WARPS) {
-    // -------------------------------------------------------------- weight producer
+    // ---------------------------------------------------------- weight producer
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
       const uint32_t bytes = WBYTES + B * (KTILE * 4);
@@ -128,160 +173,192 @@ __global__ void __maxnreg__(200) stage_kernel(const __grid_constant__ StageKerne
         int G, n;
         phase_range(ph->g, c, grid, T, G, t0, n);
         const uint8_t *w = ph->g.w;
+        if (n > 0) stamp(k, TR_W_FIRST);
         for (int i = 0; i < n; ++i) {
           if (round > 0 && !consumer_wait(smem_addr(&empty[s]), (round & 1) ^ 1, &s_abort, kp.err)) break;
           const uint32_t fb = smem_addr(&full[s]);
           mbar_arrive_expect_tx(fb, bytes);
-          bulk_g2s(smem_addr(ring + (size_t)s * STAGE_BYTES), w + (size_t)(t0 + i) * WBYTES, WBYTES, fb, pol);
-          armed[s] = gi;
-          s_issued = gi + 1;
-          ++gi;
+          bulk_g2s(smem_addr(ring + (size_t)s * SB), w + (size_t)(t0 + i) * WBYTES, WBYTES, fb, pol);
+          mbar_arrive(smem_addr(&armed[s]));
+          s_issued = ++gi;
           if (++s == S) {
             s = 0;
             ++round;
           }
         }
+        if (n > 0) stamp(k, TR_W_LAST);
       }
     }
     return;
   }
   if (warp == CONSUMER_WARPS + 1) {
-    // ---------------------------------------------------------- activation producer
-    if (lane == 0) {
-      const uint64_t pol = policy_evict_last();
-      int s = 0, gi = 0;
-      for (int k = 0; k < kp.n_phases && !s_abort; ++k) {
-        const Phase *ph = kp.phases + k;
-        if (ph->kind != PH_GEMV) continue;
-        long long T, t0;
-        int G, n;
-        phase_range(ph->g, c, grid, T, G, t0, n);
-        if (n == 0) continue;
-        if (k > 0) {
-          if (!grid_wait(kp, (unsigned)k * grid, &s_abort)) break;
-          // the activations were written by other CTAs' generic stores; order them before
-          // this thread's bulk (async-proxy) reads
-          asm volatile("fence.proxy.async.global;" ::: "memory");
-        }
-        const float *x = ph->g.x;
-        const int ldx = ph->g.ldx, n_kt = ph->g.n_kt;
-        int kt = static_cast<int>(t0 % n_kt);
-        for (int i = 0; i < n; ++i) {
-          bool ok = false;
-          for (uint32_t it = 0; it < WAIT_LIMIT; ++it) {
-            if (armed[s] == gi) {
-              ok = true;
-              break;
-            }
-            if (s_abort) break;
-            if (it >= WAIT_FAST_SPINS) __nanosleep(64);
-          }
-          if (!ok) {
-            if (!s_abort) {
+    // ------------------------------------------------------- activation producer
+    // The whole warp polls the readiness of the next 32 tiles' chunks at once; lane 0 then
+    // issues the copies of the ready prefix, in order, into the armed stages.
+    const uint64_t pol = policy_evict_last();
+    int s = 0;
+    uint32_t aph = 0;
+    for (int k = 0; k < kp.n_phases && !s_abort; ++k) {
+      const Phase *ph = kp.phases + k;
+      if (ph->kind != PH_GEMV) continue;
+      const GemvParams &g = ph->g;
+      long long T, t0;
+      int G, n;
+      phase_range(g, c, grid, T, G, t0, n);
+      if (n == 0) continue;
+      const float *x = g.x;
+      const int ldx = g.ldx, n_kt = g.n_kt;
+      int kt = static_cast<int>(t0 % n_kt);
+      int i = 0;
+      uint32_t idle = 0;
+      bool first = true;
+      while (i < n && !s_abort) {
+        const int my_kt = (kt + lane) % n_kt;
+        const bool ok = (i + lane >= n) || chunk_ready(g, my_kt);
+        const unsigned ready = __ballot_sync(0xffffffffu, ok);
+        // every lane's acquire happens before lane 0's copies (__syncwarp orders memory among
+        // the participating threads)
+        __syncwarp();
+        const int run = min(n - i, (int)__ffs(~ready) - 1 < 0 ? 32 : (int)__ffs(~ready) - 1);
+        if (run <= 0) {
+          if (++idle > WAIT_LIMIT) {
+            if (lane == 0) {
               s_abort = 1;
               atomicExch(kp.abort_flag, 1);
               atomicOr(kp.err, ERR_TIMEOUT);
             }
             break;
           }
-          const uint32_t fb = smem_addr(&full[s]);
-          const uint32_t dst = smem_addr(ring + (size_t)s * STAGE_BYTES + WBYTES);
-#pragma unroll
-          for (int b = 0; b < B; ++b)
-            bulk_g2s(dst + b * (KTILE * 4), x + (size_t)b * ldx + (size_t)kt * KTILE, KTILE * 4, fb, pol);
-          ++gi;
-          if (++s == S) s = 0;
-          if (++kt == n_kt) kt = 0;
+          if ((idle & 63) == 0 && *reinterpret_cast<volatile int *>(kp.abort_flag)) {
+            if (lane == 0) s_abort = 1;
+            break;
+          }
+          continue;
         }
+        idle = 0;
+        if (lane == 0) {
+          // the chunks were written by other CTAs' generic stores: order them before this
+          // thread's bulk (async-proxy) reads
+          asm volatile("fence.proxy.async.global;" ::: "memory");
+          if (first) stamp(k, TR_X_GO);
+          for (int j = 0; j < run; ++j) {
+            if (!consumer_wait(smem_addr(&armed[s]), aph, &s_abort, kp.err)) break;
+            const uint32_t fb = smem_addr(&full[s]);
+            const uint32_t dst = smem_addr(ring + (size_t)s * SB + WBYTES);
+            const int ktj = (kt + j) % n_kt;
+#pragma unroll
+            for (int b = 0; b < B; ++b)
+              bulk_g2s(dst + b * (KTILE * 4), x + (size_t)b * ldx + (size_t)ktj * KTILE, KTILE * 4, fb, pol);
+            if (++s == S) {
+              s = 0;
+              aph ^= 1u;
+            }
+          }
+        }
+        s = __shfl_sync(0xffffffffu, s, 0);
+        aph = __shfl_sync(0xffffffffu, aph, 0);
+        first = false;
+        i += run;
+        kt = (kt + run) % n_kt;
       }
+      if (lane == 0) stamp(k, TR_X_LAST);
     }
     return;
   }
 
   // ------------------------------------------------------------------- consumers
+  {
+    // positions never change during the step: keep them and their RoPE rows in shared memory
+    const int half = kp.head_dim / 2;
+    for (int e = tid; e < B * half; e += CONSUMER_THREADS) {
+      const int b = e / half, i = e % half;
+      int pos = kp.positions[b];
+      if (pos < 0 || pos >= kp.max_ctx) pos = 0;
+      s_cos[e] = kp.rope_cos[(size_t)pos * half + i];
+      s_sin[e] = kp.rope_sin[(size_t)pos * half + i];
+    }
+    if (tid < MAXB) s_pos[tid] = tid < B ? kp.positions[tid] : 0;
+  }
   int s = 0;
   uint32_t phase = 0;
   for (int k = 0; k < kp.n_phases; ++k) {
     const Phase *ph = kp.phases + k;
     const int kind = ph->kind;
     if (tid == 0) {
-      // the phase table is read-only: copy this phase's parameters before waiting
-      if (kind == PH_GEMV)
+      stamp(k, TR_CONS_ENTER);
+      // the phase table is read-only: this phase's parameters, with the step constants in smem
+      if (kind == PH_GEMV) {
         s_gp = ph->g;
-      else
+        s_gp.positions = s_pos;
+        if (s_gp.rope_cos) {
+          s_gp.rope_cos = s_cos;
+          s_gp.rope_sin = s_sin;
+          s_gp.rope_per_user = 1;
+        }
+        s_inv_ready = 0;
+      } else {
         s_ap = ph->a;
-      if (k > 0) grid_wait(kp, (unsigned)k * grid, &s_abort);
+        s_ap.positions = s_pos;
+      }
     }
     consumer_sync();
     if (kind == PH_GEMV) {
       const GemvParams &g = s_gp;
-      norm_scale<B>(g, s_inv, tid);
-      consumer_sync();
       long long T, t0;
       int G, n;
       phase_range(g, c, grid, T, G, t0, n);
+      if (tid == 0) stamp(k, TR_CONS_GO);
       switch (ph->epi) {
         case EPI_QKV:
-          gemv_phase<B, EPI_QKV, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv, &s_last,
-                                        &s_abort, tid);
+          gemv_phase<B, EPI_QKV, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv,
+                                      &s_inv_ready, &s_last, &s_abort, tid);
           break;
         case EPI_RESID:
           gemv_phase<B, EPI_RESID, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv,
-                                          &s_last, &s_abort, tid);
+                                        &s_inv_ready, &s_last, &s_abort, tid);
           break;
         case EPI_SWIGLU:
           gemv_phase<B, EPI_SWIGLU, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv,
-                                           &s_last, &s_abort, tid);
+                                         &s_inv_ready, &s_last, &s_abort, tid);
           break;
         case EPI_ARGMAX:
           gemv_phase<B, EPI_ARGMAX, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv,
-                                           &s_last, &s_abort, tid);
+                                         &s_inv_ready, &s_last, &s_abort, tid);
           break;
         default:
           gemv_phase<B, EPI_STORE, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv,
-                                          &s_last, &s_abort, tid);
+                                        &s_inv_ready, &s_last, &s_abort, tid);
           break;
       }
     } else {
       const AttnParams &a = s_ap;
-      // units (user, KV head, chunk), users in order; user b has n_kv_heads * nc_b units
       const int nc0 = attn_chunks(a, 0);
       const int nc1 = a.batch > 1 ? attn_chunks(a, 1) : 0;
       const int nc2 = a.batch > 2 ? attn_chunks(a, 2) : 0;
       const int nc3 = a.batch > 3 ? attn_chunks(a, 3) : 0;
-      const int hk = a.n_kv_heads;
-      const int units = (nc0 + nc1 + nc2 + nc3) * hk;
+      const int units = (nc0 + nc1 + nc2 + nc3) * a.n_kv_heads;
       for (int u = c; u < units; u += grid) {
-        int rem = u, b = 0, ncb = nc0;
-        if (rem >= nc0 * hk) {
-          rem -= nc0 * hk;
-          b = 1;
-          ncb = nc1;
-          if (rem >= nc1 * hk) {
-            rem -= nc1 * hk;
-            b = 2;
-            ncb = nc2;
-            if (rem >= nc2 * hk) {
-              rem -= nc2 * hk;
-              b = 3;
-              ncb = nc3;
-            }
-          }
-        }
-        const int kvh = rem / ncb, ch = rem % ncb;
+        int b, kvh, ch, ncb;
+        attn_unit_coords(u, a.n_kv_heads, nc0, nc1, nc2, nc3, b, kvh, ch, ncb);
+        // the cached K/V rows do not depend on this step: load them while the Q/K/V rows of
+        // this KV head are still being produced
         if (kp.head_dim == 128)
-          attn_phase_unit<128>(a, b, kvh, ch, ncb, att, &s_last, tid);
+          attn_prefetch<128, 1>(a, b, kvh, ch, att, tid);
         else
-          attn_phase_unit<64>(a, b, kvh, ch, ncb, att, &s_last, tid);
+          attn_prefetch<64, 1>(a, b, kvh, ch, att, tid);
+        if (tid == 0) {
+          if (u == c) stamp(k, TR_CONS_GO);
+          if (a.in_ready) wait_counter(a.in_ready + kvh, (unsigned)a.in_need, &s_abort, kp.err);
+        }
+        consumer_sync();
+        if (kp.head_dim == 128)
+          attn_phase_unit<128>(a, b, kvh, ch, ncb, att, &s_last, tid, 1);
+        else
+          attn_phase_unit<64>(a, b, kvh, ch, ncb, att, &s_last, tid, 1);
         consumer_sync();
       }
     }
-    // this CTA's part of phase k is written: arrive at the grid barrier
-    consumer_sync();
-    if (tid == 0) {
-      __threadfence();
-      atomicAdd(kp.bar, 1u);
-    }
+    if (tid == 0) stamp(k, TR_CONS_DONE);
   }
 
   if (s_abort && tid == 0) {
@@ -292,13 +369,14 @@ __global__ void __maxnreg__(200) stage_kernel(const __grid_constant__ StageKerne
 }
 
 // ------------------------------------------------------------------------------- launch
-size_t stage_kernel_smem(int stages, int head_dim) {
-  const size_t att = head_dim == 128 ? AttnLayout<128>::BYTES : AttnLayout<64>::BYTES;
-  return (size_t)stages * STAGE_BYTES + att + 2 * stages * sizeof(uint64_t) +
-         (RB * MAXB + 2 * CONSUMER_WARPS) * sizeof(float) + stages * sizeof(int);
+size_t stage_kernel_smem(int stages, int head_dim, int batch, int fmt) {
+  return (size_t)stages * stage_bytes(batch, fmt) + stage_kernel_attn_bytes(head_dim) +
+         3 * stages * sizeof(uint64_t) + (RB * MAXB + 2 * CONSUMER_WARPS) * sizeof(float);
 }
 
-int stage_kernel_attn_bytes(int head_dim) { return head_dim == 128 ? AttnLayout<128>::BYTES : AttnLayout<64>::BYTES; }
+int stage_kernel_attn_bytes(int head_dim) {
+  return head_dim == 128 ? AttnLayout<128, 1>::BYTES : AttnLayout<64, 1>::BYTES;
+}
 
 template <int B, int FMT>
 static cudaError_t prepare_one_stage(size_t smem) {
@@ -306,6 +384,7 @@ static cudaError_t prepare_one_stage(size_t smem) {
 }
 
 cudaError_t prepare_stage_kernel(size_t smem) {
+  // every instantiation may use up to `smem` bytes of dynamic shared memory
   cudaError_t e;
   if ((e = prepare_one_stage<1, 0>(smem)) != cudaSuccess) return e;
   if ((e = prepare_one_stage<2, 0>(smem)) != cudaSuccess) return e;

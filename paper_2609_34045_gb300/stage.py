@@ -26,7 +26,8 @@ SYNTH_NORMAL_BF16, SYNTH_INT4_WORDS, SYNTH_INT4_SCALES_BF16 = 0, 1, 2
 class KflError(RuntimeError):
     def __init__(self, code: int, where: str):
         self.code = code
-        super().__init__(f"{where}: {kfl_strerror(code)} ({code})")
+        detail = kfl_last_error_detail() if code == -4 else ""
+        super().__init__(f"{where}: {kfl_strerror(code)} ({code}){': ' + detail if detail else ''}")
 
 
 class kfl_model_cfg(C.Structure):
@@ -76,11 +77,14 @@ def lib() -> C.CDLL:
             "kfl_kv_read": ([vp, i, i, vp, vp, i], i),
             "kfl_stage_debug_capture": ([vp, vp], i),
             "kfl_stage_status": ([vp], i),
+            "kfl_stage_trace": ([vp, vp], i),
+            "kfl_stage_trace_shape": ([vp, i, C.POINTER(i), C.POINTER(i), C.POINTER(i)], i),
             "kfl_stage_profile": ([vp, i], i),
             "kfl_stage_profile_read": ([vp, C.POINTER(C.c_double), C.POINTER(C.c_int64), i], i),
             "kfl_stage_launches_per_step": ([vp, i], i),
             "kfl_stage_destroy": ([vp], None),
             "kfl_strerror": ([i], C.c_char_p),
+            "kfl_last_error_detail": ([], C.c_char_p),
             "kfl_synth_key": ([C.c_uint64, C.c_uint64], C.c_uint64),
             "kfl_synth_fill": ([vp, C.c_int64, C.c_uint64, C.c_uint64, i, C.c_float, C.c_float, C.c_int64, vp], i),
         }
@@ -115,6 +119,10 @@ def _check(rc: int, where: str) -> int:
 
 def kfl_strerror(code: int) -> str:
     return lib().kfl_strerror(code).decode()
+
+
+def kfl_last_error_detail() -> str:
+    return lib().kfl_last_error_detail().decode()
 
 
 def model_cfg(shape, max_ctx: int, max_batch: int) -> kfl_model_cfg:
@@ -225,6 +233,17 @@ def kfl_kv_read(st: Stage, local: int, user: int, k, v, on_device: bool) -> None
 
 def kfl_stage_debug_capture(st: Stage, per_layer_hidden) -> None:
     _check(lib().kfl_stage_debug_capture(st.handle, _ptr(per_layer_hidden)), "kfl_stage_debug_capture")
+
+
+def kfl_stage_trace(st: Stage, buf) -> None:
+    _check(lib().kfl_stage_trace(st.handle, _ptr(buf)), "kfl_stage_trace")
+
+
+def kfl_stage_trace_shape(st: Stage, batch: int) -> tuple:
+    n, g, sl = C.c_int(), C.c_int(), C.c_int()
+    _check(lib().kfl_stage_trace_shape(st.handle, batch, C.byref(n), C.byref(g), C.byref(sl)),
+           "kfl_stage_trace_shape")
+    return n.value, g.value, sl.value
 
 
 def kfl_stage_status(st: Stage) -> int:
