@@ -19,7 +19,7 @@ constexpr int KT = 128;           // K per bf16 tile
 constexpr int TILE_BYTES = RB * KT * 2;
 constexpr int MAXB = 4;           // users per step
 constexpr int CONSUMER_WARPS = 8;
-constexpr int GEMV_THREADS = (CONSUMER_WARPS + 1) * 32;
+constexpr int GEMV_THREADS = (CONSUMER_WARPS + 2) * 32;  // consumers, producer, epilogue warp
 constexpr int MAX_STAGES = 12;
 
 // int4 group-64 tiles: [N/RB][K/KT4][RB][KT4/8] uint32 codes then [RB][KT4/64] bf16 scales
@@ -153,6 +153,7 @@ struct StageKernelParams {
   const int *positions;       // [batch] (static during the step)
   const float *rope_cos, *rope_sin;  // [max_ctx][hd/2]
   int max_ctx;
+  int l2_ahead;               // weight tiles prefetched into L2 ahead of the ring, per CTA
 };
 
 // phase trace slots (ns, %globaltimer)
@@ -258,6 +259,18 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
       " [%0], [%1], %2, [%3], %4;" ::"r"(dst),
       "l"(src), "r"(bytes), "r"(bar), "l"(policy)
       : "memory");
+}
+
+// 1-D bulk prefetch global -> L2 (no completion tracking); 16-byte aligned, size multiple of 16.
+__device__ __forceinline__ void bulk_prefetch_l2(const void *src, uint32_t bytes, uint64_t policy) {
+  asm volatile("cp.async.bulk.prefetch.L2.global.L2::cache_hint [%0], %1, %2;" ::"l"(src), "r"(bytes), "l"(policy)
+               : "memory");
+}
+
+__device__ __forceinline__ uint64_t policy_evict_normal() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
 }
 
 // Programmatic dependent launch (PDL)

@@ -26,17 +26,19 @@ constexpr int GEMV_MAX_STAGES = 10;  // standalone kernel: two CTAs (this and th
 
 // ---------------------------------------------------------------------------- the kernel
 // FMT 0: bf16 tiles [RB][KT].  FMT 1: int4 tiles, codes [RB][KT4/8] uint32 + scales [RB][KT4/64].
+// Warps 0-7 consume tiles, warp 8 is the TMA producer, warp 9 the epilogue warp.
 template <int B, int EPI, int FMT>
 __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) gemv_kernel(const __grid_constant__ GemvParams p) {
   extern __shared__ __align__(1024) uint8_t smem[];
-  const int S = p.stages;
   constexpr int SB = stage_bytes(B, FMT);
+  const int S = p.stages;
   uint64_t *full = reinterpret_cast<uint64_t *>(smem + (size_t)S * SB);
   uint64_t *empty = full + S;
-  float *red = reinterpret_cast<float *>(empty + S);  // [RB][MAXB]
-  float *scr = red + RB * MAXB;                       // 2 * CONSUMER_WARPS words
+  uint64_t *seg_full = empty + S;
+  uint64_t *seg_empty = seg_full + NSLOT;
+  // [NSLOT][RB][MAXB], 128-byte aligned (read as float4)
+  float *red = reinterpret_cast<float *>((reinterpret_cast<uintptr_t>(seg_empty + NSLOT) + 127) & ~uintptr_t(127));
   __shared__ float s_inv[MAXB];
-  __shared__ int s_last;
   __shared__ volatile int s_abort;
   __shared__ volatile int s_issued;
 
@@ -47,11 +49,16 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
   const int G = gridDim.x, c = blockIdx.x;
   const long long t0 = (long long)c * T / G, t1 = (long long)(c + 1) * T / G;
   const int n = static_cast<int>(t1 - t0);
+  const SegRing sr = {red, seg_full, seg_empty};
 
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_addr(&full[s]), 1);
       mbar_init(smem_addr(&empty[s]), CONSUMER_WARPS);
+    }
+    for (int s = 0; s < NSLOT; ++s) {
+      mbar_init(smem_addr(&seg_full[s]), CONSUMER_WARPS);
+      mbar_init(smem_addr(&seg_empty[s]), 1);
     }
     s_abort = 0;
     s_issued = 0;
@@ -104,17 +111,22 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
     }
     return;
   }
+  if (warp == CONSUMER_WARPS + 1) {
+    // -------------------------------------------------------------- epilogue warp
+    pdl_wait();
+    norm_scale_warp<B>(p, s_inv, lane);
+    bool inv_ready = true;
+    int segc = 0;
+    gemv_epilogues<B, EPI>(p, t0, n, T, G, c, sr, segc, s_inv, inv_ready, &s_abort, lane);
+    return;
+  }
 
   // -------------------------------------------------------------------- consumers
-  pdl_wait();
-  norm_scale<B>(p, s_inv, tid);
-  consumer_sync();
-  int s = 0;
+  int s = 0, segc = 0;
   uint32_t phase = 0;
-  int inv_ready = 1;
-  gemv_consume<B, EPI, FMT>(p, smem, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv, &inv_ready, &s_last,
-                            &s_abort, tid);
+  gemv_consume<B, FMT>(p.n_kt, smem, full, empty, S, s, phase, t0, n, sr, segc, &s_abort, p.err, tid);
 
+  consumer_sync();
   if (s_abort && tid == 0) {
     // drain copies still in flight before the CTA's shared memory goes away (bounded)
     const int issued = s_issued;
@@ -125,8 +137,8 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
 
 // ---------------------------------------------------------------------------- launch
 static size_t gemv_smem_bytes(int stages, int batch, int fmt) {
-  return (size_t)stages * stage_bytes(batch, fmt) + 2 * stages * sizeof(uint64_t) +
-         (RB * MAXB + 2 * CONSUMER_WARPS) * sizeof(float);
+  return (size_t)stages * stage_bytes(batch, fmt) + (2 * stages + 2 * NSLOT) * sizeof(uint64_t) +
+         128 + NSLOT * RB * MAXB * sizeof(float);
 }
 
 template <int B, int EPI, int FMT>

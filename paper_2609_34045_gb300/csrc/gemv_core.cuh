@@ -1,10 +1,17 @@
 // Device-side building blocks of the weight-streaming GEMV, shared by the standalone GEMV
 // kernel (gemv.cu) and the persistent stage kernel (stage_kernel.cu).
 //
-// Tile layout: a matrix [N][K] is stored as tiles [N/64][K/KT][64][KT]; a consumer CTA has 8
-// warps; lane `kc = lane & 15` owns a K chunk (8 bf16 or 16 int4 codes) of the rows
-// warp*8 + (lane >> 4) + 2j, j < 4, so each warp-wide shared-memory load reads two whole tile
-// rows (conflict-free) and the activation chunk is reused over four rows.
+// Tile layout: a matrix [N][K] is stored as tiles [N/64][K/KT][64][KT]; the 8 consumer warps of
+// a CTA each own 8 rows of every tile: lane `kc = lane & 15` takes a K chunk (8 bf16 or 16 int4
+// codes) of rows warp*8 + (lane >> 4) + 2j, j < 4, so a warp-wide shared-memory load reads two
+// whole tile rows (conflict-free) and the activation chunk is reused over four rows.
+//
+// The consumer warps never stop for an epilogue: at the end of a row-block segment each warp
+// reduces its rows into a staging slot and goes on with the next tile.  One epilogue warp takes
+// the slots in the same order and does everything with latency: the partial sums of row blocks
+// shared with neighbouring CTAs (written to global memory; the last CTA to arrive on an atomic
+// ticket adds them in CTA order), the RMSNorm scale, the fused epilogue, and (persistent kernel)
+// the readiness counters.  Memory in flight therefore never drains at a segment end.
 //
 // Every global read of data written by other CTAs goes through L2 (ld.global.cg): inside the
 // persistent kernel a CTA's L1 may hold lines from an earlier phase.
@@ -18,6 +25,7 @@ namespace kfl {
 
 constexpr int CONSUMER_THREADS = CONSUMER_WARPS * 32;
 constexpr int CONSUMER_BAR = 1;  // named barrier of the consumer warps
+constexpr int NSLOT = 4;         // staging slots between the consumer warps and the epilogue warp
 
 __device__ __forceinline__ void consumer_sync() { named_bar_sync(CONSUMER_BAR, CONSUMER_THREADS); }
 
@@ -41,6 +49,7 @@ __device__ __forceinline__ int cta_of_tile(long long t, long long T, int G) {
   return static_cast<int>(((t + 1) * G - 1) / T);
 }
 
+// Bounded wait on an mbarrier phase that also ends when the CTA aborts.
 __device__ __forceinline__ bool consumer_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag,
                                               unsigned *err) {
   if (*abort_flag) return false;
@@ -56,151 +65,42 @@ __device__ __forceinline__ bool consumer_wait(uint32_t bar, uint32_t parity, vol
   return false;
 }
 
-// ---------------------------------------------------------------------------- epilogues
-// red[r * MAXB + b] holds the finished dot product of row rb*RB + r for user b (before the
-// RMSNorm scale inv[b]).  Called by the 256 consumer threads; every thread reaches every
-// barrier.
-template <int B, int EPI>
-__device__ __forceinline__ void epilogue(const GemvParams &p, int rb, const float *red, const float *inv,
-                                         float *scr, int tid) {
-  const int warp = tid >> 5, lane = tid & 31;
-  if constexpr (EPI == EPI_STORE) {
-    if (tid < RB * B) {
-      const int b = tid / RB, r = tid % RB, n = rb * RB + r;
-      if (n < p.n_rows) p.out[(size_t)b * p.ldo + n] = red[r * MAXB + b] * inv[b];
-    }
-  } else if constexpr (EPI == EPI_RESID) {
-    float sq = 0.f;
-    if (tid < RB * B) {
-      const int b = tid >> 6, r = tid & 63, n = rb * RB + r;
-      if (n < p.n_rows) {
-        const size_t o = (size_t)b * p.ldh + n;
-        const float hn = __ldcg(p.h + o) + red[r * MAXB + b] * inv[b];
-        p.h[o] = hn;
-        if (p.g_next) p.xn[o] = hn * p.g_next[n];
-        if (p.capture) p.capture[(size_t)b * p.n_rows + n] = hn;
-        sq = hn * hn;
-      }
-    }
+// Wait (one thread, bounded) until a counter written by other CTAs reaches `need`.
+__device__ __forceinline__ bool wait_counter(const unsigned *ctr, unsigned need, volatile int *abort_flag,
+                                             unsigned *err) {
+  for (uint32_t i = 0; i < 64u * WAIT_LIMIT; ++i) {
+    if (ld_acquire_gpu(ctr) >= need) return true;
+    if ((i & 255) == 255 && *abort_flag) return false;
+  }
+  *abort_flag = 1;
+  atomicOr(err, ERR_TIMEOUT);
+  return false;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
-    if (lane == 0) scr[warp] = sq;
-    named_bar_sync(1, CONSUMER_WARPS * 32);
-    if (tid < B) p.sumsq_out[rb * MAXB + tid] = scr[2 * tid] + scr[2 * tid + 1];
-  } else if constexpr (EPI == EPI_SWIGLU) {
-    if (tid < 32 * B) {
-      const int b = tid >> 5, pr = tid & 31, j = rb * (RB / 2) + pr;
-      if (2 * j < p.n_rows) {
-        const float g = red[(2 * pr) * MAXB + b] * inv[b];
-        const float u = red[(2 * pr + 1) * MAXB + b] * inv[b];
-        p.out[(size_t)b * p.ldo + j] = g / (1.0f + expf(-g)) * u;
-      }
-    }
-  } else if constexpr (EPI == EPI_QKV) {
-    if (tid < 32 * B) {
-      const int b = tid >> 5, pr = tid & 31, r0 = rb * RB + 2 * pr;
-      int pos = p.positions[b];
-      const bool ok = pos >= 0 && pos < p.max_ctx;
-      if (!ok) pos = 0;
-      if (r0 < p.n_rows) {
-        const int hd = p.head_dim, half = hd >> 1;
-        const float v1 = red[(2 * pr) * MAXB + b] * inv[b];
-        const float v2 = red[(2 * pr + 1) * MAXB + b] * inv[b];
-        if (r0 < p.n_q_rows + p.n_kv_rows) {
-          const bool is_q = r0 < p.n_q_rows;
-          const int rr = is_q ? r0 : r0 - p.n_q_rows;
-          const int head = rr / hd, i = (rr % hd) >> 1;
-          const size_t ri = (size_t)(p.rope_per_user ? b : pos) * half + i;
-          const float cs = p.rope_cos[ri];
-          const float sn = p.rope_sin[ri];
-          const float a = v1 * cs - v2 * sn;
-          const float c = v2 * cs + v1 * sn;
-          if (is_q) {
-            float *qd = p.q + (size_t)b * p.n_q_rows + head * hd;
-            qd[i] = a;
-            qd[i + half] = c;
-          } else if (ok) {
-            uint16_t *kd = p.kcache + (((size_t)b * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
-            kd[i] = f32_to_bf16_rne(a);
-            kd[i + half] = f32_to_bf16_rne(c);
-          }
-        } else if (ok) {
-          const int rr = r0 - p.n_q_rows - p.n_kv_rows;
-          const int head = rr / hd, j = rr % hd;
-          uint16_t *vd = p.vcache + (((size_t)b * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
-          vd[j] = f32_to_bf16_rne(v1);
-          vd[j + 1] = f32_to_bf16_rne(v2);
-        }
-      }
-    }
-  } else if constexpr (EPI == EPI_ARGMAX) {
-    int *scri = reinterpret_cast<int *>(scr + CONSUMER_WARPS);
-    __shared__ int s_last_am;
-    float v = -INFINITY;
-    int idx = 0x7fffffff;
-    if (tid < RB * B) {
-      const int b = tid >> 6, r = tid & 63, n = rb * RB + r;
-      if (n < p.n_rows) {
-        v = red[r * MAXB + b] * inv[b];
-        idx = n;
-      }
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, v, off);
-      const int oi = __shfl_xor_sync(0xffffffffu, idx, off);
-      if (ov > v || (ov == v && oi < idx)) { v = ov; idx = oi; }
-    }
-    if (lane == 0) { scr[warp] = v; scri[warp] = idx; }
-    named_bar_sync(1, CONSUMER_WARPS * 32);
-    if (tid < B) {
-      float bv = scr[2 * tid];
-      int bi = scri[2 * tid];
-      const float ov = scr[2 * tid + 1];
-      const int oi = scri[2 * tid + 1];
-      if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
-      p.cand_val[rb * MAXB + tid] = bv;
-      p.cand_idx[rb * MAXB + tid] = bi;
-    }
-    named_bar_sync(1, CONSUMER_WARPS * 32);
-    if (tid == 0) {
-      const unsigned prev = atom_add_acq_rel(reinterpret_cast<unsigned *>(p.argmax_ticket), 1u);
-      s_last_am = (prev == (unsigned)(p.n_rb - 1));
-      if (s_last_am) atomicExch(p.argmax_ticket, 0);
-    }
-    named_bar_sync(1, CONSUMER_WARPS * 32);
-    if (s_last_am) {
-      for (int b = 0; b < B; ++b) {
-        float bv = -INFINITY;
-        int bi = 0x7fffffff;
-        for (int r = tid; r < p.n_rb; r += CONSUMER_WARPS * 32) {
-          const float ov = __ldcg(p.cand_val + r * MAXB + b);
-          const int oi = __ldcg(p.cand_idx + r * MAXB + b);
-          if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
-        }
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) {
-          const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
-          const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-          if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
-        }
-        named_bar_sync(1, CONSUMER_WARPS * 32);
-        if (lane == 0) { scr[warp] = bv; scri[warp] = bi; }
-        named_bar_sync(1, CONSUMER_WARPS * 32);
-        if (tid == 0) {
-          bv = scr[0];
-          bi = scri[0];
-          for (int w = 1; w < CONSUMER_WARPS; ++w) {
-            if (scr[w] > bv || (scr[w] == bv && scri[w] < bi)) { bv = scr[w]; bi = scri[w]; }
-          }
-          p.next_ids[b] = (bi == 0x7fffffff) ? 0 : bi;
-        }
-      }
-    }
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  return v;
+}
+
+// (value, index) maximum with the lowest index on ties
+__device__ __forceinline__ void argmax_merge(float &v, int &i, float ov, int oi) {
+  if (ov > v || (ov == v && oi < i)) {
+    v = ov;
+    i = oi;
   }
 }
 
+__device__ __forceinline__ void warp_argmax(float &v, int &i) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, v, off);
+    const int oi = __shfl_xor_sync(0xffffffffu, i, off);
+    argmax_merge(v, i, ov, oi);
+  }
+}
 
+// ---------------------------------------------------------------------------- consumers
 // Accumulate one tile (in shared memory at `st`, activations after the weights) into acc.
 template <int B, int FMT>
 __device__ __forceinline__ void tile_compute(const uint8_t *st, int warp, int lane, float (&acc)[B][4][2]) {
@@ -268,178 +168,321 @@ __device__ __forceinline__ void tile_compute(const uint8_t *st, int warp, int la
   }
 }
 
-// RMSNorm scale of the GEMV input (1 without a norm): warp b sums the per-row-block sums of
-// squares of user b's h (lane j takes parts j, j+32, ... in order, then a fixed butterfly), so
-// the loads are independent and the order is the same on every call.  Writes inv[0..B).
-template <int B>
-__device__ __forceinline__ void norm_scale(const GemvParams &p, float *inv, int tid) {
-  const int warp = tid >> 5, lane = tid & 31;
-  if (warp < B) {
-    float v = 1.0f;
-    if (p.sumsq) {
-      float s = 0.f;
-      for (int i = lane; i < p.n_parts; i += 32) s += __ldcg(p.sumsq + i * MAXB + warp);
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-      v = 1.0f / sqrtf(s / static_cast<float>(p.d_norm) + p.eps);
-    }
-    if (lane == 0) inv[warp] = v;
-  }
-}
-
-// End of a row-block segment [seg_kt0, kt] of tile row block rb in CTA c (of G) whose tile range
-// starts at t0: reduce the lanes of each row, combine with the neighbouring CTAs that share the
-// row block (partials + atomic ticket; the last to arrive sums them in CTA order), and run the
-// epilogue once per row block.  All consumer threads call it.
-// Wait (one thread, bounded) until a counter written by other CTAs reaches `need`.
-__device__ __forceinline__ bool wait_counter(const unsigned *ctr, unsigned need, volatile int *abort_flag,
-                                             unsigned *err) {
-  for (uint32_t i = 0; i < 64u * WAIT_LIMIT; ++i) {
-    if (ld_acquire_gpu(ctr) >= need) return true;
-    if ((i & 255) == 255 && *abort_flag) return false;
-  }
-  *abort_flag = 1;
-  atomicOr(err, ERR_TIMEOUT);
-  return false;
-}
-
-template <int B, int EPI>
-__device__ __forceinline__ void segment_end(const GemvParams &p, int rb, int kt, int seg_kt0, long long t0,
-                                            long long T, int G, int c, float (&acc)[B][4][2], float *red,
-                                            float *scr, float *inv, int *inv_ready, int *s_last,
-                                            volatile int *abort_flag, int tid) {
-  const int warp = tid >> 5, lane = tid & 31, kc = lane & 15, rsub = lane >> 4;
-  float tot[B][4];
-#pragma unroll
-  for (int b = 0; b < B; ++b)
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      float v = acc[b][j][0] + acc[b][j][1];
-      v += __shfl_xor_sync(0xffffffffu, v, 8);
-      v += __shfl_xor_sync(0xffffffffu, v, 4);
-      v += __shfl_xor_sync(0xffffffffu, v, 2);
-      v += __shfl_xor_sync(0xffffffffu, v, 1);
-      tot[b][j] = v;
-    }
-  if (kc == 0) {
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-#pragma unroll
-      for (int b = 0; b < B; ++b) red[(warp * 8 + rsub + 2 * j) * MAXB + b] = tot[b][j];
-  }
-  consumer_sync();
-  bool do_epi = true;
-  if (!(seg_kt0 == 0 && kt == p.n_kt - 1)) {
-    // this row block is shared with neighbouring CTAs
-    const int first_rb = static_cast<int>(t0 / p.n_kt);
-    const int slot = (rb == first_rb) ? 0 : 1;
-    float *mine = p.partial + (size_t)(c * 2 + slot) * (RB * MAXB);
-    for (int e = tid; e < RB * MAXB; e += CONSUMER_THREADS) mine[e] = red[e];
-    consumer_sync();
-    const int c_lo = cta_of_tile((long long)rb * p.n_kt, T, G);
-    const int c_hi = cta_of_tile((long long)(rb + 1) * p.n_kt - 1, T, G);
-    if (tid == 0) {
-      // release this CTA's partials; the last to arrive acquires everyone's
-      const unsigned prev = atom_add_acq_rel(reinterpret_cast<unsigned *>(p.tickets + rb), 1u);
-      *s_last = (prev == (unsigned)(c_hi - c_lo));
-      if (*s_last) atomicExch(p.tickets + rb, 0);
-    }
-    consumer_sync();
-    do_epi = *s_last != 0;
-    if (do_epi) {
-      // issue every partial's load first (independent), then add them in CTA order
-      constexpr int MAXPART = 8;
-      for (int e = tid; e < RB * MAXB; e += CONSUMER_THREADS) {
-        float sum = 0.f;
-        for (int c0 = c_lo; c0 <= c_hi; c0 += MAXPART) {
-          float v[MAXPART];
-#pragma unroll
-          for (int j = 0; j < MAXPART; ++j) {
-            const int cc = c0 + j;
-            v[j] = 0.f;
-            if (cc <= c_hi) {
-              const int frb = static_cast<int>(((long long)cc * T / G) / p.n_kt);
-              const int sl = (rb == frb) ? 0 : 1;
-              v[j] = __ldcg(p.partial + (size_t)(cc * 2 + sl) * (RB * MAXB) + e);
-            }
-          }
-#pragma unroll
-          for (int j = 0; j < MAXPART; ++j)
-            if (c0 + j <= c_hi) sum += v[j];
-        }
-        red[e] = sum;
-      }
-      consumer_sync();
-    }
-  }
-  if (do_epi && !*inv_ready) {
-    // the RMSNorm scale needs every row block of h: in the persistent kernel wait for the
-    // phase that produces h to complete them
-    if (tid == 0 && p.norm_done) wait_counter(p.norm_done, (unsigned)p.norm_need, abort_flag, p.err);
-    consumer_sync();
-    norm_scale<B>(p, inv, tid);
-    consumer_sync();
-    if (tid == 0) *inv_ready = 1;
-  }
-  if (do_epi) epilogue<B, EPI>(p, rb, red, inv, scr, tid);
-  consumer_sync();
-  if (do_epi && tid == 0) {
-    // publish this row block (the bar.sync above ordered every consumer's stores before it)
-    if (p.out_ready) {
-      int idx;
-      if constexpr (EPI == EPI_QKV) {
-        const int r0 = rb * RB, hd = p.head_dim;
-        const int group = p.n_q_rows / p.n_kv_rows;
-        if (r0 < p.n_q_rows)
-          idx = (r0 / hd) / group;
-        else if (r0 < p.n_q_rows + p.n_kv_rows)
-          idx = (r0 - p.n_q_rows) / hd;
-        else
-          idx = (r0 - p.n_q_rows - p.n_kv_rows) / hd;
-      } else {
-        idx = (rb * p.out_unit) / p.out_kt;
-      }
-      red_add_release(p.out_ready + idx, 1u);
-    }
-    if (p.out_done) red_add_release(p.out_done, 1u);
-  }
-}
+// Staging ring between the consumer warps and the epilogue warp.
+struct SegRing {
+  float *red;      // [NSLOT][RB][MAXB]
+  uint64_t *full;  // [NSLOT], count CONSUMER_WARPS
+  uint64_t *empty; // [NSLOT], count 1
+};
 
 // Consumer side of one GEMV over this CTA's tile range [t0, t0 + n): wait for each tile's ring
-// stage, accumulate, release the stage, finish segments.  (s, phase) is the ring position,
-// carried across calls when consecutive GEMVs share one ring.
-template <int B, int EPI, int FMT>
-__device__ __forceinline__ void gemv_consume(const GemvParams &p, uint8_t *ring, uint64_t *full, uint64_t *empty,
-                                             int S, int &s, uint32_t &phase, long long t0, int n, long long T,
-                                             int G, int c, float *red, float *scr, float *inv, int *inv_ready,
-                                             int *s_last, volatile int *abort_flag, int tid) {
-  const int warp = tid >> 5, lane = tid & 31;
+// stage, accumulate, release the stage; at each segment end reduce the rows of this warp into the
+// next staging slot.  (s, phase) is the ring position and segc the staging count, both carried
+// across calls when consecutive GEMVs share the rings.
+template <int B, int FMT>
+__device__ __forceinline__ void gemv_consume(int n_kt, uint8_t *ring, uint64_t *full, uint64_t *empty, int S, int &s,
+                                             uint32_t &phase, long long t0, int n, const SegRing &sr, int &segc,
+                                             volatile int *abort_flag, unsigned *err, int tid) {
+  const int warp = tid >> 5, lane = tid & 31, kc = lane & 15, rsub = lane >> 4;
   float acc[B][4][2];
-  int seg_kt0 = 0;
-  int rb = static_cast<int>(t0 / p.n_kt);
-  int kt = static_cast<int>(t0 - (long long)rb * p.n_kt);
+  int kt = static_cast<int>(t0 % n_kt);
   for (int i = 0; i < n; ++i) {
     if (i == 0 || kt == 0) {
 #pragma unroll
       for (int b = 0; b < B; ++b)
 #pragma unroll
         for (int j = 0; j < 4; ++j) acc[b][j][0] = acc[b][j][1] = 0.f;
-      seg_kt0 = kt;
     }
-    consumer_wait(smem_addr(&full[s]), phase, abort_flag, p.err);
+    consumer_wait(smem_addr(&full[s]), phase, abort_flag, err);
     tile_compute<B, FMT>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc);
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_addr(&empty[s]));
-    if (kt == p.n_kt - 1 || i == n - 1)
-      segment_end<B, EPI>(p, rb, kt, seg_kt0, t0, T, G, c, acc, red, scr, inv, inv_ready, s_last, abort_flag, tid);
-    if (++kt == p.n_kt) {
-      kt = 0;
-      ++rb;
+    if (kt == n_kt - 1 || i == n - 1) {
+      float tot[B][4];
+#pragma unroll
+      for (int b = 0; b < B; ++b)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          float v = acc[b][j][0] + acc[b][j][1];
+          v += __shfl_xor_sync(0xffffffffu, v, 8);
+          v += __shfl_xor_sync(0xffffffffu, v, 4);
+          v += __shfl_xor_sync(0xffffffffu, v, 2);
+          v += __shfl_xor_sync(0xffffffffu, v, 1);
+          tot[b][j] = v;
+        }
+      const int slot = segc % NSLOT, use = segc / NSLOT;
+      if (use > 0) consumer_wait(smem_addr(&sr.empty[slot]), (use - 1) & 1, abort_flag, err);
+      if (kc == 0) {
+        float *rd = sr.red + slot * RB * MAXB;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+#pragma unroll
+          for (int b = 0; b < B; ++b) rd[(warp * 8 + rsub + 2 * j) * MAXB + b] = tot[b][j];
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_addr(&sr.full[slot]));
+      ++segc;
     }
+    if (++kt == n_kt) kt = 0;
     if (++s == S) {
       s = 0;
       phase ^= 1u;
     }
+  }
+}
+
+// ---------------------------------------------------------------------------- epilogue warp
+// RMSNorm scale of the GEMV input (1 without a norm): user b's scale from the per-row-block sums
+// of squares of h, the lanes taking parts j, j+32, ... in order, then a fixed butterfly, so the
+// result is the same on every call.
+template <int B>
+__device__ __forceinline__ void norm_scale_warp(const GemvParams &p, float *inv, int lane) {
+#pragma unroll
+  for (int b = 0; b < B; ++b) {
+    float v = 1.0f;
+    if (p.sumsq) {
+      float s = 0.f;
+      for (int i = lane; i < p.n_parts; i += 32) s += __ldcg(p.sumsq + i * MAXB + b);
+      s = warp_sum(s);
+      v = 1.0f / sqrtf(s / static_cast<float>(p.d_norm) + p.eps);
+    }
+    inv[b] = v;
+  }
+}
+
+// The fused epilogue of row block rb: red[r * MAXB + b] is the dot product of row rb*RB + r for
+// user b, before the RMSNorm scale inv[b].  One warp.
+template <int B, int EPI>
+__device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const float *red, const float *inv,
+                                              int lane) {
+  if constexpr (EPI == EPI_STORE) {
+    for (int e = lane; e < RB * B; e += 32) {
+      const int b = e / RB, r = e % RB, n = rb * RB + r;
+      if (n < p.n_rows) p.out[(size_t)b * p.ldo + n] = red[r * MAXB + b] * inv[b];
+    }
+  } else if constexpr (EPI == EPI_RESID) {
+#pragma unroll
+    for (int b = 0; b < B; ++b) {
+      float sq = 0.f;
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+        const int r = lane + 32 * h2, n = rb * RB + r;
+        if (n < p.n_rows) {
+          const size_t o = (size_t)b * p.ldh + n;
+          const float hn = __ldcg(p.h + o) + red[r * MAXB + b] * inv[b];
+          p.h[o] = hn;
+          if (p.g_next) p.xn[o] = hn * p.g_next[n];
+          if (p.capture) p.capture[(size_t)b * p.n_rows + n] = hn;
+          sq = fmaf(hn, hn, sq);
+        }
+      }
+      sq = warp_sum(sq);
+      if (lane == 0) p.sumsq_out[rb * MAXB + b] = sq;
+    }
+  } else if constexpr (EPI == EPI_SWIGLU) {
+    for (int e = lane; e < (RB / 2) * B; e += 32) {
+      const int b = e / (RB / 2), pr = e % (RB / 2), j = rb * (RB / 2) + pr;
+      if (2 * j < p.n_rows) {
+        const float g = red[(2 * pr) * MAXB + b] * inv[b];
+        const float u = red[(2 * pr + 1) * MAXB + b] * inv[b];
+        p.out[(size_t)b * p.ldo + j] = g / (1.0f + expf(-g)) * u;
+      }
+    }
+  } else if constexpr (EPI == EPI_QKV) {
+    const int hd = p.head_dim, half = hd >> 1;
+    for (int e = lane; e < (RB / 2) * B; e += 32) {
+      const int b = e / (RB / 2), pr = e % (RB / 2), r0 = rb * RB + 2 * pr;
+      int pos = p.positions[b];
+      const bool ok = pos >= 0 && pos < p.max_ctx;
+      if (!ok) pos = 0;
+      if (r0 >= p.n_rows) continue;
+      const float v1 = red[(2 * pr) * MAXB + b] * inv[b];
+      const float v2 = red[(2 * pr + 1) * MAXB + b] * inv[b];
+      if (r0 < p.n_q_rows + p.n_kv_rows) {
+        const bool is_q = r0 < p.n_q_rows;
+        const int rr = is_q ? r0 : r0 - p.n_q_rows;
+        const int head = rr / hd, i = (rr % hd) >> 1;
+        const size_t ri = (size_t)(p.rope_per_user ? b : pos) * half + i;
+        const float cs = p.rope_cos[ri];
+        const float sn = p.rope_sin[ri];
+        const float a = v1 * cs - v2 * sn;
+        const float c2 = v2 * cs + v1 * sn;
+        if (is_q) {
+          float *qd = p.q + (size_t)b * p.n_q_rows + head * hd;
+          qd[i] = a;
+          qd[i + half] = c2;
+        } else if (ok) {
+          uint16_t *kd = p.kcache + (((size_t)b * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
+          kd[i] = f32_to_bf16_rne(a);
+          kd[i + half] = f32_to_bf16_rne(c2);
+        }
+      } else if (ok) {
+        const int rr = r0 - p.n_q_rows - p.n_kv_rows;
+        const int head = rr / hd, j = rr % hd;
+        uint16_t *vd = p.vcache + (((size_t)b * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
+        vd[j] = f32_to_bf16_rne(v1);
+        vd[j + 1] = f32_to_bf16_rne(v2);
+      }
+    }
+  } else if constexpr (EPI == EPI_ARGMAX) {
+    // per row block: each user's best row; the last row block to finish (global ticket) reduces
+    // the candidates of all row blocks
+#pragma unroll
+    for (int b = 0; b < B; ++b) {
+      float v = -INFINITY;
+      int idx = 0x7fffffff;
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+        const int r = lane + 32 * h2, n = rb * RB + r;
+        if (n < p.n_rows) argmax_merge(v, idx, red[r * MAXB + b] * inv[b], n);
+      }
+      warp_argmax(v, idx);
+      if (lane == 0) {
+        p.cand_val[rb * MAXB + b] = v;
+        p.cand_idx[rb * MAXB + b] = idx;
+      }
+    }
+    __syncwarp();
+    unsigned prev = 0;
+    if (lane == 0) prev = atom_add_acq_rel(reinterpret_cast<unsigned *>(p.argmax_ticket), 1u);
+    prev = __shfl_sync(0xffffffffu, prev, 0);
+    if (prev == (unsigned)(p.n_rb - 1)) {
+      if (lane == 0) atomicExch(p.argmax_ticket, 0);
+      __syncwarp();
+#pragma unroll
+      for (int b = 0; b < B; ++b) {
+        float bv = -INFINITY;
+        int bi = 0x7fffffff;
+        for (int r = lane; r < p.n_rb; r += 32)
+          argmax_merge(bv, bi, __ldcg(p.cand_val + r * MAXB + b), __ldcg(p.cand_idx + r * MAXB + b));
+        warp_argmax(bv, bi);
+        if (lane == 0) p.next_ids[b] = (bi == 0x7fffffff) ? 0 : bi;
+      }
+    }
+  }
+}
+
+// Epilogue warp side of one GEMV over this CTA's tile range [t0, t0 + n): takes the staged
+// segments in order; a row block shared with neighbouring CTAs is combined (partials in global
+// memory, atomic ticket, the last to arrive sums them in CTA order); each finished row block gets
+// its epilogue and (persistent kernel) is published on the readiness counters.
+// inv / inv_ready: the RMSNorm scale of this GEMV, computed once, when first needed.
+template <int B, int EPI>
+__device__ __forceinline__ void gemv_epilogues(const GemvParams &p, long long t0, int n, long long T, int G, int c,
+                                               const SegRing &sr, int &segc, float *inv, bool &inv_ready,
+                                               volatile int *abort_flag, int lane) {
+  int i = 0;
+  while (i < n) {
+    const long long t = t0 + i;
+    const int rb = static_cast<int>(t / p.n_kt);
+    const int kt0 = static_cast<int>(t - (long long)rb * p.n_kt);
+    const int len = min(p.n_kt - kt0, n - i);
+    i += len;
+    const int slot = segc % NSLOT, use = segc / NSLOT;
+    ++segc;
+    consumer_wait(smem_addr(&sr.full[slot]), use & 1, abort_flag, p.err);
+    float *red = sr.red + slot * RB * MAXB;
+    bool do_epi = true;
+    if (!(kt0 == 0 && len == p.n_kt)) {
+      // this row block is shared with neighbouring CTAs
+      const int first_rb = static_cast<int>(t0 / p.n_kt);
+      const int myslot = (rb == first_rb) ? 0 : 1;
+      float4 *mine = reinterpret_cast<float4 *>(p.partial + (size_t)(c * 2 + myslot) * (RB * MAXB));
+      const float4 *r4 = reinterpret_cast<const float4 *>(red);
+      for (int e = lane; e < RB * MAXB / 4; e += 32) mine[e] = r4[e];
+      __syncwarp();
+      const int c_lo = cta_of_tile((long long)rb * p.n_kt, T, G);
+      const int c_hi = cta_of_tile((long long)(rb + 1) * p.n_kt - 1, T, G);
+      unsigned prev = 0;
+      if (lane == 0) {
+        // release this CTA's partials; the last to arrive acquires everyone's
+        prev = atom_add_acq_rel(reinterpret_cast<unsigned *>(p.tickets + rb), 1u);
+        if (prev == (unsigned)(c_hi - c_lo)) atomicExch(p.tickets + rb, 0);
+      }
+      prev = __shfl_sync(0xffffffffu, prev, 0);
+      __syncwarp();
+      do_epi = prev == (unsigned)(c_hi - c_lo);
+      if (do_epi) {
+        // every partial's loads first (independent), then the sums in CTA order
+        for (int e = lane; e < RB * MAXB / 4; e += 32) {
+          float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+          for (int c0 = c_lo; c0 <= c_hi; c0 += 4) {
+            float4 v[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const int cc = c0 + j;
+              v[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+              if (cc <= c_hi) {
+                const int frb = static_cast<int>(((long long)cc * T / G) / p.n_kt);
+                const int sl = (rb == frb) ? 0 : 1;
+                v[j] = __ldcg(reinterpret_cast<const float4 *>(p.partial + (size_t)(cc * 2 + sl) * (RB * MAXB)) + e);
+              }
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              if (c0 + j <= c_hi) {
+                sum.x += v[j].x;
+                sum.y += v[j].y;
+                sum.z += v[j].z;
+                sum.w += v[j].w;
+              }
+          }
+          reinterpret_cast<float4 *>(red)[e] = sum;
+        }
+        __syncwarp();
+      }
+    }
+    if (do_epi) {
+      if (!inv_ready) {
+        // the RMSNorm scale needs every row block of h: in the persistent kernel wait for the
+        // phase that produces h to complete them
+        if (lane == 0 && p.norm_done) wait_counter(p.norm_done, (unsigned)p.norm_need, abort_flag, p.err);
+        __syncwarp();
+        norm_scale_warp<B>(p, inv, lane);
+        inv_ready = true;
+      }
+      epilogue_warp<B, EPI>(p, rb, red, inv, lane);
+      __syncwarp();
+      if (lane == 0) {
+        // publish this row block (the __syncwarp above ordered every lane's stores before it)
+        if (p.out_ready) {
+          int idx;
+          if constexpr (EPI == EPI_QKV) {
+            const int r0 = rb * RB, hd = p.head_dim;
+            const int group = p.n_q_rows / p.n_kv_rows;
+            if (r0 < p.n_q_rows)
+              idx = (r0 / hd) / group;
+            else if (r0 < p.n_q_rows + p.n_kv_rows)
+              idx = (r0 - p.n_q_rows) / hd;
+            else
+              idx = (r0 - p.n_q_rows - p.n_kv_rows) / hd;
+          } else {
+            idx = (rb * p.out_unit) / p.out_kt;
+          }
+          red_add_release(p.out_ready + idx, 1u);
+        }
+        if (p.out_done) red_add_release(p.out_done, 1u);
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_addr(&sr.empty[slot]));
+  }
+}
+
+template <int B>
+__device__ __forceinline__ void gemv_epilogues_any(int epi, const GemvParams &p, long long t0, int n, long long T,
+                                                   int G, int c, const SegRing &sr, int &segc, float *inv,
+                                                   bool &inv_ready, volatile int *abort_flag, int lane) {
+  switch (epi) {
+    case EPI_QKV: gemv_epilogues<B, EPI_QKV>(p, t0, n, T, G, c, sr, segc, inv, inv_ready, abort_flag, lane); break;
+    case EPI_RESID: gemv_epilogues<B, EPI_RESID>(p, t0, n, T, G, c, sr, segc, inv, inv_ready, abort_flag, lane); break;
+    case EPI_SWIGLU:
+      gemv_epilogues<B, EPI_SWIGLU>(p, t0, n, T, G, c, sr, segc, inv, inv_ready, abort_flag, lane);
+      break;
+    case EPI_ARGMAX:
+      gemv_epilogues<B, EPI_ARGMAX>(p, t0, n, T, G, c, sr, segc, inv, inv_ready, abort_flag, lane);
+      break;
+    default: gemv_epilogues<B, EPI_STORE>(p, t0, n, T, G, c, sr, segc, inv, inv_ready, abort_flag, lane); break;
   }
 }
 

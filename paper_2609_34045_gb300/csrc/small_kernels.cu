@@ -12,7 +12,7 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
                                                          int vocab, int d, int ldh, const float *g_next,
                                                          float *h, float *xn, float *sumsq, int *positions,
                                                          int max_ctx, unsigned *err, unsigned *bar) {
-  __shared__ float part[2];
+  __shared__ float vals[64];
   const int b = blockIdx.y, tid = threadIdx.x, r = blockIdx.x * 64 + tid;
   pdl_launch_dependents();
   pdl_wait();
@@ -20,7 +20,7 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
     const int pos = positions_in[b];
     if (pos < 0 || pos >= max_ctx) atomicOr(err, ERR_POSITION);
     positions[b] = pos;
-    // grid-barrier counter and abort flag of the persistent stage kernel that follows
+    // abort flag of the persistent stage kernel that follows
     if (b == 0 && bar) {
       bar[0] = 0u;
       bar[1] = 0u;
@@ -41,12 +41,18 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
     h[(size_t)b * ldh + r] = v;
     if (g_next) xn[(size_t)b * ldh + r] = v * g_next[r];
   }
-  float sq = v * v;
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
-  if ((tid & 31) == 0) part[tid >> 5] = sq;
+  // the block's sum of squares in exactly the order of the residual epilogue (lane l: rows l
+  // and l + 32 by fma, then a butterfly), so that a stage fed this hidden state computes the same
+  // bits as the block before it did
+  vals[tid] = v;
   __syncthreads();
-  if (tid == 0) sumsq[blockIdx.x * MAXB + b] = part[0] + part[1];
+  if (tid < 32) {
+    float sq = fmaf(vals[tid], vals[tid], 0.f);
+    sq = fmaf(vals[tid + 32], vals[tid + 32], sq);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
+    if (tid == 0) sumsq[blockIdx.x * MAXB + b] = sq;
+  }
 }
 
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in, int batch,

@@ -506,6 +506,7 @@ int enqueue_persistent(kfl_stage *st, int batch, cudaStream_t s) {
   kp.rope_cos = st->rope_cos;
   kp.rope_sin = st->rope_sin;
   kp.max_ctx = st->cfg.max_ctx;
+  kp.l2_ahead = env_int("KFL_L2_AHEAD", 32);
   CK(cudaMemsetAsync(st->counters, 0, (size_t)std::max(1, st->n_phases) * st->P.ctr_stride * 4, s));
   CK(launch_stage_kernel(kp, batch, st->cfg.weight_fmt, st->P.n_sm, st->mk_smem[batch], s));
   return KFL_OK;
@@ -809,7 +810,8 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
     const size_t static_smem = 8192;  // the kernel's own __shared__ variables
     size_t smem_max = 0;
     for (int b = 1; b <= cfg->max_batch; ++b) {
-      int stages = env_int("KFL_STAGE_KERNEL_STAGES", MAX_STAGES);
+      // 96-128 KiB of weights in flight per SM streams fastest (deeper rings queue more)
+      int stages = env_int("KFL_STAGE_KERNEL_STAGES", 8);
       if (stages > MAX_STAGES) stages = MAX_STAGES;
       while (stages > 2 && stage_kernel_smem(stages, P.hd, b, cfg->weight_fmt) + static_smem > (size_t)smem_optin)
         --stages;

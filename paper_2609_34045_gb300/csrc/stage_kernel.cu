@@ -25,7 +25,7 @@
 
 namespace kfl {
 
-constexpr int MK_WARPS = CONSUMER_WARPS + 2;
+constexpr int MK_WARPS = CONSUMER_WARPS + 3;  // consumers, weight producer, activation producer, epilogue
 constexpr int MK_THREADS = MK_WARPS * 32;
 
 // Tile range of CTA c in a GEMV phase: stream-K over min(T, grid) CTAs; the rest get none.
@@ -61,30 +61,20 @@ __device__ __forceinline__ bool chunk_ready(const GemvParams &g, int kt) {
   return true;
 }
 
-// Phase bodies as separate (not inlined) functions: each gets its own register allocation, so
-// the widest one does not raise the pressure of the rest of the kernel.
-template <int B, int EPI, int FMT>
-__device__ __noinline__ void gemv_phase_call(const GemvParams &g, uint8_t *ring, uint64_t *full, uint64_t *empty,
-                                             int S, int &s, uint32_t &phase, long long t0, int n, long long T, int G,
-                                             int c, float *red, float *scr, float *inv, int *inv_ready, int *s_last,
-                                             volatile int *abort_flag, int tid) {
-  gemv_consume<B, EPI, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, inv, inv_ready, s_last,
-                            abort_flag, tid);
+// Phase bodies as separate (not inlined) functions get their own register allocation, so the
+// widest one does not raise the pressure of the rest of the kernel.
+template <int B, int FMT>
+__device__ __noinline__ void gemv_consume_call(int n_kt, uint8_t *ring, uint64_t *full, uint64_t *empty, int S,
+                                               int &s, uint32_t &phase, long long t0, int n, const SegRing &sr,
+                                               int &segc, volatile int *abort_flag, unsigned *err, int tid) {
+  gemv_consume<B, FMT>(n_kt, ring, full, empty, S, s, phase, t0, n, sr, segc, abort_flag, err, tid);
 }
 
-// Batches 1-2 inline the loop (shared-memory addressing known to the compiler); wider batches
-// call the out-of-line copy.
-template <int B, int EPI, int FMT>
-__device__ __forceinline__ void gemv_phase(const GemvParams &g, uint8_t *ring, uint64_t *full, uint64_t *empty, int S,
-                                           int &s, uint32_t &phase, long long t0, int n, long long T, int G, int c,
-                                           float *red, float *scr, float *inv, int *inv_ready, int *s_last,
-                                           volatile int *abort_flag, int tid) {
-  if constexpr (B <= 2)
-    gemv_consume<B, EPI, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, inv, inv_ready, s_last,
-                              abort_flag, tid);
-  else
-    gemv_phase_call<B, EPI, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, inv, inv_ready,
-                                 s_last, abort_flag, tid);
+template <int B>
+__device__ __noinline__ void gemv_epilogues_call(int epi, const GemvParams &p, long long t0, int n, long long T, int G,
+                                                 int c, const SegRing &sr, int &segc, float *inv, bool &inv_ready,
+                                                 volatile int *abort_flag, int lane) {
+  gemv_epilogues_any<B>(epi, p, t0, n, T, G, c, sr, segc, inv, inv_ready, abort_flag, lane);
 }
 
 template <int HD>
@@ -128,13 +118,14 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
   uint64_t *full = reinterpret_cast<uint64_t *>(att + kp.attn_bytes);
   uint64_t *empty = full + S;
   uint64_t *armed = empty + S;                        // weight tile issued (for the x producer)
-  float *red = reinterpret_cast<float *>(armed + S);  // [RB][MAXB]
-  float *scr = red + RB * MAXB;                       // 2 * CONSUMER_WARPS words
-  __shared__ GemvParams s_gp;
+  uint64_t *seg_full = armed + S;                     // staged segments (consumers -> epilogue)
+  uint64_t *seg_empty = seg_full + NSLOT;
+  // [NSLOT][RB][MAXB], 128-byte aligned (read as float4)
+  float *red = reinterpret_cast<float *>((reinterpret_cast<uintptr_t>(seg_empty + NSLOT) + 127) & ~uintptr_t(127));
+  __shared__ GemvParams s_egp;  // the epilogue warp's copy of the current GEMV's parameters
   __shared__ AttnParams s_ap;
   __shared__ float s_inv[MAXB];
   __shared__ int s_last;
-  __shared__ int s_inv_ready;
   __shared__ volatile int s_abort;
   __shared__ volatile int s_issued;
   __shared__ int s_pos[MAXB];                           // this step's positions
@@ -144,6 +135,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
   constexpr uint32_t WBYTES = FMT == 0 ? TILE_BYTES : TILE4_BYTES;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int c = blockIdx.x, grid = gridDim.x;
+  const SegRing sr = {red, seg_full, seg_empty};
   auto stamp = [&](int k, int slot) {
     if (kp.trace) kp.trace[((size_t)k * grid + c) * TRACE_SLOTS + slot] = global_ns();
   };
@@ -154,39 +146,122 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
       mbar_init(smem_addr(&empty[s]), CONSUMER_WARPS);
       mbar_init(smem_addr(&armed[s]), 1);
     }
+    for (int s = 0; s < NSLOT; ++s) {
+      mbar_init(smem_addr(&seg_full[s]), CONSUMER_WARPS);
+      mbar_init(smem_addr(&seg_empty[s]), 1);
+    }
     s_abort = 0;
     s_issued = 0;
     fence_mbar_init();
   }
+  {
+    // positions never change during the step: keep them and their RoPE rows in shared memory
+    const int half = kp.head_dim / 2;
+    for (int e = tid; e < B * half; e += MK_THREADS) {
+      const int b = e / half, i = e % half;
+      int pos = kp.positions[b];
+      if (pos < 0 || pos >= kp.max_ctx) pos = 0;
+      s_cos[e] = kp.rope_cos[(size_t)pos * half + i];
+      s_sin[e] = kp.rope_sin[(size_t)pos * half + i];
+    }
+    if (tid < MAXB) s_pos[tid] = tid < B ? kp.positions[tid] : 0;
+  }
   __syncthreads();
 
+  if (warp == CONSUMER_WARPS + 2) {
+    // ------------------------------------------------------------- epilogue warp
+    int segc = 0;
+    for (int k = 0; k < kp.n_phases && !s_abort; ++k) {
+      const Phase *ph = kp.phases + k;
+      if (ph->kind != PH_GEMV) continue;
+      long long T, t0;
+      int G, n;
+      phase_range(ph->g, c, grid, T, G, t0, n);
+      if (n == 0) continue;
+      if (lane == 0) {
+        s_egp = ph->g;
+        s_egp.positions = s_pos;
+        if (s_egp.rope_cos) {
+          s_egp.rope_cos = s_cos;
+          s_egp.rope_sin = s_sin;
+          s_egp.rope_per_user = 1;
+        }
+      }
+      __syncwarp();
+      bool inv_ready = false;
+      gemv_epilogues_call<B>(ph->epi, s_egp, t0, n, T, G, c, sr, segc, s_inv, inv_ready, &s_abort, lane);
+      __syncwarp();
+      if (lane == 0) stamp(k, TR_CONS_DONE);
+    }
+    return;
+  }
   if (warp == CONSUMER_WARPS) {
     // ---------------------------------------------------------- weight producer
+    // Two cursors over this CTA's weight tiles of every GEMV phase, in order: the ring cursor
+    // loads a tile into a free stage; the L2 cursor, l2_ahead tiles in front of it, prefetches
+    // tiles into L2, so HBM keeps streaming while the consumers wait on data (phase tails,
+    // attention) and the ring loads then hit L2.
     if (lane == 0) {
-      const uint64_t pol = policy_evict_first();
+      const uint64_t pol_ring = policy_evict_first();
+      const uint64_t pol_l2 = policy_evict_normal();
       const uint32_t bytes = WBYTES + B * (KTILE * 4);
-      int s = 0, round = 0, gi = 0;
-      for (int k = 0; k < kp.n_phases && !s_abort; ++k) {
-        const Phase *ph = kp.phases + k;
-        if (ph->kind != PH_GEMV) continue;
-        long long T, t0;
-        int G, n;
-        phase_range(ph->g, c, grid, T, G, t0, n);
-        const uint8_t *w = ph->g.w;
-        if (n > 0) stamp(k, TR_W_FIRST);
-        for (int i = 0; i < n; ++i) {
-          if (round > 0 && !consumer_wait(smem_addr(&empty[s]), (round & 1) ^ 1, &s_abort, kp.err)) break;
-          const uint32_t fb = smem_addr(&full[s]);
-          mbar_arrive_expect_tx(fb, bytes);
-          bulk_g2s(smem_addr(ring + (size_t)s * SB), w + (size_t)(t0 + i) * WBYTES, WBYTES, fb, pol);
-          mbar_arrive(smem_addr(&armed[s]));
-          s_issued = ++gi;
-          if (++s == S) {
-            s = 0;
-            ++round;
-          }
+      struct Cursor {
+        int k, i, n;
+        long long t0;
+        const uint8_t *w;
+      };
+      auto seek = [&](Cursor &cu, int from) {
+        for (int k = from; k < kp.n_phases; ++k) {
+          const Phase *ph = kp.phases + k;
+          if (ph->kind != PH_GEMV) continue;
+          long long T, t0;
+          int G, n;
+          phase_range(ph->g, c, grid, T, G, t0, n);
+          if (n == 0) continue;
+          cu.k = k;
+          cu.i = 0;
+          cu.n = n;
+          cu.t0 = t0;
+          cu.w = ph->g.w;
+          return;
         }
-        if (n > 0) stamp(k, TR_W_LAST);
+        cu.k = kp.n_phases;
+      };
+      Cursor cr, cp;
+      seek(cr, 0);
+      cp = cr;
+      int ahead = 0;  // tiles the L2 cursor is in front of the ring cursor
+      auto prefetch_up_to = [&](int want) {
+        while (ahead < want && cp.k < kp.n_phases) {
+          bulk_prefetch_l2(cp.w + (size_t)(cp.t0 + cp.i) * WBYTES, WBYTES, pol_l2);
+          ++ahead;
+          if (++cp.i == cp.n) seek(cp, cp.k + 1);
+        }
+      };
+      prefetch_up_to(kp.l2_ahead);
+      int s = 0, round = 0, gi = 0;
+      int last_k = -1;
+      while (cr.k < kp.n_phases && !s_abort) {
+        if (cr.k != last_k) {
+          stamp(cr.k, TR_W_FIRST);
+          last_k = cr.k;
+        }
+        if (round > 0 && !consumer_wait(smem_addr(&empty[s]), (round & 1) ^ 1, &s_abort, kp.err)) break;
+        const uint32_t fb = smem_addr(&full[s]);
+        mbar_arrive_expect_tx(fb, bytes);
+        bulk_g2s(smem_addr(ring + (size_t)s * SB), cr.w + (size_t)(cr.t0 + cr.i) * WBYTES, WBYTES, fb, pol_ring);
+        mbar_arrive(smem_addr(&armed[s]));
+        s_issued = ++gi;
+        if (++s == S) {
+          s = 0;
+          ++round;
+        }
+        if (ahead > 0) --ahead;
+        if (++cr.i == cr.n) {
+          stamp(cr.k, TR_W_LAST);
+          seek(cr, cr.k + 1);
+        }
+        prefetch_up_to(kp.l2_ahead);
       }
     }
     return;
@@ -267,70 +342,28 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
   }
 
   // ------------------------------------------------------------------- consumers
-  {
-    // positions never change during the step: keep them and their RoPE rows in shared memory
-    const int half = kp.head_dim / 2;
-    for (int e = tid; e < B * half; e += CONSUMER_THREADS) {
-      const int b = e / half, i = e % half;
-      int pos = kp.positions[b];
-      if (pos < 0 || pos >= kp.max_ctx) pos = 0;
-      s_cos[e] = kp.rope_cos[(size_t)pos * half + i];
-      s_sin[e] = kp.rope_sin[(size_t)pos * half + i];
-    }
-    if (tid < MAXB) s_pos[tid] = tid < B ? kp.positions[tid] : 0;
-  }
-  int s = 0;
+  int s = 0, segc = 0;
   uint32_t phase = 0;
   for (int k = 0; k < kp.n_phases; ++k) {
     const Phase *ph = kp.phases + k;
     const int kind = ph->kind;
-    if (tid == 0) {
-      stamp(k, TR_CONS_ENTER);
-      // the phase table is read-only: this phase's parameters, with the step constants in smem
-      if (kind == PH_GEMV) {
-        s_gp = ph->g;
-        s_gp.positions = s_pos;
-        if (s_gp.rope_cos) {
-          s_gp.rope_cos = s_cos;
-          s_gp.rope_sin = s_sin;
-          s_gp.rope_per_user = 1;
-        }
-        s_inv_ready = 0;
-      } else {
+    if (kind == PH_GEMV) {
+      long long T, t0;
+      int G, n;
+      phase_range(ph->g, c, grid, T, G, t0, n);
+      if (tid == 0) stamp(k, TR_CONS_GO);
+      if (B <= 2)
+        gemv_consume<B, FMT>(ph->g.n_kt, ring, full, empty, S, s, phase, t0, n, sr, segc, &s_abort, kp.err, tid);
+      else
+        gemv_consume_call<B, FMT>(ph->g.n_kt, ring, full, empty, S, s, phase, t0, n, sr, segc, &s_abort, kp.err,
+                                  tid);
+    } else {
+      if (tid == 0) {
+        stamp(k, TR_CONS_ENTER);
         s_ap = ph->a;
         s_ap.positions = s_pos;
       }
-    }
-    consumer_sync();
-    if (kind == PH_GEMV) {
-      const GemvParams &g = s_gp;
-      long long T, t0;
-      int G, n;
-      phase_range(g, c, grid, T, G, t0, n);
-      if (tid == 0) stamp(k, TR_CONS_GO);
-      switch (ph->epi) {
-        case EPI_QKV:
-          gemv_phase<B, EPI_QKV, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv,
-                                      &s_inv_ready, &s_last, &s_abort, tid);
-          break;
-        case EPI_RESID:
-          gemv_phase<B, EPI_RESID, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv,
-                                        &s_inv_ready, &s_last, &s_abort, tid);
-          break;
-        case EPI_SWIGLU:
-          gemv_phase<B, EPI_SWIGLU, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv,
-                                         &s_inv_ready, &s_last, &s_abort, tid);
-          break;
-        case EPI_ARGMAX:
-          gemv_phase<B, EPI_ARGMAX, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv,
-                                         &s_inv_ready, &s_last, &s_abort, tid);
-          break;
-        default:
-          gemv_phase<B, EPI_STORE, FMT>(g, ring, full, empty, S, s, phase, t0, n, T, G, c, red, scr, s_inv,
-                                        &s_inv_ready, &s_last, &s_abort, tid);
-          break;
-      }
-    } else {
+      consumer_sync();
       const AttnParams &a = s_ap;
       const int nc0 = attn_chunks(a, 0);
       const int nc1 = a.batch > 1 ? attn_chunks(a, 1) : 0;
@@ -357,10 +390,12 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
           attn_phase_unit<64>(a, b, kvh, ch, ncb, att, &s_last, tid, 1);
         consumer_sync();
       }
+      if (tid == 0) stamp(k, TR_CONS_DONE);
+      consumer_sync();
     }
-    if (tid == 0) stamp(k, TR_CONS_DONE);
   }
 
+  consumer_sync();
   if (s_abort && tid == 0) {
     // drain copies still in flight before the CTA's shared memory goes away (bounded)
     const int issued = s_issued;
@@ -371,7 +406,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
 // ------------------------------------------------------------------------------- launch
 size_t stage_kernel_smem(int stages, int head_dim, int batch, int fmt) {
   return (size_t)stages * stage_bytes(batch, fmt) + stage_kernel_attn_bytes(head_dim) +
-         3 * stages * sizeof(uint64_t) + (RB * MAXB + 2 * CONSUMER_WARPS) * sizeof(float);
+         (3 * stages + 2 * NSLOT) * sizeof(uint64_t) + NSLOT * RB * MAXB * sizeof(float);
 }
 
 int stage_kernel_attn_bytes(int head_dim) {
