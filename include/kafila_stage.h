@@ -201,6 +201,29 @@ const char *kfl_strerror(int code);
  * and its error string), or "" if none.  The pointer stays valid until the next failing call. */
 const char *kfl_last_error_detail(void);
 
+/* Greedy next token from a head's final hidden state WITHOUT allocating any device memory: the
+ * final RMSNorm, the lm_head product and the argmax of a KFL_LOGITS_OUT stage, as one kernel on
+ * the caller's buffers.  The paper has no counterpart; this is for callers that cannot call
+ * cudaMalloc, such as a host whose device memory is all held by its own pool or allocator, or
+ * an embedding that forbids allocation from extension code, and that keep their lm_head
+ * themselves.  Enqueued on cuda_stream (a cudaStream_t; NULL = the legacy default stream);
+ * returns without waiting.
+ *   hidden     device fp32[batch][d_model], 16-byte aligned: the stage output before the norm
+ *   final_norm device bf16[d_model], 16-byte aligned: the final RMSNorm gain
+ *   lm_head    device bf16[vocab][d_model], row-major, 16-byte aligned (not a stage's tiles)
+ *   next_ids   device int32[batch]: the lowest index among the largest logits of each user
+ * Limits (the size of its static scratch): 1 <= batch <= 4, d_model a multiple of 8 up to
+ * 16384, vocab up to 262144; larger sizes return KFL_ERR_RANGE with the limits in
+ * kfl_last_error_detail.  Its scratch is one fixed array of 131,328 bytes of device memory per
+ * GPU that loads this library, held until the process exits.  The first call on a device looks
+ * the array up and clears its ticket with a synchronous cudaMemset, so make that first call
+ * before any stream capture.  Every call on a device shares the array and leaves its contents
+ * behind; calls that overlap on the GPU (other streams, no ordering) race and give wrong ids.
+ * Errors: KFL_ERR_ARG (NULL, misaligned or rms_eps <= 0), KFL_ERR_RANGE, KFL_ERR_CUDA. */
+int kfl_head_argmax_noalloc(const float *hidden, const uint16_t *final_norm, const uint16_t *lm_head,
+                            int batch, int d_model, int vocab, float rms_eps, int32_t *next_ids,
+                            void *cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -1134,6 +1134,12 @@ extern "C" void kfl_stage_destroy(kfl_stage *st) {
 
 extern "C" const char *kfl_last_error_detail(void) { return g_last_error; }
 
+namespace kfl {
+// Lets other translation units of the library (the allocation-free entry point) set the text
+// that kfl_last_error_detail returns.
+void set_error_detail(const char *msg) { snprintf(g_last_error, sizeof(g_last_error), "%s", msg); }
+}  // namespace kfl
+
 extern "C" const char *kfl_strerror(int code) {
   switch (code) {
     case KFL_OK: return "ok";

@@ -85,6 +85,7 @@ def lib() -> C.CDLL:
             "kfl_stage_destroy": ([vp], None),
             "kfl_strerror": ([i], C.c_char_p),
             "kfl_last_error_detail": ([], C.c_char_p),
+            "kfl_head_argmax_noalloc": ([vp, vp, vp, i, i, i, C.c_float, vp, vp], i),
             "kfl_synth_key": ([C.c_uint64, C.c_uint64], C.c_uint64),
             "kfl_synth_fill": ([vp, C.c_int64, C.c_uint64, C.c_uint64, i, C.c_float, C.c_float, C.c_int64, vp], i),
         }
@@ -270,6 +271,18 @@ def kfl_stage_destroy(st: Stage) -> None:
     if st.handle:
         lib().kfl_stage_destroy(st.handle)
         st.handle = None
+
+
+def kfl_head_argmax_noalloc(hidden, final_norm, lm_head, batch: int, d_model: int, vocab: int, rms_eps: float,
+                            next_ids, stream=None) -> None:
+    """Greedy ids from device buffers without any device allocation (for callers that cannot
+    allocate).  hidden fp32 [batch][d_model], final_norm bf16 [d_model], lm_head bf16
+    [vocab][d_model] row-major, next_ids int32 [batch]; all device memory.  Enqueued on
+    ``stream`` (an int handle or None); the library's static scratch is shared by every call."""
+    rc = lib().kfl_head_argmax_noalloc(_ptr(hidden), _ptr(final_norm), _ptr(lm_head), batch, d_model, vocab,
+                                       rms_eps, _ptr(next_ids), _ptr(stream))
+    if rc < 0:
+        raise RuntimeError(f"kfl_head_argmax_noalloc: {kfl_strerror(rc)} ({rc}): {kfl_last_error_detail()}")
 
 
 def kfl_synth_key(seed: int, tag: int) -> int:
