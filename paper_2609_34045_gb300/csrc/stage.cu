@@ -506,7 +506,7 @@ int enqueue_persistent(kfl_stage *st, int batch, cudaStream_t s) {
   kp.rope_cos = st->rope_cos;
   kp.rope_sin = st->rope_sin;
   kp.max_ctx = st->cfg.max_ctx;
-  kp.l2_ahead = env_int("KFL_L2_AHEAD", 32);
+  kp.l2_ahead = env_int("KFL_L2_AHEAD", 0);
   CK(cudaMemsetAsync(st->counters, 0, (size_t)std::max(1, st->n_phases) * st->P.ctr_stride * 4, s));
   CK(launch_stage_kernel(kp, batch, st->cfg.weight_fmt, st->P.n_sm, st->mk_smem[batch], s));
   return KFL_OK;
