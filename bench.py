@@ -339,11 +339,13 @@ def run_ours(args, work):
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": False, "scaling": "weak",
-            "vs_baseline": None, "dtype": "bf16 weights, fp32 accumulate", "data": "synthetic (seeded)",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded)",
             "config": {"workload": work.name, "stage_layers": [work.l0, work.l1], "batch": b,
                        "ctx": list(work.contexts), "weights": m.weight_fmt,
                        "l2": "inputs larger than L2 (weights streamed once per step)",
-                       "parallelism": f"replicas x{world}"},
+                       "parallelism": f"replicas x{world}",
+                       "execution": ("persistent stage kernel" if launches == 3 * args.steps
+                                     else "one kernel per phase, CUDA graph + programmatic dependent launch")},
             "tokens_per_s": b * world / (ms * 1e-3),
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "peak_kind": f"{peak_kind} copy (MEASURED_PEAKS.json hbm_gbs)",

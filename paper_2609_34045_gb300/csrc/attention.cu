@@ -1,6 +1,6 @@
 // Standalone launch of the decode-attention unit (attn_core.cuh): one CTA per (chunk, KV head,
-// user); CTAs beyond a user's chunk count exit at once.  Used when the stage runs its kernels
-// one by one (per-kernel timing mode); the persistent stage kernel runs the same units itself.
+// user); CTAs beyond a user's chunk count exit at once.  Used when the stage runs one kernel per
+// phase; the persistent stage kernel runs the same units itself.
 #include "attn_core.cuh"
 
 namespace kfl {
@@ -11,10 +11,17 @@ __global__ void __launch_bounds__(ATT_THREADS) attn_kernel(const __grid_constant
   __shared__ int s_last;
   const int c = blockIdx.x, kvh = blockIdx.y, b = blockIdx.z;
   pdl_launch_dependents();
-  pdl_wait();
+  // the positions were written before the step and the cached rows [0, P) in earlier steps:
+  // load the unit's first sub-tile (all but the new row, which the Q/K/V kernel writes) while
+  // that kernel is still running
   const int nc = attn_chunks(p, b);
-  if (c >= nc) return;
-  attn_unit<HD, 2>(p, b, kvh, c, nc, sm, &s_last, threadIdx.x, 0);
+  if (c >= nc) {
+    pdl_wait();
+    return;
+  }
+  attn_prefetch<HD, 2>(p, b, kvh, c, sm, threadIdx.x);
+  pdl_wait();
+  attn_unit<HD, 2>(p, b, kvh, c, nc, sm, &s_last, threadIdx.x, 1);
 }
 
 cudaError_t prepare_attention() {

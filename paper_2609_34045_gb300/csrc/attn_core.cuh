@@ -137,27 +137,41 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
   const int start = c * p.chunk;
   const int end = min(ntok, start + p.chunk);
 
-  for (int e = tid; e < G * HD; e += ATT_THREADS) {
-    const int g = e / HD, d = e % HD;
-    sq[g * 4 * L::QQ + (d / (HD / 4)) * L::QQ + d % (HD / 4)] =
-        __ldcg(p.q + (size_t)b * p.n_heads * HD + (size_t)kvh * G * HD + e) * p.scale_log2;
+  auto load_sub = [&](int sub, int buf) {
+    const int p0 = start + sub * ATT_SUB;
+    attn_load_rows<HD, NBUF>(p, b, kvh, p0, min(ATT_SUB, end - p0), buf, -1, -1, sm, tid);
+  };
+  // the first sub-tile's copies go out first, so that their latency overlaps the q loads
+  if (prefetched)  // only the new token's row of the first sub-tile is still to load
+    attn_load_rows<HD, NBUF>(p, b, kvh, start, min(ATT_SUB, end - start), 0, P, -1, sm, tid);
+  else
+    load_sub(0, 0);
+
+  {
+    // q rows of the group: loads first (independent), then the scaled stores
+    constexpr int QPT = (ATT_MAXG * HD + ATT_THREADS - 1) / ATT_THREADS;
+    float qv[QPT];
+#pragma unroll
+    for (int i = 0; i < QPT; ++i) {
+      const int e = tid + i * ATT_THREADS;
+      qv[i] = e < G * HD ? __ldcg(p.q + (size_t)b * p.n_heads * HD + (size_t)kvh * G * HD + e) : 0.f;
+    }
+#pragma unroll
+    for (int i = 0; i < QPT; ++i) {
+      const int e = tid + i * ATT_THREADS;
+      if (e < G * HD) {
+        const int g = e / HD, d = e % HD;
+        sq[g * 4 * L::QQ + (d / (HD / 4)) * L::QQ + d % (HD / 4)] = qv[i] * p.scale_log2;
+      }
+    }
   }
   if (tid < ATT_MAXG) {
     s_m[tid] = -INFINITY;
     s_l[tid] = 0.f;
   }
 
-  auto load_sub = [&](int sub, int buf) {
-    const int p0 = start + sub * ATT_SUB;
-    attn_load_rows<HD, NBUF>(p, b, kvh, p0, min(ATT_SUB, end - p0), buf, -1, -1, sm, tid);
-  };
-
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
   const int nsub = (end - start + ATT_SUB - 1) / ATT_SUB;
-  if (prefetched)  // only the new token's row of the first sub-tile is still to load
-    attn_load_rows<HD, NBUF>(p, b, kvh, start, min(ATT_SUB, end - start), 0, P, -1, sm, tid);
-  else
-    load_sub(0, 0);
   for (int it = 0; it < nsub; ++it) {
     const int buf = NBUF == 2 ? (it & 1) : 0;
     if (NBUF == 2 && it + 1 < nsub) {
@@ -316,16 +330,26 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
   }
   att_sync();
   if (owns) {
+    // the chunks' outputs in chunk order, loaded eight at a time so that they are in flight
+    // together
     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
     const float *pg = base + og * PS + od;
-#pragma unroll 4
-    for (int cc = 0; cc < nc; ++cc) {
-      const float w = wm[cc * G + og];
-      const float4 a = __ldcg(reinterpret_cast<const float4 *>(pg + (size_t)cc * ATT_MAXG * PS));
-      O.x = fmaf(w, a.x, O.x);
-      O.y = fmaf(w, a.y, O.y);
-      O.z = fmaf(w, a.z, O.z);
-      O.w = fmaf(w, a.w, O.w);
+    for (int c0 = 0; c0 < nc; c0 += 8) {
+      float4 a[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        a[j] = c0 + j < nc ? __ldcg(reinterpret_cast<const float4 *>(pg + (size_t)(c0 + j) * ATT_MAXG * PS))
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        if (c0 + j < nc) {
+          const float w = wm[(c0 + j) * G + og];
+          O.x = fmaf(w, a[j].x, O.x);
+          O.y = fmaf(w, a[j].y, O.y);
+          O.z = fmaf(w, a[j].z, O.z);
+          O.w = fmaf(w, a[j].w, O.w);
+        }
+      }
     }
     *reinterpret_cast<float4 *>(o + og * HD + od) = O;
   }

@@ -108,8 +108,10 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   p->n_sm = n_sm;
   p->ctas_per_sm = env_int("KFL_GEMV_CTAS_PER_SM", 1);
   if (p->ctas_per_sm < 1 || p->ctas_per_sm > 2) p->ctas_per_sm = 1;
-  p->stages = env_int("KFL_GEMV_STAGES", 6);
-  if (p->stages < 2 || p->stages > 10) p->stages = 6;
+  // 10 stages (169 KiB at batch 1) leave room for one CTA per SM: the next GEMV's CTA starts on
+  // an SM when this one leaves it and fills its ring during the rest of this GEMV's tail
+  p->stages = env_int("KFL_GEMV_STAGES", 10);
+  if (p->stages < 2 || p->stages > 10) p->stages = 10;
   p->gemv_grid_max = n_sm * p->ctas_per_sm;
   int nrb = 1;
   if (p->nl > 0) {
@@ -805,7 +807,7 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
       return fail(KFL_ERR_CUDA);
   }
   // persistent stage kernel: the deepest ring that fits next to the attention buffers
-  st->persistent = env_int("KFL_PERSISTENT", 1) != 0;
+  st->persistent = env_int("KFL_PERSISTENT", 0) != 0;
   {
     const size_t static_smem = 8192;  // the kernel's own __shared__ variables
     size_t smem_max = 0;

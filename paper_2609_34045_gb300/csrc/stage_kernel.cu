@@ -405,8 +405,9 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
 
 // ------------------------------------------------------------------------------- launch
 size_t stage_kernel_smem(int stages, int head_dim, int batch, int fmt) {
+  // + 128: the staging buffer is aligned up to 128 bytes after the barriers
   return (size_t)stages * stage_bytes(batch, fmt) + stage_kernel_attn_bytes(head_dim) +
-         (3 * stages + 2 * NSLOT) * sizeof(uint64_t) + NSLOT * RB * MAXB * sizeof(float);
+         (3 * stages + 2 * NSLOT) * sizeof(uint64_t) + 128 + NSLOT * RB * MAXB * sizeof(float);
 }
 
 int stage_kernel_attn_bytes(int head_dim) {

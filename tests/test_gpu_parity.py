@@ -106,7 +106,8 @@ def test_stage_split_associativity_bit_exact():
         p.close()
 
 
-def test_deterministic_replay_and_profile_mode():
+def test_deterministic_replay_and_profile_mode(monkeypatch):
+    monkeypatch.setenv("KFL_PERSISTENT", "1")
     p = Pair(RAGGED, 0, 3, K.KFL_IS_HEAD, 3, (10, 20, 30), 64, seed=17)
     pos = np.array([10, 20, 30], dtype=np.int32)
     ids = np.array([1, 2, 3], dtype=np.int32)
@@ -130,12 +131,14 @@ def test_deterministic_replay_and_profile_mode():
     p.close()
 
 
+@pytest.mark.parametrize("persistent", [0, 1], ids=["per-kernel", "persistent"])
 @pytest.mark.parametrize("fmt_model", [RAGGED, RAGGED_INT4], ids=["bf16", "int4"])
-def test_per_kernel_mode_parity(fmt_model, monkeypatch):
-    """The stage run as one launch per phase (CUDA graph with programmatic dependent launch)."""
-    monkeypatch.setenv("KFL_PERSISTENT", "0")
+def test_execution_mode_parity(fmt_model, persistent, monkeypatch):
+    """The stage run as one launch per phase (CUDA graph with programmatic dependent launch) and
+    as the persistent stage kernel."""
+    monkeypatch.setenv("KFL_PERSISTENT", str(persistent))
     p = Pair(fmt_model, 0, 2, K.KFL_IS_HEAD, 3, (4, 77, 150), 192, seed=23)
-    assert K.kfl_stage_launches_per_step(p.st, 3) == 2 + 5 * 2 + 1
+    assert K.kfl_stage_launches_per_step(p.st, 3) == (3 if persistent else 2 + 5 * 2 + 1)
     _greedy(p, 2, np.array([1, 500, 999], dtype=np.int32))
     p.close()
 
