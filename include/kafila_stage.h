@@ -159,13 +159,14 @@ int kfl_kv_read(kfl_stage *st, int local, int user, uint16_t *k, uint16_t *v, in
  * Changing it rebuilds the stage's CUDA graphs on the next decode. */
 int kfl_stage_debug_capture(kfl_stage *st, float *per_layer_hidden);
 
-/* Phase trace of the persistent stage kernel (tuning aid).  When buf (device uint64
- * [n_phases][grid][slots], shape from kfl_stage_trace_shape) is not NULL, every later decode
- * writes %globaltimer stamps (ns) per phase and CTA: 0 consumers reach the phase, 1 they pass
- * its grid barrier, 2 they finish it, 3 the activation producer passes the barrier, 4 it issues
- * the phase's last chunk, 5/6 the weight producer issues the phase's first/last tile (slots of
- * events that do not happen are left as they were).  NULL turns it off.  Changing it rebuilds
- * the stage's CUDA graphs on the next decode. */
+/* Phase trace (tuning aid).  When buf (device uint64 [n_phases][grid][slots], shape from
+ * kfl_stage_trace_shape) is not NULL, every later decode writes %globaltimer stamps (ns) per
+ * phase and CTA.  Slots: 0 the consumers reach an attention phase / finish a GEMV's tiles,
+ * 1 the phase starts on the CTA, 2 the CTA finishes it (epilogues included), 3 its activation
+ * input is available (first chunk copied; one-kernel-per-phase: past griddepcontrol.wait),
+ * 4 the last activation chunk is copied (persistent kernel), 5/6 the first/last weight tile is
+ * issued.  Slots of events that do not happen are left as they were.  NULL turns it off.
+ * Changing it rebuilds the stage's CUDA graphs on the next decode. */
 int kfl_stage_trace(kfl_stage *st, uint64_t *buf);
 int kfl_stage_trace_shape(kfl_stage *st, int batch, int *n_phases, int *grid, int *slots);
 

@@ -11,6 +11,11 @@ __global__ void __launch_bounds__(ATT_THREADS) attn_kernel(const __grid_constant
   __shared__ int s_last;
   const int c = blockIdx.x, kvh = blockIdx.y, b = blockIdx.z;
   pdl_launch_dependents();
+  const int lin = c + gridDim.x * (kvh + gridDim.y * b);
+  auto stamp = [&](int slot) {
+    if (p.trace && lin < p.trace_grid && threadIdx.x == 0) p.trace[(size_t)lin * TRACE_SLOTS + slot] = global_ns();
+  };
+  stamp(TR_CONS_GO);
   // the positions were written before the step and the cached rows [0, P) in earlier steps:
   // load the unit's first sub-tile (all but the new row, which the Q/K/V kernel writes) while
   // that kernel is still running
@@ -21,7 +26,10 @@ __global__ void __launch_bounds__(ATT_THREADS) attn_kernel(const __grid_constant
   }
   attn_prefetch<HD, 2>(p, b, kvh, c, sm, threadIdx.x);
   pdl_wait();
-  attn_unit<HD, 2>(p, b, kvh, c, nc, sm, &s_last, threadIdx.x, 1);
+  stamp(TR_X_GO);
+  attn_unit<HD, 2>(p, b, kvh, c, nc, sm, &s_last, threadIdx.x, 1,
+                   p.trace && lin < p.trace_grid ? p.trace + (size_t)lin * TRACE_SLOTS : nullptr);
+  stamp(TR_CONS_DONE);
 }
 
 cudaError_t prepare_attention() {

@@ -109,7 +109,12 @@ __device__ __forceinline__ void attn_publish(const AttnParams &p, int kvh, int t
 
 template <int HD, int NBUF>
 __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, uint8_t *sm, int *s_last, int tid,
-                          int prefetched) {
+                          int prefetched, unsigned long long *tr = nullptr) {
+  // tr: this CTA's trace slots (tuning aid): 4 K/V in shared memory, 5 output or partial
+  // computed, 6 the merge starts (the last unit of its user and KV head)
+  auto stamp = [&](int slot) {
+    if (tr && tid == 0) tr[slot] = global_ns();
+  };
   using L = AttnLayout<HD, NBUF>;
   uint8_t *sk = sm + L::K_OFF;
   uint8_t *sv = sm + L::V_OFF;
@@ -182,6 +187,7 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
       cp_async_wait<0>();
     }
     att_sync();
+    if (it == 0) stamp(TR_X_LAST);
     const int p0 = start + it * ATT_SUB;
     const int cnt = min(ATT_SUB, end - p0);
     const uint8_t *kb = sk + buf * ATT_SUB * L::KROW;
@@ -277,6 +283,7 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
     att_sync();
   }
 
+  stamp(TR_W_FIRST);
   if (nc == 1) {
     if (owns) {
       const float il = 1.0f / s_l[og];
@@ -302,6 +309,7 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
   }
   att_sync();
   if (!*s_last) return;
+  stamp(TR_W_LAST);
   // merge: per-chunk weights 2^(m_c - M) / L staged in shared memory (the K buffers), then each
   // thread sums its 4 outputs over the chunks
   const float *base = p.partial + unit_base * (ATT_MAXG * PS);

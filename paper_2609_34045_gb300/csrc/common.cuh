@@ -110,6 +110,8 @@ struct GemvParams {
   int out_unit;               // output elements per row block (RESID 64, SWIGLU 32)
   int out_kt;                 // the consumer's tile K
   unsigned *out_done;         // row blocks completed
+  unsigned long long *trace;  // one-kernel-per-phase mode: this launch's [grid][TRACE_SLOTS]
+                              // %globaltimer stamps, or NULL
 };
 
 struct AttnParams {
@@ -128,6 +130,8 @@ struct AttnParams {
   const unsigned *in_ready;  // per KV head: Q/K/V row blocks completed
   int in_need;
   unsigned *out_ready;       // per KV head: (user, KV head) outputs completed
+  unsigned long long *trace;  // one-kernel-per-phase mode: this launch's [grid][TRACE_SLOTS], or NULL
+  int trace_grid;
 };
 
 // One phase of the persistent stage kernel: a GEMV (with its epilogue) or an attention pass.
@@ -320,6 +324,7 @@ namespace kfl {
 cudaError_t prepare_gemv();
 cudaError_t prepare_attention();
 cudaError_t launch_gemv(const GemvParams &p, int epi, int grid, cudaStream_t s, bool pdl);
+int gemv_max_stages(int batch, int fmt, int smem_optin);  // valid after prepare_gemv
 cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s, bool pdl);
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in,
                                int batch, const uint16_t *embed, int vocab, int d, int ldh,

@@ -22,7 +22,8 @@
 
 namespace kfl {
 
-constexpr int GEMV_MAX_STAGES = 10;  // standalone kernel: two CTAs (this and the next) per SM
+constexpr int GEMV_MAX_STAGES = 13;  // 13 x 16.9 KiB (batch 1) still fits one CTA's shared memory
+constexpr int GEMV_STATIC_SMEM = 2048;  // allowance for the kernel's own __shared__ variables
 
 // ---------------------------------------------------------------------------- the kernel
 // FMT 0: bf16 tiles [RB][KT].  FMT 1: int4 tiles, codes [RB][KT4/8] uint32 + scales [RB][KT4/64].
@@ -66,6 +67,10 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
   }
   __syncthreads();
   pdl_launch_dependents();
+  auto stamp = [&](int slot) {
+    if (p.trace) p.trace[(size_t)c * TRACE_SLOTS + slot] = global_ns();
+  };
+  if (tid == 0) stamp(TR_CONS_GO);
 
   if (warp == CONSUMER_WARPS) {
     // ------------------------------------------------------------------ producer
@@ -74,6 +79,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
       const uint64_t pol_x = policy_evict_last();
       const uint32_t xbytes = B * (KTILE * 4);
       const int pre = n < S ? n : S;
+      stamp(TR_W_FIRST);
       for (int i = 0; i < pre; ++i) {
         const uint32_t fb = smem_addr(&full[i]);
         mbar_arrive_expect_tx(fb, WBYTES + xbytes);
@@ -81,6 +87,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
         s_issued = i + 1;
       }
       pdl_wait();
+      stamp(TR_X_GO);
       auto issue_x = [&](int kt, int s) {
         const uint32_t fb = smem_addr(&full[s]);
         const uint32_t dst = smem_addr(smem + (size_t)s * SB + WBYTES);
@@ -108,6 +115,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
           eph ^= 1u;
         }
       }
+      stamp(TR_W_LAST);
     }
     return;
   }
@@ -118,6 +126,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
     bool inv_ready = true;
     int segc = 0;
     gemv_epilogues<B, EPI>(p, t0, n, T, G, c, sr, segc, s_inv, inv_ready, &s_abort, lane);
+    if (lane == 0) stamp(TR_CONS_DONE);
     return;
   }
 
@@ -127,6 +136,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
   gemv_consume<B, FMT>(p.n_kt, smem, full, empty, S, s, phase, t0, n, sr, segc, &s_abort, p.err, tid);
 
   consumer_sync();
+  if (tid == 0) stamp(TR_CONS_ENTER);
   if (s_abort && tid == 0) {
     // drain copies still in flight before the CTA's shared memory goes away (bounded)
     const int issued = s_issued;
@@ -180,10 +190,19 @@ static cudaError_t launch_f(const GemvParams &p, int epi, int grid, cudaStream_t
   }
 }
 
+// The deepest ring of this batch size and format that fits a CTA's shared memory.
+int gemv_max_stages(int batch, int fmt, int smem_optin) {
+  int s = GEMV_MAX_STAGES;
+  while (s > 2 && gemv_smem_bytes(s, batch, fmt) + GEMV_STATIC_SMEM > (size_t)smem_optin) --s;
+  return s;
+}
+
+static int g_smem_optin = 0;
+
 template <int B, int EPI, int FMT>
 static cudaError_t prepare_one() {
   return cudaFuncSetAttribute(gemv_kernel<B, EPI, FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)gemv_smem_bytes(GEMV_MAX_STAGES, B, FMT));
+                              (int)gemv_smem_bytes(gemv_max_stages(B, FMT, g_smem_optin), B, FMT));
 }
 
 template <int EPI, int FMT>
@@ -208,12 +227,16 @@ static cudaError_t prepare_f() {
 // Raise the dynamic shared-memory limit of every GEMV instantiation (once per device, before
 // any launch or stream capture).
 cudaError_t prepare_gemv() {
-  cudaError_t e = prepare_f<0>();
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&g_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (e != cudaSuccess) return e;
+  e = prepare_f<0>();
   return e != cudaSuccess ? e : prepare_f<1>();
 }
 
 cudaError_t launch_gemv(const GemvParams &p, int epi, int grid, cudaStream_t s, bool pdl) {
-  if (p.stages < 2 || p.stages > GEMV_MAX_STAGES) return cudaErrorInvalidValue;
+  if (p.stages < 2 || p.stages > gemv_max_stages(p.batch, p.fmt, g_smem_optin)) return cudaErrorInvalidValue;
   return p.fmt == 0 ? launch_f<0>(p, epi, grid, s, pdl) : launch_f<1>(p, epi, grid, s, pdl);
 }
 

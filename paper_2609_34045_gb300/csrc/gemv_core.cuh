@@ -250,11 +250,34 @@ __device__ __forceinline__ void norm_scale_warp(const GemvParams &p, float *inv,
   }
 }
 
+// Values the epilogue of a row block reads from global memory, loaded before the row block's
+// partial sums are combined so that their latency overlaps the combine (RESID: the residual rows
+// and the next RMSNorm gain).  Loaded after the segment's staging slot is full, which orders them
+// after the writes of earlier phases.
+struct EpiPre {
+  float h[MAXB][2];
+  float g[2];
+};
+
+template <int B, int EPI>
+__device__ __forceinline__ void epilogue_prefetch(const GemvParams &p, int rb, int lane, EpiPre &e) {
+  if constexpr (EPI == EPI_RESID) {
+#pragma unroll
+    for (int h2 = 0; h2 < 2; ++h2) {
+      const int n = rb * RB + lane + 32 * h2;
+      const bool ok = n < p.n_rows;
+#pragma unroll
+      for (int b = 0; b < B; ++b) e.h[b][h2] = ok ? __ldcg(p.h + (size_t)b * p.ldh + n) : 0.f;
+      e.g[h2] = ok && p.g_next ? p.g_next[n] : 0.f;
+    }
+  }
+}
+
 // The fused epilogue of row block rb: red[r * MAXB + b] is the dot product of row rb*RB + r for
 // user b, before the RMSNorm scale inv[b].  One warp.
 template <int B, int EPI>
 __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const float *red, const float *inv,
-                                              int lane) {
+                                              const EpiPre &pre, int lane) {
   if constexpr (EPI == EPI_STORE) {
     for (int e = lane; e < RB * B; e += 32) {
       const int b = e / RB, r = e % RB, n = rb * RB + r;
@@ -269,9 +292,9 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
         const int r = lane + 32 * h2, n = rb * RB + r;
         if (n < p.n_rows) {
           const size_t o = (size_t)b * p.ldh + n;
-          const float hn = __ldcg(p.h + o) + red[r * MAXB + b] * inv[b];
+          const float hn = pre.h[b][h2] + red[r * MAXB + b] * inv[b];
           p.h[o] = hn;
-          if (p.g_next) p.xn[o] = hn * p.g_next[n];
+          if (p.g_next) p.xn[o] = hn * pre.g[h2];
           if (p.capture) p.capture[(size_t)b * p.n_rows + n] = hn;
           sq = fmaf(hn, hn, sq);
         }
@@ -382,6 +405,8 @@ __device__ __forceinline__ void gemv_epilogues(const GemvParams &p, long long t0
     ++segc;
     consumer_wait(smem_addr(&sr.full[slot]), use & 1, abort_flag, p.err);
     float *red = sr.red + slot * RB * MAXB;
+    EpiPre pre;
+    epilogue_prefetch<B, EPI>(p, rb, lane, pre);
     bool do_epi = true;
     if (!(kt0 == 0 && len == p.n_kt)) {
       // this row block is shared with neighbouring CTAs
@@ -441,7 +466,7 @@ __device__ __forceinline__ void gemv_epilogues(const GemvParams &p, long long t0
         norm_scale_warp<B>(p, inv, lane);
         inv_ready = true;
       }
-      epilogue_warp<B, EPI>(p, rb, red, inv, lane);
+      epilogue_warp<B, EPI>(p, rb, red, inv, pre, lane);
       __syncwarp();
       if (lane == 0) {
         // publish this row block (the __syncwarp above ordered every lane's stores before it)

@@ -111,7 +111,7 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   // 10 stages (169 KiB at batch 1) leave room for one CTA per SM: the next GEMV's CTA starts on
   // an SM when this one leaves it and fills its ring during the rest of this GEMV's tail
   p->stages = env_int("KFL_GEMV_STAGES", 10);
-  if (p->stages < 2 || p->stages > 10) p->stages = 10;
+  if (p->stages < 2 || p->stages > 13) p->stages = 10;
   p->gemv_grid_max = n_sm * p->ctas_per_sm;
   int nrb = 1;
   if (p->nl > 0) {
@@ -188,6 +188,7 @@ struct kfl_stage {
   std::vector<void *> allocs;
   int alloc_count = 0, fault_at = 0;
   cudaStream_t cap_stream = nullptr;
+  int smem_optin = 0;  // shared memory a block may opt in to
   cudaGraphExec_t graph[MAXB + 1] = {};
   // persistent stage kernel
   bool persistent = true;
@@ -268,7 +269,7 @@ GemvParams base_gemv(kfl_stage *st, const Mat &m, const float *x, int ldx, int b
   g.x = x;
   g.ldx = ldx;
   g.batch = batch;
-  g.stages = st->P.stages;
+  g.stages = std::min(st->P.stages, gemv_max_stages(batch, m.fmt, st->smem_optin));
   g.rope_per_user = 0;
   g.partial = st->gemv_partial;
   g.tickets = st->tickets;
@@ -382,6 +383,19 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk, bool d
     g.argmax_ticket = st->am_ticket;
     g.next_ids = st->next_int;
     gemv(EPI_ARGMAX, g);
+  }
+  if (!dataflow && st->trace) {
+    // one kernel per phase: each launch stamps its own slice of the trace
+    const int tg = std::max(P.n_sm, P.gemv_grid_max);
+    for (size_t k = 0; k < ph.size(); ++k) {
+      unsigned long long *slice = st->trace + k * (size_t)tg * TRACE_SLOTS;
+      if (ph[k].kind == PH_GEMV) {
+        ph[k].g.trace = slice;
+      } else {
+        ph[k].a.trace = slice;
+        ph[k].a.trace_grid = tg;
+      }
+    }
   }
   if (dataflow) {
     // readiness counters: phase k publishes in region k, the phase after it reads region k
@@ -718,6 +732,7 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
   st->l1 = l1;
   st->flags = flags;
   st->dev = dev;
+  st->smem_optin = smem_optin;
   st->fault_at = env_int("KFL_FAULT_ALLOC_AT", 0);
   make_plan(cfg, l0, l1, flags, n_sm, &st->P);
   Plan &P = st->P;
@@ -1077,7 +1092,7 @@ extern "C" int kfl_stage_trace_shape(kfl_stage *st, int batch, int *n_phases, in
   if (!valid(st)) return KFL_ERR_STATE;
   if (batch < 1 || batch > st->cfg.max_batch) return KFL_ERR_RANGE;
   if (n_phases) *n_phases = (int)build_phases(st, batch, st->persist_chunk[batch]).size();
-  if (grid) *grid = st->P.n_sm;
+  if (grid) *grid = std::max(st->P.n_sm, st->P.gemv_grid_max);
   if (slots) *slots = TRACE_SLOTS;
   return KFL_OK;
 }
