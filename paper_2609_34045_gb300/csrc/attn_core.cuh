@@ -10,8 +10,11 @@
 // its (user, KV head) to finish (atomic ticket, no spin) merges the chunks in chunk order.
 // Scores are in the log2 domain (q pre-scaled by log2(e)/sqrt(hd)).
 //
-// 256 threads.  Scores: 4 lanes per position, each a quarter of the head dimension, for every
-// head.  P.V: one warp per head (two per warp at hd 64), 4 dimensions per lane.
+// 256 threads.  Scores S = q K^T and the weighted sum P V are small dense products (at most 8
+// heads x 64 positions x hd): both run on the tensor cores as warp-level m16n8k8 MMAs in TF32
+// with fp32 accumulation (the heads are the M rows, padded to 16).  q and P are rounded to TF32
+// (2^-11 relative); K and V are bf16 and exact in TF32.  Scores: warp w takes positions 8w..8w+7;
+// P V: warp w takes head dimensions hd/8 * w onwards.
 #pragma once
 
 #include <math.h>
@@ -39,17 +42,17 @@ __device__ __forceinline__ void cp_async_wait() {
 
 template <int HD, int NBUF>
 struct AttnLayout {
-  // K row: four quarters of hd/4 dims, each padded by 16 bytes, so the four lanes reading the
-  // quarters of one position and the next position's lanes hit distinct banks
-  static constexpr int QB = HD / 2 + 16;
-  static constexpr int KROW = 4 * QB;
-  static constexpr int VROW = HD * 2;
-  static constexpr int QQ = HD / 4 + 4;     // floats per padded quarter of a q row
+  // K and V rows padded by 16 bytes (4 banks) so that the MMA fragments of 8 consecutive rows
+  // fall in distinct banks; q rows (fp32) padded by 8 floats, score rows by 4
+  static constexpr int KROW = HD * 2 + 16;
+  static constexpr int VROW = HD * 2 + 16;
+  static constexpr int QS = HD + 8;
+  static constexpr int SS = ATT_SUB + 4;
   static constexpr int K_OFF = 0;
   static constexpr int V_OFF = K_OFF + NBUF * ATT_SUB * KROW;
   static constexpr int Q_OFF = V_OFF + NBUF * ATT_SUB * VROW;
-  static constexpr int S_OFF = Q_OFF + ATT_MAXG * 4 * QQ * 4;
-  static constexpr int M_OFF = S_OFF + ATT_MAXG * ATT_SUB * 4;
+  static constexpr int S_OFF = Q_OFF + ATT_MAXG * QS * 4;
+  static constexpr int M_OFF = S_OFF + ATT_MAXG * SS * 4;
   static constexpr int BYTES = M_OFF + 4 * ATT_MAXG * 4;
   static constexpr int MERGE_MAX = (NBUF * ATT_SUB * KROW) / 8;  // chunks x heads in the K buffers
   static_assert(MERGE_MAX >= 1024, "merge scratch too small");
@@ -77,12 +80,11 @@ __device__ __forceinline__ void attn_load_rows(const AttnParams &p, int b, int k
   uint8_t *sk = sm + L::K_OFF + buf * ATT_SUB * L::KROW;
   uint8_t *sv = sm + L::V_OFF + buf * ATT_SUB * L::VROW;
   constexpr int CH = HD / 8;   // 16-byte chunks per row
-  constexpr int CQ = HD / 32;  // chunks per quarter
   for (int e = tid; e < cnt * CH; e += ATT_THREADS) {
     const int r = e / CH, ch = e % CH;
     const int row = p0 + r;
     if ((only >= 0 && row != only) || row == skip) continue;
-    cp_async16(sk + r * L::KROW + (ch / CQ) * L::QB + (ch % CQ) * 16, kg + (size_t)row * HD + ch * 8);
+    cp_async16(sk + r * L::KROW + ch * 16, kg + (size_t)row * HD + ch * 8);
     cp_async16(sv + r * L::VROW + ch * 16, vg + (size_t)row * HD + ch * 8);
   }
   cp_async_commit();
@@ -105,6 +107,23 @@ __device__ __forceinline__ void attn_publish(const AttnParams &p, int kvh, int t
   if (!p.out_ready) return;
   att_sync();
   if (tid == 0) red_add_release(p.out_ready + kvh, 1u);
+}
+
+// fp32 -> TF32 (round to nearest, ties away), as the MMA's operand bits
+__device__ __forceinline__ uint32_t to_tf32(float x) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+  return r;
+}
+
+// d += a b for one m16n8k8 TF32 tile (a: 16x8 row-major, b: 8x8 column-major, fp32 accumulate).
+// Rows 8..15 of a are the zero padding of the at most 8 heads, so a1 = a3 = 0.
+__device__ __forceinline__ void mma_tf32(float (&d)[4], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
 }
 
 template <int HD, int NBUF>
@@ -166,7 +185,7 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
       const int e = tid + i * ATT_THREADS;
       if (e < G * HD) {
         const int g = e / HD, d = e % HD;
-        sq[g * 4 * L::QQ + (d / (HD / 4)) * L::QQ + d % (HD / 4)] = qv[i] * p.scale_log2;
+        sq[g * L::QS + d] = qv[i] * p.scale_log2;
       }
     }
   }
@@ -175,7 +194,20 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
     s_l[tid] = 0.f;
   }
 
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  // MMA fragment coordinates: lane = 4 * gid + tig; accumulator rows gid are heads (gid < G)
+  const int gid = lane >> 2, tig = lane & 3;
+  const bool hrow = gid < G;
+  constexpr int KS = HD / 8;    // K steps of the scores
+  constexpr int NT = HD / 64;   // P V n-tiles (8 dimensions) per warp: warp w owns dims NT*8*w ...
+  const int n_base = warp * NT * 8;
+  float acc[NT][4];
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
+  // q as A fragments.  Within each K step of 8 dimensions the MMA's k = tig, tig + 4 are taken as
+  // dimensions 2 tig, 2 tig + 1 (the same order for q and K: the dot product is unchanged), so
+  // that a lane's two K values are one 32-bit load.
+  uint32_t qa0[KS], qa2[KS];
+
   const int nsub = (end - start + ATT_SUB - 1) / ATT_SUB;
   for (int it = 0; it < nsub; ++it) {
     const int buf = NBUF == 2 ? (it & 1) : 0;
@@ -191,47 +223,41 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
     const int p0 = start + it * ATT_SUB;
     const int cnt = min(ATT_SUB, end - p0);
     const uint8_t *kb = sk + buf * ATT_SUB * L::KROW;
-    const uint8_t *vb = sv + buf * ATT_SUB * L::VROW;
-
-    // scores: lanes 4i..4i+3 share position i, each a quarter of the head dimension
-    {
-      const int pp = tid >> 2, qq = tid & 3;
-      const bool valid = pp < cnt;
-      float kf[HD / 4];
-      const uint4 *kr = reinterpret_cast<const uint4 *>(kb + pp * L::KROW + qq * L::QB);
+    uint8_t *vb = sv + buf * ATT_SUB * L::VROW;
+    if (it == 0) {
 #pragma unroll
-      for (int ch = 0; ch < HD / 32; ++ch) {
-        const uint4 k4 = valid ? kr[ch] : make_uint4(0u, 0u, 0u, 0u);
-        kf[8 * ch] = bf16_lo(k4.x); kf[8 * ch + 1] = bf16_hi(k4.x);
-        kf[8 * ch + 2] = bf16_lo(k4.y); kf[8 * ch + 3] = bf16_hi(k4.y);
-        kf[8 * ch + 4] = bf16_lo(k4.z); kf[8 * ch + 5] = bf16_hi(k4.z);
-        kf[8 * ch + 6] = bf16_lo(k4.w); kf[8 * ch + 7] = bf16_hi(k4.w);
+      for (int s8 = 0; s8 < KS; ++s8) {
+        const float2 qv = hrow ? *reinterpret_cast<const float2 *>(sq + gid * L::QS + 8 * s8 + 2 * tig)
+                               : make_float2(0.f, 0.f);
+        qa0[s8] = to_tf32(qv.x);
+        qa2[s8] = to_tf32(qv.y);
       }
+    }
+    // rows past the sub-tile's positions take part in P V with weight 0: make them finite
+    if (cnt < ATT_SUB)
+      for (int e = tid; e < (ATT_SUB - cnt) * (HD / 8); e += ATT_THREADS)
+        *reinterpret_cast<uint4 *>(vb + (cnt + e / (HD / 8)) * L::VROW + (e % (HD / 8)) * 16) = make_uint4(0u, 0u, 0u, 0u);
+
+    // scores of positions 8w .. 8w + 7 for every head (rows gid)
+    {
+      float sc[4] = {0.f, 0.f, 0.f, 0.f};
+      const uint8_t *krow = kb + (8 * warp + gid) * L::KROW + 4 * tig;
 #pragma unroll
-      for (int g = 0; g < ATT_MAXG; ++g) {
-        if (g < G) {
-          const float4 *qr = reinterpret_cast<const float4 *>(sq + g * 4 * L::QQ + qq * L::QQ);
-          float d0 = 0.f, d1 = 0.f;
-#pragma unroll
-          for (int i = 0; i < HD / 16; ++i) {
-            const float4 q4 = qr[i];
-            d0 = fmaf(kf[4 * i], q4.x, d0);
-            d1 = fmaf(kf[4 * i + 1], q4.y, d1);
-            d0 = fmaf(kf[4 * i + 2], q4.z, d0);
-            d1 = fmaf(kf[4 * i + 3], q4.w, d1);
-          }
-          float dot = d0 + d1;
-          dot += __shfl_xor_sync(0xffffffffu, dot, 1);
-          dot += __shfl_xor_sync(0xffffffffu, dot, 2);
-          if (qq == 0) ss[g * ATT_SUB + pp] = valid ? dot : -INFINITY;
-        }
+      for (int s8 = 0; s8 < KS; ++s8) {
+        const uint32_t kw = *reinterpret_cast<const uint32_t *>(krow + 16 * s8);
+        mma_tf32(sc, qa0[s8], qa2[s8], kw << 16, kw & 0xFFFF0000u);
+      }
+      if (hrow) {
+        const int pp = 8 * warp + 2 * tig;
+        *reinterpret_cast<float2 *>(ss + gid * L::SS + pp) =
+            make_float2(pp < cnt ? sc[0] : -INFINITY, pp + 1 < cnt ? sc[1] : -INFINITY);
       }
     }
     att_sync();
     // online softmax update: warp g owns head g
     if (warp < G) {
       const int g = warp;
-      const float a0 = ss[g * ATT_SUB + lane], a1 = ss[g * ATT_SUB + lane + 32];
+      const float a0 = ss[g * L::SS + lane], a1 = ss[g * L::SS + lane + 32];
       float mx = fmaxf(a0, a1);
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
@@ -241,8 +267,8 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
       float sum = e0 + e1;
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-      ss[g * ATT_SUB + lane] = e0;
-      ss[g * ATT_SUB + lane + 32] = e1;
+      ss[g * L::SS + lane] = e0;
+      ss[g * L::SS + lane + 32] = e1;
       __syncwarp();
       if (lane == 0) {
         const float alpha = exp2f(m_old - m_new);
@@ -252,32 +278,28 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
       }
     }
     att_sync();
-    // acc = acc * alpha + P . V over the sub-tile's valid positions
-    if (owns) {
-      const float al = s_alpha[og];
+    // acc = acc * alpha + P V over the sub-tile (P as A fragments, V as B fragments)
+    {
+      const float al = hrow ? s_alpha[gid] : 0.f;
 #pragma unroll
-      for (int i = 0; i < 4; ++i) acc[i] *= al;
-      const float *pr = ss + og * ATT_SUB;
-      int pp = 0;
-      for (; pp + 4 <= cnt; pp += 4) {
-        const float4 p4 = *reinterpret_cast<const float4 *>(pr + pp);
-        const float pw[4] = {p4.x, p4.y, p4.z, p4.w};
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const uint2 v2 = *reinterpret_cast<const uint2 *>(vb + (pp + k) * L::VROW + od * 2);
-          acc[0] = fmaf(pw[k], bf16_lo(v2.x), acc[0]);
-          acc[1] = fmaf(pw[k], bf16_hi(v2.x), acc[1]);
-          acc[2] = fmaf(pw[k], bf16_lo(v2.y), acc[2]);
-          acc[3] = fmaf(pw[k], bf16_hi(v2.y), acc[3]);
-        }
+      for (int nt = 0; nt < NT; ++nt) {
+        acc[nt][0] *= al;
+        acc[nt][1] *= al;
       }
-      for (; pp < cnt; ++pp) {
-        const float pw = pr[pp];
-        const uint2 v2 = *reinterpret_cast<const uint2 *>(vb + pp * L::VROW + od * 2);
-        acc[0] = fmaf(pw, bf16_lo(v2.x), acc[0]);
-        acc[1] = fmaf(pw, bf16_hi(v2.x), acc[1]);
-        acc[2] = fmaf(pw, bf16_lo(v2.y), acc[2]);
-        acc[3] = fmaf(pw, bf16_hi(v2.y), acc[3]);
+      const float *prow = ss + gid * L::SS;
+#pragma unroll
+      for (int k8 = 0; k8 < ATT_SUB / 8; ++k8) {
+        const uint32_t pa0 = hrow ? to_tf32(prow[8 * k8 + tig]) : 0u;
+        const uint32_t pa2 = hrow ? to_tf32(prow[8 * k8 + tig + 4]) : 0u;
+        const uint8_t *v0 = vb + (8 * k8 + tig) * L::VROW;
+        const uint8_t *v1 = v0 + 4 * L::VROW;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          const int n = n_base + 8 * nt + gid;
+          const uint32_t b0 = (uint32_t)(*reinterpret_cast<const uint16_t *>(v0 + 2 * n)) << 16;
+          const uint32_t b1 = (uint32_t)(*reinterpret_cast<const uint16_t *>(v1 + 2 * n)) << 16;
+          mma_tf32(acc[nt], pa0, pa2, b0, b1);
+        }
       }
     }
     att_sync();
@@ -285,9 +307,12 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
 
   stamp(TR_W_FIRST);
   if (nc == 1) {
-    if (owns) {
-      const float il = 1.0f / s_l[og];
-      *reinterpret_cast<float4 *>(o + og * HD + od) = make_float4(acc[0] * il, acc[1] * il, acc[2] * il, acc[3] * il);
+    if (hrow) {
+      const float il = 1.0f / s_l[gid];
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+        *reinterpret_cast<float2 *>(o + gid * HD + n_base + 8 * nt + 2 * tig) =
+            make_float2(acc[nt][0] * il, acc[nt][1] * il);
     }
     attn_publish(p, kvh, tid);
     return;
@@ -295,7 +320,11 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
   constexpr int PS = attn_pstride(HD);
   const size_t unit_base = ((size_t)b * p.n_kv_heads + kvh) * p.n_chunks;
   float *part = p.partial + (unit_base + c) * (ATT_MAXG * PS);
-  if (owns) *reinterpret_cast<float4 *>(part + og * PS + od) = make_float4(acc[0], acc[1], acc[2], acc[3]);
+  if (hrow) {
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+      *reinterpret_cast<float2 *>(part + gid * PS + n_base + 8 * nt + 2 * tig) = make_float2(acc[nt][0], acc[nt][1]);
+  }
   if (tid < G) {
     part[tid * PS + HD] = s_m[tid];
     part[tid * PS + HD + 1] = s_l[tid];
@@ -311,8 +340,20 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
   if (!*s_last) return;
   stamp(TR_W_LAST);
   // merge: per-chunk weights 2^(m_c - M) / L staged in shared memory (the K buffers), then each
-  // thread sums its 4 outputs over the chunks
+  // thread sums its 4 outputs over the chunks.  The chunk outputs are loaded MB at a time, the
+  // first MB before the weights are computed, so that few L2 round trips are in series (MB 8
+  // inside the persistent stage kernel, whose register budget is shared with its other roles).
+  constexpr int MB = NBUF == 2 ? 16 : 8;
   const float *base = p.partial + unit_base * (ATT_MAXG * PS);
+  const float *pg = base + og * PS + od;
+  float4 a[MB];
+  auto load_batch = [&](int c0) {
+#pragma unroll
+    for (int j = 0; j < MB; ++j)
+      a[j] = owns && c0 + j < nc ? __ldcg(reinterpret_cast<const float4 *>(pg + (size_t)(c0 + j) * ATT_MAXG * PS))
+                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+  };
+  load_batch(0);
   float *wm = reinterpret_cast<float *>(sk);
   float *wl = wm + L::MERGE_MAX;
   for (int e = tid; e < nc * G; e += ATT_THREADS) {
@@ -338,18 +379,11 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
   }
   att_sync();
   if (owns) {
-    // the chunks' outputs in chunk order, loaded eight at a time so that they are in flight
-    // together
     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
-    const float *pg = base + og * PS + od;
-    for (int c0 = 0; c0 < nc; c0 += 8) {
-      float4 a[8];
+    for (int c0 = 0; c0 < nc; c0 += MB) {
+      if (c0 > 0) load_batch(c0);
 #pragma unroll
-      for (int j = 0; j < 8; ++j)
-        a[j] = c0 + j < nc ? __ldcg(reinterpret_cast<const float4 *>(pg + (size_t)(c0 + j) * ATT_MAXG * PS))
-                           : make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
+      for (int j = 0; j < MB; ++j) {
         if (c0 + j < nc) {
           const float w = wm[(c0 + j) * G + og];
           O.x = fmaf(w, a[j].x, O.x);
