@@ -51,6 +51,17 @@ def dist_env():
     return int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)), int(os.environ.get("WORLD_SIZE", 1))
 
 
+def max_over_ranks(x: float, dist, device) -> float:
+    """The largest of every rank's x (the job is as slow as its slowest replica); x itself
+    without a process group."""
+    if dist is None:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 # ---------------------------------------------------------------------------- bytes
 
 def kernel_bytes(work, kind: str) -> int:
@@ -157,9 +168,11 @@ class ClockSampler:
 
 # ---------------------------------------------------------------------------- CPU oracle
 
-def oracle_layer_seconds(work, n_layer_steps: int, warmup: int = 1):
+def oracle_layer_seconds(work, n_layer_steps: int, warmup: int = 1, budget_s: float = 0.0):
     """Time the CPU oracle on single-block decode steps of the workload (weights and KV made
-    before timing).  Returns (seconds per layer-token, layer-steps timed, threads)."""
+    before timing): n_layer_steps steps, or with budget_s > 0 as many as fit in about budget_s
+    seconds (at least 2, at most n_layer_steps).  Returns (seconds per layer-token, layer-steps
+    timed, threads)."""
     import numpy as np
 
     import oracle
@@ -175,10 +188,14 @@ def oracle_layer_seconds(work, n_layer_steps: int, warmup: int = 1):
     for _ in range(warmup):
         st.decode(pos, hidden_in=h)
     t0 = time.perf_counter()
-    for _ in range(n_layer_steps):
+    n = 0
+    while n < n_layer_steps:
         st.decode(pos, hidden_in=h)
-    dt = (time.perf_counter() - t0) / n_layer_steps
-    return dt / work.batch, n_layer_steps, os.cpu_count()
+        n += 1
+        if budget_s > 0 and n >= 2 and time.perf_counter() - t0 >= budget_s:
+            break
+    dt = (time.perf_counter() - t0) / n
+    return dt / work.batch, n, os.cpu_count()
 
 
 def run_reference(args, work):
@@ -202,6 +219,74 @@ def run_reference(args, work):
 
 
 # ---------------------------------------------------------------------------- ours
+
+def run_splits(work, st_full, ids_all, hid_all, pos_all, args, stream):
+    """The workload's stage splits ({13, 67} = blocks [0, 13) then [13, 80), ...) run as
+    consecutive stages on this GPU, the hidden state handed over in a device buffer.  Each split
+    is checked bit for bit against the single stage over its first steps (next ids and final
+    hidden state), then timed.  Returns a list of per-split results."""
+    import torch
+
+    from paper_2609_34045_gb300 import device_inputs as di
+    from paper_2609_34045_gb300 import stage as K
+
+    m, b, d = work.model, work.batch, work.model.d_model
+    n_check = 3
+    n_time = max(10, min(200, args.steps // 10))
+    cfg = K.model_cfg(m, work.max_ctx, b)
+    res = []
+    for split in work.splits:
+        if len(split) < 2:
+            continue
+        bounds = [work.l0]
+        for n in split:
+            bounds.append(bounds[-1] + n)
+        parts = []
+        for i in range(len(split)):
+            flags = (K.KFL_EMBED_IN if (i == 0 and work.embed_in) else 0) | \
+                    (K.KFL_LOGITS_OUT if (i == len(split) - 1 and work.logits_out) else 0)
+            s_ = K.kfl_stage_create(cfg, bounds[i], bounds[i + 1], flags)
+            di.load_stage_seeded(s_, work, bounds[i], bounds[i + 1])
+            parts.append(s_)
+        hbuf = [torch.empty(b, d, dtype=torch.float32, device="cuda") for _ in range(len(split))]
+        nxt = torch.empty(b, dtype=torch.int32, device="cuda") if work.logits_out else None
+
+        def chain(i):
+            j = i % work.steps
+            for k, s_ in enumerate(parts):
+                K.kfl_stage_decode(s_, ids_all[j] if (k == 0 and ids_all is not None) else None,
+                                   (hid_all[j] if hid_all is not None else None) if k == 0 else hbuf[k - 1],
+                                   pos_all[j], b, hbuf[k], nxt if k == len(parts) - 1 else None, stream.cuda_stream)
+
+        exact = True
+        ref_h = torch.empty(b, d, dtype=torch.float32, device="cuda")
+        ref_n = torch.empty(b, dtype=torch.int32, device="cuda") if work.logits_out else None
+        for i in range(n_check):
+            chain(i)
+            K.kfl_stage_decode(st_full, ids_all[i] if ids_all is not None else None,
+                               hid_all[i] if hid_all is not None else None, pos_all[i], b, ref_h, ref_n,
+                               stream.cuda_stream)
+            torch.cuda.synchronize()
+            exact = exact and torch.equal(ref_h, hbuf[-1]) and (ref_n is None or torch.equal(ref_n, nxt))
+        for i in range(n_check, n_check + 3):
+            chain(i)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for i in range(n_time):
+            chain(n_check + 3 + i)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / n_time
+        for s_ in parts:
+            if K.kfl_stage_status(s_) != 0:
+                raise RuntimeError("device reported an error in a split stage")
+            K.kfl_stage_destroy(s_)
+        res.append({"split": list(split), "ms_per_step": ms, "us_per_layer_token": ms * 1e3 / (work.n_layers * b),
+                    "steps_timed": n_time, "bit_exact_vs_single_stage": bool(exact),
+                    "steps_compared": n_check})
+    return res
+
 
 def run_ours(args, work):
     import numpy as np
@@ -265,10 +350,8 @@ def run_ours(args, work):
     torch.cuda.synchronize()
     clk = clocks.stop()
     ms = ev0.elapsed_time(ev1) / args.steps
+    ms = max_over_ranks(ms, dist, "cuda")
     if dist:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
         dist.barrier()
     status = K.kfl_stage_status(st)
     if status != 0:
@@ -323,15 +406,14 @@ def run_ours(args, work):
     for s in range(e2e_steps):
         e2e_step(s)
     e2e_s = (time.perf_counter() - t0) / e2e_steps
-    if dist:
-        t = torch.tensor([e2e_s], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = max_over_ranks(e2e_s, dist, "cuda")
     e2e_value = e2e_s * 1e6 / (n_layers * b) / world
+
+    splits = run_splits(work, st, ids_all, hid_all, pos_all, args, stream) if work.splits and world == 1 else None
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        sec, n, cores = oracle_layer_seconds(work, 3)
+        sec, n, cores = oracle_layer_seconds(work, 64, budget_s=10.0)
         cpu = {"value": sec * 1e6, "unit": UNIT, "cores": cores, "kind": "oracle",
                "sample": f"{n} decode steps of one block (block {work.l0}) of {work.name}, fp64 numpy"}
 
@@ -360,6 +442,8 @@ def run_ours(args, work):
             "clocks": clk,
             "cpu_baseline": cpu,
         }
+        if splits is not None:
+            line["splits"] = splits
         print(json.dumps(line), flush=True)
     K.kfl_stage_destroy(st)
     if dist:
