@@ -203,10 +203,11 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
   float acc[NT][4];
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
-  // q as A fragments.  Within each K step of 8 dimensions the MMA's k = tig, tig + 4 are taken as
-  // dimensions 2 tig, 2 tig + 1 (the same order for q and K: the dot product is unchanged), so
-  // that a lane's two K values are one 32-bit load.
-  uint32_t qa0[KS], qa2[KS];
+  // q as A fragments, made from shared memory at each K step.  Within a step of 8 dimensions the
+  // MMA's k = tig, tig + 4 are taken as dimensions 2 tig, 2 tig + 1 (the same order for q and K:
+  // the dot product is unchanged), so that a lane's two K values are one 32-bit load.  q is
+  // carried as a TF32 pair (rounded, rest) so that the scores keep about fp32 precision: the
+  // softmax turns a relative error e of a score s into an error of about |s| e of its weight.
 
   const int nsub = (end - start + ATT_SUB - 1) / ATT_SUB;
   for (int it = 0; it < nsub; ++it) {
@@ -224,15 +225,6 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
     const int cnt = min(ATT_SUB, end - p0);
     const uint8_t *kb = sk + buf * ATT_SUB * L::KROW;
     uint8_t *vb = sv + buf * ATT_SUB * L::VROW;
-    if (it == 0) {
-#pragma unroll
-      for (int s8 = 0; s8 < KS; ++s8) {
-        const float2 qv = hrow ? *reinterpret_cast<const float2 *>(sq + gid * L::QS + 8 * s8 + 2 * tig)
-                               : make_float2(0.f, 0.f);
-        qa0[s8] = to_tf32(qv.x);
-        qa2[s8] = to_tf32(qv.y);
-      }
-    }
     // rows past the sub-tile's positions take part in P V with weight 0: make them finite
     if (cnt < ATT_SUB)
       for (int e = tid; e < (ATT_SUB - cnt) * (HD / 8); e += ATT_THREADS)
@@ -244,8 +236,13 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
       const uint8_t *krow = kb + (8 * warp + gid) * L::KROW + 4 * tig;
 #pragma unroll
       for (int s8 = 0; s8 < KS; ++s8) {
+        const float2 qv = hrow ? *reinterpret_cast<const float2 *>(sq + gid * L::QS + 8 * s8 + 2 * tig)
+                               : make_float2(0.f, 0.f);
+        const uint32_t qh0 = to_tf32(qv.x), qh2 = to_tf32(qv.y);
         const uint32_t kw = *reinterpret_cast<const uint32_t *>(krow + 16 * s8);
-        mma_tf32(sc, qa0[s8], qa2[s8], kw << 16, kw & 0xFFFF0000u);
+        mma_tf32(sc, qh0, qh2, kw << 16, kw & 0xFFFF0000u);
+        mma_tf32(sc, to_tf32(qv.x - __uint_as_float(qh0)), to_tf32(qv.y - __uint_as_float(qh2)), kw << 16,
+                 kw & 0xFFFF0000u);
       }
       if (hrow) {
         const int pp = 8 * warp + 2 * tig;

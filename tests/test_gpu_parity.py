@@ -5,6 +5,8 @@ user and step; greedy ids identical where the oracle's top-2 logit margin exceed
 addressing bit-exact (every slot not written is unchanged, written slots hold the new K/V).
 Everything goes through the C ABI.
 """
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -274,3 +276,44 @@ def test_config5_width_int4_head_b4():
     p = Pair(w.model, 79, 80, K.KFL_IS_HEAD, 4, w.contexts, w.max_ctx, w.seed, device_weights=True)
     _greedy(p, 1, wl.token_ids(w.seed, 97, 4, w.model.vocab))
     p.close()
+
+
+@pytest.mark.parametrize("batch", [1, 4])
+def test_int4_deep_stack_finite_and_split_bit_exact(batch):
+    # eight 72B-shaped int4 blocks: the residual stream of the seeded model grows block after block
+    # (the GEMV input h * g is not normalized), so a narrow activation type would overflow here;
+    # the stack as one stage and as stages [0, 3) + [3, 8) must agree bit for bit
+    from paper_2609_34045_gb300 import device_inputs as dev_in
+    w = wl.CONFIGS[5]
+    m = w.model
+    ctx = tuple(64 + 9 * u for u in range(batch))
+    work = dataclasses.replace(w, l1=8, batch=batch, contexts=ctx)
+    cfg = K.model_cfg(m, work.max_ctx, batch)
+    stream = torch.cuda.current_stream().cuda_stream
+
+    def make(l0, l1, flags):
+        st = K.kfl_stage_create(cfg, l0, l1, flags)
+        dev_in.load_stage_seeded(st, work, l0, l1)
+        cap = torch.zeros(l1 - l0, batch, m.d_model, device="cuda")
+        K.kfl_stage_debug_capture(st, cap)
+        return st, cap
+
+    full, capf = make(0, 8, K.KFL_EMBED_IN)
+    a, capa = make(0, 3, K.KFL_EMBED_IN)
+    c, capc = make(3, 8, 0)
+    h = torch.empty(batch, m.d_model, device="cuda")
+    out_f = torch.empty_like(h)
+    out_c = torch.empty_like(h)
+    for s in range(2):
+        ids = torch.tensor(wl.token_ids(w.seed, 300 + s, batch, m.vocab), device="cuda")
+        pos = torch.tensor([p + s for p in ctx], dtype=torch.int32, device="cuda")
+        K.kfl_stage_decode(full, ids, None, pos, batch, out_f, None, stream)
+        K.kfl_stage_decode(a, ids, None, pos, batch, h, None, stream)
+        K.kfl_stage_decode(c, None, h, pos, batch, out_c, None, stream)
+        torch.cuda.synchronize()
+        assert torch.isfinite(capf).all(), "non-finite hidden state in the int4 stack"
+        assert torch.equal(capf, torch.cat([capa, capc]))
+        assert torch.equal(out_f, out_c)
+    for st in (full, a, c):
+        assert K.kfl_stage_status(st) == 0
+        K.kfl_stage_destroy(st)
