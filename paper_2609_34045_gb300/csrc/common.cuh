@@ -22,7 +22,8 @@ constexpr int CONSUMER_WARPS = 8;
 constexpr int GEMV_THREADS = (CONSUMER_WARPS + 2) * 32;  // consumers, producer, epilogue warp
 constexpr int MAX_STAGES = 12;
 
-// int4 group-64 tiles: [N/RB][K/KT4][RB][KT4/8] uint32 codes then [RB][KT4/64] bf16 scales
+// int4 group-64 tiles: [N/RB][K/KT4], each 64 x 256 codes (8 KiB, in the order of the
+// tensor-core MMA fragments, see repack_int4_kernel) then [RB][KT4/64] bf16 scales
 constexpr int KT4 = 256;
 constexpr int TILE4_CODE_BYTES = RB * KT4 / 2;     // 8 KiB
 constexpr int TILE4_SCALE_BYTES = RB * (KT4 / 64) * 2;  // 512 B
@@ -31,8 +32,11 @@ constexpr int TILE4_BYTES = TILE4_CODE_BYTES + TILE4_SCALE_BYTES;
 // A ring stage holds one weight tile and the B users' fp32 activation chunks of its K range.
 __host__ __device__ constexpr int tile_k(int fmt) { return fmt == 0 ? KT : KT4; }
 __host__ __device__ constexpr int tile_bytes(int fmt) { return fmt == 0 ? TILE_BYTES : TILE4_BYTES; }
+// int4 stages also carry the activation multipliers of the tile (XCHUNK-element chunks x MAXB)
+constexpr int XCHUNK = 32;
+constexpr int XMUL_TILE_BYTES = (KT4 / XCHUNK) * MAXB * 4;  // 128
 __host__ __device__ constexpr int stage_bytes(int batch, int fmt) {
-  return (tile_bytes(fmt) + batch * tile_k(fmt) * 4 + 127) / 128 * 128;
+  return (tile_bytes(fmt) + batch * tile_k(fmt) * 4 + (fmt == 0 ? 0 : XMUL_TILE_BYTES) + 127) / 128 * 128;
 }
 constexpr int STAGE_BYTES_MAX = stage_bytes(MAXB, 0);
 
@@ -87,6 +91,12 @@ struct GemvParams {
   const float *rope_cos, *rope_sin;  // [max_ctx][hd/2], or [batch][hd/2] when rope_per_user
   int rope_per_user;
   int n_q_rows, n_kv_rows, head_dim, max_ctx, n_kv_heads;
+  // int4 weights: the GEMV multiplies fp16 activations on the tensor cores.  Each producer of an
+  // int4 GEMV's input stores it scaled by a power of two per XCHUNK elements (so that it fits
+  // fp16) with the multiplier that undoes it: x_true[k] = x[k] * xmul[k / XCHUNK][b].
+  const float *xmul;  // this GEMV's input multipliers [chunks][MAXB] (int4), else NULL
+  float *xmul_out;    // RESID / SWIGLU: multipliers of the output written (int4 stages), else NULL
+  int xsplit;         // activations carried as an fp16 pair (rounded, rest): Q/K/V projection
   // EPI_ARGMAX
   float *cand_val;
   int *cand_idx;
@@ -311,6 +321,17 @@ __device__ __forceinline__ unsigned atom_add_acq_rel(unsigned *p, unsigned v) {
 __device__ __forceinline__ void red_add_release(unsigned *p, unsigned v) {
   asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
+// The power of two 2^e that a chunk of values with largest magnitude m is divided by so that it
+// fits fp16 with its largest value in [2^14, 2^15) (exact: a power of two); *inv = 2^-e.  A chunk
+// of zeros gets 1.
+__device__ __forceinline__ float xchunk_scale(float m, float *inv) {
+  int e = 0;
+  if (m > 0.f) e = static_cast<int>((__float_as_uint(m) >> 23) & 0xFF) - 127 - 14;
+  e = max(-100, min(100, e));
+  *inv = __uint_as_float(static_cast<uint32_t>(127 - e) << 23);
+  return __uint_as_float(static_cast<uint32_t>(127 + e) << 23);
+}
+
 __device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned *p) {
   unsigned v;
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -329,7 +350,8 @@ cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s, 
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in,
                                int batch, const uint16_t *embed, int vocab, int d, int ldh,
                                const float *g_next, float *h, float *xn, float *sumsq,
-                               int *positions, int max_ctx, unsigned *err, unsigned *bar, cudaStream_t s);
+                               int *positions, int max_ctx, unsigned *err, unsigned *bar, float *xmul,
+                               cudaStream_t s);
 size_t stage_kernel_smem(int stages, int head_dim, int batch, int fmt);
 int stage_kernel_attn_bytes(int head_dim);
 cudaError_t prepare_stage_kernel(size_t smem);

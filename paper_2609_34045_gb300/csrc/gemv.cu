@@ -65,6 +65,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
     s_issued = 0;
     fence_mbar_init();
   }
+  for (int e = tid; e < NSLOT * RB * MAXB; e += GEMV_THREADS) red[e] = 0.f;  // int4 tiles add into it
   __syncthreads();
   pdl_launch_dependents();
   auto stamp = [&](int slot) {
@@ -77,7 +78,8 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
     if (lane == 0) {
       const uint64_t pol_w = policy_evict_first();
       const uint64_t pol_x = policy_evict_last();
-      const uint32_t xbytes = B * (KTILE * 4);
+      // int4: the tile's activation multipliers follow the activations
+      const uint32_t xbytes = B * (KTILE * 4) + (FMT == 1 ? XMUL_TILE_BYTES : 0);
       const int pre = n < S ? n : S;
       stamp(TR_W_FIRST);
       for (int i = 0; i < pre; ++i) {
@@ -94,6 +96,8 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
 #pragma unroll
         for (int b = 0; b < B; ++b)
           bulk_g2s(dst + b * (KTILE * 4), p.x + (size_t)b * p.ldx + (size_t)kt * KTILE, KTILE * 4, fb, pol_x);
+        if constexpr (FMT == 1)
+          bulk_g2s(dst + B * (KTILE * 4), p.xmul + (size_t)kt * (KT4 / XCHUNK) * MAXB, XMUL_TILE_BYTES, fb, pol_x);
       };
       int kt_x = static_cast<int>(t0 % p.n_kt);
       for (int i = 0; i < pre; ++i) {
@@ -133,7 +137,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) ge
   // -------------------------------------------------------------------- consumers
   int s = 0, segc = 0;
   uint32_t phase = 0;
-  gemv_consume<B, FMT>(p.n_kt, smem, full, empty, S, s, phase, t0, n, sr, segc, &s_abort, p.err, tid);
+  gemv_consume<B, FMT>(p.n_kt, smem, full, empty, S, s, phase, t0, n, sr, segc, &s_abort, p.err, tid, p.xsplit != 0);
 
   consumer_sync();
   if (tid == 0) stamp(TR_CONS_ENTER);

@@ -126,44 +126,100 @@ __device__ __forceinline__ void tile_compute(const uint8_t *st, int warp, int la
         for (int b = 0; b < B; ++b) ffma2(acc[b][j][0], acc[b][j][1], wl, wh, xv[b][2 * e], xv[b][2 * e + 1]);
       }
     }
-  } else {
-    // int4 tile: codes [RB][KT4/8] uint32 (32 words = 128 B per row), scales [RB][4] bf16.
-    // The lane's 16 codes of a row (two words, one scale group) are taken a word at a time so
-    // that only 8 activations per user are live.
-    const float4 *xp = reinterpret_cast<const float4 *>(st + TILE4_BYTES) + kc * 4;
-    const uint2 *cp = reinterpret_cast<const uint2 *>(st) + (warp * 8 + rsub) * (KT4 / 16) + kc;
-    const uint16_t *sp = reinterpret_cast<const uint16_t *>(st + TILE4_CODE_BYTES);
-    uint2 cw[4];
-    float sc[4];
+  }
+}
+
+// d += a b for one m16n8k16 fp16 tile (a: 16x16 row-major, b: 16x8 column-major, fp32 accumulate)
+__device__ __forceinline__ void mma_f16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                               uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Two 4-bit codes (bits 0-3 and 16-19 of w) as an fp16 pair of their signed values: the nibble,
+// with its top bit flipped, as the low mantissa bits of 1024 gives 1024 + (n ^ 8) = 1032 + code;
+// subtracting 1032 is exact.
+__device__ __forceinline__ uint32_t int4_pair_f16(uint32_t w) {
+  uint32_t r;
+  asm("lop3.b32 %0, %1, %2, %3, 0x6A;" : "=r"(r) : "r"(w), "r"(0x000F000Fu), "r"(0x64086408u));  // (w & m) ^ c
+  uint32_t d;
+  asm("fma.rn.f16x2 %0, %1, %2, %3;" : "=r"(d) : "r"(r), "r"(0x3C003C00u), "r"(0xE408E408u));  // r * 1 - 1032
+  return d;
+}
+
+// fp32 pair -> fp16 pair (round to nearest even), lo in the low half
+__device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// fp32 pair -> the fp16 pair of what rounding it to fp16 left over (x - fp16(x), rounded): with
+// the rounded pair it carries x to about 2^-22
+__device__ __forceinline__ uint32_t pack_f16x2_rest(float lo, float hi, uint32_t rounded) {
+  float rl, rh;
+  asm("{\n\t.reg .f16 l, h;\n\tmov.b32 {l, h}, %2;\n\tcvt.f32.f16 %0, l;\n\tcvt.f32.f16 %1, h;\n\t}"
+      : "=f"(rl), "=f"(rh)
+      : "r"(rounded));
+  return pack_f16x2(lo - rl, hi - rh);
+}
+
+// int4 tile (FMT 1) on the tensor cores.  Warp w takes row group r16 = w % 4 (16 rows) and K half
+// h = w / 4 (128 of the tile's 256 K): per K step of 16, one m16n8k16 MMA of the codes (exact in
+// fp16) against the users' activations (stored pre-scaled per 32 elements, rounded to fp16:
+// 2^-11 relative; columns past B are 0); each 32-element chunk's product is multiplied back by its
+// multiplier and the weights' group scale into acc.  acc[0..1]: row r16*16 + gid, users 2 tig,
+// 2 tig + 1; acc[2..3]: row + 8.
+// XSPLIT (Q/K/V projection, whose errors the attention softmax amplifies): each activation is
+// carried as an fp16 pair (rounded, rest), the rounded parts in columns 0-3, the rests in 4-7
+// (B <= 4); the two are added at the end of the row block.
+template <int B, bool XSPLIT>
+__device__ __forceinline__ void tile_compute_int4(const uint8_t *st, int warp, int lane, float (&acc)[4]) {
+  const int r16 = warp & 3, h = warp >> 2, gid = lane >> 2, tig = lane & 3;
+  const uint4 *cw = reinterpret_cast<const uint4 *>(st) + (h * 4 + r16) * 2 * 32 + lane;
+  const uint4 wq[2] = {cw[0], cw[32]};
+  const uint32_t *sp = reinterpret_cast<const uint32_t *>(st + TILE4_CODE_BYTES);
+  const uint32_t s0 = sp[(r16 * 16 + gid) * 2 + h], s1 = sp[(r16 * 16 + gid + 8) * 2 + h];
+  const int xu_id = XSPLIT ? (gid & 3) : gid;
+  const float *xs = reinterpret_cast<const float *>(st + TILE4_BYTES) + xu_id * KT4 + 128 * h + 2 * tig;
+  const bool xu = xu_id < B;
+  // multipliers [8 chunks][MAXB] after the activations; this lane's columns are users
+  // (2 tig) & 3 and (2 tig + 1) & 3 (the rest parts of XSPLIT in columns 4-7 share them)
+  const float *xm = reinterpret_cast<const float *>(st + TILE4_BYTES + B * KT4 * 4) + (2 * tig & 3);
+  const bool mu0 = (2 * tig & 3) < B, mu1 = ((2 * tig + 1) & 3) < B;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      cw[j] = cp[j * 2 * (KT4 / 16)];
-      sc[j] = bf16_to_f32(sp[(warp * 8 + rsub + 2 * j) * (KT4 / 64) + (kc >> 2)]);
-    }
+  for (int q = 0; q < 2; ++q) {
+    const float sc0 = q ? bf16_hi(s0) : bf16_lo(s0), sc1 = q ? bf16_hi(s1) : bf16_lo(s1);
 #pragma unroll
-    for (int hw = 0; hw < 2; ++hw) {
-      float xv[B][8];
+    for (int half = 0; half < 2; ++half) {
+    float c[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int b = 0; b < B; ++b) {
-        const float4 a0 = xp[b * (KT4 / 4) + 2 * hw], a1 = xp[b * (KT4 / 4) + 2 * hw + 1];
-        xv[b][0] = a0.x; xv[b][1] = a0.y; xv[b][2] = a0.z; xv[b][3] = a0.w;
-        xv[b][4] = a1.x; xv[b][5] = a1.y; xv[b][6] = a1.z; xv[b][7] = a1.w;
-      }
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const uint32_t word = hw ? cw[j].y : cw[j].x;
-        float part[B][2];
-#pragma unroll
-        for (int b = 0; b < B; ++b) part[b][0] = part[b][1] = 0.f;
-#pragma unroll
-        for (int e = 0; e < 8; e += 2) {
-          const float q0 = int4_code(word, e), q1 = int4_code(word, e + 1);
-#pragma unroll
-          for (int b = 0; b < B; ++b) ffma2(part[b][0], part[b][1], q0, q1, xv[b][e], xv[b][e + 1]);
+    for (int j = 2 * half; j < 2 * half + 2; ++j) {
+      const uint32_t w = j == 0 ? wq[q].x : j == 1 ? wq[q].y : j == 2 ? wq[q].z : wq[q].w;
+      const int k0 = 16 * (4 * q + j);
+      uint32_t b0 = 0u, b1 = 0u;
+      if (xu) {
+        const float2 x0 = *reinterpret_cast<const float2 *>(xs + k0);
+        const float2 x1 = *reinterpret_cast<const float2 *>(xs + k0 + 8);
+        b0 = pack_f16x2(x0.x, x0.y);
+        b1 = pack_f16x2(x1.x, x1.y);
+        if (XSPLIT && gid >= 4) {
+          b0 = pack_f16x2_rest(x0.x, x0.y, b0);
+          b1 = pack_f16x2_rest(x1.x, x1.y, b1);
         }
-#pragma unroll
-        for (int b = 0; b < B; ++b) ffma2(acc[b][j][0], acc[b][j][1], sc[j], sc[j], part[b][0], part[b][1]);
       }
+      mma_f16_16816(c, int4_pair_f16(w), int4_pair_f16(w >> 4), int4_pair_f16(w >> 8), int4_pair_f16(w >> 12), b0, b1);
+    }
+    // chunk h * 4 + 2 q + half of the tile: its multipliers, then the rows' group scales
+    const float2 m = *reinterpret_cast<const float2 *>(xm + (h * 4 + 2 * q + half) * MAXB);
+    const float m0 = mu0 ? m.x : 0.f, m1 = mu1 ? m.y : 0.f;
+    acc[0] = fmaf(sc0 * m0, c[0], acc[0]);
+    acc[1] = fmaf(sc0 * m1, c[1], acc[1]);
+    acc[2] = fmaf(sc1 * m0, c[2], acc[2]);
+    acc[3] = fmaf(sc1 * m1, c[3], acc[3]);
     }
   }
 }
@@ -182,42 +238,72 @@ struct SegRing {
 template <int B, int FMT>
 __device__ __forceinline__ void gemv_consume(int n_kt, uint8_t *ring, uint64_t *full, uint64_t *empty, int S, int &s,
                                              uint32_t &phase, long long t0, int n, const SegRing &sr, int &segc,
-                                             volatile int *abort_flag, unsigned *err, int tid) {
+                                             volatile int *abort_flag, unsigned *err, int tid, bool xsplit) {
   const int warp = tid >> 5, lane = tid & 31, kc = lane & 15, rsub = lane >> 4;
-  float acc[B][4][2];
+  float acc[B][4][2];   // bf16 tiles: rows warp*8 + rsub + 2j, this lane's K chunk
+  float acc4[4];        // int4 tiles (tensor cores): see tile_compute_int4
   int kt = static_cast<int>(t0 % n_kt);
   for (int i = 0; i < n; ++i) {
     if (i == 0 || kt == 0) {
+      if constexpr (FMT == 0) {
 #pragma unroll
-      for (int b = 0; b < B; ++b)
+        for (int b = 0; b < B; ++b)
 #pragma unroll
-        for (int j = 0; j < 4; ++j) acc[b][j][0] = acc[b][j][1] = 0.f;
+          for (int j = 0; j < 4; ++j) acc[b][j][0] = acc[b][j][1] = 0.f;
+      } else {
+        acc4[0] = acc4[1] = acc4[2] = acc4[3] = 0.f;
+      }
     }
     consumer_wait(smem_addr(&full[s]), phase, abort_flag, err);
-    tile_compute<B, FMT>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc);
+    if constexpr (FMT == 0)
+      tile_compute<B, FMT>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc);
+    else if (xsplit)
+      tile_compute_int4<B, true>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc4);
+    else
+      tile_compute_int4<B, false>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc4);
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_addr(&empty[s]));
     if (kt == n_kt - 1 || i == n - 1) {
-      float tot[B][4];
-#pragma unroll
-      for (int b = 0; b < B; ++b)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          float v = acc[b][j][0] + acc[b][j][1];
-          v += __shfl_xor_sync(0xffffffffu, v, 8);
-          v += __shfl_xor_sync(0xffffffffu, v, 4);
-          v += __shfl_xor_sync(0xffffffffu, v, 2);
-          v += __shfl_xor_sync(0xffffffffu, v, 1);
-          tot[b][j] = v;
-        }
       const int slot = segc % NSLOT, use = segc / NSLOT;
-      if (use > 0) consumer_wait(smem_addr(&sr.empty[slot]), (use - 1) & 1, abort_flag, err);
-      if (kc == 0) {
-        float *rd = sr.red + slot * RB * MAXB;
+      float *rd = sr.red + slot * RB * MAXB;
+      if constexpr (FMT == 0) {
+        float tot[B][4];
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
+        for (int b = 0; b < B; ++b)
 #pragma unroll
-          for (int b = 0; b < B; ++b) rd[(warp * 8 + rsub + 2 * j) * MAXB + b] = tot[b][j];
+          for (int j = 0; j < 4; ++j) {
+            float v = acc[b][j][0] + acc[b][j][1];
+            v += __shfl_xor_sync(0xffffffffu, v, 8);
+            v += __shfl_xor_sync(0xffffffffu, v, 4);
+            v += __shfl_xor_sync(0xffffffffu, v, 2);
+            v += __shfl_xor_sync(0xffffffffu, v, 1);
+            tot[b][j] = v;
+          }
+        if (use > 0) consumer_wait(smem_addr(&sr.empty[slot]), (use - 1) & 1, abort_flag, err);
+        if (kc == 0) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+#pragma unroll
+            for (int b = 0; b < B; ++b) rd[(warp * 8 + rsub + 2 * j) * MAXB + b] = tot[b][j];
+        }
+      } else {
+        // the two K halves of a row group add into the slot, which the epilogue warp left at
+        // zero: two additions per value, so the order does not change the sum
+        if (xsplit) {
+          // rounded part (columns 0-3, lanes tig < 2) + rest (columns 4-7, lanes tig + 2)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc4[v] += __shfl_down_sync(0xffffffffu, acc4[v], 2);
+        }
+        if (use > 0) consumer_wait(smem_addr(&sr.empty[slot]), (use - 1) & 1, abort_flag, err);
+        const int gid = lane >> 2, tig = lane & 3, r0 = (warp & 3) * 16 + gid;
+        if (2 * tig < B) {
+          atomicAdd(rd + r0 * MAXB + 2 * tig, acc4[0]);
+          atomicAdd(rd + (r0 + 8) * MAXB + 2 * tig, acc4[2]);
+        }
+        if (2 * tig + 1 < B) {
+          atomicAdd(rd + r0 * MAXB + 2 * tig + 1, acc4[1]);
+          atomicAdd(rd + (r0 + 8) * MAXB + 2 * tig + 1, acc4[3]);
+        }
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_addr(&sr.full[slot]));
@@ -290,11 +376,23 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
 #pragma unroll
       for (int h2 = 0; h2 < 2; ++h2) {
         const int r = lane + 32 * h2, n = rb * RB + r;
-        if (n < p.n_rows) {
-          const size_t o = (size_t)b * p.ldh + n;
-          const float hn = pre.h[b][h2] + red[r * MAXB + b] * inv[b];
+        const bool ok = n < p.n_rows;
+        const size_t o = (size_t)b * p.ldh + n;
+        const float hn = ok ? pre.h[b][h2] + red[r * MAXB + b] * inv[b] : 0.f;
+        float xv = hn * pre.g[h2];
+        if (p.xmul_out && p.g_next) {
+          // int4 stage: xn in 32-row chunks scaled to fit fp16, with their multipliers
+          float mx = fabsf(xv);
+#pragma unroll
+          for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+          float iv;
+          const float mul = xchunk_scale(mx, &iv);
+          xv *= iv;
+          if (lane == 0) p.xmul_out[(rb * 2 + h2) * MAXB + b] = mul;
+        }
+        if (ok) {
           p.h[o] = hn;
-          if (p.g_next) p.xn[o] = hn * pre.g[h2];
+          if (p.g_next) p.xn[o] = xv;
           if (p.capture) p.capture[(size_t)b * p.n_rows + n] = hn;
           sq = fmaf(hn, hn, sq);
         }
@@ -303,13 +401,28 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
       if (lane == 0) p.sumsq_out[rb * MAXB + b] = sq;
     }
   } else if constexpr (EPI == EPI_SWIGLU) {
-    for (int e = lane; e < (RB / 2) * B; e += 32) {
-      const int b = e / (RB / 2), pr = e % (RB / 2), j = rb * (RB / 2) + pr;
-      if (2 * j < p.n_rows) {
+    // lane = output (RB / 2 = 32 of them per row block), one user per pass
+#pragma unroll
+    for (int b = 0; b < B; ++b) {
+      const int pr = lane, j = rb * (RB / 2) + pr;
+      const bool ok = 2 * j < p.n_rows;
+      float a = 0.f;
+      if (ok) {
         const float g = red[(2 * pr) * MAXB + b] * inv[b];
         const float u = red[(2 * pr + 1) * MAXB + b] * inv[b];
-        p.out[(size_t)b * p.ldo + j] = g / (1.0f + expf(-g)) * u;
+        a = g / (1.0f + expf(-g)) * u;
       }
+      if (p.xmul_out) {
+        // int4 stage: the row block's 32 outputs scaled to fit fp16, with their multiplier
+        float mx = fabsf(a);
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+        float iv;
+        const float mul = xchunk_scale(mx, &iv);
+        a *= iv;
+        if (lane == 0) p.xmul_out[rb * MAXB + b] = mul;
+      }
+      if (ok) p.out[(size_t)b * p.ldo + j] = a;
     }
   } else if constexpr (EPI == EPI_QKV) {
     const int hd = p.head_dim, half = hd >> 1;
@@ -489,6 +602,9 @@ __device__ __forceinline__ void gemv_epilogues(const GemvParams &p, long long t0
         if (p.out_done) red_add_release(p.out_done, 1u);
       }
     }
+    __syncwarp();
+    // leave the slot at zero: int4 tiles add into it
+    for (int e = lane; e < RB * MAXB / 4; e += 32) reinterpret_cast<float4 *>(red)[e] = make_float4(0.f, 0.f, 0.f, 0.f);
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_addr(&sr.empty[slot]));
   }

@@ -11,7 +11,7 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
                                                          const int *positions_in, const uint16_t *embed,
                                                          int vocab, int d, int ldh, const float *g_next,
                                                          float *h, float *xn, float *sumsq, int *positions,
-                                                         int max_ctx, unsigned *err, unsigned *bar) {
+                                                         int max_ctx, unsigned *err, unsigned *bar, float *xmul) {
   __shared__ float vals[64];
   const int b = blockIdx.y, tid = threadIdx.x, r = blockIdx.x * 64 + tid;
   pdl_launch_dependents();
@@ -39,7 +39,21 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
       v = hidden_in[(size_t)b * d + r];
     }
     h[(size_t)b * ldh + r] = v;
-    if (g_next) xn[(size_t)b * ldh + r] = v * g_next[r];
+  }
+  if (g_next) {
+    // xn = h * g; for int4 weights in 32-element chunks scaled to fit fp16 (one warp per chunk),
+    // exactly as the residual epilogue writes it
+    float xv = r < d ? v * g_next[r] : 0.f;
+    if (xmul) {
+      float mx = fabsf(xv);
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+      float iv;
+      const float mul = xchunk_scale(mx, &iv);
+      xv *= iv;
+      if ((tid & 31) == 0) xmul[(blockIdx.x * 2 + (tid >> 5)) * MAXB + b] = mul;
+    }
+    if (r < d) xn[(size_t)b * ldh + r] = xv;
   }
   // the block's sum of squares in exactly the order of the residual epilogue (lane l: rows l
   // and l + 32 by fma, then a butterfly), so that a stage fed this hidden state computes the same
@@ -58,10 +72,10 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in, int batch,
                                const uint16_t *embed, int vocab, int d, int ldh, const float *g_next, float *h,
                                float *xn, float *sumsq, int *positions, int max_ctx, unsigned *err,
-                               unsigned *bar, cudaStream_t s) {
+                               unsigned *bar, float *xmul, cudaStream_t s) {
   dim3 grid((d + 63) / 64, batch);
   stage_input_kernel<<<grid, 64, 0, s>>>(ids, hidden_in, positions_in, embed, vocab, d, ldh, g_next, h, xn, sumsq,
-                                         positions, max_ctx, err, bar);
+                                         positions, max_ctx, err, bar, xmul);
   return cudaGetLastError();
 }
 
@@ -127,32 +141,51 @@ cudaError_t launch_repack_bf16(const uint16_t *src, int n_src_rows, int k, const
 
 // Repack an int4 group-64 matrix (words [n_src_rows][k/8], scales [n_src_rows][k/64]) into
 // tiles [n_rb][n_kt][RB][KT4/8 words] followed by [RB][KT4/64] bf16 scales per tile.
+// int4 tiles in the order of the tensor-core MMA fragments (tile_compute, FMT 1): the 64 x 256
+// codes of a tile are 2048 words; word ((((h * 4 + r16) * 2 + q) * 32 + lane) * 4 + j) holds the
+// eight codes lane needs for K step s = 4 q + j of K half h and row group r16 (rows r16 * 16 +
+// gid and + 8, gid = lane / 4; columns 2 tig, 2 tig + 1, 2 tig + 8, 2 tig + 9 of the step, tig =
+// lane % 4), nibble i at bits 4 i: row + 8 (i & 1), column + 8 ((i >> 1) & 1) + ((i >> 2) & 1), so
+// that (word >> 4 i) & 0x000F000F, i < 4, is the bf16 pair of one A register.  Scales stay
+// [64 rows][4 groups of 64].
 __global__ void repack_int4_kernel(const uint32_t *words, const uint16_t *scales, int n_src_rows, int k,
                                    const int *row_map, int n_rows_out, int n_rb, int n_kt, uint8_t *dst) {
-  constexpr int WPR = KT4 / 8;   // words per tile row
-  constexpr int SPR = KT4 / 64;  // scales per tile row
-  const long long total = (long long)n_rb * n_kt * RB;
+  constexpr int TW = TILE4_CODE_BYTES / 4;  // words per tile
+  constexpr int SPR = KT4 / 64;             // scales per tile row
   const int kw = k / 8, ks = k / 64;
+  const long long total = (long long)n_rb * n_kt * TW;
   for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
        e += (long long)gridDim.x * blockDim.x) {
-    const int r = static_cast<int>(e % RB);
-    const long long t = e / RB;
+    const int idx = static_cast<int>(e % TW);
+    const long long t = e / TW;
     const int kt = static_cast<int>(t % n_kt);
     const int rb = static_cast<int>(t / n_kt);
-    const int orow = rb * RB + r;
-    int srow = -1;
-    if (orow < n_rows_out) srow = row_map ? row_map[orow] : orow;
-    if (srow >= n_src_rows) srow = -1;
-    uint8_t *tile = dst + (size_t)t * TILE4_BYTES;
-    uint32_t *wd = reinterpret_cast<uint32_t *>(tile) + r * WPR;
-    uint16_t *sd = reinterpret_cast<uint16_t *>(tile + TILE4_CODE_BYTES) + r * SPR;
-    for (int j = 0; j < WPR; ++j) {
-      const int w = kt * WPR + j;
-      wd[j] = (srow >= 0 && w < kw) ? words[(size_t)srow * kw + w] : 0u;
+    const int j = idx & 3, lane = (idx >> 2) & 31, q = (idx >> 7) & 1, r16 = (idx >> 8) & 3, h = idx >> 10;
+    const int gid = lane >> 2, tig = lane & 3;
+    uint32_t out = 0;
+    for (int i = 0; i < 8; ++i) {
+      const int orow = rb * RB + r16 * 16 + gid + 8 * (i & 1);
+      const int kk = kt * KT4 + 128 * h + 16 * (4 * q + j) + 2 * tig + 8 * ((i >> 1) & 1) + ((i >> 2) & 1);
+      int srow = -1;
+      if (orow < n_rows_out) srow = row_map ? row_map[orow] : orow;
+      if (srow >= n_src_rows) srow = -1;
+      uint32_t nib = 0;
+      if (srow >= 0 && kk < k) nib = (words[(size_t)srow * kw + kk / 8] >> (4 * (kk % 8))) & 0xFu;
+      out |= nib << (4 * i);
     }
-    for (int j = 0; j < SPR; ++j) {
-      const int g = kt * SPR + j;
-      sd[j] = (srow >= 0 && g < ks) ? scales[(size_t)srow * ks + g] : uint16_t(0);
+    uint8_t *tile = dst + (size_t)t * TILE4_BYTES;
+    reinterpret_cast<uint32_t *>(tile)[idx] = out;
+    if (idx < RB) {
+      // the tile's scales, one row per thread
+      const int orow = rb * RB + idx;
+      int srow = -1;
+      if (orow < n_rows_out) srow = row_map ? row_map[orow] : orow;
+      if (srow >= n_src_rows) srow = -1;
+      uint16_t *sd = reinterpret_cast<uint16_t *>(tile + TILE4_CODE_BYTES) + idx * SPR;
+      for (int g = 0; g < SPR; ++g) {
+        const int gg = kt * SPR + g;
+        sd[g] = (srow >= 0 && gg < ks) ? scales[(size_t)srow * ks + gg] : uint16_t(0);
+      }
     }
   }
 }

@@ -143,6 +143,7 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   size_t ws = 0;
   ws += (size_t)c->max_ctx * (p->hd / 2) * 4 * 2;                      // rope tables
   ws += (size_t)MAXB * (2 * p->ldh + 2 * p->ldq + p->lda) * 4;         // h, xn, q, o, a
+  ws += (size_t)MAXB * (p->ldh + p->ldq + p->lda) / XCHUNK * 4;        // int4 input multipliers
   ws += (size_t)p->n_parts * MAXB * 4;                                 // sum of squares
   ws += 2 * MAXB * 4;                                                  // positions, next ids
   ws += (size_t)4 * p->gemv_grid_max * 2 * RB * MAXB * 4;              // stream-K partials (x4)
@@ -172,6 +173,8 @@ struct kfl_stage {
   uint16_t *kc = nullptr, *vc = nullptr;
   float *rope_cos = nullptr, *rope_sin = nullptr;
   float *h = nullptr, *xn = nullptr, *q = nullptr, *o = nullptr, *a = nullptr, *sumsq = nullptr;
+  // int4 stages: multipliers of the fp16-scaled GEMV inputs ([chunks of 32][MAXB]; o's are 1)
+  float *xn_mul = nullptr, *a_mul = nullptr, *o_mul = nullptr;
   int *pos = nullptr, *next_int = nullptr;
   int *io_pos = nullptr, *io_ids = nullptr;  // host-buffer decode staging
   float *io_hin = nullptr;
@@ -240,7 +243,7 @@ namespace {
 
 bool valid(const kfl_stage *st) { return st && st->magic == 0x4B464C53; }
 
-thread_local char g_last_error[256] = "";
+thread_local char g_last_error[512] = "";
 
 int record_cuda_error(cudaError_t e, const char *what, int line) {
   snprintf(g_last_error, sizeof(g_last_error), "%s (%s) at stage.cu:%d", cudaGetErrorString(e), what, line);
@@ -284,6 +287,7 @@ GemvParams base_gemv(kfl_stage *st, const Mat &m, const float *x, int ldx, int b
 std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk, bool dataflow = false) {
   const Plan &P = st->P;
   const kfl_model_cfg &c = st->cfg;
+  const bool i4 = c.weight_fmt == KFL_INT4_G64;
   std::vector<Phase> ph;
   auto gemv = [&](int epi, const GemvParams &g) {
     Phase x = {};
@@ -294,6 +298,9 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk, bool d
     // of the three before it (in the persistent kernel phases overlap)
     const int r = (int)ph.size() % 4;
     x.g.partial = st->gemv_partial + (size_t)r * P.gemv_grid_max * 2 * RB * MAXB;
+    // int4: the Q/K/V projection carries its activations as an fp16 pair (its errors are
+    // amplified by the attention softmax)
+    x.g.xsplit = (g.fmt == KFL_INT4_G64 && epi == EPI_QKV) ? 1 : 0;
     x.g.tickets = st->tickets + (size_t)r * P.n_rb_max;
     ph.push_back(x);
   };
@@ -318,6 +325,7 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk, bool d
       g.head_dim = P.hd;
       g.max_ctx = c.max_ctx;
       g.n_kv_heads = P.hkv;
+      if (i4) g.xmul = st->xn_mul;
       gemv(EPI_QKV, g);
     }
     {
@@ -349,6 +357,10 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk, bool d
       g.xn = st->xn;
       g.g_next = L.g_ffn;
       g.sumsq_out = st->sumsq;
+      if (i4) {
+        g.xmul = st->o_mul;
+        g.xmul_out = st->xn_mul;
+      }
       gemv(EPI_RESID, g);
     }
     {
@@ -359,6 +371,10 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk, bool d
       g.eps = c.rms_eps;
       g.out = st->a;
       g.ldo = P.lda;
+      if (i4) {
+        g.xmul = st->xn_mul;
+        g.xmul_out = st->a_mul;
+      }
       gemv(EPI_SWIGLU, g);
     }
     {
@@ -369,6 +385,10 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk, bool d
       g.g_next = (l + 1 < P.nl) ? st->layers[l + 1].g_attn : ((st->flags & KFL_LOGITS_OUT) ? st->g_final : nullptr);
       g.sumsq_out = st->sumsq;
       g.capture = st->capture ? st->capture + (size_t)l * c.max_batch * P.d : nullptr;
+      if (i4) {
+        g.xmul = st->a_mul;
+        g.xmul_out = st->xn_mul;
+      }
       gemv(EPI_RESID, g);
     }
   }
@@ -382,6 +402,7 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk, bool d
     g.cand_idx = st->cand_idx;
     g.argmax_ticket = st->am_ticket;
     g.next_ids = st->next_int;
+    if (i4) g.xmul = st->xn_mul;
     gemv(EPI_ARGMAX, g);
   }
   if (!dataflow && st->trace) {
@@ -576,7 +597,8 @@ int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const in
     std::vector<int> kinds;
     CK(cudaEventRecord(st->ev[0], s));
     CK(launch_stage_input(ids, hidden_in, positions, batch, embed ? st->embed : nullptr, P.V, P.d, P.ldh,
-                          input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, st->bar, s));
+                          input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, st->bar,
+                          st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn_mul : nullptr, s));
     CK(cudaEventRecord(st->ev[1], s));
     kinds.push_back(KFL_KERNEL_INPUT);
     int rc = enqueue_body(st, batch, s, false, &kinds, 1);
@@ -596,7 +618,8 @@ int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const in
     return KFL_OK;
   }
   CK(launch_stage_input(ids, hidden_in, positions, batch, embed ? st->embed : nullptr, P.V, P.d, P.ldh,
-                        input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, st->bar, s));
+                        input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, st->bar,
+                        st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn_mul : nullptr, s));
   if (body) {
     int rc = ensure_graph(st, batch);
     if (rc != KFL_OK) return rc;
@@ -777,6 +800,9 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
   AL(st->o, (size_t)MAXB * P.ldq * 4);
   AL(st->a, (size_t)MAXB * P.lda * 4);
   AL(st->sumsq, (size_t)P.n_parts * MAXB * 4);
+  AL(st->xn_mul, (size_t)MAXB * P.ldh / XCHUNK * 4);
+  AL(st->a_mul, (size_t)MAXB * P.lda / XCHUNK * 4);
+  AL(st->o_mul, (size_t)MAXB * P.ldq / XCHUNK * 4);
   AL(st->pos, MAXB * 4);
   AL(st->next_int, MAXB * 4);
   AL(st->gemv_partial, (size_t)4 * P.gemv_grid_max * 2 * RB * MAXB * 4);
@@ -805,8 +831,15 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
       cudaMemset(st->tickets, 0, (size_t)(4 * P.n_rb_max + 1) * 4) ||
       cudaMemset(st->counters, 0, (size_t)std::max(1, P.n_phases) * P.ctr_stride * 4) ||
       cudaMemset(st->attn_tickets, 0, (size_t)MAXB * P.hkv * 4) || cudaMemset(st->err, 0, 16) ||
-      cudaMemset(st->bar, 0, 16))
+      cudaMemset(st->bar, 0, 16) || cudaMemset(st->xn_mul, 0, (size_t)MAXB * P.ldh / XCHUNK * 4) ||
+      cudaMemset(st->a_mul, 0, (size_t)MAXB * P.lda / XCHUNK * 4))
     return fail(KFL_ERR_CUDA);
+  {
+    // the attention output needs no scaling: its multipliers are all 1
+    std::vector<float> ones((size_t)MAXB * P.ldq / XCHUNK, 1.0f);
+    if (cudaMemcpy(st->o_mul, ones.data(), ones.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+      return fail(KFL_ERR_CUDA);
+  }
   // RoPE table: angle pos * theta^(-2i/hd) in fp64, stored as fp32 cos / sin
   {
     const int half = P.hd / 2;

@@ -66,8 +66,9 @@ __device__ __forceinline__ bool chunk_ready(const GemvParams &g, int kt) {
 template <int B, int FMT>
 __device__ __noinline__ void gemv_consume_call(int n_kt, uint8_t *ring, uint64_t *full, uint64_t *empty, int S,
                                                int &s, uint32_t &phase, long long t0, int n, const SegRing &sr,
-                                               int &segc, volatile int *abort_flag, unsigned *err, int tid) {
-  gemv_consume<B, FMT>(n_kt, ring, full, empty, S, s, phase, t0, n, sr, segc, abort_flag, err, tid);
+                                               int &segc, volatile int *abort_flag, unsigned *err, int tid,
+                                               bool xsplit) {
+  gemv_consume<B, FMT>(n_kt, ring, full, empty, S, s, phase, t0, n, sr, segc, abort_flag, err, tid, xsplit);
 }
 
 template <int B>
@@ -166,6 +167,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
     }
     if (tid < MAXB) s_pos[tid] = tid < B ? kp.positions[tid] : 0;
   }
+  for (int e = tid; e < NSLOT * RB * MAXB; e += MK_THREADS) red[e] = 0.f;  // int4 tiles add into it
   __syncthreads();
 
   if (warp == CONSUMER_WARPS + 2) {
@@ -204,7 +206,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
     if (lane == 0) {
       const uint64_t pol_ring = policy_evict_first();
       const uint64_t pol_l2 = policy_evict_normal();
-      const uint32_t bytes = WBYTES + B * (KTILE * 4);
+      const uint32_t bytes = WBYTES + B * (KTILE * 4) + (FMT == 1 ? XMUL_TILE_BYTES : 0);
       struct Cursor {
         int k, i, n;
         long long t0;
@@ -324,6 +326,8 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
 #pragma unroll
             for (int b = 0; b < B; ++b)
               bulk_g2s(dst + b * (KTILE * 4), x + (size_t)b * ldx + (size_t)ktj * KTILE, KTILE * 4, fb, pol);
+            if constexpr (FMT == 1)
+              bulk_g2s(dst + B * (KTILE * 4), g.xmul + (size_t)ktj * (KT4 / XCHUNK) * MAXB, XMUL_TILE_BYTES, fb, pol);
             if (++s == S) {
               s = 0;
               aph ^= 1u;
@@ -353,10 +357,11 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
       phase_range(ph->g, c, grid, T, G, t0, n);
       if (tid == 0) stamp(k, TR_CONS_GO);
       if (B <= 2)
-        gemv_consume<B, FMT>(ph->g.n_kt, ring, full, empty, S, s, phase, t0, n, sr, segc, &s_abort, kp.err, tid);
+        gemv_consume<B, FMT>(ph->g.n_kt, ring, full, empty, S, s, phase, t0, n, sr, segc, &s_abort, kp.err, tid,
+                             ph->g.xsplit != 0);
       else
         gemv_consume_call<B, FMT>(ph->g.n_kt, ring, full, empty, S, s, phase, t0, n, sr, segc, &s_abort, kp.err,
-                                  tid);
+                                  tid, ph->g.xsplit != 0);
     } else {
       if (tid == 0) {
         stamp(k, TR_CONS_ENTER);
