@@ -68,6 +68,51 @@ __device__ __forceinline__ int attn_chunks(const AttnParams &p, int b) {
   return (P + 1 + p.chunk - 1) / p.chunk;
 }
 
+// (user, KV head, chunk) of attention unit u: users in order, n_kv_heads * nc_b units each.
+__device__ __forceinline__ void attn_unit_coords(int u, int hk, int nc0, int nc1, int nc2, int nc3, int &b, int &kvh,
+                                                 int &ch, int &ncb) {
+  int rem = u;
+  b = 0;
+  ncb = nc0;
+  if (rem >= nc0 * hk) {
+    rem -= nc0 * hk;
+    b = 1;
+    ncb = nc1;
+    if (rem >= nc1 * hk) {
+      rem -= nc1 * hk;
+      b = 2;
+      ncb = nc2;
+      if (rem >= nc2 * hk) {
+        rem -= nc2 * hk;
+        b = 3;
+        ncb = nc3;
+      }
+    }
+  }
+  kvh = rem / ncb;
+  ch = rem % ncb;
+}
+
+// Positions per unit for this step: about target_units units over the users' actual contexts
+// (a multiple of 64, at least 64), and few enough chunks per (user, KV head) for the merge to
+// take (chunks x heads <= ATT_MERGE_MAX).  Every CTA of a launch computes the same value.
+__device__ __forceinline__ int attn_chunk_size(const AttnParams &p) {
+  long long total = 0;
+  int maxp1 = 1;
+  for (int b = 0; b < p.batch; ++b) {
+    const int P = p.positions[b];
+    const int n = (P < 0 || P >= p.max_ctx) ? 1 : P + 1;
+    total += n;
+    maxp1 = max(maxp1, n);
+  }
+  const long long work = total * p.n_kv_heads;
+  const long long want = (work + p.target_units - 1) / max(1, p.target_units);
+  int chunk = static_cast<int>(max(64LL, (want + 63) / 64 * 64));
+  const int G = p.n_heads / p.n_kv_heads;
+  const int need = (maxp1 * G + ATT_MERGE_MAX - 1) / ATT_MERGE_MAX;
+  return max(chunk, (need + 63) / 64 * 64);
+}
+
 // Rows [p0, p0 + cnt) of user b / KV head kvh into K/V buffer `buf`, except `skip` (the new
 // token's row, written in this step) when skip >= 0; one cp.async group.
 template <int HD, int NBUF>
@@ -230,9 +275,10 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
       for (int e = tid; e < (ATT_SUB - cnt) * (HD / 8); e += ATT_THREADS)
         *reinterpret_cast<uint4 *>(vb + (cnt + e / (HD / 8)) * L::VROW + (e % (HD / 8)) * 16) = make_uint4(0u, 0u, 0u, 0u);
 
-    // scores of positions 8w .. 8w + 7 for every head (rows gid)
+    // scores of positions 8w .. 8w + 7 for every head (rows gid); four independent accumulator
+    // chains (K steps modulo 2, rounded and rest parts of q) so that the MMAs overlap
     {
-      float sc[4] = {0.f, 0.f, 0.f, 0.f};
+      float sp[4][4] = {};
       const uint8_t *krow = kb + (8 * warp + gid) * L::KROW + 4 * tig;
 #pragma unroll
       for (int s8 = 0; s8 < KS; ++s8) {
@@ -240,10 +286,13 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
                                : make_float2(0.f, 0.f);
         const uint32_t qh0 = to_tf32(qv.x), qh2 = to_tf32(qv.y);
         const uint32_t kw = *reinterpret_cast<const uint32_t *>(krow + 16 * s8);
-        mma_tf32(sc, qh0, qh2, kw << 16, kw & 0xFFFF0000u);
-        mma_tf32(sc, to_tf32(qv.x - __uint_as_float(qh0)), to_tf32(qv.y - __uint_as_float(qh2)), kw << 16,
-                 kw & 0xFFFF0000u);
+        mma_tf32(sp[2 * (s8 & 1)], qh0, qh2, kw << 16, kw & 0xFFFF0000u);
+        mma_tf32(sp[2 * (s8 & 1) + 1], to_tf32(qv.x - __uint_as_float(qh0)), to_tf32(qv.y - __uint_as_float(qh2)),
+                 kw << 16, kw & 0xFFFF0000u);
       }
+      float sc[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) sc[i] = (sp[0][i] + sp[2][i]) + (sp[1][i] + sp[3][i]);
       if (hrow) {
         const int pp = 8 * warp + 2 * tig;
         *reinterpret_cast<float2 *>(ss + gid * L::SS + pp) =
@@ -284,6 +333,8 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
         acc[nt][1] *= al;
       }
       const float *prow = ss + gid * L::SS;
+      // this sub-tile's P V in two chains per n-tile (even and odd K steps), then into acc
+      float pv[NT][2][4] = {};
 #pragma unroll
       for (int k8 = 0; k8 < ATT_SUB / 8; ++k8) {
         const uint32_t pa0 = hrow ? to_tf32(prow[8 * k8 + tig]) : 0u;
@@ -295,9 +346,13 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
           const int n = n_base + 8 * nt + gid;
           const uint32_t b0 = (uint32_t)(*reinterpret_cast<const uint16_t *>(v0 + 2 * n)) << 16;
           const uint32_t b1 = (uint32_t)(*reinterpret_cast<const uint16_t *>(v1 + 2 * n)) << 16;
-          mma_tf32(acc[nt], pa0, pa2, b0, b1);
+          mma_tf32(pv[nt][k8 & 1], pa0, pa2, b0, b1);
         }
       }
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc[nt][i] += pv[nt][0][i] + pv[nt][1][i];
     }
     att_sync();
   }

@@ -133,7 +133,11 @@ struct AttnParams {
   int ldo;
   float *partial;            // [batch][Hkv][n_chunks][G][hd + 2]
   int *tickets;              // [batch][Hkv]
-  int batch, n_heads, n_kv_heads, max_ctx, chunk, n_chunks;
+  int batch, n_heads, n_kv_heads, max_ctx;
+  // positions per unit: set on the device at each launch from the step's positions
+  // (attn_chunk_size), so that a step has about target_units units; the partial buffer holds
+  // n_chunks (= max_ctx / 64, rounded up) chunks per (user, KV head)
+  int chunk, n_chunks, target_units;
   float scale_log2;          // log2(e) / sqrt(hd)
   unsigned *err;
   // dataflow (persistent stage kernel only)

@@ -55,6 +55,7 @@ struct Plan {
   size_t kv_elems_per_layer;  // per cache (K or V)
   int n_sm, ctas_per_sm, stages, gemv_grid_max, n_rb_max, n_parts, attn_nchunks_max;
   int n_phases, ctr_stride;  // persistent kernel: phases per step, readiness counters per phase
+  int attn_units;            // attention units a step aims at (the kernels size chunks to it)
   size_t bytes_weights, bytes_kv, bytes_ws;
 };
 
@@ -123,6 +124,8 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   if ((flags & KFL_LOGITS_OUT) && p->lm.n_rb > nrb) nrb = p->lm.n_rb;
   p->n_rb_max = nrb;
   p->n_parts = (p->d + RB - 1) / RB;
+  // two attention CTAs fit an SM: about two units per SM over the step's actual contexts
+  p->attn_units = n_sm * std::max(1, env_int("KFL_ATTN_UNITS_PER_SM", 2));
   p->attn_nchunks_max = (c->max_ctx + 63) / 64;
   p->n_phases = 5 * p->nl + ((flags & KFL_LOGITS_OUT) ? 1 : 0);
   {
@@ -200,7 +203,6 @@ struct kfl_stage {
   unsigned *bar = nullptr;  // [0] grid-barrier counter, [1] abort flag
   Phase *phases_dev[MAXB + 1] = {};
   int n_phases = 0;
-  int persist_chunk[MAXB + 1] = {};
   bool profile = false;
   std::vector<cudaEvent_t> ev;
   double prof_ms[KFL_KERNEL_KINDS] = {};
@@ -257,8 +259,6 @@ int record_cuda_error(cudaError_t e, const char *what, int line) {
     if (_e != cudaSuccess) return record_cuda_error(_e, #x, __LINE__); \
   } while (0)
 
-// Positions per attention unit: the same in both execution modes, so they give identical bits.
-int attn_chunk_for(const kfl_stage *st, int batch) { return st->persist_chunk[batch]; }
 
 GemvParams base_gemv(kfl_stage *st, const Mat &m, const float *x, int ldx, int batch) {
   GemvParams g = {};
@@ -284,7 +284,7 @@ GemvParams base_gemv(kfl_stage *st, const Mat &m, const float *x, int ldx, int b
 // The phases of one decode step of the stage at this batch size: for every block Q/K/V (+RoPE,
 // KV append), attention, O (+residual), gate/up (+SwiGLU), down (+residual); then lm_head
 // (+argmax) for the head.  Both execution modes run exactly these.
-std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk, bool dataflow = false) {
+std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false) {
   const Plan &P = st->P;
   const kfl_model_cfg &c = st->cfg;
   const bool i4 = c.weight_fmt == KFL_INT4_G64;
@@ -344,8 +344,9 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, int attn_chunk, bool d
       a.n_heads = P.hq;
       a.n_kv_heads = P.hkv;
       a.max_ctx = c.max_ctx;
-      a.chunk = attn_chunk;
-      a.n_chunks = (c.max_ctx + attn_chunk - 1) / attn_chunk;
+      a.chunk = 64;  // the kernels size the step's chunks from its positions
+      a.n_chunks = (c.max_ctx + 63) / 64;
+      a.target_units = P.attn_units;
       a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)P.hd));
       a.err = st->err;
       ph.push_back(x);
@@ -491,7 +492,7 @@ int phase_kind_code(const Phase &ph, size_t i) {
 // `kinds` (profiling, no PDL) the k-th launch is bracketed by events ev[2(ev_base+k)] and
 // ev[2(ev_base+k)+1] and its kind appended to *kinds.
 int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector<int> *kinds, int ev_base) {
-  const std::vector<Phase> phases = build_phases(st, batch, attn_chunk_for(st, batch));
+  const std::vector<Phase> phases = build_phases(st, batch);
   int k = ev_base;
   for (size_t i = 0; i < phases.size(); ++i) {
     const Phase &ph = phases[i];
@@ -515,7 +516,7 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
 // Persistent mode: the phase table of this batch size, uploaded once (outside any capture).
 int upload_phases(kfl_stage *st, int batch) {
   if (st->phases_dev[batch]) return KFL_OK;
-  const std::vector<Phase> phases = build_phases(st, batch, st->persist_chunk[batch], true);
+  const std::vector<Phase> phases = build_phases(st, batch, true);
   void *d = nullptr;
   if (cudaMalloc(&d, phases.size() * sizeof(Phase)) != cudaSuccess) {
     cudaGetLastError();
@@ -588,7 +589,7 @@ int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const in
   const bool embed = (st->flags & KFL_EMBED_IN) != 0;
   const bool body = P.nl > 0 || (st->flags & KFL_LOGITS_OUT);
   if (st->profile) {
-    const int n_k = 2 + (int)build_phases(st, batch, attn_chunk_for(st, batch)).size();
+    const int n_k = 2 + (int)build_phases(st, batch).size();
     while ((int)st->ev.size() < 2 * n_k) {
       cudaEvent_t e;
       CK(cudaEventCreate(&e));
@@ -873,16 +874,6 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
       cudaGetLastError();
       st->persistent = false;
     }
-    for (int b = 1; b <= cfg->max_batch; ++b) {
-      // about one attention unit per SM over the reserved context
-      const long long work = (long long)cfg->max_ctx * b * P.hkv;
-      long long want = (work + P.n_sm - 1) / P.n_sm;
-      if (want < 64) want = 64;
-      int chunk = round_up((int)want, 64);
-      while ((long long)((cfg->max_ctx + chunk - 1) / chunk) * (P.hq / P.hkv) > 1024) chunk += 64;
-      if (chunk > round_up(cfg->max_ctx, 64)) chunk = round_up(cfg->max_ctx, 64);
-      st->persist_chunk[b] = chunk;
-    }
   }
   *out = st;
   return KFL_OK;
@@ -1124,7 +1115,7 @@ extern "C" int kfl_stage_trace(kfl_stage *st, uint64_t *buf) {
 extern "C" int kfl_stage_trace_shape(kfl_stage *st, int batch, int *n_phases, int *grid, int *slots) {
   if (!valid(st)) return KFL_ERR_STATE;
   if (batch < 1 || batch > st->cfg.max_batch) return KFL_ERR_RANGE;
-  if (n_phases) *n_phases = (int)build_phases(st, batch, st->persist_chunk[batch]).size();
+  if (n_phases) *n_phases = (int)build_phases(st, batch).size();
   if (grid) *grid = std::max(st->P.n_sm, st->P.gemv_grid_max);
   if (slots) *slots = TRACE_SLOTS;
   return KFL_OK;

@@ -84,31 +84,6 @@ __device__ __noinline__ void attn_phase_unit(const AttnParams &a, int b, int kvh
   attn_unit<HD, 1>(a, b, kvh, ch, nc, att, s_last, tid, prefetched);
 }
 
-// (user, KV head, chunk) of attention unit u: users in order, n_kv_heads * nc_b units each.
-__device__ __forceinline__ void attn_unit_coords(int u, int hk, int nc0, int nc1, int nc2, int nc3, int &b, int &kvh,
-                                                 int &ch, int &ncb) {
-  int rem = u;
-  b = 0;
-  ncb = nc0;
-  if (rem >= nc0 * hk) {
-    rem -= nc0 * hk;
-    b = 1;
-    ncb = nc1;
-    if (rem >= nc1 * hk) {
-      rem -= nc1 * hk;
-      b = 2;
-      ncb = nc2;
-      if (rem >= nc2 * hk) {
-        rem -= nc2 * hk;
-        b = 3;
-        ncb = nc3;
-      }
-    }
-  }
-  kvh = rem / ncb;
-  ch = rem % ncb;
-}
-
 template <int B, int FMT>
 __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_constant__ StageKernelParams kp) {
   extern __shared__ __align__(1024) uint8_t smem[];
@@ -367,6 +342,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
         stamp(k, TR_CONS_ENTER);
         s_ap = ph->a;
         s_ap.positions = s_pos;
+        s_ap.chunk = attn_chunk_size(s_ap);
       }
       consumer_sync();
       const AttnParams &a = s_ap;
