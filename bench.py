@@ -96,8 +96,10 @@ def measured_peaks():
 
 
 def kernel_source_hash() -> str:
+    """Hash of the sources the GEMV kernels are built from: a committed DRAM-traffic figure
+    counts only while they are unchanged."""
     h = hashlib.sha256()
-    for name in ("gemv.cu", "common.cuh"):
+    for name in ("gemv.cu", "gemv_core.cuh", "common.cuh"):
         with open(os.path.join(ROOT, "paper_2609_34045_gb300", "csrc", name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
