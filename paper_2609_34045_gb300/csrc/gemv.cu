@@ -155,10 +155,25 @@ static size_t gemv_smem_bytes(int stages, int batch, int fmt) {
          128 + NSLOT * RB * MAXB * sizeof(float);
 }
 
+static int g_smem_optin = 0, g_smem_per_sm = 0, g_n_sm = 0;
+
+// Dynamic shared memory of a launch.  Stream-K gives every CTA an equal share of the tiles, so a
+// grid of at most one CTA per SM assumes each CTA has its SM's issue slots to itself.  Where two
+// rings fit one SM (int4 tiles at batch 1), the block scheduler may place two CTAs of one GEMV on
+// an SM that frees up early while other SMs still hold the previous kernel's CTAs; those two then
+// share the SM and the whole GEMV waits for them.  Asking for more than half of the SM's shared
+// memory keeps such a grid at one CTA per SM.
+static size_t gemv_launch_smem(size_t need, int grid) {
+  if (grid > g_n_sm) return need;
+  const size_t half = (size_t)g_smem_per_sm / 2;
+  const size_t cap = (size_t)g_smem_optin - GEMV_STATIC_SMEM;
+  return need >= half ? need : (half < cap ? half : cap);
+}
+
 template <int B, int EPI, int FMT>
 static cudaError_t launch_one(const GemvParams &p, int grid, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
-  const size_t smem = gemv_smem_bytes(p.stages, B, FMT);
+  const size_t smem = gemv_launch_smem(gemv_smem_bytes(p.stages, B, FMT), grid);
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(GEMV_THREADS);
   cfg.dynamicSmemBytes = smem;
@@ -201,12 +216,11 @@ int gemv_max_stages(int batch, int fmt, int smem_optin) {
   return s;
 }
 
-static int g_smem_optin = 0;
-
 template <int B, int EPI, int FMT>
 static cudaError_t prepare_one() {
+  const size_t deepest = gemv_smem_bytes(gemv_max_stages(B, FMT, g_smem_optin), B, FMT);
   return cudaFuncSetAttribute(gemv_kernel<B, EPI, FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)gemv_smem_bytes(gemv_max_stages(B, FMT, g_smem_optin), B, FMT));
+                              (int)gemv_launch_smem(deepest, 1));
 }
 
 template <int EPI, int FMT>
@@ -234,6 +248,9 @@ cudaError_t prepare_gemv() {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&g_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (e == cudaSuccess)
+    e = cudaDeviceGetAttribute(&g_smem_per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&g_n_sm, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
   e = prepare_f<0>();
   return e != cudaSuccess ? e : prepare_f<1>();
