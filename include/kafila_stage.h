@@ -165,7 +165,11 @@ int kfl_stage_debug_capture(kfl_stage *st, float *per_layer_hidden);
  * 1 the phase starts on the CTA, 2 the CTA finishes it (epilogues included), 3 its activation
  * input is available (first chunk copied; one-kernel-per-phase: past griddepcontrol.wait),
  * 4 the last activation chunk is copied (persistent kernel), 5/6 the first/last weight tile is
- * issued.  Slots of events that do not happen are left as they were.  NULL turns it off.
+ * issued; one kernel per phase, a GEMV CTA's last row-block segment: 7 its sums are staged,
+ * 8 (row block shared with other CTAs) its partial is published and the ticket taken, 9 (last
+ * arriver) every partial is summed, 10 the fused epilogue is done, 11 the kind of segment (0 the
+ * CTA's alone, 1 shared, 2 shared and last).  Slots of events that do not happen are left as
+ * they were.  NULL turns it off.
  * Changing it rebuilds the stage's CUDA graphs on the next decode. */
 int kfl_stage_trace(kfl_stage *st, uint64_t *buf);
 int kfl_stage_trace_shape(kfl_stage *st, int batch, int *n_phases, int *grid, int *slots);

@@ -175,7 +175,7 @@ struct StageKernelParams {
 };
 
 // phase trace slots (ns, %globaltimer)
-constexpr int TRACE_SLOTS = 8;
+constexpr int TRACE_SLOTS = 12;
 constexpr int TR_CONS_ENTER = 0;   // consumers reach the phase
 constexpr int TR_CONS_GO = 1;      // consumers start its work
 constexpr int TR_CONS_DONE = 2;    // consumers finished the phase
@@ -183,6 +183,12 @@ constexpr int TR_X_GO = 3;         // activation producer issued the phase's fir
 constexpr int TR_X_LAST = 4;       // activation producer issued the phase's last chunk
 constexpr int TR_W_FIRST = 5;      // weight producer issued the phase's first tile
 constexpr int TR_W_LAST = 6;       // weight producer issued the phase's last tile
+// GEMV epilogue warp, last row-block segment of the CTA (one kernel per phase)
+constexpr int TR_E_SEG = 7;        // the consumers' sums of the segment are staged
+constexpr int TR_E_TICKET = 8;     // shared row block: this CTA's partial published, ticket taken
+constexpr int TR_E_SUMMED = 9;     // last arriver: every partial of the row block summed
+constexpr int TR_E_DONE = 10;      // fused epilogue of the segment done
+constexpr int TR_E_KIND = 11;      // 0 row block of this CTA alone, 1 shared (not last), 2 shared, last
 
 __device__ __forceinline__ unsigned long long global_ns() {
   unsigned long long t;

@@ -343,11 +343,26 @@ __device__ __forceinline__ void norm_scale_warp(const GemvParams &p, float *inv,
 struct EpiPre {
   float h[MAXB][2];
   float g[2];
+  float cs[MAXB], sn[MAXB];  // QKV: the RoPE cos / sin of this lane's row pair, per user
 };
 
 template <int B, int EPI>
 __device__ __forceinline__ void epilogue_prefetch(const GemvParams &p, int rb, int lane, EpiPre &e) {
-  if constexpr (EPI == EPI_RESID) {
+  if constexpr (EPI == EPI_QKV) {
+    // lane = row pair (RB / 2 = 32 of them), one user per pass (as in epilogue_warp)
+    const int hd = p.head_dim, half = hd >> 1, r0 = rb * RB + 2 * lane;
+    const bool rot = r0 < p.n_rows && r0 < p.n_q_rows + p.n_kv_rows;
+    const int rr = r0 < p.n_q_rows ? r0 : r0 - p.n_q_rows;
+    const int i = (rr % hd) >> 1;
+#pragma unroll
+    for (int b = 0; b < B; ++b) {
+      int pos = p.positions[b];
+      if (pos < 0 || pos >= p.max_ctx) pos = 0;
+      const size_t ri = (size_t)(p.rope_per_user ? b : pos) * half + i;
+      e.cs[b] = rot ? p.rope_cos[ri] : 0.f;
+      e.sn[b] = rot ? p.rope_sin[ri] : 0.f;
+    }
+  } else if constexpr (EPI == EPI_RESID) {
 #pragma unroll
     for (int h2 = 0; h2 < 2; ++h2) {
       const int n = rb * RB + lane + 32 * h2;
@@ -426,8 +441,9 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
     }
   } else if constexpr (EPI == EPI_QKV) {
     const int hd = p.head_dim, half = hd >> 1;
-    for (int e = lane; e < (RB / 2) * B; e += 32) {
-      const int b = e / (RB / 2), pr = e % (RB / 2), r0 = rb * RB + 2 * pr;
+#pragma unroll
+    for (int b = 0; b < B; ++b) {
+      const int pr = lane, r0 = rb * RB + 2 * pr;
       int pos = p.positions[b];
       const bool ok = pos >= 0 && pos < p.max_ctx;
       if (!ok) pos = 0;
@@ -438,9 +454,8 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
         const bool is_q = r0 < p.n_q_rows;
         const int rr = is_q ? r0 : r0 - p.n_q_rows;
         const int head = rr / hd, i = (rr % hd) >> 1;
-        const size_t ri = (size_t)(p.rope_per_user ? b : pos) * half + i;
-        const float cs = p.rope_cos[ri];
-        const float sn = p.rope_sin[ri];
+        const float cs = pre.cs[b];
+        const float sn = pre.sn[b];
         const float a = v1 * cs - v2 * sn;
         const float c2 = v2 * cs + v1 * sn;
         if (is_q) {
@@ -517,57 +532,81 @@ __device__ __forceinline__ void gemv_epilogues(const GemvParams &p, long long t0
     const int slot = segc % NSLOT, use = segc / NSLOT;
     ++segc;
     consumer_wait(smem_addr(&sr.full[slot]), use & 1, abort_flag, p.err);
+    unsigned long long *tr = p.trace && lane == 0 ? p.trace + (size_t)c * TRACE_SLOTS : nullptr;
+    if (tr) {
+      tr[TR_E_SEG] = global_ns();
+      tr[TR_E_KIND] = 0;
+    }
     float *red = sr.red + slot * RB * MAXB;
     EpiPre pre;
     epilogue_prefetch<B, EPI>(p, rb, lane, pre);
     bool do_epi = true;
     if (!(kt0 == 0 && len == p.n_kt)) {
-      // this row block is shared with neighbouring CTAs
-      const int first_rb = static_cast<int>(t0 / p.n_kt);
-      const int myslot = (rb == first_rb) ? 0 : 1;
-      float4 *mine = reinterpret_cast<float4 *>(p.partial + (size_t)(c * 2 + myslot) * (RB * MAXB));
-      const float4 *r4 = reinterpret_cast<const float4 *>(red);
-      for (int e = lane; e < RB * MAXB / 4; e += 32) mine[e] = r4[e];
-      __syncwarp();
+      // this row block is shared with neighbouring CTAs: the ticket counts the CTAs that have
+      // published their partial; the one that finds all the others there sums every partial
       const int c_lo = cta_of_tile((long long)rb * p.n_kt, T, G);
       const int c_hi = cta_of_tile((long long)(rb + 1) * p.n_kt - 1, T, G);
-      unsigned prev = 0;
-      if (lane == 0) {
-        // release this CTA's partials; the last to arrive acquires everyone's
-        prev = atom_add_acq_rel(reinterpret_cast<unsigned *>(p.tickets + rb), 1u);
-        if (prev == (unsigned)(c_hi - c_lo)) atomicExch(p.tickets + rb, 0);
-      }
-      prev = __shfl_sync(0xffffffffu, prev, 0);
+      const unsigned others = static_cast<unsigned>(c_hi - c_lo);
+      unsigned *ticket = reinterpret_cast<unsigned *>(p.tickets + rb);
+      unsigned seen = 0;
+      if (lane == 0) seen = ld_acquire_gpu(ticket);
+      seen = __shfl_sync(0xffffffffu, seen, 0);
       __syncwarp();
-      do_epi = prev == (unsigned)(c_hi - c_lo);
+      do_epi = seen == others;
+      if (!do_epi) {
+        const int first_rb = static_cast<int>(t0 / p.n_kt);
+        const int myslot = (rb == first_rb) ? 0 : 1;
+        float4 *mine = reinterpret_cast<float4 *>(p.partial + (size_t)(c * 2 + myslot) * (RB * MAXB));
+        const float4 *r4 = reinterpret_cast<const float4 *>(red);
+        for (int e = lane; e < RB * MAXB / 4; e += 32) mine[e] = r4[e];
+        __syncwarp();
+        unsigned prev = 0;
+        // release this CTA's partial; the last to arrive acquires everyone's
+        if (lane == 0) prev = atom_add_acq_rel(ticket, 1u);
+        prev = __shfl_sync(0xffffffffu, prev, 0);
+        __syncwarp();
+        do_epi = prev == others;
+      }
+      if (tr) {
+        tr[TR_E_TICKET] = global_ns();
+        tr[TR_E_KIND] = do_epi ? 2 : 1;
+      }
       if (do_epi) {
-        // every partial's loads first (independent), then the sums in CTA order
-        for (int e = lane; e < RB * MAXB / 4; e += 32) {
-          float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
-          for (int c0 = c_lo; c0 <= c_hi; c0 += 4) {
-            float4 v[4];
+        if (lane == 0) atomicExch(ticket, 0u);  // ready for the next use
+        // every partial in CTA order (this CTA's own from shared memory): each lane's loads of a
+        // group of four CTAs are issued together, then added
+        static_assert(RB * MAXB / 4 == 64, "two float4 per lane");
+        float4 sum[2] = {make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f)};
+        for (int c0 = c_lo; c0 <= c_hi; c0 += 4) {
+          float4 v[2][4];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const int cc = c0 + j;
-              v[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-              if (cc <= c_hi) {
-                const int frb = static_cast<int>(((long long)cc * T / G) / p.n_kt);
-                const int sl = (rb == frb) ? 0 : 1;
-                v[j] = __ldcg(reinterpret_cast<const float4 *>(p.partial + (size_t)(cc * 2 + sl) * (RB * MAXB)) + e);
+          for (int j = 0; j < 4; ++j) {
+            const int cc = c0 + j;
+            const int frb = static_cast<int>(((long long)cc * T / G) / p.n_kt);
+            const float4 *src = reinterpret_cast<const float4 *>(p.partial + (size_t)(cc * 2 + (rb == frb ? 0 : 1)) * (RB * MAXB));
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+              const int e = lane + 32 * k;
+              v[k][j] = cc > c_hi ? make_float4(0.f, 0.f, 0.f, 0.f)
+                        : cc == c ? reinterpret_cast<const float4 *>(red)[e] : __ldcg(src + e);
+            }
+          }
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (c0 + j <= c_hi) {
+#pragma unroll
+              for (int k = 0; k < 2; ++k) {
+                sum[k].x += v[k][j].x;
+                sum[k].y += v[k][j].y;
+                sum[k].z += v[k][j].z;
+                sum[k].w += v[k][j].w;
               }
             }
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-              if (c0 + j <= c_hi) {
-                sum.x += v[j].x;
-                sum.y += v[j].y;
-                sum.z += v[j].z;
-                sum.w += v[j].w;
-              }
-          }
-          reinterpret_cast<float4 *>(red)[e] = sum;
         }
+#pragma unroll
+        for (int k = 0; k < 2; ++k) reinterpret_cast<float4 *>(red)[lane + 32 * k] = sum[k];
         __syncwarp();
+        if (tr) tr[TR_E_SUMMED] = global_ns();
       }
     }
     if (do_epi) {
@@ -602,6 +641,7 @@ __device__ __forceinline__ void gemv_epilogues(const GemvParams &p, long long t0
         if (p.out_done) red_add_release(p.out_done, 1u);
       }
     }
+    if (tr) tr[TR_E_DONE] = global_ns();
     __syncwarp();
     // leave the slot at zero: int4 tiles add into it
     for (int e = lane; e < RB * MAXB / 4; e += 32) reinterpret_cast<float4 *>(red)[e] = make_float4(0.f, 0.f, 0.f, 0.f);
