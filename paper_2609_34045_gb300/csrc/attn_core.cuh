@@ -171,6 +171,15 @@ __device__ __forceinline__ void mma_tf32(float (&d)[4], uint32_t a0, uint32_t a2
       : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
 }
 
+// int4 stages: the output of heads (kvh, og), dimensions od .. od + 3, also in the O
+// projection's input form (8 lanes hold a 32-dimension chunk); every thread of the unit calls it.
+template <int HD>
+__device__ __forceinline__ void attn_out16(const AttnParams &p, int b, int kvh, int G, int og, int od, float4 v,
+                                           bool owns, int lane) {
+  if (!p.o16.hi) return;
+  act16_put_quad(p.o16, b, ((kvh * G + og) * HD + od) / XCHUNK, v, lane, owns);
+}
+
 template <int HD, int NBUF>
 __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, uint8_t *sm, int *s_last, int tid,
                           int prefetched, unsigned long long *tr = nullptr) {
@@ -199,6 +208,7 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
   if (P < 0 || P >= p.max_ctx) {
     // the stage input flagged the position; leave a defined (zero) output
     if (owns) *reinterpret_cast<float4 *>(o + og * HD + od) = make_float4(0.f, 0.f, 0.f, 0.f);
+    attn_out16<HD>(p, b, kvh, G, og, od, make_float4(0.f, 0.f, 0.f, 0.f), owns, lane);
     attn_publish(p, kvh, tid);
     return;
   }
@@ -359,12 +369,28 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
 
   stamp(TR_W_FIRST);
   if (nc == 1) {
-    if (hrow) {
-      const float il = 1.0f / s_l[gid];
+    if (!p.o16.hi) {
+      if (hrow) {
+        const float il = 1.0f / s_l[gid];
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-        *reinterpret_cast<float2 *>(o + gid * HD + n_base + 8 * nt + 2 * tig) =
-            make_float2(acc[nt][0] * il, acc[nt][1] * il);
+        for (int nt = 0; nt < NT; ++nt)
+          *reinterpret_cast<float2 *>(o + gid * HD + n_base + 8 * nt + 2 * tig) =
+              make_float2(acc[nt][0] * il, acc[nt][1] * il);
+      }
+    } else {
+      // through shared memory (the K buffers) into the output mapping of the merge
+      float *so = reinterpret_cast<float *>(sk);
+      if (hrow) {
+        const float il = 1.0f / s_l[gid];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+          *reinterpret_cast<float2 *>(so + gid * HD + n_base + 8 * nt + 2 * tig) =
+              make_float2(acc[nt][0] * il, acc[nt][1] * il);
+      }
+      att_sync();
+      const float4 v = owns ? *reinterpret_cast<const float4 *>(so + og * HD + od) : make_float4(0.f, 0.f, 0.f, 0.f);
+      if (owns) *reinterpret_cast<float4 *>(o + og * HD + od) = v;
+      attn_out16<HD>(p, b, kvh, G, og, od, v, owns, lane);
     }
     attn_publish(p, kvh, tid);
     return;
@@ -430,8 +456,8 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
     for (int cc = lane; cc < nc; cc += 32) wm[cc * G + g] = exp2f(wm[cc * G + g] - M) * invL;
   }
   att_sync();
+  float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
   if (owns) {
-    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int c0 = 0; c0 < nc; c0 += MB) {
       if (c0 > 0) load_batch(c0);
 #pragma unroll
@@ -447,6 +473,7 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
     }
     *reinterpret_cast<float4 *>(o + og * HD + od) = O;
   }
+  attn_out16<HD>(p, b, kvh, G, og, od, O, owns, lane);
   attn_publish(p, kvh, tid);
 }
 

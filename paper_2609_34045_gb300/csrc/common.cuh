@@ -29,16 +29,45 @@ constexpr int TILE4_CODE_BYTES = RB * KT4 / 2;     // 8 KiB
 constexpr int TILE4_SCALE_BYTES = RB * (KT4 / 64) * 2;  // 512 B
 constexpr int TILE4_BYTES = TILE4_CODE_BYTES + TILE4_SCALE_BYTES;
 
-// A ring stage holds one weight tile and the B users' fp32 activation chunks of its K range.
 __host__ __device__ constexpr int tile_k(int fmt) { return fmt == 0 ? KT : KT4; }
 __host__ __device__ constexpr int tile_bytes(int fmt) { return fmt == 0 ? TILE_BYTES : TILE4_BYTES; }
-// int4 stages also carry the activation multipliers of the tile (XCHUNK-element chunks x MAXB)
-constexpr int XCHUNK = 32;
-constexpr int XMUL_TILE_BYTES = (KT4 / XCHUNK) * MAXB * 4;  // 128
+// A ring stage holds one weight tile and the activations of its K range: bf16 tiles, the B
+// users' fp32 values; int4 tiles, up to 2 B fp16 source rows (struct Act16: the users' rounded
+// parts, then their rests) at a padded stride, then the tile's per-chunk constants.
+constexpr int XCHUNK = 32;                          // elements per scale chunk of an int4 input
+constexpr int X16_SRC_BYTES = KT4 * 2;              // 512
+constexpr int X16_SRC_STRIDE = X16_SRC_BYTES + 32;  // 544: the sources start on different banks
+constexpr int XC_CHUNK_FLOATS = 16;                 // per chunk: [4 lane quads][4]
+constexpr int XC_TILE_BYTES = (KT4 / XCHUNK) * XC_CHUNK_FLOATS * 4;  // 512
 __host__ __device__ constexpr int stage_bytes(int batch, int fmt) {
-  return (tile_bytes(fmt) + batch * tile_k(fmt) * 4 + (fmt == 0 ? 0 : XMUL_TILE_BYTES) + 127) / 128 * 128;
+  return fmt == 0 ? (TILE_BYTES + batch * KT * 4 + 127) / 128 * 128
+                  : (TILE4_BYTES + 2 * batch * X16_SRC_STRIDE + XC_TILE_BYTES + 127) / 128 * 128;
 }
 constexpr int STAGE_BYTES_MAX = stage_bytes(MAXB, 0);
+
+// A GEMV input of an int4 stage, in the form the tensor-core tile loop reads (tile_compute_int4).
+// Per user b, row b * ld: x divided by a power of two per XCHUNK elements (m, the multiplier
+// that undoes it, brings the chunk's largest value into [2^14, 2^15)) and rounded to fp16; in
+// each 16-element block, elements 8..15 are also divided by 16 (the decoder makes their weights
+// 16 x larger), and the block is stored in the order of the MMA's B fragments (act16_index).
+// lo (the Q/K/V projection's input only, else NULL): what rounding to fp16 left over, in fp16.
+// xc[chunk][t][0..1]: m of MMA columns 2t, 2t+1; xc[chunk][t][2..3]: minus their offset sums,
+// where column u < 4 is user u's rounded part and column u + 4 its rest, and a column's offset
+// sum is the sum over the chunk of its fp16 values times 1032 (block elements 0..7) or 1152
+// (8..15): what the decoder's offsets add to the MMA's product.
+struct Act16 {
+  uint16_t *hi;
+  uint16_t *lo;
+  float *xc;
+  int ld;  // elements per user row, a multiple of KT4
+};
+
+// Position of element k of a user's row in Act16 order: within a 16-element block, lane quad t
+// of a warp reads the 8 bytes at 4 t: elements 2t, 2t+1 (B fragment register b0) and 2t+8, 2t+9
+// (b1).
+__host__ __device__ constexpr int act16_index(int k) {
+  return (k & ~15) + ((k & 7) >> 1) * 4 + ((k & 15) < 8 ? 0 : 2) + (k & 1);
+}
 
 // ---- device error word bits ---------------------------------------------------------------
 constexpr unsigned ERR_POSITION = 1u;
@@ -91,12 +120,10 @@ struct GemvParams {
   const float *rope_cos, *rope_sin;  // [max_ctx][hd/2], or [batch][hd/2] when rope_per_user
   int rope_per_user;
   int n_q_rows, n_kv_rows, head_dim, max_ctx, n_kv_heads;
-  // int4 weights: the GEMV multiplies fp16 activations on the tensor cores.  Each producer of an
-  // int4 GEMV's input stores it scaled by a power of two per XCHUNK elements (so that it fits
-  // fp16) with the multiplier that undoes it: x_true[k] = x[k] * xmul[k / XCHUNK][b].
-  const float *xmul;  // this GEMV's input multipliers [chunks][MAXB] (int4), else NULL
-  float *xmul_out;    // RESID / SWIGLU: multipliers of the output written (int4 stages), else NULL
-  int xsplit;         // activations carried as an fp16 pair (rounded, rest): Q/K/V projection
+  // int4 weights: the GEMV multiplies fp16 activations on the tensor cores
+  Act16 xin;          // this GEMV's input (int4 stages; x and ldx are then unused)
+  Act16 xout;         // RESID / SWIGLU: the output in the same form (int4 stages; hi NULL else)
+  int xsplit;         // the input's rests are multiplied too (Q/K/V projection: xin.lo)
   // EPI_ARGMAX
   float *cand_val;
   int *cand_idx;
@@ -131,6 +158,7 @@ struct AttnParams {
   const int *positions;
   float *o;                  // [batch][ldo]
   int ldo;
+  Act16 o16;                 // int4 stages: o also in the O projection's input form (hi NULL else)
   float *partial;            // [batch][Hkv][n_chunks][G][hd + 2]
   int *tickets;              // [batch][Hkv]
   int batch, n_heads, n_kv_heads, max_ctx;
@@ -348,6 +376,98 @@ __device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned *p) {
   return v;
 }
 
+__device__ __forceinline__ uint16_t f32_to_f16_rn(float x) {
+  uint16_t h;
+  asm("cvt.rn.f16.f32 %0, %1;" : "=h"(h) : "f"(x));
+  return h;
+}
+__device__ __forceinline__ float f16_to_f32(uint16_t h) {
+  float f;
+  asm("cvt.f32.f16 %0, %1;" : "=f"(f) : "h"(h));
+  return f;
+}
+
+// Chunk ch's constants for user b (column b: rounded part, column b + 4: rest).
+__device__ __forceinline__ void act16_put_consts(const Act16 &a, int b, int ch, float m, float off_hi, float off_lo) {
+  float *c = a.xc + (size_t)ch * XC_CHUNK_FLOATS;
+  const int t = b >> 1, j = b & 1;
+  c[t * 4 + j] = m;
+  c[t * 4 + 2 + j] = -off_hi;
+  c[(t + 2) * 4 + j] = m;
+  c[(t + 2) * 4 + 2 + j] = -off_lo;
+}
+
+// Chunk ch of user b of an Act16, one element per lane (x = 0 past the vector's end); the whole
+// warp calls it.
+__device__ __forceinline__ void act16_put_warp(const Act16 &a, int b, int ch, float x, int lane) {
+  float mx = fabsf(x);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+  float iv;
+  const float m = xchunk_scale(mx, &iv);
+  const bool upper = (lane & 15) >= 8;
+  const float y = x * iv * (upper ? 0.0625f : 1.0f);
+  const float wgt = upper ? 1152.0f : 1032.0f;
+  const uint16_t h = f32_to_f16_rn(y);
+  const float yh = f16_to_f32(h);
+  const size_t idx = (size_t)b * a.ld + (size_t)ch * XCHUNK + act16_index(lane);
+  a.hi[idx] = h;
+  float oh = yh * wgt, ol = 0.f;
+  if (a.lo) {
+    const uint16_t l = f32_to_f16_rn(y - yh);
+    a.lo[idx] = l;
+    ol = f16_to_f32(l) * wgt;
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    oh += __shfl_xor_sync(0xffffffffu, oh, off);
+    ol += __shfl_xor_sync(0xffffffffu, ol, off);
+  }
+  if (lane == 0) act16_put_consts(a, b, ch, m, oh, ol);
+}
+
+// The same, with the chunk held by 8 consecutive lanes, 4 consecutive elements each (lane & 7
+// holds elements 4 (lane & 7) .. + 3); the whole warp calls it, `write` selects the lanes that
+// store.
+__device__ __forceinline__ void act16_put_quad(const Act16 &a, int b, int ch, float4 v, int lane, bool write) {
+  float mx = fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w)));
+#pragma unroll
+  for (int off = 4; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+  float iv;
+  const float m = xchunk_scale(mx, &iv);
+  const int sub = lane & 7;
+  const bool upper = (sub & 2) != 0;  // elements 4 sub .. + 3 lie in one half of a 16-block
+  const float sc = iv * (upper ? 0.0625f : 1.0f), wgt = upper ? 1152.0f : 1032.0f;
+  const float y[4] = {v.x * sc, v.y * sc, v.z * sc, v.w * sc};
+  uint16_t h[4], l[4];
+  float oh = 0.f, ol = 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    h[i] = f32_to_f16_rn(y[i]);
+    const float yh = f16_to_f32(h[i]);
+    l[i] = f32_to_f16_rn(y[i] - yh);
+    oh += yh * wgt;
+    ol += f16_to_f32(l[i]) * wgt;
+  }
+  if (!a.lo) ol = 0.f;
+#pragma unroll
+  for (int off = 4; off > 0; off >>= 1) {
+    oh += __shfl_xor_sync(0xffffffffu, oh, off);
+    ol += __shfl_xor_sync(0xffffffffu, ol, off);
+  }
+  if (write) {
+    const size_t row = (size_t)b * a.ld + (size_t)ch * XCHUNK;
+    const int i0 = act16_index(4 * sub), i2 = act16_index(4 * sub + 2);
+    *reinterpret_cast<uint32_t *>(a.hi + row + i0) = (uint32_t)h[0] | ((uint32_t)h[1] << 16);
+    *reinterpret_cast<uint32_t *>(a.hi + row + i2) = (uint32_t)h[2] | ((uint32_t)h[3] << 16);
+    if (a.lo) {
+      *reinterpret_cast<uint32_t *>(a.lo + row + i0) = (uint32_t)l[0] | ((uint32_t)l[1] << 16);
+      *reinterpret_cast<uint32_t *>(a.lo + row + i2) = (uint32_t)l[2] | ((uint32_t)l[3] << 16);
+    }
+    if (sub == 0) act16_put_consts(a, b, ch, m, oh, ol);
+  }
+}
+
 }  // namespace kfl
 
 // Kernel launchers (defined in the .cu files; used by the runtime).
@@ -360,7 +480,7 @@ cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s, 
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in,
                                int batch, const uint16_t *embed, int vocab, int d, int ldh,
                                const float *g_next, float *h, float *xn, float *sumsq,
-                               int *positions, int max_ctx, unsigned *err, unsigned *bar, float *xmul,
+                               int *positions, int max_ctx, unsigned *err, unsigned *bar, Act16 xn16,
                                cudaStream_t s);
 size_t stage_kernel_smem(int stages, int head_dim, int batch, int fmt);
 int stage_kernel_attn_bytes(int head_dim);

@@ -139,43 +139,31 @@ __device__ __forceinline__ void mma_f16_16816(float (&d)[4], uint32_t a0, uint32
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// Two 4-bit codes (bits 0-3 and 16-19 of w) as an fp16 pair of their signed values: the nibble,
-// with its top bit flipped, as the low mantissa bits of 1024 gives 1024 + (n ^ 8) = 1032 + code;
-// subtracting 1032 is exact.
-__device__ __forceinline__ uint32_t int4_pair_f16(uint32_t w) {
-  uint32_t r;
-  asm("lop3.b32 %0, %1, %2, %3, 0x6A;" : "=r"(r) : "r"(w), "r"(0x000F000Fu), "r"(0x64086408u));  // (w & m) ^ c
-  uint32_t d;
-  asm("fma.rn.f16x2 %0, %1, %2, %3;" : "=r"(d) : "r"(r), "r"(0x3C003C00u), "r"(0xE408E408u));  // r * 1 - 1032
-  return d;
-}
-
-// fp32 pair -> fp16 pair (round to nearest even), lo in the low half
-__device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
-  uint32_t r;
-  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
-  return r;
-}
-
-// fp32 pair -> the fp16 pair of what rounding it to fp16 left over (x - fp16(x), rounded): with
-// the rounded pair it carries x to about 2^-22
-__device__ __forceinline__ uint32_t pack_f16x2_rest(float lo, float hi, uint32_t rounded) {
-  float rl, rh;
-  asm("{\n\t.reg .f16 l, h;\n\tmov.b32 {l, h}, %2;\n\tcvt.f32.f16 %0, l;\n\tcvt.f32.f16 %1, h;\n\t}"
-      : "=f"(rl), "=f"(rh)
-      : "r"(rounded));
-  return pack_f16x2(lo - rl, hi - rh);
+// The A fragment of one m16n8k16 MMA from one 32-bit word of 8 offset-binary codes u = code + 8
+// (repack_int4_kernel): the nibble pairs at bits (0, 16) and (8, 24) become the fp16 pairs
+// 1024 + u (registers a0, a1: K elements 0..7 of the step), those at (4, 20) and (12, 28)
+// become 1024 + 16 u (a2, a3: elements 8..15, whose activations are stored divided by 16), each
+// with one lop3 ((w & mask) | 0x6400 in each half, with the code's top bit flipped: the stored
+// nibble is the two's-complement code).  The offsets 1032 x and 1152 x / 16 that this adds to
+// the product are taken off with the activations' offset sums (Act16).
+__device__ __forceinline__ void int4_frag_f16(uint32_t w, uint32_t &a0, uint32_t &a1, uint32_t &a2, uint32_t &a3) {
+  const uint32_t w8 = w >> 8;
+  asm("lop3.b32 %0, %1, %2, %3, 0x6A;" : "=r"(a0) : "r"(w), "r"(0x000F000Fu), "r"(0x64086408u));   // (w & m) ^ c
+  asm("lop3.b32 %0, %1, %2, %3, 0x6A;" : "=r"(a1) : "r"(w8), "r"(0x000F000Fu), "r"(0x64086408u));
+  asm("lop3.b32 %0, %1, %2, %3, 0x6A;" : "=r"(a2) : "r"(w), "r"(0x00F000F0u), "r"(0x64806480u));
+  asm("lop3.b32 %0, %1, %2, %3, 0x6A;" : "=r"(a3) : "r"(w8), "r"(0x00F000F0u), "r"(0x64806480u));
 }
 
 // int4 tile (FMT 1) on the tensor cores.  Warp w takes row group r16 = w % 4 (16 rows) and K half
-// h = w / 4 (128 of the tile's 256 K): per K step of 16, one m16n8k16 MMA of the codes (exact in
-// fp16) against the users' activations (stored pre-scaled per 32 elements, rounded to fp16:
-// 2^-11 relative; columns past B are 0); each 32-element chunk's product is multiplied back by its
-// multiplier and the weights' group scale into acc.  acc[0..1]: row r16*16 + gid, users 2 tig,
-// 2 tig + 1; acc[2..3]: row + 8.
-// XSPLIT (Q/K/V projection, whose errors the attention softmax amplifies): each activation is
-// carried as an fp16 pair (rounded, rest), the rounded parts in columns 0-3, the rests in 4-7
-// (B <= 4); the two are added at the end of the row block.
+// h = w / 4 (128 of the tile's 256 K): per K step of 16, one m16n8k16 MMA (fp16, fp32
+// accumulate) of the decoded codes against eight columns of activations, read as one 8-byte
+// shared-memory load per lane (Act16 order).  Column j is source row j % B (the users' rounded
+// parts); with XSPLIT, columns 4..7 are the rests (source rows B + (j - 4) % B).  Columns past
+// the users carry copies and are dropped at the end.  Per 32-element chunk the accumulator
+// starts at minus the columns' offset sums, so that after its two MMAs it holds the product of
+// the codes with the scaled activations; it is then multiplied back by the chunk's multiplier
+// and the rows' group scale into acc.  acc[0..1]: row r16*16 + gid, columns 2 tig, 2 tig + 1;
+// acc[2..3]: row + 8.
 template <int B, bool XSPLIT>
 __device__ __forceinline__ void tile_compute_int4(const uint8_t *st, int warp, int lane, float (&acc)[4]) {
   const int r16 = warp & 3, h = warp >> 2, gid = lane >> 2, tig = lane & 3;
@@ -183,43 +171,29 @@ __device__ __forceinline__ void tile_compute_int4(const uint8_t *st, int warp, i
   const uint4 wq[2] = {cw[0], cw[32]};
   const uint32_t *sp = reinterpret_cast<const uint32_t *>(st + TILE4_CODE_BYTES);
   const uint32_t s0 = sp[(r16 * 16 + gid) * 2 + h], s1 = sp[(r16 * 16 + gid + 8) * 2 + h];
-  const int xu_id = XSPLIT ? (gid & 3) : gid;
-  const float *xs = reinterpret_cast<const float *>(st + TILE4_BYTES) + xu_id * KT4 + 128 * h + 2 * tig;
-  const bool xu = xu_id < B;
-  // multipliers [8 chunks][MAXB] after the activations; this lane's columns are users
-  // (2 tig) & 3 and (2 tig + 1) & 3 (the rest parts of XSPLIT in columns 4-7 share them)
-  const float *xm = reinterpret_cast<const float *>(st + TILE4_BYTES + B * KT4 * 4) + (2 * tig & 3);
-  const bool mu0 = (2 * tig & 3) < B, mu1 = ((2 * tig + 1) & 3) < B;
+  const int src = XSPLIT ? (gid < 4 ? gid % B : B + (gid - 4) % B) : gid % B;
+  const uint8_t *xb = st + TILE4_BYTES + src * X16_SRC_STRIDE + h * 256 + tig * 8;
+  const float4 *xc = reinterpret_cast<const float4 *>(st + TILE4_BYTES + 2 * B * X16_SRC_STRIDE) + tig;
 #pragma unroll
   for (int q = 0; q < 2; ++q) {
     const float sc0 = q ? bf16_hi(s0) : bf16_lo(s0), sc1 = q ? bf16_hi(s1) : bf16_lo(s1);
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
-    float c[4] = {0.f, 0.f, 0.f, 0.f};
+      // chunk h * 4 + 2 q + half of the tile: multipliers and offset sums of this lane's columns
+      const float4 mc = xc[(h * 4 + 2 * q + half) * 4];
+      float c[4] = {mc.z, mc.w, mc.z, mc.w};
 #pragma unroll
-    for (int j = 2 * half; j < 2 * half + 2; ++j) {
-      const uint32_t w = j == 0 ? wq[q].x : j == 1 ? wq[q].y : j == 2 ? wq[q].z : wq[q].w;
-      const int k0 = 16 * (4 * q + j);
-      uint32_t b0 = 0u, b1 = 0u;
-      if (xu) {
-        const float2 x0 = *reinterpret_cast<const float2 *>(xs + k0);
-        const float2 x1 = *reinterpret_cast<const float2 *>(xs + k0 + 8);
-        b0 = pack_f16x2(x0.x, x0.y);
-        b1 = pack_f16x2(x1.x, x1.y);
-        if (XSPLIT && gid >= 4) {
-          b0 = pack_f16x2_rest(x0.x, x0.y, b0);
-          b1 = pack_f16x2_rest(x1.x, x1.y, b1);
-        }
+      for (int j = 2 * half; j < 2 * half + 2; ++j) {
+        const uint32_t w = j == 0 ? wq[q].x : j == 1 ? wq[q].y : j == 2 ? wq[q].z : wq[q].w;
+        const uint2 bb = *reinterpret_cast<const uint2 *>(xb + 32 * (4 * q + j));
+        uint32_t a0, a1, a2, a3;
+        int4_frag_f16(w, a0, a1, a2, a3);
+        mma_f16_16816(c, a0, a1, a2, a3, bb.x, bb.y);
       }
-      mma_f16_16816(c, int4_pair_f16(w), int4_pair_f16(w >> 4), int4_pair_f16(w >> 8), int4_pair_f16(w >> 12), b0, b1);
-    }
-    // chunk h * 4 + 2 q + half of the tile: its multipliers, then the rows' group scales
-    const float2 m = *reinterpret_cast<const float2 *>(xm + (h * 4 + 2 * q + half) * MAXB);
-    const float m0 = mu0 ? m.x : 0.f, m1 = mu1 ? m.y : 0.f;
-    acc[0] = fmaf(sc0 * m0, c[0], acc[0]);
-    acc[1] = fmaf(sc0 * m1, c[1], acc[1]);
-    acc[2] = fmaf(sc1 * m0, c[2], acc[2]);
-    acc[3] = fmaf(sc1 * m1, c[3], acc[3]);
+      acc[0] = fmaf(sc0 * mc.x, c[0], acc[0]);
+      acc[1] = fmaf(sc0 * mc.y, c[1], acc[1]);
+      acc[2] = fmaf(sc1 * mc.x, c[2], acc[2]);
+      acc[3] = fmaf(sc1 * mc.y, c[3], acc[3]);
     }
   }
 }
@@ -394,20 +368,12 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
         const bool ok = n < p.n_rows;
         const size_t o = (size_t)b * p.ldh + n;
         const float hn = ok ? pre.h[b][h2] + red[r * MAXB + b] * inv[b] : 0.f;
-        float xv = hn * pre.g[h2];
-        if (p.xmul_out && p.g_next) {
-          // int4 stage: xn in 32-row chunks scaled to fit fp16, with their multipliers
-          float mx = fabsf(xv);
-#pragma unroll
-          for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-          float iv;
-          const float mul = xchunk_scale(mx, &iv);
-          xv *= iv;
-          if (lane == 0) p.xmul_out[(rb * 2 + h2) * MAXB + b] = mul;
-        }
+        const float xv = hn * pre.g[h2];
+        // int4 stage: xn in the tensor-core input form, chunk rb * 2 + h2
+        if (p.xout.hi && p.g_next) act16_put_warp(p.xout, b, rb * 2 + h2, xv, lane);
         if (ok) {
           p.h[o] = hn;
-          if (p.g_next) p.xn[o] = xv;
+          if (p.g_next && !p.xout.hi) p.xn[o] = xv;
           if (p.capture) p.capture[(size_t)b * p.n_rows + n] = hn;
           sq = fmaf(hn, hn, sq);
         }
@@ -427,17 +393,10 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
         const float u = red[(2 * pr + 1) * MAXB + b] * inv[b];
         a = g / (1.0f + expf(-g)) * u;
       }
-      if (p.xmul_out) {
-        // int4 stage: the row block's 32 outputs scaled to fit fp16, with their multiplier
-        float mx = fabsf(a);
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-        float iv;
-        const float mul = xchunk_scale(mx, &iv);
-        a *= iv;
-        if (lane == 0) p.xmul_out[rb * MAXB + b] = mul;
-      }
-      if (ok) p.out[(size_t)b * p.ldo + j] = a;
+      if (p.xout.hi)
+        act16_put_warp(p.xout, b, rb, a, lane);  // int4 stage: the row block's 32 outputs, one chunk
+      else if (ok)
+        p.out[(size_t)b * p.ldo + j] = a;
     }
   } else if constexpr (EPI == EPI_QKV) {
     const int hd = p.head_dim, half = hd >> 1;

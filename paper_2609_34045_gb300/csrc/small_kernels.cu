@@ -11,7 +11,7 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
                                                          const int *positions_in, const uint16_t *embed,
                                                          int vocab, int d, int ldh, const float *g_next,
                                                          float *h, float *xn, float *sumsq, int *positions,
-                                                         int max_ctx, unsigned *err, unsigned *bar, float *xmul) {
+                                                         int max_ctx, unsigned *err, unsigned *bar, Act16 xn16) {
   __shared__ float vals[64];
   const int b = blockIdx.y, tid = threadIdx.x, r = blockIdx.x * 64 + tid;
   pdl_launch_dependents();
@@ -41,19 +41,13 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
     h[(size_t)b * ldh + r] = v;
   }
   if (g_next) {
-    // xn = h * g; for int4 weights in 32-element chunks scaled to fit fp16 (one warp per chunk),
+    // xn = h * g; for int4 weights in the tensor-core input form (one warp per 32-element chunk),
     // exactly as the residual epilogue writes it
-    float xv = r < d ? v * g_next[r] : 0.f;
-    if (xmul) {
-      float mx = fabsf(xv);
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-      float iv;
-      const float mul = xchunk_scale(mx, &iv);
-      xv *= iv;
-      if ((tid & 31) == 0) xmul[(blockIdx.x * 2 + (tid >> 5)) * MAXB + b] = mul;
-    }
-    if (r < d) xn[(size_t)b * ldh + r] = xv;
+    const float xv = r < d ? v * g_next[r] : 0.f;
+    if (xn16.hi)
+      act16_put_warp(xn16, b, blockIdx.x * 2 + (tid >> 5), xv, tid & 31);
+    else if (r < d)
+      xn[(size_t)b * ldh + r] = xv;
   }
   // the block's sum of squares in exactly the order of the residual epilogue (lane l: rows l
   // and l + 32 by fma, then a butterfly), so that a stage fed this hidden state computes the same
@@ -72,10 +66,10 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in, int batch,
                                const uint16_t *embed, int vocab, int d, int ldh, const float *g_next, float *h,
                                float *xn, float *sumsq, int *positions, int max_ctx, unsigned *err,
-                               unsigned *bar, float *xmul, cudaStream_t s) {
+                               unsigned *bar, Act16 xn16, cudaStream_t s) {
   dim3 grid((d + 63) / 64, batch);
   stage_input_kernel<<<grid, 64, 0, s>>>(ids, hidden_in, positions_in, embed, vocab, d, ldh, g_next, h, xn, sumsq,
-                                         positions, max_ctx, err, bar, xmul);
+                                         positions, max_ctx, err, bar, xn16);
   return cudaGetLastError();
 }
 
@@ -145,9 +139,9 @@ cudaError_t launch_repack_bf16(const uint16_t *src, int n_src_rows, int k, const
 // codes of a tile are 2048 words; word ((((h * 4 + r16) * 2 + q) * 32 + lane) * 4 + j) holds the
 // eight codes lane needs for K step s = 4 q + j of K half h and row group r16 (rows r16 * 16 +
 // gid and + 8, gid = lane / 4; columns 2 tig, 2 tig + 1, 2 tig + 8, 2 tig + 9 of the step, tig =
-// lane % 4), nibble i at bits 4 i: row + 8 (i & 1), column + 8 ((i >> 1) & 1) + ((i >> 2) & 1), so
-// that (word >> 4 i) & 0x000F000F, i < 4, is the bf16 pair of one A register.  Scales stay
-// [64 rows][4 groups of 64].
+// lane % 4), nibble i at bits 4 i: row + 8 ((i >> 1) & 1), column + 8 (i & 1) + ((i >> 2) & 1),
+// so that the nibble pairs at bits (0, 16), (8, 24), (4, 20), (12, 28) are the A registers a0,
+// a1, a2, a3 (int4_frag_f16).  Scales stay [64 rows][4 groups of 64].
 __global__ void repack_int4_kernel(const uint32_t *words, const uint16_t *scales, int n_src_rows, int k,
                                    const int *row_map, int n_rows_out, int n_rb, int n_kt, uint8_t *dst) {
   constexpr int TW = TILE4_CODE_BYTES / 4;  // words per tile
@@ -164,8 +158,8 @@ __global__ void repack_int4_kernel(const uint32_t *words, const uint16_t *scales
     const int gid = lane >> 2, tig = lane & 3;
     uint32_t out = 0;
     for (int i = 0; i < 8; ++i) {
-      const int orow = rb * RB + r16 * 16 + gid + 8 * (i & 1);
-      const int kk = kt * KT4 + 128 * h + 16 * (4 * q + j) + 2 * tig + 8 * ((i >> 1) & 1) + ((i >> 2) & 1);
+      const int orow = rb * RB + r16 * 16 + gid + 8 * ((i >> 1) & 1);
+      const int kk = kt * KT4 + 128 * h + 16 * (4 * q + j) + 2 * tig + 8 * (i & 1) + ((i >> 2) & 1);
       int srow = -1;
       if (orow < n_rows_out) srow = row_map ? row_map[orow] : orow;
       if (srow >= n_src_rows) srow = -1;

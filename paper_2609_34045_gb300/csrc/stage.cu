@@ -59,6 +59,12 @@ struct Plan {
   size_t bytes_weights, bytes_kv, bytes_ws;
 };
 
+// Bytes of one int4 GEMV input (Act16) of row length ld: MAXB fp16 rows (and their rests), and
+// the per-chunk constants.
+size_t act16_bytes(int ld, bool with_rest) {
+  return (size_t)MAXB * ld * 2 * (with_rest ? 2 : 1) + (size_t)ld / XCHUNK * XC_CHUNK_FLOATS * 4;
+}
+
 int env_int(const char *name, int dflt) {
   const char *v = std::getenv(name);
   return (v && *v) ? std::atoi(v) : dflt;
@@ -107,12 +113,15 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   p->lm = mat_shape(p->V, p->d, f);
   p->kv_elems_per_layer = (size_t)c->max_batch * p->hkv * c->max_ctx * p->hd;
   p->n_sm = n_sm;
-  p->ctas_per_sm = env_int("KFL_GEMV_CTAS_PER_SM", 1);
-  if (p->ctas_per_sm < 1 || p->ctas_per_sm > 2) p->ctas_per_sm = 1;
-  // 10 stages (169 KiB at batch 1) leave room for one CTA per SM: the next GEMV's CTA starts on
-  // an SM when this one leaves it and fills its ring during the rest of this GEMV's tail
-  p->stages = env_int("KFL_GEMV_STAGES", 10);
-  if (p->stages < 2 || p->stages > 13) p->stages = 10;
+  // Two CTAs per SM: a single CTA's consumer warps (8) leave the tile loop bound by instruction
+  // latency (int4 decoding; bf16 at batch 4), two give every SM twice the warps to hide it.  The
+  // rings are sized so that two fit an SM at every batch size: 5 bf16 stages (at most 90 KiB),
+  // 7 int4 stages (at most 93 KiB); that is about 80 KiB of weights in flight per SM.
+  const bool i4 = f == KFL_INT4_G64;
+  p->ctas_per_sm = env_int("KFL_GEMV_CTAS_PER_SM", 2);
+  if (p->ctas_per_sm < 1 || p->ctas_per_sm > 2) p->ctas_per_sm = 2;
+  p->stages = env_int("KFL_GEMV_STAGES", i4 ? 7 : 5);
+  if (p->stages < 2 || p->stages > 13) p->stages = i4 ? 7 : 5;
   p->gemv_grid_max = n_sm * p->ctas_per_sm;
   int nrb = 1;
   if (p->nl > 0) {
@@ -146,7 +155,7 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   size_t ws = 0;
   ws += (size_t)c->max_ctx * (p->hd / 2) * 4 * 2;                      // rope tables
   ws += (size_t)MAXB * (2 * p->ldh + 2 * p->ldq + p->lda) * 4;         // h, xn, q, o, a
-  ws += (size_t)MAXB * (p->ldh + p->ldq + p->lda) / XCHUNK * 4;        // int4 input multipliers
+  ws += act16_bytes(p->ldh, true) + act16_bytes(p->ldq, false) + act16_bytes(p->lda, false);  // int4 inputs
   ws += (size_t)p->n_parts * MAXB * 4;                                 // sum of squares
   ws += 2 * MAXB * 4;                                                  // positions, next ids
   ws += (size_t)4 * p->gemv_grid_max * 2 * RB * MAXB * 4;              // stream-K partials (x4)
@@ -176,8 +185,8 @@ struct kfl_stage {
   uint16_t *kc = nullptr, *vc = nullptr;
   float *rope_cos = nullptr, *rope_sin = nullptr;
   float *h = nullptr, *xn = nullptr, *q = nullptr, *o = nullptr, *a = nullptr, *sumsq = nullptr;
-  // int4 stages: multipliers of the fp16-scaled GEMV inputs ([chunks of 32][MAXB]; o's are 1)
-  float *xn_mul = nullptr, *a_mul = nullptr, *o_mul = nullptr;
+  // int4 stages: the GEMV inputs in the tensor cores' fp16 form (xn with its rests, for Q/K/V)
+  Act16 xn16 = {}, a16 = {}, o16 = {};
   int *pos = nullptr, *next_int = nullptr;
   int *io_pos = nullptr, *io_ids = nullptr;  // host-buffer decode staging
   float *io_hin = nullptr;
@@ -325,7 +334,7 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
       g.head_dim = P.hd;
       g.max_ctx = c.max_ctx;
       g.n_kv_heads = P.hkv;
-      if (i4) g.xmul = st->xn_mul;
+      if (i4) g.xin = st->xn16;
       gemv(EPI_QKV, g);
     }
     {
@@ -338,6 +347,7 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
       a.positions = st->pos;
       a.o = st->o;
       a.ldo = P.ldq;
+      if (i4) a.o16 = st->o16;
       a.partial = st->attn_partial;
       a.tickets = st->attn_tickets;
       a.batch = batch;
@@ -359,8 +369,8 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
       g.g_next = L.g_ffn;
       g.sumsq_out = st->sumsq;
       if (i4) {
-        g.xmul = st->o_mul;
-        g.xmul_out = st->xn_mul;
+        g.xin = st->o16;
+        g.xout = st->xn16;
       }
       gemv(EPI_RESID, g);
     }
@@ -373,8 +383,8 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
       g.out = st->a;
       g.ldo = P.lda;
       if (i4) {
-        g.xmul = st->xn_mul;
-        g.xmul_out = st->a_mul;
+        g.xin = st->xn16;
+        g.xout = st->a16;
       }
       gemv(EPI_SWIGLU, g);
     }
@@ -387,8 +397,8 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
       g.sumsq_out = st->sumsq;
       g.capture = st->capture ? st->capture + (size_t)l * c.max_batch * P.d : nullptr;
       if (i4) {
-        g.xmul = st->a_mul;
-        g.xmul_out = st->xn_mul;
+        g.xin = st->a16;
+        g.xout = st->xn16;
       }
       gemv(EPI_RESID, g);
     }
@@ -403,7 +413,7 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
     g.cand_idx = st->cand_idx;
     g.argmax_ticket = st->am_ticket;
     g.next_ids = st->next_int;
-    if (i4) g.xmul = st->xn_mul;
+    if (i4) g.xin = st->xn16;
     gemv(EPI_ARGMAX, g);
   }
   if (!dataflow && st->trace) {
@@ -599,7 +609,7 @@ int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const in
     CK(cudaEventRecord(st->ev[0], s));
     CK(launch_stage_input(ids, hidden_in, positions, batch, embed ? st->embed : nullptr, P.V, P.d, P.ldh,
                           input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, st->bar,
-                          st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn_mul : nullptr, s));
+                          st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn16 : Act16{}, s));
     CK(cudaEventRecord(st->ev[1], s));
     kinds.push_back(KFL_KERNEL_INPUT);
     int rc = enqueue_body(st, batch, s, false, &kinds, 1);
@@ -620,7 +630,7 @@ int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const in
   }
   CK(launch_stage_input(ids, hidden_in, positions, batch, embed ? st->embed : nullptr, P.V, P.d, P.ldh,
                         input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, st->bar,
-                        st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn_mul : nullptr, s));
+                        st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn16 : Act16{}, s));
   if (body) {
     int rc = ensure_graph(st, batch);
     if (rc != KFL_OK) return rc;
@@ -801,9 +811,22 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
   AL(st->o, (size_t)MAXB * P.ldq * 4);
   AL(st->a, (size_t)MAXB * P.lda * 4);
   AL(st->sumsq, (size_t)P.n_parts * MAXB * 4);
-  AL(st->xn_mul, (size_t)MAXB * P.ldh / XCHUNK * 4);
-  AL(st->a_mul, (size_t)MAXB * P.lda / XCHUNK * 4);
-  AL(st->o_mul, (size_t)MAXB * P.ldq / XCHUNK * 4);
+  {
+    // int4 GEMV inputs (allocated for every stage; zero where nothing writes: the padding)
+    Act16 *acts[3] = {&st->xn16, &st->o16, &st->a16};
+    const int lds[3] = {P.ldh, P.ldq, P.lda};
+    for (int i = 0; i < 3; ++i) {
+      Act16 &x = *acts[i];
+      x.ld = lds[i];
+      AL(x.hi, (size_t)MAXB * x.ld * 2);
+      if (i == 0) AL(x.lo, (size_t)MAXB * x.ld * 2);
+      AL(x.xc, (size_t)x.ld / XCHUNK * XC_CHUNK_FLOATS * 4);
+      if (cudaMemset(x.hi, 0, (size_t)MAXB * x.ld * 2) != cudaSuccess ||
+          (x.lo && cudaMemset(x.lo, 0, (size_t)MAXB * x.ld * 2) != cudaSuccess) ||
+          cudaMemset(x.xc, 0, (size_t)x.ld / XCHUNK * XC_CHUNK_FLOATS * 4) != cudaSuccess)
+        return fail(KFL_ERR_CUDA);
+    }
+  }
   AL(st->pos, MAXB * 4);
   AL(st->next_int, MAXB * 4);
   AL(st->gemv_partial, (size_t)4 * P.gemv_grid_max * 2 * RB * MAXB * 4);
@@ -832,15 +855,8 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
       cudaMemset(st->tickets, 0, (size_t)(4 * P.n_rb_max + 1) * 4) ||
       cudaMemset(st->counters, 0, (size_t)std::max(1, P.n_phases) * P.ctr_stride * 4) ||
       cudaMemset(st->attn_tickets, 0, (size_t)MAXB * P.hkv * 4) || cudaMemset(st->err, 0, 16) ||
-      cudaMemset(st->bar, 0, 16) || cudaMemset(st->xn_mul, 0, (size_t)MAXB * P.ldh / XCHUNK * 4) ||
-      cudaMemset(st->a_mul, 0, (size_t)MAXB * P.lda / XCHUNK * 4))
+      cudaMemset(st->bar, 0, 16))
     return fail(KFL_ERR_CUDA);
-  {
-    // the attention output needs no scaling: its multipliers are all 1
-    std::vector<float> ones((size_t)MAXB * P.ldq / XCHUNK, 1.0f);
-    if (cudaMemcpy(st->o_mul, ones.data(), ones.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
-      return fail(KFL_ERR_CUDA);
-  }
   // RoPE table: angle pos * theta^(-2i/hd) in fp64, stored as fp32 cos / sin
   {
     const int half = P.hd / 2;

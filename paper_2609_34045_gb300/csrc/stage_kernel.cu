@@ -181,11 +181,11 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
     if (lane == 0) {
       const uint64_t pol_ring = policy_evict_first();
       const uint64_t pol_l2 = policy_evict_normal();
-      const uint32_t bytes = WBYTES + B * (KTILE * 4) + (FMT == 1 ? XMUL_TILE_BYTES : 0);
       struct Cursor {
         int k, i, n;
         long long t0;
         const uint8_t *w;
+        uint32_t bytes;  // a stage's copies: the tile and its activations
       };
       auto seek = [&](Cursor &cu, int from) {
         for (int k = from; k < kp.n_phases; ++k) {
@@ -200,6 +200,8 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
           cu.n = n;
           cu.t0 = t0;
           cu.w = ph->g.w;
+          cu.bytes = WBYTES + (FMT == 0 ? B * (KTILE * 4)
+                                        : (ph->g.xsplit ? 2 * B : B) * X16_SRC_BYTES + XC_TILE_BYTES);
           return;
         }
         cu.k = kp.n_phases;
@@ -225,7 +227,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
         }
         if (round > 0 && !consumer_wait(smem_addr(&empty[s]), (round & 1) ^ 1, &s_abort, kp.err)) break;
         const uint32_t fb = smem_addr(&full[s]);
-        mbar_arrive_expect_tx(fb, bytes);
+        mbar_arrive_expect_tx(fb, cr.bytes);
         bulk_g2s(smem_addr(ring + (size_t)s * SB), cr.w + (size_t)(cr.t0 + cr.i) * WBYTES, WBYTES, fb, pol_ring);
         mbar_arrive(smem_addr(&armed[s]));
         s_issued = ++gi;
@@ -298,11 +300,20 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
             const uint32_t fb = smem_addr(&full[s]);
             const uint32_t dst = smem_addr(ring + (size_t)s * SB + WBYTES);
             const int ktj = (kt + j) % n_kt;
+            if constexpr (FMT == 0) {
 #pragma unroll
-            for (int b = 0; b < B; ++b)
-              bulk_g2s(dst + b * (KTILE * 4), x + (size_t)b * ldx + (size_t)ktj * KTILE, KTILE * 4, fb, pol);
-            if constexpr (FMT == 1)
-              bulk_g2s(dst + B * (KTILE * 4), g.xmul + (size_t)ktj * (KT4 / XCHUNK) * MAXB, XMUL_TILE_BYTES, fb, pol);
+              for (int b = 0; b < B; ++b)
+                bulk_g2s(dst + b * (KTILE * 4), x + (size_t)b * ldx + (size_t)ktj * KTILE, KTILE * 4, fb, pol);
+            } else {
+              const int nsrc = g.xsplit ? 2 * B : B;
+              for (int r = 0; r < nsrc; ++r) {
+                const uint16_t *src = (r < B ? g.xin.hi + (size_t)r * g.xin.ld
+                                             : g.xin.lo + (size_t)(r - B) * g.xin.ld) + (size_t)ktj * KT4;
+                bulk_g2s(dst + r * X16_SRC_STRIDE, src, X16_SRC_BYTES, fb, pol);
+              }
+              bulk_g2s(dst + 2 * B * X16_SRC_STRIDE, g.xin.xc + (size_t)ktj * (KT4 / XCHUNK) * XC_CHUNK_FLOATS,
+                       XC_TILE_BYTES, fb, pol);
+            }
             if (++s == S) {
               s = 0;
               aph ^= 1u;
