@@ -42,18 +42,19 @@ __device__ __forceinline__ void cp_async_wait() {
 
 template <int HD, int NBUF>
 struct AttnLayout {
-  // K and V rows padded by 16 bytes (4 banks) so that the MMA fragments of 8 consecutive rows
-  // fall in distinct banks; q rows (fp32) padded by 8 floats, score rows by 4
+  // K and V rows padded by 16 bytes (4 banks) so that the MMA fragments (and the transposing
+  // loads) of 8 consecutive rows fall in distinct banks; score rows padded by 4 floats
   static constexpr int KROW = HD * 2 + 16;
   static constexpr int VROW = HD * 2 + 16;
-  static constexpr int QS = HD + 8;
   static constexpr int SS = ATT_SUB + 4;
   static constexpr int K_OFF = 0;
   static constexpr int V_OFF = K_OFF + NBUF * ATT_SUB * KROW;
-  static constexpr int Q_OFF = V_OFF + NBUF * ATT_SUB * VROW;
-  static constexpr int S_OFF = Q_OFF + ATT_MAXG * QS * 4;
+  static constexpr int S_OFF = V_OFF + NBUF * ATT_SUB * VROW;
   static constexpr int M_OFF = S_OFF + ATT_MAXG * SS * 4;
-  static constexpr int BYTES = M_OFF + 4 * ATT_MAXG * 4;
+  // q and P as MMA A fragments: [K step][lane] x (rounded a0, a2, rest a0, a2)
+  static constexpr int QF_OFF = M_OFF + 4 * ATT_MAXG * 4;
+  static constexpr int PF_OFF = QF_OFF + (HD / 16) * 32 * 16;
+  static constexpr int BYTES = PF_OFF + (ATT_SUB / 16) * 32 * 16;
   static constexpr int MERGE_MAX = (NBUF * ATT_SUB * KROW) / 8;  // chunks x heads in the K buffers
   static_assert(MERGE_MAX >= 1024, "merge scratch too small");
 };
@@ -154,21 +155,30 @@ __device__ __forceinline__ void attn_publish(const AttnParams &p, int kvh, int t
   if (tid == 0) red_add_release(p.out_ready + kvh, 1u);
 }
 
-// fp32 -> TF32 (round to nearest, ties away), as the MMA's operand bits
-__device__ __forceinline__ uint32_t to_tf32(float x) {
-  uint32_t r;
-  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
-  return r;
-}
-
-// d += a b for one m16n8k8 TF32 tile (a: 16x8 row-major, b: 8x8 column-major, fp32 accumulate).
-// Rows 8..15 of a are the zero padding of the at most 8 heads, so a1 = a3 = 0.
-__device__ __forceinline__ void mma_tf32(float (&d)[4], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
+// d += a b for one m16n8k16 bf16 tile (a: 16x16 row-major, b: 16x8 column-major, fp32
+// accumulate).  Rows 8..15 of a are the zero padding of the at most 8 heads, so a1 = a3 = 0.
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
   asm volatile(
-      "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
       "{%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
+}
+
+// Four (two) 8 x 8 blocks of 16-bit values, transposed: lanes 8 i .. 8 i + 7 address the rows of
+// block i (16-byte aligned); a lane receives elements (2 (lane % 4), lane / 4) and
+// (2 (lane % 4) + 1, lane / 4) of each block, the B fragment layout of the MMA.
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3, const void *p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(smem_addr(p))
+               : "memory");
+}
+__device__ __forceinline__ void ldsm_x2_trans(uint32_t &r0, uint32_t &r1, const void *p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0,%1}, [%2];"
+               : "=r"(r0), "=r"(r1)
+               : "r"(smem_addr(p))
+               : "memory");
 }
 
 // int4 stages: the output of heads (kvh, og), dimensions od .. od + 3, also in the O
@@ -191,7 +201,6 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
   using L = AttnLayout<HD, NBUF>;
   uint8_t *sk = sm + L::K_OFF;
   uint8_t *sv = sm + L::V_OFF;
-  float *sq = reinterpret_cast<float *>(sm + L::Q_OFF);
   float *ss = reinterpret_cast<float *>(sm + L::S_OFF);
   float *s_m = reinterpret_cast<float *>(sm + L::M_OFF);
   float *s_l = s_m + ATT_MAXG;
@@ -226,43 +235,48 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
   else
     load_sub(0, 0);
 
+  // MMA fragment coordinates: lane = 4 * gid + tig; accumulator rows gid are heads (gid < G)
+  const int gid = lane >> 2, tig = lane & 3;
+  const bool hrow = gid < G;
+  constexpr int KS = HD / 16;   // K steps of the scores
+  constexpr int NT = HD / 64;   // P V n-tiles (8 dimensions) per warp: warp w owns dims NT*8*w ...
+  const int n_base = warp * NT * 8;
+  uint4 *qf = reinterpret_cast<uint4 *>(sm + L::QF_OFF);
+  uint4 *pf = reinterpret_cast<uint4 *>(sm + L::PF_OFF);
   {
-    // q rows of the group: loads first (independent), then the scaled stores
-    constexpr int QPT = (ATT_MAXG * HD + ATT_THREADS - 1) / ATT_THREADS;
-    float qv[QPT];
+    // q (scaled to log2 units) as the scores' A fragments, a bf16 pair each (rounded, rest:
+    // about 2^-17 relative, for the softmax turns a relative error e of a score s into an error
+    // of about |s| e of its weight): entry (step s, lane) = rounded a0, a2, rest a0, a2 of rows
+    // gid (heads; rows gid + 8 and gid >= G are zero)
+    if (tid < KS * 32) {
+      const int st = tid >> 5, l = tid & 31, g = l >> 2, t = l & 3;
+      uint4 f = make_uint4(0u, 0u, 0u, 0u);
+      if (g < G) {
+        const float *qg = p.q + (size_t)b * p.n_heads * HD + (size_t)(kvh * G + g) * HD + 16 * st + 2 * t;
+        const float2 x0 = __ldcg(reinterpret_cast<const float2 *>(qg));
+        const float2 x1 = __ldcg(reinterpret_cast<const float2 *>(qg + 8));
+        const float v[4] = {x0.x * p.scale_log2, x0.y * p.scale_log2, x1.x * p.scale_log2, x1.y * p.scale_log2};
+        uint16_t hi[4], lo[4];
 #pragma unroll
-    for (int i = 0; i < QPT; ++i) {
-      const int e = tid + i * ATT_THREADS;
-      qv[i] = e < G * HD ? __ldcg(p.q + (size_t)b * p.n_heads * HD + (size_t)kvh * G * HD + e) : 0.f;
-    }
-#pragma unroll
-    for (int i = 0; i < QPT; ++i) {
-      const int e = tid + i * ATT_THREADS;
-      if (e < G * HD) {
-        const int g = e / HD, d = e % HD;
-        sq[g * L::QS + d] = qv[i] * p.scale_log2;
+        for (int i = 0; i < 4; ++i) {
+          hi[i] = f32_to_bf16_rne(v[i]);
+          lo[i] = f32_to_bf16_rne(v[i] - bf16_to_f32(hi[i]));
+        }
+        f = make_uint4(hi[0] | ((uint32_t)hi[1] << 16), hi[2] | ((uint32_t)hi[3] << 16),
+                       lo[0] | ((uint32_t)lo[1] << 16), lo[2] | ((uint32_t)lo[3] << 16));
       }
+      qf[tid] = f;
     }
+    // P fragments of rows gid >= G stay zero for the whole unit
+    if (tid < (ATT_SUB / 16) * 32 && ((tid & 31) >> 2) >= G) pf[tid] = make_uint4(0u, 0u, 0u, 0u);
   }
   if (tid < ATT_MAXG) {
     s_m[tid] = -INFINITY;
     s_l[tid] = 0.f;
   }
-
-  // MMA fragment coordinates: lane = 4 * gid + tig; accumulator rows gid are heads (gid < G)
-  const int gid = lane >> 2, tig = lane & 3;
-  const bool hrow = gid < G;
-  constexpr int KS = HD / 8;    // K steps of the scores
-  constexpr int NT = HD / 64;   // P V n-tiles (8 dimensions) per warp: warp w owns dims NT*8*w ...
-  const int n_base = warp * NT * 8;
   float acc[NT][4];
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
-  // q as A fragments, made from shared memory at each K step.  Within a step of 8 dimensions the
-  // MMA's k = tig, tig + 4 are taken as dimensions 2 tig, 2 tig + 1 (the same order for q and K:
-  // the dot product is unchanged), so that a lane's two K values are one 32-bit load.  q is
-  // carried as a TF32 pair (rounded, rest) so that the scores keep about fp32 precision: the
-  // softmax turns a relative error e of a score s into an error of about |s| e of its weight.
 
   const int nsub = (end - start + ATT_SUB - 1) / ATT_SUB;
   for (int it = 0; it < nsub; ++it) {
@@ -285,20 +299,19 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
       for (int e = tid; e < (ATT_SUB - cnt) * (HD / 8); e += ATT_THREADS)
         *reinterpret_cast<uint4 *>(vb + (cnt + e / (HD / 8)) * L::VROW + (e % (HD / 8)) * 16) = make_uint4(0u, 0u, 0u, 0u);
 
-    // scores of positions 8w .. 8w + 7 for every head (rows gid); four independent accumulator
+    // scores of positions 8w .. 8w + 7 (MMA columns) for every head (rows gid): bf16 m16n8k16
+    // MMAs, K rows as the B fragments (two 32-bit loads per step); four independent accumulator
     // chains (K steps modulo 2, rounded and rest parts of q) so that the MMAs overlap
     {
       float sp[4][4] = {};
       const uint8_t *krow = kb + (8 * warp + gid) * L::KROW + 4 * tig;
 #pragma unroll
-      for (int s8 = 0; s8 < KS; ++s8) {
-        const float2 qv = hrow ? *reinterpret_cast<const float2 *>(sq + gid * L::QS + 8 * s8 + 2 * tig)
-                               : make_float2(0.f, 0.f);
-        const uint32_t qh0 = to_tf32(qv.x), qh2 = to_tf32(qv.y);
-        const uint32_t kw = *reinterpret_cast<const uint32_t *>(krow + 16 * s8);
-        mma_tf32(sp[2 * (s8 & 1)], qh0, qh2, kw << 16, kw & 0xFFFF0000u);
-        mma_tf32(sp[2 * (s8 & 1) + 1], to_tf32(qv.x - __uint_as_float(qh0)), to_tf32(qv.y - __uint_as_float(qh2)),
-                 kw << 16, kw & 0xFFFF0000u);
+      for (int s16 = 0; s16 < KS; ++s16) {
+        const uint4 f = qf[s16 * 32 + lane];
+        const uint32_t k0 = *reinterpret_cast<const uint32_t *>(krow + 32 * s16);
+        const uint32_t k1 = *reinterpret_cast<const uint32_t *>(krow + 32 * s16 + 16);
+        mma_bf16_16816(sp[2 * (s16 & 1)], f.x, f.y, k0, k1);
+        mma_bf16_16816(sp[2 * (s16 & 1) + 1], f.z, f.w, k0, k1);
       }
       float sc[4];
 #pragma unroll
@@ -310,7 +323,7 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
       }
     }
     att_sync();
-    // online softmax update: warp g owns head g
+    // online softmax update: warp g owns head g; its weights go to the P fragments as bf16 pairs
     if (warp < G) {
       const int g = warp;
       const float a0 = ss[g * L::SS + lane], a1 = ss[g * L::SS + lane + 32];
@@ -323,9 +336,17 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
       float sum = e0 + e1;
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-      ss[g * L::SS + lane] = e0;
-      ss[g * L::SS + lane + 32] = e1;
-      __syncwarp();
+      // position pp of the sub-tile: step pp / 16, lane 4 g + ((pp & 7) >> 1), register a0 or a2
+      // (pp & 8), half pp & 1
+      auto put = [&](int pp, float e) {
+        uint16_t *f = reinterpret_cast<uint16_t *>(pf + (pp >> 4) * 32 + 4 * g + ((pp & 7) >> 1));
+        const uint16_t hi = f32_to_bf16_rne(e);
+        const int r = (pp & 8) ? 1 : 0;
+        f[2 * r + (pp & 1)] = hi;
+        f[2 * (2 + r) + (pp & 1)] = f32_to_bf16_rne(e - bf16_to_f32(hi));
+      };
+      put(lane, e0);
+      put(lane + 32, e1);
       if (lane == 0) {
         const float alpha = exp2f(m_old - m_new);
         s_alpha[g] = alpha;
@@ -334,7 +355,8 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
       }
     }
     att_sync();
-    // acc = acc * alpha + P V over the sub-tile (P as A fragments, V as B fragments)
+    // acc = acc * alpha + P V over the sub-tile: P fragments from shared memory, V fragments by
+    // transposing loads (ldmatrix .trans: 8 x 8 blocks of positions x dimensions)
     {
       const float al = hrow ? s_alpha[gid] : 0.f;
 #pragma unroll
@@ -342,21 +364,25 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
         acc[nt][0] *= al;
         acc[nt][1] *= al;
       }
-      const float *prow = ss + gid * L::SS;
-      // this sub-tile's P V in two chains per n-tile (even and odd K steps), then into acc
+      // this sub-tile's P V in two chains per n-tile (rounded and rest parts of P), then into acc
       float pv[NT][2][4] = {};
+      const int mi = lane >> 3;  // the 8 x 8 block whose row this lane addresses
+      const uint8_t *vrow = vb + (8 * (mi & 1) + (lane & 7)) * L::VROW + 2 * (n_base + 8 * (mi >> 1));
 #pragma unroll
-      for (int k8 = 0; k8 < ATT_SUB / 8; ++k8) {
-        const uint32_t pa0 = hrow ? to_tf32(prow[8 * k8 + tig]) : 0u;
-        const uint32_t pa2 = hrow ? to_tf32(prow[8 * k8 + tig + 4]) : 0u;
-        const uint8_t *v0 = vb + (8 * k8 + tig) * L::VROW;
-        const uint8_t *v1 = v0 + 4 * L::VROW;
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-          const int n = n_base + 8 * nt + gid;
-          const uint32_t b0 = (uint32_t)(*reinterpret_cast<const uint16_t *>(v0 + 2 * n)) << 16;
-          const uint32_t b1 = (uint32_t)(*reinterpret_cast<const uint16_t *>(v1 + 2 * n)) << 16;
-          mma_tf32(pv[nt][k8 & 1], pa0, pa2, b0, b1);
+      for (int s16 = 0; s16 < ATT_SUB / 16; ++s16) {
+        const uint4 f = pf[s16 * 32 + lane];
+        if constexpr (NT == 2) {
+          uint32_t v0, v1, v2, v3;
+          ldsm_x4_trans(v0, v1, v2, v3, vrow + 16 * s16 * L::VROW);
+          mma_bf16_16816(pv[0][0], f.x, f.y, v0, v1);
+          mma_bf16_16816(pv[0][1], f.z, f.w, v0, v1);
+          mma_bf16_16816(pv[1][0], f.x, f.y, v2, v3);
+          mma_bf16_16816(pv[1][1], f.z, f.w, v2, v3);
+        } else {
+          uint32_t v0, v1;
+          ldsm_x2_trans(v0, v1, vrow + 16 * s16 * L::VROW);
+          mma_bf16_16816(pv[0][0], f.x, f.y, v0, v1);
+          mma_bf16_16816(pv[0][1], f.z, f.w, v0, v1);
         }
       }
 #pragma unroll

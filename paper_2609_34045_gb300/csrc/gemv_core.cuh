@@ -38,6 +38,15 @@ __device__ __forceinline__ void ffma2(float &a0, float &a1, float w0, float w1, 
       : "f"(w0), "f"(w1), "f"(x0), "f"(x1));
 }
 
+// (d0, d1) = (a0, a1) * (b0, b1) with one packed fp32x2 multiply (sm_100+)
+__device__ __forceinline__ void fmul2(float &d0, float &d1, float a0, float a1, float b0, float b1) {
+  asm("{\n\t.reg .b64 d, a, b;\n\t"
+      "mov.b64 a, {%2, %3};\n\tmov.b64 b, {%4, %5};\n\t"
+      "mul.rn.f32x2 d, a, b;\n\tmov.b64 {%0, %1}, d;\n\t}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+}
+
 // Signed 4-bit code j of a word as an exact float: the offset-binary nibble (code ^ 8) is
 // placed in the mantissa of 2^23, and 2^23 + 8 is subtracted.
 __device__ __forceinline__ float int4_code(uint32_t word, int j) {
@@ -190,10 +199,12 @@ __device__ __forceinline__ void tile_compute_int4(const uint8_t *st, int warp, i
         int4_frag_f16(w, a0, a1, a2, a3);
         mma_f16_16816(c, a0, a1, a2, a3, bb.x, bb.y);
       }
-      acc[0] = fmaf(sc0 * mc.x, c[0], acc[0]);
-      acc[1] = fmaf(sc0 * mc.y, c[1], acc[1]);
-      acc[2] = fmaf(sc1 * mc.x, c[2], acc[2]);
-      acc[3] = fmaf(sc1 * mc.y, c[3], acc[3]);
+      // acc += (sc * m) c, two columns per packed fp32x2 operation
+      float f0, f1, f2, f3;
+      fmul2(f0, f1, sc0, sc0, mc.x, mc.y);
+      fmul2(f2, f3, sc1, sc1, mc.x, mc.y);
+      ffma2(acc[0], acc[1], f0, f1, c[0], c[1]);
+      ffma2(acc[2], acc[3], f2, f3, c[2], c[3]);
     }
   }
 }
