@@ -227,6 +227,9 @@ def run_splits(work, st_full, ids_all, hid_all, pos_all, args, stream):
     consecutive stages on this GPU, the hidden state handed over in a device buffer.  Each split
     is checked bit for bit against the single stage over its first steps (next ids and final
     hidden state), then timed.  Returns a list of per-split results."""
+    import dataclasses
+
+    import numpy as np
     import torch
 
     from paper_2609_34045_gb300 import device_inputs as di
@@ -280,14 +283,84 @@ def run_splits(work, st_full, ids_all, hid_all, pos_all, args, stream):
         e1.record(stream)
         torch.cuda.synchronize()
         ms = e0.elapsed_time(e1) / n_time
+        # each stage of the chain on its own (events between the stages' launches)
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(parts) + 1)] for _ in range(n_time)]
+        for i in range(n_time):
+            j = (n_check + 3 + i) % work.steps
+            for k, s_ in enumerate(parts):
+                evs[i][k].record(stream)
+                K.kfl_stage_decode(s_, ids_all[j] if (k == 0 and ids_all is not None) else None,
+                                   (hid_all[j] if hid_all is not None else None) if k == 0 else hbuf[k - 1],
+                                   pos_all[j], b, hbuf[k], nxt if k == len(parts) - 1 else None, stream.cuda_stream)
+            evs[i][-1].record(stream)
+        torch.cuda.synchronize()
+        stage_ms = [float(np.median([evs[i][k].elapsed_time(evs[i][k + 1]) for i in range(n_time)]))
+                    for k in range(len(parts))]
+        stage_bytes = [dataclasses.replace(work, l0=bounds[k], l1=bounds[k + 1],
+                                           embed_in=work.embed_in and k == 0,
+                                           logits_out=work.logits_out and k == len(parts) - 1,
+                                           splits=()).step_bytes(n_check + 3)
+                       for k in range(len(parts))]
         for s_ in parts:
             if K.kfl_stage_status(s_) != 0:
                 raise RuntimeError("device reported an error in a split stage")
             K.kfl_stage_destroy(s_)
         res.append({"split": list(split), "ms_per_step": ms, "us_per_layer_token": ms * 1e3 / (work.n_layers * b),
                     "steps_timed": n_time, "bit_exact_vs_single_stage": bool(exact),
-                    "steps_compared": n_check})
+                    "steps_compared": n_check, "stage_ms": stage_ms, "stage_bytes": stage_bytes})
     return res
+
+
+def empty_stage_ms(work, stream, n=50):
+    """The fixed per-stage time o of the cost model (Eq. 2): a stage with no blocks that only
+    embeds the token (stage input and output kernels)."""
+    import torch
+
+    from paper_2609_34045_gb300 import device_inputs as di
+    from paper_2609_34045_gb300 import stage as K
+    from paper_2609_34045_gb300 import workload as wl
+
+    m, b = work.model, work.batch
+    st = K.kfl_stage_create(K.model_cfg(m, work.max_ctx, b), 0, 0, K.KFL_EMBED_IN)
+    di.load_stage_seeded(st, work, 0, 0)
+    ids = torch.tensor(wl.first_token_ids(m, b, work.seed), device="cuda")
+    pos = torch.tensor(wl.positions(work, 0), device="cuda")
+    out = torch.empty(b, m.d_model, dtype=torch.float32, device="cuda")
+    for _ in range(5):
+        K.kfl_stage_decode(st, ids, None, pos, b, out, None, stream.cuda_stream)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(n):
+        K.kfl_stage_decode(st, ids, None, pos, b, out, None, stream.cuda_stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    K.kfl_stage_destroy(st)
+    return e0.elapsed_time(e1) / n
+
+
+def cost_model(points, probe_gbs, o_ms):
+    """The paper's per-stage cost (Eq. 2), c = o + bytes / b: each stage's algorithmic HBM bytes
+    (its blocks' weights and KV, and the head's embedding and unembedding) over a bandwidth b.
+    points: [(bytes, measured ms)].  'probe' takes b from a copy benchmark and o from an empty
+    stage, as the planner would; 'fitted' takes (o, b) from a least-squares line through the
+    points.  Returns both, with each stage's predicted time and relative error."""
+    import numpy as np
+
+    x = np.array([p[0] for p in points], dtype=np.float64)
+    y = np.array([p[1] for p in points], dtype=np.float64)
+
+    def evaluate(o, gbs):
+        pred = o + x / (gbs * 1e6)
+        err = (pred - y) / y
+        return {"o_us": o * 1e3, "b_gbs": gbs, "pred_ms": pred.tolist(), "rel_err": err.tolist(),
+                "median_abs_err": float(np.median(np.abs(err)))}
+
+    out = {"stage_bytes": x.tolist(), "measured_ms": y.tolist(), "probe": evaluate(o_ms, probe_gbs)}
+    if len(points) >= 2 and np.ptp(x) > 0:
+        slope, icpt = np.polyfit(x, y, 1)
+        out["fitted"] = evaluate(float(icpt), float(1.0 / (slope * 1e6)))
+    return out
 
 
 def run_ours(args, work):
@@ -412,6 +485,13 @@ def run_ours(args, work):
     e2e_value = e2e_s * 1e6 / (n_layers * b) / world
 
     splits = run_splits(work, st, ids_all, hid_all, pos_all, args, stream) if work.splits and world == 1 else None
+    cost = None
+    if splits:
+        # Eq. 2 against every stage timed here: the whole model as one stage, and each split's stages
+        points = [(work.step_bytes(work.steps // 2), ms)]
+        for r in splits:
+            points += list(zip(r["stage_bytes"], r["stage_ms"]))
+        cost = cost_model(points, measured_peaks()[0], empty_stage_ms(work, stream))
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -446,6 +526,7 @@ def run_ours(args, work):
         }
         if splits is not None:
             line["splits"] = splits
+            line["cost_model"] = cost
         print(json.dumps(line), flush=True)
     K.kfl_stage_destroy(st)
     if dist:
