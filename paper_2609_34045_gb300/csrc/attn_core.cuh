@@ -108,7 +108,7 @@ __device__ __forceinline__ int attn_chunk_size(const AttnParams &p) {
   }
   const long long work = total * p.n_kv_heads;
   const long long want = (work + p.target_units - 1) / max(1, p.target_units);
-  int chunk = static_cast<int>(max(64LL, (want + 63) / 64 * 64));
+  int chunk = static_cast<int>(max((long long)p.chunk, (want + 63) / 64 * 64));  // p.chunk: the smallest
   const int G = p.n_heads / p.n_kv_heads;
   const int need = (maxp1 * G + ATT_MERGE_MAX - 1) / ATT_MERGE_MAX;
   return max(chunk, (need + 63) / 64 * 64);

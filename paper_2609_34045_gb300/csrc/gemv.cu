@@ -29,7 +29,7 @@ constexpr int GEMV_STATIC_SMEM = 2048;  // allowance for the kernel's own __shar
 // FMT 0: bf16 tiles [RB][KT].  FMT 1: int4 tiles, codes [RB][KT4/8] uint32 + scales [RB][KT4/64].
 // Warps 0-7 consume tiles, warp 8 is the TMA producer, warp 9 the epilogue warp.
 template <int B, int EPI, int FMT>
-__global__ void __launch_bounds__(GEMV_THREADS, (B <= 2 || FMT == 0) ? 2 : 1) gemv_kernel(const __grid_constant__ GemvParams p) {
+__global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_constant__ GemvParams p) {
   extern __shared__ __align__(1024) uint8_t smem[];
   constexpr int SB = stage_bytes(B, FMT);
   const int S = p.stages;

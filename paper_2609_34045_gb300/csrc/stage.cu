@@ -54,6 +54,7 @@ struct Plan {
   Mat qkv, o, gu, down, lm;
   size_t kv_elems_per_layer;  // per cache (K or V)
   int n_sm, ctas_per_sm, stages, gemv_grid_max, n_rb_max, n_parts, attn_nchunks_max;
+  int small_gemv_tiles, small_gemv_stages;  // GEMVs of at most this many tiles: one CTA per SM
   int n_phases, ctr_stride;  // persistent kernel: phases per step, readiness counters per phase
   int attn_units;            // attention units a step aims at (the kernels size chunks to it)
   size_t bytes_weights, bytes_kv, bytes_ws;
@@ -123,6 +124,12 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   p->stages = env_int("KFL_GEMV_STAGES", i4 ? 7 : 5);
   if (p->stages < 2 || p->stages > 13) p->stages = i4 ? 7 : 5;
   p->gemv_grid_max = n_sm * p->ctas_per_sm;
+  // bf16 GEMVs of 2 x SMs to 4096 tiles (the 7B Q/K/V and O: 28 tiles per row block) run one
+  // CTA per SM with 6 stages: half the CTAs share each row block, so their combine ends sooner
+  // (7B b=1: -1.4% per step); int4 ones keep two CTAs per SM, which their decoding needs, and
+  // GEMVs of fewer tiles keep one tile per CTA
+  p->small_gemv_tiles = env_int("KFL_SMALL_GEMV_TILES", i4 ? 0 : 4096);
+  p->small_gemv_stages = env_int("KFL_SMALL_GEMV_STAGES", 6);
   int nrb = 1;
   if (p->nl > 0) {
     nrb = p->qkv.n_rb;
@@ -354,7 +361,7 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
       a.n_heads = P.hq;
       a.n_kv_heads = P.hkv;
       a.max_ctx = c.max_ctx;
-      a.chunk = 64;  // the kernels size the step's chunks from its positions
+      a.chunk = std::max(1, env_int("KFL_ATTN_MIN_CHUNK", 64) / 64) * 64;  // the kernels size the step's chunks from its positions (at least this)
       a.n_chunks = (c.max_ctx + 63) / 64;
       a.target_units = P.attn_units;
       a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)P.hd));
@@ -512,8 +519,14 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
     }
     if (ph.kind == PH_GEMV) {
       const long long T = (long long)ph.g.n_rb * ph.g.n_kt;
-      const int grid = (int)(T < st->P.gemv_grid_max ? T : st->P.gemv_grid_max);
-      CK(launch_gemv(ph.g, ph.epi, grid, s, pdl));
+      int grid = (int)(T < st->P.gemv_grid_max ? T : st->P.gemv_grid_max);
+      GemvParams g = ph.g;
+      if (T <= st->P.small_gemv_tiles && T >= 2LL * st->P.n_sm && st->P.ctas_per_sm > 1) {
+        // a small GEMV: one CTA per SM with a deeper ring, so that fewer CTAs share a row block
+        grid = (int)(T < st->P.n_sm ? T : st->P.n_sm);
+        g.stages = std::min(st->P.small_gemv_stages, gemv_max_stages(batch, g.fmt, st->smem_optin));
+      }
+      CK(launch_gemv(g, ph.epi, grid, s, pdl));
     } else {
       CK(launch_attention(ph.a, st->P.hd, s, pdl));
     }
