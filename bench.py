@@ -43,7 +43,8 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=500)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--layers", type=int, default=0,
-                    help="keep only the first N blocks of the stage (small cases for profiling)")
+                    help="small case for profiling: the first N blocks of the stage as a body stage "
+                         "(no embedding, no head, no splits)")
     return ap.parse_args()
 
 
@@ -541,7 +542,8 @@ def main():
     from paper_2609_34045_gb300 import workload as wl
     work = wl.CONFIGS[args.config]
     if args.layers > 0 and args.layers < work.n_layers:
-        work = dataclasses.replace(work, l1=work.l0 + args.layers, name=f"{work.name}-first{args.layers}")
+        work = dataclasses.replace(work, l1=work.l0 + args.layers, name=f"{work.name}-first{args.layers}",
+                                   embed_in=False, logits_out=False, splits=())
     if args.impl == "reference":
         return run_reference(args, work)
     return run_ours(args, work)
