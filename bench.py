@@ -340,6 +340,45 @@ def empty_stage_ms(work, stream, n=50):
     return e0.elapsed_time(e1) / n
 
 
+def plan_example(work, fit):
+    """The planner (Algorithm 1 with head rotation, section V) on a synthetic ring driven by this
+    GPU's measured stage cost: four members stream at 1, 1/2, 1/4 and 1/8 of the fitted rate b
+    with the fitted overhead o, and hold 35, 280, 140 and 70 GB; the bottleneck of the planned
+    division against the evaluation's Uniform and Memory-proportional divisions under the same
+    costs (Eq. 2, ms per step)."""
+    import dataclasses
+
+    from paper_2609_34045_gb300 import stage as K
+
+    m = work.model
+    k = m.n_layers_total
+    cfg = K.model_cfg(m, work.max_ctx, work.batch)
+    mid = dataclasses.replace(work, l0=0, l1=1, embed_in=False, logits_out=False, splits=())
+    beta_block = float(mid.step_bytes(work.steps // 2))
+    head = dataclasses.replace(work, l0=0, l1=0, embed_in=True, logits_out=True, splits=())
+    beta_head = float(head.step_bytes(0))
+    rates = [1.0, 0.5, 0.25, 0.125]
+    rooms = [35e9, 280e9, 140e9, 70e9]
+    bw = [fit["b_gbs"] * 1e6 * r for r in rates]  # bytes per ms
+    devs = [dict(o=fit["o_us"] * 1e-3, bw=b, lim_body=K.kfl_block_limit(cfg, int(room), False),
+                 lim_head=K.kfl_block_limit(cfg, int(room), True)) for b, room in zip(bw, rooms)]
+    n, plan, rc = K.kfl_plan_ring(k, devs, 0, beta_block, beta_head, 0.05)
+
+    def bottleneck(div, h):
+        return max(devs[i]["o"] + (beta_head / bw[i] if i == h else 0.0) + div[i] * beta_block / bw[i]
+                   for i in range(len(devs)))
+    out = {"members_rate_of_measured": rates, "members_memory_gb": [r / 1e9 for r in rooms],
+           "blocks": k, "beta_block_bytes": beta_block, "beta_head_bytes": beta_head,
+           "lim_body": [d["lim_body"] for d in devs], "lim_head": [d["lim_head"] for d in devs]}
+    if rc == 0:
+        out.update(partition={"blocks": n, "head": plan["head"], "bottleneck_ms": plan["tau"]})
+    for name, w in (("uniform", None), ("memory_proportional", rooms)):
+        div = K.kfl_divide(k, len(devs), w)
+        fits = all(div[i] <= (devs[i]["lim_head"] if i == 0 else devs[i]["lim_body"]) for i in range(len(devs)))
+        out[name] = {"blocks": div, "head": 0, "bottleneck_ms": bottleneck(div, 0), "fits_memory": fits}
+    return out
+
+
 def cost_model(points, probe_gbs, o_ms):
     """The paper's per-stage cost (Eq. 2), c = o + bytes / b: each stage's algorithmic HBM bytes
     (its blocks' weights and KV, and the head's embedding and unembedding) over a bandwidth b.
@@ -493,6 +532,8 @@ def run_ours(args, work):
         for r in splits:
             points += list(zip(r["stage_bytes"], r["stage_ms"]))
         cost = cost_model(points, measured_peaks()[0], empty_stage_ms(work, stream))
+        if "fitted" in cost:
+            cost["plan_example"] = plan_example(work, cost["fitted"])
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

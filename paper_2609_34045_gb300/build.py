@@ -1,7 +1,7 @@
 """Build the in-tree CUDA library ``libkafila_stage.so`` for sm_103a with nvcc.
 
-Each ``csrc/*.cu`` file is compiled in parallel into ``_build/`` and linked into one shared
-library next to this file.  A file is recompiled only when it or a header is newer than its
+Each ``csrc/*.cu`` file (and host-only ``csrc/*.cpp`` file) is compiled in parallel into
+``_build/`` and linked into one shared library next to this file.  A file is recompiled only when it or a header is newer than its
 object.  No cmake, no torch extension machinery: the library has a plain C ABI.
 """
 from __future__ import annotations
@@ -45,11 +45,11 @@ def build(verbose: bool = False, ptxas_verbose: bool = False) -> str:
     """Compile and link; returns the library path."""
     os.makedirs(BUILD, exist_ok=True)
     cc = nvcc()
-    srcs = sorted(glob.glob(os.path.join(CSRC, "*.cu")))
+    srcs = sorted(glob.glob(os.path.join(CSRC, "*.cu")) + glob.glob(os.path.join(CSRC, "*.cpp")))
     deps = _headers()
     jobs = []
     for src in srcs:
-        obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(BUILD, os.path.splitext(os.path.basename(src))[0] + ".o")
         if _stale(obj, src, deps) or ptxas_verbose:
             cmd = [cc, *ARCH, *NVCC_FLAGS, "-I", os.path.join(ROOT, "include"), "-c", src, "-o", obj]
             if ptxas_verbose:
@@ -67,7 +67,7 @@ def build(verbose: bool = False, ptxas_verbose: bool = False) -> str:
         for src, r in outs.items():
             if r.stdout or r.stderr:
                 print(f"== {os.path.basename(src)}\n{r.stdout}{r.stderr}", file=sys.stderr)
-    objs = [os.path.join(BUILD, os.path.basename(s)[:-3] + ".o") for s in srcs]
+    objs = [os.path.join(BUILD, os.path.splitext(os.path.basename(s))[0] + ".o") for s in srcs]
     if jobs or not os.path.exists(LIB) or any(os.path.getmtime(o) > os.path.getmtime(LIB) for o in objs):
         tmp = LIB + ".tmp"
         cmd = [cc, *ARCH, "-shared", "-o", tmp, *objs, "-cudart", "static"]

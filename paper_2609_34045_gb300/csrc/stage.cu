@@ -13,6 +13,7 @@
 #include <cstring>
 #include <vector>
 
+#include "../../include/kafila_plan.h"
 #include "../../include/kafila_stage.h"
 #include "../../include/kafila_synth.h"
 #include "common.cuh"
@@ -1219,6 +1220,7 @@ extern "C" const char *kfl_strerror(int code) {
     case KFL_ERR_CUDA: return "CUDA runtime error";
     case KFL_ERR_STATE: return "stage not ready (weights not loaded) or invalid";
     case KFL_ERR_TIMEOUT: return "a bounded device-side wait gave up";
+    case KFL_ERR_INFEASIBLE: return "no division of the blocks fits the devices";
     default: return "unknown error";
   }
 }

@@ -51,6 +51,18 @@ class kfl_weights(C.Structure):
                 ("embed", C.c_void_p), ("final_norm", C.c_void_p), ("lm_head", kfl_matrix)]
 
 
+class kfl_plan_device(C.Structure):
+    _fields_ = [("o", C.c_double), ("bw", C.c_double), ("throughput", C.c_double), ("working_set", C.c_double),
+                ("lim_body", C.c_int), ("lim_head", C.c_int)]
+
+
+class kfl_plan(C.Structure):
+    _fields_ = [("tier", C.c_int), ("head", C.c_int), ("tau", C.c_double), ("tau_anchor", C.c_double),
+                ("undersized", C.c_int)]
+
+
+KFL_ERR_INFEASIBLE = -7
+
 _lib = None
 
 
@@ -88,6 +100,11 @@ def lib() -> C.CDLL:
             "kfl_head_argmax_noalloc": ([vp, vp, vp, i, i, i, C.c_float, vp, vp], i),
             "kfl_synth_key": ([C.c_uint64, C.c_uint64], C.c_uint64),
             "kfl_synth_fill": ([vp, C.c_int64, C.c_uint64, C.c_uint64, i, C.c_float, C.c_float, C.c_int64, vp], i),
+            "kfl_partition": ([i, i, vp, vp, vp, vp, C.POINTER(C.c_double)], i),
+            "kfl_plan_ring": ([i, i, C.POINTER(kfl_plan_device), i, C.c_double, C.c_double, C.c_double, vp,
+                               C.POINTER(kfl_plan)], i),
+            "kfl_divide": ([i, i, vp, vp], i),
+            "kfl_block_limit": ([C.POINTER(kfl_model_cfg), sz, i, C.POINTER(i)], i),
         }
         for name, (args, res) in sigs.items():
             f = getattr(L, name)
@@ -292,3 +309,49 @@ def kfl_synth_key(seed: int, tag: int) -> int:
 def kfl_synth_fill(dst, n: int, seed: int, tag: int, kind: int, c: float, mean: float = 0.0, start: int = 0,
                    cuda_stream: int | None = None) -> None:
     _check(lib().kfl_synth_fill(_ptr(dst), n, seed, tag, kind, c, mean, start, cuda_stream), "kfl_synth_fill")
+
+
+# ---- planner (include/kafila_plan.h): host code, no GPU needed ------------------------------
+
+def kfl_partition(k: int, fixed, per, lim):
+    """Algorithm 1: (block counts, bottleneck), or raises KflError (KFL_ERR_INFEASIBLE)."""
+    import numpy as np
+    m = len(fixed)
+    f = np.ascontiguousarray(fixed, dtype=np.float64)
+    p = np.ascontiguousarray(per, dtype=np.float64)
+    li = np.ascontiguousarray(lim, dtype=np.int32)
+    n = np.zeros(m, dtype=np.int32)
+    tau = C.c_double(0.0)
+    _check(lib().kfl_partition(k, m, f.ctypes.data, p.ctypes.data, li.ctypes.data, n.ctypes.data, C.byref(tau)),
+           "kfl_partition")
+    return n.tolist(), tau.value
+
+
+def kfl_plan_ring(k: int, devices, anchor: int, beta_block: float, beta_head: float, mu: float = 0.05):
+    """(block counts in ring order, kfl_plan fields as a dict, return code); devices: dicts with the
+    kfl_plan_device fields.  Does not raise on KFL_ERR_INFEASIBLE (the plan names the device)."""
+    import numpy as np
+    m = len(devices)
+    arr = (kfl_plan_device * m)(*[kfl_plan_device(d.get("o", 0.0), d.get("bw", 0.0), d.get("throughput", 0.0),
+                                                  d.get("working_set", 0.0), d["lim_body"], d["lim_head"])
+                                  for d in devices])
+    n = np.zeros(m, dtype=np.int32)
+    plan = kfl_plan()
+    rc = lib().kfl_plan_ring(k, m, arr, anchor, beta_block, beta_head, mu, n.ctypes.data, C.byref(plan))
+    if rc < 0 and rc != KFL_ERR_INFEASIBLE:
+        raise KflError(rc, "kfl_plan_ring")
+    return n.tolist(), {f: getattr(plan, f) for f, _ in kfl_plan._fields_}, rc
+
+
+def kfl_divide(k: int, m: int, weight=None):
+    import numpy as np
+    n = np.zeros(m, dtype=np.int32)
+    w = None if weight is None else np.ascontiguousarray(weight, dtype=np.float64)
+    _check(lib().kfl_divide(k, m, None if w is None else w.ctypes.data, n.ctypes.data), "kfl_divide")
+    return n.tolist()
+
+
+def kfl_block_limit(cfg: kfl_model_cfg, room_bytes: int, is_head: bool) -> int:
+    out = C.c_int(0)
+    _check(lib().kfl_block_limit(C.byref(cfg), room_bytes, 1 if is_head else 0, C.byref(out)), "kfl_block_limit")
+    return out.value
