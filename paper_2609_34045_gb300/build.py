@@ -19,8 +19,10 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libkafila_stage.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
+# host code: no floating-point contraction, so that it rounds the same on x86 and Arm hosts (an
+# aarch64 compiler would otherwise fuse a * b + c)
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
-              "-Xptxas", "-O3"]
+              "-Xcompiler", "-ffp-contract=off", "-Xptxas", "-O3"]
 
 
 def nvcc() -> str:
