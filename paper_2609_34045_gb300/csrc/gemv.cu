@@ -23,7 +23,7 @@
 namespace kfl {
 
 constexpr int GEMV_MAX_STAGES = 13;  // 13 x 16.9 KiB (batch 1) still fits one CTA's shared memory
-constexpr int GEMV_STATIC_SMEM = 2048;  // allowance for the kernel's own __shared__ variables
+constexpr int GEMV_STATIC_SMEM = 3072;  // allowance for the kernel's own __shared__ variables
 
 // ---------------------------------------------------------------------------- the kernel
 // FMT 0: bf16 tiles [RB][KT].  FMT 1: int4 tiles, codes [RB][KT4/8] uint32 + scales [RB][KT4/64].
@@ -42,6 +42,8 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
   __shared__ float s_inv[MAXB];
   __shared__ volatile int s_abort;
   __shared__ volatile int s_issued;
+  __shared__ __align__(16) float s_rx[RB * MAXB];  // cluster2: the partner CTA's partial
+  __shared__ __align__(8) uint64_t s_rx_bar;
 
   constexpr int KTILE = FMT == 0 ? KT : KT4;
   constexpr uint32_t WBYTES = FMT == 0 ? TILE_BYTES : TILE4_BYTES;
@@ -61,12 +63,14 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
       mbar_init(smem_addr(&seg_full[s]), CONSUMER_WARPS);
       mbar_init(smem_addr(&seg_empty[s]), 1);
     }
+    if (p.cluster2) mbar_init(smem_addr(&s_rx_bar), 1);
     s_abort = 0;
     s_issued = 0;
     fence_mbar_init();
   }
   for (int e = tid; e < NSLOT * RB * MAXB; e += GEMV_THREADS) red[e] = 0.f;  // int4 tiles add into it
   __syncthreads();
+  if (p.cluster2) cluster_sync_all();  // the partner writes s_rx / arrives on s_rx_bar only after this
   pdl_launch_dependents();
   auto stamp = [&](int slot) {
     if (p.trace) p.trace[(size_t)c * TRACE_SLOTS + slot] = global_ns();
@@ -138,7 +142,8 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
     norm_scale_warp<B>(p, s_inv, lane);
     bool inv_ready = true;
     int segc = 0;
-    gemv_epilogues<B, EPI>(p, t0, n, T, G, c, sr, segc, s_inv, inv_ready, &s_abort, lane);
+    gemv_epilogues<B, EPI>(p, t0, n, T, G, c, sr, segc, s_inv, inv_ready, &s_abort, lane,
+                           p.cluster2 ? s_rx : nullptr, &s_rx_bar);
     if (lane == 0) stamp(TR_CONS_DONE);
     return;
   }
@@ -187,11 +192,22 @@ static cudaError_t launch_one(const GemvParams &p, int grid, cudaStream_t s, boo
   cfg.blockDim = dim3(GEMV_THREADS);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  int na = 0;
+  if (pdl) {
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
+  if (p.cluster2) {
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = 2;
+    attr[na].val.clusterDim.y = 1;
+    attr[na].val.clusterDim.z = 1;
+    ++na;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cfg.numAttrs = na;
   return cudaLaunchKernelEx(&cfg, gemv_kernel<B, EPI, FMT>, p);
 }
 
@@ -267,6 +283,8 @@ cudaError_t prepare_gemv() {
 
 cudaError_t launch_gemv(const GemvParams &p, int epi, int grid, cudaStream_t s, bool pdl) {
   if (p.stages < 2 || p.stages > gemv_max_stages(p.batch, p.fmt, g_smem_optin)) return cudaErrorInvalidValue;
+  // clusters of two: each CTA exactly half the K range of one row block
+  if (p.cluster2 && (grid != 2 * p.n_rb || p.n_kt < 2)) return cudaErrorInvalidValue;
   return p.fmt == 0 ? launch_f<0>(p, epi, grid, s, pdl) : launch_f<1>(p, epi, grid, s, pdl);
 }
 

@@ -491,7 +491,8 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
 template <int B, int EPI>
 __device__ __forceinline__ void gemv_epilogues(const GemvParams &p, long long t0, int n, long long T, int G, int c,
                                                const SegRing &sr, int &segc, float *inv, bool &inv_ready,
-                                               volatile int *abort_flag, int lane) {
+                                               volatile int *abort_flag, int lane, float *rx = nullptr,
+                                               uint64_t *rx_bar = nullptr) {
   int i = 0;
   while (i < n) {
     const long long t = t0 + i;
@@ -511,7 +512,41 @@ __device__ __forceinline__ void gemv_epilogues(const GemvParams &p, long long t0
     EpiPre pre;
     epilogue_prefetch<B, EPI>(p, rb, lane, pre);
     bool do_epi = true;
-    if (!(kt0 == 0 && len == p.n_kt)) {
+    if (!(kt0 == 0 && len == p.n_kt) && rx) {
+      // a cluster of two splits this row block's K range: rank 1 (the upper half) writes its
+      // partial into rank 0's shared memory and arrives on its barrier; rank 0 adds it to its own
+      // (the lower half first, as the ticket path sums in CTA order)
+      if (cluster_ctarank() == 1) {
+        const uint32_t dst = map_to_rank(smem_addr(rx), 0);
+        const float4 *r4 = reinterpret_cast<const float4 *>(red);
+        for (int e = lane; e < RB * MAXB / 4; e += 32) st_cluster_f4(dst + e * 16, r4[e]);
+        __syncwarp();
+        if (lane == 0) mbar_arrive_remote(map_to_rank(smem_addr(rx_bar), 0));
+        do_epi = false;
+      } else {
+        int ok = 1;
+        if (lane == 0) {
+          ok = mbar_wait_cluster(smem_addr(rx_bar), 0) ? 1 : 0;
+          if (!ok) {
+            *abort_flag = 1;
+            atomicOr(p.err, ERR_TIMEOUT);
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        __syncwarp();
+        if (ok) {
+          float4 *r4 = reinterpret_cast<float4 *>(red);
+          const float4 *x4 = reinterpret_cast<const float4 *>(rx);
+          for (int e = lane; e < RB * MAXB / 4; e += 32) {
+            const float4 a = r4[e], b = x4[e];
+            r4[e] = make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
+          }
+          __syncwarp();
+        }
+        do_epi = ok != 0;
+      }
+      if (tr) tr[TR_E_KIND] = do_epi ? 2 : 1;
+    } else if (!(kt0 == 0 && len == p.n_kt)) {
       // this row block is shared with neighbouring CTAs: the ticket counts the CTAs that have
       // published their partial; the one that finds all the others there sums every partial
       const int c_lo = cta_of_tile((long long)rb * p.n_kt, T, G);

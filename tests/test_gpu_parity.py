@@ -254,6 +254,40 @@ def test_config2_width_bench_launch_shape():
     p.close()
 
 
+def test_cluster_combine_agrees_with_the_ticket_combine(monkeypatch):
+    """At the 7B widths the Q/K/V and O GEMVs run as clusters of two CTAs (each half of a row
+    block's K range) that combine through distributed shared memory; with clusters off they run
+    stream-K over one CTA per SM and combine through global memory and a ticket.  The K ranges
+    are split at other points, so the sums differ only by rounding: within 1e-5 of the RMS."""
+    from paper_2609_34045_gb300 import device_inputs as dev_in
+    w = dataclasses.replace(wl.CONFIGS[2], l1=2)
+    m = w.model
+    cfg = K.model_cfg(m, w.max_ctx, 1)
+    stream = torch.cuda.current_stream().cuda_stream
+    outs = []
+    for cluster in ("1", "0"):
+        monkeypatch.setenv("KFL_GEMV_CLUSTER2", cluster)
+        st = K.kfl_stage_create(cfg, 0, 2, 0)
+        dev_in.load_stage_seeded(st, w)
+        cap = torch.zeros(2, 1, m.d_model, device="cuda")
+        K.kfl_stage_debug_capture(st, cap)
+        out = torch.empty(1, m.d_model, device="cuda")
+        res = []
+        for s_ in range(2):
+            hid = torch.tensor(wl.hidden_in(m, s_, 1, w.seed), device="cuda")
+            pos = torch.tensor(wl.positions(w, s_), device="cuda")
+            K.kfl_stage_decode(st, None, hid, pos, 1, out, None, stream)
+            torch.cuda.synchronize()
+            res.append((out.cpu().clone(), cap.cpu().clone()))
+        assert K.kfl_stage_status(st) == 0
+        K.kfl_stage_destroy(st)
+        outs.append(res)
+    for (o1, c1), (o0, c0) in zip(*outs):
+        for a, b in ((o1, o0), (c1, c0)):
+            rms = torch.sqrt(torch.mean(b.double() ** 2)).item()
+            assert torch.max(torch.abs(a.double() - b.double())).item() <= 1e-5 * rms
+
+
 def test_config3_width_head_with_full_vocab():
     """The 32B-shaped head: embedding and lm_head over the full 152064-token vocabulary."""
     w = wl.CONFIGS[3]
