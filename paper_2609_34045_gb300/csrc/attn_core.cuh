@@ -158,7 +158,7 @@ __device__ __forceinline__ void attn_publish(const AttnParams &p, int kvh, int t
 // d += a b for one m16n8k16 bf16 tile (a: 16x16 row-major, b: 16x8 column-major, fp32
 // accumulate).  Rows 8..15 of a are the zero padding of the at most 8 heads, so a1 = a3 = 0.
 __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
-  asm volatile(
+  asm(
       "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
       "{%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])

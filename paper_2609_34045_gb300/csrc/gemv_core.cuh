@@ -141,7 +141,7 @@ __device__ __forceinline__ void tile_compute(const uint8_t *st, int warp, int la
 // d += a b for one m16n8k16 fp16 tile (a: 16x16 row-major, b: 16x8 column-major, fp32 accumulate)
 __device__ __forceinline__ void mma_f16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
                                                uint32_t b0, uint32_t b1) {
-  asm volatile(
+  asm(
       "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
       "{%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
