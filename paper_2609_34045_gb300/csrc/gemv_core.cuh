@@ -239,15 +239,51 @@ __device__ __forceinline__ void gemv_consume(int n_kt, uint8_t *ring, uint64_t *
         acc4[0] = acc4[1] = acc4[2] = acc4[3] = 0.f;
       }
     }
-    consumer_wait(smem_addr(&full[s]), phase, abort_flag, err);
-    if constexpr (FMT == 0)
-      tile_compute<B, FMT>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc);
-    else if (xsplit)
-      tile_compute_int4<B, true>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc4);
-    else
-      tile_compute_int4<B, false>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc4);
-    __syncwarp();
-    if (lane == 0) mbar_arrive(smem_addr(&empty[s]));
+    bool single = true;
+    if constexpr (FMT == 1) {
+      if (i + 1 < n && kt + 1 < n_kt) {
+        // two tiles of one row block: both stages awaited, then both computed without a barrier
+        // between them (their decoding and MMAs interleave), then both released
+        single = false;
+        int s1 = s + 1;
+        uint32_t ph1 = phase;
+        if (s1 == S) {
+          s1 = 0;
+          ph1 ^= 1u;
+        }
+        consumer_wait(smem_addr(&full[s]), phase, abort_flag, err);
+        consumer_wait(smem_addr(&full[s1]), ph1, abort_flag, err);
+        const uint8_t *st0 = ring + (size_t)s * stage_bytes(B, FMT), *st1 = ring + (size_t)s1 * stage_bytes(B, FMT);
+        if (xsplit) {
+          tile_compute_int4<B, true>(st0, warp, lane, acc4);
+          tile_compute_int4<B, true>(st1, warp, lane, acc4);
+        } else {
+          tile_compute_int4<B, false>(st0, warp, lane, acc4);
+          tile_compute_int4<B, false>(st1, warp, lane, acc4);
+        }
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(smem_addr(&empty[s]));
+          mbar_arrive(smem_addr(&empty[s1]));
+        }
+        // continue at the second tile: the segment check and the advance below are its
+        ++i;
+        ++kt;
+        s = s1;
+        phase = ph1;
+      }
+    }
+    if (single) {
+      consumer_wait(smem_addr(&full[s]), phase, abort_flag, err);
+      if constexpr (FMT == 0)
+        tile_compute<B, FMT>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc);
+      else if (xsplit)
+        tile_compute_int4<B, true>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc4);
+      else
+        tile_compute_int4<B, false>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc4);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_addr(&empty[s]));
+    }
     if (kt == n_kt - 1 || i == n - 1) {
       const int slot = segc % NSLOT, use = segc / NSLOT;
       float *rd = sr.red + slot * RB * MAXB;
