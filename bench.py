@@ -42,6 +42,9 @@ def parse():
     ap.add_argument("--profile-steps", type=int, default=20)
     ap.add_argument("--e2e-steps", type=int, default=500)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--ring", action="store_true",
+                    help="ring emulation: the 7B-shaped model as 4 stages of 7 blocks and the head's return "
+                         "leg, 4 users served pipelined (one stream per stage) vs one at a time vs batched")
     ap.add_argument("--layers", type=int, default=0,
                     help="small case for profiling: the first N blocks of the stage as a body stage "
                          "(no embedding, no head, no splits)")
@@ -576,8 +579,82 @@ def run_ours(args, work):
     return 0
 
 
+def run_ring(args):
+    """Tokens per second of 4 users around a ring of stages on this GPU (section VI, "Serving
+    several users at once"): pipelined (each stage on its own stream, working on one user's token
+    while the stage after it works on another's), the same schedule on one stream, one user alone,
+    and, for reference, all four users batched through one whole-model stage."""
+    import dataclasses
+
+    import torch
+
+    from paper_2609_34045_gb300 import device_inputs as di
+    from paper_2609_34045_gb300 import stage as K
+    from paper_2609_34045_gb300 import workload as wl
+    from paper_2609_34045_gb300.ring import Ring
+
+    users, tokens = 4, 16
+    base = wl.CONFIGS[2]
+    m = base.model
+    work = dataclasses.replace(base, name="7B-ring-4x7-u4-ctx2048", l0=0, l1=m.n_layers_total, embed_in=True,
+                               logits_out=True, batch=users, contexts=(2048, 2048, 2048, 2048), steps=6 * tokens,
+                               splits=())
+    torch.cuda.set_device(0)
+    ring = Ring(work, [7, 7, 7, 7], users)
+    first = wl.first_token_ids(m, users, work.seed)
+
+    def timed(fn):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        out = fn()
+        torch.cuda.synchronize()
+        return time.perf_counter() - t0, out
+
+    ring.run(first, 2)  # warm-up: every stage captures its graph
+    res = {}
+    t, ids_pipe = timed(lambda: ring.run(first, tokens, start=2))
+    res["pipelined_4_users"] = users * tokens / t
+    t, ids_seq = timed(lambda: ring.run(first, tokens, start=2 + tokens, sequential=True))
+    res["sequential_4_users"] = users * tokens / t
+    # one user alone: the same ring, users 1..3 idle
+    ring1_first = [first[0]]
+    ring.users, saved = 1, ring.users
+    t, _ = timed(lambda: ring.run(ring1_first, tokens, start=2 + 2 * tokens))
+    res["one_user"] = tokens / t
+    ring.users = saved
+    ring.close()
+    # all four users batched through one whole-model (head) stage
+    cfg = K.model_cfg(m, work.max_ctx, users)
+    st = K.kfl_stage_create(cfg, 0, m.n_layers_total, K.KFL_IS_HEAD)
+    di.load_stage_seeded(st, work)
+    ids = torch.tensor(first, dtype=torch.int32, device="cuda")
+    nxt = torch.zeros(users, dtype=torch.int32, device="cuda")
+    stream = torch.cuda.current_stream().cuda_stream
+
+    def batched(n, start):
+        tok = ids.clone()
+        for j in range(n):
+            pos = torch.tensor([c + start + j for c in work.contexts], dtype=torch.int32, device="cuda")
+            K.kfl_stage_decode(st, tok, None, pos, users, None, nxt, stream)
+            tok.copy_(nxt)
+    batched(2, 2 + 3 * tokens)
+    t, _ = timed(lambda: batched(tokens, 4 + 3 * tokens))
+    res["batched_4_users"] = users * tokens / t
+    K.kfl_stage_destroy(st)
+    line = {"metric": "ring tokens/s", "unit": "tokens/s", "higher_is_better": True, "n_gpus": 1,
+            "config": {"workload": work.name, "stages": [7, 7, 7, 7, "return leg"], "users": users,
+                       "tokens_per_user": tokens, "ctx": 2048, "weights": "bf16"},
+            "tokens_per_s": res,
+            "pipelined_over_sequential": res["pipelined_4_users"] / res["sequential_4_users"],
+            "data": "synthetic (seeded)", "timing": "host wall clock around synchronized runs"}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     args = parse()
+    if args.ring:
+        return run_ring(args)
     import dataclasses
 
     from paper_2609_34045_gb300 import workload as wl

@@ -130,6 +130,18 @@ int kfl_stage_decode(kfl_stage *st, const int32_t *token_ids, const float *hidde
                      const int32_t *positions, int batch, float *hidden_out, int32_t *next_ids,
                      void *cuda_stream);
 
+/* kfl_stage_decode for chosen users: batch row b serves user users[b] (device int32[batch],
+ * distinct values in [0, max_batch)), whose KV cache slot it reads and appends to; positions,
+ * token_ids, hidden_in/out and next_ids stay indexed by batch row.  This is how one stage of a
+ * ring serves one user's token at a time while other users' tokens are elsewhere in the ring
+ * (Section VI, "Serving several users at once").  A user outside [0, max_batch) is found on the
+ * device and treated like a bad position (nothing of that row is written, kfl_stage_status then
+ * reports KFL_ERR_RANGE).  Errors returned here: those of kfl_stage_decode, and KFL_ERR_ARG for
+ * users == NULL. */
+int kfl_stage_decode_users(kfl_stage *st, const int32_t *token_ids, const float *hidden_in,
+                           const int32_t *positions, const int32_t *users, int batch, float *hidden_out,
+                           int32_t *next_ids, void *cuda_stream);
+
 /* kfl_stage_decode with HOST buffers of the same shapes: copies the inputs to the device,
  * runs the step and copies the outputs back, then waits for cuda_stream.  Pinned host memory
  * makes the copies asynchronous to the host; pageable memory works too. */

@@ -120,7 +120,7 @@ template <int HD, int NBUF>
 __device__ __forceinline__ void attn_load_rows(const AttnParams &p, int b, int kvh, int p0, int cnt, int buf,
                                                int only, int skip, uint8_t *sm, int tid) {
   using L = AttnLayout<HD, NBUF>;
-  const size_t head_base = ((size_t)b * p.n_kv_heads + kvh) * p.max_ctx;
+  const size_t head_base = ((size_t)p.slots[b] * p.n_kv_heads + kvh) * p.max_ctx;
   const uint16_t *kg = p.kcache + head_base * HD;
   const uint16_t *vg = p.vcache + head_base * HD;
   uint8_t *sk = sm + L::K_OFF + buf * ATT_SUB * L::KROW;

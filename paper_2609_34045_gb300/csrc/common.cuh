@@ -117,6 +117,7 @@ struct GemvParams {
   float *q;
   uint16_t *kcache, *vcache;  // this layer's [max_batch][Hkv][max_ctx][hd]
   const int *positions;       // [batch]; never written while a step runs
+  const int *slots;           // [batch]: the KV-cache user slot of each batch row
   const float *rope_cos, *rope_sin;  // [max_ctx][hd/2], or [batch][hd/2] when rope_per_user
   int rope_per_user;
   int n_q_rows, n_kv_rows, head_dim, max_ctx, n_kv_heads;
@@ -160,6 +161,7 @@ struct AttnParams {
   const uint16_t *kcache;    // this layer's [max_batch][Hkv][max_ctx][hd]
   const uint16_t *vcache;
   const int *positions;
+  const int *slots;          // [batch]: the KV-cache user slot of each batch row
   float *o;                  // [batch][ldo]
   int ldo;
   Act16 o16;                 // int4 stages: o also in the O projection's input form (hi NULL else)
@@ -527,7 +529,7 @@ cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int
                                int batch, const uint16_t *embed, int vocab, int d, int ldh,
                                const float *g_next, float *h, float *xn, float *sumsq,
                                int *positions, int max_ctx, unsigned *err, unsigned *bar, Act16 xn16,
-                               cudaStream_t s);
+                               const int *users, int max_batch, int *slots, cudaStream_t s);
 size_t stage_kernel_smem(int stages, int head_dim, int batch, int fmt);
 int stage_kernel_attn_bytes(int head_dim);
 cudaError_t prepare_stage_kernel(size_t smem);

@@ -469,14 +469,14 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
           qd[i] = a;
           qd[i + half] = c2;
         } else if (ok) {
-          uint16_t *kd = p.kcache + (((size_t)b * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
+          uint16_t *kd = p.kcache + (((size_t)p.slots[b] * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
           kd[i] = f32_to_bf16_rne(a);
           kd[i + half] = f32_to_bf16_rne(c2);
         }
       } else if (ok) {
         const int rr = r0 - p.n_q_rows - p.n_kv_rows;
         const int head = rr / hd, j = rr % hd;
-        uint16_t *vd = p.vcache + (((size_t)b * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
+        uint16_t *vd = p.vcache + (((size_t)p.slots[b] * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
         vd[j] = f32_to_bf16_rne(v1);
         vd[j + 1] = f32_to_bf16_rne(v2);
       }

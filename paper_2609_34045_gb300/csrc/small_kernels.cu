@@ -11,14 +11,24 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
                                                          const int *positions_in, const uint16_t *embed,
                                                          int vocab, int d, int ldh, const float *g_next,
                                                          float *h, float *xn, float *sumsq, int *positions,
-                                                         int max_ctx, unsigned *err, unsigned *bar, Act16 xn16) {
+                                                         int max_ctx, unsigned *err, unsigned *bar, Act16 xn16,
+                                                         const int *users, int max_batch, int *slots) {
   __shared__ float vals[64];
   const int b = blockIdx.y, tid = threadIdx.x, r = blockIdx.x * 64 + tid;
   pdl_launch_dependents();
   pdl_wait();
   if (blockIdx.x == 0 && tid == 0) {
-    const int pos = positions_in[b];
+    int pos = positions_in[b];
     if (pos < 0 || pos >= max_ctx) atomicOr(err, ERR_POSITION);
+    // the user's KV slot (users NULL: batch row b is user b); a slot outside [0, max_batch) is
+    // flagged like a bad position, and the row's position is made invalid so that nothing of it
+    // is written
+    const int u = users ? users[b] : b;
+    if (u < 0 || u >= max_batch) {
+      atomicOr(err, ERR_POSITION);
+      pos = -1;
+    }
+    slots[b] = (u < 0 || u >= max_batch) ? 0 : u;
     positions[b] = pos;
     // abort flag of the persistent stage kernel that follows
     if (b == 0 && bar) {
@@ -66,10 +76,11 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in, int batch,
                                const uint16_t *embed, int vocab, int d, int ldh, const float *g_next, float *h,
                                float *xn, float *sumsq, int *positions, int max_ctx, unsigned *err,
-                               unsigned *bar, Act16 xn16, cudaStream_t s) {
+                               unsigned *bar, Act16 xn16, const int *users, int max_batch, int *slots,
+                               cudaStream_t s) {
   dim3 grid((d + 63) / 64, batch);
   stage_input_kernel<<<grid, 64, 0, s>>>(ids, hidden_in, positions_in, embed, vocab, d, ldh, g_next, h, xn, sumsq,
-                                         positions, max_ctx, err, bar, xn16);
+                                         positions, max_ctx, err, bar, xn16, users, max_batch, slots);
   return cudaGetLastError();
 }
 

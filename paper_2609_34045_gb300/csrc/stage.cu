@@ -167,7 +167,7 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   ws += (size_t)MAXB * (2 * p->ldh + 2 * p->ldq + p->lda) * 4;         // h, xn, q, o, a
   ws += act16_bytes(p->ldh, true) + act16_bytes(p->ldq, false) + act16_bytes(p->lda, false);  // int4 inputs
   ws += (size_t)p->n_parts * MAXB * 4;                                 // sum of squares
-  ws += 2 * MAXB * 4;                                                  // positions, next ids
+  ws += 3 * MAXB * 4;                                                  // positions, KV slots, next ids
   ws += (size_t)4 * p->gemv_grid_max * 2 * RB * MAXB * 4;              // stream-K partials (x4)
   ws += (size_t)(4 * p->n_rb_max + 1) * 4;                             // tickets (x4) + argmax ticket
   ws += (size_t)std::max(1, p->n_phases) * p->ctr_stride * 4;          // readiness counters
@@ -198,6 +198,7 @@ struct kfl_stage {
   // int4 stages: the GEMV inputs in the tensor cores' fp16 form (xn with its rests, for Q/K/V)
   Act16 xn16 = {}, a16 = {}, o16 = {};
   int *pos = nullptr, *next_int = nullptr;
+  int *slots = nullptr;  // [MAXB] KV-cache user slot of each batch row (this step)
   int *io_pos = nullptr, *io_ids = nullptr;  // host-buffer decode staging
   float *io_hin = nullptr;
   float *gemv_partial = nullptr;
@@ -337,6 +338,7 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
       g.kcache = kcl;
       g.vcache = vcl;
       g.positions = st->pos;
+      g.slots = st->slots;
       g.rope_cos = st->rope_cos;
       g.rope_sin = st->rope_sin;
       g.n_q_rows = P.qdim;
@@ -355,6 +357,7 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
       a.kcache = kcl;
       a.vcache = vcl;
       a.positions = st->pos;
+      a.slots = st->slots;
       a.o = st->o;
       a.ldo = P.ldq;
       if (i4) a.o16 = st->o16;
@@ -615,8 +618,8 @@ const float *input_g_next(const kfl_stage *st) {
   return nullptr;
 }
 
-int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const int32_t *positions, int batch,
-             float *hidden_out, int32_t *next_ids, cudaStream_t s) {
+int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const int32_t *positions,
+             const int32_t *users, int batch, float *hidden_out, int32_t *next_ids, cudaStream_t s) {
   const Plan &P = st->P;
   const bool embed = (st->flags & KFL_EMBED_IN) != 0;
   const bool body = P.nl > 0 || (st->flags & KFL_LOGITS_OUT);
@@ -631,7 +634,8 @@ int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const in
     CK(cudaEventRecord(st->ev[0], s));
     CK(launch_stage_input(ids, hidden_in, positions, batch, embed ? st->embed : nullptr, P.V, P.d, P.ldh,
                           input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, st->bar,
-                          st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn16 : Act16{}, s));
+                          st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn16 : Act16{}, users, st->cfg.max_batch,
+                          st->slots, s));
     CK(cudaEventRecord(st->ev[1], s));
     kinds.push_back(KFL_KERNEL_INPUT);
     int rc = enqueue_body(st, batch, s, false, &kinds, 1);
@@ -652,7 +656,8 @@ int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const in
   }
   CK(launch_stage_input(ids, hidden_in, positions, batch, embed ? st->embed : nullptr, P.V, P.d, P.ldh,
                         input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, st->bar,
-                        st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn16 : Act16{}, s));
+                        st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn16 : Act16{}, users, st->cfg.max_batch,
+                        st->slots, s));
   if (body) {
     int rc = ensure_graph(st, batch);
     if (rc != KFL_OK) return rc;
@@ -850,6 +855,7 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
     }
   }
   AL(st->pos, MAXB * 4);
+  AL(st->slots, MAXB * 4);
   AL(st->next_int, MAXB * 4);
   AL(st->gemv_partial, (size_t)4 * P.gemv_grid_max * 2 * RB * MAXB * 4);
   AL(st->tickets, (size_t)(4 * P.n_rb_max + 1) * 4);
@@ -873,7 +879,8 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
   if (cudaMemset(st->h, 0, (size_t)MAXB * P.ldh * 4) || cudaMemset(st->xn, 0, (size_t)MAXB * P.ldh * 4) ||
       cudaMemset(st->q, 0, (size_t)MAXB * P.ldq * 4) || cudaMemset(st->o, 0, (size_t)MAXB * P.ldq * 4) ||
       cudaMemset(st->a, 0, (size_t)MAXB * P.lda * 4) || cudaMemset(st->sumsq, 0, (size_t)P.n_parts * MAXB * 4) ||
-      cudaMemset(st->pos, 0, MAXB * 4) || cudaMemset(st->next_int, 0, MAXB * 4) ||
+      cudaMemset(st->pos, 0, MAXB * 4) || cudaMemset(st->slots, 0, MAXB * 4) ||
+      cudaMemset(st->next_int, 0, MAXB * 4) ||
       cudaMemset(st->tickets, 0, (size_t)(4 * P.n_rb_max + 1) * 4) ||
       cudaMemset(st->counters, 0, (size_t)std::max(1, P.n_phases) * P.ctr_stride * 4) ||
       cudaMemset(st->attn_tickets, 0, (size_t)MAXB * P.hkv * 4) || cudaMemset(st->err, 0, 16) ||
@@ -1025,7 +1032,18 @@ extern "C" int kfl_stage_decode(kfl_stage *st, const int32_t *token_ids, const f
   int rc = check_decode_args(st, token_ids, hidden_in, positions, batch, hidden_out, next_ids);
   if (rc) return rc;
   CK(cudaSetDevice(st->dev));
-  return run_step(st, token_ids, hidden_in, positions, batch, hidden_out, next_ids,
+  return run_step(st, token_ids, hidden_in, positions, nullptr, batch, hidden_out, next_ids,
+                  static_cast<cudaStream_t>(cuda_stream));
+}
+
+extern "C" int kfl_stage_decode_users(kfl_stage *st, const int32_t *token_ids, const float *hidden_in,
+                                      const int32_t *positions, const int32_t *users, int batch,
+                                      float *hidden_out, int32_t *next_ids, void *cuda_stream) {
+  int rc = check_decode_args(st, token_ids, hidden_in, positions, batch, hidden_out, next_ids);
+  if (rc) return rc;
+  if (!users) return KFL_ERR_ARG;
+  CK(cudaSetDevice(st->dev));
+  return run_step(st, token_ids, hidden_in, positions, users, batch, hidden_out, next_ids,
                   static_cast<cudaStream_t>(cuda_stream));
 }
 
@@ -1041,7 +1059,8 @@ extern "C" int kfl_stage_decode_host(kfl_stage *st, const int32_t *token_ids, co
   CK(cudaMemcpyAsync(st->io_pos, positions, (size_t)batch * 4, cudaMemcpyHostToDevice, s));
   if (embed) CK(cudaMemcpyAsync(st->io_ids, token_ids, (size_t)batch * 4, cudaMemcpyHostToDevice, s));
   else CK(cudaMemcpyAsync(st->io_hin, hidden_in, (size_t)batch * P.d * 4, cudaMemcpyHostToDevice, s));
-  rc = run_step(st, embed ? st->io_ids : nullptr, embed ? nullptr : st->io_hin, st->io_pos, batch, nullptr, nullptr, s);
+  rc = run_step(st, embed ? st->io_ids : nullptr, embed ? nullptr : st->io_hin, st->io_pos, nullptr, batch, nullptr,
+                nullptr, s);
   if (rc) return rc;
   if (hidden_out)
     CK(cudaMemcpy2DAsync(hidden_out, (size_t)P.d * 4, st->h, (size_t)P.ldh * 4, (size_t)P.d * 4, batch,

@@ -83,6 +83,7 @@ def lib() -> C.CDLL:
             "kfl_stage_load_head": ([vp, vp, vp, C.POINTER(kfl_matrix), i], i),
             "kfl_stage_decode": ([vp, vp, vp, vp, i, vp, vp, vp], i),
             "kfl_stage_decode_host": ([vp, vp, vp, vp, i, vp, vp, vp], i),
+            "kfl_stage_decode_users": ([vp, vp, vp, vp, vp, i, vp, vp, vp], i),
             "kfl_kv_reset": ([vp, i], i),
             "kfl_kv_fill_seeded": ([vp, i, i, C.c_uint64], i),
             "kfl_kv_write": ([vp, i, i, vp, vp, i, i], i),
@@ -224,6 +225,14 @@ def kfl_stage_decode(st: Stage, token_ids, hidden_in, positions, batch: int, hid
     positions [batch], fp32 hidden_out [batch][d], int32 next_ids [batch].  Asynchronous."""
     _check(lib().kfl_stage_decode(st.handle, _ptr(token_ids), _ptr(hidden_in), _ptr(positions), batch,
                                   _ptr(hidden_out), _ptr(next_ids), cuda_stream), "kfl_stage_decode")
+
+
+def kfl_stage_decode_users(st: Stage, token_ids, hidden_in, positions, users, batch: int, hidden_out, next_ids,
+                           cuda_stream: int | None = None) -> None:
+    """kfl_stage_decode with batch row b serving user users[b] (int32 CUDA tensor [batch])."""
+    _check(lib().kfl_stage_decode_users(st.handle, _ptr(token_ids), _ptr(hidden_in), _ptr(positions), _ptr(users),
+                                        batch, _ptr(hidden_out), _ptr(next_ids), cuda_stream),
+           "kfl_stage_decode_users")
 
 
 def kfl_stage_decode_host(st: Stage, token_ids, hidden_in, positions, batch: int, hidden_out, next_ids,

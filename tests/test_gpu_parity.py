@@ -351,3 +351,77 @@ def test_int4_deep_stack_finite_and_split_bit_exact(batch):
     for st in (full, a, c):
         assert K.kfl_stage_status(st) == 0
         K.kfl_stage_destroy(st)
+
+
+# ---------------------------------------------------------------------------- ring emulation
+
+RING = wl.ModelShape(n_layers_total=5, d_model=320, n_heads=6, n_kv_heads=2, head_dim=64, ffn=712, vocab=1000)
+
+
+def test_decode_users_addresses_the_users_kv_slots():
+    """kfl_stage_decode_users: batch row b reads and appends user users[b]'s KV slot.  Users 2 and
+    0 served as rows 0 and 1 give the same outputs as rows 0 and 1 of a batch in slot order, and
+    only slots 2 and 0 change."""
+    from paper_2609_34045_gb300 import device_inputs as dev_in
+    w = wl.Workload("ring-users", RING, 0, 2, False, False, 3, (17, 40, 65), 4, 31)
+    cfg = K.model_cfg(RING, w.max_ctx, 3)
+    stream = torch.cuda.current_stream().cuda_stream
+    outs = []
+    for users in ([2, 0], None):
+        st = K.kfl_stage_create(cfg, 0, 2, 0)
+        dev_in.load_stage_seeded(st, w)
+        before = [_kv(st, u, RING) for u in range(3)]
+        rows = users if users is not None else [0, 1]
+        pos = torch.tensor([w.contexts[u] for u in rows], dtype=torch.int32, device="cuda")
+        hid = torch.tensor(wl.hidden_in(RING, 0, 3, w.seed), device="cuda")[rows].contiguous()
+        out = torch.empty(2, RING.d_model, device="cuda")
+        K.kfl_stage_decode_users(st, None, hid, pos, torch.tensor(rows, dtype=torch.int32, device="cuda"),
+                                 2, out, None, stream)
+        torch.cuda.synchronize()
+        after = [_kv(st, u, RING) for u in range(3)]
+        changed = [not np.array_equal(before[u], after[u]) for u in range(3)]
+        outs.append((out.cpu().numpy(), changed))
+        assert K.kfl_stage_status(st) == 0
+        K.kfl_stage_destroy(st)
+    (o_perm, ch_perm), (o_id, ch_id) = outs
+    assert ch_perm == [True, False, True] and ch_id == [True, True, False]
+    # row 1 of the permuted call is user 0 at its own position: the same as row 0 of slot order
+    assert np.array_equal(o_perm[1], o_id[0])
+
+
+def _kv(st, u, model):
+    k = torch.empty(model.n_kv_heads, st.cfg.max_ctx, model.head_dim, dtype=torch.int16, device="cuda")
+    v = torch.empty_like(k)
+    K.kfl_kv_read(st, 0, u, k, v, True)
+    torch.cuda.synchronize()
+    return np.concatenate([k.cpu().numpy().ravel(), v.cpu().numpy().ravel()])
+
+
+@pytest.mark.parametrize("sequential", [False, True], ids=["pipelined", "sequential"])
+def test_ring_generates_what_one_stage_does(sequential):
+    """Three users around a ring of stages (2, 3 blocks) and the head's return leg, each stage on
+    its own stream: every user's greedy tokens equal those of the whole model as one head stage
+    serving that user (stage splits are exact)."""
+    from paper_2609_34045_gb300 import device_inputs as dev_in
+    from paper_2609_34045_gb300.ring import Ring
+    w = wl.Workload("ring", RING, 0, 5, True, True, 3, (12, 70, 33), 6, 41)
+    first = wl.first_token_ids(RING, 3, w.seed)
+    ring = Ring(w, [2, 3], 3)
+    got = ring.run(first, 5, sequential=sequential)
+    ring.close()
+    cfg = K.model_cfg(RING, ring.work.max_ctx, 3)
+    st = K.kfl_stage_create(cfg, 0, 5, K.KFL_IS_HEAD)
+    dev_in.load_stage_seeded(st, ring.work)
+    stream = torch.cuda.current_stream().cuda_stream
+    for u in range(3):
+        tok = torch.tensor([int(first[u])], dtype=torch.int32, device="cuda")
+        nxt = torch.zeros(1, dtype=torch.int32, device="cuda")
+        for t in range(5):
+            pos = torch.tensor([ring.work.contexts[u] + t], dtype=torch.int32, device="cuda")
+            K.kfl_stage_decode_users(st, tok, None, pos, torch.tensor([u], dtype=torch.int32, device="cuda"), 1,
+                                     None, nxt, stream)
+            torch.cuda.synchronize()
+            assert int(nxt.item()) == got[t][u]
+            tok.copy_(nxt)
+    assert K.kfl_stage_status(st) == 0
+    K.kfl_stage_destroy(st)
