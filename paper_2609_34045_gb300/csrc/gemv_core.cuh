@@ -365,6 +365,7 @@ struct EpiPre {
   float h[MAXB][2];
   float g[2];
   float cs[MAXB], sn[MAXB];  // QKV: the RoPE cos / sin of this lane's row pair, per user
+  int pos[MAXB], slot[MAXB]; // QKV: each user's position (-1 if invalid) and KV slot
 };
 
 template <int B, int EPI>
@@ -377,9 +378,11 @@ __device__ __forceinline__ void epilogue_prefetch(const GemvParams &p, int rb, i
     const int i = (rr % hd) >> 1;
 #pragma unroll
     for (int b = 0; b < B; ++b) {
-      int pos = p.positions[b];
-      if (pos < 0 || pos >= p.max_ctx) pos = 0;
-      const size_t ri = (size_t)(p.rope_per_user ? b : pos) * half + i;
+      const int pv = p.positions[b];
+      const bool ok = pv >= 0 && pv < p.max_ctx;
+      e.pos[b] = ok ? pv : -1;
+      e.slot[b] = p.slots[b];
+      const size_t ri = (size_t)(p.rope_per_user ? b : (ok ? pv : 0)) * half + i;
       e.cs[b] = rot ? p.rope_cos[ri] : 0.f;
       e.sn[b] = rot ? p.rope_sin[ri] : 0.f;
     }
@@ -406,6 +409,16 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
       if (n < p.n_rows) p.out[(size_t)b * p.ldo + n] = red[r * MAXB + b] * inv[b];
     }
   } else if constexpr (EPI == EPI_RESID) {
+    // every read before the first store (the compiler cannot tell the stores from these reads),
+    // so that the users' conversions and reductions overlap
+    float hv[B][2];
+#pragma unroll
+    for (int b = 0; b < B; ++b)
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+        const int r = lane + 32 * h2;
+        hv[b][h2] = rb * RB + r < p.n_rows ? pre.h[b][h2] + red[r * MAXB + b] * inv[b] : 0.f;
+      }
 #pragma unroll
     for (int b = 0; b < B; ++b) {
       float sq = 0.f;
@@ -414,7 +427,7 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
         const int r = lane + 32 * h2, n = rb * RB + r;
         const bool ok = n < p.n_rows;
         const size_t o = (size_t)b * p.ldh + n;
-        const float hn = ok ? pre.h[b][h2] + red[r * MAXB + b] * inv[b] : 0.f;
+        const float hn = hv[b][h2];
         const float xv = hn * pre.g[h2];
         // int4 stage: xn in the tensor-core input form, chunk rb * 2 + h2
         if (p.xout.hi && p.g_next) act16_put_warp(p.xout, b, rb * 2 + h2, xv, lane);
@@ -429,15 +442,21 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
       if (lane == 0) p.sumsq_out[rb * MAXB + b] = sq;
     }
   } else if constexpr (EPI == EPI_SWIGLU) {
-    // lane = output (RB / 2 = 32 of them per row block), one user per pass
+    // lane = output (RB / 2 = 32 of them per row block), one user per pass; every read first
+    float gv[B], uv[B];
+#pragma unroll
+    for (int b = 0; b < B; ++b) {
+      gv[b] = red[(2 * lane) * MAXB + b] * inv[b];
+      uv[b] = red[(2 * lane + 1) * MAXB + b] * inv[b];
+    }
 #pragma unroll
     for (int b = 0; b < B; ++b) {
       const int pr = lane, j = rb * (RB / 2) + pr;
       const bool ok = 2 * j < p.n_rows;
       float a = 0.f;
       if (ok) {
-        const float g = red[(2 * pr) * MAXB + b] * inv[b];
-        const float u = red[(2 * pr + 1) * MAXB + b] * inv[b];
+        const float g = gv[b];
+        const float u = uv[b];
         a = g / (1.0f + expf(-g)) * u;
       }
       if (p.xout.hi)
@@ -447,15 +466,22 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
     }
   } else if constexpr (EPI == EPI_QKV) {
     const int hd = p.head_dim, half = hd >> 1;
+    // every read before the first store (the compiler cannot tell the stores from these reads)
+    float rv1[B], rv2[B], iv[B];
+#pragma unroll
+    for (int b = 0; b < B; ++b) {
+      rv1[b] = red[(2 * lane) * MAXB + b];
+      rv2[b] = red[(2 * lane + 1) * MAXB + b];
+      iv[b] = inv[b];
+    }
 #pragma unroll
     for (int b = 0; b < B; ++b) {
       const int pr = lane, r0 = rb * RB + 2 * pr;
-      int pos = p.positions[b];
-      const bool ok = pos >= 0 && pos < p.max_ctx;
-      if (!ok) pos = 0;
+      const bool ok = pre.pos[b] >= 0;
+      const int pos = ok ? pre.pos[b] : 0;
       if (r0 >= p.n_rows) continue;
-      const float v1 = red[(2 * pr) * MAXB + b] * inv[b];
-      const float v2 = red[(2 * pr + 1) * MAXB + b] * inv[b];
+      const float v1 = rv1[b] * iv[b];
+      const float v2 = rv2[b] * iv[b];
       if (r0 < p.n_q_rows + p.n_kv_rows) {
         const bool is_q = r0 < p.n_q_rows;
         const int rr = is_q ? r0 : r0 - p.n_q_rows;
@@ -469,14 +495,14 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
           qd[i] = a;
           qd[i + half] = c2;
         } else if (ok) {
-          uint16_t *kd = p.kcache + (((size_t)p.slots[b] * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
+          uint16_t *kd = p.kcache + (((size_t)pre.slot[b] * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
           kd[i] = f32_to_bf16_rne(a);
           kd[i + half] = f32_to_bf16_rne(c2);
         }
       } else if (ok) {
         const int rr = r0 - p.n_q_rows - p.n_kv_rows;
         const int head = rr / hd, j = rr % hd;
-        uint16_t *vd = p.vcache + (((size_t)p.slots[b] * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
+        uint16_t *vd = p.vcache + (((size_t)pre.slot[b] * p.n_kv_heads + head) * p.max_ctx + pos) * hd;
         vd[j] = f32_to_bf16_rne(v1);
         vd[j + 1] = f32_to_bf16_rne(v2);
       }
