@@ -45,6 +45,9 @@ def parse():
     ap.add_argument("--ring", action="store_true",
                     help="ring emulation: the 7B-shaped model as 4 stages of 7 blocks and the head's return "
                          "leg, 4 users served pipelined (one stream per stage) vs one at a time vs batched")
+    ap.add_argument("--prefill", action="store_true",
+                    help="time to first token of one user on the 7B-shaped model as one head stage: the "
+                         "prompt's prefill (steps of 4 of its tokens) plus the first decode step")
     ap.add_argument("--layers", type=int, default=0,
                     help="small case for profiling: the first N blocks of the stage as a body stage "
                          "(no embedding, no head, no splits)")
@@ -580,7 +583,7 @@ def run_ours(args, work):
 
 
 def run_ring(args):
-    """Tokens per second of 4 users around a ring of stages on this GPU (section VI, "Serving
+    """Tokens per second of 4 users around a ring of stages on this GPU (section VII, "Serving
     several users at once"): pipelined (each stage on its own stream, working on one user's token
     while the stage after it works on another's), the same schedule on one stream, one user alone,
     and, for reference, all four users batched through one whole-model stage."""
@@ -651,10 +654,92 @@ def run_ring(args):
     return 0
 
 
+def run_prefill(args):
+    """Time to first token split into prefill and decode (section VI, instrumentation paragraph)
+    on the 7B-shaped model as one head stage, one user from an empty cache: the prompt goes
+    through kfl_stage_prefill (steps of max_batch = 4 of its tokens), then one decode step.  As in
+    the paper's protocol, five generations per prompt length, the first discarded as cold, the
+    median of the rest; CUDA events on the launching stream.  For comparison the same prompt one
+    token per step (kfl_stage_decode_users at batch 1)."""
+    import dataclasses
+    import statistics
+
+    import torch
+
+    from paper_2609_34045_gb300 import device_inputs as di
+    from paper_2609_34045_gb300 import stage as K
+    from paper_2609_34045_gb300 import workload as wl
+
+    lengths = (128, 512, 2048)
+    base = wl.CONFIGS[2]
+    m = base.model
+    work = dataclasses.replace(base, name="7B-head-28L-prefill", l0=0, l1=m.n_layers_total, embed_in=True,
+                               logits_out=True, batch=4, contexts=(0, 0, 0, 0), steps=max(lengths) + 64,
+                               splits=())
+    torch.cuda.set_device(0)
+    cfg = K.model_cfg(m, work.max_ctx, 4)
+    st = K.kfl_stage_create(cfg, 0, m.n_layers_total, K.KFL_IS_HEAD)
+    di.load_stage_seeded(st, work)
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+    user = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    rows = {}
+    for n in lengths:
+        ids = torch.tensor(wl.token_ids(work.seed, 90, n, m.vocab), device="cuda")
+        pos = torch.arange(n, dtype=torch.int32, device="cuda")
+        nxt = torch.zeros(n, dtype=torch.int32, device="cuda")
+        tok = torch.zeros(1, dtype=torch.int32, device="cuda")
+        first = torch.zeros(1, dtype=torch.int32, device="cuda")
+        pos_n = torch.tensor([n], dtype=torch.int32, device="cuda")
+        gens = []
+        for g in range(5):
+            torch.cuda.synchronize()
+            ev[0].record(stream)
+            K.kfl_stage_prefill(st, ids, None, pos, 0, n, None, nxt, sp)
+            ev[1].record(stream)
+            tok.copy_(nxt[n - 1:])
+            K.kfl_stage_decode_users(st, tok, None, pos_n, user, 1, None, first, sp)
+            ev[2].record(stream)
+            torch.cuda.synchronize()
+            gens.append((ev[0].elapsed_time(ev[1]), ev[1].elapsed_time(ev[2])))
+        pre = statistics.median(x[0] for x in gens[1:])
+        dec = statistics.median(x[1] for x in gens[1:])
+        rows[n] = {"prefill_ms": pre, "decode_ms": dec, "ttft_ms": pre + dec, "prefill_tokens_per_s": n / pre * 1e3}
+    # one token per step, the 512-token prompt
+    n = 512
+    ids = torch.tensor(wl.token_ids(work.seed, 90, n, m.vocab), dtype=torch.int32, device="cuda")
+    pos = torch.arange(n, dtype=torch.int32, device="cuda")
+    gens = []
+    for g in range(3):
+        torch.cuda.synchronize()
+        ev[0].record(stream)
+        for t in range(n):
+            K.kfl_stage_decode_users(st, ids[t:t + 1], None, pos[t:t + 1], user, 1, None, first, sp)
+        ev[1].record(stream)
+        torch.cuda.synchronize()
+        gens.append(ev[0].elapsed_time(ev[1]))
+    one = statistics.median(gens[1:])
+    if K.kfl_stage_status(st) != 0:
+        raise RuntimeError("device reported an error during the prefill runs")
+    K.kfl_stage_destroy(st)
+    line = {"metric": "time to first token", "unit": "ms", "higher_is_better": False, "n_gpus": 1,
+            "config": {"workload": work.name, "users": 1, "steps_of": 4, "weights": "bf16",
+                       "prompt_lengths": list(lengths)},
+            "by_prompt_length": {str(k): v for k, v in rows.items()},
+            "one_token_per_step_512": {"prefill_ms": one, "prefill_tokens_per_s": n / one * 1e3},
+            "data": "synthetic (seeded)", "protocol": "5 generations, first discarded, median",
+            "timing": "CUDA events on the launching stream"}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     args = parse()
     if args.ring:
         return run_ring(args)
+    if args.prefill:
+        return run_prefill(args)
     import dataclasses
 
     from paper_2609_34045_gb300 import workload as wl

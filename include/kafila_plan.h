@@ -72,7 +72,7 @@ typedef struct {
 int kfl_plan_ring(int k, int m, const kfl_plan_device *dev, int anchor, double beta_block, double beta_head,
                   double mu, int *n_out, kfl_plan *plan);
 
-/* The baselines of the paper's evaluation (Section VI): weight == NULL, Uniform (GPipe): k / m
+/* The baselines of the paper's evaluation (Section VII): weight == NULL, Uniform (GPipe): k / m
  * blocks each, the k mod m left over to the first devices; else Memory-proportional (exo): the
  * largest-remainder apportionment of k by weight (remainders tied: the lower index first), then
  * every device left with 0 blocks takes one from the device holding most (the lowest index on

@@ -131,16 +131,41 @@ int kfl_stage_decode(kfl_stage *st, const int32_t *token_ids, const float *hidde
                      void *cuda_stream);
 
 /* kfl_stage_decode for chosen users: batch row b serves user users[b] (device int32[batch],
- * distinct values in [0, max_batch)), whose KV cache slot it reads and appends to; positions,
- * token_ids, hidden_in/out and next_ids stay indexed by batch row.  This is how one stage of a
+ * values in [0, max_batch)), whose KV cache slot it reads and appends to; positions, token_ids,
+ * hidden_in/out and next_ids stay indexed by batch row.  A user may fill several rows (several
+ * of its tokens in one step) at distinct positions: each row attends to the slot's rows
+ * [0, P_b], the ones this step writes included.  A row repeating an earlier row's user and
+ * position is treated like a bad position.  This is how one stage of a
  * ring serves one user's token at a time while other users' tokens are elsewhere in the ring
- * (Section VI, "Serving several users at once").  A user outside [0, max_batch) is found on the
+ * (Section VII, "Serving several users at once").  A user outside [0, max_batch) is found on the
  * device and treated like a bad position (nothing of that row is written, kfl_stage_status then
  * reports KFL_ERR_RANGE).  Errors returned here: those of kfl_stage_decode, and KFL_ERR_ARG for
  * users == NULL. */
 int kfl_stage_decode_users(kfl_stage *st, const int32_t *token_ids, const float *hidden_in,
                            const int32_t *positions, const int32_t *users, int batch, float *hidden_out,
                            int32_t *next_ids, void *cuda_stream);
+
+/* Prefill: run n_tokens tokens of one user's prompt through the stage, filling the user's KV
+ * cache slot at the given positions; each token attends to the slot's rows up to its own
+ * position, earlier tokens of the same call included (time to first token is the prefill plus
+ * one decode step, Section VI, instrumentation paragraph).  The tokens go as steps of up to
+ * max_batch rows, in order, every row of a step addressing the user's slot (the decode step's
+ * kernels, each weight matrix streamed once per step); enqueued on cuda_stream, returns without
+ * waiting.
+ *   token_ids  device int32[n_tokens] (KFL_EMBED_IN), else ignored
+ *   hidden_in  device fp32[n_tokens][d_model] (without KFL_EMBED_IN)
+ *   positions  device int32[n_tokens]: token t's position, distinct, normally start + t; the
+ *              slot's rows below a token's position must be cached before the call or be
+ *              earlier tokens of it (rows never written read as whatever the slot holds)
+ *   user       the KV cache slot, in [0, max_batch)
+ *   hidden_out device fp32[n_tokens][d_model] (needed without KFL_LOGITS_OUT)
+ *   next_ids   device int32[n_tokens]: the greedy token after each prompt token
+ *              (KFL_LOGITS_OUT; the last one starts the decode)
+ * Bad positions and token ids are found on the device as in kfl_stage_decode.
+ * Errors returned here: KFL_ERR_ARG, KFL_ERR_RANGE (user), KFL_ERR_STATE, KFL_ERR_CUDA. */
+int kfl_stage_prefill(kfl_stage *st, const int32_t *token_ids, const float *hidden_in,
+                      const int32_t *positions, int user, int n_tokens, float *hidden_out,
+                      int32_t *next_ids, void *cuda_stream);
 
 /* kfl_stage_decode with HOST buffers of the same shapes: copies the inputs to the device,
  * runs the step and copies the outputs back, then waits for cuda_stream.  Pinned host memory

@@ -1,4 +1,4 @@
-"""fp64 oracle of one pipeline stage's decode step (test infrastructure only).
+"""fp64 oracle of one pipeline stage's decode step and prompt prefill (test infrastructure only).
 
 What a stage computes comes from the paper:
 
@@ -197,7 +197,7 @@ class OracleStage:
         self.k_cache[local, user, :, :n] = k_bits
         self.v_cache[local, user, :, :n] = v_bits
 
-    def _block(self, local: int, h: np.ndarray, positions: np.ndarray) -> np.ndarray:
+    def _block(self, local: int, h: np.ndarray, positions: np.ndarray, slots: np.ndarray) -> np.ndarray:
         m, w = self.m, self.layers[local]
         b = h.shape[0]
         hq, hkv, hd = m.n_heads, m.n_kv_heads, m.head_dim
@@ -205,33 +205,54 @@ class OracleStage:
         q = gemv(matrix_f64(w["wq"]), y).reshape(b, hq, hd)
         k = gemv(matrix_f64(w["wk"]), y).reshape(b, hkv, hd)
         v = gemv(matrix_f64(w["wv"]), y).reshape(b, hkv, hd)
-        o = np.empty((b, hq * hd), dtype=np.float64)
+        # every row's K/V is stored before any row attends: rows of one user at several positions
+        # (a prompt) see the earlier ones, as causal attention over the prompt does
+        qs = []
         for u in range(b):
-            p = int(positions[u])
+            p, sl = int(positions[u]), int(slots[u])
             qu, ku = q[u], k[u]
             if m.qk_norm:
                 qu = rms_norm(qu, bf16_to_f64(w["q_norm"]), m.rms_eps)
                 ku = rms_norm(ku, bf16_to_f64(w["k_norm"]), m.rms_eps)
-            qu = rope_rotate(qu, p, m.rope_theta)
-            ku = rope_rotate(ku, p, m.rope_theta)
-            self.k_cache[local, u, :, p] = round_to_bf16(ku)
-            self.v_cache[local, u, :, p] = round_to_bf16(v[u])
-            kc = bf16_to_f64(self.k_cache[local, u, :, : p + 1])
-            vc = bf16_to_f64(self.v_cache[local, u, :, : p + 1])
-            o[u] = attention_gqa(qu, kc, vc).reshape(hq * hd)
+            qs.append(rope_rotate(qu, p, m.rope_theta))
+            self.k_cache[local, sl, :, p] = round_to_bf16(rope_rotate(ku, p, m.rope_theta))
+            self.v_cache[local, sl, :, p] = round_to_bf16(v[u])
+        o = np.empty((b, hq * hd), dtype=np.float64)
+        for u in range(b):
+            p, sl = int(positions[u]), int(slots[u])
+            kc = bf16_to_f64(self.k_cache[local, sl, :, : p + 1])
+            vc = bf16_to_f64(self.v_cache[local, sl, :, : p + 1])
+            o[u] = attention_gqa(qs[u], kc, vc).reshape(hq * hd)
         h = h + gemv(matrix_f64(w["wo"]), o)
         y = rms_norm(h, bf16_to_f64(w["ffn_norm"]), m.rms_eps)
         a = swiglu(gemv(matrix_f64(w["wg"]), y), gemv(matrix_f64(w["wu"]), y))
         return h + gemv(matrix_f64(w["wd"]), a)
 
-    def decode(self, positions, token_ids=None, hidden_in=None, capture: bool = False) -> dict:
-        """One decode step for users ``0..b-1``.  Returns ``hidden_out`` (fp64 ``[b][d]``),
-        and with ``logits_out``: ``next_ids``, ``margins`` (top-2 logit gap) and ``logits``;
-        with ``capture``: ``per_layer`` (hidden after each block, ``[n][b][d]``)."""
+    def decode(self, positions, token_ids=None, hidden_in=None, capture: bool = False, users=None) -> dict:
+        """One decode step for users ``0..b-1`` (``users``: row b serves user users[b]).  Returns
+        ``hidden_out`` (fp64 ``[b][d]``), and with ``logits_out``: ``next_ids``, ``margins``
+        (top-2 logit gap) and ``logits``; with ``capture``: ``per_layer`` (hidden after each
+        block, ``[n][b][d]``)."""
         positions = np.asarray(positions, dtype=np.int64)
         b = positions.shape[0]
         if b > self.max_batch:
             raise ValueError("batch exceeds max_batch")
+        slots = np.arange(b) if users is None else np.asarray(users, dtype=np.int64)
+        return self._forward(positions, slots, token_ids, hidden_in, capture)
+
+    def prefill(self, user: int, positions, token_ids=None, hidden_in=None) -> dict:
+        """A prompt of one user in one pass: token t at positions[t] attends to the user's cached
+        rows up to its position, the prompt's earlier tokens included (causal self-attention over
+        the prompt).  Any number of tokens; the results as ``decode`` gives them, per token."""
+        positions = np.asarray(positions, dtype=np.int64)
+        if len(set(positions.tolist())) != positions.shape[0]:
+            raise ValueError("a prompt's positions must be distinct")
+        if not 0 <= user < self.max_batch:
+            raise ValueError("user outside [0, max_batch)")
+        return self._forward(positions, np.full(positions.shape[0], user), token_ids, hidden_in, False)
+
+    def _forward(self, positions, slots, token_ids, hidden_in, capture) -> dict:
+        b = positions.shape[0]
         if np.any(positions < 0) or np.any(positions >= self.max_ctx):
             raise ValueError("position outside [0, max_ctx)")
         if self.embed_in:
@@ -241,7 +262,7 @@ class OracleStage:
             h = np.array(hidden_in, dtype=np.float64).reshape(b, self.m.d_model)
         per_layer = []
         for local in range(self.l1 - self.l0):
-            h = self._block(local, h, positions)
+            h = self._block(local, h, positions, slots)
             if capture:
                 per_layer.append(h.copy())
         out = {"hidden_out": h}

@@ -114,11 +114,12 @@ __device__ __forceinline__ int attn_chunk_size(const AttnParams &p) {
   return max(chunk, (need + 63) / 64 * 64);
 }
 
-// Rows [p0, p0 + cnt) of user b / KV head kvh into K/V buffer `buf`, except `skip` (the new
-// token's row, written in this step) when skip >= 0; one cp.async group.
+// Rows [p0, p0 + cnt) of user b / KV head kvh into K/V buffer `buf`: mode 0 all of them, mode 1
+// those outside [new_lo, new_hi] (the rows this step writes), mode 2 those inside; one cp.async
+// group.
 template <int HD, int NBUF>
 __device__ __forceinline__ void attn_load_rows(const AttnParams &p, int b, int kvh, int p0, int cnt, int buf,
-                                               int only, int skip, uint8_t *sm, int tid) {
+                                               int mode, int new_lo, int new_hi, uint8_t *sm, int tid) {
   using L = AttnLayout<HD, NBUF>;
   const size_t head_base = ((size_t)p.slots[b] * p.n_kv_heads + kvh) * p.max_ctx;
   const uint16_t *kg = p.kcache + head_base * HD;
@@ -129,22 +130,37 @@ __device__ __forceinline__ void attn_load_rows(const AttnParams &p, int b, int k
   for (int e = tid; e < cnt * CH; e += ATT_THREADS) {
     const int r = e / CH, ch = e % CH;
     const int row = p0 + r;
-    if ((only >= 0 && row != only) || row == skip) continue;
+    const bool fresh = row >= new_lo && row <= new_hi;
+    if ((mode == 1 && fresh) || (mode == 2 && !fresh)) continue;
     cp_async16(sk + r * L::KROW + ch * 16, kg + (size_t)row * HD + ch * 8);
     cp_async16(sv + r * L::VROW + ch * 16, vg + (size_t)row * HD + ch * 8);
   }
   cp_async_commit();
 }
 
+// The lowest position of user b's KV slot that this step writes: its own position, or an
+// earlier one of another batch row on the same slot (several of a user's tokens in one step, as
+// in a prefill).  Rows from there to its own position are written by this step's Q/K/V phase.
+__device__ __forceinline__ int attn_step_lo(const AttnParams &p, int b) {
+  const int P = p.positions[b], sl = p.slots[b];
+  int lo = P;
+  for (int j = 0; j < p.batch; ++j) {
+    const int q = p.positions[j];
+    if (p.slots[j] == sl && q >= 0 && q < lo) lo = q;
+  }
+  return lo;
+}
+
 // Issue the loads of a unit's first sub-tile that do not depend on the current step: every row
-// but the new token's (which the QKV phase writes).  The unit then runs with prefetched = 1.
+// before the step's first new one (attn_step_lo).  The unit then runs with prefetched = 1.
+// Positions and slots are final before the step's kernels start.
 template <int HD, int NBUF>
 __device__ __forceinline__ void attn_prefetch(const AttnParams &p, int b, int kvh, int c, uint8_t *sm, int tid) {
   const int P = p.positions[b];
   if (P < 0 || P >= p.max_ctx) return;
   const int start = c * p.chunk;
   const int end = min(P + 1, start + p.chunk);
-  attn_load_rows<HD, NBUF>(p, b, kvh, start, min(ATT_SUB, end - start), 0, -1, P, sm, tid);
+  attn_load_rows<HD, NBUF>(p, b, kvh, start, min(ATT_SUB, end - start), 0, 1, attn_step_lo(p, b), P, sm, tid);
 }
 
 // The (user, KV head) output is written: publish it (persistent kernel; the bar.sync orders every
@@ -227,11 +243,11 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
 
   auto load_sub = [&](int sub, int buf) {
     const int p0 = start + sub * ATT_SUB;
-    attn_load_rows<HD, NBUF>(p, b, kvh, p0, min(ATT_SUB, end - p0), buf, -1, -1, sm, tid);
+    attn_load_rows<HD, NBUF>(p, b, kvh, p0, min(ATT_SUB, end - p0), buf, 0, 0, -1, sm, tid);
   };
   // the first sub-tile's copies go out first, so that their latency overlaps the q loads
-  if (prefetched)  // only the new token's row of the first sub-tile is still to load
-    attn_load_rows<HD, NBUF>(p, b, kvh, start, min(ATT_SUB, end - start), 0, P, -1, sm, tid);
+  if (prefetched)  // only the rows this step wrote (attn_step_lo .. P) are still to load
+    attn_load_rows<HD, NBUF>(p, b, kvh, start, min(ATT_SUB, end - start), 0, 2, attn_step_lo(p, b), P, sm, tid);
   else
     load_sub(0, 0);
 

@@ -529,7 +529,8 @@ cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int
                                int batch, const uint16_t *embed, int vocab, int d, int ldh,
                                const float *g_next, float *h, float *xn, float *sumsq,
                                int *positions, int max_ctx, unsigned *err, unsigned *bar, Act16 xn16,
-                               const int *users, int max_batch, int *slots, cudaStream_t s);
+                               const int *users, int user_all, int max_batch, int *slots,
+                               cudaStream_t s);
 size_t stage_kernel_smem(int stages, int head_dim, int batch, int fmt);
 int stage_kernel_attn_bytes(int head_dim);
 cudaError_t prepare_stage_kernel(size_t smem);

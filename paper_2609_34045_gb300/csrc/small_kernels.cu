@@ -12,7 +12,8 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
                                                          int vocab, int d, int ldh, const float *g_next,
                                                          float *h, float *xn, float *sumsq, int *positions,
                                                          int max_ctx, unsigned *err, unsigned *bar, Act16 xn16,
-                                                         const int *users, int max_batch, int *slots) {
+                                                         const int *users, int user_all, int max_batch,
+                                                         int *slots) {
   __shared__ float vals[64];
   const int b = blockIdx.y, tid = threadIdx.x, r = blockIdx.x * 64 + tid;
   pdl_launch_dependents();
@@ -20,14 +21,21 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
   if (blockIdx.x == 0 && tid == 0) {
     int pos = positions_in[b];
     if (pos < 0 || pos >= max_ctx) atomicOr(err, ERR_POSITION);
-    // the user's KV slot (users NULL: batch row b is user b); a slot outside [0, max_batch) is
-    // flagged like a bad position, and the row's position is made invalid so that nothing of it
-    // is written
-    const int u = users ? users[b] : b;
+    // the user's KV slot (users NULL: user_all for every row if >= 0, else batch row b is user
+    // b); a slot outside [0, max_batch) is flagged like a bad position, and the row's position is
+    // made invalid so that nothing of it is written.  Rows of one user must hold distinct
+    // positions (each writes its own cache row): a repeat of an earlier row's is flagged the same.
+    auto slot_of = [&](int j) { return users ? users[j] : (user_all >= 0 ? user_all : j); };
+    const int u = slot_of(b);
     if (u < 0 || u >= max_batch) {
       atomicOr(err, ERR_POSITION);
       pos = -1;
     }
+    for (int j = 0; j < b && pos >= 0; ++j)
+      if (slot_of(j) == u && positions_in[j] == pos) {
+        atomicOr(err, ERR_POSITION);
+        pos = -1;
+      }
     slots[b] = (u < 0 || u >= max_batch) ? 0 : u;
     positions[b] = pos;
     // abort flag of the persistent stage kernel that follows
@@ -76,11 +84,11 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in, int batch,
                                const uint16_t *embed, int vocab, int d, int ldh, const float *g_next, float *h,
                                float *xn, float *sumsq, int *positions, int max_ctx, unsigned *err,
-                               unsigned *bar, Act16 xn16, const int *users, int max_batch, int *slots,
-                               cudaStream_t s) {
+                               unsigned *bar, Act16 xn16, const int *users, int user_all, int max_batch,
+                               int *slots, cudaStream_t s) {
   dim3 grid((d + 63) / 64, batch);
   stage_input_kernel<<<grid, 64, 0, s>>>(ids, hidden_in, positions_in, embed, vocab, d, ldh, g_next, h, xn, sumsq,
-                                         positions, max_ctx, err, bar, xn16, users, max_batch, slots);
+                                         positions, max_ctx, err, bar, xn16, users, user_all, max_batch, slots);
   return cudaGetLastError();
 }
 

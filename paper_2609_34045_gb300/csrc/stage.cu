@@ -618,8 +618,11 @@ const float *input_g_next(const kfl_stage *st) {
   return nullptr;
 }
 
+// One step over `batch` rows.  Row b's KV slot: users[b] (device) when users is non-NULL, else
+// user_all for every row when user_all >= 0, else b.
 int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const int32_t *positions,
-             const int32_t *users, int batch, float *hidden_out, int32_t *next_ids, cudaStream_t s) {
+             const int32_t *users, int user_all, int batch, float *hidden_out, int32_t *next_ids,
+             cudaStream_t s) {
   const Plan &P = st->P;
   const bool embed = (st->flags & KFL_EMBED_IN) != 0;
   const bool body = P.nl > 0 || (st->flags & KFL_LOGITS_OUT);
@@ -634,8 +637,8 @@ int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const in
     CK(cudaEventRecord(st->ev[0], s));
     CK(launch_stage_input(ids, hidden_in, positions, batch, embed ? st->embed : nullptr, P.V, P.d, P.ldh,
                           input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, st->bar,
-                          st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn16 : Act16{}, users, st->cfg.max_batch,
-                          st->slots, s));
+                          st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn16 : Act16{}, users, user_all,
+                          st->cfg.max_batch, st->slots, s));
     CK(cudaEventRecord(st->ev[1], s));
     kinds.push_back(KFL_KERNEL_INPUT);
     int rc = enqueue_body(st, batch, s, false, &kinds, 1);
@@ -656,8 +659,8 @@ int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const in
   }
   CK(launch_stage_input(ids, hidden_in, positions, batch, embed ? st->embed : nullptr, P.V, P.d, P.ldh,
                         input_g_next(st), st->h, st->xn, st->sumsq, st->pos, st->cfg.max_ctx, st->err, st->bar,
-                        st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn16 : Act16{}, users, st->cfg.max_batch,
-                        st->slots, s));
+                        st->cfg.weight_fmt == KFL_INT4_G64 ? st->xn16 : Act16{}, users, user_all,
+                        st->cfg.max_batch, st->slots, s));
   if (body) {
     int rc = ensure_graph(st, batch);
     if (rc != KFL_OK) return rc;
@@ -1032,7 +1035,7 @@ extern "C" int kfl_stage_decode(kfl_stage *st, const int32_t *token_ids, const f
   int rc = check_decode_args(st, token_ids, hidden_in, positions, batch, hidden_out, next_ids);
   if (rc) return rc;
   CK(cudaSetDevice(st->dev));
-  return run_step(st, token_ids, hidden_in, positions, nullptr, batch, hidden_out, next_ids,
+  return run_step(st, token_ids, hidden_in, positions, nullptr, -1, batch, hidden_out, next_ids,
                   static_cast<cudaStream_t>(cuda_stream));
 }
 
@@ -1043,8 +1046,32 @@ extern "C" int kfl_stage_decode_users(kfl_stage *st, const int32_t *token_ids, c
   if (rc) return rc;
   if (!users) return KFL_ERR_ARG;
   CK(cudaSetDevice(st->dev));
-  return run_step(st, token_ids, hidden_in, positions, users, batch, hidden_out, next_ids,
+  return run_step(st, token_ids, hidden_in, positions, users, -1, batch, hidden_out, next_ids,
                   static_cast<cudaStream_t>(cuda_stream));
+}
+
+extern "C" int kfl_stage_prefill(kfl_stage *st, const int32_t *token_ids, const float *hidden_in,
+                                 const int32_t *positions, int user, int n_tokens, float *hidden_out,
+                                 int32_t *next_ids, void *cuda_stream) {
+  if (!valid(st)) return KFL_ERR_STATE;
+  if (n_tokens < 1 || !positions) return KFL_ERR_ARG;
+  if ((st->flags & KFL_EMBED_IN) ? !token_ids : !hidden_in) return KFL_ERR_ARG;
+  if ((st->flags & KFL_LOGITS_OUT) ? !next_ids : !hidden_out) return KFL_ERR_ARG;
+  if (user < 0 || user >= st->cfg.max_batch) return KFL_ERR_RANGE;
+  if (!st->loaded()) return KFL_ERR_STATE;
+  CK(cudaSetDevice(st->dev));
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  const int d = st->P.d;
+  // the prompt in chunks of max_batch consecutive tokens: each chunk is one step whose rows all
+  // address the user's KV slot, so a token attends to the chunk's earlier tokens too
+  for (int t0 = 0; t0 < n_tokens; t0 += st->cfg.max_batch) {
+    const int n = std::min(st->cfg.max_batch, n_tokens - t0);
+    const int rc = run_step(st, token_ids ? token_ids + t0 : nullptr, hidden_in ? hidden_in + (size_t)t0 * d : nullptr,
+                            positions + t0, nullptr, user, n, hidden_out ? hidden_out + (size_t)t0 * d : nullptr,
+                            next_ids ? next_ids + t0 : nullptr, s);
+    if (rc != KFL_OK) return rc;
+  }
+  return KFL_OK;
 }
 
 extern "C" int kfl_stage_decode_host(kfl_stage *st, const int32_t *token_ids, const float *hidden_in,
@@ -1059,8 +1086,8 @@ extern "C" int kfl_stage_decode_host(kfl_stage *st, const int32_t *token_ids, co
   CK(cudaMemcpyAsync(st->io_pos, positions, (size_t)batch * 4, cudaMemcpyHostToDevice, s));
   if (embed) CK(cudaMemcpyAsync(st->io_ids, token_ids, (size_t)batch * 4, cudaMemcpyHostToDevice, s));
   else CK(cudaMemcpyAsync(st->io_hin, hidden_in, (size_t)batch * P.d * 4, cudaMemcpyHostToDevice, s));
-  rc = run_step(st, embed ? st->io_ids : nullptr, embed ? nullptr : st->io_hin, st->io_pos, nullptr, batch, nullptr,
-                nullptr, s);
+  rc = run_step(st, embed ? st->io_ids : nullptr, embed ? nullptr : st->io_hin, st->io_pos, nullptr, -1, batch,
+                nullptr, nullptr, s);
   if (rc) return rc;
   if (hidden_out)
     CK(cudaMemcpy2DAsync(hidden_out, (size_t)P.d * 4, st->h, (size_t)P.ldh * 4, (size_t)P.d * 4, batch,

@@ -5,7 +5,7 @@ blocks, each member runs its contiguous block range in turn, and the hidden stat
 head for the final RMSNorm, lm_head and sampler (the head's return leg).  Decoding one user is
 sequential around the ring, so at any instant one stage computes and the others wait; several
 users' requests fill that bubble, each stage working on one user's token while another stage works
-on the next user's (section VI, "Serving several users at once"; Eq. 1's compute term).
+on the next user's (section VII, "Serving several users at once"; Eq. 1's compute term).
 
 Here every member is a stage of the library on this GPU, with its own CUDA stream, and the return
 leg is a stage of its own (no blocks, KFL_LOGITS_OUT).  A stage serves one user per call

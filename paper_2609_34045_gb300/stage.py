@@ -84,6 +84,7 @@ def lib() -> C.CDLL:
             "kfl_stage_decode": ([vp, vp, vp, vp, i, vp, vp, vp], i),
             "kfl_stage_decode_host": ([vp, vp, vp, vp, i, vp, vp, vp], i),
             "kfl_stage_decode_users": ([vp, vp, vp, vp, vp, i, vp, vp, vp], i),
+            "kfl_stage_prefill": ([vp, vp, vp, vp, i, i, vp, vp, vp], i),
             "kfl_kv_reset": ([vp, i], i),
             "kfl_kv_fill_seeded": ([vp, i, i, C.c_uint64], i),
             "kfl_kv_write": ([vp, i, i, vp, vp, i, i], i),
@@ -233,6 +234,15 @@ def kfl_stage_decode_users(st: Stage, token_ids, hidden_in, positions, users, ba
     _check(lib().kfl_stage_decode_users(st.handle, _ptr(token_ids), _ptr(hidden_in), _ptr(positions), _ptr(users),
                                         batch, _ptr(hidden_out), _ptr(next_ids), cuda_stream),
            "kfl_stage_decode_users")
+
+
+def kfl_stage_prefill(st: Stage, token_ids, hidden_in, positions, user: int, n_tokens: int, hidden_out, next_ids,
+                      cuda_stream: int | None = None) -> None:
+    """n_tokens prompt tokens of one user (KV slot `user`) through the stage, in steps of up to
+    max_batch rows: int32 token_ids [n] or fp32 hidden_in [n][d], int32 positions [n], fp32
+    hidden_out [n][d], int32 next_ids [n] (CUDA tensors).  Asynchronous."""
+    _check(lib().kfl_stage_prefill(st.handle, _ptr(token_ids), _ptr(hidden_in), _ptr(positions), user, n_tokens,
+                                   _ptr(hidden_out), _ptr(next_ids), cuda_stream), "kfl_stage_prefill")
 
 
 def kfl_stage_decode_host(st: Stage, token_ids, hidden_in, positions, batch: int, hidden_out, next_ids,

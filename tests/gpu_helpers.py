@@ -159,6 +159,8 @@ class Pair:
                 mask[written] = False
                 assert np.array_equal(kg[:, mask], self.k0[layer, u][:, mask])
                 assert np.array_equal(vg[:, mask], self.v0[layer, u][:, mask])
+                if not written:
+                    continue
                 for cache_g, cache_o in ((kg, self.ora.k_cache), (vg, self.ora.v_cache)):
                     g = oracle.bf16_to_f64(cache_g[:, written])
                     r = oracle.bf16_to_f64(cache_o[layer, u][:, written])

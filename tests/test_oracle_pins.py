@@ -295,6 +295,83 @@ def pin_stage_split_associativity():
         ids = o_full["next_ids"]
 
 
+def _torch_prefill(model, layers, head, kcache, vcache, start, ids, causal=True):
+    """A prompt of one user (cache [layer][Hkv][ctx][hd] bf16 bits, filled below `start`) in
+    matrix form: every token's K/V appended at start + t, then one masked attention with torch's
+    F.scaled_dot_product_attention, token t seeing cache rows <= start + t (causal=False: the
+    whole prompt, to show the check can fail)."""
+    def bf(bits):
+        if isinstance(bits, tuple):
+            return _int4_by_lut(bits)
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(torch.float64)
+    d, hq, hkv, hd = model.d_model, model.n_heads, model.n_kv_heads, model.head_dim
+    T = len(ids)
+    h = bf(head["embed"][ids])
+    kc = [bf(k.copy()) for k in kcache]
+    vc = [bf(v.copy()) for v in vcache]
+    pos = torch.arange(start, start + T, dtype=torch.float64)
+    freq = torch.tensor([model.rope_theta ** (-(2.0 * i) / hd) for i in range(hd // 2)], dtype=torch.float64)
+    rot = torch.polar(torch.ones(T, hd // 2, dtype=torch.float64), pos[:, None] * freq[None, :])
+
+    def rope(x):  # [T][heads][hd]
+        z = torch.complex(x[..., : hd // 2], x[..., hd // 2:]) * rot[:, None, :]
+        return torch.cat([z.real, z.imag], dim=-1)
+    ctx = start + T
+    seen = torch.arange(ctx)[None, :] <= (start + torch.arange(T))[:, None]
+    mask = seen if causal else torch.ones(T, ctx, dtype=torch.bool)
+    for li, w in enumerate(layers):
+        y = F.rms_norm(h, (d,), weight=bf(w["attn_norm"]), eps=model.rms_eps)
+        q = rope(F.linear(y, bf(w["wq"])).view(T, hq, hd))
+        k = rope(F.linear(y, bf(w["wk"])).view(T, hkv, hd))
+        v = F.linear(y, bf(w["wv"])).view(T, hkv, hd)
+        kc[li][:, start:ctx] = k.transpose(0, 1).to(torch.float32).to(torch.bfloat16).to(torch.float64)
+        vc[li][:, start:ctx] = v.transpose(0, 1).to(torch.float32).to(torch.bfloat16).to(torch.float64)
+        K = kc[li][:, :ctx].repeat_interleave(hq // hkv, 0)
+        V = vc[li][:, :ctx].repeat_interleave(hq // hkv, 0)
+        o = F.scaled_dot_product_attention(q.transpose(0, 1), K, V, attn_mask=mask)  # [hq][T][hd]
+        h = h + F.linear(o.transpose(0, 1).reshape(T, hq * hd), bf(w["wo"]))
+        y = F.rms_norm(h, (d,), weight=bf(w["ffn_norm"]), eps=model.rms_eps)
+        h = h + F.linear(F.silu(F.linear(y, bf(w["wg"]))) * F.linear(y, bf(w["wu"])), bf(w["wd"]))
+    y = F.rms_norm(h, (d,), weight=bf(head["final_norm"]), eps=model.rms_eps)
+    z = F.linear(y, bf(head["lm_head"]))
+    return h.numpy(), z.numpy(), kc, vc
+
+
+def pin_prefill_vs_torch():
+    # user 1 (9 cached rows) takes a prompt of 6 tokens at positions 9..14; user 0 is untouched
+    st = _small_stage(0, 3, True, True)
+    k0 = [st.k_cache[i, 1].copy() for i in range(3)]
+    v0 = [st.v_cache[i, 1].copy() for i in range(3)]
+    other = (st.k_cache[:, 0].copy(), st.v_cache[:, 0].copy())
+    ids = np.array([3, 44, 17, 17, 0, 49])
+    out = st.prefill(1, np.arange(9, 15), token_ids=ids)
+    layers = [st.layers[i] for i in range(3)]
+    h, z, kc, vc = _torch_prefill(SMALL, layers, st.head, k0, v0, 9, ids)
+    assert np.allclose(out["hidden_out"], h, rtol=1e-11, atol=1e-12)
+    assert np.allclose(out["logits"], z, rtol=1e-11, atol=1e-12)
+    for i in range(3):
+        assert np.array_equal(oracle.bf16_to_f64(st.k_cache[i, 1]), kc[i].numpy())
+        assert np.array_equal(oracle.bf16_to_f64(st.v_cache[i, 1]), vc[i].numpy())
+    assert np.array_equal(st.k_cache[:, 0], other[0]) and np.array_equal(st.v_cache[:, 0], other[1])
+    # the same check without the causal mask fails: it tests what each token sees
+    h_all, _, _, _ = _torch_prefill(SMALL, layers, st.head, k0, v0, 9, ids, causal=False)
+    assert not np.allclose(out["hidden_out"], h_all, rtol=1e-6, atol=1e-6)
+
+
+def pin_prefill_is_sequential_decode():
+    # one pass over the prompt equals one decode step per token (and from an empty cache)
+    for start in (0, 9):
+        a = _small_stage(0, 3, True, True)
+        b = _small_stage(0, 3, True, True)
+        ids = np.array([8, 1, 30, 30, 12])
+        pa = a.prefill(1, np.arange(start, start + 5), token_ids=ids)
+        for t in range(5):
+            ob = b.decode(np.array([start + t]), token_ids=ids[t:t + 1], users=[1])
+            assert np.allclose(pa["hidden_out"][t], ob["hidden_out"][0], rtol=1e-12, atol=1e-13)
+            assert pa["next_ids"][t] == ob["next_ids"][0]
+        assert np.array_equal(a.k_cache, b.k_cache) and np.array_equal(a.v_cache, b.v_cache)
+
+
 SMALL_INT4 = wl.ModelShape(n_layers_total=2, d_model=128, n_heads=4, n_kv_heads=2, head_dim=32, ffn=192,
                            vocab=40, weight_fmt="int4_g64")
 
@@ -305,7 +382,8 @@ def pin_int4_stage_vs_torch():
 
 PINS = [pin_bf16_golden, pin_bf16_vs_torch, pin_int4_exhaustive, pin_int4_groups, pin_gemv_bruteforce,
         pin_rms_norm, pin_rope, pin_softmax, pin_attention, pin_silu, pin_argmax, pin_stage_vs_torch,
-        pin_kv_slots, pin_stage_split_associativity, pin_int4_stage_vs_torch]
+        pin_kv_slots, pin_stage_split_associativity, pin_int4_stage_vs_torch, pin_prefill_vs_torch,
+        pin_prefill_is_sequential_decode]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -432,8 +510,8 @@ def test_planted_transposed_gemv_is_caught(monkeypatch):
 def test_planted_residual_drop_is_caught(monkeypatch):
     orig = ost.OracleStage._block
 
-    def no_residual(self, local, h, positions):
-        return orig(self, local, h, positions) - h
+    def no_residual(self, local, h, positions, slots):
+        return orig(self, local, h, positions, slots) - h
 
     monkeypatch.setattr(ost.OracleStage, "_block", no_residual)
     with pytest.raises(AssertionError):
