@@ -657,10 +657,11 @@ def run_ring(args):
 def run_prefill(args):
     """Time to first token split into prefill and decode (section VI, instrumentation paragraph)
     on the 7B-shaped model as one head stage, one user from an empty cache: the prompt goes
-    through kfl_stage_prefill (steps of max_batch = 4 of its tokens), then one decode step.  As in
-    the paper's protocol, five generations per prompt length, the first discarded as cold, the
-    median of the rest; CUDA events on the launching stream.  For comparison the same prompt one
-    token per step (kfl_stage_decode_users at batch 1)."""
+    through kfl_stage_prefill, then one decode step.  The prefill is the dense path (tensor-core
+    matrix products over the prompt's tokens); for comparison the 512-token prompt also in steps
+    of max_batch = 4 tokens through the decode kernels, and one token per step
+    (kfl_stage_decode_users at batch 1).  As in the paper's protocol, five generations per case,
+    the first discarded as cold, the median of the rest; CUDA events on the launching stream."""
     import dataclasses
     import statistics
 
@@ -684,8 +685,9 @@ def run_prefill(args):
     sp = stream.cuda_stream
     user = torch.zeros(1, dtype=torch.int32, device="cuda")
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
-    rows = {}
-    for n in lengths:
+
+    def ttft(n, dense):
+        os.environ["KFL_PREFILL_DENSE_MIN"] = "1" if dense else str(1 << 30)
         ids = torch.tensor(wl.token_ids(work.seed, 90, n, m.vocab), device="cuda")
         pos = torch.arange(n, dtype=torch.int32, device="cuda")
         nxt = torch.zeros(n, dtype=torch.int32, device="cuda")
@@ -705,11 +707,19 @@ def run_prefill(args):
             gens.append((ev[0].elapsed_time(ev[1]), ev[1].elapsed_time(ev[2])))
         pre = statistics.median(x[0] for x in gens[1:])
         dec = statistics.median(x[1] for x in gens[1:])
-        rows[n] = {"prefill_ms": pre, "decode_ms": dec, "ttft_ms": pre + dec, "prefill_tokens_per_s": n / pre * 1e3}
+        # the weight products only (attention's products excluded)
+        flops = 2.0 * n * (m.n_layers_total * sum(r * c for r, c in m.matrix_shapes().values()) + m.vocab * m.d_model)
+        return {"prefill_ms": pre, "decode_ms": dec, "ttft_ms": pre + dec, "prefill_tokens_per_s": n / pre * 1e3,
+                "matmul_tflops": flops / pre / 1e9}
+
+    rows = {n: ttft(n, True) for n in lengths}
+    steps512 = ttft(512, False)
+    os.environ.pop("KFL_PREFILL_DENSE_MIN", None)
     # one token per step, the 512-token prompt
     n = 512
     ids = torch.tensor(wl.token_ids(work.seed, 90, n, m.vocab), dtype=torch.int32, device="cuda")
     pos = torch.arange(n, dtype=torch.int32, device="cuda")
+    first = torch.zeros(1, dtype=torch.int32, device="cuda")
     gens = []
     for g in range(3):
         torch.cuda.synchronize()
@@ -724,9 +734,10 @@ def run_prefill(args):
         raise RuntimeError("device reported an error during the prefill runs")
     K.kfl_stage_destroy(st)
     line = {"metric": "time to first token", "unit": "ms", "higher_is_better": False, "n_gpus": 1,
-            "config": {"workload": work.name, "users": 1, "steps_of": 4, "weights": "bf16",
+            "config": {"workload": work.name, "users": 1, "weights": "bf16",
                        "prompt_lengths": list(lengths)},
-            "by_prompt_length": {str(k): v for k, v in rows.items()},
+            "dense_by_prompt_length": {str(k): v for k, v in rows.items()},
+            "steps_of_4_512": steps512,
             "one_token_per_step_512": {"prefill_ms": one, "prefill_tokens_per_s": n / one * 1e3},
             "data": "synthetic (seeded)", "protocol": "5 generations, first discarded, median",
             "timing": "CUDA events on the launching stream"}

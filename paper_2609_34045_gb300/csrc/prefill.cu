@@ -1,0 +1,777 @@
+// Dense prompt prefill kernels (sm_103a): the tcgen05 GEMM with its fused epilogues, causal
+// attention of the prompt's tokens over the user's KV cache, row RMSNorm, the prompt's input rows
+// and the greedy argmax over the column tiles.
+//
+// The prefill computes what one decode step per prompt token computes (section III: a stage
+// applies its block range to every token; the head's sampler is greedy), with the tokens of a
+// pass as the rows of dense matrix products instead of one weight pass per token.
+#include <cudaTypedefs.h>
+
+#include <cmath>
+
+#include "../../include/kafila_gemm.h"
+#include "prefill.cuh"
+
+namespace kfl {
+
+// ---------------------------------------------------------------------------- tcgen05 / TMA
+namespace {
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Tensor-memory allocation by one whole warp; the base address is written to shared memory.
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t cols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(cols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t cols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(cols) : "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major operand in the 128-byte swizzled layout: rows of
+// 128 bytes (64 bf16 of K), groups of 8 rows 1024 bytes apart (the stride byte offset); the
+// leading byte offset is unused in this layout (1 by convention); descriptor version 1; swizzle
+// mode 2 (128 bytes).  A slice of 16 K values starts 32 bytes further within the row.
+__device__ __forceinline__ uint64_t sdesc_k_sw128(uint32_t addr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((addr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;
+  d |= (uint64_t)(1024 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulator (bits 4-5 = 1), A and B bf16 (bits 7-9
+// and 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 in bits 17-22, M >> 4 in bits 24-28.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int m, int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16_ss(uint32_t d_tmem, uint64_t da, uint64_t db, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(da), "l"(db), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive on an mbarrier of this CTA once every MMA this thread issued before has completed.
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+
+// 32 consecutive fp32 columns of this thread's tensor-memory lane (warp w reads lanes 32 w ..).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int c0, int c1, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *map, int c0, int c1, int c2, int c3,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], "
+      "[%6];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  return (uint32_t)f32_to_bf16_rne(lo) | ((uint32_t)f32_to_bf16_rne(hi) << 16);
+}
+
+// x as two bf16 terms: hi = bf16(x), lo = bf16(x - hi) (the difference is exact in fp32).
+__device__ __forceinline__ void split_bf16(float x, uint16_t &hi, uint16_t &lo) {
+  hi = f32_to_bf16_rne(x);
+  lo = f32_to_bf16_rne(x - bf16_to_f32(hi));
+}
+// Two values as packed pairs of their hi and lo terms.
+__device__ __forceinline__ void split_pack(float x0, float x1, uint32_t &hi, uint32_t &lo) {
+  uint16_t h0, l0, h1, l1;
+  split_bf16(x0, h0, l0);
+  split_bf16(x1, h1, l1);
+  hi = (uint32_t)h0 | ((uint32_t)h1 << 16);
+  lo = (uint32_t)l0 | ((uint32_t)l1 << 16);
+}
+
+// ---------------------------------------------------------------------------- GEMM epilogues
+// Thread = one token t of the tile (its tensor-memory lane); v[j] = Y[t][n + j], j < 32.
+
+template <int MODE>
+struct EpiState {
+  float best = -INFINITY;
+  int bidx = 0x7FFFFFFF;
+};
+
+template <int MODE>
+__device__ __forceinline__ void epilogue32(const PrefillEpiParams &ep, int t, int n, const uint32_t (&r)[32],
+                                           EpiState<MODE> &st) {
+  float v[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+  if constexpr (MODE == PE_STORE || MODE == PE_RESID) {
+    float *row = ep.out + (size_t)t * ep.ldo + n;
+    if (n + 32 <= ep.N) {
+#pragma unroll
+      for (int j = 0; j < 32; j += 4) {
+        float4 y = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+        if constexpr (MODE == PE_RESID) {
+          const float4 h = *reinterpret_cast<const float4 *>(row + j);
+          y.x += h.x;
+          y.y += h.y;
+          y.z += h.z;
+          y.w += h.w;
+        }
+        *reinterpret_cast<float4 *>(row + j) = y;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (n + j < ep.N) row[j] = (MODE == PE_RESID ? row[j] : 0.f) + v[j];
+    }
+  } else if constexpr (MODE == PE_SWIGLU) {
+    // 16 outputs j0 .. j0 + 15, as hi and lo terms
+    const int j0 = n >> 1;
+    uint32_t w[8], wl[8];
+#pragma unroll
+    for (int i = 0; i < 16; i += 2) {
+      const float g0 = v[2 * i], u0 = v[2 * i + 1], g1 = v[2 * i + 2], u1 = v[2 * i + 3];
+      split_pack(g0 / (1.0f + expf(-g0)) * u0, g1 / (1.0f + expf(-g1)) * u1, w[i / 2], wl[i / 2]);
+    }
+    uint16_t *row = ep.out16 + (size_t)t * ep.ldo16 + j0;
+    uint16_t *rlo = ep.out16lo + (size_t)t * ep.ldo16 + j0;
+    if (n + 32 <= ep.N) {
+      reinterpret_cast<uint4 *>(row)[0] = make_uint4(w[0], w[1], w[2], w[3]);
+      reinterpret_cast<uint4 *>(row)[1] = make_uint4(w[4], w[5], w[6], w[7]);
+      reinterpret_cast<uint4 *>(rlo)[0] = make_uint4(wl[0], wl[1], wl[2], wl[3]);
+      reinterpret_cast<uint4 *>(rlo)[1] = make_uint4(wl[4], wl[5], wl[6], wl[7]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        if (n + 2 * i + 1 < ep.N) {
+          row[i] = (uint16_t)(w[i / 2] >> (16 * (i & 1)));
+          rlo[i] = (uint16_t)(wl[i / 2] >> (16 * (i & 1)));
+        }
+    }
+  } else if constexpr (MODE == PE_QKV) {
+    const int pos = ep.positions[t];
+    if (pos < 0) return;
+    const int half = ep.hd / 2;
+    if (n < ep.qdim + ep.kvdim) {
+      // 16 RoPE pairs (i, i + hd/2) of one head
+      const bool is_q = n < ep.qdim;
+      const int r0 = is_q ? n : n - ep.qdim;
+      const int head = r0 / ep.hd, i0 = (r0 % ep.hd) / 2;
+      const float *cs = ep.rope_cos + (size_t)pos * half + i0;
+      const float *sn = ep.rope_sin + (size_t)pos * half + i0;
+      uint16_t *dst;
+      if (is_q) {
+        dst = ep.out16 + (size_t)t * ep.ldo16 + (size_t)head * ep.hd;
+      } else {
+        dst = ep.kcache + (((size_t)ep.slot * ep.hkv + head) * ep.max_ctx + pos) * ep.hd;
+      }
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const float x1 = v[2 * i], x2 = v[2 * i + 1], c = cs[i], s = sn[i];
+        dst[i0 + i] = f32_to_bf16_rne(x1 * c - x2 * s);
+        dst[i0 + i + half] = f32_to_bf16_rne(x2 * c + x1 * s);
+      }
+    } else {
+      const int r0 = n - ep.qdim - ep.kvdim;
+      const int head = r0 / ep.hd, j0 = r0 % ep.hd;
+      uint16_t *dst = ep.vcache + (((size_t)ep.slot * ep.hkv + head) * ep.max_ctx + pos) * ep.hd + j0;
+      uint32_t w[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) w[i] = pack_bf16(v[2 * i], v[2 * i + 1]);
+#pragma unroll
+      for (int i = 0; i < 16; i += 4) reinterpret_cast<uint4 *>(dst)[i / 4] = make_uint4(w[i], w[i + 1], w[i + 2], w[i + 3]);
+    }
+  } else if constexpr (MODE == PE_ARGMAX) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (n + j < ep.N && v[j] > st.best) {
+        st.best = v[j];
+        st.bidx = n + j;
+      }
+  }
+}
+
+// ---------------------------------------------------------------------------- GEMM kernel
+template <int MODE>
+__global__ void __launch_bounds__(PG_THREADS, 1)
+    prefill_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_a2,
+                        const __grid_constant__ CUtensorMap tm_b, int n_kblocks, PrefillEpiParams ep) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t s_full[PG_STAGES], s_empty[PG_STAGES], s_accum;
+  __shared__ uint32_t s_tmem;
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int t0 = blockIdx.x * PG_M, n0 = blockIdx.y * PG_N;
+  // the swizzled tiles start on a 1024-byte boundary
+  const uint32_t raw = smem_addr(smem_raw);
+  const uint32_t sa = (raw + 1023u) & ~1023u;      // [stage][hi, lo] activation tiles
+  const uint32_t sb = sa + PG_STAGES * 2 * PG_A_BYTES;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < PG_STAGES; ++s) {
+      mbar_init(smem_addr(&s_full[s]), 1);
+      mbar_init(smem_addr(&s_empty[s]), 1);
+    }
+    mbar_init(smem_addr(&s_accum), 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+  if (warp == 0) tmem_alloc(smem_addr(&s_tmem), PG_TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+
+  if (threadIdx.x == 0) {
+    // ---- TMA producer
+    int issued[PG_STAGES] = {};
+    bool ok = true;
+    for (int kb = 0; kb < n_kblocks; ++kb) {
+      const int s = kb % PG_STAGES;
+      const uint32_t use = kb / PG_STAGES;
+      if (use > 0 && !mbar_wait(smem_addr(&s_empty[s]), (use - 1) & 1)) {
+        ok = false;
+        break;
+      }
+      const uint32_t full = smem_addr(&s_full[s]);
+      mbar_arrive_expect_tx(full, 2 * PG_A_BYTES + PG_B_BYTES);
+      tma_load_2d(sa + s * 2 * PG_A_BYTES, &tm_a, kb * PG_K, t0, full);
+      tma_load_2d(sa + s * 2 * PG_A_BYTES + PG_A_BYTES, &tm_a2, kb * PG_K, t0, full);
+      // weight tiles: (column within the K tile, row within the row block, K tile, row block)
+      tma_load_4d(sb + s * PG_B_BYTES, &tm_b, (kb & 1) * PG_K, 0, kb >> 1, n0 / RB, full);
+      ++issued[s];
+    }
+    if (!ok) {
+      atomicOr(ep.err, ERR_TIMEOUT);
+      // let the copies in flight land before the CTA's shared memory is released
+      for (int s = 0; s < PG_STAGES; ++s)
+        if (issued[s] > 0) mbar_wait(smem_addr(&s_full[s]), (issued[s] - 1) & 1);
+    }
+  } else if (threadIdx.x == 32) {
+    // ---- MMA issuer
+    constexpr uint32_t idesc = idesc_bf16_f32(PG_M, PG_N);
+    for (int kb = 0; kb < n_kblocks; ++kb) {
+      const int s = kb % PG_STAGES;
+      if (!mbar_wait(smem_addr(&s_full[s]), (kb / PG_STAGES) & 1)) {
+        atomicOr(ep.err, ERR_TIMEOUT);
+        break;
+      }
+      tc_fence_after();
+      const uint32_t a = sa + s * 2 * PG_A_BYTES, b = sb + s * PG_B_BYTES;
+#pragma unroll
+      for (int k = 0; k < PG_K / 16; ++k) {
+        const uint64_t db = sdesc_k_sw128(b + 32 * k);
+        mma_bf16_ss(tmem, sdesc_k_sw128(a + 32 * k), db, idesc, (kb | k) != 0);
+        mma_bf16_ss(tmem, sdesc_k_sw128(a + PG_A_BYTES + 32 * k), db, idesc, 1);
+      }
+      mma_commit(smem_addr(&s_empty[s]));  // the stage is free once these MMAs have read it
+    }
+    mma_commit(smem_addr(&s_accum));  // the accumulator is complete (or, after a timeout, idle)
+  }
+  __syncwarp();
+
+  // ---- epilogue: warp w holds tokens t0 + 32 w + lane
+  const bool ready = __all_sync(0xffffffffu, mbar_wait(smem_addr(&s_accum), 0));
+  if (!ready && lane == 0) atomicOr(ep.err, ERR_TIMEOUT);
+  tc_fence_after();
+  const int t = t0 + warp * 32 + lane;
+  EpiState<MODE> st;
+  if (ready) {
+    for (int c = 0; c < PG_N / 32; ++c) {
+      const int n = n0 + 32 * c;
+      if (n >= ep.N) break;  // uniform across the warp
+      uint32_t r[32];
+      tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + 32 * c, r);
+      if (t < ep.T) epilogue32<MODE>(ep, t, n, r, st);
+    }
+    if constexpr (MODE == PE_ARGMAX) {
+      if (t < ep.T) {
+        ep.amax[(size_t)t * ep.n_tiles + blockIdx.y] = st.best;
+        ep.aidx[(size_t)t * ep.n_tiles + blockIdx.y] = st.bidx;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, PG_TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------------------- attention
+// Causal attention of a block of 64 prompt tokens (4 warps x 16) for one query head over the
+// user's cache rows [0, position]: S = Q K^T and O = P V on bf16 m16n8k16 MMAs, softmax online
+// over key blocks of 64 rows double-buffered in shared memory (rows padded by 16 bytes so the
+// matrix loads are free of bank conflicts).
+
+constexpr int PA_ROWS = 64;
+constexpr int PA_THREADS = 128;
+
+__device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3, uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr)
+               : "memory");
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3, uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr)
+               : "memory");
+}
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
+template <int HD>
+struct PaLayout {
+  static constexpr int ROW = (HD + 8) * 2;  // bytes per padded row
+  static constexpr int TILE = PA_ROWS * ROW;
+  static constexpr int Q_OFF = 0;
+  static constexpr int K_OFF = TILE;          // 2 buffers
+  static constexpr int V_OFF = 3 * TILE;      // 2 buffers
+  static constexpr int POS_OFF = 5 * TILE;    // int [64]
+  static constexpr int BYTES = POS_OFF + PA_ROWS * 4;
+};
+
+// Rows [r0, r0 + 64) of a [rows][HD] bf16 matrix (row stride ld elements) into a padded tile;
+// rows at or above `limit` are zero.
+template <int HD>
+__device__ __forceinline__ void pa_load_tile(uint8_t *tile, const uint16_t *src, size_t ld, int r0, int limit) {
+  constexpr int CH = HD / 8;
+  for (int e = threadIdx.x; e < PA_ROWS * CH; e += PA_THREADS) {
+    const int r = e / CH, ch = e % CH;
+    uint8_t *dst = tile + r * PaLayout<HD>::ROW + ch * 16;
+    if (r0 + r < limit)
+      cp_async16(smem_addr(dst), src + (size_t)(r0 + r) * ld + ch * 8);
+    else
+      *reinterpret_cast<uint4 *>(dst) = make_uint4(0, 0, 0, 0);
+  }
+}
+
+template <int HD>
+__global__ void __launch_bounds__(PA_THREADS) prefill_attn_kernel(PrefillAttnParams p) {
+  using L = PaLayout<HD>;
+  extern __shared__ __align__(16) uint8_t sm[];
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int g = lane / 4, c = lane % 4;
+  // the longest blocks (latest tokens) first
+  const int qb = gridDim.x - 1 - blockIdx.x;
+  const int h = blockIdx.y, kvh = h / (p.n_heads / p.n_kv_heads);
+  const int t0 = qb * PA_ROWS;
+  int *s_pos = reinterpret_cast<int *>(sm + L::POS_OFF);
+  if (threadIdx.x < PA_ROWS) s_pos[threadIdx.x] = t0 + threadIdx.x < p.T ? p.positions[t0 + threadIdx.x] : -1;
+  pa_load_tile<HD>(sm + L::Q_OFF, p.q + h * HD, p.ldq, t0, p.T);
+  cp_async_commit();
+  __syncthreads();
+  int max_pos = -1;
+  for (int i = 0; i < PA_ROWS; ++i) max_pos = max(max_pos, s_pos[i]);
+  const int n_kb = (max_pos + PA_ROWS) / PA_ROWS;  // key blocks covering [0, max_pos]
+  const int kv_limit = min(max_pos + 1, p.max_ctx);
+  const size_t head_base = ((size_t)p.slot * p.n_kv_heads + kvh) * p.max_ctx * HD;
+  const uint16_t *kg = p.kcache + head_base, *vg = p.vcache + head_base;
+  if (n_kb > 0) {
+    pa_load_tile<HD>(sm + L::K_OFF, kg, HD, 0, kv_limit);
+    pa_load_tile<HD>(sm + L::V_OFF, vg, HD, 0, kv_limit);
+  }
+  cp_async_commit();
+  const int qp0 = s_pos[16 * warp + g], qp1 = s_pos[16 * warp + g + 8];
+  cp_async_wait_all();
+  __syncthreads();
+  // Q fragments of this warp's 16 rows
+  uint32_t qf[HD / 16][4];
+  {
+    const uint32_t qbase = smem_addr(sm + L::Q_OFF) + (16 * warp + (lane % 16)) * L::ROW + (lane / 16) * 16;
+#pragma unroll
+    for (int kk = 0; kk < HD / 16; ++kk) ldsm_x4(qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3], qbase + kk * 32);
+  }
+  float oacc[HD / 8][4] = {};
+  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+  for (int kb = 0; kb < n_kb; ++kb) {
+    const int buf = kb & 1;
+    if (kb + 1 < n_kb) {  // the next block loads while this one is used
+      pa_load_tile<HD>(sm + L::K_OFF + (buf ^ 1) * L::TILE, kg, HD, (kb + 1) * PA_ROWS, kv_limit);
+      pa_load_tile<HD>(sm + L::V_OFF + (buf ^ 1) * L::TILE, vg, HD, (kb + 1) * PA_ROWS, kv_limit);
+    }
+    cp_async_commit();
+    const uint32_t kbase = smem_addr(sm + L::K_OFF + buf * L::TILE);
+    const uint32_t vbase = smem_addr(sm + L::V_OFF + buf * L::TILE);
+    // S = Q K^T: 8 key tiles of 8
+    float s[8][4];
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+      s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+#pragma unroll
+      for (int kk = 0; kk < HD / 16; kk += 2) {
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4(b0, b1, b2, b3, kbase + (nt * 8 + (lane % 8)) * L::ROW + kk * 32 + (lane / 8) * 16);
+        mma16816(s[nt], qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3], b0, b1);
+        mma16816(s[nt], qf[kk + 1][0], qf[kk + 1][1], qf[kk + 1][2], qf[kk + 1][3], b2, b3);
+      }
+    }
+    // scale, causal mask, online softmax (rows g and g + 8 of the warp)
+    float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+      const int kp = kb * PA_ROWS + nt * 8 + 2 * c;
+      s[nt][0] = kp <= qp0 ? s[nt][0] * p.scale_log2 : -INFINITY;
+      s[nt][1] = kp + 1 <= qp0 ? s[nt][1] * p.scale_log2 : -INFINITY;
+      s[nt][2] = kp <= qp1 ? s[nt][2] * p.scale_log2 : -INFINITY;
+      s[nt][3] = kp + 1 <= qp1 ? s[nt][3] * p.scale_log2 : -INFINITY;
+      mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]));
+      mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]));
+    }
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+    const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+    // rows with no visible key yet keep m = -inf; their factors stay 0 / 1
+    const float base0 = mn0 == -INFINITY ? 0.f : mn0, base1 = mn1 == -INFINITY ? 0.f : mn1;
+    const float corr0 = exp2f(m0 - base0), corr1 = exp2f(m1 - base1);
+    m0 = mn0;
+    m1 = mn1;
+    float rs0 = 0.f, rs1 = 0.f;
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+      s[nt][0] = exp2f(s[nt][0] - base0);
+      s[nt][1] = exp2f(s[nt][1] - base0);
+      s[nt][2] = exp2f(s[nt][2] - base1);
+      s[nt][3] = exp2f(s[nt][3] - base1);
+      rs0 += s[nt][0] + s[nt][1];
+      rs1 += s[nt][2] + s[nt][3];
+    }
+    l0 = l0 * corr0 + rs0;
+    l1 = l1 * corr1 + rs1;
+#pragma unroll
+    for (int dt = 0; dt < HD / 8; ++dt) {
+      oacc[dt][0] *= corr0;
+      oacc[dt][1] *= corr0;
+      oacc[dt][2] *= corr1;
+      oacc[dt][3] *= corr1;
+    }
+    // O += P V: 4 key steps of 16; V fragments by transposed matrix loads
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t a0 = pack_bf16(s[2 * j][0], s[2 * j][1]), a1 = pack_bf16(s[2 * j][2], s[2 * j][3]);
+      const uint32_t a2 = pack_bf16(s[2 * j + 1][0], s[2 * j + 1][1]), a3 = pack_bf16(s[2 * j + 1][2], s[2 * j + 1][3]);
+#pragma unroll
+      for (int dt = 0; dt < HD / 8; dt += 2) {
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4_t(b0, b1, b2, b3,
+                  vbase + (j * 16 + (lane % 8) + ((lane / 8) & 1) * 8) * L::ROW + (dt + lane / 16) * 16);
+        mma16816(oacc[dt], a0, a1, a2, a3, b0, b1);
+        mma16816(oacc[dt + 1], a0, a1, a2, a3, b2, b3);
+      }
+    }
+    cp_async_wait_all();
+    __syncthreads();
+  }
+  // row sums over the quad, normalize, store bf16
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+  const float inv0 = l0 > 0.f ? 1.f / l0 : 0.f, inv1 = l1 > 0.f ? 1.f / l1 : 0.f;
+  const int ta = t0 + 16 * warp + g, tb = ta + 8;
+#pragma unroll
+  for (int dt = 0; dt < HD / 8; ++dt) {
+    const int col = h * HD + dt * 8 + 2 * c;
+    uint32_t hi, lo;
+    if (ta < p.T) {
+      split_pack(oacc[dt][0] * inv0, oacc[dt][1] * inv0, hi, lo);
+      *reinterpret_cast<uint32_t *>(p.o + (size_t)ta * p.ldo + col) = hi;
+      *reinterpret_cast<uint32_t *>(p.o_lo + (size_t)ta * p.ldo + col) = lo;
+    }
+    if (tb < p.T) {
+      split_pack(oacc[dt][2] * inv1, oacc[dt][3] * inv1, hi, lo);
+      *reinterpret_cast<uint32_t *>(p.o + (size_t)tb * p.ldo + col) = hi;
+      *reinterpret_cast<uint32_t *>(p.o_lo + (size_t)tb * p.ldo + col) = lo;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------- small kernels
+// One block per prompt token: its input row (embedding row or given hidden state) and its
+// position, refused (-1, ERR_POSITION) outside [0, max_ctx) or when an earlier token of the pass
+// holds the same position.
+__global__ void prefill_input_kernel(const int *ids, const float *hidden_in, const int *positions_in, int T,
+                                     const uint16_t *embed, int vocab, int d, int ldh, float *h, int *positions,
+                                     int max_ctx, unsigned *err) {
+  const int t = blockIdx.x;
+  __shared__ int s_bad;
+  if (threadIdx.x == 0) s_bad = 0;
+  __syncthreads();
+  const int pos = positions_in[t];
+  for (int j = threadIdx.x; j < t; j += blockDim.x)
+    if (positions_in[j] == pos) s_bad = 1;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const bool ok = pos >= 0 && pos < max_ctx && !s_bad;
+    if (!ok) atomicOr(err, ERR_POSITION);
+    positions[t] = ok ? pos : -1;
+  }
+  int id = 0;
+  if (embed) {
+    id = ids[t];
+    if (id < 0 || id >= vocab) {
+      if (threadIdx.x == 0) atomicOr(err, ERR_TOKEN);
+      id = 0;
+    }
+  }
+  for (int i = threadIdx.x; i < d; i += blockDim.x)
+    h[(size_t)t * ldh + i] = embed ? bf16_to_f32(embed[(size_t)id * d + i]) : hidden_in[(size_t)t * d + i];
+}
+
+// x[t] = h[t] / rms(h[t]) * g as hi and lo bf16 terms, one block per token.
+__global__ void prefill_rmsnorm_kernel(const float *h, int ldh, int d, const float *g, float eps, uint16_t *x,
+                                       uint16_t *x_lo, int ldx) {
+  const int t = blockIdx.x;
+  const float *row = h + (size_t)t * ldh;
+  float ss = 0.f;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) ss += row[i] * row[i];
+  __shared__ float red[32];
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if (threadIdx.x % 32 == 0) red[threadIdx.x / 32] = ss;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    float v = threadIdx.x < blockDim.x / 32 ? red[threadIdx.x] : 0.f;
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if (threadIdx.x == 0) red[0] = v;
+  }
+  __syncthreads();
+  const float inv = rsqrtf(red[0] / d + eps);
+  for (int i = threadIdx.x; i < d; i += blockDim.x)
+    split_bf16(row[i] * inv * g[i], x[(size_t)t * ldx + i], x_lo[(size_t)t * ldx + i]);
+}
+
+// fp32 rows [T][K] (stride ldx) -> hi and lo bf16 terms (stride ld).
+__global__ void split_rows_kernel(const float *x, int K, int ldx, uint16_t *hi, uint16_t *lo, int ld) {
+  const int t = blockIdx.x;
+  for (int i = threadIdx.x; i < K; i += blockDim.x)
+    split_bf16(x[(size_t)t * ldx + i], hi[(size_t)t * ld + i], lo[(size_t)t * ld + i]);
+}
+
+// next_ids[t]: the lowest index among the largest logits, over the column tiles' partial maxima.
+__global__ void prefill_argmax_kernel(const float *amax, const int *aidx, int n_tiles, int T, int *next_ids) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= T) return;
+  float best = -INFINITY;
+  int bi = 0;
+  for (int j = 0; j < n_tiles; ++j) {
+    const float v = amax[(size_t)t * n_tiles + j];
+    if (v > best) {
+      best = v;
+      bi = aidx[(size_t)t * n_tiles + j];
+    }
+  }
+  next_ids[t] = bi;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    else
+      cudaGetLastError();
+  }
+  return fn;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------- host side
+// Activation rows [rows][K] bf16 at row stride ld (a multiple of 8): boxes of 64 columns x PG_M
+// rows; columns >= K and rows >= rows read as zero.
+int encode_act_map(CUtensorMap *map, const uint16_t *base, int K, int rows, int ld) {
+  auto fn = encode_fn();
+  if (!fn || ld % 8 != 0 || (reinterpret_cast<uintptr_t>(base) & 15) != 0) return -1;
+  const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+  const cuuint32_t box[2] = {PG_K, PG_M};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t *>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS
+             ? 0
+             : -1;
+}
+
+// Weight tiles [n_rb][n_kt][RB][KT] bf16 as a 4-D tensor (column, row, K tile, row block):
+// boxes of 64 columns x RB rows x 1 K tile x PG_N / RB row blocks; row blocks >= n_rb read as zero.
+int encode_tiles_map(CUtensorMap *map, const uint8_t *tiles, int n_kt, int n_rb) {
+  auto fn = encode_fn();
+  if (!fn) return -1;
+  const cuuint64_t dims[4] = {(cuuint64_t)KT, (cuuint64_t)RB, (cuuint64_t)n_kt, (cuuint64_t)n_rb};
+  const cuuint64_t strides[3] = {(cuuint64_t)KT * 2, (cuuint64_t)TILE_BYTES, (cuuint64_t)TILE_BYTES * n_kt};
+  const cuuint32_t box[4] = {PG_K, RB, 1, PG_N / RB};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<uint8_t *>(tiles), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS
+             ? 0
+             : -1;
+}
+
+template <int MODE>
+static cudaError_t launch_mode(const CUtensorMap &a, const CUtensorMap &a2, const CUtensorMap &b, int n_kt,
+                               const PrefillEpiParams &ep, cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(prefill_gemm_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)PG_SMEM);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  const dim3 grid((ep.T + PG_M - 1) / PG_M, (ep.N + PG_N - 1) / PG_N);
+  prefill_gemm_kernel<MODE><<<grid, PG_THREADS, PG_SMEM, s>>>(a, a2, b, 2 * n_kt, ep);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prefill_gemm(int mode, const CUtensorMap &a, const CUtensorMap &a2, const CUtensorMap &b,
+                                int n_kt, const PrefillEpiParams &ep, cudaStream_t s) {
+  if (ep.T <= 0 || ep.N <= 0) return cudaSuccess;
+  switch (mode) {
+    case PE_STORE: return launch_mode<PE_STORE>(a, a2, b, n_kt, ep, s);
+    case PE_RESID: return launch_mode<PE_RESID>(a, a2, b, n_kt, ep, s);
+    case PE_SWIGLU: return launch_mode<PE_SWIGLU>(a, a2, b, n_kt, ep, s);
+    case PE_QKV: return launch_mode<PE_QKV>(a, a2, b, n_kt, ep, s);
+    case PE_ARGMAX: return launch_mode<PE_ARGMAX>(a, a2, b, n_kt, ep, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+template <int HD>
+static cudaError_t launch_attn_hd(const PrefillAttnParams &p, cudaStream_t s) {
+  static bool attr = false;
+  const int bytes = PaLayout<HD>::BYTES;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(prefill_attn_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  const dim3 grid((p.T + PA_ROWS - 1) / PA_ROWS, p.n_heads);
+  prefill_attn_kernel<HD><<<grid, PA_THREADS, bytes, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prefill_attention(const PrefillAttnParams &p, int hd, cudaStream_t s) {
+  if (p.T <= 0) return cudaSuccess;
+  return hd == 128 ? launch_attn_hd<128>(p, s) : launch_attn_hd<64>(p, s);
+}
+
+cudaError_t launch_prefill_input(const int *ids, const float *hidden_in, const int *positions_in, int T,
+                                 const uint16_t *embed, int vocab, int d, int ldh, float *h, int *positions,
+                                 int max_ctx, unsigned *err, cudaStream_t s) {
+  prefill_input_kernel<<<T, 256, 0, s>>>(ids, hidden_in, positions_in, T, embed, vocab, d, ldh, h, positions,
+                                         max_ctx, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prefill_rmsnorm(const float *h, int ldh, int T, int d, const float *g, float eps, uint16_t *x,
+                                   uint16_t *x_lo, int ldx, cudaStream_t s) {
+  prefill_rmsnorm_kernel<<<T, 256, 0, s>>>(h, ldh, d, g, eps, x, x_lo, ldx);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_split_bf16(const float *x, int T, int K, int ldx, uint16_t *hi, uint16_t *lo, int ld,
+                              cudaStream_t s) {
+  split_rows_kernel<<<T, 256, 0, s>>>(x, K, ldx, hi, lo, ld);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prefill_argmax(const float *amax, const int *aidx, int n_tiles, int T, int *next_ids,
+                                  cudaStream_t s) {
+  prefill_argmax_kernel<<<(T + 127) / 128, 128, 0, s>>>(amax, aidx, n_tiles, T, next_ids);
+  return cudaGetLastError();
+}
+
+}  // namespace kfl
+
+// ---------------------------------------------------------------------------- C ABI
+extern "C" int kfl_matmul_bf16w(const float *x, int T, int K, int ldx, const uint16_t *w, int N, float *y, int ldy,
+                                void *cuda_stream) {
+  using namespace kfl;
+  if (!x || !w || !y || T < 1 || K < 1 || N < 1 || ldx < K || ldy < N || ldy % 4 != 0 ||
+      (reinterpret_cast<uintptr_t>(y) & 15) != 0)
+    return KFL_ERR_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  const int n_rb = (N + RB - 1) / RB, n_kt = (K + KT - 1) / KT, ld = (K + 63) / 64 * 64;
+  void *mem = nullptr;
+  const size_t tile_bytes = (size_t)n_rb * n_kt * TILE_BYTES, x_bytes = (size_t)T * ld * 2;
+  if (cudaMalloc(&mem, tile_bytes + 2 * x_bytes + 16) != cudaSuccess) {
+    cudaGetLastError();
+    return KFL_ERR_OOM;
+  }
+  uint8_t *tiles = static_cast<uint8_t *>(mem);
+  uint16_t *xhi = reinterpret_cast<uint16_t *>(tiles + tile_bytes);
+  uint16_t *xlo = xhi + (size_t)T * ld;
+  unsigned *err = reinterpret_cast<unsigned *>(xlo + (size_t)T * ld);
+  int rc = KFL_OK;
+  CUtensorMap mh, ml, mb;
+  if (cudaMemsetAsync(err, 0, 4, s) != cudaSuccess || launch_split_bf16(x, T, K, ldx, xhi, xlo, ld, s) != cudaSuccess ||
+      launch_repack_bf16(w, N, K, nullptr, N, n_rb, n_kt, tiles, s) != cudaSuccess) {
+    rc = KFL_ERR_CUDA;
+  } else if (encode_act_map(&mh, xhi, K, T, ld) || encode_act_map(&ml, xlo, K, T, ld) ||
+             encode_tiles_map(&mb, tiles, n_kt, n_rb)) {
+    rc = KFL_ERR_CUDA;
+  } else {
+    PrefillEpiParams e = {};
+    e.T = T;
+    e.N = N;
+    e.out = y;
+    e.ldo = ldy;
+    e.err = err;
+    unsigned h_err = 0;
+    if (launch_prefill_gemm(PE_STORE, mh, ml, mb, n_kt, e, s) != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess ||
+        cudaMemcpy(&h_err, err, 4, cudaMemcpyDeviceToHost) != cudaSuccess)
+      rc = KFL_ERR_CUDA;
+    else if (h_err & ERR_TIMEOUT)
+      rc = KFL_ERR_TIMEOUT;
+  }
+  cudaStreamSynchronize(s);
+  cudaFree(mem);
+  cudaGetLastError();
+  return rc;
+}

@@ -17,6 +17,7 @@
 #include "../../include/kafila_stage.h"
 #include "../../include/kafila_synth.h"
 #include "common.cuh"
+#include "prefill.cuh"
 
 using namespace kfl;
 
@@ -227,6 +228,17 @@ struct kfl_stage {
   std::vector<cudaEvent_t> ev;
   double prof_ms[KFL_KERNEL_KINDS] = {};
   int64_t prof_n[KFL_KERNEL_KINDS] = {};
+  // dense prefill (bf16 stages): the workspace of one pass of up to pf_cap tokens, allocated at
+  // the first dense prefill, and the tensor maps of the weight tiles (per layer: Q/K/V, O,
+  // gate/up, down; then lm_head)
+  int pf_cap = 0;
+  float *pf_h = nullptr;
+  uint16_t *pf_q = nullptr;
+  uint16_t *pf_x[2] = {}, *pf_o[2] = {}, *pf_a[2] = {};  // GEMM inputs as hi and lo bf16 terms
+  int *pf_pos = nullptr, *pf_aidx = nullptr;
+  float *pf_amax = nullptr;
+  std::vector<void *> pf_allocs;
+  std::vector<CUtensorMap> pf_maps;
   int magic = 0x4B464C53;
 
   int alloc(void **p, size_t bytes) {
@@ -670,6 +682,152 @@ int run_step(kfl_stage *st, const int32_t *ids, const float *hidden_in, const in
   return KFL_OK;
 }
 
+// ---- dense prefill (bf16 weights) ---------------------------------------------------------
+constexpr int PF_PASS = 2048;  // tokens per pass of the dense prefill
+
+int pf_ld(int n) { return round_up(n, 64); }
+
+// Workspace for passes of up to `tokens` tokens (grown, never shrunk) and the weight maps.
+int ensure_prefill(kfl_stage *st, int tokens) {
+  const Plan &P = st->P;
+  const int cap = std::min(PF_PASS, round_up(tokens, PG_M));
+  if (cap > st->pf_cap) {
+    for (void *p : st->pf_allocs) cudaFree(p);
+    st->pf_allocs.clear();
+    st->pf_cap = 0;
+    auto get = [&](void **p, size_t bytes) {
+      if (cudaMalloc(p, bytes) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+      }
+      st->pf_allocs.push_back(*p);
+      return true;
+    };
+    const int n_tiles = (P.V + PG_N - 1) / PG_N;
+    bool ok = get((void **)&st->pf_h, (size_t)cap * P.ldh * 4) && get((void **)&st->pf_q, (size_t)cap * pf_ld(P.qdim) * 2);
+    for (int j = 0; j < 2; ++j)
+      ok = ok && get((void **)&st->pf_x[j], (size_t)cap * pf_ld(P.d) * 2) &&
+           get((void **)&st->pf_o[j], (size_t)cap * pf_ld(P.qdim) * 2) &&
+           get((void **)&st->pf_a[j], (size_t)cap * pf_ld(P.F) * 2);
+    if (!ok || !get((void **)&st->pf_pos, (size_t)cap * 4) ||
+        !get((void **)&st->pf_amax, (size_t)cap * n_tiles * 4) ||
+        !get((void **)&st->pf_aidx, (size_t)cap * n_tiles * 4))
+      return KFL_ERR_OOM;
+    st->pf_cap = cap;
+  }
+  if (st->pf_maps.empty()) {
+    std::vector<CUtensorMap> maps(4 * P.nl + 1);
+    for (int l = 0; l < P.nl; ++l) {
+      const LayerDev &L = st->layers[l];
+      const Mat *m[4] = {&L.qkv, &L.o, &L.gu, &L.down};
+      for (int j = 0; j < 4; ++j)
+        if (encode_tiles_map(&maps[4 * l + j], m[j]->tiles, m[j]->n_kt, m[j]->n_rb)) return KFL_ERR_CUDA;
+    }
+    if ((st->flags & KFL_LOGITS_OUT) && encode_tiles_map(&maps[4 * P.nl], st->lm.tiles, st->lm.n_kt, st->lm.n_rb))
+      return KFL_ERR_CUDA;
+    st->pf_maps = std::move(maps);
+  }
+  return KFL_OK;
+}
+
+// The prompt in passes of up to pf_cap tokens.  Per pass and block: RMSNorm -> Q/K/V GEMM (RoPE,
+// K/V appended to the user's slot) -> causal attention over the slot -> O GEMM + residual ->
+// RMSNorm -> gate/up GEMM (SwiGLU) -> down GEMM + residual; the head: final RMSNorm -> lm_head GEMM
+// with the greedy argmax.
+int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in, const int32_t *positions, int user,
+                      int T, float *hidden_out, int32_t *next_ids, cudaStream_t s) {
+  const Plan &P = st->P;
+  int rc = ensure_prefill(st, T);
+  if (rc != KFL_OK) return rc;
+  const bool embed = (st->flags & KFL_EMBED_IN) != 0;
+  const int ldx = pf_ld(P.d), ldq = pf_ld(P.qdim), lda = pf_ld(P.F);
+  const float eps = st->cfg.rms_eps;
+  for (int t0 = 0; t0 < T; t0 += st->pf_cap) {
+    const int n = std::min(st->pf_cap, T - t0);
+    CK(launch_prefill_input(ids ? ids + t0 : nullptr, hidden_in ? hidden_in + (size_t)t0 * P.d : nullptr,
+                            positions + t0, n, embed ? st->embed : nullptr, P.V, P.d, P.ldh, st->pf_h, st->pf_pos,
+                            st->cfg.max_ctx, st->err, s));
+    CUtensorMap mx[2], mo[2], ma[2];
+    for (int j = 0; j < 2; ++j)
+      if (encode_act_map(&mx[j], st->pf_x[j], P.d, n, ldx) || encode_act_map(&mo[j], st->pf_o[j], P.qdim, n, ldq) ||
+          encode_act_map(&ma[j], st->pf_a[j], P.F, n, lda))
+        return KFL_ERR_CUDA;
+    for (int l = 0; l < P.nl; ++l) {
+      const LayerDev &L = st->layers[l];
+      uint16_t *kcl = st->kc + (size_t)l * P.kv_elems_per_layer;
+      uint16_t *vcl = st->vc + (size_t)l * P.kv_elems_per_layer;
+      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, L.g_attn, eps, st->pf_x[0], st->pf_x[1], ldx, s));
+      PrefillEpiParams e = {};
+      e.T = n;
+      e.err = st->err;
+      e.N = L.qkv.N;
+      e.out16 = st->pf_q;
+      e.ldo16 = ldq;
+      e.kcache = kcl;
+      e.vcache = vcl;
+      e.positions = st->pf_pos;
+      e.slot = user;
+      e.hd = P.hd;
+      e.hkv = P.hkv;
+      e.qdim = P.qdim;
+      e.kvdim = P.kvdim;
+      e.max_ctx = st->cfg.max_ctx;
+      e.rope_cos = st->rope_cos;
+      e.rope_sin = st->rope_sin;
+      CK(launch_prefill_gemm(PE_QKV, mx[0], mx[1], st->pf_maps[4 * l], L.qkv.n_kt, e, s));
+      PrefillAttnParams a = {};
+      a.q = st->pf_q;
+      a.ldq = ldq;
+      a.o = st->pf_o[0];
+      a.o_lo = st->pf_o[1];
+      a.ldo = ldq;
+      a.kcache = kcl;
+      a.vcache = vcl;
+      a.positions = st->pf_pos;
+      a.slot = user;
+      a.T = n;
+      a.n_heads = P.hq;
+      a.n_kv_heads = P.hkv;
+      a.max_ctx = st->cfg.max_ctx;
+      a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)P.hd));
+      CK(launch_prefill_attention(a, P.hd, s));
+      PrefillEpiParams r = {};
+      r.T = n;
+      r.err = st->err;
+      r.N = P.d;
+      r.out = st->pf_h;
+      r.ldo = P.ldh;
+      CK(launch_prefill_gemm(PE_RESID, mo[0], mo[1], st->pf_maps[4 * l + 1], L.o.n_kt, r, s));
+      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, L.g_ffn, eps, st->pf_x[0], st->pf_x[1], ldx, s));
+      PrefillEpiParams g = {};
+      g.T = n;
+      g.err = st->err;
+      g.N = 2 * P.F;
+      g.out16 = st->pf_a[0];
+      g.out16lo = st->pf_a[1];
+      g.ldo16 = lda;
+      CK(launch_prefill_gemm(PE_SWIGLU, mx[0], mx[1], st->pf_maps[4 * l + 2], L.gu.n_kt, g, s));
+      CK(launch_prefill_gemm(PE_RESID, ma[0], ma[1], st->pf_maps[4 * l + 3], L.down.n_kt, r, s));
+    }
+    if (st->flags & KFL_LOGITS_OUT) {
+      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, st->g_final, eps, st->pf_x[0], st->pf_x[1], ldx, s));
+      PrefillEpiParams z = {};
+      z.T = n;
+      z.err = st->err;
+      z.N = P.V;
+      z.amax = st->pf_amax;
+      z.aidx = st->pf_aidx;
+      z.n_tiles = (P.V + PG_N - 1) / PG_N;
+      CK(launch_prefill_gemm(PE_ARGMAX, mx[0], mx[1], st->pf_maps[4 * P.nl], st->lm.n_kt, z, s));
+      CK(launch_prefill_argmax(st->pf_amax, st->pf_aidx, z.n_tiles, n, next_ids + t0, s));
+    }
+    if (hidden_out)
+      CK(cudaMemcpy2DAsync(hidden_out + (size_t)t0 * P.d, (size_t)P.d * 4, st->pf_h, (size_t)P.ldh * 4,
+                           (size_t)P.d * 4, n, cudaMemcpyDeviceToDevice, s));
+  }
+  return KFL_OK;
+}
+
 // host or device source -> device pointer (a temporary copy for host sources)
 int to_device(kfl_stage *st, const void *src, size_t bytes, int on_device, void **out, std::vector<void *> &tmp) {
   if (on_device) {
@@ -1061,9 +1219,12 @@ extern "C" int kfl_stage_prefill(kfl_stage *st, const int32_t *token_ids, const 
   if (!st->loaded()) return KFL_ERR_STATE;
   CK(cudaSetDevice(st->dev));
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  // bf16 weights: the dense path from KFL_PREFILL_DENSE_MIN tokens on (default 16)
+  if (st->cfg.weight_fmt == KFL_BF16 && n_tokens >= env_int("KFL_PREFILL_DENSE_MIN", 16))
+    return run_prefill_dense(st, token_ids, hidden_in, positions, user, n_tokens, hidden_out, next_ids, s);
   const int d = st->P.d;
-  // the prompt in chunks of max_batch consecutive tokens: each chunk is one step whose rows all
-  // address the user's KV slot, so a token attends to the chunk's earlier tokens too
+  // else the prompt in chunks of max_batch consecutive tokens: each chunk is one decode step whose
+  // rows all address the user's KV slot, so a token attends to the chunk's earlier tokens too
   for (int t0 = 0; t0 < n_tokens; t0 += st->cfg.max_batch) {
     const int n = std::min(st->cfg.max_batch, n_tokens - t0);
     const int rc = run_step(st, token_ids ? token_ids + t0 : nullptr, hidden_in ? hidden_in + (size_t)t0 * d : nullptr,
@@ -1252,6 +1413,7 @@ extern "C" void kfl_stage_destroy(kfl_stage *st) {
   for (cudaEvent_t e : st->ev) cudaEventDestroy(e);
   if (st->cap_stream) cudaStreamDestroy(st->cap_stream);
   for (void *p : st->allocs) cudaFree(p);
+  for (void *p : st->pf_allocs) cudaFree(p);
   cudaGetLastError();
   st->magic = 0;
   delete st;

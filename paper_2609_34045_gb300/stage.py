@@ -85,6 +85,7 @@ def lib() -> C.CDLL:
             "kfl_stage_decode_host": ([vp, vp, vp, vp, i, vp, vp, vp], i),
             "kfl_stage_decode_users": ([vp, vp, vp, vp, vp, i, vp, vp, vp], i),
             "kfl_stage_prefill": ([vp, vp, vp, vp, i, i, vp, vp, vp], i),
+            "kfl_matmul_bf16w": ([vp, i, i, i, vp, i, vp, i, vp], i),
             "kfl_kv_reset": ([vp, i], i),
             "kfl_kv_fill_seeded": ([vp, i, i, C.c_uint64], i),
             "kfl_kv_write": ([vp, i, i, vp, vp, i, i], i),
@@ -243,6 +244,12 @@ def kfl_stage_prefill(st: Stage, token_ids, hidden_in, positions, user: int, n_t
     hidden_out [n][d], int32 next_ids [n] (CUDA tensors).  Asynchronous."""
     _check(lib().kfl_stage_prefill(st.handle, _ptr(token_ids), _ptr(hidden_in), _ptr(positions), user, n_tokens,
                                    _ptr(hidden_out), _ptr(next_ids), cuda_stream), "kfl_stage_prefill")
+
+
+def kfl_matmul_bf16w(x, T: int, K_: int, ldx: int, w, N: int, y, ldy: int, cuda_stream: int | None = None) -> None:
+    """y[T][N] (fp32, row stride ldy) = x[T][K] (fp32, row stride ldx) times w[N][K]^T (bf16 bits)
+    on the tensor cores: the prefill's matrix product on its own.  CUDA tensors; synchronous."""
+    _check(lib().kfl_matmul_bf16w(_ptr(x), T, K_, ldx, _ptr(w), N, _ptr(y), ldy, cuda_stream), "kfl_matmul_bf16w")
 
 
 def kfl_stage_decode_host(st: Stage, token_ids, hidden_in, positions, batch: int, hidden_out, next_ids,

@@ -1,7 +1,8 @@
 """GPU parity of the prompt prefill (kfl_stage_prefill) against the oracle's prefill.
 
-A prompt of one user goes through the stage as steps of up to max_batch rows on the user's KV
-slot; the oracle runs the whole prompt in one pass (causal attention over the prompt).  Bar as
+A prompt of one user goes through the stage either as steps of up to max_batch rows on the user's
+KV slot (the decode kernels) or, for bf16 weights, densely (tensor-core matrix products over all
+its tokens, causal attention over the slot); the oracle runs the whole prompt in one pass.  Bar as
 for decode: every token's output within max-abs 1e-2 of the oracle's RMS, greedy ids equal where
 the oracle's top-2 margin exceeds 1e-2, the user's written cache rows within tolerance and every
 other row of every slot bit-identical.
@@ -57,27 +58,53 @@ def _prefill(pair, user, start, n, seed, embed):
     return o
 
 
-# (model, stage layers, flags, contexts of users 0..2, prefilled user, tokens): prompts that end
-# mid-step (11 = 4 + 4 + 3), fill whole steps, are one token, cross the 64-position sub-tiles and
-# start from an empty cache
+@pytest.fixture(params=["steps", "dense"])
+def path(request, monkeypatch):
+    """Which prefill path a bf16 stage takes: the decode steps or the dense one."""
+    monkeypatch.setenv("KFL_PREFILL_DENSE_MIN", "1" if request.param == "dense" else str(1 << 30))
+    return request.param
+
+
+# (model, stage layers, flags, contexts of users 0..2, prefilled user, tokens, max_ctx): prompts
+# that end mid-step (11 = 4 + 4 + 3), fill whole steps, are one token, cross the 64-position
+# sub-tiles and the dense path's 128-token tiles, start from an empty cache, and (2100 tokens)
+# take two dense passes
 CASES = [
-    ("bf16-head-ragged", RAGGED, 0, 3, K.KFL_IS_HEAD, (5, 130, 58), 2, 11),
-    ("bf16-body-hidden", RAGGED, 1, 3, 0, (17, 40, 61), 1, 8),
-    ("bf16-one-token", RAGGED, 0, 2, K.KFL_IS_HEAD, (3, 9, 20), 0, 1),
-    ("hd128-empty-cache", RAGGED128, 0, 2, K.KFL_IS_HEAD, (0, 100, 7), 0, 9),
-    ("int4-head", RAGGED_INT4, 0, 2, K.KFL_IS_HEAD, (9, 70, 131), 1, 7),
+    ("bf16-head-ragged", RAGGED, 0, 3, K.KFL_IS_HEAD, (5, 130, 58), 2, 11, 192),
+    ("bf16-body-hidden", RAGGED, 1, 3, 0, (17, 40, 61), 1, 8, 192),
+    ("bf16-one-token", RAGGED, 0, 2, K.KFL_IS_HEAD, (3, 9, 20), 0, 1, 192),
+    ("hd128-empty-cache", RAGGED128, 0, 2, K.KFL_IS_HEAD, (0, 100, 7), 0, 9, 192),
+    ("bf16-head-300", RAGGED, 0, 3, K.KFL_IS_HEAD, (5, 30, 70), 2, 300, 448),
+    ("hd128-200", RAGGED128, 0, 2, K.KFL_IS_HEAD, (0, 100, 7), 1, 200, 320),
+    ("int4-head", RAGGED_INT4, 0, 2, K.KFL_IS_HEAD, (9, 70, 131), 1, 7, 192),
 ]
 
 
-@pytest.mark.parametrize("name,model,l0,l1,flags,contexts,user,n", CASES, ids=[c[0] for c in CASES])
-def test_prefill_matches_the_oracle(name, model, l0, l1, flags, contexts, user, n):
-    p = Pair(model, l0, l1, flags, 3, contexts, 192, seed=23, max_batch=4)
+@pytest.mark.parametrize("name,model,l0,l1,flags,contexts,user,n,max_ctx", CASES, ids=[c[0] for c in CASES])
+def test_prefill_matches_the_oracle(name, model, l0, l1, flags, contexts, user, n, max_ctx, path):
+    if path == "dense" and model.weight_fmt != "bf16":
+        pytest.skip("the dense prefill takes bf16 weights; int4 stages prefill in steps")
+    if path == "steps" and n > 64:
+        pytest.skip("long prompts: the dense path only (the steps path is covered by the short ones)")
+    p = Pair(model, l0, l1, flags, 3, contexts, max_ctx, seed=23, max_batch=4)
     _prefill(p, user, contexts[user], n, 23, bool(flags & K.KFL_EMBED_IN))
     p.compare_kv()
     p.close()
 
 
-def test_decode_after_prefill_matches_the_oracle():
+def test_two_dense_passes(monkeypatch):
+    """A prompt longer than one dense pass (2048 tokens): the second pass attends to the first's
+    cache rows."""
+    monkeypatch.setenv("KFL_PREFILL_DENSE_MIN", "1")
+    small = wl.ModelShape(n_layers_total=1, d_model=128, n_heads=2, n_kv_heads=1, head_dim=64, ffn=256,
+                          vocab=300)
+    p = Pair(small, 0, 1, K.KFL_IS_HEAD, 1, (40,), 2176, seed=37, max_batch=1)
+    _prefill(p, 0, 40, 2100, 37, True)
+    p.compare_kv()
+    p.close()
+
+
+def test_decode_after_prefill_matches_the_oracle(path):
     """Prefill user 1's prompt, then decode all three users; user 1 continues after its prompt."""
     model, contexts, n = RAGGED, (20, 33, 64), 6
     p = Pair(model, 0, 3, K.KFL_IS_HEAD, 3, contexts, 192, seed=29, max_batch=4)
@@ -91,7 +118,7 @@ def test_decode_after_prefill_matches_the_oracle():
     p.close()
 
 
-def test_repeated_position_is_reported():
+def test_repeated_position_is_reported(path):
     """Two tokens of one user at the same position in one step: the later one is refused on the
     device (status KFL_ERR_RANGE) and the stage stays usable."""
     p = Pair(RAGGED, 0, 1, K.KFL_IS_HEAD, 2, (5, 6), 64, seed=31, max_batch=4)
