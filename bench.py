@@ -48,6 +48,14 @@ def parse():
     ap.add_argument("--prefill", action="store_true",
                     help="time to first token of one user on the 7B-shaped model as one head stage: the "
                          "prompt's prefill (steps of 4 of its tokens) plus the first decode step")
+    ap.add_argument("--prompt-lengths", default="128,512,2048",
+                    help="--prefill: prompt lengths (comma-separated)")
+    ap.add_argument("--prefill-gens", type=int, default=5,
+                    help="--prefill: generations per case (the first is discarded)")
+    ap.add_argument("--prefill-dense-only", action="store_true",
+                    help="--prefill: skip the decode-step comparisons (for launch lists)")
+    ap.add_argument("--prefill-layers", type=int, default=0,
+                    help="--prefill: the head stage holds only the first N blocks (small case for profiling)")
     ap.add_argument("--layers", type=int, default=0,
                     help="small case for profiling: the first N blocks of the stage as a body stage "
                          "(no embedding, no head, no splits)")
@@ -671,15 +679,17 @@ def run_prefill(args):
     from paper_2609_34045_gb300 import stage as K
     from paper_2609_34045_gb300 import workload as wl
 
-    lengths = (128, 512, 2048)
+    lengths = tuple(int(x) for x in args.prompt_lengths.split(","))
+    gens = max(2, args.prefill_gens)
     base = wl.CONFIGS[2]
     m = base.model
-    work = dataclasses.replace(base, name="7B-head-28L-prefill", l0=0, l1=m.n_layers_total, embed_in=True,
+    nl = args.prefill_layers if 0 < args.prefill_layers < m.n_layers_total else m.n_layers_total
+    work = dataclasses.replace(base, name=f"7B-head-{nl}L-prefill", l0=0, l1=nl, embed_in=True,
                                logits_out=True, batch=4, contexts=(0, 0, 0, 0), steps=max(lengths) + 64,
                                splits=())
     torch.cuda.set_device(0)
     cfg = K.model_cfg(m, work.max_ctx, 4)
-    st = K.kfl_stage_create(cfg, 0, m.n_layers_total, K.KFL_IS_HEAD)
+    st = K.kfl_stage_create(cfg, 0, nl, K.KFL_IS_HEAD)
     di.load_stage_seeded(st, work)
     stream = torch.cuda.current_stream()
     sp = stream.cuda_stream
@@ -694,8 +704,8 @@ def run_prefill(args):
         tok = torch.zeros(1, dtype=torch.int32, device="cuda")
         first = torch.zeros(1, dtype=torch.int32, device="cuda")
         pos_n = torch.tensor([n], dtype=torch.int32, device="cuda")
-        gens = []
-        for g in range(5):
+        times = []
+        for g in range(gens):
             torch.cuda.synchronize()
             ev[0].record(stream)
             K.kfl_stage_prefill(st, ids, None, pos, 0, n, None, nxt, sp)
@@ -704,32 +714,40 @@ def run_prefill(args):
             K.kfl_stage_decode_users(st, tok, None, pos_n, user, 1, None, first, sp)
             ev[2].record(stream)
             torch.cuda.synchronize()
-            gens.append((ev[0].elapsed_time(ev[1]), ev[1].elapsed_time(ev[2])))
-        pre = statistics.median(x[0] for x in gens[1:])
-        dec = statistics.median(x[1] for x in gens[1:])
+            times.append((ev[0].elapsed_time(ev[1]), ev[1].elapsed_time(ev[2])))
+        pre = statistics.median(x[0] for x in times[1:])
+        dec = statistics.median(x[1] for x in times[1:])
         # the weight products only (attention's products excluded)
-        flops = 2.0 * n * (m.n_layers_total * sum(r * c for r, c in m.matrix_shapes().values()) + m.vocab * m.d_model)
+        flops = 2.0 * n * (nl * sum(r * c for r, c in m.matrix_shapes().values()) + m.vocab * m.d_model)
         return {"prefill_ms": pre, "decode_ms": dec, "ttft_ms": pre + dec, "prefill_tokens_per_s": n / pre * 1e3,
                 "matmul_tflops": flops / pre / 1e9}
 
     rows = {n: ttft(n, True) for n in lengths}
-    steps512 = ttft(512, False)
     os.environ.pop("KFL_PREFILL_DENSE_MIN", None)
-    # one token per step, the 512-token prompt
-    n = 512
+    if args.prefill_dense_only:
+        K.kfl_stage_destroy(st)
+        print(json.dumps({"metric": "time to first token", "unit": "ms", "higher_is_better": False, "n_gpus": 1,
+                          "config": {"workload": work.name, "users": 1, "weights": "bf16",
+                                     "prompt_lengths": list(lengths)},
+                          "dense_by_prompt_length": {str(k): v for k, v in rows.items()}}), flush=True)
+        return 0
+    n = 512 if 512 in lengths else lengths[0]
+    steps512 = ttft(n, False)
+    os.environ.pop("KFL_PREFILL_DENSE_MIN", None)
+    # one token per step
     ids = torch.tensor(wl.token_ids(work.seed, 90, n, m.vocab), dtype=torch.int32, device="cuda")
     pos = torch.arange(n, dtype=torch.int32, device="cuda")
     first = torch.zeros(1, dtype=torch.int32, device="cuda")
-    gens = []
-    for g in range(3):
+    times = []
+    for g in range(min(gens, 3)):
         torch.cuda.synchronize()
         ev[0].record(stream)
         for t in range(n):
             K.kfl_stage_decode_users(st, ids[t:t + 1], None, pos[t:t + 1], user, 1, None, first, sp)
         ev[1].record(stream)
         torch.cuda.synchronize()
-        gens.append(ev[0].elapsed_time(ev[1]))
-    one = statistics.median(gens[1:])
+        times.append(ev[0].elapsed_time(ev[1]))
+    one = statistics.median(times[1:])
     if K.kfl_stage_status(st) != 0:
         raise RuntimeError("device reported an error during the prefill runs")
     K.kfl_stage_destroy(st)
@@ -737,9 +755,9 @@ def run_prefill(args):
             "config": {"workload": work.name, "users": 1, "weights": "bf16",
                        "prompt_lengths": list(lengths)},
             "dense_by_prompt_length": {str(k): v for k, v in rows.items()},
-            "steps_of_4_512": steps512,
-            "one_token_per_step_512": {"prefill_ms": one, "prefill_tokens_per_s": n / one * 1e3},
-            "data": "synthetic (seeded)", "protocol": "5 generations, first discarded, median",
+            f"steps_of_4_{n}": steps512,
+            f"one_token_per_step_{n}": {"prefill_ms": one, "prefill_tokens_per_s": n / one * 1e3},
+            "data": "synthetic (seeded)", "protocol": f"{gens} generations, first discarded, median",
             "timing": "CUDA events on the launching stream"}
     print(json.dumps(line), flush=True)
     return 0
