@@ -183,20 +183,35 @@ __device__ __forceinline__ void epilogue32(const PrefillEpiParams &ep, int t, in
       const bool is_q = n < ep.qdim;
       const int r0 = is_q ? n : n - ep.qdim;
       const int head = r0 / ep.hd, i0 = (r0 % ep.hd) / 2;
-      const float *cs = ep.rope_cos + (size_t)pos * half + i0;
-      const float *sn = ep.rope_sin + (size_t)pos * half + i0;
+      // the 16 factors of each kind are 64 contiguous, 64-byte aligned bytes
+      const float4 *cs = reinterpret_cast<const float4 *>(ep.rope_cos + (size_t)pos * half + i0);
+      const float4 *sn = reinterpret_cast<const float4 *>(ep.rope_sin + (size_t)pos * half + i0);
+      float c[16], sv[16];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float4 a = cs[j], b = sn[j];
+        c[4 * j] = a.x, c[4 * j + 1] = a.y, c[4 * j + 2] = a.z, c[4 * j + 3] = a.w;
+        sv[4 * j] = b.x, sv[4 * j + 1] = b.y, sv[4 * j + 2] = b.z, sv[4 * j + 3] = b.w;
+      }
       uint16_t *dst;
       if (is_q) {
         dst = ep.out16 + (size_t)t * ep.ldo16 + (size_t)head * ep.hd;
       } else {
         dst = ep.kcache + (((size_t)ep.slot * ep.hkv + head) * ep.max_ctx + pos) * ep.hd;
       }
+      // rotated first halves -> dst[i0 ..], second halves -> dst[i0 + hd/2 ..]: 32 bytes each
+      uint32_t w1[8], w2[8];
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const float x1 = v[2 * i], x2 = v[2 * i + 1], c = cs[i], s = sn[i];
-        dst[i0 + i] = f32_to_bf16_rne(x1 * c - x2 * s);
-        dst[i0 + i + half] = f32_to_bf16_rne(x2 * c + x1 * s);
+      for (int i = 0; i < 16; i += 2) {
+        const float a1 = v[2 * i], a2 = v[2 * i + 1], b1 = v[2 * i + 2], b2 = v[2 * i + 3];
+        w1[i / 2] = pack_bf16(a1 * c[i] - a2 * sv[i], b1 * c[i + 1] - b2 * sv[i + 1]);
+        w2[i / 2] = pack_bf16(a2 * c[i] + a1 * sv[i], b2 * c[i + 1] + b1 * sv[i + 1]);
       }
+      uint4 *d1 = reinterpret_cast<uint4 *>(dst + i0), *d2 = reinterpret_cast<uint4 *>(dst + i0 + half);
+      d1[0] = make_uint4(w1[0], w1[1], w1[2], w1[3]);
+      d1[1] = make_uint4(w1[4], w1[5], w1[6], w1[7]);
+      d2[0] = make_uint4(w2[0], w2[1], w2[2], w2[3]);
+      d2[1] = make_uint4(w2[4], w2[5], w2[6], w2[7]);
     } else {
       const int r0 = n - ep.qdim - ep.kvdim;
       const int head = r0 / ep.hd, j0 = r0 % ep.hd;
@@ -227,6 +242,10 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
   __shared__ uint32_t s_tmem;
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int t0 = blockIdx.x * PG_M, n0 = blockIdx.y * PG_N;
+  // split-K: split blockIdx.z of ep.splits takes K blocks [kb0, kb1)
+  const int kb0 = (int)((long long)blockIdx.z * n_kblocks / ep.splits);
+  const int kb1 = (int)((long long)(blockIdx.z + 1) * n_kblocks / ep.splits);
+  const int nkb = kb1 - kb0;
   // the swizzled tiles start on a 1024-byte boundary
   const uint32_t raw = smem_addr(smem_raw);
   const uint32_t sa = (raw + 1023u) & ~1023u;      // [stage][hi, lo] activation tiles
@@ -251,9 +270,9 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
     // ---- TMA producer
     int issued[PG_STAGES] = {};
     bool ok = true;
-    for (int kb = 0; kb < n_kblocks; ++kb) {
-      const int s = kb % PG_STAGES;
-      const uint32_t use = kb / PG_STAGES;
+    for (int j = 0; j < nkb; ++j) {
+      const int s = j % PG_STAGES, kb = kb0 + j;
+      const uint32_t use = j / PG_STAGES;
       if (use > 0 && !mbar_wait(smem_addr(&s_empty[s]), (use - 1) & 1)) {
         ok = false;
         break;
@@ -275,9 +294,9 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
   } else if (threadIdx.x == 32) {
     // ---- MMA issuer
     constexpr uint32_t idesc = idesc_bf16_f32(PG_M, PG_N);
-    for (int kb = 0; kb < n_kblocks; ++kb) {
-      const int s = kb % PG_STAGES;
-      if (!mbar_wait(smem_addr(&s_full[s]), (kb / PG_STAGES) & 1)) {
+    for (int j = 0; j < nkb; ++j) {
+      const int s = j % PG_STAGES;
+      if (!mbar_wait(smem_addr(&s_full[s]), (j / PG_STAGES) & 1)) {
         atomicOr(ep.err, ERR_TIMEOUT);
         break;
       }
@@ -286,7 +305,7 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
 #pragma unroll
       for (int k = 0; k < PG_K / 16; ++k) {
         const uint64_t db = sdesc_k_sw128(b + 32 * k);
-        mma_bf16_ss(tmem, sdesc_k_sw128(a + 32 * k), db, idesc, (kb | k) != 0);
+        mma_bf16_ss(tmem, sdesc_k_sw128(a + 32 * k), db, idesc, (j | k) != 0);
         mma_bf16_ss(tmem, sdesc_k_sw128(a + PG_A_BYTES + 32 * k), db, idesc, 1);
       }
       mma_commit(smem_addr(&s_empty[s]));  // the stage is free once these MMAs have read it
@@ -296,12 +315,64 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
   __syncwarp();
 
   // ---- epilogue: warp w holds tokens t0 + 32 w + lane
-  const bool ready = __all_sync(0xffffffffu, mbar_wait(smem_addr(&s_accum), 0));
-  if (!ready && lane == 0) atomicOr(ep.err, ERR_TIMEOUT);
+  // block-uniform: the split path synchronises the whole block
+  const bool ready = __syncthreads_and(mbar_wait(smem_addr(&s_accum), 0)) != 0;
+  if (!ready && threadIdx.x == 0) atomicOr(ep.err, ERR_TIMEOUT);
   tc_fence_after();
-  const int t = t0 + warp * 32 + lane;
+  const int row = warp * 32 + lane, t = t0 + row;
   EpiState<MODE> st;
-  if (ready) {
+  if (ep.splits > 1) {
+    // split-K over a cluster of S = ep.splits CTAs (rank = blockIdx.z).  Column chunk c (32
+    // columns) of the tile belongs to rank c / (8 / S).  Every CTA pushes each chunk of its fp32
+    // accumulator into the owner's shared memory (posted remote stores; the pipeline buffers are
+    // idle now), at [own rank][row][chunk within the owner's share]; after the cluster barrier
+    // each owner sums its chunks over the ranks in rank order (deterministic) from its own shared
+    // memory and runs the epilogue.  The first barrier keeps a CTA from writing into a peer whose
+    // pipeline still uses that memory.  Both barriers are reached by every CTA, whatever its
+    // pipeline did.
+    const int S = ep.splits, per = (PG_N / 32) / S, ld = per * 32 + 4;
+    float *red = reinterpret_cast<float *>(smem_raw + (sa - raw));  // [S][PG_M][ld]
+    cluster_sync_all();
+    if (ready) {
+      for (int c = 0; c < PG_N / 32; ++c) {
+        if (n0 + 32 * c >= ep.N) break;
+        uint32_t r[32];
+        tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + 32 * c, r);
+        const int owner = c / per;
+        const uint32_t dst = map_to_rank(smem_addr(red + ((size_t)blockIdx.z * PG_M + row) * ld + (c % per) * 32),
+                                         owner);
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          st_cluster_f4(dst + 16 * j, make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                                                  __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3])));
+      }
+    }
+    cluster_sync_all();
+    if (ready) {
+      for (int cc = 0; cc < per; ++cc) {
+        const int n = n0 + 32 * (blockIdx.z * per + cc);
+        if (n >= ep.N) break;
+        float acc[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) acc[j] = 0.f;
+        for (int q = 0; q < S; ++q) {
+          const float4 *src = reinterpret_cast<const float4 *>(red + ((size_t)q * PG_M + row) * ld + cc * 32);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float4 v4 = src[j];
+            acc[4 * j] += v4.x;
+            acc[4 * j + 1] += v4.y;
+            acc[4 * j + 2] += v4.z;
+            acc[4 * j + 3] += v4.w;
+          }
+        }
+        uint32_t r[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(acc[j]);
+        if (t < ep.T) epilogue32<MODE>(ep, t, n, r, st);
+      }
+    }
+  } else if (ready) {
     for (int c = 0; c < PG_N / 32; ++c) {
       const int n = n0 + 32 * c;
       if (n >= ep.N) break;  // uniform across the warp
@@ -309,6 +380,8 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
       tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + 32 * c, r);
       if (t < ep.T) epilogue32<MODE>(ep, t, n, r, st);
     }
+  }
+  if (ready) {
     if constexpr (MODE == PE_ARGMAX) {
       if (t < ep.T) {
         ep.amax[(size_t)t * ep.n_tiles + blockIdx.y] = st.best;
@@ -657,21 +730,66 @@ int encode_tiles_map(CUtensorMap *map, const uint8_t *tiles, int n_kt, int n_rb)
 template <int MODE>
 static cudaError_t launch_mode(const CUtensorMap &a, const CUtensorMap &a2, const CUtensorMap &b, int n_kt,
                                const PrefillEpiParams &ep, cudaStream_t s) {
-  static bool attr = false;
-  if (!attr) {
+  static bool smem_set = false;
+  if (!smem_set) {
     cudaError_t e = cudaFuncSetAttribute(prefill_gemm_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)PG_SMEM);
     if (e != cudaSuccess) return e;
-    attr = true;
+    smem_set = true;
   }
-  const dim3 grid((ep.T + PG_M - 1) / PG_M, (ep.N + PG_N - 1) / PG_N);
-  prefill_gemm_kernel<MODE><<<grid, PG_THREADS, PG_SMEM, s>>>(a, a2, b, 2 * n_kt, ep);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(PG_THREADS);
+  cfg.dynamicSmemBytes = PG_SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  // the largest split count not above the chosen one whose cluster fits on the device
+  static int fits[9] = {};  // 0 unknown, 1 yes, -1 no
+  PrefillEpiParams e = ep;
+  while (e.splits > 1) {
+    if (fits[e.splits] == 0) {
+      attr[0].val.clusterDim.z = e.splits;
+      cfg.gridDim = dim3(1, 1, e.splits);
+      int n = 0;
+      fits[e.splits] = cudaOccupancyMaxActiveClusters(&n, prefill_gemm_kernel<MODE>, &cfg) == cudaSuccess && n > 0 ? 1 : -1;
+      cudaGetLastError();
+    }
+    if (fits[e.splits] > 0) break;
+    e.splits /= 2;
+  }
+  attr[0].val.clusterDim.z = e.splits;
+  cfg.gridDim = dim3((e.T + PG_M - 1) / PG_M, (e.N + PG_N - 1) / PG_N, e.splits);
+  return cudaLaunchKernelEx(&cfg, prefill_gemm_kernel<MODE>, a, a2, b, 2 * n_kt, e);
+}
+
+int prefill_splits(int T, int N, int n_kt, int n_sm) {
+  const long long base = (long long)((T + PG_M - 1) / PG_M) * ((N + PG_N - 1) / PG_N);
+  const int n_kb = 2 * n_kt;
+  // waves x (K blocks per split + a fixed cost per CTA of about 6 K blocks: pipeline fill and
+  // epilogue; 1.5 more for the cluster reduction), over the split counts 1, 2, 4, 8 that keep
+  // at least 4 K blocks each
+  int best = 1;
+  double best_t = 1e30;
+  for (int S = 1; S <= 8 && n_kb / S >= 4; S *= 2) {
+    const double waves = (double)((base * S + n_sm - 1) / n_sm);
+    const double t = waves * ((double)n_kb / S + 6.0 + (S > 1 ? 1.5 : 0.0));
+    if (t < best_t - 1e-9) {
+      best_t = t;
+      best = S;
+    }
+  }
+  return best;
 }
 
 cudaError_t launch_prefill_gemm(int mode, const CUtensorMap &a, const CUtensorMap &a2, const CUtensorMap &b,
                                 int n_kt, const PrefillEpiParams &ep, cudaStream_t s) {
   if (ep.T <= 0 || ep.N <= 0) return cudaSuccess;
+  if (ep.splits != 1 && ep.splits != 2 && ep.splits != 4 && ep.splits != 8) return cudaErrorInvalidValue;
+  if (mode == PE_ARGMAX && ep.splits != 1) return cudaErrorInvalidValue;  // partial maxima are per tile
   switch (mode) {
     case PE_STORE: return launch_mode<PE_STORE>(a, a2, b, n_kt, ep, s);
     case PE_RESID: return launch_mode<PE_RESID>(a, a2, b, n_kt, ep, s);
@@ -738,6 +856,12 @@ extern "C" int kfl_matmul_bf16w(const float *x, int T, int K, int ldx, const uin
     return KFL_ERR_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   const int n_rb = (N + RB - 1) / RB, n_kt = (K + KT - 1) / KT, ld = (K + 63) / 64 * 64;
+  int dev = 0, n_sm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+    cudaGetLastError();
+    return KFL_ERR_CUDA;
+  }
+  const int splits = prefill_splits(T, N, n_kt, n_sm);
   void *mem = nullptr;
   const size_t tile_bytes = (size_t)n_rb * n_kt * TILE_BYTES, x_bytes = (size_t)T * ld * 2;
   if (cudaMalloc(&mem, tile_bytes + 2 * x_bytes + 16) != cudaSuccess) {
@@ -750,7 +874,8 @@ extern "C" int kfl_matmul_bf16w(const float *x, int T, int K, int ldx, const uin
   unsigned *err = reinterpret_cast<unsigned *>(xlo + (size_t)T * ld);
   int rc = KFL_OK;
   CUtensorMap mh, ml, mb;
-  if (cudaMemsetAsync(err, 0, 4, s) != cudaSuccess || launch_split_bf16(x, T, K, ldx, xhi, xlo, ld, s) != cudaSuccess ||
+  if (cudaMemsetAsync(err, 0, 4, s) != cudaSuccess ||
+      launch_split_bf16(x, T, K, ldx, xhi, xlo, ld, s) != cudaSuccess ||
       launch_repack_bf16(w, N, K, nullptr, N, n_rb, n_kt, tiles, s) != cudaSuccess) {
     rc = KFL_ERR_CUDA;
   } else if (encode_act_map(&mh, xhi, K, T, ld) || encode_act_map(&ml, xlo, K, T, ld) ||
@@ -763,6 +888,7 @@ extern "C" int kfl_matmul_bf16w(const float *x, int T, int K, int ldx, const uin
     e.out = y;
     e.ldo = ldy;
     e.err = err;
+    e.splits = splits;
     unsigned h_err = 0;
     if (launch_prefill_gemm(PE_STORE, mh, ml, mb, n_kt, e, s) != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess ||
         cudaMemcpy(&h_err, err, 4, cudaMemcpyDeviceToHost) != cudaSuccess)

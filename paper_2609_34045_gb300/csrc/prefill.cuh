@@ -55,6 +55,9 @@ struct PrefillEpiParams {
   float *amax;
   int *aidx;
   int n_tiles;
+  // split-K: 1, 2, 4 or 8 CTAs per output tile, launched as a cluster that reduces through
+  // distributed shared memory (PE_ARGMAX: 1)
+  int splits;
   unsigned *err;           // ERR_TIMEOUT if a pipeline wait gave up
 };
 
@@ -72,6 +75,9 @@ struct PrefillAttnParams {
 // Host side (prefill.cu).
 int encode_act_map(CUtensorMap *map, const uint16_t *base, int K, int rows, int ld);
 int encode_tiles_map(CUtensorMap *map, const uint8_t *tiles, int n_kt, int n_rb);
+// Splits of K (1, 2, 4 or 8) for a GEMM of T tokens x N rows (n_kt K tiles) on n_sm SMs: the
+// count that minimises an estimate of waves x work per CTA.
+int prefill_splits(int T, int N, int n_kt, int n_sm);
 cudaError_t launch_prefill_gemm(int mode, const CUtensorMap &a_hi, const CUtensorMap &a_lo, const CUtensorMap &b,
                                 int n_kt, const PrefillEpiParams &ep, cudaStream_t s);
 cudaError_t launch_prefill_attention(const PrefillAttnParams &p, int hd, cudaStream_t s);

@@ -730,6 +730,13 @@ int ensure_prefill(kfl_stage *st, int tokens) {
   return KFL_OK;
 }
 
+// One prefill GEMM with the split count chosen for its shape.
+cudaError_t pf_gemm(kfl_stage *st, int mode, const CUtensorMap &a, const CUtensorMap &a2, const CUtensorMap &b,
+                    int n_kt, PrefillEpiParams e, cudaStream_t s) {
+  e.splits = mode == PE_ARGMAX ? 1 : prefill_splits(e.T, e.N, n_kt, st->P.n_sm);
+  return launch_prefill_gemm(mode, a, a2, b, n_kt, e, s);
+}
+
 // The prompt in passes of up to pf_cap tokens.  Per pass and block: RMSNorm -> Q/K/V GEMM (RoPE,
 // K/V appended to the user's slot) -> causal attention over the slot -> O GEMM + residual ->
 // RMSNorm -> gate/up GEMM (SwiGLU) -> down GEMM + residual; the head: final RMSNorm -> lm_head GEMM
@@ -774,7 +781,7 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
       e.max_ctx = st->cfg.max_ctx;
       e.rope_cos = st->rope_cos;
       e.rope_sin = st->rope_sin;
-      CK(launch_prefill_gemm(PE_QKV, mx[0], mx[1], st->pf_maps[4 * l], L.qkv.n_kt, e, s));
+      CK(pf_gemm(st, PE_QKV, mx[0], mx[1], st->pf_maps[4 * l], L.qkv.n_kt, e, s));
       PrefillAttnParams a = {};
       a.q = st->pf_q;
       a.ldq = ldq;
@@ -797,7 +804,7 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
       r.N = P.d;
       r.out = st->pf_h;
       r.ldo = P.ldh;
-      CK(launch_prefill_gemm(PE_RESID, mo[0], mo[1], st->pf_maps[4 * l + 1], L.o.n_kt, r, s));
+      CK(pf_gemm(st, PE_RESID, mo[0], mo[1], st->pf_maps[4 * l + 1], L.o.n_kt, r, s));
       CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, L.g_ffn, eps, st->pf_x[0], st->pf_x[1], ldx, s));
       PrefillEpiParams g = {};
       g.T = n;
@@ -806,8 +813,8 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
       g.out16 = st->pf_a[0];
       g.out16lo = st->pf_a[1];
       g.ldo16 = lda;
-      CK(launch_prefill_gemm(PE_SWIGLU, mx[0], mx[1], st->pf_maps[4 * l + 2], L.gu.n_kt, g, s));
-      CK(launch_prefill_gemm(PE_RESID, ma[0], ma[1], st->pf_maps[4 * l + 3], L.down.n_kt, r, s));
+      CK(pf_gemm(st, PE_SWIGLU, mx[0], mx[1], st->pf_maps[4 * l + 2], L.gu.n_kt, g, s));
+      CK(pf_gemm(st, PE_RESID, ma[0], ma[1], st->pf_maps[4 * l + 3], L.down.n_kt, r, s));
     }
     if (st->flags & KFL_LOGITS_OUT) {
       CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, st->g_final, eps, st->pf_x[0], st->pf_x[1], ldx, s));
@@ -818,7 +825,7 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
       z.amax = st->pf_amax;
       z.aidx = st->pf_aidx;
       z.n_tiles = (P.V + PG_N - 1) / PG_N;
-      CK(launch_prefill_gemm(PE_ARGMAX, mx[0], mx[1], st->pf_maps[4 * P.nl], st->lm.n_kt, z, s));
+      CK(pf_gemm(st, PE_ARGMAX, mx[0], mx[1], st->pf_maps[4 * P.nl], st->lm.n_kt, z, s));
       CK(launch_prefill_argmax(st->pf_amax, st->pf_aidx, z.n_tiles, n, next_ids + t0, s));
     }
     if (hidden_out)
