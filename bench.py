@@ -54,6 +54,9 @@ def parse():
                     help="--prefill: generations per case (the first is discarded)")
     ap.add_argument("--prefill-dense-only", action="store_true",
                     help="--prefill: skip the decode-step comparisons (for launch lists)")
+    ap.add_argument("--prefill-config", type=int, default=2, choices=[2, 5],
+                    help="--prefill: the model of this workload as one whole-model head stage "
+                         "(2: 7B-shaped bf16, 5: 72B-shaped int4)")
     ap.add_argument("--prefill-layers", type=int, default=0,
                     help="--prefill: the head stage holds only the first N blocks (small case for profiling)")
     ap.add_argument("--layers", type=int, default=0,
@@ -681,10 +684,11 @@ def run_prefill(args):
 
     lengths = tuple(int(x) for x in args.prompt_lengths.split(","))
     gens = max(2, args.prefill_gens)
-    base = wl.CONFIGS[2]
+    base = wl.CONFIGS[args.prefill_config]
     m = base.model
     nl = args.prefill_layers if 0 < args.prefill_layers < m.n_layers_total else m.n_layers_total
-    work = dataclasses.replace(base, name=f"7B-head-{nl}L-prefill", l0=0, l1=nl, embed_in=True,
+    shape = "7B" if args.prefill_config == 2 else "72B-int4"
+    work = dataclasses.replace(base, name=f"{shape}-head-{nl}L-prefill", l0=0, l1=nl, embed_in=True,
                                logits_out=True, batch=4, contexts=(0, 0, 0, 0), steps=max(lengths) + 64,
                                splits=())
     torch.cuda.set_device(0)
@@ -727,7 +731,7 @@ def run_prefill(args):
     if args.prefill_dense_only:
         K.kfl_stage_destroy(st)
         print(json.dumps({"metric": "time to first token", "unit": "ms", "higher_is_better": False, "n_gpus": 1,
-                          "config": {"workload": work.name, "users": 1, "weights": "bf16",
+                          "config": {"workload": work.name, "users": 1, "weights": m.weight_fmt,
                                      "prompt_lengths": list(lengths)},
                           "dense_by_prompt_length": {str(k): v for k, v in rows.items()}}), flush=True)
         return 0
@@ -752,7 +756,7 @@ def run_prefill(args):
         raise RuntimeError("device reported an error during the prefill runs")
     K.kfl_stage_destroy(st)
     line = {"metric": "time to first token", "unit": "ms", "higher_is_better": False, "n_gpus": 1,
-            "config": {"workload": work.name, "users": 1, "weights": "bf16",
+            "config": {"workload": work.name, "users": 1, "weights": m.weight_fmt,
                        "prompt_lengths": list(lengths)},
             "dense_by_prompt_length": {str(k): v for k, v in rows.items()},
             f"steps_of_4_{n}": steps512,

@@ -44,10 +44,12 @@ __device__ __forceinline__ uint64_t sdesc_k_sw128(uint32_t addr) {
   return d;
 }
 
-// Instruction descriptor of kind::f16: fp32 accumulator (bits 4-5 = 1), A and B bf16 (bits 7-9
-// and 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 in bits 17-22, M >> 4 in bits 24-28.
-__host__ __device__ constexpr uint32_t idesc_bf16_f32(int m, int n) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+// Instruction descriptor of kind::f16: fp32 accumulator (bits 4-5 = 1), A and B both bf16 (bits
+// 7-9 and 10-12 = 1) or both fp16 (0), both K-major (bits 15, 16 = 0), N >> 3 in bits 17-22,
+// M >> 4 in bits 24-28.
+__host__ __device__ constexpr uint32_t idesc_kind_f16(int m, int n, bool bf16) {
+  return (1u << 4) | ((bf16 ? 1u : 0u) << 7) | ((bf16 ? 1u : 0u) << 10) | ((uint32_t)(n >> 3) << 17) |
+         ((uint32_t)(m >> 4) << 24);
 }
 
 __device__ __forceinline__ void mma_bf16_ss(uint32_t d_tmem, uint64_t da, uint64_t db, uint32_t idesc,
@@ -106,11 +108,22 @@ __device__ __forceinline__ void split_bf16(float x, uint16_t &hi, uint16_t &lo) 
   hi = f32_to_bf16_rne(x);
   lo = f32_to_bf16_rne(x - bf16_to_f32(hi));
 }
+// The same with fp16 terms (about 2^-22 relative left; |x| must stay below 65504).
+__device__ __forceinline__ void split_f16(float x, uint16_t &hi, uint16_t &lo) {
+  hi = f32_to_f16_rn(x);
+  lo = f32_to_f16_rn(x - f16_to_f32(hi));
+}
+__device__ __forceinline__ void split_term(float x, uint16_t &hi, uint16_t &lo, int f16) {
+  if (f16)
+    split_f16(x, hi, lo);
+  else
+    split_bf16(x, hi, lo);
+}
 // Two values as packed pairs of their hi and lo terms.
-__device__ __forceinline__ void split_pack(float x0, float x1, uint32_t &hi, uint32_t &lo) {
+__device__ __forceinline__ void split_pack(float x0, float x1, uint32_t &hi, uint32_t &lo, int f16 = 0) {
   uint16_t h0, l0, h1, l1;
-  split_bf16(x0, h0, l0);
-  split_bf16(x1, h1, l1);
+  split_term(x0, h0, l0, f16);
+  split_term(x1, h1, l1, f16);
   hi = (uint32_t)h0 | ((uint32_t)h1 << 16);
   lo = (uint32_t)l0 | ((uint32_t)l1 << 16);
 }
@@ -157,7 +170,7 @@ __device__ __forceinline__ void epilogue32(const PrefillEpiParams &ep, int t, in
 #pragma unroll
     for (int i = 0; i < 16; i += 2) {
       const float g0 = v[2 * i], u0 = v[2 * i + 1], g1 = v[2 * i + 2], u1 = v[2 * i + 3];
-      split_pack(g0 / (1.0f + expf(-g0)) * u0, g1 / (1.0f + expf(-g1)) * u1, w[i / 2], wl[i / 2]);
+      split_pack(g0 / (1.0f + expf(-g0)) * u0, g1 / (1.0f + expf(-g1)) * u1, w[i / 2], wl[i / 2], ep.f16);
     }
     uint16_t *row = ep.out16 + (size_t)t * ep.ldo16 + j0;
     uint16_t *rlo = ep.out16lo + (size_t)t * ep.ldo16 + j0;
@@ -293,7 +306,8 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
     }
   } else if (threadIdx.x == 32) {
     // ---- MMA issuer
-    constexpr uint32_t idesc = idesc_bf16_f32(PG_M, PG_N);
+    // A and B always share one type: both bf16, or (int4 stages) both fp16
+    const uint32_t idesc = ep.f16 ? idesc_kind_f16(PG_M, PG_N, false) : idesc_kind_f16(PG_M, PG_N, true);
     for (int j = 0; j < nkb; ++j) {
       const int s = j % PG_STAGES;
       if (!mbar_wait(smem_addr(&s_full[s]), (j / PG_STAGES) & 1)) {
@@ -588,12 +602,12 @@ __global__ void __launch_bounds__(PA_THREADS) prefill_attn_kernel(PrefillAttnPar
     const int col = h * HD + dt * 8 + 2 * c;
     uint32_t hi, lo;
     if (ta < p.T) {
-      split_pack(oacc[dt][0] * inv0, oacc[dt][1] * inv0, hi, lo);
+      split_pack(oacc[dt][0] * inv0, oacc[dt][1] * inv0, hi, lo, p.f16);
       *reinterpret_cast<uint32_t *>(p.o + (size_t)ta * p.ldo + col) = hi;
       *reinterpret_cast<uint32_t *>(p.o_lo + (size_t)ta * p.ldo + col) = lo;
     }
     if (tb < p.T) {
-      split_pack(oacc[dt][2] * inv1, oacc[dt][3] * inv1, hi, lo);
+      split_pack(oacc[dt][2] * inv1, oacc[dt][3] * inv1, hi, lo, p.f16);
       *reinterpret_cast<uint32_t *>(p.o + (size_t)tb * p.ldo + col) = hi;
       *reinterpret_cast<uint32_t *>(p.o_lo + (size_t)tb * p.ldo + col) = lo;
     }
@@ -634,7 +648,7 @@ __global__ void prefill_input_kernel(const int *ids, const float *hidden_in, con
 
 // x[t] = h[t] / rms(h[t]) * g as hi and lo bf16 terms, one block per token.
 __global__ void prefill_rmsnorm_kernel(const float *h, int ldh, int d, const float *g, float eps, uint16_t *x,
-                                       uint16_t *x_lo, int ldx) {
+                                       uint16_t *x_lo, int ldx, int f16) {
   const int t = blockIdx.x;
   const float *row = h + (size_t)t * ldh;
   float ss = 0.f;
@@ -651,7 +665,45 @@ __global__ void prefill_rmsnorm_kernel(const float *h, int ldh, int d, const flo
   __syncthreads();
   const float inv = rsqrtf(red[0] / d + eps);
   for (int i = threadIdx.x; i < d; i += blockDim.x)
-    split_bf16(row[i] * inv * g[i], x[(size_t)t * ldx + i], x_lo[(size_t)t * ldx + i]);
+    split_term(row[i] * inv * g[i], x[(size_t)t * ldx + i], x_lo[(size_t)t * ldx + i], f16);
+}
+
+// One thread per 8 consecutive outputs of one row (16 bytes): the int4 tile stores the nibble of
+// (row rb*64 + r16*16 + gid + 8 ((i >> 1) & 1), column kt*256 + 128 h + 16 (4 q + j) + 2 tig +
+// 8 (i & 1) + ((i >> 2) & 1)) as nibble i of word j + 4 lane + 128 q + 256 r16 + 1024 h
+// (lane = 4 gid + tig), and the row's group scales after the codes; so the 8 columns
+// 16 m + 8 e .. + 7 of a row come from lanes tig = 0..3, nibbles i with i & 1 = e.
+__global__ void dequant_int4_f16_kernel(const uint8_t *tiles4, int n_rb, int n_kt, uint16_t *dst) {
+  const long long total = (long long)n_rb * n_kt * RB * (KT4 / 8);
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int c8 = (int)(e % (KT4 / 8));      // 8-column chunk within the int4 tile (0..31)
+    const long long rt = e / (KT4 / 8);
+    const int r = (int)(rt % RB);              // row within the row block
+    const long long t = rt / RB;               // int4 tile index rb * n_kt + kt
+    const int col0 = c8 * 8;                   // 0..248
+    const int h = col0 >> 7, m = (col0 >> 4) & 7, ebit = (col0 >> 3) & 1;
+    const int q = m >> 2, j = m & 3, r16 = r >> 4, gid = r & 7, rhalf = (r >> 3) & 1;
+    const uint8_t *tile = tiles4 + (size_t)t * TILE4_BYTES;
+    const uint32_t *words = reinterpret_cast<const uint32_t *>(tile);
+    const float sc = bf16_to_f32(reinterpret_cast<const uint16_t *>(tile + TILE4_CODE_BYTES)[r * (KT4 / 64) + (col0 >> 6)]);
+    uint16_t out[8];
+#pragma unroll
+    for (int tig = 0; tig < 4; ++tig) {
+      const uint32_t w = words[j + 4 * (4 * gid + tig) + 128 * q + 256 * r16 + 1024 * h];
+#pragma unroll
+      for (int b = 0; b < 2; ++b) {
+        const int i = ebit | (rhalf << 1) | (b << 2);
+        const int nib = (int)((w >> (4 * i)) & 0xFu);
+        out[2 * tig + b] = f32_to_f16_rn((float)(nib >= 8 ? nib - 16 : nib) * sc);
+      }
+    }
+    // fp16 tile (rb, 2 kt + h): row r, columns (col0 & 127) ..
+    const long long rb = t / n_kt, kt = t % n_kt;
+    uint16_t *d = dst + ((size_t)(rb * 2 * n_kt + 2 * kt + h) * RB + r) * KT + (col0 & 127);
+    *reinterpret_cast<uint4 *>(d) = make_uint4(out[0] | (uint32_t)out[1] << 16, out[2] | (uint32_t)out[3] << 16,
+                                               out[4] | (uint32_t)out[5] << 16, out[6] | (uint32_t)out[7] << 16);
+  }
 }
 
 // fp32 rows [T][K] (stride ldx) -> hi and lo bf16 terms (stride ld).
@@ -828,8 +880,13 @@ cudaError_t launch_prefill_input(const int *ids, const float *hidden_in, const i
 }
 
 cudaError_t launch_prefill_rmsnorm(const float *h, int ldh, int T, int d, const float *g, float eps, uint16_t *x,
-                                   uint16_t *x_lo, int ldx, cudaStream_t s) {
-  prefill_rmsnorm_kernel<<<T, 256, 0, s>>>(h, ldh, d, g, eps, x, x_lo, ldx);
+                                   uint16_t *x_lo, int ldx, int f16, cudaStream_t s) {
+  prefill_rmsnorm_kernel<<<T, 256, 0, s>>>(h, ldh, d, g, eps, x, x_lo, ldx, f16);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dequant_int4_f16(const uint8_t *tiles4, int n_rb, int n_kt, uint16_t *dst, cudaStream_t s) {
+  dequant_int4_f16_kernel<<<8 * 152, 256, 0, s>>>(tiles4, n_rb, n_kt, dst);
   return cudaGetLastError();
 }
 

@@ -39,6 +39,7 @@ enum PrefillEpi : int {
 
 struct PrefillEpiParams {
   int T, N;                // valid tokens and columns
+  int f16;                 // operands are fp16 (int4 stages: weights dequantized to fp16), else bf16
   float *out;              // PE_STORE / PE_RESID: fp32 [T][ldo]
   int ldo;
   uint16_t *out16;         // PE_SWIGLU: hi term, bf16 [T][ldo16] (N / 2 columns); PE_QKV: q, bf16 [T][ldo16]
@@ -64,8 +65,8 @@ struct PrefillEpiParams {
 struct PrefillAttnParams {
   const uint16_t *q;       // [T][ldq] bf16, RoPE applied, heads in natural order
   int ldq;
-  uint16_t *o, *o_lo;      // [T][ldo] bf16: the output as hi and lo terms
-  int ldo;
+  uint16_t *o, *o_lo;      // [T][ldo]: the output as hi and lo terms (fp16 if f16, else bf16)
+  int ldo, f16;
   const uint16_t *kcache, *vcache;  // this layer's [max_batch][Hkv][max_ctx][hd]
   const int *positions;    // [T], -1: refused (output 0)
   int slot, T, n_heads, n_kv_heads, max_ctx;
@@ -85,7 +86,9 @@ cudaError_t launch_prefill_input(const int *ids, const float *hidden_in, const i
                                  const uint16_t *embed, int vocab, int d, int ldh, float *h, int *positions,
                                  int max_ctx, unsigned *err, cudaStream_t s);
 cudaError_t launch_prefill_rmsnorm(const float *h, int ldh, int T, int d, const float *g, float eps, uint16_t *x,
-                                   uint16_t *x_lo, int ldx, cudaStream_t s);
+                                   uint16_t *x_lo, int ldx, int f16, cudaStream_t s);
+// int4 group-64 tiles [n_rb][n_kt][TILE4_BYTES] -> fp16 tiles [n_rb][2 n_kt][RB][KT] of code x scale.
+cudaError_t launch_dequant_int4_f16(const uint8_t *tiles4, int n_rb, int n_kt, uint16_t *dst, cudaStream_t s);
 cudaError_t launch_split_bf16(const float *x, int T, int K, int ldx, uint16_t *hi, uint16_t *lo, int ld,
                               cudaStream_t s);
 cudaError_t launch_prefill_argmax(const float *amax, const int *aidx, int n_tiles, int T, int *next_ids,

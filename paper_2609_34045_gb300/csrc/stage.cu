@@ -238,7 +238,11 @@ struct kfl_stage {
   int *pf_pos = nullptr, *pf_aidx = nullptr;
   float *pf_amax = nullptr;
   std::vector<void *> pf_allocs;
+  // bf16 stages: the maps of every layer's weight tiles [4 l + j] (Q/K/V, O, gate/up, down), then
+  // lm_head.  int4 stages: one map per matrix kind [j] (then lm_head) over pf_w16, the fp16 tiles
+  // of the matrix being multiplied (dequantized just before its GEMM)
   std::vector<CUtensorMap> pf_maps;
+  uint16_t *pf_w16 = nullptr;
   int magic = 0x4B464C53;
 
   int alloc(void **p, size_t bytes) {
@@ -715,6 +719,24 @@ int ensure_prefill(kfl_stage *st, int tokens) {
       return KFL_ERR_OOM;
     st->pf_cap = cap;
   }
+  if (st->pf_maps.empty() && st->cfg.weight_fmt == KFL_INT4_G64) {
+    // the fp16 scratch holds the largest matrix; its maps are per matrix kind
+    const Mat *kinds[5] = {&P.qkv, &P.o, &P.gu, &P.down, &P.lm};
+    const int n_kinds = (st->flags & KFL_LOGITS_OUT) ? 5 : 4;
+    size_t most = 0;
+    for (int j = 0; j < n_kinds; ++j) most = std::max(most, (size_t)kinds[j]->n_rb * 2 * kinds[j]->n_kt * TILE_BYTES);
+    if (cudaMalloc((void **)&st->pf_w16, most) != cudaSuccess) {
+      cudaGetLastError();
+      st->pf_w16 = nullptr;
+      return KFL_ERR_OOM;
+    }
+    std::vector<CUtensorMap> maps(5);
+    for (int j = 0; j < n_kinds; ++j)
+      if (encode_tiles_map(&maps[j], reinterpret_cast<const uint8_t *>(st->pf_w16), 2 * kinds[j]->n_kt,
+                           kinds[j]->n_rb))
+        return KFL_ERR_CUDA;
+    st->pf_maps = std::move(maps);
+  }
   if (st->pf_maps.empty()) {
     std::vector<CUtensorMap> maps(4 * P.nl + 1);
     for (int l = 0; l < P.nl; ++l) {
@@ -730,11 +752,26 @@ int ensure_prefill(kfl_stage *st, int tokens) {
   return KFL_OK;
 }
 
-// One prefill GEMM with the split count chosen for its shape.
-cudaError_t pf_gemm(kfl_stage *st, int mode, const CUtensorMap &a, const CUtensorMap &a2, const CUtensorMap &b,
-                    int n_kt, PrefillEpiParams e, cudaStream_t s) {
+// One prefill GEMM with matrix j of block l (j = 4: lm_head) and the split count chosen for its
+// shape.  int4 stages first dequantize the matrix into the fp16 scratch.
+cudaError_t pf_gemm(kfl_stage *st, int mode, const CUtensorMap &a, const CUtensorMap &a2, int l, int j,
+                    PrefillEpiParams e, cudaStream_t s) {
+  const Mat &m = j == 4 ? st->lm
+                        : (j == 0 ? st->layers[l].qkv : j == 1 ? st->layers[l].o : j == 2 ? st->layers[l].gu : st->layers[l].down);
+  const bool i4 = st->cfg.weight_fmt == KFL_INT4_G64;
+  int n_kt = m.n_kt;
+  const CUtensorMap *b;
+  if (i4) {
+    cudaError_t err = launch_dequant_int4_f16(m.tiles, m.n_rb, m.n_kt, st->pf_w16, s);
+    if (err != cudaSuccess) return err;
+    b = &st->pf_maps[j];
+    n_kt = 2 * m.n_kt;  // K tiles of 128 fp16
+  } else {
+    b = &st->pf_maps[j == 4 ? 4 * st->P.nl : 4 * l + j];
+  }
+  e.f16 = i4 ? 1 : 0;
   e.splits = mode == PE_ARGMAX ? 1 : prefill_splits(e.T, e.N, n_kt, st->P.n_sm);
-  return launch_prefill_gemm(mode, a, a2, b, n_kt, e, s);
+  return launch_prefill_gemm(mode, a, a2, *b, n_kt, e, s);
 }
 
 // The prompt in passes of up to pf_cap tokens.  Per pass and block: RMSNorm -> Q/K/V GEMM (RoPE,
@@ -747,6 +784,7 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
   int rc = ensure_prefill(st, T);
   if (rc != KFL_OK) return rc;
   const bool embed = (st->flags & KFL_EMBED_IN) != 0;
+  const int i4 = st->cfg.weight_fmt == KFL_INT4_G64 ? 1 : 0;
   const int ldx = pf_ld(P.d), ldq = pf_ld(P.qdim), lda = pf_ld(P.F);
   const float eps = st->cfg.rms_eps;
   for (int t0 = 0; t0 < T; t0 += st->pf_cap) {
@@ -763,7 +801,7 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
       const LayerDev &L = st->layers[l];
       uint16_t *kcl = st->kc + (size_t)l * P.kv_elems_per_layer;
       uint16_t *vcl = st->vc + (size_t)l * P.kv_elems_per_layer;
-      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, L.g_attn, eps, st->pf_x[0], st->pf_x[1], ldx, s));
+      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, L.g_attn, eps, st->pf_x[0], st->pf_x[1], ldx, i4, s));
       PrefillEpiParams e = {};
       e.T = n;
       e.err = st->err;
@@ -781,13 +819,14 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
       e.max_ctx = st->cfg.max_ctx;
       e.rope_cos = st->rope_cos;
       e.rope_sin = st->rope_sin;
-      CK(pf_gemm(st, PE_QKV, mx[0], mx[1], st->pf_maps[4 * l], L.qkv.n_kt, e, s));
+      CK(pf_gemm(st, PE_QKV, mx[0], mx[1], l, 0, e, s));
       PrefillAttnParams a = {};
       a.q = st->pf_q;
       a.ldq = ldq;
       a.o = st->pf_o[0];
       a.o_lo = st->pf_o[1];
       a.ldo = ldq;
+      a.f16 = i4;
       a.kcache = kcl;
       a.vcache = vcl;
       a.positions = st->pf_pos;
@@ -804,8 +843,8 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
       r.N = P.d;
       r.out = st->pf_h;
       r.ldo = P.ldh;
-      CK(pf_gemm(st, PE_RESID, mo[0], mo[1], st->pf_maps[4 * l + 1], L.o.n_kt, r, s));
-      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, L.g_ffn, eps, st->pf_x[0], st->pf_x[1], ldx, s));
+      CK(pf_gemm(st, PE_RESID, mo[0], mo[1], l, 1, r, s));
+      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, L.g_ffn, eps, st->pf_x[0], st->pf_x[1], ldx, i4, s));
       PrefillEpiParams g = {};
       g.T = n;
       g.err = st->err;
@@ -813,11 +852,11 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
       g.out16 = st->pf_a[0];
       g.out16lo = st->pf_a[1];
       g.ldo16 = lda;
-      CK(pf_gemm(st, PE_SWIGLU, mx[0], mx[1], st->pf_maps[4 * l + 2], L.gu.n_kt, g, s));
-      CK(pf_gemm(st, PE_RESID, ma[0], ma[1], st->pf_maps[4 * l + 3], L.down.n_kt, r, s));
+      CK(pf_gemm(st, PE_SWIGLU, mx[0], mx[1], l, 2, g, s));
+      CK(pf_gemm(st, PE_RESID, ma[0], ma[1], l, 3, r, s));
     }
     if (st->flags & KFL_LOGITS_OUT) {
-      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, st->g_final, eps, st->pf_x[0], st->pf_x[1], ldx, s));
+      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, st->g_final, eps, st->pf_x[0], st->pf_x[1], ldx, i4, s));
       PrefillEpiParams z = {};
       z.T = n;
       z.err = st->err;
@@ -825,7 +864,7 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
       z.amax = st->pf_amax;
       z.aidx = st->pf_aidx;
       z.n_tiles = (P.V + PG_N - 1) / PG_N;
-      CK(pf_gemm(st, PE_ARGMAX, mx[0], mx[1], st->pf_maps[4 * P.nl], st->lm.n_kt, z, s));
+      CK(pf_gemm(st, PE_ARGMAX, mx[0], mx[1], -1, 4, z, s));
       CK(launch_prefill_argmax(st->pf_amax, st->pf_aidx, z.n_tiles, n, next_ids + t0, s));
     }
     if (hidden_out)
@@ -1226,8 +1265,8 @@ extern "C" int kfl_stage_prefill(kfl_stage *st, const int32_t *token_ids, const 
   if (!st->loaded()) return KFL_ERR_STATE;
   CK(cudaSetDevice(st->dev));
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
-  // bf16 weights: the dense path from KFL_PREFILL_DENSE_MIN tokens on (default 16)
-  if (st->cfg.weight_fmt == KFL_BF16 && n_tokens >= env_int("KFL_PREFILL_DENSE_MIN", 16))
+  // the dense path from KFL_PREFILL_DENSE_MIN tokens on (default 16)
+  if (n_tokens >= env_int("KFL_PREFILL_DENSE_MIN", 16))
     return run_prefill_dense(st, token_ids, hidden_in, positions, user, n_tokens, hidden_out, next_ids, s);
   const int d = st->P.d;
   // else the prompt in chunks of max_batch consecutive tokens: each chunk is one decode step whose
@@ -1421,6 +1460,7 @@ extern "C" void kfl_stage_destroy(kfl_stage *st) {
   if (st->cap_stream) cudaStreamDestroy(st->cap_stream);
   for (void *p : st->allocs) cudaFree(p);
   for (void *p : st->pf_allocs) cudaFree(p);
+  if (st->pf_w16) cudaFree(st->pf_w16);
   cudaGetLastError();
   st->magic = 0;
   delete st;

@@ -1,8 +1,9 @@
 """GPU parity of the prompt prefill (kfl_stage_prefill) against the oracle's prefill.
 
 A prompt of one user goes through the stage either as steps of up to max_batch rows on the user's
-KV slot (the decode kernels) or, for bf16 weights, densely (tensor-core matrix products over all
-its tokens, causal attention over the slot); the oracle runs the whole prompt in one pass.  Bar as
+KV slot (the decode kernels) or densely (tensor-core matrix products over all its tokens, causal
+attention over the slot; int4 weights dequantized to fp16 first); the oracle runs the whole prompt
+in one pass.  Bar as
 for decode: every token's output within max-abs 1e-2 of the oracle's RMS, greedy ids equal where
 the oracle's top-2 margin exceeds 1e-2, the user's written cache rows within tolerance and every
 other row of every slot bit-identical.
@@ -77,13 +78,12 @@ CASES = [
     ("bf16-head-300", RAGGED, 0, 3, K.KFL_IS_HEAD, (5, 30, 70), 2, 300, 448),
     ("hd128-200", RAGGED128, 0, 2, K.KFL_IS_HEAD, (0, 100, 7), 1, 200, 320),
     ("int4-head", RAGGED_INT4, 0, 2, K.KFL_IS_HEAD, (9, 70, 131), 1, 7, 192),
+    ("int4-head-260", RAGGED_INT4, 0, 2, K.KFL_IS_HEAD, (9, 70, 131), 2, 260, 448),
 ]
 
 
 @pytest.mark.parametrize("name,model,l0,l1,flags,contexts,user,n,max_ctx", CASES, ids=[c[0] for c in CASES])
 def test_prefill_matches_the_oracle(name, model, l0, l1, flags, contexts, user, n, max_ctx, path):
-    if path == "dense" and model.weight_fmt != "bf16":
-        pytest.skip("the dense prefill takes bf16 weights; int4 stages prefill in steps")
     if path == "steps" and n > 64:
         pytest.skip("long prompts: the dense path only (the steps path is covered by the short ones)")
     p = Pair(model, l0, l1, flags, 3, contexts, max_ctx, seed=23, max_batch=4)
