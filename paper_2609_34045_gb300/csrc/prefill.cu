@@ -246,7 +246,8 @@ __device__ __forceinline__ void epilogue32(const PrefillEpiParams &ep, int t, in
 }
 
 // ---------------------------------------------------------------------------- GEMM kernel
-template <int MODE>
+// SPLIT: the launch is a cluster of ep.splits > 1 CTAs per tile (split-K); else ep.splits is 1.
+template <int MODE, bool SPLIT>
 __global__ void __launch_bounds__(PG_THREADS, 1)
     prefill_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_a2,
                         const __grid_constant__ CUtensorMap tm_b, int n_kblocks, PrefillEpiParams ep) {
@@ -256,8 +257,8 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int t0 = blockIdx.x * PG_M, n0 = blockIdx.y * PG_N;
   // split-K: split blockIdx.z of ep.splits takes K blocks [kb0, kb1)
-  const int kb0 = (int)((long long)blockIdx.z * n_kblocks / ep.splits);
-  const int kb1 = (int)((long long)(blockIdx.z + 1) * n_kblocks / ep.splits);
+  const int kb0 = SPLIT ? (int)((long long)blockIdx.z * n_kblocks / ep.splits) : 0;
+  const int kb1 = SPLIT ? (int)((long long)(blockIdx.z + 1) * n_kblocks / ep.splits) : n_kblocks;
   const int nkb = kb1 - kb0;
   // the swizzled tiles start on a 1024-byte boundary
   const uint32_t raw = smem_addr(smem_raw);
@@ -335,7 +336,7 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
   tc_fence_after();
   const int row = warp * 32 + lane, t = t0 + row;
   EpiState<MODE> st;
-  if (ep.splits > 1) {
+  if constexpr (SPLIT) {
     // split-K over a cluster of S = ep.splits CTAs (rank = blockIdx.z).  Column chunk c (32
     // columns) of the tile belongs to rank c / (8 / S).  Every CTA pushes each chunk of its fp32
     // accumulator into the owner's shared memory (posted remote stores; the pipeline buffers are
@@ -784,8 +785,11 @@ static cudaError_t launch_mode(const CUtensorMap &a, const CUtensorMap &a2, cons
                                const PrefillEpiParams &ep, cudaStream_t s) {
   static bool smem_set = false;
   if (!smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(prefill_gemm_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)PG_SMEM);
+    cudaError_t e = cudaFuncSetAttribute(prefill_gemm_kernel<MODE, false>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PG_SMEM);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(prefill_gemm_kernel<MODE, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)PG_SMEM);
     if (e != cudaSuccess) return e;
     smem_set = true;
   }
@@ -807,15 +811,20 @@ static cudaError_t launch_mode(const CUtensorMap &a, const CUtensorMap &a2, cons
       attr[0].val.clusterDim.z = e.splits;
       cfg.gridDim = dim3(1, 1, e.splits);
       int n = 0;
-      fits[e.splits] = cudaOccupancyMaxActiveClusters(&n, prefill_gemm_kernel<MODE>, &cfg) == cudaSuccess && n > 0 ? 1 : -1;
+      fits[e.splits] =
+          cudaOccupancyMaxActiveClusters(&n, prefill_gemm_kernel<MODE, true>, &cfg) == cudaSuccess && n > 0 ? 1 : -1;
       cudaGetLastError();
     }
     if (fits[e.splits] > 0) break;
     e.splits /= 2;
   }
-  attr[0].val.clusterDim.z = e.splits;
   cfg.gridDim = dim3((e.T + PG_M - 1) / PG_M, (e.N + PG_N - 1) / PG_N, e.splits);
-  return cudaLaunchKernelEx(&cfg, prefill_gemm_kernel<MODE>, a, a2, b, 2 * n_kt, e);
+  if (e.splits == 1) {
+    cfg.numAttrs = 0;
+    return cudaLaunchKernelEx(&cfg, prefill_gemm_kernel<MODE, false>, a, a2, b, 2 * n_kt, e);
+  }
+  attr[0].val.clusterDim.z = e.splits;
+  return cudaLaunchKernelEx(&cfg, prefill_gemm_kernel<MODE, true>, a, a2, b, 2 * n_kt, e);
 }
 
 int prefill_splits(int T, int N, int n_kt, int n_sm) {

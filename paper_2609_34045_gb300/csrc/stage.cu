@@ -241,8 +241,13 @@ struct kfl_stage {
   // bf16 stages: the maps of every layer's weight tiles [4 l + j] (Q/K/V, O, gate/up, down), then
   // lm_head.  int4 stages: one map per matrix kind [j] (then lm_head) over pf_w16, the fp16 tiles
   // of the matrix being multiplied (dequantized just before its GEMM)
-  std::vector<CUtensorMap> pf_maps;
-  uint16_t *pf_w16 = nullptr;
+  std::vector<CUtensorMap> pf_maps;  // int4: [buffer * 5 + kind]
+  uint16_t *pf_w16[2] = {};
+  // int4: matrix g + 1 of a pass is dequantized on pf_side into buffer (g + 1) % 2 while GEMM g
+  // reads buffer g % 2; pf_deq[b] marks a buffer filled, pf_used[b] its GEMM done
+  cudaStream_t pf_side = nullptr;
+  cudaEvent_t pf_deq[2] = {}, pf_used[2] = {};
+  int pf_seq = 0;  // GEMMs of the current pass issued so far
   int magic = 0x4B464C53;
 
   int alloc(void **p, size_t bytes) {
@@ -725,16 +730,23 @@ int ensure_prefill(kfl_stage *st, int tokens) {
     const int n_kinds = (st->flags & KFL_LOGITS_OUT) ? 5 : 4;
     size_t most = 0;
     for (int j = 0; j < n_kinds; ++j) most = std::max(most, (size_t)kinds[j]->n_rb * 2 * kinds[j]->n_kt * TILE_BYTES);
-    if (cudaMalloc((void **)&st->pf_w16, most) != cudaSuccess) {
-      cudaGetLastError();
-      st->pf_w16 = nullptr;
-      return KFL_ERR_OOM;
-    }
-    std::vector<CUtensorMap> maps(5);
-    for (int j = 0; j < n_kinds; ++j)
-      if (encode_tiles_map(&maps[j], reinterpret_cast<const uint8_t *>(st->pf_w16), 2 * kinds[j]->n_kt,
-                           kinds[j]->n_rb))
+    for (int b = 0; b < 2; ++b) {
+      if (cudaMalloc((void **)&st->pf_w16[b], most) != cudaSuccess) {
+        cudaGetLastError();
+        st->pf_w16[b] = nullptr;
+        return KFL_ERR_OOM;
+      }
+      if (cudaEventCreateWithFlags(&st->pf_deq[b], cudaEventDisableTiming) != cudaSuccess ||
+          cudaEventCreateWithFlags(&st->pf_used[b], cudaEventDisableTiming) != cudaSuccess)
         return KFL_ERR_CUDA;
+    }
+    if (cudaStreamCreateWithFlags(&st->pf_side, cudaStreamNonBlocking) != cudaSuccess) return KFL_ERR_CUDA;
+    std::vector<CUtensorMap> maps(10);
+    for (int b = 0; b < 2; ++b)
+      for (int j = 0; j < n_kinds; ++j)
+        if (encode_tiles_map(&maps[b * 5 + j], reinterpret_cast<const uint8_t *>(st->pf_w16[b]), 2 * kinds[j]->n_kt,
+                             kinds[j]->n_rb))
+          return KFL_ERR_CUDA;
     st->pf_maps = std::move(maps);
   }
   if (st->pf_maps.empty()) {
@@ -752,26 +764,75 @@ int ensure_prefill(kfl_stage *st, int tokens) {
   return KFL_OK;
 }
 
+// Matrix j of block l (j = 4: lm_head).
+const Mat &pf_mat(const kfl_stage *st, int l, int j) {
+  if (j == 4) return st->lm;
+  const LayerDev &L = st->layers[l];
+  return j == 0 ? L.qkv : j == 1 ? L.o : j == 2 ? L.gu : L.down;
+}
+
+// The g-th GEMM of a pass multiplies matrix (g / 4, g % 4) of the blocks, then (head) the lm_head.
+bool pf_seq_matrix(const kfl_stage *st, int g, int *l, int *j) {
+  if (g < 4 * st->P.nl) {
+    *l = g / 4;
+    *j = g % 4;
+    return true;
+  }
+  if (g == 4 * st->P.nl && (st->flags & KFL_LOGITS_OUT)) {
+    *l = -1;
+    *j = 4;
+    return true;
+  }
+  return false;
+}
+
+// int4: dequantize the g-th matrix of the pass into buffer g % 2 on the side stream, once the GEMM
+// that last read that buffer (g - 2) is done.
+cudaError_t pf_dequant(kfl_stage *st, int g) {
+  int l, j;
+  if (!pf_seq_matrix(st, g, &l, &j)) return cudaSuccess;
+  const Mat &m = pf_mat(st, l, j);
+  cudaError_t err = cudaStreamWaitEvent(st->pf_side, st->pf_used[g % 2], 0);
+  if (err == cudaSuccess) err = launch_dequant_int4_f16(m.tiles, m.n_rb, m.n_kt, st->pf_w16[g % 2], st->pf_side);
+  if (err == cudaSuccess) err = cudaEventRecord(st->pf_deq[g % 2], st->pf_side);
+  return err;
+}
+
+// int4: start of a pass on stream s: both buffers free once s's earlier work is done; the first
+// matrix is dequantized.
+cudaError_t pf_pass_begin(kfl_stage *st, cudaStream_t s) {
+  st->pf_seq = 0;
+  if (st->cfg.weight_fmt != KFL_INT4_G64) return cudaSuccess;
+  cudaError_t err = cudaEventRecord(st->pf_used[0], s);
+  if (err == cudaSuccess) err = cudaEventRecord(st->pf_used[1], s);
+  if (err == cudaSuccess) err = pf_dequant(st, 0);
+  return err;
+}
+
 // One prefill GEMM with matrix j of block l (j = 4: lm_head) and the split count chosen for its
-// shape.  int4 stages first dequantize the matrix into the fp16 scratch.
+// shape.  int4 stages read the matrix's fp16 copy, dequantized ahead on the side stream (the
+// next one is started before this GEMM, so dequantization overlaps the products).
 cudaError_t pf_gemm(kfl_stage *st, int mode, const CUtensorMap &a, const CUtensorMap &a2, int l, int j,
                     PrefillEpiParams e, cudaStream_t s) {
-  const Mat &m = j == 4 ? st->lm
-                        : (j == 0 ? st->layers[l].qkv : j == 1 ? st->layers[l].o : j == 2 ? st->layers[l].gu : st->layers[l].down);
+  const Mat &m = pf_mat(st, l, j);
   const bool i4 = st->cfg.weight_fmt == KFL_INT4_G64;
   int n_kt = m.n_kt;
   const CUtensorMap *b;
+  const int g = st->pf_seq++;
   if (i4) {
-    cudaError_t err = launch_dequant_int4_f16(m.tiles, m.n_rb, m.n_kt, st->pf_w16, s);
+    cudaError_t err = pf_dequant(st, g + 1);
+    if (err == cudaSuccess) err = cudaStreamWaitEvent(s, st->pf_deq[g % 2], 0);
     if (err != cudaSuccess) return err;
-    b = &st->pf_maps[j];
+    b = &st->pf_maps[(g % 2) * 5 + j];
     n_kt = 2 * m.n_kt;  // K tiles of 128 fp16
   } else {
     b = &st->pf_maps[j == 4 ? 4 * st->P.nl : 4 * l + j];
   }
   e.f16 = i4 ? 1 : 0;
   e.splits = mode == PE_ARGMAX ? 1 : prefill_splits(e.T, e.N, n_kt, st->P.n_sm);
-  return launch_prefill_gemm(mode, a, a2, *b, n_kt, e, s);
+  cudaError_t err = launch_prefill_gemm(mode, a, a2, *b, n_kt, e, s);
+  if (err == cudaSuccess && i4) err = cudaEventRecord(st->pf_used[g % 2], s);
+  return err;
 }
 
 // The prompt in passes of up to pf_cap tokens.  Per pass and block: RMSNorm -> Q/K/V GEMM (RoPE,
@@ -792,6 +853,7 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
     CK(launch_prefill_input(ids ? ids + t0 : nullptr, hidden_in ? hidden_in + (size_t)t0 * P.d : nullptr,
                             positions + t0, n, embed ? st->embed : nullptr, P.V, P.d, P.ldh, st->pf_h, st->pf_pos,
                             st->cfg.max_ctx, st->err, s));
+    CK(pf_pass_begin(st, s));
     CUtensorMap mx[2], mo[2], ma[2];
     for (int j = 0; j < 2; ++j)
       if (encode_act_map(&mx[j], st->pf_x[j], P.d, n, ldx) || encode_act_map(&mo[j], st->pf_o[j], P.qdim, n, ldq) ||
@@ -1460,7 +1522,12 @@ extern "C" void kfl_stage_destroy(kfl_stage *st) {
   if (st->cap_stream) cudaStreamDestroy(st->cap_stream);
   for (void *p : st->allocs) cudaFree(p);
   for (void *p : st->pf_allocs) cudaFree(p);
-  if (st->pf_w16) cudaFree(st->pf_w16);
+  for (int b = 0; b < 2; ++b) {
+    if (st->pf_w16[b]) cudaFree(st->pf_w16[b]);
+    if (st->pf_deq[b]) cudaEventDestroy(st->pf_deq[b]);
+    if (st->pf_used[b]) cudaEventDestroy(st->pf_used[b]);
+  }
+  if (st->pf_side) cudaStreamDestroy(st->pf_side);
   cudaGetLastError();
   st->magic = 0;
   delete st;
