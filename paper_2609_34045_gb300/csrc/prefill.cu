@@ -7,6 +7,7 @@
 // pass as the rows of dense matrix products instead of one weight pass per token.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cmath>
 
 #include "../../include/kafila_gemm.h"
@@ -246,8 +247,9 @@ __device__ __forceinline__ void epilogue32(const PrefillEpiParams &ep, int t, in
 }
 
 // ---------------------------------------------------------------------------- GEMM kernel
-// SPLIT: the launch is a cluster of ep.splits > 1 CTAs per tile (split-K); else ep.splits is 1.
-template <int MODE, bool SPLIT>
+// Split-K: the launch is a cluster of ep.splits (2, 4 or 8) CTAs per output tile (blockIdx.z =
+// rank); unsplit GEMMs run prefill_gemm_persistent.
+template <int MODE>
 __global__ void __launch_bounds__(PG_THREADS, 1)
     prefill_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_a2,
                         const __grid_constant__ CUtensorMap tm_b, int n_kblocks, PrefillEpiParams ep) {
@@ -257,8 +259,8 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int t0 = blockIdx.x * PG_M, n0 = blockIdx.y * PG_N;
   // split-K: split blockIdx.z of ep.splits takes K blocks [kb0, kb1)
-  const int kb0 = SPLIT ? (int)((long long)blockIdx.z * n_kblocks / ep.splits) : 0;
-  const int kb1 = SPLIT ? (int)((long long)(blockIdx.z + 1) * n_kblocks / ep.splits) : n_kblocks;
+  const int kb0 = (int)((long long)blockIdx.z * n_kblocks / ep.splits);
+  const int kb1 = (int)((long long)(blockIdx.z + 1) * n_kblocks / ep.splits);
   const int nkb = kb1 - kb0;
   // the swizzled tiles start on a 1024-byte boundary
   const uint32_t raw = smem_addr(smem_raw);
@@ -336,7 +338,7 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
   tc_fence_after();
   const int row = warp * 32 + lane, t = t0 + row;
   EpiState<MODE> st;
-  if constexpr (SPLIT) {
+  {
     // split-K over a cluster of S = ep.splits CTAs (rank = blockIdx.z).  Column chunk c (32
     // columns) of the tile belongs to rank c / (8 / S).  Every CTA pushes each chunk of its fp32
     // accumulator into the owner's shared memory (posted remote stores; the pipeline buffers are
@@ -387,17 +389,9 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
         if (t < ep.T) epilogue32<MODE>(ep, t, n, r, st);
       }
     }
-  } else if (ready) {
-    for (int c = 0; c < PG_N / 32; ++c) {
-      const int n = n0 + 32 * c;
-      if (n >= ep.N) break;  // uniform across the warp
-      uint32_t r[32];
-      tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + 32 * c, r);
-      if (t < ep.T) epilogue32<MODE>(ep, t, n, r, st);
-    }
   }
   if (ready) {
-    if constexpr (MODE == PE_ARGMAX) {
+    if constexpr (MODE == PE_ARGMAX) {  // not launched split (partial maxima are per tile); kept general
       if (t < ep.T) {
         ep.amax[(size_t)t * ep.n_tiles + blockIdx.y] = st.best;
         ep.aidx[(size_t)t * ep.n_tiles + blockIdx.y] = st.bidx;
@@ -409,6 +403,168 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
   if (warp == 0) {
     tc_fence_after();
     tmem_dealloc(tmem, PG_TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------------------- persistent GEMM
+// The unsplit GEMM as a persistent kernel: one CTA per SM takes tiles c, c + grid, ...  The TMA
+// ring runs on across tile boundaries, and two accumulators (all 512 TMEM columns) let the MMAs of
+// the next tile proceed while four epilogue warps drain the previous one.  Warp 0 lane 0 issues
+// TMA, warp 1 lane 0 issues MMAs, warps 2-5 run the epilogue (warp w reads TMEM lanes
+// 32 (w % 4) ..).  Every wait is bounded; a CTA that gives up sets ERR_TIMEOUT, lets its copies
+// and MMAs in flight complete (bounded), frees its TMEM and returns.
+constexpr int PP_THREADS = 192;
+constexpr int PP_TMEM_COLS = 2 * PG_N;
+
+template <int MODE>
+__global__ void __launch_bounds__(PP_THREADS, 1)
+    prefill_gemm_persistent(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_a2,
+                            const __grid_constant__ CUtensorMap tm_b, int n_kblocks, PrefillEpiParams ep) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t s_full[PG_STAGES], s_empty[PG_STAGES], s_acc_full[2], s_acc_empty[2], s_drain;
+  __shared__ uint32_t s_tmem;
+  __shared__ int s_abort;
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int t_tiles = (ep.T + PG_M - 1) / PG_M, n_tiles = (ep.N + PG_N - 1) / PG_N;
+  const int tiles = t_tiles * n_tiles;
+  const uint32_t raw = smem_addr(smem_raw);
+  const uint32_t sa = (raw + 1023u) & ~1023u;  // [stage][hi, lo] activation tiles
+  const uint32_t sb = sa + PG_STAGES * 2 * PG_A_BYTES;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < PG_STAGES; ++s) {
+      mbar_init(smem_addr(&s_full[s]), 1);
+      mbar_init(smem_addr(&s_empty[s]), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(smem_addr(&s_acc_full[b]), 1);
+      mbar_init(smem_addr(&s_acc_empty[b]), 4);  // one arrival per epilogue warp
+    }
+    mbar_init(smem_addr(&s_drain), 1);
+    s_abort = 0;
+    fence_mbar_init();
+  }
+  __syncwarp();
+  if (warp == 0) tmem_alloc(smem_addr(&s_tmem), PP_TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+  volatile int *abort_flag = &s_abort;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---- TMA producer: k-block it of the CTA's sequence uses stage it % S
+      int issued[PG_STAGES] = {};
+      long long it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
+        const int t0 = (tile % t_tiles) * PG_M, n0 = (tile / t_tiles) * PG_N;
+        for (int kb = 0; kb < n_kblocks; ++kb, ++it) {
+          const int s = (int)(it % PG_STAGES);
+          const uint32_t use = (uint32_t)(it / PG_STAGES);
+          if (*abort_flag || (use > 0 && !mbar_wait(smem_addr(&s_empty[s]), (use - 1) & 1))) {
+            ok = false;
+            break;
+          }
+          const uint32_t full = smem_addr(&s_full[s]);
+          mbar_arrive_expect_tx(full, 2 * PG_A_BYTES + PG_B_BYTES);
+          tma_load_2d(sa + s * 2 * PG_A_BYTES, &tm_a, kb * PG_K, t0, full);
+          tma_load_2d(sa + s * 2 * PG_A_BYTES + PG_A_BYTES, &tm_a2, kb * PG_K, t0, full);
+          tma_load_4d(sb + s * PG_B_BYTES, &tm_b, (kb & 1) * PG_K, 0, kb >> 1, n0 / RB, full);
+          ++issued[s];
+        }
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        atomicOr(ep.err, ERR_TIMEOUT);
+        for (int s = 0; s < PG_STAGES; ++s)
+          if (issued[s] > 0) mbar_wait(smem_addr(&s_full[s]), (issued[s] - 1) & 1);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---- MMA issuer: tile i of this CTA accumulates into TMEM columns (i % 2) * PG_N
+      const uint32_t idesc = ep.f16 ? idesc_kind_f16(PG_M, PG_N, false) : idesc_kind_f16(PG_M, PG_N, true);
+      long long it = 0;
+      int i = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x, ++i) {
+        const int buf = i & 1;
+        if (i >= 2 && !mbar_wait(smem_addr(&s_acc_empty[buf]), ((i >> 1) - 1) & 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem + (uint32_t)(buf * PG_N);
+        for (int kb = 0; kb < n_kblocks; ++kb, ++it) {
+          const int s = (int)(it % PG_STAGES);
+          if (*abort_flag || !mbar_wait(smem_addr(&s_full[s]), (uint32_t)(it / PG_STAGES) & 1)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a = sa + s * 2 * PG_A_BYTES, b = sb + s * PG_B_BYTES;
+#pragma unroll
+          for (int k = 0; k < PG_K / 16; ++k) {
+            const uint64_t db = sdesc_k_sw128(b + 32 * k);
+            mma_bf16_ss(d, sdesc_k_sw128(a + 32 * k), db, idesc, (kb | k) != 0);
+            mma_bf16_ss(d, sdesc_k_sw128(a + PG_A_BYTES + 32 * k), db, idesc, 1);
+          }
+          mma_commit(smem_addr(&s_empty[s]));
+        }
+        if (ok) mma_commit(smem_addr(&s_acc_full[buf]));
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        atomicOr(ep.err, ERR_TIMEOUT);
+      }
+      // every MMA issued has completed before TMEM can be freed
+      mma_commit(smem_addr(&s_drain));
+      mbar_wait(smem_addr(&s_drain), 0);
+    }
+    __syncwarp();
+  } else {
+    // ---- epilogue warps 2..5: TMEM lanes 32 q .. 32 q + 31 (q = warp % 4) are tokens t0 + 32 q + lane
+    const int q = warp & 3, row = 32 * q + lane;
+    int i = 0;
+    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++i) {
+      const int buf = i & 1;
+      const bool ready = __all_sync(0xffffffffu, !*abort_flag && mbar_wait(smem_addr(&s_acc_full[buf]), (i >> 1) & 1));
+      if (!ready) {
+        if (lane == 0) {
+          *abort_flag = 1;
+          atomicOr(ep.err, ERR_TIMEOUT);
+        }
+        break;
+      }
+      tc_fence_after();
+      const int t_tile = tile % t_tiles, n_tile = tile / t_tiles;
+      const int t = t_tile * PG_M + row, n0 = n_tile * PG_N;
+      EpiState<MODE> st;
+      for (int c = 0; c < PG_N / 32; ++c) {
+        const int n = n0 + 32 * c;
+        if (n >= ep.N) break;  // uniform across the warp
+        uint32_t r[32];
+        tmem_ld32(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * PG_N + 32 * c), r);
+        if (t < ep.T) epilogue32<MODE>(ep, t, n, r, st);
+      }
+      if constexpr (MODE == PE_ARGMAX) {
+        if (t < ep.T) {
+          ep.amax[(size_t)t * ep.n_tiles + n_tile] = st.best;
+          ep.aidx[(size_t)t * ep.n_tiles + n_tile] = st.bidx;
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_addr(&s_acc_empty[buf]));
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, PP_TMEM_COLS);
   }
 }
 
@@ -785,11 +941,10 @@ static cudaError_t launch_mode(const CUtensorMap &a, const CUtensorMap &a2, cons
                                const PrefillEpiParams &ep, cudaStream_t s) {
   static bool smem_set = false;
   if (!smem_set) {
-    cudaError_t e = cudaFuncSetAttribute(prefill_gemm_kernel<MODE, false>,
+    cudaError_t e = cudaFuncSetAttribute(prefill_gemm_persistent<MODE>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PG_SMEM);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(prefill_gemm_kernel<MODE, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)PG_SMEM);
+      e = cudaFuncSetAttribute(prefill_gemm_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PG_SMEM);
     if (e != cudaSuccess) return e;
     smem_set = true;
   }
@@ -812,7 +967,7 @@ static cudaError_t launch_mode(const CUtensorMap &a, const CUtensorMap &a2, cons
       cfg.gridDim = dim3(1, 1, e.splits);
       int n = 0;
       fits[e.splits] =
-          cudaOccupancyMaxActiveClusters(&n, prefill_gemm_kernel<MODE, true>, &cfg) == cudaSuccess && n > 0 ? 1 : -1;
+          cudaOccupancyMaxActiveClusters(&n, prefill_gemm_kernel<MODE>, &cfg) == cudaSuccess && n > 0 ? 1 : -1;
       cudaGetLastError();
     }
     if (fits[e.splits] > 0) break;
@@ -820,11 +975,22 @@ static cudaError_t launch_mode(const CUtensorMap &a, const CUtensorMap &a2, cons
   }
   cfg.gridDim = dim3((e.T + PG_M - 1) / PG_M, (e.N + PG_N - 1) / PG_N, e.splits);
   if (e.splits == 1) {
+    // one persistent CTA per SM (fewer if there are fewer tiles)
+    static int n_sm = 0;
+    if (!n_sm) {
+      int dev = 0;
+      if (cudaGetDevice(&dev) != cudaSuccess ||
+          cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return cudaErrorInvalidDevice;
+    }
+    const long long tiles = (long long)cfg.gridDim.x * cfg.gridDim.y;
+    cfg.gridDim = dim3((unsigned)std::min<long long>(tiles, n_sm));
+    cfg.blockDim = dim3(PP_THREADS);
     cfg.numAttrs = 0;
-    return cudaLaunchKernelEx(&cfg, prefill_gemm_kernel<MODE, false>, a, a2, b, 2 * n_kt, e);
+    return cudaLaunchKernelEx(&cfg, prefill_gemm_persistent<MODE>, a, a2, b, 2 * n_kt, e);
   }
   attr[0].val.clusterDim.z = e.splits;
-  return cudaLaunchKernelEx(&cfg, prefill_gemm_kernel<MODE, true>, a, a2, b, 2 * n_kt, e);
+  return cudaLaunchKernelEx(&cfg, prefill_gemm_kernel<MODE>, a, a2, b, 2 * n_kt, e);
 }
 
 int prefill_splits(int T, int N, int n_kt, int n_sm) {
