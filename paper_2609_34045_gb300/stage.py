@@ -14,6 +14,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libkafila_stage.so")
 
 KFL_OK = 0
+KFL_ERR_ARG, KFL_ERR_RANGE, KFL_ERR_OOM, KFL_ERR_CUDA, KFL_ERR_STATE, KFL_ERR_TIMEOUT = -1, -2, -3, -4, -5, -6
 KFL_BF16 = 0
 KFL_INT4_G64 = 1
 KFL_EMBED_IN = 1
@@ -239,9 +240,10 @@ def kfl_stage_decode_users(st: Stage, token_ids, hidden_in, positions, users, ba
 
 def kfl_stage_prefill(st: Stage, token_ids, hidden_in, positions, user: int, n_tokens: int, hidden_out, next_ids,
                       cuda_stream: int | None = None) -> None:
-    """n_tokens prompt tokens of one user (KV slot `user`) through the stage, in steps of up to
-    max_batch rows: int32 token_ids [n] or fp32 hidden_in [n][d], int32 positions [n], fp32
-    hidden_out [n][d], int32 next_ids [n] (CUDA tensors).  Asynchronous."""
+    """n_tokens prompt tokens of one user (KV slot `user`) through the stage (the dense tensor-core
+    path, or for short prompts steps of up to max_batch rows): int32 token_ids [n] or fp32
+    hidden_in [n][d], int32 positions [n], fp32 hidden_out [n][d], int32 next_ids [n] (CUDA
+    tensors).  Asynchronous."""
     _check(lib().kfl_stage_prefill(st.handle, _ptr(token_ids), _ptr(hidden_in), _ptr(positions), user, n_tokens,
                                    _ptr(hidden_out), _ptr(next_ids), cuda_stream), "kfl_stage_prefill")
 

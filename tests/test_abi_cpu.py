@@ -90,3 +90,21 @@ def test_null_handles_are_rejected(lib):
     assert L.kfl_kv_reset(None, -1) == -5
     assert L.kfl_stage_status(None) == -5
     L.kfl_stage_destroy(None)  # no-op
+
+
+def test_prefill_and_matmul_argument_errors_without_a_gpu(lib):
+    """The entry points refuse bad arguments before touching the device."""
+    class NoStage:
+        handle = None  # a NULL stage pointer
+
+    with pytest.raises(K.KflError) as e:
+        K.kfl_stage_prefill(NoStage(), None, None, None, 0, 4, None, None)
+    assert e.value.code == K.KFL_ERR_STATE
+    for args in ((None, 4, 64, 64, None, 8, None, 8),       # NULL pointers
+                 (1 << 20, 0, 64, 64, 1 << 21, 8, 1 << 22, 8),  # T < 1
+                 (1 << 20, 4, 64, 60, 1 << 21, 8, 1 << 22, 8),  # ldx < K
+                 (1 << 20, 4, 64, 64, 1 << 21, 8, 1 << 22, 6),  # ldy < N
+                 (1 << 20, 4, 64, 64, 1 << 21, 8, (1 << 22) + 4, 8)):  # y not 16-byte aligned
+        with pytest.raises(K.KflError) as e:
+            K.kfl_matmul_bf16w(*args)
+        assert e.value.code == K.KFL_ERR_ARG
