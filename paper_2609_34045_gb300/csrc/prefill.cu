@@ -253,6 +253,7 @@ template <int MODE>
 __global__ void __launch_bounds__(PG_THREADS, 1)
     prefill_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_a2,
                         const __grid_constant__ CUtensorMap tm_b, int n_kblocks, PrefillEpiParams ep) {
+  static_assert(MODE != PE_ARGMAX, "the argmax partials are per whole tile: lm_head is never split");
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t s_full[PG_STAGES], s_empty[PG_STAGES], s_accum;
   __shared__ uint32_t s_tmem;
@@ -387,14 +388,6 @@ __global__ void __launch_bounds__(PG_THREADS, 1)
 #pragma unroll
         for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(acc[j]);
         if (t < ep.T) epilogue32<MODE>(ep, t, n, r, st);
-      }
-    }
-  }
-  if (ready) {
-    if constexpr (MODE == PE_ARGMAX) {  // not launched split (partial maxima are per tile); kept general
-      if (t < ep.T) {
-        ep.amax[(size_t)t * ep.n_tiles + blockIdx.y] = st.best;
-        ep.aidx[(size_t)t * ep.n_tiles + blockIdx.y] = st.bidx;
       }
     }
   }
@@ -943,8 +936,10 @@ static cudaError_t launch_mode(const CUtensorMap &a, const CUtensorMap &a2, cons
   if (!smem_set) {
     cudaError_t e = cudaFuncSetAttribute(prefill_gemm_persistent<MODE>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PG_SMEM);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(prefill_gemm_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)PG_SMEM);
+    if constexpr (MODE != PE_ARGMAX)
+      if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(prefill_gemm_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)PG_SMEM);
     if (e != cudaSuccess) return e;
     smem_set = true;
   }
@@ -958,39 +953,41 @@ static cudaError_t launch_mode(const CUtensorMap &a, const CUtensorMap &a2, cons
   attr[0].val.clusterDim.y = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  // the largest split count not above the chosen one whose cluster fits on the device
-  static int fits[9] = {};  // 0 unknown, 1 yes, -1 no
   PrefillEpiParams e = ep;
-  while (e.splits > 1) {
-    if (fits[e.splits] == 0) {
+  if constexpr (MODE != PE_ARGMAX) {
+    // the largest split count not above the chosen one whose cluster fits on the device
+    static int fits[9] = {};  // 0 unknown, 1 yes, -1 no
+    while (e.splits > 1) {
+      if (fits[e.splits] == 0) {
+        attr[0].val.clusterDim.z = e.splits;
+        cfg.gridDim = dim3(1, 1, e.splits);
+        int n = 0;
+        fits[e.splits] =
+            cudaOccupancyMaxActiveClusters(&n, prefill_gemm_kernel<MODE>, &cfg) == cudaSuccess && n > 0 ? 1 : -1;
+        cudaGetLastError();
+      }
+      if (fits[e.splits] > 0) break;
+      e.splits /= 2;
+    }
+    if (e.splits > 1) {
+      cfg.gridDim = dim3((e.T + PG_M - 1) / PG_M, (e.N + PG_N - 1) / PG_N, e.splits);
       attr[0].val.clusterDim.z = e.splits;
-      cfg.gridDim = dim3(1, 1, e.splits);
-      int n = 0;
-      fits[e.splits] =
-          cudaOccupancyMaxActiveClusters(&n, prefill_gemm_kernel<MODE>, &cfg) == cudaSuccess && n > 0 ? 1 : -1;
-      cudaGetLastError();
+      return cudaLaunchKernelEx(&cfg, prefill_gemm_kernel<MODE>, a, a2, b, 2 * n_kt, e);
     }
-    if (fits[e.splits] > 0) break;
-    e.splits /= 2;
   }
-  cfg.gridDim = dim3((e.T + PG_M - 1) / PG_M, (e.N + PG_N - 1) / PG_N, e.splits);
-  if (e.splits == 1) {
-    // one persistent CTA per SM (fewer if there are fewer tiles)
-    static int n_sm = 0;
-    if (!n_sm) {
-      int dev = 0;
-      if (cudaGetDevice(&dev) != cudaSuccess ||
-          cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-        return cudaErrorInvalidDevice;
-    }
-    const long long tiles = (long long)cfg.gridDim.x * cfg.gridDim.y;
-    cfg.gridDim = dim3((unsigned)std::min<long long>(tiles, n_sm));
-    cfg.blockDim = dim3(PP_THREADS);
-    cfg.numAttrs = 0;
-    return cudaLaunchKernelEx(&cfg, prefill_gemm_persistent<MODE>, a, a2, b, 2 * n_kt, e);
+  // one persistent CTA per SM (fewer if there are fewer tiles)
+  static int n_sm = 0;
+  if (!n_sm) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return cudaErrorInvalidDevice;
   }
-  attr[0].val.clusterDim.z = e.splits;
-  return cudaLaunchKernelEx(&cfg, prefill_gemm_kernel<MODE>, a, a2, b, 2 * n_kt, e);
+  const long long tiles = (long long)((e.T + PG_M - 1) / PG_M) * ((e.N + PG_N - 1) / PG_N);
+  cfg.gridDim = dim3((unsigned)std::min<long long>(tiles, n_sm));
+  cfg.blockDim = dim3(PP_THREADS);
+  cfg.numAttrs = 0;
+  return cudaLaunchKernelEx(&cfg, prefill_gemm_persistent<MODE>, a, a2, b, 2 * n_kt, e);
 }
 
 int prefill_splits(int T, int N, int n_kt, int n_sm) {

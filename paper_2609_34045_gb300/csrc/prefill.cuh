@@ -11,10 +11,12 @@ namespace kfl {
 // ---- the prefill GEMM: Y[T][N] = X[T][K] W[N][K]^T ------------------------------------------
 // X is fp32 in meaning and given as two bf16 terms, X = Xhi + Xlo (Xhi = bf16(X), Xlo =
 // bf16(X - Xhi), about 2^-16 relative error left), so that the products keep the accuracy of the
-// decode path's fp32 activations; W is bf16 as stored.  One CTA computes a tile of PG_M tokens x
-// PG_N weight rows with tcgen05.mma (M = PG_M, N = PG_N, K = 16 per instruction; each K slice
-// once with Xhi and once with Xlo against the same W slice), the fp32 accumulator in tensor
-// memory.  Operands reach shared memory by TMA with the 128-byte swizzle, PG_K = 64 bf16 (one
+// decode path's fp32 activations; W is bf16 as stored (int4 stages: fp16 tiles dequantized from
+// the int4 ones, with fp16 terms of X).  An output tile is PG_M tokens x PG_N weight rows,
+// computed with tcgen05.mma (M = PG_M, N = PG_N, K = 16 per instruction; each K slice once with
+// Xhi and once with Xlo against the same W slice), the fp32 accumulator in tensor memory: by a
+// persistent CTA per SM with two accumulators (prefill_gemm_persistent), or, split over K, by a
+// cluster of 2, 4 or 8 CTAs that reduce through distributed shared memory (prefill_gemm_kernel).  Operands reach shared memory by TMA with the 128-byte swizzle, PG_K = 64 bf16 (one
 // swizzle row) per pipeline stage: Xhi and Xlo through 2-D maps of the activation rows, W through
 // a 4-D map of the decode path's weight tiles [N/RB][K/KT][RB][KT] (one box = PG_N / RB row
 // blocks x 64 columns of one K tile), so the prefill streams the weights from where the decode
@@ -25,8 +27,8 @@ constexpr int PG_K = 64;
 constexpr int PG_STAGES = 3;
 constexpr int PG_A_BYTES = PG_M * PG_K * 2;  // 16 KiB per term
 constexpr int PG_B_BYTES = PG_N * PG_K * 2;  // 32 KiB
-constexpr int PG_THREADS = 128;              // 4 warps: TMA (thread 0), MMA (thread 32); all: epilogue
-constexpr int PG_TMEM_COLS = PG_N;           // fp32 accumulator columns
+constexpr int PG_THREADS = 128;              // split kernel: TMA (thread 0), MMA (thread 32); all: epilogue
+constexpr int PG_TMEM_COLS = PG_N;           // split kernel: fp32 accumulator columns
 constexpr size_t PG_SMEM = (size_t)PG_STAGES * (2 * PG_A_BYTES + PG_B_BYTES) + 1024;  // + alignment slack
 
 enum PrefillEpi : int {
