@@ -730,17 +730,25 @@ int ensure_prefill(kfl_stage *st, int tokens) {
     const int n_kinds = (st->flags & KFL_LOGITS_OUT) ? 5 : 4;
     size_t most = 0;
     for (int j = 0; j < n_kinds; ++j) most = std::max(most, (size_t)kinds[j]->n_rb * 2 * kinds[j]->n_kt * TILE_BYTES);
+    // each resource is made once (a call that failed part way keeps what it made, and the next
+    // call completes the set; kfl_stage_destroy frees them)
     for (int b = 0; b < 2; ++b) {
-      if (cudaMalloc((void **)&st->pf_w16[b], most) != cudaSuccess) {
+      if (!st->pf_w16[b] && cudaMalloc((void **)&st->pf_w16[b], most) != cudaSuccess) {
         cudaGetLastError();
         st->pf_w16[b] = nullptr;
         return KFL_ERR_OOM;
       }
-      if (cudaEventCreateWithFlags(&st->pf_deq[b], cudaEventDisableTiming) != cudaSuccess ||
-          cudaEventCreateWithFlags(&st->pf_used[b], cudaEventDisableTiming) != cudaSuccess)
+      if ((!st->pf_deq[b] && cudaEventCreateWithFlags(&st->pf_deq[b], cudaEventDisableTiming) != cudaSuccess) ||
+          (!st->pf_used[b] && cudaEventCreateWithFlags(&st->pf_used[b], cudaEventDisableTiming) != cudaSuccess)) {
+        cudaGetLastError();
         return KFL_ERR_CUDA;
+      }
     }
-    if (cudaStreamCreateWithFlags(&st->pf_side, cudaStreamNonBlocking) != cudaSuccess) return KFL_ERR_CUDA;
+    if (!st->pf_side && cudaStreamCreateWithFlags(&st->pf_side, cudaStreamNonBlocking) != cudaSuccess) {
+      cudaGetLastError();
+      st->pf_side = nullptr;
+      return KFL_ERR_CUDA;
+    }
     std::vector<CUtensorMap> maps(10);
     for (int b = 0; b < 2; ++b)
       for (int j = 0; j < n_kinds; ++j)
