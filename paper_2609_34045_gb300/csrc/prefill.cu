@@ -796,13 +796,17 @@ __global__ void prefill_input_kernel(const int *ids, const float *hidden_in, con
     h[(size_t)t * ldh + i] = embed ? bf16_to_f32(embed[(size_t)id * d + i]) : hidden_in[(size_t)t * d + i];
 }
 
-// x[t] = h[t] / rms(h[t]) * g as hi and lo bf16 terms, one block per token.
+// x[t] = h[t] / rms(h[t]) * g as hi and lo 16-bit terms, one block per token, four elements per
+// thread step (d a multiple of 8; h, g and x rows 16-byte aligned).
 __global__ void prefill_rmsnorm_kernel(const float *h, int ldh, int d, const float *g, float eps, uint16_t *x,
                                        uint16_t *x_lo, int ldx, int f16) {
-  const int t = blockIdx.x;
-  const float *row = h + (size_t)t * ldh;
+  const int t = blockIdx.x, d4 = d / 4;
+  const float4 *row = reinterpret_cast<const float4 *>(h + (size_t)t * ldh);
   float ss = 0.f;
-  for (int i = threadIdx.x; i < d; i += blockDim.x) ss += row[i] * row[i];
+  for (int i = threadIdx.x; i < d4; i += blockDim.x) {
+    const float4 v = row[i];
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
   __shared__ float red[32];
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
   if (threadIdx.x % 32 == 0) red[threadIdx.x / 32] = ss;
@@ -814,8 +818,16 @@ __global__ void prefill_rmsnorm_kernel(const float *h, int ldh, int d, const flo
   }
   __syncthreads();
   const float inv = rsqrtf(red[0] / d + eps);
-  for (int i = threadIdx.x; i < d; i += blockDim.x)
-    split_term(row[i] * inv * g[i], x[(size_t)t * ldx + i], x_lo[(size_t)t * ldx + i], f16);
+  const float4 *g4 = reinterpret_cast<const float4 *>(g);
+  uint2 *xh = reinterpret_cast<uint2 *>(x + (size_t)t * ldx), *xl = reinterpret_cast<uint2 *>(x_lo + (size_t)t * ldx);
+  for (int i = threadIdx.x; i < d4; i += blockDim.x) {
+    const float4 v = row[i], gg = g4[i];
+    uint2 hi, lo;
+    split_pack(v.x * inv * gg.x, v.y * inv * gg.y, hi.x, lo.x, f16);
+    split_pack(v.z * inv * gg.z, v.w * inv * gg.w, hi.y, lo.y, f16);
+    xh[i] = hi;
+    xl[i] = lo;
+  }
 }
 
 // One thread per 8 consecutive outputs of one row (16 bytes): the int4 tile stores the nibble of
@@ -863,20 +875,31 @@ __global__ void split_rows_kernel(const float *x, int K, int ldx, uint16_t *hi, 
     split_bf16(x[(size_t)t * ldx + i], hi[(size_t)t * ld + i], lo[(size_t)t * ld + i]);
 }
 
-// next_ids[t]: the lowest index among the largest logits, over the column tiles' partial maxima.
+// next_ids[t]: the lowest index among the largest logits, over the column tiles' partial maxima;
+// one warp per token (each lane scans every 32nd tile, then the warp keeps the largest value and,
+// among equal values, the lowest index).
 __global__ void prefill_argmax_kernel(const float *amax, const int *aidx, int n_tiles, int T, int *next_ids) {
-  const int t = blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= T) return;
+  const int t = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32, lane = threadIdx.x % 32;
+  if (t >= T) return;  // uniform per warp
   float best = -INFINITY;
-  int bi = 0;
-  for (int j = 0; j < n_tiles; ++j) {
+  int bi = 0x7FFFFFFF;
+  for (int j = lane; j < n_tiles; j += 32) {
     const float v = amax[(size_t)t * n_tiles + j];
-    if (v > best) {
+    const int i = aidx[(size_t)t * n_tiles + j];
+    if (v > best || (v == best && i < bi)) {
       best = v;
-      bi = aidx[(size_t)t * n_tiles + j];
+      bi = i;
     }
   }
-  next_ids[t] = bi;
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, best, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+    if (ov > best || (ov == best && oi < bi)) {
+      best = ov;
+      bi = oi;
+    }
+  }
+  if (lane == 0) next_ids[t] = bi == 0x7FFFFFFF ? 0 : bi;
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -1070,7 +1093,7 @@ cudaError_t launch_split_bf16(const float *x, int T, int K, int ldx, uint16_t *h
 
 cudaError_t launch_prefill_argmax(const float *amax, const int *aidx, int n_tiles, int T, int *next_ids,
                                   cudaStream_t s) {
-  prefill_argmax_kernel<<<(T + 127) / 128, 128, 0, s>>>(amax, aidx, n_tiles, T, next_ids);
+  prefill_argmax_kernel<<<(T + 3) / 4, 128, 0, s>>>(amax, aidx, n_tiles, T, next_ids);
   return cudaGetLastError();
 }
 
