@@ -337,25 +337,29 @@ def _torch_prefill(model, layers, head, kcache, vcache, start, ids, causal=True)
     return h.numpy(), z.numpy(), kc, vc
 
 
-def pin_prefill_vs_torch():
+def _check_prefill_vs_torch(model, n_layers):
     # user 1 (9 cached rows) takes a prompt of 6 tokens at positions 9..14; user 0 is untouched
-    st = _small_stage(0, 3, True, True)
-    k0 = [st.k_cache[i, 1].copy() for i in range(3)]
-    v0 = [st.v_cache[i, 1].copy() for i in range(3)]
+    st = _small_stage(0, n_layers, True, True, model=model)
+    k0 = [st.k_cache[i, 1].copy() for i in range(n_layers)]
+    v0 = [st.v_cache[i, 1].copy() for i in range(n_layers)]
     other = (st.k_cache[:, 0].copy(), st.v_cache[:, 0].copy())
-    ids = np.array([3, 44, 17, 17, 0, 49])
+    ids = np.array([3, 44, 17, 17, 0, 39]) % model.vocab
     out = st.prefill(1, np.arange(9, 15), token_ids=ids)
-    layers = [st.layers[i] for i in range(3)]
-    h, z, kc, vc = _torch_prefill(SMALL, layers, st.head, k0, v0, 9, ids)
+    layers = [st.layers[i] for i in range(n_layers)]
+    h, z, kc, vc = _torch_prefill(model, layers, st.head, k0, v0, 9, ids)
     assert np.allclose(out["hidden_out"], h, rtol=1e-11, atol=1e-12)
     assert np.allclose(out["logits"], z, rtol=1e-11, atol=1e-12)
-    for i in range(3):
+    for i in range(n_layers):
         assert np.array_equal(oracle.bf16_to_f64(st.k_cache[i, 1]), kc[i].numpy())
         assert np.array_equal(oracle.bf16_to_f64(st.v_cache[i, 1]), vc[i].numpy())
     assert np.array_equal(st.k_cache[:, 0], other[0]) and np.array_equal(st.v_cache[:, 0], other[1])
     # the same check without the causal mask fails: it tests what each token sees
-    h_all, _, _, _ = _torch_prefill(SMALL, layers, st.head, k0, v0, 9, ids, causal=False)
+    h_all, _, _, _ = _torch_prefill(model, layers, st.head, k0, v0, 9, ids, causal=False)
     assert not np.allclose(out["hidden_out"], h_all, rtol=1e-6, atol=1e-6)
+
+
+def pin_prefill_vs_torch():
+    _check_prefill_vs_torch(SMALL, 3)
 
 
 def pin_prefill_is_sequential_decode():
@@ -380,10 +384,15 @@ def pin_int4_stage_vs_torch():
     _check_stage_vs_torch(SMALL_INT4, 2)
 
 
+def pin_int4_prefill_vs_torch():
+    # int4 weights decoded through the golden code table on the torch side
+    _check_prefill_vs_torch(SMALL_INT4, 2)
+
+
 PINS = [pin_bf16_golden, pin_bf16_vs_torch, pin_int4_exhaustive, pin_int4_groups, pin_gemv_bruteforce,
         pin_rms_norm, pin_rope, pin_softmax, pin_attention, pin_silu, pin_argmax, pin_stage_vs_torch,
         pin_kv_slots, pin_stage_split_associativity, pin_int4_stage_vs_torch, pin_prefill_vs_torch,
-        pin_prefill_is_sequential_decode]
+        pin_prefill_is_sequential_decode, pin_int4_prefill_vs_torch]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
