@@ -376,6 +376,20 @@ def pin_prefill_is_sequential_decode():
         assert np.array_equal(a.k_cache, b.k_cache) and np.array_equal(a.v_cache, b.v_cache)
 
 
+def pin_prefill_in_two_calls():
+    # a prompt prefilled in two calls (the second attending to the first's cache rows) equals one call
+    a = _small_stage(0, 3, True, True)
+    b = _small_stage(0, 3, True, True)
+    ids = np.array([8, 1, 30, 30, 12, 7, 49])
+    one = a.prefill(0, np.arange(5, 12), token_ids=ids)
+    first = b.prefill(0, np.arange(5, 8), token_ids=ids[:3])
+    second = b.prefill(0, np.arange(8, 12), token_ids=ids[3:])
+    both = np.concatenate([first["hidden_out"], second["hidden_out"]])
+    assert np.allclose(one["hidden_out"], both, rtol=1e-12, atol=1e-13)
+    assert np.array_equal(one["next_ids"], np.concatenate([first["next_ids"], second["next_ids"]]))
+    assert np.array_equal(a.k_cache, b.k_cache) and np.array_equal(a.v_cache, b.v_cache)
+
+
 SMALL_INT4 = wl.ModelShape(n_layers_total=2, d_model=128, n_heads=4, n_kv_heads=2, head_dim=32, ffn=192,
                            vocab=40, weight_fmt="int4_g64")
 
@@ -392,7 +406,7 @@ def pin_int4_prefill_vs_torch():
 PINS = [pin_bf16_golden, pin_bf16_vs_torch, pin_int4_exhaustive, pin_int4_groups, pin_gemv_bruteforce,
         pin_rms_norm, pin_rope, pin_softmax, pin_attention, pin_silu, pin_argmax, pin_stage_vs_torch,
         pin_kv_slots, pin_stage_split_associativity, pin_int4_stage_vs_torch, pin_prefill_vs_torch,
-        pin_prefill_is_sequential_decode, pin_int4_prefill_vs_torch]
+        pin_prefill_is_sequential_decode, pin_int4_prefill_vs_torch, pin_prefill_in_two_calls]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
