@@ -358,7 +358,7 @@ def empty_stage_ms(work, stream, n=50):
 
 
 def plan_example(work, fit):
-    """The planner (Algorithm 1 with head rotation, section V) on a synthetic ring driven by this
+    """The planner (the exact fixed-order division with head rotation, section V) on a synthetic ring driven by this
     GPU's measured stage cost: four members stream at 1, 1/2, 1/4 and 1/8 of the fitted rate b
     with the fitted overhead o, and hold 35, 280, 140 and 70 GB; the bottleneck of the planned
     division against the evaluation's Uniform and Memory-proportional divisions under the same

@@ -1,7 +1,7 @@
 /* Kafila block placement over a ring of devices: host-side planner (no GPU needed).
  *
  * Follows the paper's planner: the stage cost of Eq. 2 (Section V-A), the exact chain-on-chain
- * block placement for a fixed device order (Section V-B "Block placement", Algorithm 1), head
+ * block placement for a fixed device order (Section V-B "Block placement"), head
  * placement by rotation with a noise margin (Section V-B, the head paragraph), and the three
  * admission tiers with the final memory check (Section V-C "Admission").
  *
@@ -24,15 +24,17 @@ extern "C" {
 
 #define KFL_ERR_INFEASIBLE (-7) /* no division of the blocks fits the devices (limits, or m > k) */
 
-/* Algorithm 1 (Partition): exact chain-on-chain placement of k blocks on devices 0..m-1 in this
- * order.  Device i holding n blocks costs fixed[i] + n * per[i] (Eq. 2: fixed = o_i, plus
- * beta_head / b_i for the head; per = beta_block / b_i) and holds at most lim[i] blocks.
- * Writes n_out[i] >= 1 with sum k, n_out[i] <= lim[i], minimizing the bottleneck
- * max_i fixed[i] + n_out[i] * per[i], and that bottleneck to *tau_out.  Among the optimal
- * divisions it returns the one the left-to-right pass builds (each device takes as many blocks as
- * the bottleneck allows, keeping one for every device after it).
+/* Exact chain-on-chain placement of k blocks on devices 0..m-1 in this order (Section V-B,
+ * "Block placement": the problem the paper's Partition solves).  Device i holding n blocks costs
+ * fixed[i] + n * per[i] (Eq. 2: fixed = o_i, plus beta_head / b_i for the head;
+ * per = beta_block / b_i) and holds at most lim[i] blocks.  Writes n_out[i] >= 1 with sum k,
+ * n_out[i] <= lim[i], minimizing the bottleneck max_i fixed[i] + n_out[i] * per[i], and that
+ * bottleneck to *tau_out (the largest cost of the returned division, so exactly attained).
+ * Method: each device starts with one block; the remaining k - m go one at a time to the device
+ * whose cost after taking one more is lowest (the lower index on ties).  O(m + k log m).
+ * Among the optimal divisions it returns the one this hand-out builds.
  * Errors: KFL_ERR_ARG (k < 1, m < 1, NULL arrays, a non-finite fixed or per, per <= 0, lim < 0),
- * KFL_ERR_INFEASIBLE (no division exists: sum of limits < k, or m > k). */
+ * KFL_ERR_INFEASIBLE (no division exists: a limit of 0, the limits sum below k, or m > k). */
 int kfl_partition(int k, int m, const double *fixed, const double *per, const int *lim, int *n_out,
                   double *tau_out);
 

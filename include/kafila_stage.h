@@ -258,8 +258,8 @@ const char *kfl_last_error_detail(void);
  * 16384, vocab up to 262144; larger sizes return KFL_ERR_RANGE with the limits in
  * kfl_last_error_detail.  Its scratch is one fixed array of 131,328 bytes of device memory per
  * GPU that loads this library, held until the process exits.  The first call on a device looks
- * the array up and clears its ticket with a synchronous cudaMemset, so make that first call
- * before any stream capture.  Every call on a device shares the array and leaves its contents
+ * the array up, clears its ticket with cudaMemset and waits for the device (cudaDeviceSynchronize),
+ * so make that first call before any stream capture.  Every call on a device shares the array and leaves its contents
  * behind; calls that overlap on the GPU (other streams, no ordering) race and give wrong ids.
  * Errors: KFL_ERR_ARG (NULL, misaligned or rms_eps <= 0), KFL_ERR_RANGE, KFL_ERR_CUDA. */
 int kfl_head_argmax_noalloc(const float *hidden, const uint16_t *final_norm, const uint16_t *lm_head,

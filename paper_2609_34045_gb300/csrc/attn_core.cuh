@@ -11,10 +11,11 @@
 // Scores are in the log2 domain (q pre-scaled by log2(e)/sqrt(hd)).
 //
 // 256 threads.  Scores S = q K^T and the weighted sum P V are small dense products (at most 8
-// heads x 64 positions x hd): both run on the tensor cores as warp-level m16n8k8 MMAs in TF32
-// with fp32 accumulation (the heads are the M rows, padded to 16).  q and P are rounded to TF32
-// (2^-11 relative); K and V are bf16 and exact in TF32.  Scores: warp w takes positions 8w..8w+7;
-// P V: warp w takes head dimensions hd/8 * w onwards.
+// heads x 64 positions x hd): both run on the tensor cores as warp-level bf16 m16n8k16 MMAs with
+// fp32 accumulation (the heads are the M rows, padded to 16).  q and P enter as bf16 pairs
+// (rounded value and the bf16 rounding of the rest, each pair multiplied separately: about 2^-17
+// relative); K and V are the cache's bf16 values, exact.  Scores: warp w takes positions
+// 8w..8w+7; P V: warp w takes head dimensions hd/8 * w onwards.
 #pragma once
 
 #include <math.h>

@@ -7,8 +7,9 @@
 // until the process exits, and every call on that GPU shares it.
 //
 // Set-up happens on the first call on each device (with that device current): the array's
-// device address is looked up with cudaGetSymbolAddress and its ticket cleared with a
-// synchronous cudaMemset, so that first call belongs before any stream capture.  The last
+// device address is looked up with cudaGetSymbolAddress, its ticket cleared with cudaMemset
+// and the device synchronized (the memset is ordered only on the legacy default stream), so that
+// first call belongs before any stream capture.  The last
 // block of each launch puts the ticket back to zero; the candidates are rewritten by every
 // launch before they are read.  The array keeps the last call's contents, and calls that
 // overlap on the GPU (different streams with no ordering between them) race on it.
@@ -44,7 +45,8 @@ std::mutex g_setup_mutex;
 unsigned char *g_scratch_dev[NA_MAX_DEVICES] = {};
 
 // The device address of the scratch on the current device, set up once per device: the symbol's
-// address is looked up and the ticket cleared (the kernel leaves it at zero after every call).
+// address is looked up and the ticket cleared, and the device is synchronized so that the clear has
+// finished before any stream uses it (the kernel leaves the ticket at zero after every call).
 int scratch_for_current_device(unsigned char **out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= NA_MAX_DEVICES) {
@@ -59,7 +61,10 @@ int scratch_for_current_device(unsigned char **out) {
       cudaGetLastError();
       return KFL_ERR_CUDA;
     }
+    // cudaMemset is ordered only on the legacy default stream and may return before it is done;
+    // waiting for the device makes the clear complete before a call on any stream reads it
     e = cudaMemset(static_cast<unsigned char *>(p) + NA_CAND_BYTES, 0, 256);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
       cudaGetLastError();
       return KFL_ERR_CUDA;

@@ -1,63 +1,59 @@
-// Block placement over a ring (host code): Algorithm 1 (Partition), head placement by
-// rotation, the admission tiers, the evaluation's baseline divisions and the per-device block
+// Block placement over a ring (host code): the exact fixed-order division of Section V-B, head
+// placement by rotation, the admission tiers, the evaluation's baseline divisions and the per-device block
 // limit.  See include/kafila_plan.h for the contract of each entry point.
 #include <algorithm>
 #include <cmath>
+#include <functional>
 #include <limits>
+#include <queue>
+#include <utility>
 #include <vector>
 
 #include "../../include/kafila_plan.h"
 
 namespace {
 
-// The cost of n blocks on device i, written once so that the candidates and every test against
-// a bound evaluate the same expression (a candidate is then never rejected by rounding).
+// The cost of n blocks on device i (Eq. 2), written once so that every cost compared or returned
+// is the same expression.
 inline double cost(double fixed, double per, int n) { return fixed + static_cast<double>(n) * per; }
 
-// The largest n in [0, cap] with cost(fixed, per, n) <= tau (cost is increasing in n).
-int most_blocks_within(double fixed, double per, double tau, int cap) {
-  if (cap <= 0 || cost(fixed, per, 0) > tau) return 0;
-  double q = std::floor((tau - fixed) / per);
-  int n = q >= static_cast<double>(cap) ? cap : (q < 0.0 ? 0 : static_cast<int>(q));
-  while (n < cap && cost(fixed, per, n + 1) <= tau) ++n;
-  while (n > 0 && cost(fixed, per, n) > tau) --n;
-  return n;
-}
-
-// The Feasible pass of Algorithm 1 for bound tau: left to right, each device takes as many blocks
-// as the bound and its limit allow while leaving one for every device after it.
-bool feasible(int k, int m, const double *fixed, const double *per, const int *lim, double tau, int *n) {
-  int left = k;
-  for (int i = 0; i < m; ++i) {
-    if (fixed[i] > tau) return false;
-    const int ni = std::min(most_blocks_within(fixed[i], per[i], tau, lim[i]), left - (m - 1 - i));
-    if (ni < 1) return false;
-    n[i] = ni;
-    left -= ni;
-  }
-  return left == 0;
-}
-
+// Fixed-order chain division (Section V-B, "Block placement"): k contiguous blocks over devices
+// 0..m-1 in ring order, device i holding 1 <= n_i <= lim(i) blocks at cost(i, n_i), minimizing
+// the largest cost.  Which blocks a device holds does not change its cost, only how many, so any
+// counts within the limits that sum to k are a valid chain.
+//
+// Every device starts with its one obligatory block; the other k - m are handed out one at a
+// time, each to the device whose cost after taking it is lowest (the lower ring index on ties).
+// A device's successive costs never decrease, so the handed-out blocks are the k - m cheapest
+// increments that any division could take, and the resulting maximum is the smallest any
+// division reaches.  The bottleneck is the maximum of costs of the returned division itself,
+// evaluated with the same expression as every other cost, so it is exactly attained.
 int partition_impl(int k, int m, const double *fixed, const double *per, const int *lim, int *n_out,
                    double *tau_out) {
-  // the bottleneck of any division is fixed(i) + n per(i) for some device i and count n
-  std::vector<double> cand;
-  for (int i = 0; i < m; ++i)
-    for (int n = 1; n <= std::min(k, lim[i]); ++n) cand.push_back(cost(fixed[i], per[i], n));
-  std::sort(cand.begin(), cand.end());
-  std::vector<int> n(m);
-  // smallest feasible candidate (feasibility is monotone in the bound)
-  size_t lo = 0, hi = cand.size();
-  while (lo < hi) {
-    const size_t mid = lo + (hi - lo) / 2;
-    if (feasible(k, m, fixed, per, lim, cand[mid], n.data()))
-      hi = mid;
-    else
-      lo = mid + 1;
+  if (m > k) return KFL_ERR_INFEASIBLE;
+  long long room = 0;
+  for (int i = 0; i < m; ++i) {
+    if (lim[i] < 1) return KFL_ERR_INFEASIBLE;
+    room += std::min(lim[i], k);
   }
-  if (lo == cand.size()) return KFL_ERR_INFEASIBLE;
-  feasible(k, m, fixed, per, lim, cand[lo], n_out);
-  *tau_out = cand[lo];
+  if (room < k) return KFL_ERR_INFEASIBLE;
+  using Next = std::pair<double, int>;  // (cost with one more block, device)
+  std::priority_queue<Next, std::vector<Next>, std::greater<Next>> next;
+  double tau = -std::numeric_limits<double>::infinity();
+  for (int i = 0; i < m; ++i) {
+    n_out[i] = 1;
+    tau = std::max(tau, cost(fixed[i], per[i], 1));
+    if (lim[i] > 1) next.push({cost(fixed[i], per[i], 2), i});
+  }
+  for (int given = m; given < k; ++given) {
+    const Next t = next.top();
+    next.pop();
+    const int i = t.second;
+    ++n_out[i];
+    tau = std::max(tau, t.first);
+    if (n_out[i] < lim[i]) next.push({cost(fixed[i], per[i], n_out[i] + 1), i});
+  }
+  *tau_out = tau;
   return KFL_OK;
 }
 

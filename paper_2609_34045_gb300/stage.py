@@ -342,7 +342,8 @@ def kfl_synth_fill(dst, n: int, seed: int, tag: int, kind: int, c: float, mean: 
 # ---- planner (include/kafila_plan.h): host code, no GPU needed ------------------------------
 
 def kfl_partition(k: int, fixed, per, lim):
-    """Algorithm 1: (block counts, bottleneck), or raises KflError (KFL_ERR_INFEASIBLE)."""
+    """The exact fixed-order division of section V-B: (block counts, bottleneck), or raises
+    KflError (KFL_ERR_INFEASIBLE)."""
     import numpy as np
     m = len(fixed)
     f = np.ascontiguousarray(fixed, dtype=np.float64)

@@ -1,4 +1,4 @@
-"""Ring planner (Algorithm 1, head rotation, admission tiers): the brute-force oracle pinned by
+"""Ring planner (the exact fixed-order division, head rotation, admission tiers): the brute-force oracle pinned by
 hand-derived cases, then the C library's planner against the oracle on random instances.  Host
 code only: no GPU."""
 import math
