@@ -5,10 +5,13 @@ One step = one decode step of the 7B-shaped body stage (blocks [0, 14) of a 28-b
 context 2048 pre-filled) unless --config picks another workload.  Each timed step decodes the
 next position of the workload's 64-step run (positions wrap after 64 steps).
 
-Prints one JSON line: metric "stage decode us/layer/token" (lower is better), the roofline of
-the dominant kernel (gate/up GEMV) against the measured HBM copy bandwidth, the whole step's
-HBM fraction, an end-to-end figure through the host-buffer C-ABI call, SM clocks sampled
-during the timed region, and the CPU oracle timed on a bounded sample (cpu_baseline).
+Prints one JSON line: metric "stage decode us/layer/token" (lower is better; the median of
+--reps timed regions of --steps steps), the roofline of the dominant kernel (gate/up GEMV)
+against the measured HBM copy bandwidth, the whole step's HBM fraction, an end-to-end figure
+through the host-buffer C-ABI call, SM clocks sampled during the timed regions, and the CPU
+oracle timed on a bounded sample (cpu_baseline).  With the default workload, ``also`` carries
+the 32B-shaped head (b = 1), the 72B-shaped body with four ragged users (b = 4) and the 80-block
+int4 72B-shaped model (b = 1 and b = 4), each timed the same way.
 
 ``--impl reference`` times the CPU oracle instead (this workload has no runnable reference
 implementation: the paper ships none).
@@ -35,13 +38,16 @@ UNIT = "us/layer/token"
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", type=int, default=2)
     ap.add_argument("--profile-steps", type=int, default=20)
     ap.add_argument("--e2e-steps", type=int, default=500)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--reps", type=int, default=5, help="timed regions of --steps steps each (median reported)")
+    ap.add_argument("--no-also", action="store_true",
+                    help="skip the other workloads (32B head, 72B body b=4, 72B int4 b=1 and b=4)")
     ap.add_argument("--ring", action="store_true",
                     help="ring emulation: the 7B-shaped model as 4 stages of 7 blocks and the head's return "
                          "leg, 4 users served pipelined (one stream per stage) vs one at a time vs batched")
@@ -420,6 +426,134 @@ def cost_model(points, probe_gbs, o_ms):
     return out
 
 
+def step_inputs(work):
+    """Device tensors of every step's positions and inputs (token ids, else hidden states)."""
+    import numpy as np
+    import torch
+
+    from paper_2609_34045_gb300 import workload as wl
+    m, b = work.model, work.batch
+    pos_all = torch.tensor(np.stack([wl.positions(work, s) for s in range(work.steps)]), dtype=torch.int32,
+                           device="cuda")
+    if work.embed_in:
+        ids_all = torch.tensor(np.stack([wl.token_ids(work.seed, wl.ids_tag(s), b, m.vocab)
+                                         for s in range(work.steps)]), dtype=torch.int32, device="cuda")
+        return pos_all, ids_all, None
+    hid_all = torch.tensor(np.stack([wl.hidden_in(m, s, b, work.seed) for s in range(work.steps)]),
+                           dtype=torch.float32, device="cuda")
+    return pos_all, None, hid_all
+
+
+def time_steps(st, work, inputs, steps, warmup, reps, stream, dist, clocks=None):
+    """Decode steps of stage ``st``: ``warmup`` untimed, then ``reps`` timed regions of exactly
+    ``steps`` steps, each bracketed by a barrier and a device synchronization, timed with CUDA
+    events on the launching stream (the max over ranks).  Returns (ms per step of each region,
+    clock record or None)."""
+    import torch
+
+    from paper_2609_34045_gb300 import stage as K
+    pos_all, ids_all, hid_all = inputs
+    b, d = work.batch, work.model.d_model
+    out = torch.empty(b, d, dtype=torch.float32, device="cuda")
+    nxt = torch.empty(b, dtype=torch.int32, device="cuda") if work.logits_out else None
+
+    def step(s):
+        i = s % work.steps
+        K.kfl_stage_decode(st, ids_all[i] if ids_all is not None else None,
+                           hid_all[i] if hid_all is not None else None, pos_all[i], b, out, nxt,
+                           stream.cuda_stream)
+
+    for s in range(warmup):
+        step(s)
+    torch.cuda.synchronize()
+    if clocks is not None:
+        clocks.start()
+        time.sleep(0.3)  # let the sampler take its first reading
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    times = []
+    for r in range(reps):
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for s in range(steps):
+            step(warmup + r * steps + s)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        times.append(max_over_ranks(ev0.elapsed_time(ev1) / steps, dist, "cuda"))
+    clk = clocks.stop() if clocks is not None else None
+    status = K.kfl_stage_status(st)
+    if status != 0:
+        raise RuntimeError(f"device reported {K.kfl_strerror(status)} during the benchmark")
+    return times, clk
+
+
+def per_kernel_profile(st, work, inputs, n_steps, stream):
+    """Per-kernel time (the library's profile mode: CUDA events around each launch on the
+    stage's stream) and achieved GB/s of each kernel kind."""
+    from paper_2609_34045_gb300 import stage as K
+    K.kfl_stage_profile(st, True)
+    time_steps(st, work, inputs, n_steps, 0, 1, stream, None)
+    prof = K.kfl_stage_profile_read(st)
+    K.kfl_stage_profile(st, False)
+    kinds = [k for k in ("qkv", "attn", "oproj", "gateup", "down", "lmhead") if prof[k][1] > 0]
+    return {k: {"us": 1e3 * prof[k][0] / prof[k][1], "launches_per_step": prof[k][1] / n_steps,
+                "gbs": (kernel_bytes(work, k) / (prof[k][0] / prof[k][1] * 1e-3) / 1e9) if prof[k][0] else None}
+            for k in kinds}
+
+
+def also_workloads(args, stream, local):
+    """The batch-4 and int4 workloads measured in the same run, each as its own timed regions:
+    the 32B-shaped head (b = 1), the 72B-shaped body with four ragged users (b = 4), and the
+    80-block int4 72B-shaped model at b = 1 and b = 4 (one stage with four users' KV slots; b = 1
+    decodes user 0).  Per workload: ms per step (median, min, max over the regions), the step's
+    algorithmic bytes over its time, per-kernel times, and the clocks during its regions."""
+    import dataclasses
+
+    from paper_2609_34045_gb300 import device_inputs as di
+    from paper_2609_34045_gb300 import stage as K
+    from paper_2609_34045_gb300 import workload as wl
+
+    peak, _ = measured_peaks()
+    also_steps = max(1, min(args.steps, 40))
+    res = {}
+
+    def measure(work, st):
+        inputs = step_inputs(work)
+        times, clk = time_steps(st, work, inputs, also_steps, max(3, args.warmup), args.reps, stream, None,
+                                ClockSampler(local))
+        ms = statistics.median(times)
+        sb = work.step_bytes(0)
+        gbs = sb / (ms * 1e-3) / 1e9
+        return {"workload": work.name, "batch": work.batch, "stage_layers": [work.l0, work.l1],
+                "weights": work.model.weight_fmt, "ctx": list(work.contexts),
+                "ms_per_step": ms, "ms_per_step_min": min(times), "ms_per_step_max": max(times),
+                "regions": len(times), "steps_per_region": also_steps,
+                "us_per_layer_token": ms * 1e3 / (max(1, work.n_layers) * work.batch),
+                "tokens_per_s": work.batch / (ms * 1e-3),
+                "step_roofline": {"bytes_per_step": sb, "achieved_gbs": gbs, "frac_of_measured": gbs / peak,
+                                  "frac_of_8tbs": gbs / 8000.0},
+                "per_kernel": per_kernel_profile(st, work, inputs, min(args.profile_steps, 10), stream),
+                "clocks": clk}
+
+    for n in (3, 4):
+        work = wl.CONFIGS[n]
+        st = K.kfl_stage_create(K.model_cfg(work.model, work.max_ctx, work.batch), work.l0, work.l1,
+                                (K.KFL_EMBED_IN if work.embed_in else 0) | (K.KFL_LOGITS_OUT if work.logits_out else 0))
+        di.load_stage_seeded(st, work)
+        res[f"config{n}"] = measure(work, st)
+        K.kfl_stage_destroy(st)
+    w6 = wl.CONFIGS[6]
+    st = K.kfl_stage_create(K.model_cfg(w6.model, w6.max_ctx, 4), w6.l0, w6.l1, K.KFL_IS_HEAD)
+    di.load_stage_seeded(st, w6)
+    w5 = dataclasses.replace(wl.CONFIGS[5], splits=())
+    assert w5.max_ctx == w6.max_ctx and w5.contexts[0] == w6.contexts[0]
+    res["config5"] = measure(w5, st)
+    res["config6"] = measure(dataclasses.replace(w6, splits=()), st)
+    K.kfl_stage_destroy(st)
+    return res
+
+
 def run_ours(args, work):
     import numpy as np
     import torch
@@ -446,70 +580,28 @@ def run_ours(args, work):
     b, d = work.batch, m.d_model
     stream = torch.cuda.current_stream()
     n_pos = work.steps
-    pos_all = torch.tensor(np.stack([wl.positions(work, s) for s in range(n_pos)]), dtype=torch.int32,
-                           device="cuda")
-    if work.embed_in:
-        ids_all = torch.tensor(np.stack([wl.token_ids(work.seed, wl.ids_tag(s), b, m.vocab) for s in range(n_pos)]),
-                               dtype=torch.int32, device="cuda")
-        hid_all = None
-    else:
-        ids_all = None
-        hid_all = torch.tensor(np.stack([wl.hidden_in(m, s, b, work.seed) for s in range(n_pos)]),
-                               dtype=torch.float32, device="cuda")
-    out = torch.empty(b, d, dtype=torch.float32, device="cuda")
-    nxt = torch.empty(b, dtype=torch.int32, device="cuda") if work.logits_out else None
+    inputs = step_inputs(work)
+    pos_all, ids_all, hid_all = inputs
 
-    def step(s):
-        i = s % n_pos
-        K.kfl_stage_decode(st, ids_all[i] if ids_all is not None else None,
-                           hid_all[i] if hid_all is not None else None, pos_all[i], b, out, nxt,
-                           stream.cuda_stream)
-
-    for s in range(args.warmup):
-        step(s)
-    torch.cuda.synchronize()
+    times, clk = time_steps(st, work, inputs, args.steps, args.warmup, args.reps, stream, dist,
+                            ClockSampler(local))
+    ms = statistics.median(times)
     if dist:
         dist.barrier()
-    clocks = ClockSampler(local)
-    clocks.start()
-    time.sleep(0.3)  # let the sampler take its first reading
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    torch.cuda.synchronize()
-    ev0.record(stream)
-    for s in range(args.steps):
-        step(s)
-    ev1.record(stream)
-    torch.cuda.synchronize()
-    clk = clocks.stop()
-    ms = ev0.elapsed_time(ev1) / args.steps
-    ms = max_over_ranks(ms, dist, "cuda")
-    if dist:
-        dist.barrier()
-    status = K.kfl_stage_status(st)
-    if status != 0:
-        raise RuntimeError(f"device reported {K.kfl_strerror(status)} during the benchmark")
 
     n_layers = max(1, work.n_layers)
     value = ms * 1e3 / (n_layers * b) / world
     launches = K.kfl_stage_launches_per_step(st, b) * args.steps
 
     # per-kernel timing (kernels one by one with CUDA events on the launching stream)
-    K.kfl_stage_profile(st, True)
-    for s in range(args.profile_steps):
-        step(s)
-    prof = K.kfl_stage_profile_read(st)
-    K.kfl_stage_profile(st, False)
-    kinds = [k for k in ("qkv", "attn", "oproj", "gateup", "down", "lmhead") if prof[k][1] > 0]
-    dom = max(kinds, key=lambda k: prof[k][0])
-    dom_ms = prof[dom][0] / prof[dom][1]
+    per_kernel = per_kernel_profile(st, work, inputs, args.profile_steps, stream)
+    dom = max(per_kernel, key=lambda k: per_kernel[k]["us"] * per_kernel[k]["launches_per_step"])
+    dom_ms = per_kernel[dom]["us"] * 1e-3
     dom_bytes = kernel_bytes(work, dom)
     peak, peak_kind = measured_peaks()
     achieved = dom_bytes / (dom_ms * 1e-3) / 1e9
     step_bytes = work.step_bytes(0)
     step_gbs = step_bytes / (ms * 1e-3) / 1e9
-    per_kernel = {k: {"us": 1e3 * prof[k][0] / prof[k][1], "launches_per_step": prof[k][1] / args.profile_steps,
-                      "gbs": (kernel_bytes(work, k) / (prof[k][0] / prof[k][1] * 1e-3) / 1e9) if prof[k][0] else None}
-                  for k in kinds}
 
     # end to end through the host-buffer C-ABI call (pinned host memory, copies timed)
     e2e_steps = min(args.e2e_steps, args.steps)
@@ -551,6 +643,11 @@ def run_ours(args, work):
         cost = cost_model(points, measured_peaks()[0], empty_stage_ms(work, stream))
         if "fitted" in cost:
             cost["plan_example"] = plan_example(work, cost["fitted"])
+    K.kfl_stage_destroy(st)
+
+    also = None
+    if world == 1 and args.config == 2 and args.layers == 0 and not args.no_also:
+        also = also_workloads(args, stream, local)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -565,10 +662,14 @@ def run_ours(args, work):
             "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded)",
             "config": {"workload": work.name, "stage_layers": [work.l0, work.l1], "batch": b,
                        "ctx": list(work.contexts), "weights": m.weight_fmt,
+                       "arithmetic": ("fp32 FMA on bf16 weights" if m.weight_fmt == "bf16"
+                                      else "fp16 x int4-as-fp16 tensor-core MMA, fp32 accumulation"),
                        "l2": "inputs larger than L2 (weights streamed once per step)",
                        "parallelism": f"replicas x{world}",
+                       "timing": f"median of {len(times)} timed regions of {args.steps} steps each",
                        "execution": ("persistent stage kernel" if launches == 3 * args.steps
                                      else "one kernel per phase, CUDA graph + programmatic dependent launch")},
+            "repeats": {"ms_per_step": times, "median": ms, "min": min(times), "max": max(times)},
             "tokens_per_s": b * world / (ms * 1e-3),
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "peak_kind": f"{peak_kind} copy (MEASURED_PEAKS.json hbm_gbs)",
@@ -579,15 +680,16 @@ def run_ours(args, work):
             "per_kernel": per_kernel,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "steps": e2e_steps},
-            "gpu_launches": launches,
+            "gpu_launches": launches * len(times),
             "clocks": clk,
             "cpu_baseline": cpu,
         }
         if splits is not None:
             line["splits"] = splits
             line["cost_model"] = cost
+        if also is not None:
+            line["also"] = also
         print(json.dumps(line), flush=True)
-    K.kfl_stage_destroy(st)
     if dist:
         dist.destroy_process_group()
     return 0

@@ -39,9 +39,10 @@ __all__ = [
 def bf16_to_f64(bits) -> np.ndarray:
     """bf16 bit patterns -> fp64.  A bf16 value is the top 16 bits of an fp32 value, so the
     conversion is exact."""
-    b = np.asarray(bits, dtype=np.uint16)
+    u = np.asarray(bits, dtype=np.uint16).astype(np.uint32)
+    u <<= np.uint32(16)
     with np.errstate(invalid="ignore"):
-        return (b.astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
+        return u.view(np.float32).astype(np.float64)
 
 
 def round_to_bf16(x) -> np.ndarray:
@@ -58,14 +59,19 @@ def round_to_bf16(x) -> np.ndarray:
     return r.astype(np.uint16)
 
 
+# the signed value of each 4-bit pattern (two's complement: 0x8 -> -8, 0xF -> -1)
+_NIBBLE_VALUE = np.array([n - 16 if n >= 8 else n for n in range(16)], dtype=np.int8)
+
+
 def int4_codes(words) -> np.ndarray:
     """Signed 4-bit codes of packed words: code ``j`` of a uint32 word is bits [4j, 4j+4),
     low nibble first along K, two's complement (0x8 -> -8, 0xF -> -1).  Returns int8
-    ``[..., 8 * words]``."""
+    ``[..., 8 * words]``.  Byte ``i`` of a word (little-endian) holds codes 2i (its low nibble)
+    and 2i + 1 (its high nibble)."""
     w = np.asarray(words, dtype=np.uint32)
-    nib = np.stack([(w >> np.uint32(4 * j)) & np.uint32(0xF) for j in range(8)], axis=-1).astype(np.int16)
-    nib = np.where(nib >= 8, nib - 16, nib).astype(np.int8)
-    return nib.reshape(*w.shape[:-1], w.shape[-1] * 8)
+    b = np.ascontiguousarray(w, dtype="<u4").view(np.uint8).reshape(*w.shape, 4)
+    q = np.stack([_NIBBLE_VALUE[b & 0xF], _NIBBLE_VALUE[b >> 4]], axis=-1)
+    return q.reshape(*w.shape[:-1], w.shape[-1] * 8)
 
 
 def dequant_int4_g64(words, scales) -> np.ndarray:
@@ -73,7 +79,8 @@ def dequant_int4_g64(words, scales) -> np.ndarray:
     ``w[n][k] = code(n, k) * scale[n][k // 64]``."""
     q = int4_codes(words).astype(np.float64)
     s = bf16_to_f64(scales)
-    return q * np.repeat(s, 64, axis=-1)
+    groups = q.reshape(*q.shape[:-1], q.shape[-1] // 64, 64)  # [..., group][64 codes]
+    return (groups * s[..., None]).reshape(q.shape)
 
 
 def matrix_f64(m) -> np.ndarray:

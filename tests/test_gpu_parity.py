@@ -11,7 +11,8 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_helpers import Pair, ensure_built
+import oracle
+from gpu_helpers import HIDDEN_TOL, ID_MARGIN, Pair, ensure_built
 from paper_2609_34045_gb300 import stage as K
 from paper_2609_34045_gb300 import workload as wl
 
@@ -242,17 +243,7 @@ def test_device_generator_is_bit_identical_to_host():
 
 
 # ---------------------------------------------------------------------------- full widths
-
-def test_config2_width_bench_launch_shape():
-    """The 7B-shaped body stage at its full width and context, b = 1 (the benchmark's kernels
-    and launch shapes), on two of its blocks."""
-    w = wl.CONFIGS[2]
-    p = Pair(w.model, 0, 2, 0, 1, w.contexts, w.max_ctx, w.seed, device_weights=True)
-    for s in range(2):
-        p.step(s, hidden=wl.hidden_in(w.model, s, 1, w.seed))
-    p.compare_kv()
-    p.close()
-
+# (every block of each benchmark workload against the oracle: test_gpu_deep.py)
 
 def test_cluster_combine_agrees_with_the_ticket_combine(monkeypatch):
     """At the 7B widths the Q/K/V and O GEMVs run as clusters of two CTAs (each half of a row
@@ -286,23 +277,6 @@ def test_cluster_combine_agrees_with_the_ticket_combine(monkeypatch):
         for a, b in ((o1, o0), (c1, c0)):
             rms = torch.sqrt(torch.mean(b.double() ** 2)).item()
             assert torch.max(torch.abs(a.double() - b.double())).item() <= 1e-5 * rms
-
-
-def test_config3_width_head_with_full_vocab():
-    """The 32B-shaped head: embedding and lm_head over the full 152064-token vocabulary."""
-    w = wl.CONFIGS[3]
-    p = Pair(w.model, 56, 57, K.KFL_IS_HEAD, 1, w.contexts, w.max_ctx, w.seed, device_weights=True)
-    _greedy(p, 2, wl.first_token_ids(w.model, 1, w.seed))
-    p.close()
-
-
-def test_config4_width_four_ragged_users():
-    w = wl.CONFIGS[4]
-    p = Pair(w.model, 0, 1, 0, 4, w.contexts, w.max_ctx, w.seed, device_weights=True)
-    for s in range(2):
-        p.step(s, hidden=wl.hidden_in(w.model, s, 4, w.seed))
-    p.compare_kv()
-    p.close()
 
 
 def test_config5_width_int4_head_b4():
@@ -358,10 +332,24 @@ def test_int4_deep_stack_finite_and_split_bit_exact(batch):
 RING = wl.ModelShape(n_layers_total=5, d_model=320, n_heads=6, n_kv_heads=2, head_dim=64, ffn=712, vocab=1000)
 
 
+def _ring_oracle(work, l0, l1, embed, logits, users):
+    """The oracle stage of blocks [l0, l1) of ``work.model`` with ``users`` KV slots filled over
+    the workload's contexts (host weights from the same seeded generator)."""
+    ora = oracle.OracleStage(work.model, l0, l1, embed, logits, users, work.max_ctx)
+    for i, layer in enumerate(range(l0, l1)):
+        ora.load_layer(i, wl.layer_weights(work.model, layer, work.seed))
+        for u in range(users):
+            ora.set_kv(i, u, *wl.kv_prefill(work.model, layer, u, work.contexts[u], work.seed))
+    if embed or logits:
+        ora.load_head(wl.head_weights(work.model, work.seed, embed, logits))
+    return ora
+
+
 def test_decode_users_addresses_the_users_kv_slots():
     """kfl_stage_decode_users: batch row b reads and appends user users[b]'s KV slot.  Users 2 and
-    0 served as rows 0 and 1 give the same outputs as rows 0 and 1 of a batch in slot order, and
-    only slots 2 and 0 change."""
+    0 served as rows 0 and 1 match the oracle's decode with the same users mapping (every block's
+    hidden state and the new K/V rows), give the same outputs as rows 0 and 1 of a batch in slot
+    order, and change only slots 2 and 0."""
     from paper_2609_34045_gb300 import device_inputs as dev_in
     w = wl.Workload("ring-users", RING, 0, 2, False, False, 3, (17, 40, 65), 4, 31)
     cfg = K.model_cfg(RING, w.max_ctx, 3)
@@ -370,6 +358,8 @@ def test_decode_users_addresses_the_users_kv_slots():
     for users in ([2, 0], None):
         st = K.kfl_stage_create(cfg, 0, 2, 0)
         dev_in.load_stage_seeded(st, w)
+        cap = torch.zeros(2, 3, RING.d_model, device="cuda")
+        K.kfl_stage_debug_capture(st, cap)
         before = [_kv(st, u, RING) for u in range(3)]
         rows = users if users is not None else [0, 1]
         pos = torch.tensor([w.contexts[u] for u in rows], dtype=torch.int32, device="cuda")
@@ -381,6 +371,28 @@ def test_decode_users_addresses_the_users_kv_slots():
         after = [_kv(st, u, RING) for u in range(3)]
         changed = [not np.array_equal(before[u], after[u]) for u in range(3)]
         outs.append((out.cpu().numpy(), changed))
+        if users is not None:
+            ora = _ring_oracle(w, 0, 2, False, False, 3)
+            o = ora.decode(pos.cpu().numpy(), hidden_in=hid.cpu().numpy(), users=users, capture=True)
+            c = cap.cpu().numpy()
+            for layer in range(2):
+                for r in range(2):
+                    ref = o["per_layer"][layer][r]
+                    assert np.max(np.abs(c[layer, r] - ref)) <= HIDDEN_TOL * np.sqrt(np.mean(ref * ref)), (layer, r)
+            for r in range(2):
+                ref = o["hidden_out"][r]
+                assert np.max(np.abs(out[r].cpu().numpy() - ref)) <= HIDDEN_TOL * np.sqrt(np.mean(ref * ref))
+            for layer in range(2):
+                for r, u in enumerate(users):
+                    k = np.zeros((RING.n_kv_heads, w.max_ctx, RING.head_dim), dtype=np.uint16)
+                    v = np.zeros_like(k)
+                    K.kfl_kv_read(st, layer, u, k, v, False)
+                    p_ = w.contexts[u]
+                    for g, r_ in ((k, ora.k_cache), (v, ora.v_cache)):
+                        gg = oracle.bf16_to_f64(g[:, p_])
+                        rr = oracle.bf16_to_f64(r_[layer, u][:, p_])
+                        rms = np.sqrt(np.mean(rr * rr))
+                        assert np.all(np.abs(gg - rr) <= HIDDEN_TOL * rms + 2.0 ** -7 * np.abs(rr))
         assert K.kfl_stage_status(st) == 0
         K.kfl_stage_destroy(st)
     (o_perm, ch_perm), (o_id, ch_id) = outs
@@ -401,7 +413,9 @@ def _kv(st, u, model):
 def test_ring_generates_what_one_stage_does(sequential):
     """Three users around a ring of stages (2, 3 blocks) and the head's return leg, each stage on
     its own stream: every user's greedy tokens equal those of the whole model as one head stage
-    serving that user (stage splits are exact)."""
+    serving that user (stage splits are exact), and the oracle's greedy token at every step
+    (the oracle fed the ring's previous token; where its top-2 margin is within 1e-2, the ring's
+    token must be one of its near-largest logits)."""
     from paper_2609_34045_gb300 import device_inputs as dev_in
     from paper_2609_34045_gb300.ring import Ring
     w = wl.Workload("ring", RING, 0, 5, True, True, 3, (12, 70, 33), 6, 41)
@@ -425,3 +439,14 @@ def test_ring_generates_what_one_stage_does(sequential):
             tok.copy_(nxt)
     assert K.kfl_stage_status(st) == 0
     K.kfl_stage_destroy(st)
+    ora = _ring_oracle(ring.work, 0, 5, True, True, 3)
+    for u in range(3):
+        tok = int(first[u])
+        for t in range(5):
+            o = ora.decode(np.array([ring.work.contexts[u] + t]), token_ids=np.array([tok]), users=[u])
+            if o["margins"][0] > ID_MARGIN:
+                assert got[t][u] == int(o["next_ids"][0]), (u, t, got[t][u], o["next_ids"])
+            else:
+                z = o["logits"][0]
+                assert z[got[t][u]] >= np.max(z) - 2 * ID_MARGIN
+            tok = got[t][u]

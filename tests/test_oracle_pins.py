@@ -390,6 +390,28 @@ def pin_prefill_in_two_calls():
     assert np.array_equal(a.k_cache, b.k_cache) and np.array_equal(a.v_cache, b.v_cache)
 
 
+def pin_steps_of_several_users_in_one_call():
+    # two users' rows over three steps in one call (rows at positions P_u + s, each on its user's
+    # slot) equal the three steps one at a time: a row sees its user's rows of earlier steps and
+    # no later ones, and the other user's slot not at all
+    def stage():
+        st = oracle.OracleStage(SMALL, 0, 3, False, False, 6, 32)
+        for i in range(3):
+            st.load_layer(i, wl.layer_weights(SMALL, i, 78))
+            for u, n in enumerate((5, 11)):
+                st.set_kv(i, u, *wl.kv_prefill(SMALL, i, u, n, 78))
+        return st
+    a, b = stage(), stage()
+    hid = [wl.hidden_in(SMALL, s, 2, 78) for s in range(3)]
+    pos = [np.array([5 + s, 11 + s]) for s in range(3)]
+    one = a.decode(np.concatenate(pos), hidden_in=np.concatenate(hid), users=[0, 1] * 3, capture=True)
+    for s in range(3):
+        o = b.decode(pos[s], hidden_in=hid[s], capture=True)
+        assert np.allclose(one["hidden_out"][2 * s:2 * s + 2], o["hidden_out"], rtol=1e-12, atol=1e-13)
+        assert np.allclose(one["per_layer"][:, 2 * s:2 * s + 2], o["per_layer"], rtol=1e-12, atol=1e-13)
+    assert np.array_equal(a.k_cache, b.k_cache) and np.array_equal(a.v_cache, b.v_cache)
+
+
 SMALL_INT4 = wl.ModelShape(n_layers_total=2, d_model=128, n_heads=4, n_kv_heads=2, head_dim=32, ffn=192,
                            vocab=40, weight_fmt="int4_g64")
 
@@ -406,7 +428,8 @@ def pin_int4_prefill_vs_torch():
 PINS = [pin_bf16_golden, pin_bf16_vs_torch, pin_int4_exhaustive, pin_int4_groups, pin_gemv_bruteforce,
         pin_rms_norm, pin_rope, pin_softmax, pin_attention, pin_silu, pin_argmax, pin_stage_vs_torch,
         pin_kv_slots, pin_stage_split_associativity, pin_int4_stage_vs_torch, pin_prefill_vs_torch,
-        pin_prefill_is_sequential_decode, pin_int4_prefill_vs_torch, pin_prefill_in_two_calls]
+        pin_prefill_is_sequential_decode, pin_int4_prefill_vs_torch, pin_prefill_in_two_calls,
+        pin_steps_of_several_users_in_one_call]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
