@@ -52,7 +52,10 @@ extern "C" {
  * epsilon and the RoPE base.  max_ctx is the number of KV slots reserved per user and
  * max_batch the number of users (batch slots); together they are the session's declared
  * context and concurrency, at which the cache is reserved (section V-C, the block limit
- * lim(i); section V-D, admission).  qk_norm must be 0 (per-head Q/K RMSNorm is not built). */
+ * lim(i); section V-D, admission).  qk_norm: 0, or 1 for Qwen3-family blocks (the models served
+ * in section VI): each head of q and of k is RMS-normalised over head_dim with its own gain (the
+ * layer's q_norm, k_norm; epsilon rms_eps) before RoPE.  A qk_norm stage runs one kernel per
+ * phase (KFL_PERSISTENT is ignored) and prefills through decode steps. */
 typedef struct {
   int n_layers_total, d_model, n_heads, n_kv_heads, head_dim, ffn, vocab;
   float rms_eps, rope_theta;
@@ -68,10 +71,12 @@ typedef struct {
   const void *scales;
 } kfl_matrix;
 
-/* One decoder block's weights: RMSNorm gains (bf16 [d_model]), Q/K/V/O and gate/up/down. */
+/* One decoder block's weights: RMSNorm gains (bf16 [d_model]), Q/K/V/O and gate/up/down, and
+ * with qk_norm the per-head Q and K RMSNorm gains (bf16 [head_dim]; ignored without qk_norm). */
 typedef struct {
   const uint16_t *attn_norm, *ffn_norm;
   kfl_matrix wq, wk, wv, wo, wg, wu, wd;
+  const uint16_t *q_norm, *k_norm;
 } kfl_layer_weights;
 
 /* A stage's weights.  layers[i] is global block l0 + i (n_layers = l1 - l0 entries).  embed

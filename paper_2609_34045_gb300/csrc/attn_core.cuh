@@ -203,7 +203,7 @@ __device__ __forceinline__ void ldsm_x2_trans(uint32_t &r0, uint32_t &r1, const 
 template <int HD>
 __device__ __forceinline__ void attn_out16(const AttnParams &p, int b, int kvh, int G, int og, int od, float4 v,
                                            bool owns, int lane) {
-  if (!p.o16.hi) return;
+  if (!p.o16.base) return;
   act16_put_quad(p.o16, b, ((kvh * G + og) * HD + od) / XCHUNK, v, lane, owns);
 }
 
@@ -412,7 +412,7 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
 
   stamp(TR_W_FIRST);
   if (nc == 1) {
-    if (!p.o16.hi) {
+    if (!p.o16.base) {
       if (hrow) {
         const float il = 1.0f / s_l[gid];
 #pragma unroll

@@ -32,41 +32,71 @@ constexpr int TILE4_BYTES = TILE4_CODE_BYTES + TILE4_SCALE_BYTES;
 __host__ __device__ constexpr int tile_k(int fmt) { return fmt == 0 ? KT : KT4; }
 __host__ __device__ constexpr int tile_bytes(int fmt) { return fmt == 0 ? TILE_BYTES : TILE4_BYTES; }
 // A ring stage holds one weight tile and the activations of its K range: bf16 tiles, the B
-// users' fp32 values; int4 tiles, up to 2 B fp16 source rows (struct Act16: the users' rounded
-// parts, then their rests) at a padded stride, then the tile's per-chunk constants.
+// users' fp32 values; int4 tiles, one K tile's block of its Act16 input (below): the chunk
+// constants, then fp16 source rows at a padded stride.
 constexpr int XCHUNK = 32;                          // elements per scale chunk of an int4 input
 constexpr int X16_SRC_BYTES = KT4 * 2;              // 512
-constexpr int X16_SRC_STRIDE = X16_SRC_BYTES + 32;  // 544: the sources start on different banks
-constexpr int XC_CHUNK_FLOATS = 16;                 // per chunk: [4 lane quads][4]
-constexpr int XC_TILE_BYTES = (KT4 / XCHUNK) * XC_CHUNK_FLOATS * 4;  // 512
+// 576: the sources start on different halves of the banks, so that the 16-byte B-fragment loads of
+// one quarter warp (two sources) fall in distinct banks
+constexpr int X16_SRC_STRIDE = X16_SRC_BYTES + 64;
+constexpr int XC_CHUNK_FLOATS = 32;                 // per chunk: [4 lane quads][8]
+constexpr int XC_TILE_BYTES = (KT4 / XCHUNK) * XC_CHUNK_FLOATS * 4;  // 1024
+// Bytes of one K tile's block of an Act16 (rest: with the rests' rows), and the part of it a
+// GEMV at batch B copies into a ring stage: the constants and the rounded parts of users
+// 0..B-1, or (xsplit) all MAXB rounded parts and the rests of users 0..B-1.
+__host__ __device__ constexpr int act16_tile_bytes(int rest) {
+  return XC_TILE_BYTES + (rest ? 2 : 1) * MAXB * X16_SRC_STRIDE;
+}
+__host__ __device__ constexpr int act16_copy_bytes(int batch, int xsplit) {
+  return XC_TILE_BYTES + (xsplit ? MAXB + batch : batch) * X16_SRC_STRIDE;
+}
 __host__ __device__ constexpr int stage_bytes(int batch, int fmt) {
   return fmt == 0 ? (TILE_BYTES + batch * KT * 4 + 127) / 128 * 128
-                  : (TILE4_BYTES + 2 * batch * X16_SRC_STRIDE + XC_TILE_BYTES + 127) / 128 * 128;
+                  : (TILE4_BYTES + act16_copy_bytes(batch, 1) + 127) / 128 * 128;
 }
 constexpr int STAGE_BYTES_MAX = stage_bytes(MAXB, 0);
 
 // A GEMV input of an int4 stage, in the form the tensor-core tile loop reads (tile_compute_int4).
-// Per user b, row b * ld: x divided by a power of two per XCHUNK elements (m, the multiplier
-// that undoes it, brings the chunk's largest value into [2^14, 2^15)) and rounded to fp16; in
-// each 16-element block, elements 8..15 are also divided by 16 (the decoder makes their weights
-// 16 x larger), and the block is stored in the order of the MMA's B fragments (act16_index).
-// lo (the Q/K/V projection's input only, else NULL): what rounding to fp16 left over, in fp16.
-// xc[chunk][t][0..1]: m of MMA columns 2t, 2t+1; xc[chunk][t][2..3]: minus their offset sums,
-// where column u < 4 is user u's rounded part and column u + 4 its rest, and a column's offset
-// sum is the sum over the chunk of its fp16 values times 1032 (block elements 0..7) or 1152
-// (8..15): what the decoder's offsets add to the MMA's product.
+// Per user b: x divided by a power of two per XCHUNK elements (m, the multiplier that undoes it,
+// brings the chunk's largest value into [2^14, 2^15)) and rounded to fp16; in each 16-element
+// block, elements 8..15 are also divided by 16 (the decoder makes their weights 16 x larger);
+// each 32-element chunk is stored in the order of the MMA's B fragments of its two 16-element K
+// steps (act16_index).  The Q/K/V projection's input also keeps what rounding to fp16 left
+// over (the rest), in fp16.
+// Layout, tile-major so that a ring stage's activations are one contiguous copy: per K tile of
+// KT4 elements a block of act16_tile_bytes(rest) bytes, holding
+//   [0, XC_TILE_BYTES): the chunk constants, per chunk [t][0..7] for MMA columns 2t, 2t+1:
+//     minus their offset sums twice over (the MMA's accumulator quad of rows gid and gid + 8),
+//     then their multipliers m and two unused floats; column u < 4 is user u's rounded part and
+//     column u + 4 its rest, and a column's offset sum is the sum over the chunk of its fp16
+//     values times 1032 (block elements 0..7) or 1152 (8..15): what the decoder's offsets add
+//     to the MMA's product;
+//   then source rows of X16_SRC_STRIDE bytes: rows 0..MAXB-1 the users' rounded parts, rows
+//     MAXB..2 MAXB-1 their rests (rest only).
 struct Act16 {
-  uint16_t *hi;
-  uint16_t *lo;
-  float *xc;
-  int ld;  // elements per user row, a multiple of KT4
+  uint8_t *base;  // NULL: the stage has no int4 input of this kind
+  int ld;         // elements per user row, a multiple of KT4
+  int rest;       // 1: the rests are stored
 };
 
-// Position of element k of a user's row in Act16 order: within a 16-element block, lane quad t
-// of a warp reads the 8 bytes at 4 t: elements 2t, 2t+1 (B fragment register b0) and 2t+8, 2t+9
-// (b1).
+// Position of element k of a user's row in Act16 order: within a 32-element chunk, lane quad t
+// of a warp reads the 16 bytes at 16 t: elements 2t, 2t+1 (B fragment register b0) and 2t+8,
+// 2t+9 (b1) of the chunk's first 16-element block, then the same of its second block.
 __host__ __device__ constexpr int act16_index(int k) {
-  return (k & ~15) + ((k & 7) >> 1) * 4 + ((k & 15) < 8 ? 0 : 2) + (k & 1);
+  return (k & ~31) + ((k & 7) >> 1) * 8 + ((k >> 4) & 1) * 4 + ((k & 15) < 8 ? 0 : 2) + (k & 1);
+}
+
+__host__ __device__ inline uint8_t *act16_tile(const Act16 &a, int kt) {
+  return a.base + (size_t)kt * act16_tile_bytes(a.rest);
+}
+// Element k of source row r (r < MAXB: user r's rounded part; MAXB + u: user u's rest).
+__host__ __device__ inline uint16_t *act16_elem(const Act16 &a, int r, int k) {
+  return reinterpret_cast<uint16_t *>(act16_tile(a, k / KT4) + XC_TILE_BYTES + r * X16_SRC_STRIDE) +
+         act16_index(k % KT4);
+}
+// The constants of chunk ch.
+__host__ __device__ inline float *act16_consts(const Act16 &a, int ch) {
+  return reinterpret_cast<float *>(act16_tile(a, ch / (KT4 / XCHUNK))) + (ch % (KT4 / XCHUNK)) * XC_CHUNK_FLOATS;
 }
 
 // ---- device error word bits ---------------------------------------------------------------
@@ -121,10 +151,14 @@ struct GemvParams {
   const float *rope_cos, *rope_sin;  // [max_ctx][hd/2], or [batch][hd/2] when rope_per_user
   int rope_per_user;
   int n_q_rows, n_kv_rows, head_dim, max_ctx, n_kv_heads;
+  // stages with QK-norm: the projection (rows in GEMV order, after the RMSNorm scale) goes to
+  // qk_raw[b * ld_raw + n] instead, and qknorm_rope_kernel normalises, rotates and appends it
+  float *qk_raw;
+  int ld_raw;
   // int4 weights: the GEMV multiplies fp16 activations on the tensor cores
   Act16 xin;          // this GEMV's input (int4 stages; x and ldx are then unused)
-  Act16 xout;         // RESID / SWIGLU: the output in the same form (int4 stages; hi NULL else)
-  int xsplit;         // the input's rests are multiplied too (Q/K/V projection: xin.lo)
+  Act16 xout;         // RESID / SWIGLU: the output in the same form (int4 stages; base NULL else)
+  int xsplit;         // the input's rests are multiplied too (Q/K/V projection)
   // one kernel per phase: launched as clusters of two CTAs, grid 2 n_rb, each CTA half the K
   // range of one row block; the second hands its partial to the first through distributed
   // shared memory instead of global memory and a ticket
@@ -164,7 +198,7 @@ struct AttnParams {
   const int *slots;          // [batch]: the KV-cache user slot of each batch row
   float *o;                  // [batch][ldo]
   int ldo;
-  Act16 o16;                 // int4 stages: o also in the O projection's input form (hi NULL else)
+  Act16 o16;                 // int4 stages: o also in the O projection's input form (base NULL else)
   float *partial;            // [batch][Hkv][n_chunks][G][hd + 2]
   int *tickets;              // [batch][Hkv]
   int batch, n_heads, n_kv_heads, max_ctx;
@@ -182,7 +216,22 @@ struct AttnParams {
   int trace_grid;
 };
 
-// One phase of the persistent stage kernel: a GEMV (with its epilogue) or an attention pass.
+// QK-norm (per-head RMSNorm of q and k over head_dim, then RoPE, then the KV append) of the
+// Q/K/V projection of stages with qk_norm, between the projection and attention.
+struct QkNormParams {
+  const float *raw;                  // [batch][ld_raw]: q, k, v rows in GEMV order (RoPE pairs adjacent)
+  int ld_raw;
+  const float *g_q, *g_k;            // [hd] gains
+  float *q;                          // [batch][Hq * hd]: normalised, rotated q
+  uint16_t *kcache, *vcache;         // this layer's [max_batch][Hkv][max_ctx][hd]
+  const int *positions, *slots;      // [batch] (a position of -1: the row is invalid)
+  const float *rope_cos, *rope_sin;  // [max_ctx][hd/2]
+  int batch, n_heads, n_kv_heads, head_dim, max_ctx;
+  float eps;
+};
+
+// One phase of a step: a GEMV (with its epilogue) or an attention pass (preceded, in stages with
+// QK-norm, by the QK-norm kernel: qn.raw non-NULL).
 enum PhaseKind : int { PH_GEMV = 0, PH_ATTN = 1 };
 
 struct Phase {
@@ -190,6 +239,7 @@ struct Phase {
   int epi;
   GemvParams g;
   AttnParams a;
+  QkNormParams qn;
 };
 
 struct StageKernelParams {
@@ -437,12 +487,14 @@ __device__ __forceinline__ float f16_to_f32(uint16_t h) {
 
 // Chunk ch's constants for user b (column b: rounded part, column b + 4: rest).
 __device__ __forceinline__ void act16_put_consts(const Act16 &a, int b, int ch, float m, float off_hi, float off_lo) {
-  float *c = a.xc + (size_t)ch * XC_CHUNK_FLOATS;
+  float *c = act16_consts(a, ch);
   const int t = b >> 1, j = b & 1;
-  c[t * 4 + j] = m;
-  c[t * 4 + 2 + j] = -off_hi;
-  c[(t + 2) * 4 + j] = m;
-  c[(t + 2) * 4 + 2 + j] = -off_lo;
+  c[t * 8 + j] = -off_hi;
+  c[t * 8 + 2 + j] = -off_hi;
+  c[t * 8 + 4 + j] = m;
+  c[(t + 2) * 8 + j] = -off_lo;
+  c[(t + 2) * 8 + 2 + j] = -off_lo;
+  c[(t + 2) * 8 + 4 + j] = m;
 }
 
 // Chunk ch of user b of an Act16, one element per lane (x = 0 past the vector's end); the whole
@@ -458,12 +510,12 @@ __device__ __forceinline__ void act16_put_warp(const Act16 &a, int b, int ch, fl
   const float wgt = upper ? 1152.0f : 1032.0f;
   const uint16_t h = f32_to_f16_rn(y);
   const float yh = f16_to_f32(h);
-  const size_t idx = (size_t)b * a.ld + (size_t)ch * XCHUNK + act16_index(lane);
-  a.hi[idx] = h;
+  const int k = ch * XCHUNK + lane;
+  *act16_elem(a, b, k) = h;
   float oh = yh * wgt, ol = 0.f;
-  if (a.lo) {
+  if (a.rest) {
     const uint16_t l = f32_to_f16_rn(y - yh);
-    a.lo[idx] = l;
+    *act16_elem(a, MAXB + b, k) = l;
     ol = f16_to_f32(l) * wgt;
   }
 #pragma unroll
@@ -497,20 +549,19 @@ __device__ __forceinline__ void act16_put_quad(const Act16 &a, int b, int ch, fl
     oh += yh * wgt;
     ol += f16_to_f32(l[i]) * wgt;
   }
-  if (!a.lo) ol = 0.f;
+  if (!a.rest) ol = 0.f;
 #pragma unroll
   for (int off = 4; off > 0; off >>= 1) {
     oh += __shfl_xor_sync(0xffffffffu, oh, off);
     ol += __shfl_xor_sync(0xffffffffu, ol, off);
   }
   if (write) {
-    const size_t row = (size_t)b * a.ld + (size_t)ch * XCHUNK;
-    const int i0 = act16_index(4 * sub), i2 = act16_index(4 * sub + 2);
-    *reinterpret_cast<uint32_t *>(a.hi + row + i0) = (uint32_t)h[0] | ((uint32_t)h[1] << 16);
-    *reinterpret_cast<uint32_t *>(a.hi + row + i2) = (uint32_t)h[2] | ((uint32_t)h[3] << 16);
-    if (a.lo) {
-      *reinterpret_cast<uint32_t *>(a.lo + row + i0) = (uint32_t)l[0] | ((uint32_t)l[1] << 16);
-      *reinterpret_cast<uint32_t *>(a.lo + row + i2) = (uint32_t)l[2] | ((uint32_t)l[3] << 16);
+    const int k0 = ch * XCHUNK + 4 * sub;
+    *reinterpret_cast<uint32_t *>(act16_elem(a, b, k0)) = (uint32_t)h[0] | ((uint32_t)h[1] << 16);
+    *reinterpret_cast<uint32_t *>(act16_elem(a, b, k0 + 2)) = (uint32_t)h[2] | ((uint32_t)h[3] << 16);
+    if (a.rest) {
+      *reinterpret_cast<uint32_t *>(act16_elem(a, MAXB + b, k0)) = (uint32_t)l[0] | ((uint32_t)l[1] << 16);
+      *reinterpret_cast<uint32_t *>(act16_elem(a, MAXB + b, k0 + 2)) = (uint32_t)l[2] | ((uint32_t)l[3] << 16);
     }
     if (sub == 0) act16_put_consts(a, b, ch, m, oh, ol);
   }
@@ -525,6 +576,7 @@ cudaError_t prepare_attention();
 cudaError_t launch_gemv(const GemvParams &p, int epi, int grid, cudaStream_t s, bool pdl);
 int gemv_max_stages(int batch, int fmt, int smem_optin);  // valid after prepare_gemv
 cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s, bool pdl);
+cudaError_t launch_qknorm(const QkNormParams &p, cudaStream_t s, bool pdl);
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in,
                                int batch, const uint16_t *embed, int vocab, int d, int ldh,
                                const float *g_next, float *h, float *xn, float *sumsq,

@@ -82,9 +82,8 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
     if (lane == 0) {
       const uint64_t pol_w = policy_evict_first();
       const uint64_t pol_x = policy_evict_last();
-      // int4: B (Q/K/V projection: 2 B) fp16 source rows, then the tile's chunk constants
-      const int nsrc = p.xsplit ? 2 * B : B;
-      const uint32_t xbytes = FMT == 0 ? B * (KTILE * 4) : nsrc * X16_SRC_BYTES + XC_TILE_BYTES;
+      // int4: the K tile's block of the Act16 input, one contiguous copy
+      const uint32_t xbytes = FMT == 0 ? B * (KTILE * 4) : act16_copy_bytes(B, p.xsplit);
       const int pre = n < S ? n : S;
       stamp(TR_W_FIRST);
       for (int i = 0; i < pre; ++i) {
@@ -103,13 +102,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
           for (int b = 0; b < B; ++b)
             bulk_g2s(dst + b * (KTILE * 4), p.x + (size_t)b * p.ldx + (size_t)kt * KTILE, KTILE * 4, fb, pol_x);
         } else {
-          for (int r = 0; r < nsrc; ++r) {
-            const uint16_t *src = (r < B ? p.xin.hi + (size_t)r * p.xin.ld : p.xin.lo + (size_t)(r - B) * p.xin.ld) +
-                                  (size_t)kt * KT4;
-            bulk_g2s(dst + r * X16_SRC_STRIDE, src, X16_SRC_BYTES, fb, pol_x);
-          }
-          bulk_g2s(dst + 2 * B * X16_SRC_STRIDE, p.xin.xc + (size_t)kt * (KT4 / XCHUNK) * XC_CHUNK_FLOATS,
-                   XC_TILE_BYTES, fb, pol_x);
+          bulk_g2s(dst, act16_tile(p.xin, kt), xbytes, fb, pol_x);
         }
       };
       int kt_x = static_cast<int>(t0 % p.n_kt);

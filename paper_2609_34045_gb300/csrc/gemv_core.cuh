@@ -163,16 +163,27 @@ __device__ __forceinline__ void int4_frag_f16(uint32_t w, uint32_t &a0, uint32_t
   asm("lop3.b32 %0, %1, %2, %3, 0x6A;" : "=r"(a3) : "r"(w8), "r"(0x00F000F0u), "r"(0x64806480u));
 }
 
+// d = a b + c for one m16n8k16 fp16 tile, the accumulator seeded from c
+__device__ __forceinline__ void mma_f16_16816_seed(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                                    uint32_t b0, uint32_t b1, float4 c) {
+  asm(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%10,%11,%12,%13};"
+      : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(c.x), "f"(c.y), "f"(c.z), "f"(c.w));
+}
+
 // int4 tile (FMT 1) on the tensor cores.  Warp w takes row group r16 = w % 4 (16 rows) and K half
 // h = w / 4 (128 of the tile's 256 K): per K step of 16, one m16n8k16 MMA (fp16, fp32
-// accumulate) of the decoded codes against eight columns of activations, read as one 8-byte
-// shared-memory load per lane (Act16 order).  Column j is source row j % B (the users' rounded
-// parts); with XSPLIT, columns 4..7 are the rests (source rows B + (j - 4) % B).  Columns past
-// the users carry copies and are dropped at the end.  Per 32-element chunk the accumulator
-// starts at minus the columns' offset sums, so that after its two MMAs it holds the product of
-// the codes with the scaled activations; it is then multiplied back by the chunk's multiplier
-// and the rows' group scale into acc.  acc[0..1]: row r16*16 + gid, columns 2 tig, 2 tig + 1;
-// acc[2..3]: row + 8.
+// accumulate) of the decoded codes against eight columns of activations; one 16-byte
+// shared-memory load per lane gives the B fragments of both K steps of a 32-element chunk (Act16
+// order).  Column j is source row j % B (the users' rounded parts); with XSPLIT, columns 4..7
+// are the rests (source rows MAXB + (j - 4) % B).  Columns past the users carry copies and are
+// dropped at the end.  A chunk's first MMA seeds the accumulator with minus the columns' offset
+// sums (stored as the accumulator quad), so that after its two MMAs it holds the product of the
+// codes with the scaled activations; the two chunks of a weight group are multiplied back by
+// their multipliers and summed (packed fp32x2), then scaled by the rows' group scale into acc.
+// acc[0..1]: row r16*16 + gid, columns 2 tig, 2 tig + 1; acc[2..3]: row + 8.
 template <int B, bool XSPLIT>
 __device__ __forceinline__ void tile_compute_int4(const uint8_t *st, int warp, int lane, float (&acc)[4]) {
   const int r16 = warp & 3, h = warp >> 2, gid = lane >> 2, tig = lane & 3;
@@ -180,32 +191,39 @@ __device__ __forceinline__ void tile_compute_int4(const uint8_t *st, int warp, i
   const uint4 wq[2] = {cw[0], cw[32]};
   const uint32_t *sp = reinterpret_cast<const uint32_t *>(st + TILE4_CODE_BYTES);
   const uint32_t s0 = sp[(r16 * 16 + gid) * 2 + h], s1 = sp[(r16 * 16 + gid + 8) * 2 + h];
-  const int src = XSPLIT ? (gid < 4 ? gid % B : B + (gid - 4) % B) : gid % B;
-  const uint8_t *xb = st + TILE4_BYTES + src * X16_SRC_STRIDE + h * 256 + tig * 8;
-  const float4 *xc = reinterpret_cast<const float4 *>(st + TILE4_BYTES + 2 * B * X16_SRC_STRIDE) + tig;
+  const int src = XSPLIT ? (gid < 4 ? gid % B : MAXB + (gid - 4) % B) : gid % B;
+  const uint4 *xb =
+      reinterpret_cast<const uint4 *>(st + TILE4_BYTES + XC_TILE_BYTES + src * X16_SRC_STRIDE + h * 256) + tig;
+  const float4 *xc = reinterpret_cast<const float4 *>(st + TILE4_BYTES) + tig * 2;
 #pragma unroll
   for (int q = 0; q < 2; ++q) {
-    const float sc0 = q ? bf16_hi(s0) : bf16_lo(s0), sc1 = q ? bf16_hi(s1) : bf16_lo(s1);
+    float2 g0, g1;  // rows gid, gid + 8: the group's two chunks, each times its multipliers
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
-      // chunk h * 4 + 2 q + half of the tile: multipliers and offset sums of this lane's columns
-      const float4 mc = xc[(h * 4 + 2 * q + half) * 4];
-      float c[4] = {mc.z, mc.w, mc.z, mc.w};
-#pragma unroll
-      for (int j = 2 * half; j < 2 * half + 2; ++j) {
-        const uint32_t w = j == 0 ? wq[q].x : j == 1 ? wq[q].y : j == 2 ? wq[q].z : wq[q].w;
-        const uint2 bb = *reinterpret_cast<const uint2 *>(xb + 32 * (4 * q + j));
-        uint32_t a0, a1, a2, a3;
-        int4_frag_f16(w, a0, a1, a2, a3);
-        mma_f16_16816(c, a0, a1, a2, a3, bb.x, bb.y);
+      const int ch = h * 4 + 2 * q + half;  // chunk of the tile
+      const float4 seed = xc[ch * 8];
+      const float4 mm = xc[ch * 8 + 1];
+      const uint4 bb = xb[(2 * q + half) * 4];
+      uint32_t a0, a1, a2, a3;
+      float c[4];
+      int4_frag_f16(half ? wq[q].z : wq[q].x, a0, a1, a2, a3);
+      mma_f16_16816_seed(c, a0, a1, a2, a3, bb.x, bb.y, seed);
+      int4_frag_f16(half ? wq[q].w : wq[q].y, a0, a1, a2, a3);
+      mma_f16_16816(c, a0, a1, a2, a3, bb.z, bb.w);
+      const float2 m2 = make_float2(mm.x, mm.y);
+      if (half == 0) {
+        g0 = __fmul2_rn(m2, make_float2(c[0], c[1]));
+        g1 = __fmul2_rn(m2, make_float2(c[2], c[3]));
+      } else {
+        g0 = __ffma2_rn(m2, make_float2(c[0], c[1]), g0);
+        g1 = __ffma2_rn(m2, make_float2(c[2], c[3]), g1);
       }
-      // acc += (sc * m) c, two columns per packed fp32x2 operation
-      float f0, f1, f2, f3;
-      fmul2(f0, f1, sc0, sc0, mc.x, mc.y);
-      fmul2(f2, f3, sc1, sc1, mc.x, mc.y);
-      ffma2(acc[0], acc[1], f0, f1, c[0], c[1]);
-      ffma2(acc[2], acc[3], f2, f3, c[2], c[3]);
     }
+    const float sc0 = q ? bf16_hi(s0) : bf16_lo(s0), sc1 = q ? bf16_hi(s1) : bf16_lo(s1);
+    acc[0] = fmaf(sc0, g0.x, acc[0]);
+    acc[1] = fmaf(sc0, g0.y, acc[1]);
+    acc[2] = fmaf(sc1, g1.x, acc[2]);
+    acc[3] = fmaf(sc1, g1.y, acc[3]);
   }
 }
 
@@ -430,10 +448,10 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
         const float hn = hv[b][h2];
         const float xv = hn * pre.g[h2];
         // int4 stage: xn in the tensor-core input form, chunk rb * 2 + h2
-        if (p.xout.hi && p.g_next) act16_put_warp(p.xout, b, rb * 2 + h2, xv, lane);
+        if (p.xout.base && p.g_next) act16_put_warp(p.xout, b, rb * 2 + h2, xv, lane);
         if (ok) {
           p.h[o] = hn;
-          if (p.g_next && !p.xout.hi) p.xn[o] = xv;
+          if (p.g_next && !p.xout.base) p.xn[o] = xv;
           if (p.capture) p.capture[(size_t)b * p.n_rows + n] = hn;
           sq = fmaf(hn, hn, sq);
         }
@@ -459,7 +477,7 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
         const float u = uv[b];
         a = g / (1.0f + expf(-g)) * u;
       }
-      if (p.xout.hi)
+      if (p.xout.base)
         act16_put_warp(p.xout, b, rb, a, lane);  // int4 stage: the row block's 32 outputs, one chunk
       else if (ok)
         p.out[(size_t)b * p.ldo + j] = a;
@@ -482,6 +500,12 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
       if (r0 >= p.n_rows) continue;
       const float v1 = rv1[b] * iv[b];
       const float v2 = rv2[b] * iv[b];
+      if (p.qk_raw) {  // QK-norm stage: the kernel after this one rotates and appends
+        float *rw = p.qk_raw + (size_t)b * p.ld_raw + r0;
+        rw[0] = v1;
+        rw[1] = v2;
+        continue;
+      }
       if (r0 < p.n_q_rows + p.n_kv_rows) {
         const bool is_q = r0 < p.n_q_rows;
         const int rr = is_q ? r0 : r0 - p.n_q_rows;

@@ -62,7 +62,7 @@ __global__ void __launch_bounds__(64) stage_input_kernel(const int *ids, const f
     // xn = h * g; for int4 weights in the tensor-core input form (one warp per 32-element chunk),
     // exactly as the residual epilogue writes it
     const float xv = r < d ? v * g_next[r] : 0.f;
-    if (xn16.hi)
+    if (xn16.base)
       act16_put_warp(xn16, b, blockIdx.x * 2 + (tid >> 5), xv, tid & 31);
     else if (r < d)
       xn[(size_t)b * ldh + r] = xv;
@@ -114,6 +114,79 @@ cudaError_t launch_stage_output(const float *h, int ldh, int d, int batch, float
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, stage_output_kernel, h, ldh, d, hidden_out, next_in, next_ids);
+}
+
+// QK-norm of Qwen3-family blocks (the served models of section VI): each head of q and of k is
+// RMS-normalised over head_dim with its gain (g_q, g_k), then rotated (RoPE at the row's
+// position); q goes to the attention input, k and v (bf16, nearest even) to the row's KV slot.
+// One CTA per (head of Q, K or V, batch row), one thread per rotation pair (i, i + hd/2), whose
+// two values are adjacent rows of the projection (GEMV order).  The norm's sum of squares is
+// reduced in a fixed order (butterfly within a warp, then the warps in order), as the other
+// norms of the path are.
+template <int HD>
+__global__ void __launch_bounds__(HD / 2) qknorm_rope_kernel(QkNormParams p) {
+  constexpr int HALF = HD / 2, NW = HALF / 32;
+  __shared__ float s_part[NW];
+  pdl_launch_dependents();
+  pdl_wait();
+  const int head = blockIdx.x, b = blockIdx.y, i = threadIdx.x;
+  const int nq = p.n_heads, nk = p.n_kv_heads;
+  const float *raw = p.raw + (size_t)b * p.ld_raw;
+  const int pv = p.positions[b];
+  const bool ok = pv >= 0 && pv < p.max_ctx;
+  const size_t slot_base = (size_t)p.slots[b] * nk;
+  if (head >= nq + nk) {  // V rows are in natural order: no norm, no rotation
+    if (!ok) return;
+    const int vh = head - nq - nk;
+    const float2 x = *reinterpret_cast<const float2 *>(raw + (size_t)(nq + nk) * HD + (size_t)vh * HD + 2 * i);
+    uint16_t *vd = p.vcache + ((slot_base + vh) * p.max_ctx + pv) * HD;
+    vd[2 * i] = f32_to_bf16_rne(x.x);
+    vd[2 * i + 1] = f32_to_bf16_rne(x.y);
+    return;
+  }
+  const bool is_q = head < nq;
+  const float2 x = *reinterpret_cast<const float2 *>(raw + (size_t)head * HD + 2 * i);
+  float s = x.x * x.x + x.y * x.y;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+  if constexpr (NW > 1) {
+    if ((i & 31) == 0) s_part[i >> 5] = s;
+    __syncthreads();
+    s = 0.f;
+#pragma unroll
+    for (int w = 0; w < NW; ++w) s += s_part[w];
+  }
+  const float r = 1.0f / sqrtf(s / static_cast<float>(HD) + p.eps);
+  const float *g = is_q ? p.g_q : p.g_k;
+  const float y1 = x.x * r * g[i], y2 = x.y * r * g[i + HALF];
+  const size_t ri = (size_t)(ok ? pv : 0) * HALF + i;
+  const float cs = p.rope_cos[ri], sn = p.rope_sin[ri];
+  const float a = y1 * cs - y2 * sn;
+  const float c2 = y2 * cs + y1 * sn;
+  if (is_q) {
+    float *qd = p.q + (size_t)b * nq * HD + (size_t)head * HD;
+    qd[i] = a;
+    qd[i + HALF] = c2;
+  } else if (ok) {
+    uint16_t *kd = p.kcache + ((slot_base + (head - nq)) * p.max_ctx + pv) * HD;
+    kd[i] = f32_to_bf16_rne(a);
+    kd[i + HALF] = f32_to_bf16_rne(c2);
+  }
+}
+
+cudaError_t launch_qknorm(const QkNormParams &p, cudaStream_t s, bool pdl) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.n_heads + 2 * p.n_kv_heads, p.batch);
+  cfg.blockDim = dim3(p.head_dim / 2);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  if (p.head_dim == 128) return cudaLaunchKernelEx(&cfg, qknorm_rope_kernel<128>, p);
+  if (p.head_dim == 64) return cudaLaunchKernelEx(&cfg, qknorm_rope_kernel<64>, p);
+  return cudaErrorInvalidValue;
 }
 
 // Repack a bf16 matrix src [n_src_rows][k] into tiles [n_rb][n_kt][RB][KT]: output row r is

@@ -46,6 +46,7 @@ Mat mat_shape(int N, int K, int fmt) {
 struct LayerDev {
   Mat qkv, o, gu, down;
   float *g_attn = nullptr, *g_ffn = nullptr;
+  float *g_q = nullptr, *g_k = nullptr;  // QK-norm gains [hd] (qk_norm stages)
   bool loaded = false;
 };
 
@@ -53,6 +54,7 @@ struct LayerDev {
 struct Plan {
   int d, hq, hkv, hd, F, V, qdim, kvdim, nl;
   int ldh, ldq, lda;  // activation row strides, multiples of 256 floats
+  int ld_raw;         // QK-norm stages: row stride of the raw Q/K/V projection (else 0)
   Mat qkv, o, gu, down, lm;
   size_t kv_elems_per_layer;  // per cache (K or V)
   int n_sm, ctas_per_sm, stages, gemv_grid_max, n_rb_max, n_parts, attn_nchunks_max;
@@ -65,9 +67,7 @@ struct Plan {
 
 // Bytes of one int4 GEMV input (Act16) of row length ld: MAXB fp16 rows (and their rests), and
 // the per-chunk constants.
-size_t act16_bytes(int ld, bool with_rest) {
-  return (size_t)MAXB * ld * 2 * (with_rest ? 2 : 1) + (size_t)ld / XCHUNK * XC_CHUNK_FLOATS * 4;
-}
+size_t act16_bytes(int ld, bool with_rest) { return (size_t)(ld / KT4) * act16_tile_bytes(with_rest ? 1 : 0); }
 
 int env_int(const char *name, int dflt) {
   const char *v = std::getenv(name);
@@ -88,7 +88,7 @@ int validate_cfg(const kfl_model_cfg *c, int l0, int l1, int flags) {
     return KFL_ERR_ARG;
   if (c->max_ctx <= 0 || c->max_batch <= 0 || c->max_batch > MAXB) return KFL_ERR_ARG;
   if (c->max_ctx > (1 << 20)) return KFL_ERR_ARG;
-  if (c->qk_norm != 0) return KFL_ERR_ARG;
+  if (c->qk_norm != 0 && c->qk_norm != 1) return KFL_ERR_ARG;
   if (!(c->rms_eps > 0.f) || !(c->rope_theta > 0.f)) return KFL_ERR_ARG;
   if (l0 < 0 || l1 < l0 || l1 > c->n_layers_total) return KFL_ERR_ARG;
   if (flags & ~KFL_IS_HEAD) return KFL_ERR_ARG;
@@ -109,6 +109,7 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   p->ldh = round_up(p->d, 256);
   p->ldq = round_up(p->qdim, 256);
   p->lda = round_up(p->F, 256);
+  p->ld_raw = c->qk_norm ? round_up(p->qdim + 2 * p->kvdim, 256) : 0;
   const int f = c->weight_fmt;
   p->qkv = mat_shape(p->qdim + 2 * p->kvdim, p->d, f);
   p->o = mat_shape(p->d, p->qdim, f);
@@ -158,14 +159,15 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
 
   size_t w = 0;
   if (p->nl > 0)
-    w += (size_t)p->nl * (p->qkv.bytes + p->o.bytes + p->gu.bytes + p->down.bytes + 2 * (size_t)p->d * 4);
+    w += (size_t)p->nl * (p->qkv.bytes + p->o.bytes + p->gu.bytes + p->down.bytes + 2 * (size_t)p->d * 4 +
+                          (c->qk_norm ? 2 * (size_t)p->hd * 4 : 0));
   if (flags & KFL_EMBED_IN) w += (size_t)p->V * p->d * 2;
   if (flags & KFL_LOGITS_OUT) w += p->lm.bytes + (size_t)p->d * 4;
   p->bytes_weights = w;
   p->bytes_kv = 2 * (size_t)p->nl * p->kv_elems_per_layer * 2;
   size_t ws = 0;
   ws += (size_t)c->max_ctx * (p->hd / 2) * 4 * 2;                      // rope tables
-  ws += (size_t)MAXB * (2 * p->ldh + 2 * p->ldq + p->lda) * 4;         // h, xn, q, o, a
+  ws += (size_t)MAXB * (2 * p->ldh + 2 * p->ldq + p->lda + p->ld_raw) * 4;  // h, xn, q, o, a, raw Q/K/V
   ws += act16_bytes(p->ldh, true) + act16_bytes(p->ldq, false) + act16_bytes(p->lda, false);  // int4 inputs
   ws += (size_t)p->n_parts * MAXB * 4;                                 // sum of squares
   ws += 3 * MAXB * 4;                                                  // positions, KV slots, next ids
@@ -196,6 +198,7 @@ struct kfl_stage {
   uint16_t *kc = nullptr, *vc = nullptr;
   float *rope_cos = nullptr, *rope_sin = nullptr;
   float *h = nullptr, *xn = nullptr, *q = nullptr, *o = nullptr, *a = nullptr, *sumsq = nullptr;
+  float *qk_raw = nullptr;  // QK-norm stages: the Q/K/V projection before the norm and RoPE
   // int4 stages: the GEMV inputs in the tensor cores' fp16 form (xn with its rests, for Q/K/V)
   Act16 xn16 = {}, a16 = {}, o16 = {};
   int *pos = nullptr, *next_int = nullptr;
@@ -367,6 +370,10 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
       g.head_dim = P.hd;
       g.max_ctx = c.max_ctx;
       g.n_kv_heads = P.hkv;
+      if (c.qk_norm) {
+        g.qk_raw = st->qk_raw;
+        g.ld_raw = P.ld_raw;
+      }
       if (i4) g.xin = st->xn16;
       gemv(EPI_QKV, g);
     }
@@ -393,6 +400,26 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
       a.target_units = P.attn_units;
       a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)P.hd));
       a.err = st->err;
+      if (c.qk_norm) {
+        QkNormParams &n = x.qn;
+        n.raw = st->qk_raw;
+        n.ld_raw = P.ld_raw;
+        n.g_q = L.g_q;
+        n.g_k = L.g_k;
+        n.q = st->q;
+        n.kcache = kcl;
+        n.vcache = vcl;
+        n.positions = st->pos;
+        n.slots = st->slots;
+        n.rope_cos = st->rope_cos;
+        n.rope_sin = st->rope_sin;
+        n.batch = batch;
+        n.n_heads = P.hq;
+        n.n_kv_heads = P.hkv;
+        n.head_dim = P.hd;
+        n.max_ctx = c.max_ctx;
+        n.eps = c.rms_eps;
+      }
       ph.push_back(x);
     }
     {
@@ -561,6 +588,7 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
       }
       CK(launch_gemv(g, ph.epi, grid, s, pdl));
     } else {
+      if (ph.qn.raw) CK(launch_qknorm(ph.qn, s, pdl));  // QK-norm stages: norm, RoPE, KV append
       CK(launch_attention(ph.a, st->P.hd, s, pdl));
     }
     if (kinds) CK(cudaEventRecord(st->ev[2 * k + 1], s));
@@ -1096,6 +1124,10 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
     AL(L.down.tiles, L.down.bytes);
     AL(L.g_attn, (size_t)P.d * 4);
     AL(L.g_ffn, (size_t)P.d * 4);
+    if (cfg->qk_norm) {
+      AL(L.g_q, (size_t)P.hd * 4);
+      AL(L.g_k, (size_t)P.hd * 4);
+    }
   }
   if (flags & KFL_EMBED_IN) AL(st->embed, (size_t)P.V * P.d * 2);
   if (flags & KFL_LOGITS_OUT) {
@@ -1114,6 +1146,7 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
   AL(st->q, (size_t)MAXB * P.ldq * 4);
   AL(st->o, (size_t)MAXB * P.ldq * 4);
   AL(st->a, (size_t)MAXB * P.lda * 4);
+  if (cfg->qk_norm) AL(st->qk_raw, (size_t)MAXB * P.ld_raw * 4);
   AL(st->sumsq, (size_t)P.n_parts * MAXB * 4);
   {
     // int4 GEMV inputs (allocated for every stage; zero where nothing writes: the padding)
@@ -1122,13 +1155,10 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
     for (int i = 0; i < 3; ++i) {
       Act16 &x = *acts[i];
       x.ld = lds[i];
-      AL(x.hi, (size_t)MAXB * x.ld * 2);
-      if (i == 0) AL(x.lo, (size_t)MAXB * x.ld * 2);
-      AL(x.xc, (size_t)x.ld / XCHUNK * XC_CHUNK_FLOATS * 4);
-      if (cudaMemset(x.hi, 0, (size_t)MAXB * x.ld * 2) != cudaSuccess ||
-          (x.lo && cudaMemset(x.lo, 0, (size_t)MAXB * x.ld * 2) != cudaSuccess) ||
-          cudaMemset(x.xc, 0, (size_t)x.ld / XCHUNK * XC_CHUNK_FLOATS * 4) != cudaSuccess)
-        return fail(KFL_ERR_CUDA);
+      x.rest = i == 0 ? 1 : 0;
+      const size_t bytes = act16_bytes(x.ld, x.rest != 0);
+      AL(x.base, bytes);
+      if (cudaMemset(x.base, 0, bytes) != cudaSuccess) return fail(KFL_ERR_CUDA);
     }
   }
   AL(st->pos, MAXB * 4);
@@ -1178,7 +1208,8 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
       return fail(KFL_ERR_CUDA);
   }
   // persistent stage kernel: the deepest ring that fits next to the attention buffers
-  st->persistent = env_int("KFL_PERSISTENT", 0) != 0;
+  // the persistent stage kernel has no QK-norm phase: QK-norm stages run one kernel per phase
+  st->persistent = env_int("KFL_PERSISTENT", 0) != 0 && !cfg->qk_norm;
   {
     const size_t static_smem = 8192;  // the kernel's own __shared__ variables
     size_t smem_max = 0;
@@ -1206,6 +1237,7 @@ extern "C" int kfl_stage_load_layer(kfl_stage *st, int local, const kfl_layer_we
   if (!w) return KFL_ERR_ARG;
   if (local < 0 || local >= st->P.nl) return KFL_ERR_RANGE;
   if (!w->attn_norm || !w->ffn_norm) return KFL_ERR_ARG;
+  if (st->cfg.qk_norm && (!w->q_norm || !w->k_norm)) return KFL_ERR_ARG;
   CK(cudaSetDevice(st->dev));
   const Plan &P = st->P;
   LayerDev &L = st->layers[local];
@@ -1214,6 +1246,10 @@ extern "C" int kfl_stage_load_layer(kfl_stage *st, int local, const kfl_layer_we
   do {
     if ((rc = load_gain(st, w->attn_norm, P.d, on_device, L.g_attn, tmp))) break;
     if ((rc = load_gain(st, w->ffn_norm, P.d, on_device, L.g_ffn, tmp))) break;
+    if (st->cfg.qk_norm) {
+      if ((rc = load_gain(st, w->q_norm, P.hd, on_device, L.g_q, tmp))) break;
+      if ((rc = load_gain(st, w->k_norm, P.hd, on_device, L.g_k, tmp))) break;
+    }
     // Q/K/V: q and k rows of each head reordered so that the RoPE pair (i, i + hd/2) is adjacent
     std::vector<int> map(P.qdim + 2 * P.kvdim);
     for (int r = 0; r < (int)map.size(); ++r) {
@@ -1335,8 +1371,9 @@ extern "C" int kfl_stage_prefill(kfl_stage *st, const int32_t *token_ids, const 
   if (!st->loaded()) return KFL_ERR_STATE;
   CK(cudaSetDevice(st->dev));
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
-  // the dense path from KFL_PREFILL_DENSE_MIN tokens on (default 16)
-  if (n_tokens >= env_int("KFL_PREFILL_DENSE_MIN", 16))
+  // the dense path from KFL_PREFILL_DENSE_MIN tokens on (default 16); QK-norm stages take the
+  // decode-step path (the dense path has no QK-norm epilogue)
+  if (n_tokens >= env_int("KFL_PREFILL_DENSE_MIN", 16) && !st->cfg.qk_norm)
     return run_prefill_dense(st, token_ids, hidden_in, positions, user, n_tokens, hidden_out, next_ids, s);
   const int d = st->P.d;
   // else the prompt in chunks of max_batch consecutive tokens: each chunk is one decode step whose
@@ -1517,7 +1554,7 @@ extern "C" int kfl_stage_launches_per_step(kfl_stage *st, int batch) {
   if (!valid(st)) return KFL_ERR_STATE;
   (void)batch;
   const int body = 5 * st->P.nl + ((st->flags & KFL_LOGITS_OUT) ? 1 : 0);
-  if (st->profile || !st->persistent) return 2 + body;
+  if (st->profile || !st->persistent) return 2 + body + (st->cfg.qk_norm ? st->P.nl : 0);
   return 2 + (body > 0 ? 1 : 0);
 }
 

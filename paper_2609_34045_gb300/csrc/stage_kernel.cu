@@ -200,8 +200,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
           cu.n = n;
           cu.t0 = t0;
           cu.w = ph->g.w;
-          cu.bytes = WBYTES + (FMT == 0 ? B * (KTILE * 4)
-                                        : (ph->g.xsplit ? 2 * B : B) * X16_SRC_BYTES + XC_TILE_BYTES);
+          cu.bytes = WBYTES + (FMT == 0 ? B * (KTILE * 4) : act16_copy_bytes(B, ph->g.xsplit));
           return;
         }
         cu.k = kp.n_phases;
@@ -305,14 +304,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
               for (int b = 0; b < B; ++b)
                 bulk_g2s(dst + b * (KTILE * 4), x + (size_t)b * ldx + (size_t)ktj * KTILE, KTILE * 4, fb, pol);
             } else {
-              const int nsrc = g.xsplit ? 2 * B : B;
-              for (int r = 0; r < nsrc; ++r) {
-                const uint16_t *src = (r < B ? g.xin.hi + (size_t)r * g.xin.ld
-                                             : g.xin.lo + (size_t)(r - B) * g.xin.ld) + (size_t)ktj * KT4;
-                bulk_g2s(dst + r * X16_SRC_STRIDE, src, X16_SRC_BYTES, fb, pol);
-              }
-              bulk_g2s(dst + 2 * B * X16_SRC_STRIDE, g.xin.xc + (size_t)ktj * (KT4 / XCHUNK) * XC_CHUNK_FLOATS,
-                       XC_TILE_BYTES, fb, pol);
+              bulk_g2s(dst, act16_tile(g.xin, ktj), act16_copy_bytes(B, g.xsplit), fb, pol);
             }
             if (++s == S) {
               s = 0;

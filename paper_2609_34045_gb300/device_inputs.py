@@ -39,6 +39,9 @@ def layer_weights(model: wl.ModelShape, layer: int, seed: int, device="cuda") ->
     w = {}
     for name in ("attn_norm", "ffn_norm"):
         w[name] = normal_bf16(seed, wl.layer_tag(layer, name), model.d_model, 0.02, mean=1.0, device=device)
+    if model.qk_norm:
+        for name in ("q_norm", "k_norm"):
+            w[name] = normal_bf16(seed, wl.layer_tag(layer, name), model.head_dim, 0.02, mean=1.0, device=device)
     for name, (rows, cols) in model.matrix_shapes().items():
         w[name] = matrix(model.weight_fmt, seed, wl.layer_tag(layer, name), wl.layer_tag(layer, name, True),
                          rows, cols, device)

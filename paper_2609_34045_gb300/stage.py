@@ -44,7 +44,8 @@ class kfl_matrix(C.Structure):
 
 class kfl_layer_weights(C.Structure):
     _fields_ = [("attn_norm", C.c_void_p), ("ffn_norm", C.c_void_p)] + \
-               [(n, kfl_matrix) for n in ("wq", "wk", "wv", "wo", "wg", "wu", "wd")]
+               [(n, kfl_matrix) for n in ("wq", "wk", "wv", "wo", "wg", "wu", "wd")] + \
+               [("q_norm", C.c_void_p), ("k_norm", C.c_void_p)]
 
 
 class kfl_weights(C.Structure):
@@ -194,6 +195,8 @@ def _layer(w: dict) -> kfl_layer_weights:
     lw.ffn_norm = _ptr(w["ffn_norm"])
     for n in ("wq", "wk", "wv", "wo", "wg", "wu", "wd"):
         setattr(lw, n, _matrix(w[n]))
+    lw.q_norm = _ptr(w.get("q_norm"))
+    lw.k_norm = _ptr(w.get("k_norm"))
     return lw
 
 

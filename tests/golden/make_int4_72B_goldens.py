@@ -75,7 +75,18 @@ class Embedding:
         return wl.normal_bf16_at(self.seed, wl.head_tag("embed"), idx, 0.02).reshape(len(ids), d)
 
 
+def _no_huge_page_advice() -> None:
+    """numpy asks the kernel for transparent huge pages on large arrays; where the kernel then
+    compacts memory on every allocation, the oracle's multi-gigabyte temporaries crawl.  Only
+    the allocation advice changes, not any value."""
+    core = getattr(np, "_core", None) or getattr(np, "core", None)
+    setter = getattr(getattr(core, "multiarray", None), "_set_madvise_hugepage", None)
+    if setter is not None:
+        setter(False)
+
+
 def main() -> int:
+    _no_huge_page_advice()
     work = wl.CONFIGS[6]
     m, seed, b = work.model, work.seed, work.batch
     assert work.contexts == (8192,) * 4 and wl.CONFIGS[5].seed == seed

@@ -61,7 +61,19 @@ def test_memory_bytes_counts_weights_and_cache(lib):
     assert n_head - n >= 2 * w.model.vocab * w.model.d_model * 2
 
 
-@pytest.mark.parametrize("field,value", [("max_batch", 5), ("max_batch", 0), ("head_dim", 96), ("qk_norm", 1),
+def test_qk_norm_stage_counts_its_gains_and_raw_projection(lib):
+    # QK-norm adds two fp32 gains of head_dim per block and one raw Q/K/V row per user
+    w = wl.CONFIGS[2]
+    cfg = K.model_cfg(w.model, w.max_ctx, w.batch)
+    n0 = K.kfl_stage_memory_bytes(cfg, 0, 14, 0)
+    cfg.qk_norm = 1
+    n1 = K.kfl_stage_memory_bytes(cfg, 0, 14, 0)
+    m = w.model
+    ld_raw = (m.q_dim + 2 * m.kv_dim + 255) // 256 * 256
+    assert n1 - n0 == 14 * 2 * m.head_dim * 4 + 4 * ld_raw * 4
+
+
+@pytest.mark.parametrize("field,value", [("max_batch", 5), ("max_batch", 0), ("head_dim", 96), ("qk_norm", 2),
                                          ("n_kv_heads", 3), ("max_ctx", 0), ("weight_fmt", 7)])
 def test_bad_config_is_refused_before_any_allocation(lib, field, value):
     w = wl.CONFIGS[1]

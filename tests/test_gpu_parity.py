@@ -81,6 +81,41 @@ def test_int4_head_stage(batch):
     p.close()
 
 
+# Qwen3-family blocks: per-head RMSNorm of q and k before RoPE (QK-norm), with head_dim 64 and
+# 128, bf16 and int4 weights, ragged users
+QK64 = dataclasses.replace(RAGGED, qk_norm=True)
+QK128 = dataclasses.replace(RAGGED128, ffn=576, qk_norm=True)
+
+
+@pytest.mark.parametrize("fmt", ["bf16", "int4_g64"])
+@pytest.mark.parametrize("model", [QK64, QK128], ids=["hd64", "hd128"])
+def test_qk_norm_stage(model, fmt):
+    m = dataclasses.replace(model, weight_fmt=fmt, ffn=model.ffn // 64 * 64 if fmt != "bf16" else model.ffn)
+    p = Pair(m, 0, 2, K.KFL_IS_HEAD, 3, (4, 77, 150), 192, seed=24)
+    assert K.kfl_stage_launches_per_step(p.st, 3) == 2 + 5 * 2 + 1 + 2  # QK-norm: one more launch per block
+    _greedy(p, 3, np.array([1, 500, 776], dtype=np.int32) % m.vocab)
+    p.close()
+
+
+def test_qk_norm_body_stage_hidden_in_and_split():
+    # a body stage with hidden_in, then the same blocks as two stages: bit for bit the one stage
+    m = dataclasses.replace(RAGGED, qk_norm=True)
+    p = Pair(m, 0, 3, 0, 2, (30, 90), 128, seed=25)
+    a = Pair(m, 0, 1, 0, 2, (30, 90), 128, seed=25)
+    b = Pair(m, 1, 3, 0, 2, (30, 90), 128, seed=25)
+    for s_ in range(2):
+        h = wl.hidden_in(m, s_, 2, 25)
+        p.step(s_, hidden=h)
+        pos = np.array([30 + s_, 90 + s_], dtype=np.int32)
+        ha, _ = a.gpu_step(pos, hidden=h)
+        hb, _ = b.gpu_step(pos, hidden=ha)
+        hp, _ = p.gpu_step(pos, hidden=h)  # the same step again: it rewrites the same slots
+        assert np.array_equal(hp, hb)
+    p.compare_kv()
+    for x in (p, a, b):
+        x.close()
+
+
 def test_empty_tail_stage_is_head_return_leg():
     # l0 == l1 with LOGITS_OUT: final norm, lm_head and argmax of a received hidden state
     p = Pair(RAGGED, 3, 3, K.KFL_LOGITS_OUT, 2, (0, 0), 64, seed=15)

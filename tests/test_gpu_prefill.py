@@ -8,6 +8,8 @@ for decode: every token's output within max-abs 1e-2 of the oracle's RMS, greedy
 the oracle's top-2 margin exceeds 1e-2, the user's written cache rows within tolerance and every
 other row of every slot bit-identical.
 """
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -79,6 +81,8 @@ CASES = [
     ("hd128-200", RAGGED128, 0, 2, K.KFL_IS_HEAD, (0, 100, 7), 1, 200, 320),
     ("int4-head", RAGGED_INT4, 0, 2, K.KFL_IS_HEAD, (9, 70, 131), 1, 7, 192),
     ("int4-head-260", RAGGED_INT4, 0, 2, K.KFL_IS_HEAD, (9, 70, 131), 2, 260, 448),
+    # QK-norm stages prefill through decode steps whatever the prompt length
+    ("qknorm-head-40", dataclasses.replace(RAGGED, qk_norm=True), 0, 3, K.KFL_IS_HEAD, (5, 30, 70), 1, 40, 192),
 ]
 
 
