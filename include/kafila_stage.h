@@ -39,6 +39,9 @@ extern "C" {
 #define KFL_ERR_CUDA (-4)    /* a CUDA runtime call failed (no device, launch failure, ...) */
 #define KFL_ERR_STATE (-5)   /* decode before the weights were loaded, or a destroyed stage */
 #define KFL_ERR_TIMEOUT (-6) /* a bounded device-side wait gave up (reported by kfl_stage_status) */
+#define KFL_ERR_OVERFLOW (-8) /* an int4 stage's dense prefill met an activation fp16 cannot hold
+                                 (|x| >= 65520 or not finite); that prefill's outputs and cache
+                                 rows are not valid (reported by kfl_stage_status) */
 
 /* ---- weight formats and stage flags --------------------------------------------------- */
 #define KFL_BF16 0     /* bf16 matrices */
@@ -153,10 +156,14 @@ int kfl_stage_decode_users(kfl_stage *st, const int32_t *token_ids, const float 
 /* Prefill: run n_tokens tokens of one user's prompt through the stage, filling the user's KV
  * cache slot at the given positions; each token attends to the slot's rows up to its own
  * position, earlier tokens of the same call included (time to first token is the prefill plus
- * one decode step, Section VI, instrumentation paragraph).  The tokens go as steps of up to
- * max_batch rows, in order, every row of a step addressing the user's slot (the decode step's
- * kernels, each weight matrix streamed once per step); enqueued on cuda_stream, returns without
- * waiting.
+ * one decode step, Section VI, instrumentation paragraph).  From KFL_PREFILL_DENSE_MIN tokens
+ * (environment, default 16) the prompt runs densely: passes of up to 2048 tokens through
+ * tensor-core matrix products (tcgen05) and causal attention, each activation carried as two
+ * 16-bit terms (bf16 with bf16 weights; fp16 with int4 weights, dequantized to fp16 tiles in
+ * device memory the stage allocates at its first dense prefill).  Shorter prompts, and every
+ * prompt of a qk_norm stage, go as steps of up to max_batch rows, in order, every row of a step
+ * addressing the user's slot (the decode step's kernels).  Enqueued on cuda_stream, returns
+ * without waiting.
  *   token_ids  device int32[n_tokens] (KFL_EMBED_IN), else ignored
  *   hidden_in  device fp32[n_tokens][d_model] (without KFL_EMBED_IN)
  *   positions  device int32[n_tokens]: token t's position, distinct, normally start + t; the
@@ -166,7 +173,10 @@ int kfl_stage_decode_users(kfl_stage *st, const int32_t *token_ids, const float 
  *   hidden_out device fp32[n_tokens][d_model] (needed without KFL_LOGITS_OUT)
  *   next_ids   device int32[n_tokens]: the greedy token after each prompt token
  *              (KFL_LOGITS_OUT; the last one starts the decode)
- * Bad positions and token ids are found on the device as in kfl_stage_decode.
+ * Bad positions and token ids are found on the device as in kfl_stage_decode.  In an int4
+ * stage's dense prefill an activation beyond the fp16 range (|x| >= 65520, or not finite) is
+ * found on the device too: kfl_stage_status then reports KFL_ERR_OVERFLOW and the call's
+ * outputs and cache rows are not valid.
  * Errors returned here: KFL_ERR_ARG, KFL_ERR_RANGE (user), KFL_ERR_STATE, KFL_ERR_CUDA. */
 int kfl_stage_prefill(kfl_stage *st, const int32_t *token_ids, const float *hidden_in,
                       const int32_t *positions, int user, int n_tokens, float *hidden_out,
@@ -217,8 +227,9 @@ int kfl_stage_trace(kfl_stage *st, uint64_t *buf);
 int kfl_stage_trace_shape(kfl_stage *st, int batch, int *n_phases, int *grid, int *slots);
 
 /* Sticky device-side error word of the stage: waits for the device, then returns KFL_OK,
- * KFL_ERR_RANGE (a bad position or token id was seen) or KFL_ERR_TIMEOUT (a bounded wait
- * gave up), and clears it. */
+ * KFL_ERR_TIMEOUT (a bounded wait gave up), KFL_ERR_RANGE (a bad position or token id was
+ * seen) or KFL_ERR_OVERFLOW (an int4 dense prefill met an activation fp16 cannot hold), in this
+ * order of precedence, and clears it. */
 int kfl_stage_status(kfl_stage *st);
 
 /* Per-kernel timing: with enable = 1 later decodes run their kernels one by one (no CUDA

@@ -103,6 +103,7 @@ __host__ __device__ inline float *act16_consts(const Act16 &a, int ch) {
 constexpr unsigned ERR_POSITION = 1u;
 constexpr unsigned ERR_TOKEN = 2u;
 constexpr unsigned ERR_TIMEOUT = 4u;
+constexpr unsigned ERR_F16_RANGE = 8u;  // an int4 prefill activation beyond the fp16 range
 
 // bounded waits: spins before backing off, total polls before giving up (~1-2 s)
 constexpr uint32_t WAIT_FAST_SPINS = 1024;

@@ -120,8 +120,11 @@ __device__ __forceinline__ void split_term(float x, uint16_t &hi, uint16_t &lo, 
   else
     split_bf16(x, hi, lo);
 }
-// Two values as packed pairs of their hi and lo terms.
-__device__ __forceinline__ void split_pack(float x0, float x1, uint32_t &hi, uint32_t &lo, int f16 = 0) {
+// Two values as packed pairs of their hi and lo terms.  fp16 terms of a value that fp16 cannot
+// hold (|x| >= 65520 rounds to infinity, or not finite) set ERR_F16_RANGE in *err.
+__device__ __forceinline__ void split_pack(float x0, float x1, uint32_t &hi, uint32_t &lo, int f16 = 0,
+                                           unsigned *err = nullptr) {
+  if (f16 && err && !(fabsf(x0) < 65520.f && fabsf(x1) < 65520.f)) atomicOr(err, ERR_F16_RANGE);
   uint16_t h0, l0, h1, l1;
   split_term(x0, h0, l0, f16);
   split_term(x1, h1, l1, f16);
@@ -171,7 +174,7 @@ __device__ __forceinline__ void epilogue32(const PrefillEpiParams &ep, int t, in
 #pragma unroll
     for (int i = 0; i < 16; i += 2) {
       const float g0 = v[2 * i], u0 = v[2 * i + 1], g1 = v[2 * i + 2], u1 = v[2 * i + 3];
-      split_pack(g0 / (1.0f + expf(-g0)) * u0, g1 / (1.0f + expf(-g1)) * u1, w[i / 2], wl[i / 2], ep.f16);
+      split_pack(g0 / (1.0f + expf(-g0)) * u0, g1 / (1.0f + expf(-g1)) * u1, w[i / 2], wl[i / 2], ep.f16, ep.err);
     }
     uint16_t *row = ep.out16 + (size_t)t * ep.ldo16 + j0;
     uint16_t *rlo = ep.out16lo + (size_t)t * ep.ldo16 + j0;
@@ -752,12 +755,12 @@ __global__ void __launch_bounds__(PA_THREADS) prefill_attn_kernel(PrefillAttnPar
     const int col = h * HD + dt * 8 + 2 * c;
     uint32_t hi, lo;
     if (ta < p.T) {
-      split_pack(oacc[dt][0] * inv0, oacc[dt][1] * inv0, hi, lo, p.f16);
+      split_pack(oacc[dt][0] * inv0, oacc[dt][1] * inv0, hi, lo, p.f16, p.err);
       *reinterpret_cast<uint32_t *>(p.o + (size_t)ta * p.ldo + col) = hi;
       *reinterpret_cast<uint32_t *>(p.o_lo + (size_t)ta * p.ldo + col) = lo;
     }
     if (tb < p.T) {
-      split_pack(oacc[dt][2] * inv1, oacc[dt][3] * inv1, hi, lo, p.f16);
+      split_pack(oacc[dt][2] * inv1, oacc[dt][3] * inv1, hi, lo, p.f16, p.err);
       *reinterpret_cast<uint32_t *>(p.o + (size_t)tb * p.ldo + col) = hi;
       *reinterpret_cast<uint32_t *>(p.o_lo + (size_t)tb * p.ldo + col) = lo;
     }
@@ -799,7 +802,7 @@ __global__ void prefill_input_kernel(const int *ids, const float *hidden_in, con
 // x[t] = h[t] / rms(h[t]) * g as hi and lo 16-bit terms, one block per token, four elements per
 // thread step (d a multiple of 8; h, g and x rows 16-byte aligned).
 __global__ void prefill_rmsnorm_kernel(const float *h, int ldh, int d, const float *g, float eps, uint16_t *x,
-                                       uint16_t *x_lo, int ldx, int f16) {
+                                       uint16_t *x_lo, int ldx, int f16, unsigned *err) {
   const int t = blockIdx.x, d4 = d / 4;
   const float4 *row = reinterpret_cast<const float4 *>(h + (size_t)t * ldh);
   float ss = 0.f;
@@ -823,8 +826,8 @@ __global__ void prefill_rmsnorm_kernel(const float *h, int ldh, int d, const flo
   for (int i = threadIdx.x; i < d4; i += blockDim.x) {
     const float4 v = row[i], gg = g4[i];
     uint2 hi, lo;
-    split_pack(v.x * inv * gg.x, v.y * inv * gg.y, hi.x, lo.x, f16);
-    split_pack(v.z * inv * gg.z, v.w * inv * gg.w, hi.y, lo.y, f16);
+    split_pack(v.x * inv * gg.x, v.y * inv * gg.y, hi.x, lo.x, f16, err);
+    split_pack(v.z * inv * gg.z, v.w * inv * gg.w, hi.y, lo.y, f16, err);
     xh[i] = hi;
     xl[i] = lo;
   }
@@ -1075,8 +1078,8 @@ cudaError_t launch_prefill_input(const int *ids, const float *hidden_in, const i
 }
 
 cudaError_t launch_prefill_rmsnorm(const float *h, int ldh, int T, int d, const float *g, float eps, uint16_t *x,
-                                   uint16_t *x_lo, int ldx, int f16, cudaStream_t s) {
-  prefill_rmsnorm_kernel<<<T, 256, 0, s>>>(h, ldh, d, g, eps, x, x_lo, ldx, f16);
+                                   uint16_t *x_lo, int ldx, int f16, unsigned *err, cudaStream_t s) {
+  prefill_rmsnorm_kernel<<<T, 256, 0, s>>>(h, ldh, d, g, eps, x, x_lo, ldx, f16, err);
   return cudaGetLastError();
 }
 

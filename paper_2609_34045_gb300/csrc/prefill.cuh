@@ -61,7 +61,8 @@ struct PrefillEpiParams {
   // split-K: 1, 2, 4 or 8 CTAs per output tile, launched as a cluster that reduces through
   // distributed shared memory (PE_ARGMAX: 1)
   int splits;
-  unsigned *err;           // ERR_TIMEOUT if a pipeline wait gave up
+  unsigned *err;           // ERR_TIMEOUT if a pipeline wait gave up; ERR_F16_RANGE (PE_SWIGLU, fp16
+                           // terms) if a value is beyond the fp16 range
 };
 
 struct PrefillAttnParams {
@@ -73,6 +74,7 @@ struct PrefillAttnParams {
   const int *positions;    // [T], -1: refused (output 0)
   int slot, T, n_heads, n_kv_heads, max_ctx;
   float scale_log2;        // log2(e) / sqrt(hd)
+  unsigned *err;           // ERR_F16_RANGE if an fp16 output term cannot hold its value
 };
 
 // Host side (prefill.cu).
@@ -88,7 +90,7 @@ cudaError_t launch_prefill_input(const int *ids, const float *hidden_in, const i
                                  const uint16_t *embed, int vocab, int d, int ldh, float *h, int *positions,
                                  int max_ctx, unsigned *err, cudaStream_t s);
 cudaError_t launch_prefill_rmsnorm(const float *h, int ldh, int T, int d, const float *g, float eps, uint16_t *x,
-                                   uint16_t *x_lo, int ldx, int f16, cudaStream_t s);
+                                   uint16_t *x_lo, int ldx, int f16, unsigned *err, cudaStream_t s);
 // int4 group-64 tiles [n_rb][n_kt][TILE4_BYTES] -> fp16 tiles [n_rb][2 n_kt][RB][KT] of code x scale.
 cudaError_t launch_dequant_int4_f16(const uint8_t *tiles4, int n_rb, int n_kt, uint16_t *dst, cudaStream_t s);
 cudaError_t launch_split_bf16(const float *x, int T, int K, int ldx, uint16_t *hi, uint16_t *lo, int ld,

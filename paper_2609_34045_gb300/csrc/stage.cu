@@ -899,7 +899,7 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
       const LayerDev &L = st->layers[l];
       uint16_t *kcl = st->kc + (size_t)l * P.kv_elems_per_layer;
       uint16_t *vcl = st->vc + (size_t)l * P.kv_elems_per_layer;
-      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, L.g_attn, eps, st->pf_x[0], st->pf_x[1], ldx, i4, s));
+      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, L.g_attn, eps, st->pf_x[0], st->pf_x[1], ldx, i4, st->err, s));
       PrefillEpiParams e = {};
       e.T = n;
       e.err = st->err;
@@ -934,6 +934,7 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
       a.n_kv_heads = P.hkv;
       a.max_ctx = st->cfg.max_ctx;
       a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)P.hd));
+      a.err = st->err;
       CK(launch_prefill_attention(a, P.hd, s));
       PrefillEpiParams r = {};
       r.T = n;
@@ -942,7 +943,7 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
       r.out = st->pf_h;
       r.ldo = P.ldh;
       CK(pf_gemm(st, PE_RESID, mo[0], mo[1], l, 1, r, s));
-      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, L.g_ffn, eps, st->pf_x[0], st->pf_x[1], ldx, i4, s));
+      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, L.g_ffn, eps, st->pf_x[0], st->pf_x[1], ldx, i4, st->err, s));
       PrefillEpiParams g = {};
       g.T = n;
       g.err = st->err;
@@ -954,7 +955,7 @@ int run_prefill_dense(kfl_stage *st, const int32_t *ids, const float *hidden_in,
       CK(pf_gemm(st, PE_RESID, ma[0], ma[1], l, 3, r, s));
     }
     if (st->flags & KFL_LOGITS_OUT) {
-      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, st->g_final, eps, st->pf_x[0], st->pf_x[1], ldx, i4, s));
+      CK(launch_prefill_rmsnorm(st->pf_h, P.ldh, n, P.d, st->g_final, eps, st->pf_x[0], st->pf_x[1], ldx, i4, st->err, s));
       PrefillEpiParams z = {};
       z.T = n;
       z.err = st->err;
@@ -1528,6 +1529,7 @@ extern "C" int kfl_stage_status(kfl_stage *st) {
   CK(cudaMemset(st->err, 0, 4));
   if (e & ERR_TIMEOUT) return KFL_ERR_TIMEOUT;
   if (e & (ERR_POSITION | ERR_TOKEN)) return KFL_ERR_RANGE;
+  if (e & ERR_F16_RANGE) return KFL_ERR_OVERFLOW;
   return KFL_OK;
 }
 
@@ -1595,6 +1597,7 @@ extern "C" const char *kfl_strerror(int code) {
     case KFL_ERR_CUDA: return "CUDA runtime error";
     case KFL_ERR_STATE: return "stage not ready (weights not loaded) or invalid";
     case KFL_ERR_TIMEOUT: return "a bounded device-side wait gave up";
+    case KFL_ERR_OVERFLOW: return "an int4 prefill activation is beyond the fp16 range";
     case KFL_ERR_INFEASIBLE: return "no division of the blocks fits the devices";
     default: return "unknown error";
   }

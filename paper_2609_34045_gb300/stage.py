@@ -64,6 +64,7 @@ class kfl_plan(C.Structure):
 
 
 KFL_ERR_INFEASIBLE = -7
+KFL_ERR_OVERFLOW = -8
 
 _lib = None
 

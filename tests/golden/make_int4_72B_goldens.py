@@ -25,8 +25,9 @@ Stored (``int4_72B_80L_step0.npz``):
   those blocks;
 * provenance: the seed, this script's SHA-256, the oracle's SHA-256.
 
-Run from the repository root: ``python tests/golden/make_int4_72B_goldens.py`` (about an hour on
-eight cores, 30 GB of host memory).
+Run from the repository root: ``python tests/golden/make_int4_72B_goldens.py [output.npz]``
+(about 20 minutes on sixteen cores, 30 GB of host memory; the output defaults to the file beside
+this script).
 """
 from __future__ import annotations
 
@@ -85,7 +86,7 @@ def _no_huge_page_advice() -> None:
         setter(False)
 
 
-def main() -> int:
+def main(out: str = OUT) -> int:
     _no_huge_page_advice()
     work = wl.CONFIGS[6]
     m, seed, b = work.model, work.seed, work.batch
@@ -131,16 +132,16 @@ def main() -> int:
         print(f"block {layer}: rms {rms[layer].round(3).tolist()}  ({time.time() - t0:.0f} s)", flush=True)
         del st
     np.savez_compressed(
-        OUT, seed=np.int64(seed), positions=pos.astype(np.int64), token_ids=ids.astype(np.int64),
+        out, seed=np.int64(seed), positions=pos.astype(np.int64), token_ids=ids.astype(np.int64),
         per_layer_rms=rms, sample_cols=cols, per_layer_sample=samp,
         full_layers=np.array(FULL_LAYERS, dtype=np.int64), full_states=np.stack([full[x] for x in FULL_LAYERS]),
         next_ids=next_ids.astype(np.int64), margins=margins, top_ids=top.astype(np.int64), top_logits=top_logits,
         kv_layers=np.array(KV_LAYERS, dtype=np.int64), k_new=np.stack(k_new), v_new=np.stack(v_new),
         script_sha256=np.array(sha256(os.path.abspath(__file__))),
         oracle_sha256=np.array(sha256(os.path.join(ROOT, "oracle", "stage.py"))))
-    print("wrote", OUT, f"({time.time() - t0:.0f} s)")
+    print("wrote", out, f"({time.time() - t0:.0f} s)")
     return 0
 
 
 if __name__ == "__main__":
-    sys.exit(main())
+    sys.exit(main(*sys.argv[1:2]))

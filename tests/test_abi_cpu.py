@@ -44,7 +44,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 def test_strerror(lib):
     assert K.kfl_strerror(0) == "ok"
-    for code in range(-6, 0):
+    for code in range(-8, 0):
         assert K.kfl_strerror(code) != "unknown error"
     assert K.kfl_strerror(-99) == "unknown error"
 

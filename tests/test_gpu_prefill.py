@@ -137,3 +137,27 @@ def test_repeated_position_is_reported(path):
     K.kfl_stage_prefill(p.st, ids, None, pos, 0, 2, None, nxt, torch.cuda.current_stream().cuda_stream)
     assert K.kfl_stage_status(p.st) == 0
     p.close()
+
+
+def test_int4_dense_prefill_reports_fp16_overflow(monkeypatch):
+    """The int4 dense prefill carries activations as fp16 terms.  Host-made RMSNorm gains of 2^17
+    make every normalised input larger than fp16 can hold: kfl_stage_status reports
+    KFL_ERR_OVERFLOW (a status read back on the host; nothing faults).  The same stage with its
+    seeded gains reports nothing."""
+    monkeypatch.setenv("KFL_PREFILL_DENSE_MIN", "1")
+    m = RAGGED_INT4
+    cfg = K.model_cfg(m, 128, 1)
+    for big in (False, True):
+        st = K.kfl_stage_create(cfg, 0, 1, K.KFL_IS_HEAD)
+        w = wl.layer_weights(m, 0, 41)
+        if big:
+            w["attn_norm"] = np.full(m.d_model, 0x4800, dtype=np.uint16)  # bf16 2^17
+        K.kfl_stage_load_layer(st, 0, w, on_device=False)
+        K.kfl_stage_load_head(st, wl.head_weights(m, 41), on_device=False)
+        n = 20
+        ids = torch.tensor(wl.token_ids(41, 5, n, m.vocab), device="cuda")
+        pos = torch.arange(n, dtype=torch.int32, device="cuda")
+        nxt = torch.zeros(n, dtype=torch.int32, device="cuda")
+        K.kfl_stage_prefill(st, ids, None, pos, 0, n, None, nxt, torch.cuda.current_stream().cuda_stream)
+        assert K.kfl_stage_status(st) == (K.KFL_ERR_OVERFLOW if big else 0)
+        K.kfl_stage_destroy(st)
