@@ -363,10 +363,33 @@ def empty_stage_ms(work, stream, n=50):
     return e0.elapsed_time(e1) / n
 
 
+def block_probe_stage(work, stream, o_ms, n=30):
+    """The per-format bandwidth probe of Eq. 2: one block of the workload's model, in its weight
+    format, at its batch and context, run as a body stage of its own (a device can time this
+    before any division of the blocks).  b = the block's algorithmic bytes / (its step time - o),
+    in GB/s, with o the empty stage's fixed time."""
+    import dataclasses
+
+    import torch
+
+    from paper_2609_34045_gb300 import device_inputs as di
+    from paper_2609_34045_gb300 import stage as K
+
+    one = dataclasses.replace(work, l0=0, l1=1, embed_in=False, logits_out=False, splits=())
+    st = K.kfl_stage_create(K.model_cfg(one.model, one.max_ctx, one.batch), 0, 1, 0)
+    di.load_stage_seeded(st, one)
+    inputs = step_inputs(one)
+    times, _ = time_steps(st, one, inputs, n, 5, 3, stream, None)
+    K.kfl_stage_destroy(st)
+    ms = statistics.median(times)
+    return one.step_bytes(0) / ((ms - o_ms) * 1e-3) / 1e9, ms
+
+
 def plan_example(work, fit):
-    """The planner (the exact fixed-order division with head rotation, section V) on a synthetic ring driven by this
-    GPU's measured stage cost: four members stream at 1, 1/2, 1/4 and 1/8 of the fitted rate b
-    with the fitted overhead o, and hold 35, 280, 140 and 70 GB; the bottleneck of the planned
+    """The planner (the exact fixed-order division with head rotation, section V) on a synthetic
+    ring driven by this GPU's measured stage cost: four members stream at 1, 1/2, 1/4 and 1/8 of
+    the probed rate b with the probed overhead o, and hold 35, 280, 140 and 70 GB; the bottleneck
+    of the planned
     division against the evaluation's Uniform and Memory-proportional divisions under the same
     costs (Eq. 2, ms per step)."""
     import dataclasses
@@ -402,12 +425,15 @@ def plan_example(work, fit):
     return out
 
 
-def cost_model(points, probe_gbs, o_ms):
+def cost_model(points, probe_gbs, o_ms, block_probe_gbs=None):
     """The paper's per-stage cost (Eq. 2), c = o + bytes / b: each stage's algorithmic HBM bytes
     (its blocks' weights and KV, and the head's embedding and unembedding) over a bandwidth b.
     points: [(bytes, measured ms)].  'probe' takes b from a copy benchmark and o from an empty
-    stage, as the planner would; 'fitted' takes (o, b) from a least-squares line through the
-    points.  Returns both, with each stage's predicted time and relative error."""
+    stage; 'block_probe' (when given) takes b from one block of the model run in the stage's own
+    weight format before any placement (block_probe_stage); both are what a planner can measure
+    ahead of dividing the blocks.  'fitted' takes (o, b) from a least-squares line through the
+    points (it needs the stages it predicts).  Returns each, with each stage's predicted time and
+    relative error."""
     import numpy as np
 
     x = np.array([p[0] for p in points], dtype=np.float64)
@@ -420,6 +446,8 @@ def cost_model(points, probe_gbs, o_ms):
                 "median_abs_err": float(np.median(np.abs(err)))}
 
     out = {"stage_bytes": x.tolist(), "measured_ms": y.tolist(), "probe": evaluate(o_ms, probe_gbs)}
+    if block_probe_gbs:
+        out["block_probe"] = evaluate(o_ms, block_probe_gbs)
     if len(points) >= 2 and np.ptp(x) > 0:
         slope, icpt = np.polyfit(x, y, 1)
         out["fitted"] = evaluate(float(icpt), float(1.0 / (slope * 1e6)))
@@ -640,9 +668,12 @@ def run_ours(args, work):
         points = [(work.step_bytes(work.steps // 2), ms)]
         for r in splits:
             points += list(zip(r["stage_bytes"], r["stage_ms"]))
-        cost = cost_model(points, measured_peaks()[0], empty_stage_ms(work, stream))
-        if "fitted" in cost:
-            cost["plan_example"] = plan_example(work, cost["fitted"])
+        o_ms = empty_stage_ms(work, stream)
+        probe_gbs, probe_ms = block_probe_stage(work, stream, o_ms)
+        cost = cost_model(points, measured_peaks()[0], o_ms, probe_gbs)
+        cost["block_probe_step_ms"] = probe_ms
+        # the planner runs on what it can measure before placing blocks: the block probe
+        cost["plan_example"] = plan_example(work, {"o_us": o_ms * 1e3, "b_gbs": probe_gbs})
     K.kfl_stage_destroy(st)
 
     also = None

@@ -21,6 +21,7 @@ constexpr int MAXB = 4;           // users per step
 constexpr int CONSUMER_WARPS = 8;
 constexpr int GEMV_THREADS = (CONSUMER_WARPS + 2) * 32;  // consumers, producer, epilogue warp
 constexpr int MAX_STAGES = 12;
+constexpr int MAX_CLUSTER = 8;  // CTAs of a split-K GEMV cluster (the portable cluster size)
 
 // int4 group-64 tiles: [N/RB][K/KT4], each 64 x 256 codes (8 KiB, in the order of the
 // tensor-core MMA fragments, see repack_int4_kernel) then [RB][KT4/64] bf16 scales
@@ -160,10 +161,11 @@ struct GemvParams {
   Act16 xin;          // this GEMV's input (int4 stages; x and ldx are then unused)
   Act16 xout;         // RESID / SWIGLU: the output in the same form (int4 stages; base NULL else)
   int xsplit;         // the input's rests are multiplied too (Q/K/V projection)
-  // one kernel per phase: launched as clusters of two CTAs, grid 2 n_rb, each CTA half the K
-  // range of one row block; the second hands its partial to the first through distributed
-  // shared memory instead of global memory and a ticket
-  int cluster2;
+  // one kernel per phase, cluster > 1: launched as clusters of `cluster` CTAs (at most
+  // MAX_CLUSTER), grid cluster x n_rb, each CTA 1/cluster of the K range of one row block; ranks
+  // 1.. hand their partials to rank 0 through distributed shared memory instead of global
+  // memory and a ticket
+  int cluster;
   // EPI_ARGMAX
   float *cand_val;
   int *cand_idx;
@@ -576,6 +578,7 @@ cudaError_t prepare_gemv();
 cudaError_t prepare_attention();
 cudaError_t launch_gemv(const GemvParams &p, int epi, int grid, cudaStream_t s, bool pdl);
 int gemv_max_stages(int batch, int fmt, int smem_optin);  // valid after prepare_gemv
+int gemv_stages_for(int batch, int fmt, int cluster, int per_sm);  // valid after prepare_gemv
 cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s, bool pdl);
 cudaError_t launch_qknorm(const QkNormParams &p, cudaStream_t s, bool pdl);
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in,

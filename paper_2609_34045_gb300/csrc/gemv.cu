@@ -42,8 +42,9 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
   __shared__ float s_inv[MAXB];
   __shared__ volatile int s_abort;
   __shared__ volatile int s_issued;
-  __shared__ __align__(16) float s_rx[RB * MAXB];  // cluster2: the partner CTA's partial
-  __shared__ __align__(8) uint64_t s_rx_bar;
+  __shared__ __align__(8) uint64_t s_rx_bar;  // cluster: rank 0 waits here for the other ranks' partials
+  // cluster: [cluster - 1][RB][MAXB] partials of ranks 1.., after the staging slots
+  float *rx = red + NSLOT * RB * MAXB;
 
   constexpr int KTILE = FMT == 0 ? KT : KT4;
   constexpr uint32_t WBYTES = FMT == 0 ? TILE_BYTES : TILE4_BYTES;
@@ -63,14 +64,14 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
       mbar_init(smem_addr(&seg_full[s]), CONSUMER_WARPS);
       mbar_init(smem_addr(&seg_empty[s]), 1);
     }
-    if (p.cluster2) mbar_init(smem_addr(&s_rx_bar), 1);
+    if (p.cluster > 1) mbar_init(smem_addr(&s_rx_bar), p.cluster - 1);
     s_abort = 0;
     s_issued = 0;
     fence_mbar_init();
   }
   for (int e = tid; e < NSLOT * RB * MAXB; e += GEMV_THREADS) red[e] = 0.f;  // int4 tiles add into it
   __syncthreads();
-  if (p.cluster2) cluster_sync_all();  // the partner writes s_rx / arrives on s_rx_bar only after this
+  if (p.cluster > 1) cluster_sync_all();  // the other ranks write rx / arrive on s_rx_bar only after this
   pdl_launch_dependents();
   auto stamp = [&](int slot) {
     if (p.trace) p.trace[(size_t)c * TRACE_SLOTS + slot] = global_ns();
@@ -136,7 +137,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
     bool inv_ready = true;
     int segc = 0;
     gemv_epilogues<B, EPI>(p, t0, n, T, G, c, sr, segc, s_inv, inv_ready, &s_abort, lane,
-                           p.cluster2 ? s_rx : nullptr, &s_rx_bar);
+                           p.cluster > 1 ? rx : nullptr, &s_rx_bar);
     if (lane == 0) stamp(TR_CONS_DONE);
     return;
   }
@@ -157,9 +158,9 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
 }
 
 // ---------------------------------------------------------------------------- launch
-static size_t gemv_smem_bytes(int stages, int batch, int fmt) {
+static size_t gemv_smem_bytes(int stages, int batch, int fmt, int cluster = 1) {
   return (size_t)stages * stage_bytes(batch, fmt) + (2 * stages + 2 * NSLOT) * sizeof(uint64_t) +
-         128 + NSLOT * RB * MAXB * sizeof(float);
+         128 + (NSLOT + (cluster > 1 ? cluster - 1 : 0)) * RB * MAXB * sizeof(float);
 }
 
 static int g_smem_optin = 0, g_smem_per_sm = 0, g_n_sm = 0;
@@ -180,7 +181,7 @@ static size_t gemv_launch_smem(size_t need, int grid) {
 template <int B, int EPI, int FMT>
 static cudaError_t launch_one(const GemvParams &p, int grid, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
-  const size_t smem = gemv_launch_smem(gemv_smem_bytes(p.stages, B, FMT), grid);
+  const size_t smem = gemv_launch_smem(gemv_smem_bytes(p.stages, B, FMT, p.cluster), grid);
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(GEMV_THREADS);
   cfg.dynamicSmemBytes = smem;
@@ -192,9 +193,9 @@ static cudaError_t launch_one(const GemvParams &p, int grid, cudaStream_t s, boo
     attr[na].val.programmaticStreamSerializationAllowed = 1;
     ++na;
   }
-  if (p.cluster2) {
+  if (p.cluster > 1) {
     attr[na].id = cudaLaunchAttributeClusterDimension;
-    attr[na].val.clusterDim.x = 2;
+    attr[na].val.clusterDim.x = p.cluster;
     attr[na].val.clusterDim.y = 1;
     attr[na].val.clusterDim.z = 1;
     ++na;
@@ -228,6 +229,18 @@ static cudaError_t launch_f(const GemvParams &p, int epi, int grid, cudaStream_t
 }
 
 // The deepest ring of this batch size and format that fits a CTA's shared memory.
+// The deepest ring such that `per_sm` CTAs of a GEMV with this cluster size fit one SM's shared
+// memory (each also holds its static shared memory and the per-CTA reservation).
+int gemv_stages_for(int batch, int fmt, int cluster, int per_sm) {
+  int s = GEMV_MAX_STAGES;
+  auto fits = [&](int st) {
+    const size_t cta = gemv_smem_bytes(st, batch, fmt, cluster) + GEMV_STATIC_SMEM;
+    return cta <= (size_t)g_smem_optin && (size_t)per_sm * (cta + 1024) <= (size_t)g_smem_per_sm;
+  };
+  while (s > 2 && !fits(s)) --s;
+  return s;
+}
+
 int gemv_max_stages(int batch, int fmt, int smem_optin) {
   int s = GEMV_MAX_STAGES;
   while (s > 2 && gemv_smem_bytes(s, batch, fmt) + GEMV_STATIC_SMEM > (size_t)smem_optin) --s;
@@ -236,9 +249,9 @@ int gemv_max_stages(int batch, int fmt, int smem_optin) {
 
 template <int B, int EPI, int FMT>
 static cudaError_t prepare_one() {
-  const size_t deepest = gemv_smem_bytes(gemv_max_stages(B, FMT, g_smem_optin), B, FMT);
+  // every launch asks for at most this (a deepest ring, or a cluster's partials with a shallower one)
   return cudaFuncSetAttribute(gemv_kernel<B, EPI, FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)gemv_launch_smem(deepest, 1));
+                              g_smem_optin - GEMV_STATIC_SMEM);
 }
 
 template <int EPI, int FMT>
@@ -276,8 +289,11 @@ cudaError_t prepare_gemv() {
 
 cudaError_t launch_gemv(const GemvParams &p, int epi, int grid, cudaStream_t s, bool pdl) {
   if (p.stages < 2 || p.stages > gemv_max_stages(p.batch, p.fmt, g_smem_optin)) return cudaErrorInvalidValue;
-  // clusters of two: each CTA exactly half the K range of one row block
-  if (p.cluster2 && (grid != 2 * p.n_rb || p.n_kt < 2)) return cudaErrorInvalidValue;
+  // clusters: each CTA exactly 1/cluster of the K range of one row block
+  if (p.cluster > 1 && (p.cluster > MAX_CLUSTER || grid != p.cluster * p.n_rb || p.n_kt < p.cluster))
+    return cudaErrorInvalidValue;
+  if (gemv_smem_bytes(p.stages, p.batch, p.fmt, p.cluster) + GEMV_STATIC_SMEM > (size_t)g_smem_optin)
+    return cudaErrorInvalidValue;
   return p.fmt == 0 ? launch_f<0>(p, epi, grid, s, pdl) : launch_f<1>(p, epi, grid, s, pdl);
 }
 

@@ -599,11 +599,12 @@ __device__ __forceinline__ void gemv_epilogues(const GemvParams &p, long long t0
     epilogue_prefetch<B, EPI>(p, rb, lane, pre);
     bool do_epi = true;
     if (!(kt0 == 0 && len == p.n_kt) && rx) {
-      // a cluster of two splits this row block's K range: rank 1 (the upper half) writes its
-      // partial into rank 0's shared memory and arrives on its barrier; rank 0 adds it to its own
-      // (the lower half first, as the ticket path sums in CTA order)
-      if (cluster_ctarank() == 1) {
-        const uint32_t dst = map_to_rank(smem_addr(rx), 0);
+      // a cluster of p.cluster CTAs splits this row block's K range: ranks 1.. write their
+      // partials into rank 0's shared memory (slot rank - 1) and arrive on its barrier; rank 0
+      // adds them to its own in rank order (K order, as the ticket path sums in CTA order)
+      const uint32_t rank = cluster_ctarank();
+      if (rank != 0) {
+        const uint32_t dst = map_to_rank(smem_addr(rx + (rank - 1) * (RB * MAXB)), 0);
         const float4 *r4 = reinterpret_cast<const float4 *>(red);
         for (int e = lane; e < RB * MAXB / 4; e += 32) st_cluster_f4(dst + e * 16, r4[e]);
         __syncwarp();
@@ -624,8 +625,12 @@ __device__ __forceinline__ void gemv_epilogues(const GemvParams &p, long long t0
           float4 *r4 = reinterpret_cast<float4 *>(red);
           const float4 *x4 = reinterpret_cast<const float4 *>(rx);
           for (int e = lane; e < RB * MAXB / 4; e += 32) {
-            const float4 a = r4[e], b = x4[e];
-            r4[e] = make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
+            float4 a = r4[e];
+            for (int j = 0; j + 1 < p.cluster; ++j) {
+              const float4 b = x4[j * (RB * MAXB / 4) + e];
+              a = make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
+            }
+            r4[e] = a;
           }
           __syncwarp();
         }

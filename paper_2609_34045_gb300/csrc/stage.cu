@@ -59,7 +59,7 @@ struct Plan {
   size_t kv_elems_per_layer;  // per cache (K or V)
   int n_sm, ctas_per_sm, stages, gemv_grid_max, n_rb_max, n_parts, attn_nchunks_max;
   int small_gemv_tiles, small_gemv_stages;  // GEMVs of at most this many tiles: one CTA per SM
-  int cluster2;                             // small GEMVs may run as clusters of two (see enqueue_body)
+  int cluster;                              // small GEMVs run as clusters of this many CTAs (see enqueue_body)
   int n_phases, ctr_stride;  // persistent kernel: phases per step, readiness counters per phase
   int attn_units;            // attention units a step aims at (the kernels size chunks to it)
   size_t bytes_weights, bytes_kv, bytes_ws;
@@ -134,7 +134,8 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   // GEMVs of fewer tiles keep one tile per CTA
   p->small_gemv_tiles = env_int("KFL_SMALL_GEMV_TILES", i4 ? 0 : 4096);
   p->small_gemv_stages = env_int("KFL_SMALL_GEMV_STAGES", 6);
-  p->cluster2 = env_int("KFL_GEMV_CLUSTER2", 1);
+  p->cluster = env_int("KFL_GEMV_CLUSTER", 3);
+  if (p->cluster > MAX_CLUSTER) p->cluster = MAX_CLUSTER;
   int nrb = 1;
   if (p->nl > 0) {
     nrb = p->qkv.n_rb;
@@ -577,13 +578,16 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
       GemvParams g = ph.g;
       if (T <= st->P.small_gemv_tiles && T >= 2LL * st->P.n_sm && st->P.ctas_per_sm > 1) {
         // a small GEMV: one CTA per SM with a deeper ring, so that fewer CTAs share a row block;
-        // with few enough row blocks, clusters of two CTAs split each one's K range and combine
-        // through distributed shared memory
+        // with few enough row blocks, clusters of N CTAs split each one's K range and combine
+        // through distributed shared memory (N row blocks' worth of CTAs at one or two per SM)
         grid = (int)(T < st->P.n_sm ? T : st->P.n_sm);
         g.stages = std::min(st->P.small_gemv_stages, gemv_max_stages(batch, g.fmt, st->smem_optin));
-        if (st->P.cluster2 && 2 * g.n_rb <= st->P.n_sm && g.n_kt >= 2) {
-          grid = 2 * g.n_rb;
-          g.cluster2 = 1;
+        const int N = st->P.cluster;
+        if (N >= 2 && g.n_kt >= N && (long long)N * g.n_rb <= 2LL * st->P.n_sm) {
+          const int per_sm = N * g.n_rb <= st->P.n_sm ? 1 : 2;
+          grid = N * g.n_rb;
+          g.cluster = N;
+          g.stages = std::min(st->P.small_gemv_stages, gemv_stages_for(batch, g.fmt, N, per_sm));
         }
       }
       CK(launch_gemv(g, ph.epi, grid, s, pdl));

@@ -20,5 +20,15 @@ def test_fit_recovers_overhead_and_bandwidth():
     assert f["median_abs_err"] < 1e-12
 
 
+def test_block_probe_is_evaluated_like_the_copy_probe():
+    pts = [(6e9, 2.0), (12e9, 3.0)]
+    r = bench.cost_model(pts, 6000.0, 0.5, block_probe_gbs=4000.0)
+    # 0.5 ms + 6e9 B / 4e12 B/s = 2.0 ms (exact), 0.5 + 3.0 = 3.5 ms (+1/6)
+    b = r["block_probe"]
+    assert abs(b["pred_ms"][0] - 2.0) < 1e-12 and abs(b["pred_ms"][1] - 3.5) < 1e-12
+    assert abs(b["median_abs_err"] - (0 + 1 / 6) / 2) < 1e-12
+    assert "block_probe" not in bench.cost_model(pts, 6000.0, 0.5)
+
+
 def test_single_point_has_no_fit():
     assert "fitted" not in bench.cost_model([(1e9, 1.0)], 6000.0, 0.1)

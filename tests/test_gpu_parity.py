@@ -280,19 +280,21 @@ def test_device_generator_is_bit_identical_to_host():
 # ---------------------------------------------------------------------------- full widths
 # (every block of each benchmark workload against the oracle: test_gpu_deep.py)
 
-def test_cluster_combine_agrees_with_the_ticket_combine(monkeypatch):
-    """At the 7B widths the Q/K/V and O GEMVs run as clusters of two CTAs (each half of a row
-    block's K range) that combine through distributed shared memory; with clusters off they run
-    stream-K over one CTA per SM and combine through global memory and a ticket.  The K ranges
-    are split at other points, so the sums differ only by rounding: within 1e-5 of the RMS."""
+@pytest.mark.parametrize("cluster", ["2", "3", "4", "8"])
+def test_cluster_combine_agrees_with_the_ticket_combine(cluster, monkeypatch):
+    """At the 7B widths the Q/K/V and O GEMVs run as clusters of N CTAs (each 1/N of a row
+    block's K range, at one or two CTAs per SM) that combine through distributed shared memory;
+    with clusters off they run stream-K over one CTA per SM and combine through global memory and
+    a ticket.  The K ranges are split at other points, so the sums differ only by rounding: within
+    1e-5 of the RMS."""
     from paper_2609_34045_gb300 import device_inputs as dev_in
     w = dataclasses.replace(wl.CONFIGS[2], l1=2)
     m = w.model
     cfg = K.model_cfg(m, w.max_ctx, 1)
     stream = torch.cuda.current_stream().cuda_stream
     outs = []
-    for cluster in ("1", "0"):
-        monkeypatch.setenv("KFL_GEMV_CLUSTER2", cluster)
+    for n in (cluster, "0"):
+        monkeypatch.setenv("KFL_GEMV_CLUSTER", n)
         st = K.kfl_stage_create(cfg, 0, 2, 0)
         dev_in.load_stage_seeded(st, w)
         cap = torch.zeros(2, 1, m.d_model, device="cuda")
