@@ -12,9 +12,10 @@
 //
 // 256 threads.  Scores S = q K^T and the weighted sum P V are small dense products (at most 8
 // heads x 64 positions x hd): both run on the tensor cores as warp-level bf16 m16n8k16 MMAs with
-// fp32 accumulation (the heads are the M rows, padded to 16).  q and P enter as bf16 pairs
-// (rounded value and the bf16 rounding of the rest, each pair multiplied separately: about 2^-17
-// relative); K and V are the cache's bf16 values, exact.  Scores: warp w takes positions
+// fp32 accumulation.  q and P enter as bf16 pairs (rounded value and the bf16 rounding of the
+// rest: about 2^-17 relative), the rounded parts in the A operand's rows 0..7 (the heads) and the
+// rests in rows 8..15, so one MMA gives both products; K and V are the cache's bf16 values,
+// exact.  Scores: warp w takes positions
 // 8w..8w+7; P V: warp w takes head dimensions hd/8 * w onwards.
 #pragma once
 
@@ -173,13 +174,13 @@ __device__ __forceinline__ void attn_publish(const AttnParams &p, int kvh, int t
 }
 
 // d += a b for one m16n8k16 bf16 tile (a: 16x16 row-major, b: 16x8 column-major, fp32
-// accumulate).  Rows 8..15 of a are the zero padding of the at most 8 heads, so a1 = a3 = 0.
-__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
-  asm(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+// accumulate).  Rows 0..7 of a hold the heads' rounded parts and rows 8..15 their rests (bf16
+// pairs of q or P), so accumulator rows g and g + 8, which one lane holds, add up to head g's.
+__device__ __forceinline__ void mma_bf16_full(float (&d)[4], const uint4 &a, uint32_t b0, uint32_t b1) {
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
       "{%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
+      : "r"(a.x), "r"(a.y), "r"(a.z), "r"(a.w), "r"(b0), "r"(b1));
 }
 
 // Four (two) 8 x 8 blocks of 16-bit values, transposed: lanes 8 i .. 8 i + 7 address the rows of
@@ -263,8 +264,8 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
   {
     // q (scaled to log2 units) as the scores' A fragments, a bf16 pair each (rounded, rest:
     // about 2^-17 relative, for the softmax turns a relative error e of a score s into an error
-    // of about |s| e of its weight): entry (step s, lane) = rounded a0, a2, rest a0, a2 of rows
-    // gid (heads; rows gid + 8 and gid >= G are zero)
+    // of about |s| e of its weight): entry (step s, lane) = registers a0..a3, rows gid the
+    // heads' rounded parts and rows gid + 8 their rests; rows of heads >= G are zero
     if (tid < KS * 32) {
       const int st = tid >> 5, l = tid & 31, g = l >> 2, t = l & 3;
       uint4 f = make_uint4(0u, 0u, 0u, 0u);
@@ -279,8 +280,8 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
           hi[i] = f32_to_bf16_rne(v[i]);
           lo[i] = f32_to_bf16_rne(v[i] - bf16_to_f32(hi[i]));
         }
-        f = make_uint4(hi[0] | ((uint32_t)hi[1] << 16), hi[2] | ((uint32_t)hi[3] << 16),
-                       lo[0] | ((uint32_t)lo[1] << 16), lo[2] | ((uint32_t)lo[3] << 16));
+        f = make_uint4(hi[0] | ((uint32_t)hi[1] << 16), lo[0] | ((uint32_t)lo[1] << 16),
+                       hi[2] | ((uint32_t)hi[3] << 16), lo[2] | ((uint32_t)lo[3] << 16));
       }
       qf[tid] = f;
     }
@@ -316,27 +317,25 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
       for (int e = tid; e < (ATT_SUB - cnt) * (HD / 8); e += ATT_THREADS)
         *reinterpret_cast<uint4 *>(vb + (cnt + e / (HD / 8)) * L::VROW + (e % (HD / 8)) * 16) = make_uint4(0u, 0u, 0u, 0u);
 
-    // scores of positions 8w .. 8w + 7 (MMA columns) for every head (rows gid): bf16 m16n8k16
-    // MMAs, K rows as the B fragments (two 32-bit loads per step); four independent accumulator
-    // chains (K steps modulo 2, rounded and rest parts of q) so that the MMAs overlap
+    // scores of positions 8w .. 8w + 7 (MMA columns) for every head (rows gid, rests gid + 8):
+    // bf16 m16n8k16 MMAs, K rows as the B fragments (two 32-bit loads per step); two
+    // independent accumulator chains (K steps modulo 2) so that the MMAs overlap
     {
-      float sp[4][4] = {};
+      float sp[2][4] = {};
       const uint8_t *krow = kb + (8 * warp + gid) * L::KROW + 4 * tig;
 #pragma unroll
       for (int s16 = 0; s16 < KS; ++s16) {
         const uint4 f = qf[s16 * 32 + lane];
         const uint32_t k0 = *reinterpret_cast<const uint32_t *>(krow + 32 * s16);
         const uint32_t k1 = *reinterpret_cast<const uint32_t *>(krow + 32 * s16 + 16);
-        mma_bf16_16816(sp[2 * (s16 & 1)], f.x, f.y, k0, k1);
-        mma_bf16_16816(sp[2 * (s16 & 1) + 1], f.z, f.w, k0, k1);
+        mma_bf16_full(sp[s16 & 1], f, k0, k1);
       }
-      float sc[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) sc[i] = (sp[0][i] + sp[2][i]) + (sp[1][i] + sp[3][i]);
       if (hrow) {
+        const float s0 = (sp[0][0] + sp[1][0]) + (sp[0][2] + sp[1][2]);
+        const float s1 = (sp[0][1] + sp[1][1]) + (sp[0][3] + sp[1][3]);
         const int pp = 8 * warp + 2 * tig;
         *reinterpret_cast<float2 *>(ss + gid * L::SS + pp) =
-            make_float2(pp < cnt ? sc[0] : -INFINITY, pp + 1 < cnt ? sc[1] : -INFINITY);
+            make_float2(pp < cnt ? s0 : -INFINITY, pp + 1 < cnt ? s1 : -INFINITY);
       }
     }
     att_sync();
@@ -353,14 +352,14 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
       float sum = e0 + e1;
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-      // position pp of the sub-tile: step pp / 16, lane 4 g + ((pp & 7) >> 1), register a0 or a2
-      // (pp & 8), half pp & 1
+      // position pp of the sub-tile: step pp / 16, lane 4 g + ((pp & 7) >> 1), registers a0
+      // (rounded part) and a1 (rest) or, for pp & 8, a2 and a3; half pp & 1
       auto put = [&](int pp, float e) {
         uint16_t *f = reinterpret_cast<uint16_t *>(pf + (pp >> 4) * 32 + 4 * g + ((pp & 7) >> 1));
         const uint16_t hi = f32_to_bf16_rne(e);
-        const int r = (pp & 8) ? 1 : 0;
-        f[2 * r + (pp & 1)] = hi;
-        f[2 * (2 + r) + (pp & 1)] = f32_to_bf16_rne(e - bf16_to_f32(hi));
+        const int reg = (pp & 8) ? 2 : 0;
+        f[2 * reg + (pp & 1)] = hi;
+        f[2 * (reg + 1) + (pp & 1)] = f32_to_bf16_rne(e - bf16_to_f32(hi));
       };
       put(lane, e0);
       put(lane + 32, e1);
@@ -375,13 +374,13 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
     // acc = acc * alpha + P V over the sub-tile: P fragments from shared memory, V fragments by
     // transposing loads (ldmatrix .trans: 8 x 8 blocks of positions x dimensions)
     {
+      // rows gid (P's rounded parts) and gid + 8 (rests) are both head gid's
       const float al = hrow ? s_alpha[gid] : 0.f;
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt) {
-        acc[nt][0] *= al;
-        acc[nt][1] *= al;
-      }
-      // this sub-tile's P V in two chains per n-tile (rounded and rest parts of P), then into acc
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc[nt][i] *= al;
+      // this sub-tile's P V in two chains per n-tile (K steps modulo 2), then into acc
       float pv[NT][2][4] = {};
       const int mi = lane >> 3;  // the 8 x 8 block whose row this lane addresses
       const uint8_t *vrow = vb + (8 * (mi & 1) + (lane & 7)) * L::VROW + 2 * (n_base + 8 * (mi >> 1));
@@ -391,15 +390,12 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
         if constexpr (NT == 2) {
           uint32_t v0, v1, v2, v3;
           ldsm_x4_trans(v0, v1, v2, v3, vrow + 16 * s16 * L::VROW);
-          mma_bf16_16816(pv[0][0], f.x, f.y, v0, v1);
-          mma_bf16_16816(pv[0][1], f.z, f.w, v0, v1);
-          mma_bf16_16816(pv[1][0], f.x, f.y, v2, v3);
-          mma_bf16_16816(pv[1][1], f.z, f.w, v2, v3);
+          mma_bf16_full(pv[0][s16 & 1], f, v0, v1);
+          mma_bf16_full(pv[1][s16 & 1], f, v2, v3);
         } else {
           uint32_t v0, v1;
           ldsm_x2_trans(v0, v1, vrow + 16 * s16 * L::VROW);
-          mma_bf16_16816(pv[0][0], f.x, f.y, v0, v1);
-          mma_bf16_16816(pv[0][1], f.z, f.w, v0, v1);
+          mma_bf16_full(pv[0][s16 & 1], f, v0, v1);
         }
       }
 #pragma unroll
@@ -418,7 +414,7 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
           *reinterpret_cast<float2 *>(o + gid * HD + n_base + 8 * nt + 2 * tig) =
-              make_float2(acc[nt][0] * il, acc[nt][1] * il);
+              make_float2((acc[nt][0] + acc[nt][2]) * il, (acc[nt][1] + acc[nt][3]) * il);
       }
     } else {
       // through shared memory (the K buffers) into the output mapping of the merge
@@ -428,7 +424,7 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
           *reinterpret_cast<float2 *>(so + gid * HD + n_base + 8 * nt + 2 * tig) =
-              make_float2(acc[nt][0] * il, acc[nt][1] * il);
+              make_float2((acc[nt][0] + acc[nt][2]) * il, (acc[nt][1] + acc[nt][3]) * il);
       }
       att_sync();
       const float4 v = owns ? *reinterpret_cast<const float4 *>(so + og * HD + od) : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -444,7 +440,8 @@ __device__ void attn_unit(const AttnParams &p, int b, int kvh, int c, int nc, ui
   if (hrow) {
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt)
-      *reinterpret_cast<float2 *>(part + gid * PS + n_base + 8 * nt + 2 * tig) = make_float2(acc[nt][0], acc[nt][1]);
+      *reinterpret_cast<float2 *>(part + gid * PS + n_base + 8 * nt + 2 * tig) =
+          make_float2(acc[nt][0] + acc[nt][2], acc[nt][1] + acc[nt][3]);
   }
   if (tid < G) {
     part[tid * PS + HD] = s_m[tid];

@@ -22,6 +22,7 @@ constexpr int CONSUMER_WARPS = 8;
 constexpr int GEMV_THREADS = (CONSUMER_WARPS + 2) * 32;  // consumers, producer, epilogue warp
 constexpr int MAX_STAGES = 12;
 constexpr int MAX_CLUSTER = 8;  // CTAs of a split-K GEMV cluster (the portable cluster size)
+constexpr int MAX_CLUSTER_ATT = 16;  // CTAs of an attention cluster (non-portable above 8)
 
 // int4 group-64 tiles: [N/RB][K/KT4], each 64 x 256 codes (8 KiB, in the order of the
 // tensor-core MMA fragments, see repack_int4_kernel) then [RB][KT4/64] bf16 scales
@@ -209,6 +210,10 @@ struct AttnParams {
   // (attn_chunk_size), so that a step has about target_units units; the partial buffer holds
   // n_chunks (= max_ctx / 64, rounded up) chunks per (user, KV head)
   int chunk, n_chunks, target_units;
+  // one kernel per phase: > 0 runs attn_cluster_kernel, one thread-block cluster of `cluster`
+  // CTAs per (user, KV head) that split its positions and merge through distributed shared
+  // memory (partial, tickets, chunk and target_units are then unused)
+  int cluster;
   float scale_log2;          // log2(e) / sqrt(hd)
   unsigned *err;
   // dataflow (persistent stage kernel only)
@@ -311,6 +316,19 @@ __device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
   uint32_t r;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
   return r;
+}
+__device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ float ld_cluster_f32(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+  return v;
 }
 __device__ __forceinline__ void st_cluster_f4(uint32_t addr, float4 v) {
   asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(v.x), "f"(v.y), "f"(v.z),
@@ -581,6 +599,9 @@ int gemv_max_stages(int batch, int fmt, int smem_optin);  // valid after prepare
 int gemv_stages_for(int batch, int fmt, int cluster, int per_sm);  // valid after prepare_gemv
 cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s, bool pdl);
 cudaError_t launch_qknorm(const QkNormParams &p, cudaStream_t s, bool pdl);
+cudaError_t prepare_attention_cluster();
+int attention_cluster_size(int head_dim, int want);  // valid after prepare_attention_cluster
+cudaError_t launch_attention_cluster(const AttnParams &p, int head_dim, cudaStream_t s, bool pdl);
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in,
                                int batch, const uint16_t *embed, int vocab, int d, int ldh,
                                const float *g_next, float *h, float *xn, float *sumsq,

@@ -62,6 +62,7 @@ struct Plan {
   int cluster;                              // small GEMVs run as clusters of this many CTAs (see enqueue_body)
   int n_phases, ctr_stride;  // persistent kernel: phases per step, readiness counters per phase
   int attn_units;            // attention units a step aims at (the kernels size chunks to it)
+  int attn_cluster_max;      // one kernel per phase: the largest attention cluster (0: unit kernel)
   size_t bytes_weights, bytes_kv, bytes_ws;
 };
 
@@ -317,7 +318,7 @@ GemvParams base_gemv(kfl_stage *st, const Mat &m, const float *x, int ldx, int b
   g.x = x;
   g.ldx = ldx;
   g.batch = batch;
-  g.stages = std::min(st->P.stages, gemv_max_stages(batch, m.fmt, st->smem_optin));
+  g.stages = std::min(st->P.stages, gemv_stages_for(batch, m.fmt, 1, st->P.ctas_per_sm));
   g.rope_per_user = 0;
   g.partial = st->gemv_partial;
   g.tickets = st->tickets;
@@ -399,6 +400,17 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
       a.chunk = std::max(1, env_int("KFL_ATTN_MIN_CHUNK", 64) / 64) * 64;  // the kernels size the step's chunks from its positions (at least this)
       a.n_chunks = (c.max_ctx + 63) / 64;
       a.target_units = P.attn_units;
+      if (!dataflow && P.attn_cluster_max >= 2) {
+        // one cluster per (user, KV head): the largest power of two up to the maximum with at
+        // most two CTAs per SM in all
+        int cl = P.attn_cluster_max;
+        while (cl > 2 && (long long)cl * batch * P.hkv > 2LL * P.n_sm) cl >>= 1;
+        // the clusters cannot balance ragged users or spread a long context over idle SMs: they
+        // are taken when each CTA has at most five 64-position sub-tiles at the longest context
+        // (the merge latency then dominates) or when they give every SM at least one CTA
+        const int per_cta = (c.max_ctx + cl - 1) / cl;
+        if (per_cta <= 5 * 64 || (long long)cl * batch * P.hkv >= P.n_sm) a.cluster = cl;
+      }
       a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)P.hd));
       a.err = st->err;
       if (c.qk_norm) {
@@ -560,6 +572,29 @@ int phase_kind_code(const Phase &ph, size_t i) {
   }
 }
 
+// The launch shape of a GEMV phase in the one-kernel-per-phase mode: sets g's ring depth and
+// cluster size and returns its grid.  Every shape is a stream-K split: CTA c streams tiles
+// [c T / G, (c + 1) T / G) (a cluster of N CTAs per row block is the split with G = N n_rb).
+int gemv_launch_shape(const kfl_stage *st, int batch, GemvParams &g) {
+  const long long T = (long long)g.n_rb * g.n_kt;
+  int grid = (int)(T < st->P.gemv_grid_max ? T : st->P.gemv_grid_max);
+  if (T <= st->P.small_gemv_tiles && T >= 2LL * st->P.n_sm && st->P.ctas_per_sm > 1) {
+    // a small GEMV: one CTA per SM with a deeper ring, so that fewer CTAs share a row block;
+    // with few enough row blocks, clusters of N CTAs split each one's K range and combine
+    // through distributed shared memory (N row blocks' worth of CTAs at one or two per SM)
+    grid = (int)(T < st->P.n_sm ? T : st->P.n_sm);
+    g.stages = std::min(st->P.small_gemv_stages, gemv_max_stages(batch, g.fmt, st->smem_optin));
+    const int N = st->P.cluster;
+    if (N >= 2 && g.n_kt >= N && (long long)N * g.n_rb <= 2LL * st->P.n_sm) {
+      const int per_sm = N * g.n_rb <= st->P.n_sm ? 1 : 2;
+      grid = N * g.n_rb;
+      g.cluster = N;
+      g.stages = std::min(st->P.small_gemv_stages, gemv_stages_for(batch, g.fmt, N, per_sm));
+    }
+  }
+  return grid;
+}
+
 // Per-kernel mode: one launch per phase on stream s (chained with PDL when pdl is set).  With
 // `kinds` (profiling, no PDL) the k-th launch is bracketed by events ev[2(ev_base+k)] and
 // ev[2(ev_base+k)+1] and its kind appended to *kinds.
@@ -573,27 +608,15 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
       kinds->push_back(phase_kind_code(ph, i));
     }
     if (ph.kind == PH_GEMV) {
-      const long long T = (long long)ph.g.n_rb * ph.g.n_kt;
-      int grid = (int)(T < st->P.gemv_grid_max ? T : st->P.gemv_grid_max);
       GemvParams g = ph.g;
-      if (T <= st->P.small_gemv_tiles && T >= 2LL * st->P.n_sm && st->P.ctas_per_sm > 1) {
-        // a small GEMV: one CTA per SM with a deeper ring, so that fewer CTAs share a row block;
-        // with few enough row blocks, clusters of N CTAs split each one's K range and combine
-        // through distributed shared memory (N row blocks' worth of CTAs at one or two per SM)
-        grid = (int)(T < st->P.n_sm ? T : st->P.n_sm);
-        g.stages = std::min(st->P.small_gemv_stages, gemv_max_stages(batch, g.fmt, st->smem_optin));
-        const int N = st->P.cluster;
-        if (N >= 2 && g.n_kt >= N && (long long)N * g.n_rb <= 2LL * st->P.n_sm) {
-          const int per_sm = N * g.n_rb <= st->P.n_sm ? 1 : 2;
-          grid = N * g.n_rb;
-          g.cluster = N;
-          g.stages = std::min(st->P.small_gemv_stages, gemv_stages_for(batch, g.fmt, N, per_sm));
-        }
-      }
+      const int grid = gemv_launch_shape(st, batch, g);
       CK(launch_gemv(g, ph.epi, grid, s, pdl));
     } else {
       if (ph.qn.raw) CK(launch_qknorm(ph.qn, s, pdl));  // QK-norm stages: norm, RoPE, KV append
-      CK(launch_attention(ph.a, st->P.hd, s, pdl));
+      if (ph.a.cluster > 0)
+        CK(launch_attention_cluster(ph.a, st->P.hd, s, pdl));
+      else
+        CK(launch_attention(ph.a, st->P.hd, s, pdl));
     }
     if (kinds) CK(cudaEventRecord(st->ev[2 * k + 1], s));
     ++k;
@@ -1095,6 +1118,7 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
   CK(cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev));
   CK(prepare_gemv());
   CK(prepare_attention());
+  CK(prepare_attention_cluster());
   int smem_optin = 0;
   CK(cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev));
   kfl_stage *st = new kfl_stage();
@@ -1107,6 +1131,10 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
   st->fault_at = env_int("KFL_FAULT_ALLOC_AT", 0);
   make_plan(cfg, l0, l1, flags, n_sm, &st->P);
   Plan &P = st->P;
+  {
+    const int want = env_int("KFL_ATTN_CLUSTER", MAX_CLUSTER_ATT);
+    P.attn_cluster_max = want >= 2 ? attention_cluster_size(P.hd, std::min(want, MAX_CLUSTER_ATT)) : 0;
+  }
   auto fail = [&](int code) {
     kfl_stage_destroy(st);
     return code;

@@ -153,16 +153,18 @@ def test_deterministic_replay_and_profile_mode(monkeypatch):
     c1 = p.cap.cpu().numpy().copy()
     h2, n2 = p.gpu_step(pos, ids=ids)  # rewrites the same slots with the same values
     assert np.array_equal(h1, h2) and np.array_equal(n1, n2)
-    # per-kernel mode (one launch per phase, events around each) gives the same bits as the
-    # persistent stage kernel
+    # per-kernel mode (one launch per phase, events around each) against the persistent stage
+    # kernel: its attention splits the positions differently (one cluster per user and KV head),
+    # so the sums differ by rounding only
     assert K.kfl_stage_launches_per_step(p.st, 3) == 3
     K.kfl_stage_profile(p.st, True)
     assert K.kfl_stage_launches_per_step(p.st, 3) == 2 + 5 * 3 + 1
     h3, n3 = p.gpu_step(pos, ids=ids)
     prof = K.kfl_stage_profile_read(p.st)
     K.kfl_stage_profile(p.st, False)
-    assert np.array_equal(h1, h3) and np.array_equal(n1, n3)
-    assert np.array_equal(c1, p.cap.cpu().numpy())
+    for a, b in ((h1, h3), (c1, p.cap.cpu().numpy())):
+        assert np.max(np.abs(a - b)) <= 1e-5 * np.sqrt(np.mean(b.astype(np.float64) ** 2))
+    assert np.array_equal(n1, n3)
     assert prof["qkv"][1] == 3 and prof["attn"][1] == 3 and prof["oproj"][1] == 3 and prof["down"][1] == 3
     assert prof["lmhead"][1] == 1 and prof["gateup"][1] == 3
     assert all(ms > 0 for ms, n in prof.values() if n > 0)
@@ -275,6 +277,17 @@ def test_device_generator_is_bit_identical_to_host():
     K.kfl_synth_fill(t, 1000, 7, 9, K.SYNTH_NORMAL_BF16, float(wl.normal_scale(1.0)), 0.0, start=(1 << 33) + 5)
     idx = np.arange((1 << 33) + 5, (1 << 33) + 1005, dtype=np.uint64)
     assert np.array_equal(t.cpu().numpy().view(np.uint16), wl.normal_bf16_at(7, 9, idx, 1.0))
+
+
+@pytest.mark.parametrize("attn_cluster", ["16", "2", "0"])
+def test_attention_kernels_ragged_users(attn_cluster, monkeypatch):
+    """One kernel per phase, attention either as one thread-block cluster per (user, KV head)
+    whose CTAs merge through distributed shared memory (16 or 2 CTAs) or as the unit kernel with
+    its global chunk partials (0): each against the oracle, ragged users crossing sub-tiles."""
+    monkeypatch.setenv("KFL_ATTN_CLUSTER", attn_cluster)
+    p = Pair(RAGGED, 0, 3, K.KFL_IS_HEAD, 4, (0, 63, 64, 250), 320, seed=26)
+    _greedy(p, 3, wl.token_ids(26, 97, 4, RAGGED.vocab))
+    p.close()
 
 
 # ---------------------------------------------------------------------------- full widths
