@@ -25,12 +25,23 @@ constexpr int MAX_CLUSTER = 8;  // CTAs of a split-K GEMV cluster (the portable 
 constexpr int MAX_CLUSTER_ATT = 16;  // CTAs of an attention cluster (non-portable above 8)
 
 // int4 group-64 tiles: [N/RB][K/KT4], each 64 x 256 codes (8 KiB, in the order of the
-// tensor-core MMA fragments, see repack_int4_kernel) then [RB][KT4/64] bf16 scales
+// tensor-core MMA fragments, see repack_int4_kernel) then RB x KT4/64 bf16 scales (in the order of
+// tile4_scale_index)
 constexpr int KT4 = 256;
 constexpr int TILE4_CODE_BYTES = RB * KT4 / 2;     // 8 KiB
 constexpr int TILE4_SCALE_BYTES = RB * (KT4 / 64) * 2;  // 512 B
 constexpr int TILE4_BYTES = TILE4_CODE_BYTES + TILE4_SCALE_BYTES;
 
+// Position (in bf16 units, after the codes) of the scale of row r (0..63) and weight group g4
+// (0..3) of an int4 tile: grouped by the consumer warp that reads them (weight group g4), then by
+// the lane's row gid = r % 8, so that one 16-byte load gives a lane the scales of rows gid and
+// gid + 8 of all four row groups r / 16 of its group.
+__host__ __device__ constexpr int tile4_scale_index(int r, int g4) {
+  return ((g4 * 8 + (r & 7)) * 4 + (r >> 4)) * 2 + ((r >> 3) & 1);
+}
+// A weight-ring depth usable by this format: int4 rings have an even number of stages (each stage
+// then belongs to one of the two consumer teams, gemv_consume_int4).
+__host__ __device__ constexpr int ring_depth(int fmt, int stages) { return fmt == 0 ? stages : (stages & ~1); }
 __host__ __device__ constexpr int tile_k(int fmt) { return fmt == 0 ? KT : KT4; }
 __host__ __device__ constexpr int tile_bytes(int fmt) { return fmt == 0 ? TILE_BYTES : TILE4_BYTES; }
 // A ring stage holds one weight tile and the activations of its K range: bf16 tiles, the B
@@ -41,8 +52,8 @@ constexpr int X16_SRC_BYTES = KT4 * 2;              // 512
 // 576: the sources start on different halves of the banks, so that the 16-byte B-fragment loads of
 // one quarter warp (two sources) fall in distinct banks
 constexpr int X16_SRC_STRIDE = X16_SRC_BYTES + 64;
-constexpr int XC_CHUNK_FLOATS = 32;                 // per chunk: [4 lane quads][8]
-constexpr int XC_TILE_BYTES = (KT4 / XCHUNK) * XC_CHUNK_FLOATS * 4;  // 1024
+constexpr int XC_GROUP_BYTES = 192;                 // per weight group (two chunks): 3 x [4 lane quads][4]
+constexpr int XC_TILE_BYTES = (KT4 / (2 * XCHUNK)) * XC_GROUP_BYTES;  // 768
 // Bytes of one K tile's block of an Act16 (rest: with the rests' rows), and the part of it a
 // GEMV at batch B copies into a ring stage: the constants and the rounded parts of users
 // 0..B-1, or (xsplit) all MAXB rounded parts and the rests of users 0..B-1.
@@ -67,9 +78,10 @@ constexpr int STAGE_BYTES_MAX = stage_bytes(MAXB, 0);
 // over (the rest), in fp16.
 // Layout, tile-major so that a ring stage's activations are one contiguous copy: per K tile of
 // KT4 elements a block of act16_tile_bytes(rest) bytes, holding
-//   [0, XC_TILE_BYTES): the chunk constants, per chunk [t][0..7] for MMA columns 2t, 2t+1:
-//     minus their offset sums twice over (the MMA's accumulator quad of rows gid and gid + 8),
-//     then their multipliers m and two unused floats; column u < 4 is user u's rounded part and
+//   [0, XC_TILE_BYTES): the chunk constants, per weight group of two chunks (a, b) three blocks
+//     [t][0..3] for MMA columns 2t, 2t+1: chunk a's seed, chunk b's seed, then the multipliers
+//     (m_a(2t), m_a(2t+1), m_b(2t), m_b(2t+1)); a seed is minus the columns' offset sums twice over
+//     (the MMA's accumulator quad of rows gid and gid + 8); column u < 4 is user u's rounded part and
 //     column u + 4 its rest, and a column's offset sum is the sum over the chunk of its fp16
 //     values times 1032 (block elements 0..7) or 1152 (8..15): what the decoder's offsets add
 //     to the MMA's product;
@@ -96,9 +108,9 @@ __host__ __device__ inline uint16_t *act16_elem(const Act16 &a, int r, int k) {
   return reinterpret_cast<uint16_t *>(act16_tile(a, k / KT4) + XC_TILE_BYTES + r * X16_SRC_STRIDE) +
          act16_index(k % KT4);
 }
-// The constants of chunk ch.
+// The constants block of the weight group holding chunk ch.
 __host__ __device__ inline float *act16_consts(const Act16 &a, int ch) {
-  return reinterpret_cast<float *>(act16_tile(a, ch / (KT4 / XCHUNK))) + (ch % (KT4 / XCHUNK)) * XC_CHUNK_FLOATS;
+  return reinterpret_cast<float *>(act16_tile(a, ch / (KT4 / XCHUNK)) + ((ch % (KT4 / XCHUNK)) >> 1) * XC_GROUP_BYTES);
 }
 
 // ---- device error word bits ---------------------------------------------------------------
@@ -508,14 +520,12 @@ __device__ __forceinline__ float f16_to_f32(uint16_t h) {
 
 // Chunk ch's constants for user b (column b: rounded part, column b + 4: rest).
 __device__ __forceinline__ void act16_put_consts(const Act16 &a, int b, int ch, float m, float off_hi, float off_lo) {
-  float *c = act16_consts(a, ch);
+  float *g = act16_consts(a, ch);
+  float *seed = g + (ch & 1) * 16, *mult = g + 32 + (ch & 1) * 2;
   const int t = b >> 1, j = b & 1;
-  c[t * 8 + j] = -off_hi;
-  c[t * 8 + 2 + j] = -off_hi;
-  c[t * 8 + 4 + j] = m;
-  c[(t + 2) * 8 + j] = -off_lo;
-  c[(t + 2) * 8 + 2 + j] = -off_lo;
-  c[(t + 2) * 8 + 4 + j] = m;
+  seed[t * 4 + j] = seed[t * 4 + 2 + j] = -off_hi;
+  seed[(t + 2) * 4 + j] = seed[(t + 2) * 4 + 2 + j] = -off_lo;
+  mult[t * 4 + j] = mult[(t + 2) * 4 + j] = m;
 }
 
 // Chunk ch of user b of an Act16, one element per lane (x = 0 past the vector's end); the whole

@@ -26,7 +26,7 @@ constexpr int GEMV_MAX_STAGES = 13;  // 13 x 16.9 KiB (batch 1) still fits one C
 constexpr int GEMV_STATIC_SMEM = 3072;  // allowance for the kernel's own __shared__ variables
 
 // ---------------------------------------------------------------------------- the kernel
-// FMT 0: bf16 tiles [RB][KT].  FMT 1: int4 tiles, codes [RB][KT4/8] uint32 + scales [RB][KT4/64].
+// FMT 0: bf16 tiles [RB][KT].  FMT 1: int4 tiles, codes [RB][KT4/8] uint32 + RB x KT4/64 scales.
 // Warps 0-7 consume tiles, warp 8 is the TMA producer, warp 9 the epilogue warp.
 template <int B, int EPI, int FMT>
 __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_constant__ GemvParams p) {
@@ -37,14 +37,14 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
   uint64_t *empty = full + S;
   uint64_t *seg_full = empty + S;
   uint64_t *seg_empty = seg_full + NSLOT;
-  // [NSLOT][RB][MAXB], 128-byte aligned (read as float4)
+  // staging slots (SegRing: seg_floats(FMT) floats), 128-byte aligned (read as float4)
   float *red = reinterpret_cast<float *>((reinterpret_cast<uintptr_t>(seg_empty + NSLOT) + 127) & ~uintptr_t(127));
   __shared__ float s_inv[MAXB];
   __shared__ volatile int s_abort;
   __shared__ volatile int s_issued;
   __shared__ __align__(8) uint64_t s_rx_bar;  // cluster: rank 0 waits here for the other ranks' partials
   // cluster: [cluster - 1][RB][MAXB] partials of ranks 1.., after the staging slots
-  float *rx = red + NSLOT * RB * MAXB;
+  float *rx = red + seg_floats(FMT);
 
   constexpr int KTILE = FMT == 0 ? KT : KT4;
   constexpr uint32_t WBYTES = FMT == 0 ? TILE_BYTES : TILE4_BYTES;
@@ -53,12 +53,12 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
   const int G = gridDim.x, c = blockIdx.x;
   const long long t0 = (long long)c * T / G, t1 = (long long)(c + 1) * T / G;
   const int n = static_cast<int>(t1 - t0);
-  const SegRing sr = {red, seg_full, seg_empty};
+  const SegRing sr = {red, seg_full, seg_empty, seg_slots(FMT), seg_subs(FMT)};
 
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_addr(&full[s]), 1);
-      mbar_init(smem_addr(&empty[s]), CONSUMER_WARPS);
+      mbar_init(smem_addr(&empty[s]), ring_empty_count(FMT));
     }
     for (int s = 0; s < NSLOT; ++s) {
       mbar_init(smem_addr(&seg_full[s]), CONSUMER_WARPS);
@@ -69,7 +69,7 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
     s_issued = 0;
     fence_mbar_init();
   }
-  for (int e = tid; e < NSLOT * RB * MAXB; e += GEMV_THREADS) red[e] = 0.f;  // int4 tiles add into it
+  for (int e = tid; e < seg_floats(FMT); e += GEMV_THREADS) red[e] = 0.f;  // int4 tiles add into it
   __syncthreads();
   if (p.cluster > 1) cluster_sync_all();  // the other ranks write rx / arrive on s_rx_bar only after this
   pdl_launch_dependents();
@@ -145,7 +145,13 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
   // -------------------------------------------------------------------- consumers
   int s = 0, segc = 0;
   uint32_t phase = 0;
-  gemv_consume<B, FMT>(p.n_kt, smem, full, empty, S, s, phase, t0, n, sr, segc, &s_abort, p.err, tid, p.xsplit != 0);
+  if constexpr (FMT == 1) {
+    // only the Q/K/V projection multiplies its input's rests (GemvParams::xsplit)
+    gemv_consume_int4<B, EPI == EPI_QKV>(p.n_kt, smem, full, empty, S, s, phase, t0, n, sr, segc, &s_abort, p.err,
+                                         tid);
+  } else {
+    gemv_consume<B, FMT>(p.n_kt, smem, full, empty, S, s, phase, t0, n, sr, segc, &s_abort, p.err, tid, false);
+  }
 
   consumer_sync();
   if (tid == 0) stamp(TR_CONS_ENTER);
@@ -159,8 +165,8 @@ __global__ void __launch_bounds__(GEMV_THREADS, 2) gemv_kernel(const __grid_cons
 
 // ---------------------------------------------------------------------------- launch
 static size_t gemv_smem_bytes(int stages, int batch, int fmt, int cluster = 1) {
-  return (size_t)stages * stage_bytes(batch, fmt) + (2 * stages + 2 * NSLOT) * sizeof(uint64_t) +
-         128 + (NSLOT + (cluster > 1 ? cluster - 1 : 0)) * RB * MAXB * sizeof(float);
+  return (size_t)stages * stage_bytes(batch, fmt) + (2 * stages + 2 * NSLOT) * sizeof(uint64_t) + 128 +
+         (seg_floats(fmt) + (cluster > 1 ? cluster - 1 : 0) * RB * MAXB) * sizeof(float);
 }
 
 static int g_smem_optin = 0, g_smem_per_sm = 0, g_n_sm = 0;
@@ -238,13 +244,13 @@ int gemv_stages_for(int batch, int fmt, int cluster, int per_sm) {
     return cta <= (size_t)g_smem_optin && (size_t)per_sm * (cta + 1024) <= (size_t)g_smem_per_sm;
   };
   while (s > 2 && !fits(s)) --s;
-  return s;
+  return ring_depth(fmt, s);
 }
 
 int gemv_max_stages(int batch, int fmt, int smem_optin) {
   int s = GEMV_MAX_STAGES;
   while (s > 2 && gemv_smem_bytes(s, batch, fmt) + GEMV_STATIC_SMEM > (size_t)smem_optin) --s;
-  return s;
+  return ring_depth(fmt, s);
 }
 
 template <int B, int EPI, int FMT>
@@ -289,11 +295,14 @@ cudaError_t prepare_gemv() {
 
 cudaError_t launch_gemv(const GemvParams &p, int epi, int grid, cudaStream_t s, bool pdl) {
   if (p.stages < 2 || p.stages > gemv_max_stages(p.batch, p.fmt, g_smem_optin)) return cudaErrorInvalidValue;
+  if (p.stages != ring_depth(p.fmt, p.stages)) return cudaErrorInvalidValue;  // int4: an even ring
   // clusters: each CTA exactly 1/cluster of the K range of one row block
   if (p.cluster > 1 && (p.cluster > MAX_CLUSTER || grid != p.cluster * p.n_rb || p.n_kt < p.cluster))
     return cudaErrorInvalidValue;
   if (gemv_smem_bytes(p.stages, p.batch, p.fmt, p.cluster) + GEMV_STATIC_SMEM > (size_t)g_smem_optin)
     return cudaErrorInvalidValue;
+  // the int4 consumers take the rests exactly when the Q/K/V projection runs (a template choice)
+  if (p.fmt == 1 && (p.xsplit != 0) != (epi == EPI_QKV)) return cudaErrorInvalidValue;
   return p.fmt == 0 ? launch_f<0>(p, epi, grid, s, pdl) : launch_f<1>(p, epi, grid, s, pdl);
 }
 

@@ -59,8 +59,11 @@ __device__ __forceinline__ int cta_of_tile(long long t, long long T, int G) {
 }
 
 // Bounded wait on an mbarrier phase that also ends when the CTA aborts.
+// The first poll comes before the abort flag is read: in a running ring the phase is usually
+// complete already, and then the wait costs one poll.
 __device__ __forceinline__ bool consumer_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag,
                                               unsigned *err) {
+  if (mbar_try_wait(bar, parity)) return true;
   if (*abort_flag) return false;
   for (uint32_t i = 0; i < WAIT_LIMIT; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -173,66 +176,169 @@ __device__ __forceinline__ void mma_f16_16816_seed(float (&d)[4], uint32_t a0, u
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(c.x), "f"(c.y), "f"(c.z), "f"(c.w));
 }
 
-// int4 tile (FMT 1) on the tensor cores.  Warp w takes row group r16 = w % 4 (16 rows) and K half
-// h = w / 4 (128 of the tile's 256 K): per K step of 16, one m16n8k16 MMA (fp16, fp32
-// accumulate) of the decoded codes against eight columns of activations; one 16-byte
-// shared-memory load per lane gives the B fragments of both K steps of a 32-element chunk (Act16
-// order).  Column j is source row j % B (the users' rounded parts); with XSPLIT, columns 4..7
-// are the rests (source rows MAXB + (j - 4) % B).  Columns past the users carry copies and are
-// dropped at the end.  A chunk's first MMA seeds the accumulator with minus the columns' offset
-// sums (stored as the accumulator quad), so that after its two MMAs it holds the product of the
-// codes with the scaled activations; the two chunks of a weight group are multiplied back by
-// their multipliers and summed (packed fp32x2), then scaled by the rows' group scale into acc.
-// acc[0..1]: row r16*16 + gid, columns 2 tig, 2 tig + 1; acc[2..3]: row + 8.
+// int4 tile (FMT 1) on the tensor cores.  The consumer warps form two teams of four: team
+// w / 4 takes every other tile of the CTA's range, and warp w takes weight group g4 = w % 4 (64
+// of the tile's 256 K) of all four row groups (64 rows).  Per K step of 16, one m16n8k16 MMA
+// (fp16, fp32 accumulate) of the decoded codes against eight columns of activations; so every
+// B fragment, seed and multiplier a warp loads from shared memory serves four MMAs, one per row
+// group (a warp per row group would load them four times over, and shared-memory wavefronts,
+// not instructions, would bound the kernel).  Column j is source row j % B (the users' rounded
+// parts); with XSPLIT, columns 4..7 are the rests (source rows MAXB + (j - 4) % B).  Columns past
+// the users carry copies and are dropped at the end.  A chunk's first MMA seeds the accumulator
+// with minus the columns' offset sums, so that after its two MMAs it holds the product of the
+// codes with the scaled activations; the group's two chunks are multiplied back by their
+// multipliers and summed (packed fp32x2), then scaled by the rows' group scale into acc.
+// acc[r16][0..1]: row r16*16 + gid, columns 2 tig, 2 tig + 1; acc[r16][2..3]: row + 8.
+
+// Byte offsets, within a ring stage, of one consumer lane's operands (fixed for the whole GEMV).
+struct Int4Lane {
+  uint32_t cw;  // code words of row group 0 (uint4: the group's four K steps); row group r16 at + 1024 r16
+  uint32_t sc;  // scales of rows gid and gid + 8 of the four row groups (tile4_scale_index), 16 bytes
+  uint32_t xb;  // B fragments of the group's first chunk (its second at + 64)
+  uint32_t xc;  // the group's constants: seed a, seed b (+ 64), multipliers (+ 128)
+};
+
 template <int B, bool XSPLIT>
-__device__ __forceinline__ void tile_compute_int4(const uint8_t *st, int warp, int lane, float (&acc)[4]) {
-  const int r16 = warp & 3, h = warp >> 2, gid = lane >> 2, tig = lane & 3;
-  const uint4 *cw = reinterpret_cast<const uint4 *>(st) + (h * 4 + r16) * 2 * 32 + lane;
-  const uint4 wq[2] = {cw[0], cw[32]};
-  const uint32_t *sp = reinterpret_cast<const uint32_t *>(st + TILE4_CODE_BYTES);
-  const uint32_t s0 = sp[(r16 * 16 + gid) * 2 + h], s1 = sp[(r16 * 16 + gid + 8) * 2 + h];
+__device__ __forceinline__ Int4Lane int4_lane(int warp, int lane) {
+  const int g4 = warp & 3, h = g4 >> 1, q = g4 & 1, gid = lane >> 2, tig = lane & 3;
   const int src = XSPLIT ? (gid < 4 ? gid % B : MAXB + (gid - 4) % B) : gid % B;
-  const uint4 *xb =
-      reinterpret_cast<const uint4 *>(st + TILE4_BYTES + XC_TILE_BYTES + src * X16_SRC_STRIDE + h * 256) + tig;
-  const float4 *xc = reinterpret_cast<const float4 *>(st + TILE4_BYTES) + tig * 2;
+  Int4Lane L;
+  L.cw = static_cast<uint32_t>(((h * 8 + q) * 32 + lane) * 16);
+  L.sc = static_cast<uint32_t>(TILE4_CODE_BYTES + 2 * tile4_scale_index(gid, g4));
+  L.xb = static_cast<uint32_t>(TILE4_BYTES + XC_TILE_BYTES + src * X16_SRC_STRIDE + g4 * 128 + tig * 16);
+  L.xc = static_cast<uint32_t>(TILE4_BYTES + g4 * XC_GROUP_BYTES + tig * 16);
+  return L;
+}
+
+template <int B, bool XSPLIT>
+__device__ __forceinline__ void tile_compute_int4(const uint8_t *st, const Int4Lane &L, float (&acc)[4][4]) {
+  uint4 w[4];
 #pragma unroll
-  for (int q = 0; q < 2; ++q) {
-    float2 g0, g1;  // rows gid, gid + 8: the group's two chunks, each times its multipliers
+  for (int r16 = 0; r16 < 4; ++r16) w[r16] = *reinterpret_cast<const uint4 *>(st + L.cw + r16 * 1024);
+  const uint4 sc = *reinterpret_cast<const uint4 *>(st + L.sc);  // row groups 0..3: (row gid, row gid + 8)
+  const uint4 ba = *reinterpret_cast<const uint4 *>(st + L.xb);
+  const uint4 bb = *reinterpret_cast<const uint4 *>(st + L.xb + 64);
+  const float4 seed_a = *reinterpret_cast<const float4 *>(st + L.xc);
+  const float4 seed_b = *reinterpret_cast<const float4 *>(st + L.xc + 64);
+  const float4 mq = *reinterpret_cast<const float4 *>(st + L.xc + 128);  // (m_a, m_b) of the two columns
+  const float2 ma = make_float2(mq.x, mq.y), mb = make_float2(mq.z, mq.w);
 #pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      const int ch = h * 4 + 2 * q + half;  // chunk of the tile
-      const float4 seed = xc[ch * 8];
-      const float4 mm = xc[ch * 8 + 1];
-      const uint4 bb = xb[(2 * q + half) * 4];
-      uint32_t a0, a1, a2, a3;
-      float c[4];
-      int4_frag_f16(half ? wq[q].z : wq[q].x, a0, a1, a2, a3);
-      mma_f16_16816_seed(c, a0, a1, a2, a3, bb.x, bb.y, seed);
-      int4_frag_f16(half ? wq[q].w : wq[q].y, a0, a1, a2, a3);
-      mma_f16_16816(c, a0, a1, a2, a3, bb.z, bb.w);
-      const float2 m2 = make_float2(mm.x, mm.y);
-      if (half == 0) {
-        g0 = __fmul2_rn(m2, make_float2(c[0], c[1]));
-        g1 = __fmul2_rn(m2, make_float2(c[2], c[3]));
-      } else {
-        g0 = __ffma2_rn(m2, make_float2(c[0], c[1]), g0);
-        g1 = __ffma2_rn(m2, make_float2(c[2], c[3]), g1);
-      }
-    }
-    const float sc0 = q ? bf16_hi(s0) : bf16_lo(s0), sc1 = q ? bf16_hi(s1) : bf16_lo(s1);
-    acc[0] = fmaf(sc0, g0.x, acc[0]);
-    acc[1] = fmaf(sc0, g0.y, acc[1]);
-    acc[2] = fmaf(sc1, g1.x, acc[2]);
-    acc[3] = fmaf(sc1, g1.y, acc[3]);
+  for (int r16 = 0; r16 < 4; ++r16) {
+    uint32_t a0, a1, a2, a3;
+    float ca[4], cb[4];
+    int4_frag_f16(w[r16].x, a0, a1, a2, a3);
+    mma_f16_16816_seed(ca, a0, a1, a2, a3, ba.x, ba.y, seed_a);
+    int4_frag_f16(w[r16].z, a0, a1, a2, a3);
+    mma_f16_16816_seed(cb, a0, a1, a2, a3, bb.x, bb.y, seed_b);
+    int4_frag_f16(w[r16].y, a0, a1, a2, a3);
+    mma_f16_16816(ca, a0, a1, a2, a3, ba.z, ba.w);
+    int4_frag_f16(w[r16].w, a0, a1, a2, a3);
+    mma_f16_16816(cb, a0, a1, a2, a3, bb.z, bb.w);
+    float2 g0 = __fmul2_rn(ma, make_float2(ca[0], ca[1]));
+    float2 g1 = __fmul2_rn(ma, make_float2(ca[2], ca[3]));
+    g0 = __ffma2_rn(mb, make_float2(cb[0], cb[1]), g0);
+    g1 = __ffma2_rn(mb, make_float2(cb[2], cb[3]), g1);
+    const uint32_t sw = r16 == 0 ? sc.x : r16 == 1 ? sc.y : r16 == 2 ? sc.z : sc.w;
+    const float sc0 = bf16_lo(sw), sc1 = bf16_hi(sw);
+    acc[r16][0] = fmaf(sc0, g0.x, acc[r16][0]);
+    acc[r16][1] = fmaf(sc0, g0.y, acc[r16][1]);
+    acc[r16][2] = fmaf(sc1, g1.x, acc[r16][2]);
+    acc[r16][3] = fmaf(sc1, g1.y, acc[r16][3]);
   }
 }
 
-// Staging ring between the consumer warps and the epilogue warp.
+// Staging ring between the consumer warps and the epilogue warp: nslot slots of nsub sub-slots
+// of [RB][MAXB] sums.  bf16 tiles: 4 slots of one sub-slot, each value written by one lane.  int4
+// tiles: 2 slots of 4 sub-slots, sub-slot g4 receiving exactly two additions (one per team) onto
+// zero, so that the order does not change the sum; the epilogue warp adds the sub-slots in order.
 struct SegRing {
-  float *red;      // [NSLOT][RB][MAXB]
-  uint64_t *full;  // [NSLOT], count CONSUMER_WARPS
-  uint64_t *empty; // [NSLOT], count 1
+  float *red;      // [nslot][nsub][RB][MAXB]
+  uint64_t *full;  // [nslot], count CONSUMER_WARPS
+  uint64_t *empty; // [nslot], count 1
+  int nslot, nsub;
 };
+__host__ __device__ constexpr int seg_slots(int fmt) { return fmt == 0 ? NSLOT : 2; }
+__host__ __device__ constexpr int seg_subs(int fmt) { return fmt == 0 ? 1 : 4; }
+__host__ __device__ constexpr int seg_floats(int fmt) { return seg_slots(fmt) * seg_subs(fmt) * RB * MAXB; }
+
+// Arrivals that release a weight-ring stage: one per consumer warp (bf16 tiles, lane 0 after a
+// __syncwarp) or one per thread of the team that consumed it (int4 tiles: no warp barrier in the
+// tile loop).
+__host__ __device__ constexpr int ring_empty_count(int fmt) { return fmt == 0 ? CONSUMER_WARPS : CONSUMER_THREADS / 2; }
+
+// int4 consumer side of one GEMV over this CTA's tile range [t0, t0 + n).  The ring depth S is
+// even and ring stage r belongs to team r % 2: tile i of the range, in stage (s + i) % S, is
+// team (s + i) % 2's.  (Were a stage used by both teams in turn, a warp could come back to it for
+// the use after next while the other team's use is still landing, and a parity wait cannot tell
+// those two phases apart.)  Per segment (the tiles of one row block) a warp waits for each of its
+// team's tiles, computes its weight group of it and releases it with every lane, then adds the
+// segment's sums into its sub-slot of the next staging slot.  (s, phase), the ring position of
+// the range's first tile, comes back advanced by n, as the persistent kernel carries it across
+// GEMVs that share the ring.
+template <int B, bool XSPLIT>
+__device__ __forceinline__ void gemv_consume_int4(int n_kt, uint8_t *ring, uint64_t *full, uint64_t *empty, int S,
+                                                  int &s, uint32_t &phase, long long t0, int n, const SegRing &sr,
+                                                  int &segc, volatile int *abort_flag, unsigned *err, int tid) {
+  constexpr uint32_t SB = stage_bytes(B, 1);
+  const int warp = tid >> 5, lane = tid & 31, team = warp >> 2;
+  const Int4Lane L = int4_lane<B, XSPLIT>(warp, lane);
+  const uint32_t full0 = smem_addr(full), empty0 = smem_addr(empty);
+  // this team's ring position: its first tile of the range, (team ^ s) & 1
+  const int par = (team ^ s) & 1;  // tile i is this team's when (i & 1) == par
+  int ms = s + par;
+  uint32_t mph = phase;
+  if (ms >= S) {
+    ms -= S;
+    mph ^= 1u;
+  }
+  int kt = static_cast<int>(t0 % n_kt);
+  int i = 0;
+  while (i < n) {
+    const int seg = min(n_kt - kt, n - i);
+    float acc[4][4] = {};
+    for (int j = (par ^ i) & 1; j < seg; j += 2) {
+      consumer_wait(full0 + 8u * ms, mph, abort_flag, err);
+      tile_compute_int4<B, XSPLIT>(ring + (size_t)ms * SB, L, acc);
+      mbar_arrive(empty0 + 8u * ms);
+      ms += 2;
+      if (ms >= S) {
+        ms -= S;
+        mph ^= 1u;
+      }
+    }
+    i += seg;
+    kt = 0;
+    const int slot = segc % sr.nslot, use = segc / sr.nslot;
+    float *rd = sr.red + (slot * sr.nsub + (warp & 3)) * RB * MAXB;
+    if (XSPLIT) {
+      // rounded part (columns 0-3, lanes tig < 2) + rest (columns 4-7, lanes tig + 2)
+#pragma unroll
+      for (int r16 = 0; r16 < 4; ++r16)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) acc[r16][v] += __shfl_down_sync(0xffffffffu, acc[r16][v], 2);
+    }
+    if (use > 0) consumer_wait(smem_addr(&sr.empty[slot]), (use - 1) & 1, abort_flag, err);
+    const int gid = lane >> 2, tig = lane & 3;
+#pragma unroll
+    for (int r16 = 0; r16 < 4; ++r16) {
+      const int r0 = r16 * 16 + gid;
+      if (2 * tig < B) {
+        atomicAdd(rd + r0 * MAXB + 2 * tig, acc[r16][0]);
+        atomicAdd(rd + (r0 + 8) * MAXB + 2 * tig, acc[r16][2]);
+      }
+      if (2 * tig + 1 < B) {
+        atomicAdd(rd + r0 * MAXB + 2 * tig + 1, acc[r16][1]);
+        atomicAdd(rd + (r0 + 8) * MAXB + 2 * tig + 1, acc[r16][3]);
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_addr(&sr.full[slot]));
+    ++segc;
+  }
+  const int adv = s + n;
+  s = adv % S;
+  phase ^= static_cast<uint32_t>((adv / S) & 1);
+}
 
 // Consumer side of one GEMV over this CTA's tile range [t0, t0 + n): wait for each tile's ring
 // stage, accumulate, release the stage; at each segment end reduce the rows of this warp into the
@@ -242,70 +348,29 @@ template <int B, int FMT>
 __device__ __forceinline__ void gemv_consume(int n_kt, uint8_t *ring, uint64_t *full, uint64_t *empty, int S, int &s,
                                              uint32_t &phase, long long t0, int n, const SegRing &sr, int &segc,
                                              volatile int *abort_flag, unsigned *err, int tid, bool xsplit) {
-  const int warp = tid >> 5, lane = tid & 31, kc = lane & 15, rsub = lane >> 4;
-  float acc[B][4][2];   // bf16 tiles: rows warp*8 + rsub + 2j, this lane's K chunk
-  float acc4[4];        // int4 tiles (tensor cores): see tile_compute_int4
-  int kt = static_cast<int>(t0 % n_kt);
-  for (int i = 0; i < n; ++i) {
-    if (i == 0 || kt == 0) {
-      if constexpr (FMT == 0) {
+  if constexpr (FMT == 1) {
+    if (xsplit)
+      gemv_consume_int4<B, true>(n_kt, ring, full, empty, S, s, phase, t0, n, sr, segc, abort_flag, err, tid);
+    else
+      gemv_consume_int4<B, false>(n_kt, ring, full, empty, S, s, phase, t0, n, sr, segc, abort_flag, err, tid);
+  } else {
+    const int warp = tid >> 5, lane = tid & 31, kc = lane & 15, rsub = lane >> 4;
+    float acc[B][4][2];  // rows warp*8 + rsub + 2j, this lane's K chunk
+    int kt = static_cast<int>(t0 % n_kt);
+    for (int i = 0; i < n; ++i) {
+      if (i == 0 || kt == 0) {
 #pragma unroll
         for (int b = 0; b < B; ++b)
 #pragma unroll
           for (int j = 0; j < 4; ++j) acc[b][j][0] = acc[b][j][1] = 0.f;
-      } else {
-        acc4[0] = acc4[1] = acc4[2] = acc4[3] = 0.f;
       }
-    }
-    bool single = true;
-    if constexpr (FMT == 1) {
-      if (i + 1 < n && kt + 1 < n_kt) {
-        // two tiles of one row block: both stages awaited, then both computed without a barrier
-        // between them (their decoding and MMAs interleave), then both released
-        single = false;
-        int s1 = s + 1;
-        uint32_t ph1 = phase;
-        if (s1 == S) {
-          s1 = 0;
-          ph1 ^= 1u;
-        }
-        consumer_wait(smem_addr(&full[s]), phase, abort_flag, err);
-        consumer_wait(smem_addr(&full[s1]), ph1, abort_flag, err);
-        const uint8_t *st0 = ring + (size_t)s * stage_bytes(B, FMT), *st1 = ring + (size_t)s1 * stage_bytes(B, FMT);
-        if (xsplit) {
-          tile_compute_int4<B, true>(st0, warp, lane, acc4);
-          tile_compute_int4<B, true>(st1, warp, lane, acc4);
-        } else {
-          tile_compute_int4<B, false>(st0, warp, lane, acc4);
-          tile_compute_int4<B, false>(st1, warp, lane, acc4);
-        }
-        __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(smem_addr(&empty[s]));
-          mbar_arrive(smem_addr(&empty[s1]));
-        }
-        // continue at the second tile: the segment check and the advance below are its
-        ++i;
-        ++kt;
-        s = s1;
-        phase = ph1;
-      }
-    }
-    if (single) {
       consumer_wait(smem_addr(&full[s]), phase, abort_flag, err);
-      if constexpr (FMT == 0)
-        tile_compute<B, FMT>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc);
-      else if (xsplit)
-        tile_compute_int4<B, true>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc4);
-      else
-        tile_compute_int4<B, false>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc4);
+      tile_compute<B, FMT>(ring + (size_t)s * stage_bytes(B, FMT), warp, lane, acc);
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_addr(&empty[s]));
-    }
-    if (kt == n_kt - 1 || i == n - 1) {
-      const int slot = segc % NSLOT, use = segc / NSLOT;
-      float *rd = sr.red + slot * RB * MAXB;
-      if constexpr (FMT == 0) {
+      if (kt == n_kt - 1 || i == n - 1) {
+        const int slot = segc % sr.nslot, use = segc / sr.nslot;
+        float *rd = sr.red + slot * RB * MAXB;
         float tot[B][4];
 #pragma unroll
         for (int b = 0; b < B; ++b)
@@ -325,36 +390,19 @@ __device__ __forceinline__ void gemv_consume(int n_kt, uint8_t *ring, uint64_t *
 #pragma unroll
             for (int b = 0; b < B; ++b) rd[(warp * 8 + rsub + 2 * j) * MAXB + b] = tot[b][j];
         }
-      } else {
-        // the two K halves of a row group add into the slot, which the epilogue warp left at
-        // zero: two additions per value, so the order does not change the sum
-        if (xsplit) {
-          // rounded part (columns 0-3, lanes tig < 2) + rest (columns 4-7, lanes tig + 2)
-#pragma unroll
-          for (int v = 0; v < 4; ++v) acc4[v] += __shfl_down_sync(0xffffffffu, acc4[v], 2);
-        }
-        if (use > 0) consumer_wait(smem_addr(&sr.empty[slot]), (use - 1) & 1, abort_flag, err);
-        const int gid = lane >> 2, tig = lane & 3, r0 = (warp & 3) * 16 + gid;
-        if (2 * tig < B) {
-          atomicAdd(rd + r0 * MAXB + 2 * tig, acc4[0]);
-          atomicAdd(rd + (r0 + 8) * MAXB + 2 * tig, acc4[2]);
-        }
-        if (2 * tig + 1 < B) {
-          atomicAdd(rd + r0 * MAXB + 2 * tig + 1, acc4[1]);
-          atomicAdd(rd + (r0 + 8) * MAXB + 2 * tig + 1, acc4[3]);
-        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_addr(&sr.full[slot]));
+        ++segc;
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_addr(&sr.full[slot]));
-      ++segc;
-    }
-    if (++kt == n_kt) kt = 0;
-    if (++s == S) {
-      s = 0;
-      phase ^= 1u;
+      if (++kt == n_kt) kt = 0;
+      if (++s == S) {
+        s = 0;
+        phase ^= 1u;
+      }
     }
   }
 }
+
 
 // ---------------------------------------------------------------------------- epilogue warp
 // RMSNorm scale of the GEMV input (1 without a norm): user b's scale from the per-row-block sums
@@ -586,7 +634,7 @@ __device__ __forceinline__ void gemv_epilogues(const GemvParams &p, long long t0
     const int kt0 = static_cast<int>(t - (long long)rb * p.n_kt);
     const int len = min(p.n_kt - kt0, n - i);
     i += len;
-    const int slot = segc % NSLOT, use = segc / NSLOT;
+    const int slot = segc % sr.nslot, use = segc / sr.nslot;
     ++segc;
     consumer_wait(smem_addr(&sr.full[slot]), use & 1, abort_flag, p.err);
     unsigned long long *tr = p.trace && lane == 0 ? p.trace + (size_t)c * TRACE_SLOTS : nullptr;
@@ -594,7 +642,21 @@ __device__ __forceinline__ void gemv_epilogues(const GemvParams &p, long long t0
       tr[TR_E_SEG] = global_ns();
       tr[TR_E_KIND] = 0;
     }
-    float *red = sr.red + slot * RB * MAXB;
+    float *red = sr.red + slot * sr.nsub * RB * MAXB;
+    if (sr.nsub > 1) {
+      // int4 tiles: the sub-slots' sums in sub-slot order into the first, the others back to zero
+      float4 *r4 = reinterpret_cast<float4 *>(red);
+      for (int e = lane; e < RB * MAXB / 4; e += 32) {
+        float4 a = r4[e];
+        for (int j = 1; j < sr.nsub; ++j) {
+          const float4 v = r4[j * (RB * MAXB / 4) + e];
+          a = make_float4(a.x + v.x, a.y + v.y, a.z + v.z, a.w + v.w);
+          r4[j * (RB * MAXB / 4) + e] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        r4[e] = a;
+      }
+      __syncwarp();
+    }
     EpiPre pre;
     epilogue_prefetch<B, EPI>(p, rb, lane, pre);
     bool do_epi = true;

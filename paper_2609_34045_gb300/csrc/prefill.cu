@@ -851,7 +851,7 @@ __global__ void dequant_int4_f16_kernel(const uint8_t *tiles4, int n_rb, int n_k
     const int q = m >> 2, j = m & 3, r16 = r >> 4, gid = r & 7, rhalf = (r >> 3) & 1;
     const uint8_t *tile = tiles4 + (size_t)t * TILE4_BYTES;
     const uint32_t *words = reinterpret_cast<const uint32_t *>(tile);
-    const float sc = bf16_to_f32(reinterpret_cast<const uint16_t *>(tile + TILE4_CODE_BYTES)[r * (KT4 / 64) + (col0 >> 6)]);
+    const float sc = bf16_to_f32(reinterpret_cast<const uint16_t *>(tile + TILE4_CODE_BYTES)[tile4_scale_index(r, col0 >> 6)]);
     uint16_t out[8];
 #pragma unroll
     for (int tig = 0; tig < 4; ++tig) {

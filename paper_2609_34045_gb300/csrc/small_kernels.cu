@@ -226,14 +226,15 @@ cudaError_t launch_repack_bf16(const uint16_t *src, int n_src_rows, int k, const
 }
 
 // Repack an int4 group-64 matrix (words [n_src_rows][k/8], scales [n_src_rows][k/64]) into
-// tiles [n_rb][n_kt][RB][KT4/8 words] followed by [RB][KT4/64] bf16 scales per tile.
+// tiles [n_rb][n_kt][RB][KT4/8 words] followed by RB x KT4/64 bf16 scales per tile.
 // int4 tiles in the order of the tensor-core MMA fragments (tile_compute, FMT 1): the 64 x 256
 // codes of a tile are 2048 words; word ((((h * 4 + r16) * 2 + q) * 32 + lane) * 4 + j) holds the
 // eight codes lane needs for K step s = 4 q + j of K half h and row group r16 (rows r16 * 16 +
 // gid and + 8, gid = lane / 4; columns 2 tig, 2 tig + 1, 2 tig + 8, 2 tig + 9 of the step, tig =
 // lane % 4), nibble i at bits 4 i: row + 8 ((i >> 1) & 1), column + 8 (i & 1) + ((i >> 2) & 1),
 // so that the nibble pairs at bits (0, 16), (8, 24), (4, 20), (12, 28) are the A registers a0,
-// a1, a2, a3 (int4_frag_f16).  Scales stay [64 rows][4 groups of 64].
+// a1, a2, a3 (int4_frag_f16).  The 64 x 4 scales are stored in the order of tile4_scale_index
+// (a lane's rows gid and gid + 8, both groups of its K half, in 8 consecutive bytes).
 __global__ void repack_int4_kernel(const uint32_t *words, const uint16_t *scales, int n_src_rows, int k,
                                    const int *row_map, int n_rows_out, int n_rb, int n_kt, uint8_t *dst) {
   constexpr int TW = TILE4_CODE_BYTES / 4;  // words per tile
@@ -267,10 +268,10 @@ __global__ void repack_int4_kernel(const uint32_t *words, const uint16_t *scales
       int srow = -1;
       if (orow < n_rows_out) srow = row_map ? row_map[orow] : orow;
       if (srow >= n_src_rows) srow = -1;
-      uint16_t *sd = reinterpret_cast<uint16_t *>(tile + TILE4_CODE_BYTES) + idx * SPR;
+      uint16_t *sd = reinterpret_cast<uint16_t *>(tile + TILE4_CODE_BYTES);
       for (int g = 0; g < SPR; ++g) {
         const int gg = kt * SPR + g;
-        sd[g] = (srow >= 0 && gg < ks) ? scales[(size_t)srow * ks + gg] : uint16_t(0);
+        sd[tile4_scale_index(idx, g)] = (srow >= 0 && gg < ks) ? scales[(size_t)srow * ks + gg] : uint16_t(0);
       }
     }
   }

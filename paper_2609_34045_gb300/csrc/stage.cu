@@ -121,13 +121,14 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   p->n_sm = n_sm;
   // Two CTAs per SM: a single CTA's consumer warps (8) leave the tile loop bound by instruction
   // latency (int4 decoding; bf16 at batch 4), two give every SM twice the warps to hide it.  The
-  // rings are sized so that two fit an SM at every batch size: 5 bf16 stages (at most 90 KiB),
-  // 7 int4 stages (at most 93 KiB); that is about 80 KiB of weights in flight per SM.
+  // rings are sized so that two fit an SM at every batch size: 5 bf16 stages (at most 90 KiB);
+  // int4 rings take the deepest even depth up to 8 that fits (8 at batch 1, 6 at batch 4, with
+  // its staging slots): 70-100 KiB of weights in flight per SM.
   const bool i4 = f == KFL_INT4_G64;
   p->ctas_per_sm = env_int("KFL_GEMV_CTAS_PER_SM", 2);
   if (p->ctas_per_sm < 1 || p->ctas_per_sm > 2) p->ctas_per_sm = 2;
-  p->stages = env_int("KFL_GEMV_STAGES", i4 ? 7 : 5);
-  if (p->stages < 2 || p->stages > 13) p->stages = i4 ? 7 : 5;
+  p->stages = env_int("KFL_GEMV_STAGES", i4 ? 8 : 5);
+  if (p->stages < 2 || p->stages > 13) p->stages = i4 ? 8 : 5;
   p->gemv_grid_max = n_sm * p->ctas_per_sm;
   // bf16 GEMVs of 2 x SMs to 4096 tiles (the 7B Q/K/V and O: 28 tiles per row block) run one
   // CTA per SM with 6 stages: half the CTAs share each row block, so their combine ends sooner
@@ -318,7 +319,7 @@ GemvParams base_gemv(kfl_stage *st, const Mat &m, const float *x, int ldx, int b
   g.x = x;
   g.ldx = ldx;
   g.batch = batch;
-  g.stages = std::min(st->P.stages, gemv_stages_for(batch, m.fmt, 1, st->P.ctas_per_sm));
+  g.stages = ring_depth(m.fmt, std::min(st->P.stages, gemv_stages_for(batch, m.fmt, 1, st->P.ctas_per_sm)));
   g.rope_per_user = 0;
   g.partial = st->gemv_partial;
   g.tickets = st->tickets;
@@ -583,13 +584,13 @@ int gemv_launch_shape(const kfl_stage *st, int batch, GemvParams &g) {
     // with few enough row blocks, clusters of N CTAs split each one's K range and combine
     // through distributed shared memory (N row blocks' worth of CTAs at one or two per SM)
     grid = (int)(T < st->P.n_sm ? T : st->P.n_sm);
-    g.stages = std::min(st->P.small_gemv_stages, gemv_max_stages(batch, g.fmt, st->smem_optin));
+    g.stages = ring_depth(g.fmt, std::min(st->P.small_gemv_stages, gemv_max_stages(batch, g.fmt, st->smem_optin)));
     const int N = st->P.cluster;
     if (N >= 2 && g.n_kt >= N && (long long)N * g.n_rb <= 2LL * st->P.n_sm) {
       const int per_sm = N * g.n_rb <= st->P.n_sm ? 1 : 2;
       grid = N * g.n_rb;
       g.cluster = N;
-      g.stages = std::min(st->P.small_gemv_stages, gemv_stages_for(batch, g.fmt, N, per_sm));
+      g.stages = ring_depth(g.fmt, std::min(st->P.small_gemv_stages, gemv_stages_for(batch, g.fmt, N, per_sm)));
     }
   }
   return grid;
@@ -1252,6 +1253,7 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
       if (stages > MAX_STAGES) stages = MAX_STAGES;
       while (stages > 2 && stage_kernel_smem(stages, P.hd, b, cfg->weight_fmt) + static_smem > (size_t)smem_optin)
         --stages;
+      stages = ring_depth(cfg->weight_fmt, stages);
       st->mk_stages[b] = stages;
       st->mk_smem[b] = stage_kernel_smem(stages, P.hd, b, cfg->weight_fmt);
       if (st->mk_smem[b] > smem_max) smem_max = st->mk_smem[b];

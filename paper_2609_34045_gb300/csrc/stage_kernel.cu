@@ -96,7 +96,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
   uint64_t *armed = empty + S;                        // weight tile issued (for the x producer)
   uint64_t *seg_full = armed + S;                     // staged segments (consumers -> epilogue)
   uint64_t *seg_empty = seg_full + NSLOT;
-  // [NSLOT][RB][MAXB], 128-byte aligned (read as float4)
+  // staging slots (SegRing: seg_floats(FMT) floats), 128-byte aligned (read as float4)
   float *red = reinterpret_cast<float *>((reinterpret_cast<uintptr_t>(seg_empty + NSLOT) + 127) & ~uintptr_t(127));
   __shared__ GemvParams s_egp;  // the epilogue warp's copy of the current GEMV's parameters
   __shared__ AttnParams s_ap;
@@ -111,7 +111,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
   constexpr uint32_t WBYTES = FMT == 0 ? TILE_BYTES : TILE4_BYTES;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int c = blockIdx.x, grid = gridDim.x;
-  const SegRing sr = {red, seg_full, seg_empty};
+  const SegRing sr = {red, seg_full, seg_empty, seg_slots(FMT), seg_subs(FMT)};
   auto stamp = [&](int k, int slot) {
     if (kp.trace) kp.trace[((size_t)k * grid + c) * TRACE_SLOTS + slot] = global_ns();
   };
@@ -119,7 +119,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_addr(&full[s]), 1);
-      mbar_init(smem_addr(&empty[s]), CONSUMER_WARPS);
+      mbar_init(smem_addr(&empty[s]), ring_empty_count(FMT));
       mbar_init(smem_addr(&armed[s]), 1);
     }
     for (int s = 0; s < NSLOT; ++s) {
@@ -142,7 +142,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
     }
     if (tid < MAXB) s_pos[tid] = tid < B ? kp.positions[tid] : 0;
   }
-  for (int e = tid; e < NSLOT * RB * MAXB; e += MK_THREADS) red[e] = 0.f;  // int4 tiles add into it
+  for (int e = tid; e < seg_floats(FMT); e += MK_THREADS) red[e] = 0.f;  // int4 tiles add into it
   __syncthreads();
 
   if (warp == CONSUMER_WARPS + 2) {
@@ -391,7 +391,7 @@ __global__ void __launch_bounds__(MK_THREADS, 1) stage_kernel(const __grid_const
 size_t stage_kernel_smem(int stages, int head_dim, int batch, int fmt) {
   // + 128: the staging buffer is aligned up to 128 bytes after the barriers
   return (size_t)stages * stage_bytes(batch, fmt) + stage_kernel_attn_bytes(head_dim) +
-         (3 * stages + 2 * NSLOT) * sizeof(uint64_t) + 128 + NSLOT * RB * MAXB * sizeof(float);
+         (3 * stages + 2 * NSLOT) * sizeof(uint64_t) + 128 + seg_floats(fmt) * sizeof(float);
 }
 
 int stage_kernel_attn_bytes(int head_dim) {
@@ -433,7 +433,7 @@ static cudaError_t launch_stage_one(const StageKernelParams &kp, int grid, size_
 
 cudaError_t launch_stage_kernel(const StageKernelParams &kp, int batch, int fmt, int grid, size_t smem,
                                 cudaStream_t s) {
-  if (kp.stages < 2 || kp.stages > MAX_STAGES) return cudaErrorInvalidValue;
+  if (kp.stages < 2 || kp.stages > MAX_STAGES || kp.stages != ring_depth(fmt, kp.stages)) return cudaErrorInvalidValue;
   if (fmt == 0) {
     switch (batch) {
       case 1: return launch_stage_one<1, 0>(kp, grid, smem, s);
