@@ -4,29 +4,106 @@
 // User b's token at position P_b attends to its cached slots [0, P_b] (its own K/V were appended
 // before this kernel), query head h reading KV head h / G.  The cluster's C CTAs split the
 // positions in whole 64-position sub-tiles: CTA r takes sub-tiles [r n / C, (r + 1) n / C) of the
-// n = ceil((P_b + 1) / 64).  Each keeps an online-softmax state (running max m, running sum l,
-// unnormalised weighted sum of V) per head; the C partial states then meet through distributed
-// shared memory: CTA r merges its share of the output's 32-element chunks, reading every CTA's
-// (m, l) and partial sums in CTA order (deterministic), and writes them (int4 stages: also in
-// the O projection's input form).  No global partial buffer, ticket or last-unit merge.
+// n = ceil((P_b + 1) / 64).
 //
-// Scores S = q K^T and the weighted sum P V run as bf16 m16n8k16 MMAs with fp32 accumulation.
-// q and P enter as bf16 pairs (rounded value, bf16 of the rest: about 2^-17 relative): rows
-// 0..7 of the MMA's A operand hold the heads' rounded parts and rows 8..15 their rests, so one
-// MMA yields both products and the head's value is the sum of accumulator rows g and g + 8,
-// which the same lane holds.  K and V are the cache's bf16 values, exact.  Scores: warp w takes
-// positions 8w..8w+7; P V: warp w takes head dimensions hd/8 * w onwards; softmax: warp g takes
-// head g.  Scores are in the log2 domain (q pre-scaled by log2(e)/sqrt(hd)).
+// Inside a CTA one producer warp streams the sub-tiles' K and V rows into a ring of shared-memory
+// stages with 2-D TMA copies (boxes of 64 positions x 64 dimensions, 128-byte swizzle: the
+// fragment loads of 8 consecutive rows fall in distinct banks without padding), and four consumer
+// warps each take 16 positions of every stage.  A consumer warp keeps its own online-softmax state
+// (running max m, running sum l, unnormalised weighted sum of V) per head and needs no block
+// barrier in its loop: the scores of its 16 positions (two m16n8k16 accumulator tiles) are, after
+// the softmax, exactly the A fragments of its P V product, so P never leaves the registers.
+// After the loop the four warp states merge into the CTA's (in shared memory), and the C CTA
+// states meet through distributed shared memory: CTA r merges its share of the output's
+// 32-element chunks, reading every CTA's (m, l) and partial sums in CTA order (deterministic), and
+// writes them (int4 stages: also in the O projection's input form).
+//
+// Scores S = q K^T and P V run as bf16 m16n8k16 MMAs with fp32 accumulation.  q and P enter as
+// bf16 pairs (rounded value, bf16 of the rest: about 2^-17 relative): rows 0..7 of the MMA's A
+// operand hold the heads' rounded parts and rows 8..15 their rests, so one MMA yields both
+// products and the head's value is the sum of accumulator rows g and g + 8, which the same lane
+// holds.  K and V are the cache's bf16 values, exact.  Scores are in the log2 domain (q
+// pre-scaled by log2(e)/sqrt(hd)).
+#include <cuda.h>  // CUtensorMap
+#include <cudaTypedefs.h>  // the type of cuTensorMapEncodeTiled
+
 #include "attn_core.cuh"
 
 namespace kfl {
 
+constexpr int ATC_WARPS = 4;                       // consumer warps, 16 positions of a stage each
+constexpr int ATC_THREADS = (ATC_WARPS + 1) * 32;  // + the producer warp
+constexpr int ATC_STAGES = 3;
+
 template <int HD>
-__global__ void __launch_bounds__(ATT_THREADS) attn_cluster_kernel(const __grid_constant__ AttnParams p) {
-  using L = AttnLayout<HD, 2>;
-  extern __shared__ __align__(128) uint8_t sm[];
+struct AtcLayout {
+  static constexpr int BOXES = HD / 64;                  // 64-dimension boxes of a row
+  static constexpr int BOX_BYTES = ATT_SUB * 128;        // 64 positions x 64 bf16, swizzled
+  static constexpr int KV_BYTES = BOXES * BOX_BYTES;     // the K (or V) rows of one stage
+  static constexpr int STAGE_BYTES = 2 * KV_BYTES;
+  static constexpr int QF_OFF = ATC_STAGES * STAGE_BYTES;  // q as A fragments [HD / 16][32] uint4
+  static constexpr int BAR_OFF = QF_OFF + (HD / 16) * 32 * 16;
+  static constexpr int BYTES = BAR_OFF + 2 * ATC_STAGES * 8;
+  static constexpr int SMEM = BYTES + 1024;              // + the alignment of the swizzled boxes
+  // after the loop, in the stage buffers: the warps' sums [ATC_WARPS][ATT_MAXG][HD], then the
+  // CTA's merged sums [ATT_MAXG][HD] (read by the cluster)
+  static constexpr int PART_OFF = ATC_WARPS * ATT_MAXG * HD * 4;
+  static_assert(PART_OFF + ATT_MAXG * HD * 4 <= ATC_STAGES * STAGE_BYTES, "merge scratch");
+};
+
+// Byte offset of 16-byte chunk c of row r in a box of 128-byte rows written with the 128-byte
+// swizzle (the chunk index is XORed with the row's index modulo 8).
+__device__ __forceinline__ uint32_t swz128(int r, int c) { return static_cast<uint32_t>(r * 128 + ((c ^ (r & 7)) << 4)); }
+
+__device__ __forceinline__ void atc_tma_load(uint32_t dst, const CUtensorMap *map, int c0, int c1, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3, uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr)
+               : "memory");
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3, uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr)
+               : "memory");
+}
+
+__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// (rounded, rest) bf16 pairs of two weights as the packed registers of one A-fragment row pair
+__device__ __forceinline__ void bf16_pair2(float x0, float x1, uint32_t &hi, uint32_t &lo) {
+  const uint16_t h0 = f32_to_bf16_rne(x0), h1 = f32_to_bf16_rne(x1);
+  hi = (uint32_t)h0 | ((uint32_t)h1 << 16);
+  lo = (uint32_t)f32_to_bf16_rne(x0 - bf16_to_f32(h0)) | ((uint32_t)f32_to_bf16_rne(x1 - bf16_to_f32(h1)) << 16);
+}
+
+template <int HD>
+__global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_constant__ AttnParams p,
+                                                                   const __grid_constant__ CUtensorMap kmap,
+                                                                   const __grid_constant__ CUtensorMap vmap) {
+  using L = AtcLayout<HD>;
+  extern __shared__ uint8_t sm_raw[];
+  uint8_t *sm = sm_raw + ((1024u - (smem_addr(sm_raw) & 1023u)) & 1023u);
   __shared__ float s_w[MAX_CLUSTER_ATT][ATT_MAXG];  // merge: (m, then weight) of each CTA and head
   __shared__ float s_lw[MAX_CLUSTER_ATT][ATT_MAXG];
+  __shared__ float s_wm[ATC_WARPS][ATT_MAXG];       // each consumer warp's (m, then weight) per head
+  __shared__ float s_wl[ATC_WARPS][ATT_MAXG];
+  __shared__ float s_m[ATT_MAXG], s_l[ATT_MAXG];     // this CTA's state, read by the cluster
+  __shared__ volatile int s_abort;
   pdl_launch_dependents();
   const int C = p.cluster;
   const int pair = blockIdx.x / C, r = blockIdx.x % C;  // r: the CTA's rank in its cluster
@@ -34,201 +111,232 @@ __global__ void __launch_bounds__(ATT_THREADS) attn_cluster_kernel(const __grid_
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int G = p.n_heads / p.n_kv_heads;
   const int gid = lane >> 2, tig = lane & 3;
-  const bool hrow = gid < G;
   auto stamp = [&](int slot) {
     if (p.trace && (int)blockIdx.x < p.trace_grid && tid == 0)
       p.trace[(size_t)blockIdx.x * TRACE_SLOTS + slot] = global_ns();
   };
   stamp(TR_CONS_GO);
-  uint8_t *sk = sm + L::K_OFF;
-  uint8_t *sv = sm + L::V_OFF;
-  float *ss = reinterpret_cast<float *>(sm + L::S_OFF);
-  float *s_m = reinterpret_cast<float *>(sm + L::M_OFF);
-  float *s_l = s_m + ATT_MAXG;
-  float *s_alpha = s_l + ATT_MAXG;
+  uint64_t *full = reinterpret_cast<uint64_t *>(sm + L::BAR_OFF);
+  uint64_t *empty = full + ATC_STAGES;
   uint4 *qf = reinterpret_cast<uint4 *>(sm + L::QF_OFF);
-  uint4 *pf = reinterpret_cast<uint4 *>(sm + L::PF_OFF);
+  const uint32_t sm0 = smem_addr(sm);
 
   const int P = p.positions[b];
   const bool valid = P >= 0 && P < p.max_ctx;
   int start = 0, end = 0;
   if (valid) {
-    const int nsub = (P + ATT_SUB) / ATT_SUB;
-    start = static_cast<int>((long long)r * nsub / C) * ATT_SUB;
-    end = min(P + 1, static_cast<int>((long long)(r + 1) * nsub / C) * ATT_SUB);
+    const int nsub_all = (P + ATT_SUB) / ATT_SUB;
+    start = static_cast<int>((long long)r * nsub_all / C) * ATT_SUB;
+    end = min(P + 1, static_cast<int>((long long)(r + 1) * nsub_all / C) * ATT_SUB);
   }
   const int nsub = end > start ? (end - start + ATT_SUB - 1) / ATT_SUB : 0;
-  // the cached rows [0, lo) were written by earlier steps: the first two sub-tiles' copies of
-  // them go out while the Q/K/V projection may still run; rows from lo (written by this step)
-  // after the wait
-  const int lo = valid ? attn_step_lo(p, b) : 0;
-  for (int sub = 0; sub < 2 && sub < nsub; ++sub) {
-    const int p0 = start + sub * ATT_SUB;
-    attn_load_rows<HD, 2>(p, b, kvh, p0, min(ATT_SUB, end - p0), sub, 1, lo, P, sm, tid);
+  if (tid == 0) {
+    for (int s = 0; s < ATC_STAGES; ++s) {
+      mbar_init(smem_addr(&full[s]), 1);
+      mbar_init(smem_addr(&empty[s]), ATC_WARPS * 32);
+    }
+    s_abort = 0;
+    fence_mbar_init();
   }
-  pdl_wait();
-  stamp(TR_X_GO);
-  for (int sub = 0; sub < 2 && sub < nsub; ++sub) {
-    const int p0 = start + sub * ATT_SUB;
-    attn_load_rows<HD, 2>(p, b, kvh, p0, min(ATT_SUB, end - p0), sub, 2, lo, P, sm, tid);
-  }
+  __syncthreads();
 
   constexpr int KS = HD / 16;  // K steps of the scores
-  constexpr int NT = HD / 64;  // P V n-tiles (8 dimensions) per warp: warp w owns dims NT*8*w ...
-  const int n_base = warp * NT * 8;
-  {
+  constexpr int NT = HD / 8;   // n-tiles (8 dimensions) of P V
+  if (warp == ATC_WARPS) {
+    // ------------------------------------------------------------------ producer
+    // The cached rows [0, lo) were written by earlier steps: sub-tiles below lo go out while the
+    // Q/K/V projection may still run, the rest after the wait on it.
+    if (lane == 0 && nsub > 0) {
+      const int lo = attn_step_lo(p, b);
+      const int row0 = (p.slots[b] * p.n_kv_heads + kvh) * p.max_ctx;
+      bool waited = false;
+      int issued = 0;
+      for (int t = 0; t < nsub; ++t) {
+        const int s = t % ATC_STAGES;
+        if (t >= ATC_STAGES && !mbar_wait(smem_addr(&empty[s]), ((t / ATC_STAGES) - 1) & 1)) {
+          s_abort = 1;
+          atomicOr(p.err, ERR_TIMEOUT);
+          break;
+        }
+        if (s_abort) break;
+        const int p0 = start + t * ATT_SUB;
+        if (!waited && p0 + ATT_SUB > lo) {
+          pdl_wait();
+          waited = true;
+        }
+        const uint32_t fb = smem_addr(&full[s]);
+        mbar_arrive_expect_tx(fb, L::STAGE_BYTES);
+        const uint32_t kd = sm0 + s * L::STAGE_BYTES, vd = kd + L::KV_BYTES;
+#pragma unroll
+        for (int hb = 0; hb < L::BOXES; ++hb) {
+          atc_tma_load(kd + hb * L::BOX_BYTES, &kmap, 64 * hb, row0 + p0, fb);
+          atc_tma_load(vd + hb * L::BOX_BYTES, &vmap, 64 * hb, row0 + p0, fb);
+        }
+        ++issued;
+      }
+      // copies still in flight land before the shared memory is reused (bounded)
+      for (int t = issued > ATC_STAGES ? issued - ATC_STAGES : 0; t < issued; ++t)
+        mbar_wait(smem_addr(&full[t % ATC_STAGES]), (t / ATC_STAGES) & 1);
+    }
+  } else {
+    // ------------------------------------------------------------------ consumers
+    pdl_wait();  // q and this step's K/V rows come from the Q/K/V projection
     // q (scaled to log2 units) as the scores' A fragments: entry (step, lane) = registers a0..a3:
     // rows gid (the heads' rounded parts) and gid + 8 (their rests), columns 2 tig, 2 tig + 1
     // (a0, a1) and + 8 (a2, a3); rows of heads >= G are zero
-    if (tid < KS * 32) {
-      const int st = tid >> 5, l = tid & 31, g = l >> 2, t = l & 3;
+    for (int e = tid; e < KS * 32; e += ATC_WARPS * 32) {
+      const int st = e >> 5, l = e & 31, g = l >> 2, t = l & 3;
       uint4 f = make_uint4(0u, 0u, 0u, 0u);
       if (valid && g < G) {
         const float *qg = p.q + (size_t)b * p.n_heads * HD + (size_t)(kvh * G + g) * HD + 16 * st + 2 * t;
         const float2 x0 = __ldcg(reinterpret_cast<const float2 *>(qg));
         const float2 x1 = __ldcg(reinterpret_cast<const float2 *>(qg + 8));
-        const float v[4] = {x0.x * p.scale_log2, x0.y * p.scale_log2, x1.x * p.scale_log2, x1.y * p.scale_log2};
-        uint16_t hi[4], lo_[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          hi[i] = f32_to_bf16_rne(v[i]);
-          lo_[i] = f32_to_bf16_rne(v[i] - bf16_to_f32(hi[i]));
-        }
-        f = make_uint4(hi[0] | ((uint32_t)hi[1] << 16), lo_[0] | ((uint32_t)lo_[1] << 16),
-                       hi[2] | ((uint32_t)hi[3] << 16), lo_[2] | ((uint32_t)lo_[3] << 16));
+        bf16_pair2(x0.x * p.scale_log2, x0.y * p.scale_log2, f.x, f.y);
+        bf16_pair2(x1.x * p.scale_log2, x1.y * p.scale_log2, f.z, f.w);
       }
-      qf[tid] = f;
+      qf[e] = f;
     }
-    // P fragments of rows of heads >= G stay zero
-    if (tid < (ATT_SUB / 16) * 32 && ((tid & 31) >> 2) >= G) pf[tid] = make_uint4(0u, 0u, 0u, 0u);
-  }
-  if (tid < ATT_MAXG) {
-    s_m[tid] = -INFINITY;
-    s_l[tid] = 0.f;
-  }
-  float acc[NT][4];  // rows gid (P's rounded parts) and gid + 8 (rests): both head gid's
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
+    named_bar_sync(ATT_BAR, ATC_WARPS * 32);
 
-  for (int it = 0; it < nsub; ++it) {
-    const int buf = it & 1;
-    if (it + 1 < nsub) {
-      // sub-tiles 0 and 1 were issued above; from sub-tile 2 on, each goes out one step ahead.
-      // Every copy group but the newest is then complete, this sub-tile's among them
-      if (it >= 1) {
-        const int p0 = start + (it + 1) * ATT_SUB;
-        attn_load_rows<HD, 2>(p, b, kvh, p0, min(ATT_SUB, end - p0), buf ^ 1, 0, 0, -1, sm, tid);
+    const int w0 = warp * 16;  // this warp's positions within a stage
+    float m_run = -INFINITY, l_run = 0.f;  // head gid
+    float acc[NT][4];  // rows gid (P's rounded parts) and gid + 8 (rests): both head gid's
+#pragma unroll
+    for (int d = 0; d < NT; ++d) acc[d][0] = acc[d][1] = acc[d][2] = acc[d][3] = 0.f;
+    for (int t = 0; t < nsub; ++t) {
+      const int s = t % ATC_STAGES;
+      if (s_abort) break;
+      if (!mbar_wait(smem_addr(&full[s]), (t / ATC_STAGES) & 1)) {
+        s_abort = 1;
+        atomicOr(p.err, ERR_TIMEOUT);
+        break;
       }
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
-    }
-    att_sync();
-    const int p0 = start + it * ATT_SUB;
-    const int cnt = min(ATT_SUB, end - p0);
-    const uint8_t *kb = sk + buf * ATT_SUB * L::KROW;
-    uint8_t *vb = sv + buf * ATT_SUB * L::VROW;
-    // rows past the sub-tile's positions take part in P V with weight 0: make them finite
-    if (cnt < ATT_SUB)
-      for (int e = tid; e < (ATT_SUB - cnt) * (HD / 8); e += ATT_THREADS)
-        *reinterpret_cast<uint4 *>(vb + (cnt + e / (HD / 8)) * L::VROW + (e % (HD / 8)) * 16) = make_uint4(0u, 0u, 0u, 0u);
-    {
-      // scores of positions 8w .. 8w + 7 (MMA columns) for every head: one MMA per K step (two
-      // accumulator chains by K-step parity); head gid's score = rows gid + gid + 8
-      float sp[2][4] = {};
-      const uint8_t *krow = kb + (8 * warp + gid) * L::KROW + 4 * tig;
+      const int nv = min(ATT_SUB, end - (start + t * ATT_SUB)) - w0;  // valid positions of this warp
+      const uint32_t kb = sm0 + s * L::STAGE_BYTES, vb = kb + L::KV_BYTES;
+      if (nv > 0) {
+        if (nv < 16) {
+          // rows past the last position take part in P V with weight 0: make them finite
+          uint8_t *vg = sm + s * L::STAGE_BYTES + L::KV_BYTES;
+          for (int e = lane; e < (16 - nv) * 8 * L::BOXES; e += 32) {
+            const int row = w0 + nv + e / (8 * L::BOXES), rest = e % (8 * L::BOXES);
+            *reinterpret_cast<uint4 *>(vg + (rest >> 3) * L::BOX_BYTES + row * 128 + (rest & 7) * 16) =
+                make_uint4(0u, 0u, 0u, 0u);
+          }
+          // these stores come before the stage's next TMA write (another proxy) in every order
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          __syncwarp();
+        }
+        // scores of positions w0 + 8 j + (2 tig, 2 tig + 1), n-tile j = 0, 1, for head gid: two
+        // accumulator chains per n-tile (K-step parity)
+        float sc[2][2][4] = {};
+        const int mi = lane >> 3, rr = lane & 7;
 #pragma unroll
-      for (int s16 = 0; s16 < KS; ++s16) {
-        const uint4 f = qf[s16 * 32 + lane];
-        const uint32_t k0 = *reinterpret_cast<const uint32_t *>(krow + 32 * s16);
-        const uint32_t k1 = *reinterpret_cast<const uint32_t *>(krow + 32 * s16 + 16);
-        mma_bf16_full(sp[s16 & 1], f, k0, k1);
-      }
-      if (hrow) {
-        const float s0 = (sp[0][0] + sp[1][0]) + (sp[0][2] + sp[1][2]);
-        const float s1 = (sp[0][1] + sp[1][1]) + (sp[0][3] + sp[1][3]);
-        const int pp = 8 * warp + 2 * tig;
-        *reinterpret_cast<float2 *>(ss + gid * L::SS + pp) =
-            make_float2(pp < cnt ? s0 : -INFINITY, pp + 1 < cnt ? s1 : -INFINITY);
-      }
-    }
-    att_sync();
-    // online softmax update: warp g owns head g; its weights go to the P fragments as bf16
-    // pairs (rounded part in rows g, rest in rows g + 8)
-    if (warp < G) {
-      const int g = warp;
-      const float a0 = ss[g * L::SS + lane], a1 = ss[g * L::SS + lane + 32];
-      float mx = fmaxf(a0, a1);
+        for (int k2 = 0; k2 < KS / 2; ++k2) {
+          const uint4 qa = qf[(2 * k2) * 32 + lane], qb = qf[(2 * k2 + 1) * 32 + lane];
+          const int ch = 4 * k2 + mi;  // the 16-byte chunk of dimensions this lane addresses
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-      const float m_old = s_m[g];
-      const float m_new = fmaxf(m_old, mx);
-      const float e0 = exp2f(a0 - m_new), e1 = exp2f(a1 - m_new);
-      float sum = e0 + e1;
+          for (int j = 0; j < 2; ++j) {
+            uint32_t k0, k1, k2r, k3;
+            ldsm_x4(k0, k1, k2r, k3, kb + (ch >> 3) * L::BOX_BYTES + swz128(w0 + 8 * j + rr, ch & 7));
+            mma_bf16(sc[j][0], qa.x, qa.y, qa.z, qa.w, k0, k1);
+            mma_bf16(sc[j][1], qb.x, qb.y, qb.z, qb.w, k2r, k3);
+          }
+        }
+        float sv[2][2];
+        float mx = -INFINITY;
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-      // position pp of the sub-tile: step pp / 16, lane 4 g + ((pp & 7) >> 1), register a0 / a1
-      // (columns 2 tig, 2 tig + 1) or a2 / a3 (pp & 8), half pp & 1
-      auto put = [&](int pp, float e) {
-        uint16_t *f = reinterpret_cast<uint16_t *>(pf + (pp >> 4) * 32 + 4 * g + ((pp & 7) >> 1));
-        const uint16_t hi = f32_to_bf16_rne(e);
-        const int reg = (pp & 8) ? 2 : 0;
-        f[2 * reg + (pp & 1)] = hi;
-        f[2 * (reg + 1) + (pp & 1)] = f32_to_bf16_rne(e - bf16_to_f32(hi));
-      };
-      put(lane, e0);
-      put(lane + 32, e1);
-      if (lane == 0) {
-        const float alpha = exp2f(m_old - m_new);
-        s_alpha[g] = alpha;
-        s_l[g] = s_l[g] * alpha + sum;
-        s_m[g] = m_new;
-      }
-    }
-    att_sync();
-    // acc = acc * alpha + P V over the sub-tile: P fragments from shared memory, V fragments by
-    // transposing loads (ldmatrix .trans: 8 x 8 blocks of positions x dimensions)
-    {
-      const float al = hrow ? s_alpha[gid] : 0.f;
+        for (int j = 0; j < 2; ++j)
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
+          for (int e = 0; e < 2; ++e) {
+            const float v = (sc[j][0][e] + sc[j][1][e]) + (sc[j][0][e + 2] + sc[j][1][e + 2]);
+            sv[j][e] = 8 * j + 2 * tig + e < nv ? v : -INFINITY;
+            mx = fmaxf(mx, sv[j][e]);
+          }
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+        const float m_new = fmaxf(m_run, mx);
+        // a head with no finite score yet keeps weight 0 and scale 1
+        const float alpha = m_new == -INFINITY ? 1.f : exp2f(m_run - m_new);
+        float pr[2][2], lsum = 0.f;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) acc[nt][i] *= al;
-      float pv[NT][2][4] = {};
-      const int mi = lane >> 3;  // the 8 x 8 block whose row this lane addresses
-      const uint8_t *vrow = vb + (8 * (mi & 1) + (lane & 7)) * L::VROW + 2 * (n_base + 8 * (mi >> 1));
+        for (int j = 0; j < 2; ++j)
 #pragma unroll
-      for (int s16 = 0; s16 < ATT_SUB / 16; ++s16) {
-        const uint4 f = pf[s16 * 32 + lane];
-        if constexpr (NT == 2) {
+          for (int e = 0; e < 2; ++e) {
+            pr[j][e] = m_new == -INFINITY ? 0.f : exp2f(sv[j][e] - m_new);
+            lsum += pr[j][e];
+          }
+        lsum += __shfl_xor_sync(0xffffffffu, lsum, 1);
+        lsum += __shfl_xor_sync(0xffffffffu, lsum, 2);
+        l_run = l_run * alpha + lsum;
+        m_run = m_new;
+        if (__any_sync(0xffffffffu, alpha != 1.f)) {
+#pragma unroll
+          for (int d = 0; d < NT; ++d)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) acc[d][i] *= alpha;
+        }
+        // P as the A fragment of P V over the warp's 16 positions: a0 / a2 the rounded parts of
+        // positions (2 tig, 2 tig + 1) and (8 + 2 tig, 9 + 2 tig), a1 / a3 their rests
+        uint32_t a0, a1, a2, a3;
+        bf16_pair2(pr[0][0], pr[0][1], a0, a1);
+        bf16_pair2(pr[1][0], pr[1][1], a2, a3);
+        // acc += P V: V fragments by transposing loads (8 x 8 blocks of positions x dimensions)
+        const int vrow = w0 + 8 * (mi & 1) + rr;
+#pragma unroll
+        for (int d2 = 0; d2 < NT / 2; ++d2) {
+          const int ch = 2 * d2 + (mi >> 1);
           uint32_t v0, v1, v2, v3;
-          ldsm_x4_trans(v0, v1, v2, v3, vrow + 16 * s16 * L::VROW);
-          mma_bf16_full(pv[0][s16 & 1], f, v0, v1);
-          mma_bf16_full(pv[1][s16 & 1], f, v2, v3);
-        } else {
-          uint32_t v0, v1;
-          ldsm_x2_trans(v0, v1, vrow + 16 * s16 * L::VROW);
-          mma_bf16_full(pv[0][s16 & 1], f, v0, v1);
+          ldsm_x4_t(v0, v1, v2, v3, vb + (ch >> 3) * L::BOX_BYTES + swz128(vrow, ch & 7));
+          mma_bf16(acc[2 * d2], a0, a1, a2, a3, v0, v1);
+          mma_bf16(acc[2 * d2 + 1], a0, a1, a2, a3, v2, v3);
         }
       }
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int i = 0; i < 4; ++i) acc[nt][i] += pv[nt][0][i] + pv[nt][1][i];
+      mbar_arrive(smem_addr(&empty[s]));
     }
-    att_sync();
+    // this warp's state: (m, l) per head, sums [warp][head][HD] (rounded + rest rows) in the
+    // stage buffers, once every consumer warp has read its last stage (the copies have all landed:
+    // each was awaited)
+    named_bar_sync(ATT_BAR, ATC_WARPS * 32);
+    if (tig == 0 && gid < G) {
+      s_wm[warp][gid] = m_run;
+      s_wl[warp][gid] = l_run;
+    }
+    float *ws = reinterpret_cast<float *>(sm) + (size_t)warp * ATT_MAXG * HD;
+    if (gid < G) {
+#pragma unroll
+      for (int d = 0; d < NT; ++d)
+        *reinterpret_cast<float2 *>(ws + gid * HD + 8 * d + 2 * tig) =
+            make_float2(acc[d][0] + acc[d][2], acc[d][1] + acc[d][3]);
+    }
+  }
+  __syncthreads();
+  // the CTA's state: per head M = max of the warps' m, each warp's weight 2^(m_w - M), l and the
+  // sums combined in warp order (unnormalised, relative to M)
+  if (tid < G) {
+    const int g = tid;
+    float M = -INFINITY;
+    for (int w = 0; w < ATC_WARPS; ++w) M = fmaxf(M, s_wm[w][g]);
+    float Ls = 0.f;
+    for (int w = 0; w < ATC_WARPS; ++w) {
+      const float e = M == -INFINITY ? 0.f : exp2f(s_wm[w][g] - M);
+      s_wm[w][g] = e;
+      Ls += s_wl[w][g] * e;
+    }
+    s_m[g] = M;
+    s_l[g] = Ls;
+  }
+  __syncthreads();
+  float *part = reinterpret_cast<float *>(sm + L::PART_OFF);
+  {
+    const float *wsum = reinterpret_cast<const float *>(sm);
+    for (int e = tid; e < G * HD; e += ATC_THREADS) {
+      const int g = e / HD;
+      float v = 0.f;
+      for (int w = 0; w < ATC_WARPS; ++w) v = fmaf(s_wm[w][g], wsum[(size_t)w * ATT_MAXG * HD + e], v);
+      part[e] = v;
+    }
   }
   stamp(TR_W_FIRST);
-
-  // this CTA's partial state into its own shared memory (the K buffers): sums [G][HD], and the
-  // (m, l) of each head, read by the cluster after the barrier
-  float *part = reinterpret_cast<float *>(sk);
-  if (hrow) {
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt)
-      *reinterpret_cast<float2 *>(part + gid * HD + n_base + 8 * nt + 2 * tig) =
-          make_float2(acc[nt][0] + acc[nt][2], acc[nt][1] + acc[nt][3]);
-  }
   cluster_sync_all();
   stamp(TR_W_LAST);
 
@@ -248,15 +356,16 @@ __global__ void __launch_bounds__(ATT_THREADS) attn_cluster_kernel(const __grid_
       float M = -INFINITY;
       for (int q = 0; q < C; ++q) M = fmaxf(M, s_w[q][g]);
       float Ls = 0.f;
-      for (int q = 0; q < C; ++q) Ls += s_lw[q][g] * exp2f(s_w[q][g] - M);
+      for (int q = 0; q < C; ++q) Ls += s_lw[q][g] * (s_w[q][g] == -INFINITY ? 0.f : exp2f(s_w[q][g] - M));
       const float inv = 1.0f / Ls;
-      for (int q = 0; q < C; ++q) s_w[q][g] = exp2f(s_w[q][g] - M) * inv;
+      for (int q = 0; q < C; ++q) s_w[q][g] = (s_w[q][g] == -INFINITY ? 0.f : exp2f(s_w[q][g] - M)) * inv;
     }
     __syncthreads();
   }
-  {
-    // lane groups of 8 take one chunk each (4 elements per lane): warp w chunks c0 + 4w .. + 3
-    const int jj = c0 + warp * 4 + (lane >> 3);
+  // lane groups of 8 take one chunk each (4 elements per lane); the warps walk the CTA's chunks
+  // in groups of 4 per warp (every warp calls act16_put_quad as a whole)
+  for (int cb = c0 + warp * 4; cb < c1; cb += (ATC_WARPS + 1) * 4) {
+    const int jj = cb + (lane >> 3);
     const bool mine = jj < c1;
     const int jc = mine ? jj : c0;
     const int g = jc / (HD / XCHUNK), d0 = (jc % (HD / XCHUNK)) * XCHUNK + 4 * (lane & 7);
@@ -283,8 +392,7 @@ __global__ void __launch_bounds__(ATT_THREADS) attn_cluster_kernel(const __grid_
     }
     float *o = p.o + (size_t)b * p.ldo + (size_t)kvh * G * HD;
     if (mine) *reinterpret_cast<float4 *>(o + g * HD + d0) = O;
-    if (p.o16.base && (warp * 4 < c1 - c0))  // the whole warp calls it; `mine` selects the lanes that store
-      act16_put_quad(p.o16, b, ((kvh * G + g) * HD + d0) / XCHUNK, O, lane, mine);
+    if (p.o16.base) act16_put_quad(p.o16, b, ((kvh * G + g) * HD + d0) / XCHUNK, O, lane, mine);
   }
   // no CTA leaves while another may still read its shared memory
   cluster_sync_all();
@@ -294,10 +402,10 @@ __global__ void __launch_bounds__(ATT_THREADS) attn_cluster_kernel(const __grid_
 cudaError_t prepare_attention_cluster() {
   cudaError_t e;
   if ((e = cudaFuncSetAttribute(attn_cluster_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                AttnLayout<128, 2>::BYTES)) != cudaSuccess)
+                                AtcLayout<128>::SMEM)) != cudaSuccess)
     return e;
   if ((e = cudaFuncSetAttribute(attn_cluster_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                AttnLayout<64, 2>::BYTES)) != cudaSuccess)
+                                AtcLayout<64>::SMEM)) != cudaSuccess)
     return e;
   if ((e = cudaFuncSetAttribute(attn_cluster_kernel<128>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) !=
       cudaSuccess)
@@ -311,8 +419,8 @@ int attention_cluster_size(int head_dim, int want) {
   for (int c = want; c >= 2; c >>= 1) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(c);
-    cfg.blockDim = dim3(ATT_THREADS);
-    cfg.dynamicSmemBytes = head_dim == 128 ? AttnLayout<128, 2>::BYTES : AttnLayout<64, 2>::BYTES;
+    cfg.blockDim = dim3(ATC_THREADS);
+    cfg.dynamicSmemBytes = head_dim == 128 ? AtcLayout<128>::SMEM : AtcLayout<64>::SMEM;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = c;
@@ -333,11 +441,12 @@ int attention_cluster_size(int head_dim, int want) {
 }
 
 template <int HD>
-static cudaError_t launch_cluster_hd(const AttnParams &p, cudaStream_t s, bool pdl) {
+static cudaError_t launch_cluster_hd(const AttnParams &p, const CUtensorMap &km, const CUtensorMap &vm,
+                                     cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.batch * p.n_kv_heads * p.cluster);
-  cfg.blockDim = dim3(ATT_THREADS);
-  cfg.dynamicSmemBytes = AttnLayout<HD, 2>::BYTES;
+  cfg.blockDim = dim3(ATC_THREADS);
+  cfg.dynamicSmemBytes = AtcLayout<HD>::SMEM;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   int na = 0;
@@ -353,16 +462,46 @@ static cudaError_t launch_cluster_hd(const AttnParams &p, cudaStream_t s, bool p
   }
   cfg.attrs = attr;
   cfg.numAttrs = na;
-  return cudaLaunchKernelEx(&cfg, attn_cluster_kernel<HD>, p);
+  return cudaLaunchKernelEx(&cfg, attn_cluster_kernel<HD>, p, km, vm);
 }
 
-cudaError_t launch_attention_cluster(const AttnParams &p, int head_dim, cudaStream_t s, bool pdl) {
+cudaError_t launch_attention_cluster(const AttnParams &p, const CUtensorMap &km, const CUtensorMap &vm, int head_dim,
+                                     cudaStream_t s, bool pdl) {
   if (p.n_heads % p.n_kv_heads != 0 || p.n_heads / p.n_kv_heads > ATT_MAXG || p.cluster < 1 ||
       p.cluster > MAX_CLUSTER_ATT)
     return cudaErrorInvalidValue;
-  if (head_dim == 128) return launch_cluster_hd<128>(p, s, pdl);
-  if (head_dim == 64) return launch_cluster_hd<64>(p, s, pdl);
+  if (head_dim == 128) return launch_cluster_hd<128>(p, km, vm, s, pdl);
+  if (head_dim == 64) return launch_cluster_hd<64>(p, km, vm, s, pdl);
   return cudaErrorInvalidValue;
+}
+
+// The K (or V) cache of one layer, [max_batch][n_kv_heads][max_ctx][head_dim] bf16, as a 2-D
+// tensor of head_dim columns and max_batch * n_kv_heads * max_ctx rows, read in boxes of 64
+// positions x 64 dimensions with the 128-byte swizzle; rows past the end read as zero.
+int encode_kv_map(CUtensorMap *map, const uint16_t *base, int head_dim, long long rows) {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void *f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess) {
+      cudaGetLastError();
+      return -1;
+    }
+    fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  }
+  if ((head_dim != 64 && head_dim != 128) || (reinterpret_cast<uintptr_t>(base) & 15) != 0 || rows < 1 ||
+      rows > 0x7FFFFFFFLL)
+    return -1;
+  const cuuint64_t dims[2] = {(cuuint64_t)head_dim, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)head_dim * 2};
+  const cuuint32_t box[2] = {64, (cuuint32_t)ATT_SUB};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t *>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS
+             ? 0
+             : -1;
 }
 
 }  // namespace kfl

@@ -1,6 +1,7 @@
 // Internal definitions shared by the stage-decode kernels and the runtime (sm_103a only).
 #pragma once
 
+#include <cuda.h>  // CUtensorMap (the type only; maps are encoded through the runtime's entry point)
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -611,7 +612,9 @@ cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s, 
 cudaError_t launch_qknorm(const QkNormParams &p, cudaStream_t s, bool pdl);
 cudaError_t prepare_attention_cluster();
 int attention_cluster_size(int head_dim, int want);  // valid after prepare_attention_cluster
-cudaError_t launch_attention_cluster(const AttnParams &p, int head_dim, cudaStream_t s, bool pdl);
+cudaError_t launch_attention_cluster(const AttnParams &p, const CUtensorMap &kmap, const CUtensorMap &vmap,
+                                     int head_dim, cudaStream_t s, bool pdl);
+int encode_kv_map(CUtensorMap *map, const uint16_t *base, int head_dim, long long rows);
 cudaError_t launch_stage_input(const int *ids, const float *hidden_in, const int *positions_in,
                                int batch, const uint16_t *embed, int vocab, int d, int ldh,
                                const float *g_next, float *h, float *xn, float *sumsq,

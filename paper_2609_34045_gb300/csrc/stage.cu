@@ -248,6 +248,7 @@ struct kfl_stage {
   // lm_head.  int4 stages: one map per matrix kind [j] (then lm_head) over pf_w16, the fp16 tiles
   // of the matrix being multiplied (dequantized just before its GEMM)
   std::vector<CUtensorMap> pf_maps;  // int4: [buffer * 5 + kind]
+  std::vector<CUtensorMap> kv_maps;  // attention clusters: layer l's K cache [2 l] and V cache [2 l + 1]
   uint16_t *pf_w16[2] = {};
   // int4: matrix g + 1 of a pass is dequantized on pf_side into buffer (g + 1) % 2 while GEMM g
   // reads buffer g % 2; pf_deq[b] marks a buffer filled, pf_used[b] its GEMM done
@@ -614,8 +615,8 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
       CK(launch_gemv(g, ph.epi, grid, s, pdl));
     } else {
       if (ph.qn.raw) CK(launch_qknorm(ph.qn, s, pdl));  // QK-norm stages: norm, RoPE, KV append
-      if (ph.a.cluster > 0)
-        CK(launch_attention_cluster(ph.a, st->P.hd, s, pdl));
+      if (ph.a.cluster > 0)  // phases come five per block: Q/K/V, attention, O, gate/up, down
+        CK(launch_attention_cluster(ph.a, st->kv_maps[2 * (i / 5)], st->kv_maps[2 * (i / 5) + 1], st->P.hd, s, pdl));
       else
         CK(launch_attention(ph.a, st->P.hd, s, pdl));
     }
@@ -1216,6 +1217,13 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
   if (P.nl > 0) {
     if (cudaMemset(st->kc, 0, (size_t)P.nl * P.kv_elems_per_layer * 2) != cudaSuccess) return fail(KFL_ERR_CUDA);
     if (cudaMemset(st->vc, 0, (size_t)P.nl * P.kv_elems_per_layer * 2) != cudaSuccess) return fail(KFL_ERR_CUDA);
+    // the attention clusters read each layer's cache through TMA tensor maps
+    st->kv_maps.resize(2 * (size_t)P.nl);
+    const long long rows = (long long)cfg->max_batch * P.hkv * cfg->max_ctx;
+    for (int l = 0; l < P.nl; ++l)
+      if (encode_kv_map(&st->kv_maps[2 * l], st->kc + (size_t)l * P.kv_elems_per_layer, P.hd, rows) ||
+          encode_kv_map(&st->kv_maps[2 * l + 1], st->vc + (size_t)l * P.kv_elems_per_layer, P.hd, rows))
+        return fail(KFL_ERR_CUDA);
   }
   if (cudaMemset(st->h, 0, (size_t)MAXB * P.ldh * 4) || cudaMemset(st->xn, 0, (size_t)MAXB * P.ldh * 4) ||
       cudaMemset(st->q, 0, (size_t)MAXB * P.ldq * 4) || cudaMemset(st->o, 0, (size_t)MAXB * P.ldq * 4) ||
