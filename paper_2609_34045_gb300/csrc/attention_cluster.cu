@@ -33,22 +33,23 @@ namespace kfl {
 
 constexpr int ATC_WARPS = 4;                       // consumer warps, 16 positions of a stage each
 constexpr int ATC_THREADS = (ATC_WARPS + 1) * 32;  // + the producer warp
-constexpr int ATC_STAGES = 3;
 
+// Shared memory of a CTA with a ring of S stages: the stages, q's A fragments, the barriers.
 template <int HD>
 struct AtcLayout {
   static constexpr int BOXES = HD / 64;                  // 64-dimension boxes of a row
   static constexpr int BOX_BYTES = ATT_SUB * 128;        // 64 positions x 64 bf16, swizzled
   static constexpr int KV_BYTES = BOXES * BOX_BYTES;     // the K (or V) rows of one stage
   static constexpr int STAGE_BYTES = 2 * KV_BYTES;
-  static constexpr int QF_OFF = ATC_STAGES * STAGE_BYTES;  // q as A fragments [HD / 16][32] uint4
-  static constexpr int BAR_OFF = QF_OFF + (HD / 16) * 32 * 16;
-  static constexpr int BYTES = BAR_OFF + 2 * ATC_STAGES * 8;
-  static constexpr int SMEM = BYTES + 1024;              // + the alignment of the swizzled boxes
+  static constexpr int QF_BYTES = (HD / 16) * 32 * 16;   // q as A fragments [HD / 16][32] uint4
+  __host__ __device__ static constexpr int qf_off(int S) { return S * STAGE_BYTES; }
+  __host__ __device__ static constexpr int bar_off(int S) { return qf_off(S) + QF_BYTES; }
+  // + 1024: the alignment of the swizzled boxes
+  __host__ __device__ static constexpr int smem(int S) { return bar_off(S) + 2 * S * 8 + 1024; }
   // after the loop, in the stage buffers: the warps' sums [ATC_WARPS][ATT_MAXG][HD], then the
   // CTA's merged sums [ATT_MAXG][HD] (read by the cluster)
   static constexpr int PART_OFF = ATC_WARPS * ATT_MAXG * HD * 4;
-  static_assert(PART_OFF + ATT_MAXG * HD * 4 <= ATC_STAGES * STAGE_BYTES, "merge scratch");
+  static_assert(PART_OFF + ATT_MAXG * HD * 4 <= STAGE_BYTES, "merge scratch");
 };
 
 // Byte offset of 16-byte chunk c of row r in a box of 128-byte rows written with the 128-byte
@@ -116,9 +117,10 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
       p.trace[(size_t)blockIdx.x * TRACE_SLOTS + slot] = global_ns();
   };
   stamp(TR_CONS_GO);
-  uint64_t *full = reinterpret_cast<uint64_t *>(sm + L::BAR_OFF);
-  uint64_t *empty = full + ATC_STAGES;
-  uint4 *qf = reinterpret_cast<uint4 *>(sm + L::QF_OFF);
+  const int S = p.stages;  // ring depth
+  uint64_t *full = reinterpret_cast<uint64_t *>(sm + L::bar_off(S));
+  uint64_t *empty = full + S;
+  uint4 *qf = reinterpret_cast<uint4 *>(sm + L::qf_off(S));
   const uint32_t sm0 = smem_addr(sm);
 
   const int P = p.positions[b];
@@ -131,7 +133,7 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
   }
   const int nsub = end > start ? (end - start + ATT_SUB - 1) / ATT_SUB : 0;
   if (tid == 0) {
-    for (int s = 0; s < ATC_STAGES; ++s) {
+    for (int s = 0; s < S; ++s) {
       mbar_init(smem_addr(&full[s]), 1);
       mbar_init(smem_addr(&empty[s]), ATC_WARPS * 32);
     }
@@ -152,8 +154,8 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
       bool waited = false;
       int issued = 0;
       for (int t = 0; t < nsub; ++t) {
-        const int s = t % ATC_STAGES;
-        if (t >= ATC_STAGES && !mbar_wait(smem_addr(&empty[s]), ((t / ATC_STAGES) - 1) & 1)) {
+        const int s = t % S;
+        if (t >= S && !mbar_wait(smem_addr(&empty[s]), ((t / S) - 1) & 1)) {
           s_abort = 1;
           atomicOr(p.err, ERR_TIMEOUT);
           break;
@@ -175,8 +177,7 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
         ++issued;
       }
       // copies still in flight land before the shared memory is reused (bounded)
-      for (int t = issued > ATC_STAGES ? issued - ATC_STAGES : 0; t < issued; ++t)
-        mbar_wait(smem_addr(&full[t % ATC_STAGES]), (t / ATC_STAGES) & 1);
+      for (int t = issued > S ? issued - S : 0; t < issued; ++t) mbar_wait(smem_addr(&full[t % S]), (t / S) & 1);
     }
   } else {
     // ------------------------------------------------------------------ consumers
@@ -204,9 +205,9 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
 #pragma unroll
     for (int d = 0; d < NT; ++d) acc[d][0] = acc[d][1] = acc[d][2] = acc[d][3] = 0.f;
     for (int t = 0; t < nsub; ++t) {
-      const int s = t % ATC_STAGES;
+      const int s = t % S;
       if (s_abort) break;
-      if (!mbar_wait(smem_addr(&full[s]), (t / ATC_STAGES) & 1)) {
+      if (!mbar_wait(smem_addr(&full[s]), (t / S) & 1)) {
         s_abort = 1;
         atomicOr(p.err, ERR_TIMEOUT);
         break;
@@ -402,10 +403,10 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
 cudaError_t prepare_attention_cluster() {
   cudaError_t e;
   if ((e = cudaFuncSetAttribute(attn_cluster_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                AtcLayout<128>::SMEM)) != cudaSuccess)
+                                AtcLayout<128>::smem(ATT_RING_MAX))) != cudaSuccess)
     return e;
   if ((e = cudaFuncSetAttribute(attn_cluster_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                AtcLayout<64>::SMEM)) != cudaSuccess)
+                                AtcLayout<64>::smem(ATT_RING_MAX))) != cudaSuccess)
     return e;
   if ((e = cudaFuncSetAttribute(attn_cluster_kernel<128>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) !=
       cudaSuccess)
@@ -413,14 +414,14 @@ cudaError_t prepare_attention_cluster() {
   return cudaFuncSetAttribute(attn_cluster_kernel<64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
 }
 
-// The largest cluster size up to `want` (a power of two) that the device schedules for this
-// kernel, or 0 if none.
-int attention_cluster_size(int head_dim, int want) {
-  for (int c = want; c >= 2; c >>= 1) {
+// The largest cluster size up to `want` that the device schedules for this kernel with a ring of
+// `stages` sub-tiles, or 0 if none.
+int attention_cluster_size(int head_dim, int want, int stages) {
+  for (int c = want; c >= 2; --c) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(c);
     cfg.blockDim = dim3(ATC_THREADS);
-    cfg.dynamicSmemBytes = head_dim == 128 ? AtcLayout<128>::SMEM : AtcLayout<64>::SMEM;
+    cfg.dynamicSmemBytes = head_dim == 128 ? AtcLayout<128>::smem(stages) : AtcLayout<64>::smem(stages);
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = c;
@@ -446,7 +447,7 @@ static cudaError_t launch_cluster_hd(const AttnParams &p, const CUtensorMap &km,
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.batch * p.n_kv_heads * p.cluster);
   cfg.blockDim = dim3(ATC_THREADS);
-  cfg.dynamicSmemBytes = AtcLayout<HD>::SMEM;
+  cfg.dynamicSmemBytes = AtcLayout<HD>::smem(p.stages);
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   int na = 0;
@@ -468,7 +469,7 @@ static cudaError_t launch_cluster_hd(const AttnParams &p, const CUtensorMap &km,
 cudaError_t launch_attention_cluster(const AttnParams &p, const CUtensorMap &km, const CUtensorMap &vm, int head_dim,
                                      cudaStream_t s, bool pdl) {
   if (p.n_heads % p.n_kv_heads != 0 || p.n_heads / p.n_kv_heads > ATT_MAXG || p.cluster < 1 ||
-      p.cluster > MAX_CLUSTER_ATT)
+      p.cluster > MAX_CLUSTER_ATT || p.stages < 2 || p.stages > ATT_RING_MAX)
     return cudaErrorInvalidValue;
   if (head_dim == 128) return launch_cluster_hd<128>(p, km, vm, s, pdl);
   if (head_dim == 64) return launch_cluster_hd<64>(p, km, vm, s, pdl);

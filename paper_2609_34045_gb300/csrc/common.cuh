@@ -225,8 +225,10 @@ struct AttnParams {
   int chunk, n_chunks, target_units;
   // one kernel per phase: > 0 runs attn_cluster_kernel, one thread-block cluster of `cluster`
   // CTAs per (user, KV head) that split its positions and merge through distributed shared
-  // memory (partial, tickets, chunk and target_units are then unused)
+  // memory (partial, tickets, chunk and target_units are then unused), each with a ring of
+  // `stages` sub-tiles (three: two CTAs fit an SM; two: three)
   int cluster;
+  int stages;
   float scale_log2;          // log2(e) / sqrt(hd)
   unsigned *err;
   // dataflow (persistent stage kernel only)
@@ -611,7 +613,8 @@ int gemv_stages_for(int batch, int fmt, int cluster, int per_sm);  // valid afte
 cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s, bool pdl);
 cudaError_t launch_qknorm(const QkNormParams &p, cudaStream_t s, bool pdl);
 cudaError_t prepare_attention_cluster();
-int attention_cluster_size(int head_dim, int want);  // valid after prepare_attention_cluster
+constexpr int ATT_RING_MAX = 3;  // attention clusters: the deepest ring (sub-tiles); two CTAs fit an SM
+int attention_cluster_size(int head_dim, int want, int stages);  // valid after prepare_attention_cluster
 cudaError_t launch_attention_cluster(const AttnParams &p, const CUtensorMap &kmap, const CUtensorMap &vmap,
                                      int head_dim, cudaStream_t s, bool pdl);
 int encode_kv_map(CUtensorMap *map, const uint16_t *base, int head_dim, long long rows);

@@ -63,6 +63,8 @@ struct Plan {
   int n_phases, ctr_stride;  // persistent kernel: phases per step, readiness counters per phase
   int attn_units;            // attention units a step aims at (the kernels size chunks to it)
   int attn_cluster_max;      // one kernel per phase: the largest attention cluster (0: unit kernel)
+  int attn_stages;           // attention clusters: ring depth (sub-tiles) of a CTA
+  int attn_cluster_sub;      // clusters are taken up to this many 64-position sub-tiles per CTA
   size_t bytes_weights, bytes_kv, bytes_ws;
 };
 
@@ -150,6 +152,7 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   p->n_parts = (p->d + RB - 1) / RB;
   // two attention CTAs fit an SM: about two units per SM over the step's actual contexts
   p->attn_units = n_sm * std::max(1, env_int("KFL_ATTN_UNITS_PER_SM", 2));
+  p->attn_cluster_sub = env_int("KFL_ATTN_CLUSTER_SUB", 1 << 20);
   p->attn_nchunks_max = (c->max_ctx + 63) / 64;
   p->n_phases = 5 * p->nl + ((flags & KFL_LOGITS_OUT) ? 1 : 0);
   {
@@ -404,14 +407,21 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
       a.target_units = P.attn_units;
       if (!dataflow && P.attn_cluster_max >= 2) {
         // one cluster per (user, KV head): the largest power of two up to the maximum with at
-        // most two CTAs per SM in all
-        int cl = P.attn_cluster_max;
-        while (cl > 2 && (long long)cl * batch * P.hkv > 2LL * P.n_sm) cl >>= 1;
-        // the clusters cannot balance ragged users or spread a long context over idle SMs: they
-        // are taken when each CTA has at most five 64-position sub-tiles at the longest context
-        // (the merge latency then dominates) or when they give every SM at least one CTA
+        // most as many CTAs as fit the SMs at once (power-of-two clusters and two or three
+        // CTAs per SM measured fastest; clusters sized to fill the SMs exactly and one CTA per SM
+        // with a deeper ring were slower)
+        int cl = 1;
+        while (cl * 2 <= P.attn_cluster_max) cl *= 2;
+        const long long slots = (long long)P.n_sm * (P.attn_stages <= 2 ? 3 : 2);
+        while (cl > 2 && (long long)cl * batch * P.hkv > slots) cl >>= 1;
+        a.stages = P.attn_stages;
+        // the clusters cannot balance ragged users or spread a long context over idle SMs, but
+        // their CTAs stream without block barriers: they are taken unless a CTA would have more
+        // than KFL_ATTN_CLUSTER_SUB 64-position sub-tiles at the longest context while the
+        // clusters leave SMs idle (by default always: measured no slower than the unit kernel
+        // on every workload, 72B int4 b=1 20.0 against 22.4 us per block)
         const int per_cta = (c.max_ctx + cl - 1) / cl;
-        if (per_cta <= 5 * 64 || (long long)cl * batch * P.hkv >= P.n_sm) a.cluster = cl;
+        if (per_cta <= P.attn_cluster_sub * 64 || (long long)cl * batch * P.hkv >= P.n_sm) a.cluster = cl;
       }
       a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)P.hd));
       a.err = st->err;
@@ -1135,7 +1145,8 @@ extern "C" int kfl_stage_create(const kfl_model_cfg *cfg, int l0, int l1, int fl
   Plan &P = st->P;
   {
     const int want = env_int("KFL_ATTN_CLUSTER", MAX_CLUSTER_ATT);
-    P.attn_cluster_max = want >= 2 ? attention_cluster_size(P.hd, std::min(want, MAX_CLUSTER_ATT)) : 0;
+    P.attn_stages = std::max(2, std::min(ATT_RING_MAX, env_int("KFL_ATTN_STAGES", 3)));
+    P.attn_cluster_max = want >= 2 ? attention_cluster_size(P.hd, std::min(want, MAX_CLUSTER_ATT), P.attn_stages) : 0;
   }
   auto fail = [&](int code) {
     kfl_stage_destroy(st);
