@@ -14,9 +14,11 @@
 // barrier in its loop: the scores of its 16 positions (two m16n8k16 accumulator tiles) are, after
 // the softmax, exactly the A fragments of its P V product, so P never leaves the registers.
 // After the loop the four warp states merge into the CTA's (in shared memory), and the C CTA
-// states meet through distributed shared memory: CTA r merges its share of the output's
-// 32-element chunks, reading every CTA's (m, l) and partial sums in CTA order (deterministic), and
-// writes them (int4 stages: also in the O projection's input form).
+// states meet in distributed shared memory: every CTA sends its (m, l) per head to all CTAs of
+// the cluster and its sums of each 32-element output chunk to the CTA that merges that chunk, with
+// asynchronous stores whose bytes complete on the receiver's mbarrier (no round trip, no cluster
+// barrier between sending and merging); CTA r then adds its chunks' sums in CTA order
+// (deterministic) and writes them (int4 stages: also in the O projection's input form).
 //
 // Scores S = q K^T and P V run as bf16 m16n8k16 MMAs with fp32 accumulation.  q and P enter as
 // bf16 pairs (rounded value, bf16 of the rest: about 2^-17 relative): rows 0..7 of the MMA's A
@@ -46,10 +48,8 @@ struct AtcLayout {
   __host__ __device__ static constexpr int bar_off(int S) { return qf_off(S) + QF_BYTES; }
   // + 1024: the alignment of the swizzled boxes
   __host__ __device__ static constexpr int smem(int S) { return bar_off(S) + 2 * S * 8 + 1024; }
-  // after the loop, in the stage buffers: the warps' sums [ATC_WARPS][ATT_MAXG][HD], then the
-  // CTA's merged sums [ATT_MAXG][HD] (read by the cluster)
-  static constexpr int PART_OFF = ATC_WARPS * ATT_MAXG * HD * 4;
-  static_assert(PART_OFF + ATT_MAXG * HD * 4 <= STAGE_BYTES, "merge scratch");
+  // after the loop, in the stage buffers: the warps' sums [ATC_WARPS][ATT_MAXG][HD]
+  static_assert(ATC_WARPS * ATT_MAXG * HD * 4 <= STAGE_BYTES, "merge scratch");
 };
 
 // Byte offset of 16-byte chunk c of row r in a box of 128-byte rows written with the 128-byte
@@ -85,6 +85,29 @@ __device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
+// Asynchronous stores into another CTA of the cluster that count their bytes on that CTA's
+// mbarrier (complete_tx): the receiver learns that every store has landed from the barrier alone.
+__device__ __forceinline__ void st_async_f4(uint32_t addr, float4 v, uint32_t bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(addr),
+               "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(bar)
+               : "memory");
+}
+__device__ __forceinline__ void st_async_f2(uint32_t addr, float a, float b, uint32_t bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.f32 [%0], {%1, %2}, [%3];" ::"r"(addr),
+               "f"(a), "f"(b), "r"(bar)
+               : "memory");
+}
+// The cluster barrier in two halves, so that a CTA does other work between its arrival and its wait.
+__device__ __forceinline__ void cluster_arrive_release() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait_acquire() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 // (rounded, rest) bf16 pairs of two weights as the packed registers of one A-fragment row pair
 __device__ __forceinline__ void bf16_pair2(float x0, float x1, uint32_t &hi, uint32_t &lo) {
   const uint16_t h0 = f32_to_bf16_rne(x0), h1 = f32_to_bf16_rne(x1);
@@ -99,8 +122,13 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
   using L = AtcLayout<HD>;
   extern __shared__ uint8_t sm_raw[];
   uint8_t *sm = sm_raw + ((1024u - (smem_addr(sm_raw) & 1023u)) & 1023u);
-  __shared__ float s_w[MAX_CLUSTER_ATT][ATT_MAXG];  // merge: (m, then weight) of each CTA and head
-  __shared__ float s_lw[MAX_CLUSTER_ATT][ATT_MAXG];
+  // the cluster merge: what every CTA of the cluster sends this one (its (m, l) per head, and its
+  // sums of this CTA's output chunks, [source CTA][chunk - c0][XCHUNK]), the barrier that counts
+  // those bytes, and each source CTA's weight per head
+  __shared__ __align__(16) float s_recv[(ATT_MAXG * 128 / XCHUNK + MAX_CLUSTER_ATT) * XCHUNK];
+  __shared__ __align__(8) float2 s_rml[MAX_CLUSTER_ATT][ATT_MAXG];
+  __shared__ __align__(8) uint64_t s_rbar;
+  __shared__ float s_w[MAX_CLUSTER_ATT][ATT_MAXG];
   __shared__ float s_wm[ATC_WARPS][ATT_MAXG];       // each consumer warp's (m, then weight) per head
   __shared__ float s_wl[ATC_WARPS][ATT_MAXG];
   __shared__ float s_m[ATT_MAXG], s_l[ATT_MAXG];     // this CTA's state, read by the cluster
@@ -112,10 +140,15 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int G = p.n_heads / p.n_kv_heads;
   const int gid = lane >> 2, tig = lane & 3;
-  auto stamp = [&](int slot) {
-    if (p.trace && (int)blockIdx.x < p.trace_grid && tid == 0)
-      p.trace[(size_t)blockIdx.x * TRACE_SLOTS + slot] = global_ns();
+  // trace slots of an attention CTA: go (start), enter (consumers past the wait on Q/K/V), x_go
+  // (q's fragments built), x_last (first stage landed), kind (warp 0 done with the first stage),
+  // seg (warp 0 done with its stages), ticket
+  // (every consumer warp done), summed (producer past its wait on Q/K/V), w_first / w_last (around
+  // the first cluster barrier), epi (cluster weights computed), done (end)
+  auto stamp_by = [&](bool who, int slot) {
+    if (p.trace && (int)blockIdx.x < p.trace_grid && who) p.trace[(size_t)blockIdx.x * TRACE_SLOTS + slot] = global_ns();
   };
+  auto stamp = [&](int slot) { stamp_by(tid == 0, slot); };
   stamp(TR_CONS_GO);
   const int S = p.stages;  // ring depth
   uint64_t *full = reinterpret_cast<uint64_t *>(sm + L::bar_off(S));
@@ -132,15 +165,26 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
     end = min(P + 1, static_cast<int>((long long)(r + 1) * nsub_all / C) * ATT_SUB);
   }
   const int nsub = end > start ? (end - start + ATT_SUB - 1) / ATT_SUB : 0;
+  // output chunks of XCHUNK elements of the pair's G x HD: CTA r merges [c0, c1)
+  const int nch = G * HD / XCHUNK;
+  const int c0 = static_cast<int>((long long)r * nch / C), c1 = static_cast<int>((long long)(r + 1) * nch / C);
+  const int own = (nch + C - 1) / C;  // rows of s_recv per source CTA
+  const uint32_t rbar = smem_addr(&s_rbar);
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(smem_addr(&full[s]), 1);
       mbar_init(smem_addr(&empty[s]), ATC_WARPS * 32);
     }
+    // every CTA of the cluster sends its (m, l) of the G heads and its sums of chunks [c0, c1)
+    mbar_init(rbar, 1);
+    mbar_arrive_expect_tx(rbar, static_cast<uint32_t>(C * (G * 8 + (c1 - c0) * XCHUNK * 4)));
     s_abort = 0;
     fence_mbar_init();
   }
   __syncthreads();
+  // the other CTAs send into this one's shared memory only after its barrier is initialised: they
+  // wait on the cluster barrier after the loop (this arrival makes the initialisation visible)
+  cluster_arrive_release();
 
   constexpr int KS = HD / 16;  // K steps of the scores
   constexpr int NT = HD / 8;   // n-tiles (8 dimensions) of P V
@@ -165,6 +209,7 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
         if (!waited && p0 + ATT_SUB > lo) {
           pdl_wait();
           waited = true;
+          stamp_by(true, TR_E_SUMMED);
         }
         const uint32_t fb = smem_addr(&full[s]);
         mbar_arrive_expect_tx(fb, L::STAGE_BYTES);
@@ -182,22 +227,34 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
   } else {
     // ------------------------------------------------------------------ consumers
     pdl_wait();  // q and this step's K/V rows come from the Q/K/V projection
+    stamp(TR_CONS_ENTER);
     // q (scaled to log2 units) as the scores' A fragments: entry (step, lane) = registers a0..a3:
     // rows gid (the heads' rounded parts) and gid + 8 (their rests), columns 2 tig, 2 tig + 1
     // (a0, a1) and + 8 (a2, a3); rows of heads >= G are zero
-    for (int e = tid; e < KS * 32; e += ATC_WARPS * 32) {
+    // (every load is issued before any is used: one round trip to L2)
+    constexpr int QPT = KS / ATC_WARPS;  // entries per consumer thread
+    static_assert(QPT * ATC_WARPS == KS, "q fragments per thread");
+    float2 xq[QPT][2];
+#pragma unroll
+    for (int i = 0; i < QPT; ++i) {
+      const int e = tid + i * ATC_WARPS * 32;
       const int st = e >> 5, l = e & 31, g = l >> 2, t = l & 3;
-      uint4 f = make_uint4(0u, 0u, 0u, 0u);
+      xq[i][0] = xq[i][1] = make_float2(0.f, 0.f);
       if (valid && g < G) {
         const float *qg = p.q + (size_t)b * p.n_heads * HD + (size_t)(kvh * G + g) * HD + 16 * st + 2 * t;
-        const float2 x0 = __ldcg(reinterpret_cast<const float2 *>(qg));
-        const float2 x1 = __ldcg(reinterpret_cast<const float2 *>(qg + 8));
-        bf16_pair2(x0.x * p.scale_log2, x0.y * p.scale_log2, f.x, f.y);
-        bf16_pair2(x1.x * p.scale_log2, x1.y * p.scale_log2, f.z, f.w);
+        xq[i][0] = __ldcg(reinterpret_cast<const float2 *>(qg));
+        xq[i][1] = __ldcg(reinterpret_cast<const float2 *>(qg + 8));
       }
-      qf[e] = f;
+    }
+#pragma unroll
+    for (int i = 0; i < QPT; ++i) {
+      uint4 f;
+      bf16_pair2(xq[i][0].x * p.scale_log2, xq[i][0].y * p.scale_log2, f.x, f.y);
+      bf16_pair2(xq[i][1].x * p.scale_log2, xq[i][1].y * p.scale_log2, f.z, f.w);
+      qf[tid + i * ATC_WARPS * 32] = f;
     }
     named_bar_sync(ATT_BAR, ATC_WARPS * 32);
+    stamp(TR_X_GO);
 
     const int w0 = warp * 16;  // this warp's positions within a stage
     float m_run = -INFINITY, l_run = 0.f;  // head gid
@@ -212,6 +269,7 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
         atomicOr(p.err, ERR_TIMEOUT);
         break;
       }
+      if (t == 0) stamp(TR_X_LAST);
       const int nv = min(ATT_SUB, end - (start + t * ATT_SUB)) - w0;  // valid positions of this warp
       const uint32_t kb = sm0 + s * L::STAGE_BYTES, vb = kb + L::KV_BYTES;
       if (nv > 0) {
@@ -293,11 +351,14 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
         }
       }
       mbar_arrive(smem_addr(&empty[s]));
+      if (t == 0) stamp(TR_E_KIND);
     }
+    stamp(TR_E_SEG);
     // this warp's state: (m, l) per head, sums [warp][head][HD] (rounded + rest rows) in the
     // stage buffers, once every consumer warp has read its last stage (the copies have all landed:
     // each was awaited)
     named_bar_sync(ATT_BAR, ATC_WARPS * 32);
+    stamp(TR_E_TICKET);
     if (tig == 0 && gid < G) {
       s_wm[warp][gid] = m_run;
       s_wl[warp][gid] = l_run;
@@ -327,44 +388,64 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
     s_l[g] = Ls;
   }
   __syncthreads();
-  float *part = reinterpret_cast<float *>(sm + L::PART_OFF);
+  stamp(TR_W_FIRST);
+  // every CTA's receive barrier is initialised
+  __syncwarp();
+  cluster_wait_acquire();
+  stamp(TR_W_LAST);
+  // send: this CTA's (m, l) of every head to every CTA of the cluster, and its sums (the warps'
+  // sums weighted in warp order) of each output chunk to the CTA that merges the chunk, the
+  // largest o with o nch / C <= j
+  if (tid < C * G) {
+    const int q = tid / G, g = tid % G;
+    st_async_f2(map_to_rank(smem_addr(&s_rml[r][g]), q), s_m[g], s_l[g], map_to_rank(rbar, q));
+  }
   {
     const float *wsum = reinterpret_cast<const float *>(sm);
-    for (int e = tid; e < G * HD; e += ATC_THREADS) {
-      const int g = e / HD;
-      float v = 0.f;
-      for (int w = 0; w < ATC_WARPS; ++w) v = fmaf(s_wm[w][g], wsum[(size_t)w * ATT_MAXG * HD + e], v);
-      part[e] = v;
+    for (int e4 = tid; e4 < G * HD / 4; e4 += ATC_THREADS) {
+      const int e = 4 * e4, g = e / HD;
+      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int w = 0; w < ATC_WARPS; ++w) {
+        const float sw = s_wm[w][g];
+        const float4 x = *reinterpret_cast<const float4 *>(wsum + (size_t)w * ATT_MAXG * HD + e);
+        v.x = fmaf(sw, x.x, v.x);
+        v.y = fmaf(sw, x.y, v.y);
+        v.z = fmaf(sw, x.z, v.z);
+        v.w = fmaf(sw, x.w, v.w);
+      }
+      const int j = e / XCHUNK;
+      const int o = ((j + 1) * C - 1) / nch;
+      const int jl = j - static_cast<int>((long long)o * nch / C);
+      st_async_f4(map_to_rank(smem_addr(s_recv + ((size_t)r * own + jl) * XCHUNK + e % XCHUNK), o), v,
+                  map_to_rank(rbar, o));
     }
   }
-  stamp(TR_W_FIRST);
-  cluster_sync_all();
-  stamp(TR_W_LAST);
+  // no CTA leaves while another may still send to it (its wait at the end)
+  __syncwarp();
+  cluster_arrive_relaxed();
 
-  // merge: CTA r takes chunks [r nch / C, (r + 1) nch / C) of the pair's G x HD outputs
-  const int nch = G * HD / XCHUNK;
-  const int c0 = static_cast<int>((long long)r * nch / C), c1 = static_cast<int>((long long)(r + 1) * nch / C);
-  if (valid) {
-    // every CTA's (m, l) per head, then each head's weights 2^(m_q - M) / L in CTA order
-    if (tid < C * G) {
-      const int q = tid / G, g = tid % G;
-      s_w[q][g] = ld_cluster_f32(map_to_rank(smem_addr(s_m + g), q));
-      s_lw[q][g] = ld_cluster_f32(map_to_rank(smem_addr(s_l + g), q));
-    }
-    __syncthreads();
-    if (tid < G) {
-      const int g = tid;
-      float M = -INFINITY;
-      for (int q = 0; q < C; ++q) M = fmaxf(M, s_w[q][g]);
-      float Ls = 0.f;
-      for (int q = 0; q < C; ++q) Ls += s_lw[q][g] * (s_w[q][g] == -INFINITY ? 0.f : exp2f(s_w[q][g] - M));
-      const float inv = 1.0f / Ls;
-      for (int q = 0; q < C; ++q) s_w[q][g] = (s_w[q][g] == -INFINITY ? 0.f : exp2f(s_w[q][g] - M)) * inv;
-    }
-    __syncthreads();
+  // receive: every CTA's (m, l) and sums of chunks [c0, c1) have landed (bounded)
+  if (!mbar_wait_cluster(rbar, 0)) {
+    if (tid == 0) atomicOr(p.err, ERR_TIMEOUT);
   }
+  // each CTA's weight per head, 2^(m_q - M) / L with M the largest m and L = sum of l_q 2^(m_q - M)
+  // (one warp per head, lane q holding CTA q; a head no CTA has seen gets weight 0)
+  for (int g = warp; g < G; g += ATC_WARPS + 1) {
+    const float2 ml = lane < C ? s_rml[lane][g] : make_float2(-INFINITY, 0.f);
+    float M = ml.x;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    const float e = ml.x == -INFINITY ? 0.f : exp2f(ml.x - M);
+    float Ls = ml.y * e;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) Ls += __shfl_xor_sync(0xffffffffu, Ls, off);
+    if (lane < C) s_w[lane][g] = Ls > 0.f ? e * (1.0f / Ls) : 0.f;
+  }
+  __syncthreads();
+  stamp(TR_E_DONE);
   // lane groups of 8 take one chunk each (4 elements per lane); the warps walk the CTA's chunks
-  // in groups of 4 per warp (every warp calls act16_put_quad as a whole)
+  // in groups of 4 per warp (every warp calls act16_put_quad as a whole); the CTAs' sums are
+  // added in CTA order
   for (int cb = c0 + warp * 4; cb < c1; cb += (ATC_WARPS + 1) * 4) {
     const int jj = cb + (lane >> 3);
     const bool mine = jj < c1;
@@ -372,31 +453,22 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
     const int g = jc / (HD / XCHUNK), d0 = (jc % (HD / XCHUNK)) * XCHUNK + 4 * (lane & 7);
     float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
     if (valid && mine) {
-      // the CTAs' sums are loaded four at a time before any is used, so that the distributed
-      // shared memory round trips overlap; then added in CTA order
-      const uint32_t src = smem_addr(part + g * HD + d0);
-      for (int q0 = 0; q0 < C; q0 += 4) {
-        float4 v[4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) v[j] = q0 + j < C ? ld_cluster_f4(map_to_rank(src, q0 + j)) : make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          if (q0 + j < C) {
-            const float w = s_w[q0 + j][g];
-            O.x = fmaf(w, v[j].x, O.x);
-            O.y = fmaf(w, v[j].y, O.y);
-            O.z = fmaf(w, v[j].z, O.z);
-            O.w = fmaf(w, v[j].w, O.w);
-          }
-        }
+      const float *src = s_recv + (size_t)(jc - c0) * XCHUNK + 4 * (lane & 7);
+      for (int q = 0; q < C; ++q) {
+        const float4 v = *reinterpret_cast<const float4 *>(src + (size_t)q * own * XCHUNK);
+        const float w = s_w[q][g];
+        O.x = fmaf(w, v.x, O.x);
+        O.y = fmaf(w, v.y, O.y);
+        O.z = fmaf(w, v.z, O.z);
+        O.w = fmaf(w, v.w, O.w);
       }
     }
     float *o = p.o + (size_t)b * p.ldo + (size_t)kvh * G * HD;
     if (mine) *reinterpret_cast<float4 *>(o + g * HD + d0) = O;
     if (p.o16.base) act16_put_quad(p.o16, b, ((kvh * G + g) * HD + d0) / XCHUNK, O, lane, mine);
   }
-  // no CTA leaves while another may still read its shared memory
-  cluster_sync_all();
+  __syncwarp();
+  cluster_wait_acquire();
   stamp(TR_CONS_DONE);
 }
 
