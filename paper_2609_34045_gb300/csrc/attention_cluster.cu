@@ -3,8 +3,8 @@
 //
 // User b's token at position P_b attends to its cached slots [0, P_b] (its own K/V were appended
 // before this kernel), query head h reading KV head h / G.  The cluster's C CTAs split the
-// positions in whole 64-position sub-tiles: CTA r takes sub-tiles [r n / C, (r + 1) n / C) of the
-// n = ceil((P_b + 1) / 64).
+// positions in whole 64-position sub-tiles: CTA r takes sub-tiles [ceil(r n / C), ceil((r + 1) n / C))
+// of the n = ceil((P_b + 1) / 64).
 //
 // Inside a CTA one producer warp streams the sub-tiles' K and V rows into a ring of shared-memory
 // stages with 2-D TMA copies (boxes of 64 positions x 64 dimensions, 128-byte swizzle: the
@@ -116,7 +116,7 @@ __device__ __forceinline__ void bf16_pair2(float x0, float x1, uint32_t &hi, uin
 }
 
 template <int HD>
-__global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_constant__ AttnParams p,
+__global__ void __launch_bounds__(ATC_THREADS, 2) attn_cluster_kernel(const __grid_constant__ AttnParams p,
                                                                    const __grid_constant__ CUtensorMap kmap,
                                                                    const __grid_constant__ CUtensorMap vmap) {
   using L = AtcLayout<HD>;
@@ -133,7 +133,7 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
   __shared__ float s_wl[ATC_WARPS][ATT_MAXG];
   __shared__ float s_m[ATT_MAXG], s_l[ATT_MAXG];     // this CTA's state, read by the cluster
   __shared__ volatile int s_abort;
-  pdl_launch_dependents();
+  if (p.launch_at == 0) pdl_launch_dependents();
   const int C = p.cluster;
   const int pair = blockIdx.x / C, r = blockIdx.x % C;  // r: the CTA's rank in its cluster
   const int b = pair / p.n_kv_heads, kvh = pair % p.n_kv_heads;
@@ -143,8 +143,9 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
   // trace slots of an attention CTA: go (start), enter (consumers past the wait on Q/K/V), x_go
   // (q's fragments built), x_last (first stage landed), kind (warp 0 done with the first stage),
   // seg (warp 0 done with its stages), ticket
-  // (every consumer warp done), summed (producer past its wait on Q/K/V), w_first / w_last (around
-  // the first cluster barrier), epi (cluster weights computed), done (end)
+  // (every consumer warp done), summed (producer past its wait on Q/K/V), w_last (producer issued
+  // its first sub-tile), w_first (before the cluster barrier), epi (cluster weights computed), done
+  // (end)
   auto stamp_by = [&](bool who, int slot) {
     if (p.trace && (int)blockIdx.x < p.trace_grid && who) p.trace[(size_t)blockIdx.x * TRACE_SLOTS + slot] = global_ns();
   };
@@ -156,13 +157,40 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
   uint4 *qf = reinterpret_cast<uint4 *>(sm + L::qf_off(S));
   const uint32_t sm0 = smem_addr(sm);
 
-  const int P = p.positions[b];
+  // the step's positions and KV slots: the producer loads every user's at once (it needs the
+  // lowest row this step writes into its user's slot, attn_step_lo), the others this user's
+  // position; the tensor maps' descriptors are fetched meanwhile
+  int P = -1, slot = 0, lo = 0;
+  if (warp == ATC_WARPS && lane == 0) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&kmap)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&vmap)) : "memory");
+    int pj[MAXB], sj[MAXB];
+#pragma unroll
+    for (int j = 0; j < MAXB; ++j) {
+      pj[j] = j < p.batch ? p.positions[j] : -1;
+      sj[j] = j < p.batch ? p.slots[j] : -1;
+    }
+#pragma unroll
+    for (int j = 0; j < MAXB; ++j)
+      if (j == b) {
+        P = pj[j];
+        slot = sj[j];
+      }
+    lo = P;
+#pragma unroll
+    for (int j = 0; j < MAXB; ++j)
+      if (sj[j] == slot && pj[j] >= 0 && pj[j] < lo) lo = pj[j];
+  } else {
+    P = p.positions[b];
+  }
   const bool valid = P >= 0 && P < p.max_ctx;
   int start = 0, end = 0;
   if (valid) {
     const int nsub_all = (P + ATT_SUB) / ATT_SUB;
-    start = static_cast<int>((long long)r * nsub_all / C) * ATT_SUB;
-    end = min(P + 1, static_cast<int>((long long)(r + 1) * nsub_all / C) * ATT_SUB);
+    // rounded up: the larger shares go to the first CTAs, so that the last one, which holds the
+    // rows this step writes and loads them only after the wait on Q/K/V, has the fewest
+    start = static_cast<int>(((long long)r * nsub_all + C - 1) / C) * ATT_SUB;
+    end = min(P + 1, static_cast<int>(((long long)(r + 1) * nsub_all + C - 1) / C) * ATT_SUB);
   }
   const int nsub = end > start ? (end - start + ATT_SUB - 1) / ATT_SUB : 0;
   // output chunks of XCHUNK elements of the pair's G x HD: CTA r merges [c0, c1)
@@ -193,8 +221,7 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
     // The cached rows [0, lo) were written by earlier steps: sub-tiles below lo go out while the
     // Q/K/V projection may still run, the rest after the wait on it.
     if (lane == 0 && nsub > 0) {
-      const int lo = attn_step_lo(p, b);
-      const int row0 = (p.slots[b] * p.n_kv_heads + kvh) * p.max_ctx;
+      const int row0 = (slot * p.n_kv_heads + kvh) * p.max_ctx;
       bool waited = false;
       int issued = 0;
       for (int t = 0; t < nsub; ++t) {
@@ -220,7 +247,9 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
           atc_tma_load(vd + hb * L::BOX_BYTES, &vmap, 64 * hb, row0 + p0, fb);
         }
         ++issued;
+        if (t == 0) stamp_by(true, TR_W_LAST);
       }
+      if (p.launch_at == 1) pdl_launch_dependents();
       // copies still in flight land before the shared memory is reused (bounded)
       for (int t = issued > S ? issued - S : 0; t < issued; ++t) mbar_wait(smem_addr(&full[t % S]), (t / S) & 1);
     }
@@ -256,6 +285,10 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
     named_bar_sync(ATT_BAR, ATC_WARPS * 32);
     stamp(TR_X_GO);
 
+    // q's A fragments stay in registers for the whole loop
+    uint4 qr[KS];
+#pragma unroll
+    for (int k = 0; k < KS; ++k) qr[k] = qf[k * 32 + lane];
     const int w0 = warp * 16;  // this warp's positions within a stage
     float m_run = -INFINITY, l_run = 0.f;  // head gid
     float acc[NT][4];  // rows gid (P's rounded parts) and gid + 8 (rests): both head gid's
@@ -286,19 +319,37 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
           __syncwarp();
         }
         // scores of positions w0 + 8 j + (2 tig, 2 tig + 1), n-tile j = 0, 1, for head gid: two
-        // accumulator chains per n-tile (K-step parity)
-        float sc[2][2][4] = {};
+        // accumulator chains per n-tile (K-step parity); every K fragment is loaded first (one
+        // round of shared-memory latency per stage, not one per K step)
         const int mi = lane >> 3, rr = lane & 7;
+        uint32_t kf[KS / 2][2][4];
 #pragma unroll
         for (int k2 = 0; k2 < KS / 2; ++k2) {
-          const uint4 qa = qf[(2 * k2) * 32 + lane], qb = qf[(2 * k2 + 1) * 32 + lane];
           const int ch = 4 * k2 + mi;  // the 16-byte chunk of dimensions this lane addresses
 #pragma unroll
+          for (int j = 0; j < 2; ++j)
+            ldsm_x4(kf[k2][j][0], kf[k2][j][1], kf[k2][j][2], kf[k2][j][3],
+                    kb + (ch >> 3) * L::BOX_BYTES + swz128(w0 + 8 * j + rr, ch & 7));
+        }
+        float sc[2][2][4] = {};
+#pragma unroll
+        for (int k2 = 0; k2 < KS / 2; ++k2) {
+          const uint4 qa = qr[2 * k2], qb = qr[2 * k2 + 1];
+#pragma unroll
           for (int j = 0; j < 2; ++j) {
-            uint32_t k0, k1, k2r, k3;
-            ldsm_x4(k0, k1, k2r, k3, kb + (ch >> 3) * L::BOX_BYTES + swz128(w0 + 8 * j + rr, ch & 7));
-            mma_bf16(sc[j][0], qa.x, qa.y, qa.z, qa.w, k0, k1);
-            mma_bf16(sc[j][1], qb.x, qb.y, qb.z, qb.w, k2r, k3);
+            mma_bf16(sc[j][0], qa.x, qa.y, qa.z, qa.w, kf[k2][j][0], kf[k2][j][1]);
+            mma_bf16(sc[j][1], qb.x, qb.y, qb.z, qb.w, kf[k2][j][2], kf[k2][j][3]);
+          }
+        }
+        // V's fragments (8 x 8 blocks of positions x dimensions, by transposing loads), in flight
+        // during the softmax
+        uint32_t vf[NT / 2][4];
+        {
+          const int vrow = w0 + 8 * (mi & 1) + rr;
+#pragma unroll
+          for (int d2 = 0; d2 < NT / 2; ++d2) {
+            const int ch = 2 * d2 + (mi >> 1);
+            ldsm_x4_t(vf[d2][0], vf[d2][1], vf[d2][2], vf[d2][3], vb + (ch >> 3) * L::BOX_BYTES + swz128(vrow, ch & 7));
           }
         }
         float sv[2][2];
@@ -339,21 +390,18 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
         uint32_t a0, a1, a2, a3;
         bf16_pair2(pr[0][0], pr[0][1], a0, a1);
         bf16_pair2(pr[1][0], pr[1][1], a2, a3);
-        // acc += P V: V fragments by transposing loads (8 x 8 blocks of positions x dimensions)
-        const int vrow = w0 + 8 * (mi & 1) + rr;
+        // acc += P V
 #pragma unroll
         for (int d2 = 0; d2 < NT / 2; ++d2) {
-          const int ch = 2 * d2 + (mi >> 1);
-          uint32_t v0, v1, v2, v3;
-          ldsm_x4_t(v0, v1, v2, v3, vb + (ch >> 3) * L::BOX_BYTES + swz128(vrow, ch & 7));
-          mma_bf16(acc[2 * d2], a0, a1, a2, a3, v0, v1);
-          mma_bf16(acc[2 * d2 + 1], a0, a1, a2, a3, v2, v3);
+          mma_bf16(acc[2 * d2], a0, a1, a2, a3, vf[d2][0], vf[d2][1]);
+          mma_bf16(acc[2 * d2 + 1], a0, a1, a2, a3, vf[d2][2], vf[d2][3]);
         }
       }
       mbar_arrive(smem_addr(&empty[s]));
       if (t == 0) stamp(TR_E_KIND);
     }
     stamp(TR_E_SEG);
+    if (p.launch_at == 2) pdl_launch_dependents();
     // this warp's state: (m, l) per head, sums [warp][head][HD] (rounded + rest rows) in the
     // stage buffers, once every consumer warp has read its last stage (the copies have all landed:
     // each was awaited)
@@ -392,7 +440,6 @@ __global__ void __launch_bounds__(ATC_THREADS) attn_cluster_kernel(const __grid_
   // every CTA's receive barrier is initialised
   __syncwarp();
   cluster_wait_acquire();
-  stamp(TR_W_LAST);
   // send: this CTA's (m, l) of every head to every CTA of the cluster, and its sums (the warps'
   // sums weighted in warp order) of each output chunk to the CTA that merges the chunk, the
   // largest o with o nch / C <= j
@@ -540,7 +587,7 @@ static cudaError_t launch_cluster_hd(const AttnParams &p, const CUtensorMap &km,
 
 cudaError_t launch_attention_cluster(const AttnParams &p, const CUtensorMap &km, const CUtensorMap &vm, int head_dim,
                                      cudaStream_t s, bool pdl) {
-  if (p.n_heads % p.n_kv_heads != 0 || p.n_heads / p.n_kv_heads > ATT_MAXG || p.cluster < 1 ||
+  if (p.batch < 1 || p.batch > MAXB || p.n_heads % p.n_kv_heads != 0 || p.n_heads / p.n_kv_heads > ATT_MAXG || p.cluster < 1 ||
       p.cluster > MAX_CLUSTER_ATT || p.stages < 2 || p.stages > ATT_RING_MAX)
     return cudaErrorInvalidValue;
   if (head_dim == 128) return launch_cluster_hd<128>(p, km, vm, s, pdl);

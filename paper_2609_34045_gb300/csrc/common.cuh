@@ -229,6 +229,7 @@ struct AttnParams {
   // `stages` sub-tiles (three: two CTAs fit an SM; two: three)
   int cluster;
   int stages;
+  int launch_at;             // the next kernel may launch: 0 at once, 1 when every sub-tile is issued, 2 after the loop
   float scale_log2;          // log2(e) / sqrt(hd)
   unsigned *err;
   // dataflow (persistent stage kernel only)

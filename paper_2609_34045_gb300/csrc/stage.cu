@@ -65,6 +65,8 @@ struct Plan {
   int attn_cluster_max;      // one kernel per phase: the largest attention cluster (0: unit kernel)
   int attn_stages;           // attention clusters: ring depth (sub-tiles) of a CTA
   int attn_cluster_sub;      // clusters are taken up to this many 64-position sub-tiles per CTA
+  int attn_launch_at;        // AttnParams::launch_at, for O projections of at most attn_late_max_mb MiB
+  int attn_late_max_mb;
   size_t bytes_weights, bytes_kv, bytes_ws;
 };
 
@@ -153,6 +155,12 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   // two attention CTAs fit an SM: about two units per SM over the step's actual contexts
   p->attn_units = n_sm * std::max(1, env_int("KFL_ATTN_UNITS_PER_SM", 2));
   p->attn_cluster_sub = env_int("KFL_ATTN_CLUSTER_SUB", 1 << 20);
+  // a small O projection's CTAs launch once the attention CTAs have left their loop: earlier,
+  // their weight prefetch (most of the matrix) delays the attention's own loads (7B b=1, 26 MB:
+  // -2.7% per step; 72B int4, 36 MB: -0.7%); a larger one's prefetch is worth starting at once
+  // (32B, 52 MB: +0.7% late; 72B bf16, 134 MB: +1.1%)
+  p->attn_launch_at = env_int("KFL_ATTN_LAUNCH", 2);
+  p->attn_late_max_mb = env_int("KFL_ATTN_LATE_MAX_MB", 48);
   p->attn_nchunks_max = (c->max_ctx + 63) / 64;
   p->n_phases = 5 * p->nl + ((flags & KFL_LOGITS_OUT) ? 1 : 0);
   {
@@ -415,6 +423,7 @@ std::vector<Phase> build_phases(kfl_stage *st, int batch, bool dataflow = false)
         const long long slots = (long long)P.n_sm * (P.attn_stages <= 2 ? 3 : 2);
         while (cl > 2 && (long long)cl * batch * P.hkv > slots) cl >>= 1;
         a.stages = P.attn_stages;
+        a.launch_at = P.o.bytes <= (size_t)P.attn_late_max_mb << 20 ? P.attn_launch_at : 0;
         // the clusters cannot balance ragged users or spread a long context over idle SMs, but
         // their CTAs stream without block barriers: they are taken unless a CTA would have more
         // than KFL_ATTN_CLUSTER_SUB 64-position sub-tiles at the longest context while the
