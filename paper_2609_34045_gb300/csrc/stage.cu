@@ -67,6 +67,7 @@ struct Plan {
   int attn_cluster_sub;      // clusters are taken up to this many 64-position sub-tiles per CTA
   int attn_launch_at;        // AttnParams::launch_at, for O projections of at most attn_late_max_mb MiB
   int attn_late_max_mb;
+  int down_cluster;          // the down projection as clusters of this many CTAs per row block (0: stream-K)
   size_t bytes_weights, bytes_kv, bytes_ws;
 };
 
@@ -161,6 +162,18 @@ void make_plan(const kfl_model_cfg *c, int l0, int l1, int flags, int n_sm, Plan
   // (32B, 52 MB: +0.7% late; 72B bf16, 134 MB: +1.1%)
   p->attn_launch_at = env_int("KFL_ATTN_LAUNCH", 2);
   p->attn_late_max_mb = env_int("KFL_ATTN_LATE_MAX_MB", 48);
+  // a bf16 down projection over few row blocks (every row block shared by four or more CTAs in
+  // the stream-K split) runs as clusters of 3 or 4 CTAs per row block, which combine through
+  // distributed shared memory instead of the ticket's partial sums in global memory (the last
+  // arriver's loads, round trips of about a microsecond each while the next kernel streams):
+  // 7B b=1 -2.2% per step (4), 32B -0.6% (3); clusters of 2 (72B bf16, int4) measured slower, as
+  // did clusters of 5 (56 clusters of 5 do not all fit the SMs at once); some slots are left for
+  // the packing of clusters into the GPCs
+  {
+    int N = std::min(4, (2 * n_sm - 32) / std::max(1, p->down.n_rb));
+    if (f != KFL_BF16 || N < 3 || p->down.n_kt < N) N = 0;
+    p->down_cluster = std::min(MAX_CLUSTER, env_int("KFL_DOWN_CLUSTER", N));
+  }
   p->attn_nchunks_max = (c->max_ctx + 63) / 64;
   p->n_phases = 5 * p->nl + ((flags & KFL_LOGITS_OUT) ? 1 : 0);
   {
@@ -596,9 +609,17 @@ int phase_kind_code(const Phase &ph, size_t i) {
 // The launch shape of a GEMV phase in the one-kernel-per-phase mode: sets g's ring depth and
 // cluster size and returns its grid.  Every shape is a stream-K split: CTA c streams tiles
 // [c T / G, (c + 1) T / G) (a cluster of N CTAs per row block is the split with G = N n_rb).
-int gemv_launch_shape(const kfl_stage *st, int batch, GemvParams &g) {
+int gemv_launch_shape(const kfl_stage *st, int batch, GemvParams &g, int big_cluster = 0) {
   const long long T = (long long)g.n_rb * g.n_kt;
   int grid = (int)(T < st->P.gemv_grid_max ? T : st->P.gemv_grid_max);
+  if (big_cluster >= 2 && g.n_kt >= big_cluster && (long long)big_cluster * g.n_rb <= 2LL * st->P.n_sm &&
+      st->P.ctas_per_sm > 1 && T > st->P.small_gemv_tiles) {
+    const int N = big_cluster;
+    const int per_sm = N * g.n_rb <= st->P.n_sm ? 1 : 2;
+    g.cluster = N;
+    g.stages = ring_depth(g.fmt, std::min(st->P.stages, gemv_stages_for(batch, g.fmt, N, per_sm)));
+    return N * g.n_rb;
+  }
   if (T <= st->P.small_gemv_tiles && T >= 2LL * st->P.n_sm && st->P.ctas_per_sm > 1) {
     // a small GEMV: one CTA per SM with a deeper ring, so that fewer CTAs share a row block;
     // with few enough row blocks, clusters of N CTAs split each one's K range and combine
@@ -630,7 +651,7 @@ int enqueue_body(kfl_stage *st, int batch, cudaStream_t s, bool pdl, std::vector
     }
     if (ph.kind == PH_GEMV) {
       GemvParams g = ph.g;
-      const int grid = gemv_launch_shape(st, batch, g);
+      const int grid = gemv_launch_shape(st, batch, g, i % 5 == 4 ? st->P.down_cluster : 0);
       CK(launch_gemv(g, ph.epi, grid, s, pdl));
     } else {
       if (ph.qn.raw) CK(launch_qknorm(ph.qn, s, pdl));  // QK-norm stages: norm, RoPE, KV append
