@@ -690,7 +690,9 @@ def run_ours(args, work):
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": False, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded)",
+            # the arithmetic type of the weight products: fp32 FMAs on bf16 weights; fp16
+            # tensor-core products (fp32 accumulation) on int4 weights
+            "vs_baseline": None, "dtype": "f32" if m.weight_fmt == "bf16" else "f16", "data": "synthetic (seeded)",
             "config": {"workload": work.name, "stage_layers": [work.l0, work.l1], "batch": b,
                        "ctx": list(work.contexts), "weights": m.weight_fmt,
                        "arithmetic": ("fp32 FMA on bf16 weights" if m.weight_fmt == "bf16"
