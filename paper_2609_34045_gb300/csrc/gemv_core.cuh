@@ -467,7 +467,7 @@ __device__ __forceinline__ void epilogue_prefetch(const GemvParams &p, int rb, i
 // The fused epilogue of row block rb: red[r * MAXB + b] is the dot product of row rb*RB + r for
 // user b, before the RMSNorm scale inv[b].  One warp.
 template <int B, int EPI>
-__device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const float *red, const float *inv,
+__device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, float *red, const float *inv,
                                               const EpiPre &pre, int lane) {
   if constexpr (EPI == EPI_STORE) {
     for (int e = lane; e < RB * B; e += 32) {
@@ -475,17 +475,18 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
       if (n < p.n_rows) p.out[(size_t)b * p.ldo + n] = red[r * MAXB + b] * inv[b];
     }
   } else if constexpr (EPI == EPI_RESID) {
-    // every read before the first store (the compiler cannot tell the stores from these reads),
-    // so that the users' conversions and reductions overlap
-    float hv[B][2];
+    // the new h of every user first, in place of the sums (each lane its own elements), then one
+    // user at a time through a loop that is not unrolled: the users' stores and conversions run
+    // the same instructions, which a CTA fetches once (the epilogue runs once per row block, so
+    // unrolled over the users its code would be fetched cold four times over)
 #pragma unroll
     for (int b = 0; b < B; ++b)
 #pragma unroll
       for (int h2 = 0; h2 < 2; ++h2) {
         const int r = lane + 32 * h2;
-        hv[b][h2] = rb * RB + r < p.n_rows ? pre.h[b][h2] + red[r * MAXB + b] * inv[b] : 0.f;
+        red[r * MAXB + b] = rb * RB + r < p.n_rows ? pre.h[b][h2] + red[r * MAXB + b] * inv[b] : 0.f;
       }
-#pragma unroll
+#pragma unroll 1
     for (int b = 0; b < B; ++b) {
       float sq = 0.f;
 #pragma unroll
@@ -493,7 +494,7 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
         const int r = lane + 32 * h2, n = rb * RB + r;
         const bool ok = n < p.n_rows;
         const size_t o = (size_t)b * p.ldh + n;
-        const float hn = hv[b][h2];
+        const float hn = red[r * MAXB + b];
         const float xv = hn * pre.g[h2];
         // int4 stage: xn in the tensor-core input form, chunk rb * 2 + h2
         if (p.xout.base && p.g_next) act16_put_warp(p.xout, b, rb * 2 + h2, xv, lane);
@@ -508,21 +509,16 @@ __device__ __forceinline__ void epilogue_warp(const GemvParams &p, int rb, const
       if (lane == 0) p.sumsq_out[rb * MAXB + b] = sq;
     }
   } else if constexpr (EPI == EPI_SWIGLU) {
-    // lane = output (RB / 2 = 32 of them per row block), one user per pass; every read first
-    float gv[B], uv[B];
-#pragma unroll
-    for (int b = 0; b < B; ++b) {
-      gv[b] = red[(2 * lane) * MAXB + b] * inv[b];
-      uv[b] = red[(2 * lane + 1) * MAXB + b] * inv[b];
-    }
-#pragma unroll
+    // lane = output (RB / 2 = 32 of them per row block), one user per pass of a loop that is not
+    // unrolled (as in RESID)
+#pragma unroll 1
     for (int b = 0; b < B; ++b) {
       const int pr = lane, j = rb * (RB / 2) + pr;
       const bool ok = 2 * j < p.n_rows;
       float a = 0.f;
       if (ok) {
-        const float g = gv[b];
-        const float u = uv[b];
+        const float g = red[(2 * lane) * MAXB + b] * inv[b];
+        const float u = red[(2 * lane + 1) * MAXB + b] * inv[b];
         a = g / (1.0f + expf(-g)) * u;
       }
       if (p.xout.base)
